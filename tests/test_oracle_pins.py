@@ -1,0 +1,338 @@
+"""Pins of the fp64 CPU oracle to things other than itself.
+
+Every check here compares the oracle with a library routine on a special case,
+a closed form, an invariant the paper states, or brute force on tiny inputs.
+The paper prints no worked numeric example, so no value is copied from it.
+"""
+
+import itertools
+import math
+
+import numpy as np
+import pytest
+import scipy.stats
+import torch
+
+import oracle
+from paper_2608_08878_gb300 import synth
+
+
+def bits(x):
+    return synth.f32_to_bf16_bits(np.asarray(x, dtype=np.float32))
+
+
+def widen(b):
+    return synth.bf16_bits_to_f32(b).astype(np.float64)
+
+
+def rand_bits(rng, *shape, scale=1.0):
+    return bits(rng.standard_normal(shape).astype(np.float32) * np.float32(scale))
+
+
+def sdpa_gqa(q_bits, k_bits, v_bits):
+    """torch's scaled_dot_product_attention in fp64 for one KV head's query group."""
+    q = torch.from_numpy(widen(q_bits))[None, :, None, :]          # [1, G, 1, d]
+    G = q.shape[1]
+    k = torch.from_numpy(widen(k_bits))[None, None].expand(1, G, -1, -1)
+    v = torch.from_numpy(widen(v_bits))[None, None].expand(1, G, -1, -1)
+    o = torch.nn.functional.scaled_dot_product_attention(q, k, v)
+    return o[0, :, 0, :].numpy()
+
+
+def softmax_rows(q_bits, k_bits):
+    q = torch.from_numpy(widen(q_bits))
+    k = torch.from_numpy(widen(k_bits))
+    return torch.softmax(q @ k.T / math.sqrt(q.shape[1]), dim=-1).numpy()  # [G][n]
+
+
+# --------------------------------------------------------------------------
+# Attention and entropy
+# --------------------------------------------------------------------------
+
+@pytest.mark.parametrize("n,d,G", [(1, 64, 2), (37, 64, 4), (300, 128, 4)])
+def test_attention_equals_torch_sdpa(n, d, G):
+    rng = np.random.default_rng(n + d)
+    q, k, v = rand_bits(rng, G, d), rand_bits(rng, n, d, scale=2.0), rand_bits(rng, n, d)
+    o, Hq = oracle.attend(q, k, v)
+    np.testing.assert_allclose(o, sdpa_gqa(q, k, v), rtol=1e-12, atol=1e-12)
+    a = softmax_rows(q, k)
+    np.testing.assert_allclose(a.sum(-1), 1.0, rtol=1e-12)
+    np.testing.assert_allclose(Hq, [scipy.stats.entropy(a[h]) for h in range(G)], rtol=1e-10, atol=1e-12)
+    assert np.all(Hq >= -1e-12) and np.all(Hq <= math.log(n) + 1e-9)
+
+
+def test_entropy_uniform_and_one_hot():
+    d, n = 64, 50
+    q = bits(np.ones((2, d)))
+    k = bits(np.zeros((n, d)))
+    v = bits(np.random.default_rng(0).standard_normal((n, d)))
+    _, Hq = oracle.attend(q, k, v)
+    np.testing.assert_allclose(Hq, math.log(n), rtol=1e-13)
+    k2 = np.zeros((n, d), dtype=np.float32)
+    k2[7] = 8.0  # one key far along q: its logit is 64 above the rest
+    o, Hq2 = oracle.attend(q, bits(k2), v)
+    assert np.all(Hq2 < 1e-20)
+    np.testing.assert_allclose(o[0], widen(v[7]), rtol=1e-20, atol=1e-20)
+
+
+# --------------------------------------------------------------------------
+# Step: features against library routines, closed forms and brute force
+# --------------------------------------------------------------------------
+
+def _mlp(hidden=16, layernorm=1, seed=3):
+    return synth.policy_weights(seed, hidden), hidden, layernorm
+
+
+def test_step_features_against_libraries():
+    rng = np.random.default_rng(5)
+    d, G, T = 32, 4, 40
+    row = oracle.OracleRow(d, G, window=64, alpha_mode=0, capacity=64)
+    kp, vp = rand_bits(rng, T, d), rand_bits(rng, T, d)
+    row.append(kp, vp)
+    q, kn, vn = rand_bits(rng, G, d), rand_bits(rng, d), rand_bits(rng, d)
+    mlp, H, ln = _mlp()
+    r = row.step(q, kn, vn, mlp, H, ln)
+    K = np.concatenate([kp, kn[None]])
+    V = np.concatenate([vp, vn[None]])
+    a = softmax_rows(q, K)                                  # [G][n]
+    at = torch.from_numpy(a)
+    np.testing.assert_allclose(r["o"], sdpa_gqa(q, K, V), rtol=1e-12, atol=1e-12)
+    f = r["feat"]
+    np.testing.assert_allclose(f[:, 0], at.mean(0).numpy(), rtol=1e-12)                    # alpha
+    np.testing.assert_allclose(f[:, 1], np.linalg.norm(widen(V), axis=1), rtol=1e-13)     # |v|
+    np.testing.assert_allclose(f[:, 2], at.var(0, unbiased=False).numpy(), rtol=1e-9, atol=1e-20)
+    # first step: the window holds one query step -> H_i = sum_h a_h H_h / sum_h a_h
+    Hq = np.array([scipy.stats.entropy(a[h]) for h in range(G)])
+    np.testing.assert_allclose(r["Hq"], Hq, rtol=1e-10)
+    np.testing.assert_allclose(f[:, 3], (a * Hq[:, None]).sum(0) / a.sum(0), rtol=1e-10)
+    np.testing.assert_allclose(f[:, 4], np.arange(T + 1) / T, rtol=1e-15)                   # pos
+    np.testing.assert_array_equal(r["pos"], np.arange(T + 1))
+
+
+def test_mlp_equals_torch_sequential():
+    rng = np.random.default_rng(9)
+    x = rng.standard_normal((200, 5)) * np.array([0.1, 10.0, 0.01, 3.0, 1.0])
+    for hidden, layernorm in [(128, 1), (64, 0), (7, 1)]:
+        blob = synth.policy_weights(11, hidden)
+        # blob: [W1 5H | b1 H | gamma H | beta H | w2 H | b2]; give LayerNorm a
+        # non-trivial gain and shift so both are exercised.
+        blob[6 * hidden:7 * hidden] = 1.0 + 0.1 * np.arange(hidden, dtype=np.float32)
+        blob[7 * hidden:8 * hidden] = (0.1 * rng.standard_normal(hidden)).astype(np.float32)
+        W1 = blob[:5 * hidden].reshape(hidden, 5)
+        b1 = blob[5 * hidden:6 * hidden]
+        gamma = blob[6 * hidden:7 * hidden]
+        beta = blob[7 * hidden:8 * hidden]
+        w2 = blob[8 * hidden:9 * hidden]
+        b2 = blob[9 * hidden]
+        lin1 = torch.nn.Linear(5, hidden).double()
+        lin2 = torch.nn.Linear(hidden, 1).double()
+        with torch.no_grad():
+            lin1.weight.copy_(torch.from_numpy(W1.astype(np.float64)))
+            lin1.bias.copy_(torch.from_numpy(b1.astype(np.float64)))
+            lin2.weight.copy_(torch.from_numpy(w2.astype(np.float64))[None])
+            lin2.bias.fill_(float(b2))
+        layers = [lin1]
+        if layernorm:
+            lnm = torch.nn.LayerNorm(hidden, eps=1e-5).double()
+            with torch.no_grad():
+                lnm.weight.copy_(torch.from_numpy(gamma.astype(np.float64)))
+                lnm.bias.copy_(torch.from_numpy(beta.astype(np.float64)))
+            layers.append(lnm)
+        layers += [torch.nn.ReLU(), lin2]
+        ref = torch.nn.Sequential(*layers)(torch.from_numpy(x)).detach().numpy()[:, 0]
+        np.testing.assert_allclose(oracle.policy(x, blob, hidden, layernorm), ref, rtol=1e-12, atol=1e-12)
+
+
+def test_uniform_keys_closed_forms():
+    """All keys equal: every query attends uniformly, so a = 1/n, sigma = 0,
+    H_q = ln n and (with a constant cache size) H_i = ln n for every token;
+    cumulative alpha is (steps since insertion) / n."""
+    d, G, B, T = 16, 2, 9, 20
+    kc = bits(np.full((1, d), 0.5))
+    rng = np.random.default_rng(1)
+    mlp, H, ln = _mlp(8, 1)
+    for mode in (0, 1):
+        row = oracle.OracleRow(d, G, window=4, alpha_mode=mode, capacity=T + 1)
+        row.append(np.repeat(kc, T, 0), rand_bits(rng, T, d))
+        inserted = {p: 0 for p in range(T)}
+        for step in range(10):
+            r = row.step(rand_bits(rng, G, d), kc[0], rand_bits(rng, d), mlp, H, ln)
+            n = len(r["pos"])
+            inserted[int(r["pos"][-1])] = step
+            np.testing.assert_allclose(r["Hq"], math.log(n), rtol=1e-13)
+            assert np.all(r["feat"][:, 2] == 0.0)
+            if step >= 4:  # the cache held B + 1 tokens at every step of the window
+                np.testing.assert_allclose(r["feat"][:, 3], math.log(B + 1), rtol=1e-12)
+            if mode == 0:
+                np.testing.assert_allclose(r["feat"][:, 0], 1.0 / n, rtol=1e-13)
+            elif step >= 1:
+                want = [(step - max(inserted[int(p)], 1) + 1) / (B + 1) + (1.0 / (T + 1) if inserted[int(p)] == 0 else 0.0)
+                        for p in r["pos"]]
+                np.testing.assert_allclose(r["feat"][:, 0], want, rtol=1e-12)
+            row.evict(B)
+
+
+def _bruteforce_run(alpha_mode, w, steps, seed):
+    rng = np.random.default_rng(seed)
+    d, G, T, B = 8, 2, 6, 5
+    mlp, H, ln = _mlp(8, 1)
+    row = oracle.OracleRow(d, G, window=w, alpha_mode=alpha_mode, capacity=T + steps + 1)
+    kp, vp = rand_bits(rng, T, d), rand_bits(rng, T, d)
+    row.append(kp, vp)
+    store_k = {p: kp[p] for p in range(T)}
+    history = []  # per step: (dict pos -> a [G], H [G])
+    for step in range(steps):
+        q, kn, vn = rand_bits(rng, G, d, scale=1.5), rand_bits(rng, d), rand_bits(rng, d)
+        r = row.step(q, kn, vn, mlp, H, ln)
+        pos = r["pos"]
+        store_k[int(pos[-1])] = kn
+        K = np.stack([store_k[int(p)] for p in pos])
+        a = softmax_rows(q, K)
+        Hq = np.array([scipy.stats.entropy(a[h]) for h in range(G)])
+        history.append(({int(p): a[:, i] for i, p in enumerate(pos)}, Hq))
+        S_w, Z_w, acc = row.window_sums()
+        for i, p in enumerate(pos):
+            Z = S = 0.0
+            for amap, Hh in history[-w:]:
+                if int(p) in amap:
+                    Z += amap[int(p)].sum()
+                    S += (amap[int(p)] * Hh).sum()
+            np.testing.assert_allclose(Z_w[i], Z, rtol=1e-12)
+            np.testing.assert_allclose(S_w[i], S, rtol=1e-12)
+            np.testing.assert_allclose(r["feat"][i, 3], S / Z, rtol=1e-12)
+            if alpha_mode == 1:
+                cum = sum(amap[int(p)].mean() for amap, _ in history if int(p) in amap)
+                np.testing.assert_allclose(r["feat"][i, 0], cum, rtol=1e-12)
+        row.evict(B)
+    return row
+
+
+@pytest.mark.parametrize("w,alpha_mode", [(1, 0), (3, 0), (3, 1), (64, 0)])
+def test_window_sums_brute_force(w, alpha_mode):
+    _bruteforce_run(alpha_mode, w, steps=12, seed=w + 10 * alpha_mode)
+
+
+# --------------------------------------------------------------------------
+# Top-B selection and pruning
+# --------------------------------------------------------------------------
+
+def _lexsort_keep(scores, pos, B):
+    s = np.asarray(scores, dtype=np.float64)
+    nan = np.isnan(s)
+    key = np.where(nan, 0.0, -s)  # descending score; -0 and +0 compare equal
+    order = np.lexsort((pos, key, nan))
+    return set(int(pos[i]) for i in order[:B])
+
+
+def _row_with_n(n, d=4, G=1):
+    rng = np.random.default_rng(n)
+    row = oracle.OracleRow(d, G, window=4, alpha_mode=0, capacity=n + 1)
+    row.append(rand_bits(rng, n, d), rand_bits(rng, n, d))
+    return row
+
+
+def test_evict_matches_lexsort_with_ties_zeros_and_nan():
+    rng = np.random.default_rng(2)
+    for n, B in [(1, 1), (10, 3), (64, 17), (100, 100), (100, 150)]:
+        scores = rng.integers(-3, 4, n).astype(np.float32)  # many ties
+        scores[rng.random(n) < 0.1] = -0.0
+        scores[rng.random(n) < 0.05] = np.nan
+        row = _row_with_n(n)
+        pos = row.positions()
+        want = _lexsort_keep(scores, pos, B)
+        assert row.evict(B, scores) == min(n, B)
+        assert set(row.positions().tolist()) == want
+        assert np.all(np.diff(row.positions()) > 0)
+
+
+def test_evict_brute_force_subsets():
+    """The kept set is the B-subset whose ranking keys (score, -position) sort
+    highest, found by enumerating every subset."""
+    rng = np.random.default_rng(4)
+    for trial in range(30):
+        n = int(rng.integers(1, 8))
+        B = int(rng.integers(1, n + 1))
+        scores = rng.integers(-2, 3, n).astype(np.float32)
+        row = _row_with_n(n)
+        pos = row.positions()
+        best = None
+        for sub in itertools.combinations(range(n), B):
+            key = sorted(((float(scores[i]), -int(pos[i])) for i in sub), reverse=True)
+            if best is None or key > best[0]:
+                best = (key, set(int(pos[i]) for i in sub))
+        row.evict(B, scores)
+        assert set(row.positions().tolist()) == best[1]
+
+
+def test_prune_keeps_bytes_and_budget_invariants():
+    wl = synth.TINY
+    L, b, g = 0, 0, 1
+    kp, vp = synth.prompt_row(wl, L, b, g)
+    row = oracle.OracleRow(wl.head_dim, wl.group, wl.window, 0, wl.capacity)
+    row.append(kp, vp)
+    src_k = {p: kp[p] for p in range(wl.prompt_len)}
+    src_v = {p: vp[p] for p in range(wl.prompt_len)}
+    mlp = synth.policy_weights(wl.policy_seed, wl.mlp_hidden)
+    for step in range(wl.steps):
+        q, kn, vn = synth.step_row(wl, step, L, b, g)
+        n_before = len(row) + 1
+        r = row.step(q, kn, vn, mlp, wl.mlp_hidden, wl.layernorm)
+        newest = int(r["pos"][-1])
+        src_k[newest], src_v[newest] = kn, vn
+        assert newest == wl.prompt_len + step and len(r["pos"]) == n_before
+        row.evict(wl.budget)
+        assert len(row) == min(n_before, wl.budget)
+        k, v = row.kv_bits()
+        for i, p in enumerate(row.positions()):
+            assert np.array_equal(k[i], src_k[int(p)]) and np.array_equal(v[i], src_v[int(p)])
+
+
+def test_budget_at_least_n_is_full_cache_attention():
+    rng = np.random.default_rng(8)
+    d, G, T = 32, 4, 25
+    mlp, H, ln = _mlp()
+    row = oracle.OracleRow(d, G, 64, 0, T + 20)
+    K, V = rand_bits(rng, T, d), rand_bits(rng, T, d)
+    row.append(K, V)
+    for step in range(10):
+        q, kn, vn = rand_bits(rng, G, d), rand_bits(rng, d), rand_bits(rng, d)
+        r = row.step(q, kn, vn, mlp, H, ln)
+        K, V = np.concatenate([K, kn[None]]), np.concatenate([V, vn[None]])
+        np.testing.assert_allclose(r["o"], sdpa_gqa(q, K, V), rtol=1e-12, atol=1e-12)
+        assert row.evict(T + 20) == len(K)
+
+
+def test_paper_eviction_error_bound():
+    """Sec. 3.1 (Reward): |o - o_hat| <= 2 C eps, with C = max |v_i| and eps the
+    full-cache attention mass on the evicted tokens, against an unpruned
+    teacher row fed the same inputs."""
+    wl = synth.TINY.with_(prompt_len=96, budget=24, steps=20)
+    mlp = synth.policy_weights(0, wl.mlp_hidden)
+    kp, vp = synth.prompt_row(wl, 0, 0, 0)
+    teacher = oracle.OracleRow(wl.head_dim, wl.group, wl.window, 0, wl.prompt_len + wl.steps + 1)
+    student = oracle.OracleRow(wl.head_dim, wl.group, wl.window, 0, wl.prompt_len + wl.steps + 1)
+    teacher.append(kp, vp)
+    student.append(kp, vp)
+    K = kp
+    for step in range(wl.steps):
+        q, kn, vn = synth.step_row(wl, step, 0, 0, 0)
+        rt = teacher.step(q, kn, vn, mlp, wl.mlp_hidden, wl.layernorm)
+        rs = student.step(q, kn, vn, mlp, wl.mlp_hidden, wl.layernorm)
+        K = np.concatenate([K, kn[None]])
+        a = softmax_rows(q, K)
+        kept = np.isin(rt["pos"], rs["pos"])
+        eps = a[:, ~kept].sum(1)
+        Vt = widen(teacher.kv_bits()[1])
+        C = np.linalg.norm(Vt, axis=1).max()
+        err = np.linalg.norm(rt["o"] - rs["o"], axis=1)
+        assert np.all(err <= 2 * C * eps + 1e-12), (step, err, eps)
+        if step > 0:
+            assert np.all(eps > 0)
+        student.evict(wl.budget)
+
+
+def test_capacity_overflow_leaves_row_unchanged():
+    row = _row_with_n(4)
+    with pytest.raises(OverflowError):
+        row.append(np.zeros((2, 4), np.uint16), np.zeros((2, 4), np.uint16))
+    assert len(row) == 4
