@@ -1,0 +1,423 @@
+"""Decode-step throughput of the budgeted KV-eviction hot path on GB300.
+
+One step = dc_decode_step + dc_evict over every layer and sequence of the
+workload: Mistral-7B KV shape (32 layers, 32 query / 8 KV heads, head_dim 128),
+batch 8, 32K-token prompt compressed to a 25% budget (8192 tokens per row), one
+token appended and one evicted per row per step. Inputs are synthetic and
+seeded; the prompt compression (first decode step) happens before warm-up.
+
+Prints one JSON line (rank 0). ``--impl reference`` times the fp64 CPU oracle
+on the host cores instead (a bounded sample of the same workload).
+"""
+
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "decode steps/s and HBM GB/s (% of 8 TB/s) at Mistral-7B shape, 25% budget"
+UNIT = "decode steps/s"
+NOMINAL_HBM_GBS = 8000.0
+
+
+def measured_peaks():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            return json.load(f), "measured"
+    except Exception:
+        return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0}, "fallback"
+
+
+def workload():
+    from paper_2608_08878_gb300 import synth
+    return synth.MISTRAL_FULL
+
+
+def row_bytes_per_step(n: int, d: int, alpha_mode: int = 0) -> int:
+    """Algorithmic HBM bytes of one row's decode step over n tokens (after the
+    append): K and V read once (4d bytes per token), position read (4), window
+    sums S and Z read and written (32), cumulative alpha read and written in
+    alpha_mode 1 (8)."""
+    return n * (4 * d + 36 + (8 if alpha_mode else 0))
+
+
+def step_bytes(wl, n: int, moved_per_row: float = 1.0) -> float:
+    """Whole-step algorithmic bytes: every row's pass over its n tokens, the
+    append (new key and value, 4d bytes, plus 20 bytes of position and window
+    state written) and the compaction moves (each moved token's K/V and 20
+    bytes of state read and written; one per row in the steady state)."""
+    d = wl.head_dim
+    per_row = row_bytes_per_step(n, d, wl.alpha_mode) + (4 * d + 20) + moved_per_row * 2 * (4 * d + 20)
+    return wl.rows * per_row
+
+
+class ClockSampler:
+    """nvidia-smi clock/throttle samples while the timed region runs."""
+
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index: str):
+        self.index = index
+        self.proc = None
+        self.lines = []
+
+    def __enter__(self):
+        try:
+            self.proc = subprocess.Popen(["nvidia-smi", "-i", self.index, f"--query-gpu={self.FIELDS}",
+                                          "--format=csv,noheader,nounits", "-lms", "200"],
+                                         stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            self.thread = threading.Thread(target=self._read, daemon=True)
+            self.thread.start()
+        except Exception:
+            self.proc = None
+        return self
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append(line.strip())
+
+    def __exit__(self, *a):
+        if self.proc:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except Exception:
+                self.proc.kill()
+            self.thread.join(timeout=2)
+
+    def summary(self):
+        sm, mx, reasons = [], None, set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for ln in self.lines:
+            parts = [p.strip() for p in ln.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                sm.append(float(parts[1]))
+                mx = float(parts[2])
+            except ValueError:
+                continue
+            for nm, val in zip(names, parts[5:9]):
+                if val.lower().startswith("active"):
+                    reasons.add(nm)
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": mx,
+                "reasons": sorted(reasons), "samples": len(sm)}
+
+
+def gpu_index_for_smi(local_rank: int) -> str:
+    vis = os.environ.get("CUDA_VISIBLE_DEVICES")
+    if vis:
+        ids = [x.strip() for x in vis.split(",") if x.strip()]
+        if local_rank < len(ids):
+            return ids[local_rank]
+    return str(local_rank)
+
+
+# ---------------------------------------------------------------------------
+# CPU oracle leg (cpu_baseline and --impl reference)
+# ---------------------------------------------------------------------------
+
+def oracle_sample(wl, seconds: float = 12.0, threads: int | None = None, warm_steps: int | None = None):
+    """Times the fp64 oracle on a bounded sample: `threads` rows of the steady
+    state (n = budget + 1 after the append), each run for several decode steps
+    with a full entropy window, rows in parallel on host threads. Returns
+    decode steps/s of the whole workload extrapolated from the sample."""
+    import numpy as np
+    import oracle
+    from paper_2608_08878_gb300 import synth
+    oracle.build()
+    cores = os.cpu_count() or 1
+    threads = threads or max(1, min(16, cores))
+    warm_steps = wl.window if warm_steps is None else warm_steps
+    blob = synth.policy_weights(wl.policy_seed, wl.mlp_hidden)
+    sample_rows = [int(r) for r in np.linspace(0, wl.rows - 1, threads).astype(int)]
+    rows = {}
+
+    def setup(r):
+        layer, b, g = wl.row_coords(r)
+        o = oracle.OracleRow(wl.head_dim, wl.group, wl.window, wl.alpha_mode, wl.budget + 2)
+        k, v = synth.prompt_row(wl, layer, b, g, 0, wl.budget)
+        o.append(k, v)
+        for s in range(warm_steps):
+            qb, kb, vb = synth.step_row(wl, s, layer, b, g)
+            o.step(qb, kb, vb, blob, wl.mlp_hidden, wl.layernorm)
+            o.evict(wl.budget)
+        rows[r] = o
+
+    ts = [threading.Thread(target=setup, args=(r,)) for r in sample_rows]
+    [t.start() for t in ts]
+    [t.join() for t in ts]
+    # timed: each thread steps its row until the time budget is used
+    counts = {r: 0 for r in sample_rows}
+    deadline = [0.0]
+
+    def run(r):
+        layer, b, g = wl.row_coords(r)
+        o = rows[r]
+        s = warm_steps
+        while time.perf_counter() < deadline[0] or counts[r] == 0:
+            qb, kb, vb = synth.step_row(wl, s, layer, b, g)
+            o.step(qb, kb, vb, blob, wl.mlp_hidden, wl.layernorm)
+            o.evict(wl.budget)
+            counts[r] += 1
+            s += 1
+
+    t0 = time.perf_counter()
+    deadline[0] = t0 + seconds
+    ts = [threading.Thread(target=run, args=(r,)) for r in sample_rows]
+    [t.start() for t in ts]
+    [t.join() for t in ts]
+    el = time.perf_counter() - t0
+    row_steps = sum(counts.values())
+    steps_per_s = row_steps / wl.rows / el
+    return {"value": steps_per_s, "unit": UNIT, "cores": len(sample_rows), "kind": "oracle",
+            "sample": (f"{len(sample_rows)} rows (of {wl.rows}) at the steady state n={wl.budget + 1}, "
+                       f"full w={wl.window} window, {row_steps} row-steps in {el:.1f}s on "
+                       f"{len(sample_rows)} host threads; value = row-steps / rows / s")}
+
+
+# ---------------------------------------------------------------------------
+# GPU leg
+# ---------------------------------------------------------------------------
+
+def run_gpu(args):
+    import torch
+    from paper_2608_08878_gb300 import build, dc, synth, synth_device
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local_rank = int(os.environ.get("LOCAL_RANK", "0"))
+    torch.cuda.set_device(local_rank)
+    dist = None
+    if world > 1:
+        import torch.distributed as tdist
+        tdist.init_process_group("nccl", device_id=torch.device("cuda", local_rank))
+        dist = tdist
+    if local_rank == 0:
+        build.build()
+    if dist:
+        dist.barrier()
+    wl = workload()
+    wl = wl.with_(seed=wl.seed + 1000 * rank)
+    K, W = args.steps, args.warmup
+    stream = torch.cuda.current_stream()
+    cache = dc.DistillCache(wl.layers, wl.kv_heads, wl.head_dim, wl.capacity, wl.budget,
+                            batch=wl.batch, q_heads=wl.q_heads, window=wl.window,
+                            mlp_hidden=wl.mlp_hidden, layernorm=wl.layernorm, engine=args.engine,
+                            seed=wl.policy_seed)
+    chunk = 4096
+    for t0 in range(0, wl.prompt_len, chunk):
+        k, v = synth_device.prompt(wl, t0, min(chunk, wl.prompt_len - t0))
+        cache.append(k, v)
+        del k, v
+    # all step inputs resident in HBM before timing
+    inputs = [synth_device.step_inputs(wl, s) for s in range(1 + W + K)]
+    out = torch.empty((wl.layers, wl.batch, wl.q_heads, wl.head_dim), dtype=torch.float32, device="cuda")
+    # step 0: prompt compression (32769 -> 8192 tokens per row), timed apart
+    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    ev0.record(stream)
+    cache.decode_step(*inputs[0], out=out)
+    cache.evict()
+    ev1.record(stream)
+    torch.cuda.synchronize()
+    first_ms = ev0.elapsed_time(ev1)
+    for s in range(1, 1 + W):
+        cache.decode_step(*inputs[s], out=out)
+        cache.evict()
+    n_steady = cache.length()[0] + 1
+    cache.profile(True)
+    torch.cuda.synchronize()
+    if dist:
+        dist.barrier()
+    torch.cuda.synchronize()
+    with ClockSampler(gpu_index_for_smi(local_rank)) as clk:
+        ev0.record(stream)
+        for s in range(1 + W, 1 + W + K):
+            cache.decode_step(*inputs[s], out=out)
+            cache.evict()
+        ev1.record(stream)
+        torch.cuda.synchronize()
+    el_ms = ev0.elapsed_time(ev1)
+    prof = cache.profile_read()
+    cache.profile(False)
+    if dist:
+        t = torch.tensor([el_ms], device="cuda")
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        el_ms = float(t.item())
+    ms_per_step = el_ms / K
+    value = world * K / (el_ms / 1e3)
+    bytes_step = step_bytes(wl, n_steady)
+    gbs = bytes_step / (ms_per_step / 1e3) / 1e9
+    peaks, peak_src = measured_peaks()
+
+    # dominant kernel: roofline from the live per-launch events
+    dom = max((ph for ph in prof if prof[ph][1] > 0), key=lambda ph: prof[ph][0])
+    dom_ms, dom_n = prof[dom]
+    per_launch_ms = dom_ms / dom_n
+    if dom == "attend" and args.engine == 1:
+        alg = wl.rows * n_steady * (2 * wl.head_dim + 4)  # K read + positions
+    elif dom == "score":
+        alg = wl.rows * n_steady * (2 * wl.head_dim + 36)  # V read + positions + window sums R/W
+    else:
+        alg = wl.rows * row_bytes_per_step(n_steady, wl.head_dim, wl.alpha_mode)
+    achieved = alg / (per_launch_ms / 1e3) / 1e9
+    gpu_launches = int(sum(v[1] for v in prof.values()))
+
+    # full-cache comparator on the same inputs (the uncompressed prompt)
+    full = None
+    if not args.no_full and rank == 0:
+        del cache
+        torch.cuda.empty_cache()
+        fc = dc.DistillCache(wl.layers, wl.kv_heads, wl.head_dim, wl.prompt_len + 1, wl.budget,
+                             batch=wl.batch, q_heads=wl.q_heads, window=wl.window, engine=args.engine)
+        for t0 in range(0, wl.prompt_len, chunk):
+            k, v = synth_device.prompt(wl, t0, min(chunk, wl.prompt_len - t0))
+            fc.append(k, v)
+            del k, v
+        for s in range(W):
+            fc.full_decode(inputs[s][0], out=out)
+        kf = min(K, 32)
+        torch.cuda.synchronize()
+        ev0.record(stream)
+        for s in range(kf):
+            fc.full_decode(inputs[1 + W + s][0], out=out)
+        ev1.record(stream)
+        torch.cuda.synchronize()
+        fms = ev0.elapsed_time(ev1) / kf
+        fbytes = wl.rows * wl.prompt_len * 4 * wl.head_dim
+        full = {"ms_per_step": fms, "steps_per_s": 1e3 / fms, "n_tokens_per_row": wl.prompt_len,
+                "gbs": fbytes / (fms / 1e3) / 1e9, "speedup_of_eviction_step": fms / ms_per_step}
+        del fc
+        torch.cuda.empty_cache()
+        cache = None
+
+    # end to end through the public API with host buffers (rank 0 does it too
+    # on every rank: each rank its own replica)
+    e2e = None
+    if not args.no_e2e:
+        e2e = run_e2e(wl, args, inputs)
+
+    res = None
+    if rank == 0:
+        res = {
+            "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": K, "warmup": W,
+            "ms_per_step": ms_per_step, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+            "dtype": "bf16", "data": "synthetic",
+            "config": {"workload": wl.name, "layers": wl.layers, "batch": wl.batch, "q_heads": wl.q_heads,
+                       "kv_heads": wl.kv_heads, "head_dim": wl.head_dim, "context": wl.prompt_len,
+                       "budget": wl.budget, "window": wl.window, "policy": f"5-{wl.mlp_hidden}-LN-ReLU-1",
+                       "engine": ["fused", "split"][args.engine], "parallelism": f"replicas x{world}",
+                       "l2": f"inputs larger than L2: {bytes_step / 1e9:.2f} GB streamed per step vs 129 MB L2",
+                       "steady_tokens_per_row": n_steady},
+            "hbm": {"algorithmic_bytes_per_step": bytes_step, "gbs": gbs,
+                    "frac_of_8tbs": gbs / NOMINAL_HBM_GBS,
+                    "frac_of_measured": gbs / peaks["hbm_gbs"], "peak_source": peak_src},
+            "first_step_ms": first_ms,
+            "roofline": {"bound": "hbm", "kernel": dom, "achieved": achieved, "peak": peaks["hbm_gbs"],
+                         "unit": "GB/s", "frac": achieved / peaks["hbm_gbs"], "traffic": None,
+                         "peak_source": f"{peak_src} copy bandwidth",
+                         "per_launch_ms": per_launch_ms, "algorithmic_bytes_per_launch": alg},
+            "phases_ms_per_step": {k: v[0] / K for k, v in prof.items() if v[1]},
+            "gpu_launches": gpu_launches,
+            "clocks": clk.summary(),
+            "full_cache": full,
+            "e2e": e2e,
+        }
+    if dist:
+        dist.barrier()
+        dist.destroy_process_group()
+    return res
+
+
+def run_e2e(wl, args, inputs):
+    """The same steps through dc_decode_step_host: pinned host inputs copied in
+    and the attention output copied out inside the timed region."""
+    import torch
+    from paper_2608_08878_gb300 import dc, synth_device
+    cache = dc.DistillCache(wl.layers, wl.kv_heads, wl.head_dim, wl.capacity, wl.budget,
+                            batch=wl.batch, q_heads=wl.q_heads, window=wl.window, engine=args.engine,
+                            seed=wl.policy_seed)
+    chunk = 4096
+    for t0 in range(0, wl.prompt_len, chunk):
+        k, v = synth_device.prompt(wl, t0, min(chunk, wl.prompt_len - t0))
+        cache.append(k, v)
+        del k, v
+    host = [tuple(x.cpu().pin_memory() for x in inp) for inp in inputs]
+    out = torch.empty((wl.layers, wl.batch, wl.q_heads, wl.head_dim), dtype=torch.float32).pin_memory()
+    W, K = args.warmup, args.steps
+    for s in range(0, 1 + W):
+        cache.decode_step_host(*host[s], out)
+        cache.evict()
+    torch.cuda.synchronize()
+    t0 = time.perf_counter()
+    for s in range(1 + W, 1 + W + K):
+        cache.decode_step_host(*host[s], out)
+        cache.evict()
+    cache.sync()
+    el = time.perf_counter() - t0
+    h2d = sum(x.numel() * x.element_size() for x in host[0])
+    d2h = out.numel() * out.element_size()
+    cache.close()
+    return {"value": K / el, "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
+            "ms_per_step": el / K * 1e3}
+
+
+def run_reference(args):
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return None
+    wl = workload()
+    cb = oracle_sample(wl, seconds=args.cpu_seconds)
+    return {"impl": "reference", "metric": METRIC, "value": cb["value"], "unit": UNIT,
+            "n_gpus": int(os.environ.get("WORLD_SIZE", "1")), "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": 1e3 / cb["value"], "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": {"workload": wl.name, "layers": wl.layers, "batch": wl.batch,
+                       "context": wl.prompt_len, "budget": wl.budget},
+            "cpu_baseline": cb,
+            "e2e": {"value": cb["value"], "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+
+
+def main():
+    ap = argparse.ArgumentParser(description=__doc__.splitlines()[0])
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=200)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--engine", type=int, default=0, help="0 fused, 1 split")
+    ap.add_argument("--cpu-seconds", type=float, default=12.0)
+    ap.add_argument("--no-cpu", action="store_true")
+    ap.add_argument("--no-full", action="store_true")
+    ap.add_argument("--no-e2e", action="store_true")
+    args = ap.parse_args()
+    if args.warmup < 3:
+        ap.error("--warmup must be >= 3")
+    if args.impl == "reference":
+        res = run_reference(args)
+        if res:
+            print(json.dumps(res), flush=True)
+        return
+    # the oracle's host threads start before any GPU work
+    cpu = None
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    if not args.no_cpu and rank == 0 and world == 1:
+        cpu = oracle_sample(workload(), seconds=args.cpu_seconds)
+    res = run_gpu(args)
+    if res is not None:
+        res["cpu_baseline"] = cpu
+        print(json.dumps(res), flush=True)
+
+
+if __name__ == "__main__":
+    main()

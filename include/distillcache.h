@@ -1,0 +1,199 @@
+/*
+ * distillcache.h -- C ABI of the GB300 (sm_103a) DistillCache decode step.
+ *
+ * A cache holds R = layers * batch * kv_heads independent rows. Each row is the
+ * key/value cache of one (layer, sequence, KV head) plus per-token eviction
+ * state. One decode step of the paper's inference loop (Algorithm 1) is
+ *
+ *     dc_decode_step   forward pass over C_t (the cache including the new
+ *                      pair), token features x_i and policy scores s_i;
+ *     dc_evict         argtop_B of the scores and prune of the cache.
+ *
+ * The problem statement (Sec. 3.1, Problem Formulation) asks for a pruned cache
+ * C'_t of at most B tokens; the features are those of Sec. 3.1.1 (State Space)
+ * and the policy is the MLP of Sec. 3.1.2 (Action Space) with the widths of
+ * App. D (Training Details).
+ *
+ * Conventions for every call:
+ *   - Pointers are DEVICE pointers unless the name says host. bf16 tensors are
+ *     passed as `const void*` holding IEEE bfloat16 values, row-major, densely
+ *     packed. The caller owns inputs and outputs; the library owns the cache,
+ *     its state, its scratch and the policy weights.
+ *   - Work is enqueued on the stream given at creation (cfg->stream, a
+ *     cudaStream_t; NULL is the legacy default stream) and is asynchronous,
+ *     except where a call says it synchronises.
+ *   - Every call returns a dc_status. No C++ exception crosses the ABI. A CUDA
+ *     error makes the handle unusable: later calls return DC_ERR_CUDA and
+ *     dc_last_error() gives the message. Invalid arguments leave the cache
+ *     unchanged.
+ *   - Calls on one handle must not run concurrently from several host threads.
+ */
+#ifndef DISTILLCACHE_H
+#define DISTILLCACHE_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+  DC_OK = 0,
+  DC_ERR_INVALID_ARG = 1, /* bad pointer, size or shape; nothing was done */
+  DC_ERR_CAPACITY = 2,    /* the rows would exceed `capacity` tokens */
+  DC_ERR_OOM = 3,         /* device allocation failed at creation */
+  DC_ERR_CUDA = 4,        /* a CUDA call failed; the handle is now unusable */
+  DC_ERR_DEVICE = 5,      /* a kernel reported an error through its status word */
+  DC_ERR_STATE = 6        /* call out of order (e.g. evict with no scores) */
+} dc_status;
+
+typedef struct dc_cache dc_cache;
+
+typedef struct {
+  int batch;          /* sequences per layer (default 1) */
+  int q_heads;        /* query heads per layer (default 4 * kv_heads) */
+  int window;         /* w of the entropy feature H_i (default 64, Sec. 3.1.1) */
+  int mlp_hidden;     /* hidden width of the policy MLP (default 128, App. D) */
+  int layernorm;      /* 1: LayerNorm after the first layer (default, App. D) */
+  int alpha_mode;     /* 0: alpha_i from the most recent pass (Sec. 3.1.1, default);
+                         1: cumulative since insertion */
+  int engine;         /* 0: fused (one kernel streams K/V once per step, default);
+                         1: split (separate attention, feature and scoring kernels) */
+  int keep_features;  /* 1: also store x_i [R][capacity][5] fp32 for inspection */
+  unsigned long long seed; /* policy weight seed (dc_policy_init) */
+  void* stream;       /* cudaStream_t */
+} dc_config;
+
+/* Fills *cfg with the defaults above (batch 1, q_heads 0 meaning 4 * kv_heads,
+ * seed 0, stream NULL). */
+dc_status dc_config_default(dc_config* cfg);
+
+/* Creates a cache of `layers` x cfg->batch x `kv_heads` rows, each able to hold
+ * `capacity` tokens of `head_dim` dimensions, with default budget `budget`.
+ * Requirements: head_dim in {64, 128}; q_heads % kv_heads == 0 and
+ * q_heads / kv_heads in {1, 2, 4, 8}; 1 <= budget < capacity; window in
+ * [1, 1024]; mlp_hidden in [1, 256] and a multiple of 32 when >= 32.
+ * The policy weights are initialised from cfg->seed as dc_policy_init does.
+ * Synchronises the device once (allocation). cfg may be NULL (defaults). */
+dc_status dc_cache_create(int layers, int kv_heads, int head_dim, int capacity, int budget,
+                          const dc_config* cfg, dc_cache** out);
+
+/* Frees every device buffer of the handle (synchronises its stream). NULL is a
+ * no-op. A handle must not be used after it is destroyed. */
+dc_status dc_cache_destroy(dc_cache* h);
+
+/* Number of floats in a policy blob of hidden width H: 9 * H + 1. Layout
+ * (fp32): [W1 (H x 5, row-major) | b1 (H) | gamma (H) | beta (H) | w2 (H) | b2],
+ * i.e. s = w2 . relu(LN(W1 x + b1) * gamma + beta) + b2, with the feature order
+ * x = [alpha, |v|_2, sigma, H, pos] (Sec. 3.1.1). */
+size_t dc_policy_blob_len(int hidden);
+
+/* Host-only: the seeded initial weights. Linear layers draw uniformly from
+ * [-1/sqrt(fan_in), 1/sqrt(fan_in)] (PyTorch's default rule) from a
+ * SplitMix64 stream; gamma = 1, beta = 0. `host_out` holds n >= blob_len
+ * floats. Needs no GPU. */
+dc_status dc_policy_init(unsigned long long seed, int hidden, float* host_out, size_t n);
+
+/* Replaces the policy weights with a host fp32 blob of dc_policy_blob_len(H)
+ * floats (H = cfg->mlp_hidden). The blob is copied before the call returns. */
+dc_status dc_policy_set_weights(dc_cache* h, const float* host_blob, size_t n);
+
+/* Appends n_tokens tokens to every row without queries (prompt loading).
+ * k, v: bf16 [layers][batch][kv_heads][n_tokens][head_dim]. Positions continue
+ * from the number of tokens seen. DC_ERR_CAPACITY (cache unchanged) if the
+ * rows would exceed capacity. */
+dc_status dc_append(dc_cache* h, const void* k, const void* v, int n_tokens);
+
+/* One decode step (Algorithm 1, forward pass, feature extraction and scoring):
+ * appends (k_new, v_new) to every row, attends with q over the whole unpruned
+ * row (the new token included), writes the attention output, updates the
+ * token features and scores every cached token. The scores stay on the device
+ * for dc_evict.
+ *   q:     bf16 [layers][batch][q_heads][head_dim]; query head j uses KV head
+ *          j / (q_heads / kv_heads).
+ *   k_new, v_new: bf16 [layers][batch][kv_heads][head_dim].
+ *   out:   fp32 [layers][batch][q_heads][head_dim].
+ * DC_ERR_CAPACITY (cache unchanged) if a row is full. */
+dc_status dc_decode_step(dc_cache* h, const void* q, const void* k_new, const void* v_new,
+                         float* out);
+
+/* The same step with HOST buffers of the same shapes (pinned memory is fastest);
+ * the copies run on the handle's stream and the call synchronises it before it
+ * returns, so `out_host` is ready. */
+dc_status dc_decode_step_host(dc_cache* h, const void* q_host, const void* k_new_host,
+                              const void* v_new_host, float* out_host);
+
+/* argtop_B and prune (Algorithm 1): every row keeps its min(n, B) highest-scored
+ * tokens (ties: lower position first; -0 equals +0; NaN ranks last) and
+ * compacts them into its first min(n, B) slots. Survivors below that bound do
+ * not move; each survivor above it moves into the lowest free slot, in
+ * ascending slot order. budget <= 0 uses the configured budget. Needs the
+ * scores of a decode step since the last append/evict (else DC_ERR_STATE). */
+dc_status dc_evict(dc_cache* h, int budget);
+
+/* Full-cache comparator: softmax attention of q over the current rows with no
+ * append, features or eviction (the "Full" row of the paper's latency table).
+ * q and out as in dc_decode_step. */
+dc_status dc_full_decode(dc_cache* h, const void* q, float* out);
+
+/* Current tokens per row (every row holds the same number) and tokens seen. */
+dc_status dc_get_length(dc_cache* h, int* n, long long* seen);
+
+typedef enum {
+  DC_BUF_K = 0,     /* bf16 [R][capacity][head_dim] */
+  DC_BUF_V = 1,     /* bf16 [R][capacity][head_dim] */
+  DC_BUF_POS = 2,   /* int32 [R][capacity] absolute position of each slot */
+  DC_BUF_S = 3,     /* fp64 [R][capacity] entropy-weighted window mass S_i */
+  DC_BUF_Z = 4,     /* fp64 [R][capacity] window mass Z_i */
+  DC_BUF_ACC = 5,   /* fp32 [R][capacity] cumulative alpha (alpha_mode 1) */
+  DC_BUF_SCORE = 6, /* fp32 [R][capacity] policy scores of the last step */
+  DC_BUF_FEAT = 7,  /* fp32 [R][capacity][5] features (keep_features only) */
+  DC_BUF_HQ = 8     /* fp32 [R][q_heads / kv_heads] entropy of each head, last step */
+} dc_buffer;
+
+/* Size in bytes of one row of an internal buffer (0 if the handle has none of
+ * it); every buffer above is laid out as [R][row]. */
+dc_status dc_buffer_bytes(dc_cache* h, dc_buffer which, size_t* row_bytes);
+
+/* Copies rows [row0, row0 + nrows) of an internal buffer into device memory
+ * `dst` of `bytes` bytes (bytes must equal nrows * row_bytes) on the handle's
+ * stream. DC_ERR_INVALID_ARG if the range is outside [0, R). */
+dc_status dc_copy_buffer(dc_cache* h, dc_buffer which, int row0, int nrows, void* dst, size_t bytes);
+
+/* Kernel phases of the calls above, for launch counting and timing. */
+typedef enum {
+  DC_PHASE_APPEND = 0,  /* new pairs written into the rows */
+  DC_PHASE_ATTEND = 1,  /* attention pass over K (split) or the whole fused step */
+  DC_PHASE_STATS = 2,   /* softmax statistics and window-ring push (split) */
+  DC_PHASE_SCORE = 3,   /* attention output, features and policy scores (split) */
+  DC_PHASE_COMBINE = 4, /* per-split output merge (split) */
+  DC_PHASE_EVICT = 5,   /* top-B select and compaction */
+  DC_PHASE_FULL = 6,    /* full-cache comparator */
+  DC_PHASE_COUNT = 7
+} dc_phase;
+
+/* Name of a phase ("append", "attend", ...), or "" if out of range. */
+const char* dc_phase_name(int phase);
+
+/* Turns per-launch CUDA-event timing on (1) or off (0) and zeroes the
+ * counters. Events are recorded on the handle's stream around every kernel. */
+dc_status dc_profile_enable(dc_cache* h, int on);
+
+/* Synchronises the stream and reads, per phase, the summed kernel time in ms
+ * (timed launches only) and the number of launches since the last enable.
+ * ms and launches each hold DC_PHASE_COUNT values (either may be NULL). */
+dc_status dc_profile_read(dc_cache* h, double* ms, long long* launches);
+
+/* Waits for all work enqueued on the handle's stream; reports any device
+ * status the kernels raised (DC_ERR_DEVICE). */
+dc_status dc_sync(dc_cache* h);
+
+/* Message of the last error on the handle (or of the last failed create when
+ * h is NULL). Valid until the next call on the handle. */
+const char* dc_last_error(const dc_cache* h);
+
+#ifdef __cplusplus
+}
+#endif
+#endif

@@ -1,0 +1,92 @@
+"""Builds the CUDA libraries in-tree with nvcc for sm_103a.
+
+* ``libdistillcache.so`` -- the decode-step kernels and the C ABI of
+  ``include/distillcache.h``;
+* ``libdc_synth.so``     -- the device side of the seeded input generator.
+
+Each translation unit compiles in parallel; nothing is installed elsewhere.
+"""
+
+from __future__ import annotations
+
+import concurrent.futures as cf
+import os
+import shutil
+import subprocess
+import sys
+
+HERE = os.path.dirname(os.path.abspath(__file__))
+CSRC = os.path.join(HERE, "csrc")
+BUILD = os.path.join(HERE, "_build")
+INCLUDE = os.path.join(os.path.dirname(HERE), "include")
+
+LIB_MAIN = os.path.join(HERE, "libdistillcache.so")
+LIB_SYNTH = os.path.join(HERE, "libdc_synth.so")
+
+MAIN_SOURCES = ["dc_cache.cu", "dc_split.cu", "dc_evict.cu", "dc_full.cu"]
+SYNTH_SOURCES = ["synth.cu"]
+
+ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
+NVCC_FLAGS = ARCH + ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-Xcompiler", "-O2",
+                     "--expt-relaxed-constexpr", "-I", CSRC, "-I", INCLUDE]
+
+
+def nvcc() -> str:
+    for cand in (os.environ.get("NVCC"), shutil.which("nvcc"), "/usr/local/cuda/bin/nvcc"):
+        if cand and os.path.exists(cand):
+            return cand
+    raise RuntimeError("nvcc not found")
+
+
+def _deps() -> list[str]:
+    out = []
+    for d in (CSRC, INCLUDE):
+        for f in os.listdir(d):
+            if f.endswith((".cu", ".cuh", ".h")):
+                out.append(os.path.join(d, f))
+    return out
+
+
+def _stale(target: str, inputs: list[str]) -> bool:
+    if not os.path.exists(target):
+        return True
+    t = os.path.getmtime(target)
+    return any(os.path.getmtime(i) > t for i in inputs)
+
+
+def _compile(src: str, extra: list[str], verbose: bool) -> str:
+    obj = os.path.join(BUILD, os.path.basename(src).replace(".cu", ".o"))
+    if _stale(obj, _deps()):
+        cmd = [nvcc()] + NVCC_FLAGS + extra + ["-c", os.path.join(CSRC, src), "-o", obj]
+        if verbose:
+            cmd.insert(1, "-Xptxas=-v")
+        res = subprocess.run(cmd, capture_output=True, text=True)
+        if res.returncode != 0:
+            raise RuntimeError(f"nvcc failed for {src}:\n{res.stdout}\n{res.stderr}")
+        if verbose and res.stderr:
+            sys.stderr.write(res.stderr)
+    return obj
+
+
+def _link(objs: list[str], target: str, libs: list[str]) -> None:
+    if _stale(target, objs):
+        tmp = target + f".tmp{os.getpid()}"
+        cmd = [nvcc()] + ARCH + ["-shared", "-o", tmp] + objs + libs
+        res = subprocess.run(cmd, capture_output=True, text=True)
+        if res.returncode != 0:
+            raise RuntimeError(f"link of {target} failed:\n{res.stdout}\n{res.stderr}")
+        os.replace(tmp, target)
+
+
+def build(verbose: bool = False) -> tuple[str, str]:
+    os.makedirs(BUILD, exist_ok=True)
+    srcs = MAIN_SOURCES + SYNTH_SOURCES
+    with cf.ThreadPoolExecutor(max_workers=min(8, len(srcs))) as ex:
+        objs = dict(zip(srcs, ex.map(lambda s: _compile(s, [], verbose), srcs)))
+    _link([objs[s] for s in MAIN_SOURCES], LIB_MAIN, [])
+    _link([objs[s] for s in SYNTH_SOURCES], LIB_SYNTH, [])
+    return LIB_MAIN, LIB_SYNTH
+
+
+if __name__ == "__main__":
+    print(build(verbose="-v" in sys.argv))

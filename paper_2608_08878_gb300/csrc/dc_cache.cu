@@ -1,0 +1,513 @@
+// dc_cache.cu -- host side of the C ABI (include/distillcache.h): the cache
+// handle, its device buffers, argument checks, status codes and the launch
+// sequence of each call.
+#include <cuda_runtime.h>
+
+#include <cmath>
+#include <cstdio>
+#include <cstring>
+#include <string>
+#include <vector>
+
+#include "../../include/distillcache.h"
+#include "dc_common.cuh"
+#include "dc_kernels.h"
+
+namespace {
+
+constexpr unsigned kMagic = 0x44434331u;  // "DCC1"
+constexpr unsigned kDead = 0xDEADDEADu;
+
+thread_local std::string g_create_error;
+
+// SplitMix64 output function (Steele, Lea, Flood).
+uint64_t splitmix64(uint64_t x) {
+  uint64_t z = x + 0x9E3779B97F4A7C15ull;
+  z = (z ^ (z >> 30)) * 0xBF58476D1CE4E5B9ull;
+  z = (z ^ (z >> 27)) * 0x94D049BB133111EBull;
+  return z ^ (z >> 31);
+}
+
+constexpr uint64_t kTagPolicy = 0x504F4C00ull;
+
+}  // namespace
+
+struct dc_cache {
+  unsigned magic = kMagic;
+  int layers = 0, kv_heads = 0, head_dim = 0, capacity = 0, budget = 0;
+  dc_config cfg{};
+  cudaStream_t stream = nullptr;
+  int num_sms = 0;
+  dc::Dev dev{};
+  // host-side state (every row holds the same number of tokens)
+  int n = 0;
+  long long seen = 0;
+  long long steps = 0;
+  bool have_scores = false;
+  std::vector<int> ring_pnew;  // newest position at the step held by each ring slot
+  // staging for dc_decode_step_host
+  void* st_q = nullptr;
+  void* st_k = nullptr;
+  void* st_v = nullptr;
+  float* st_out = nullptr;
+  std::vector<void*> allocs;
+  std::string err;
+  bool broken = false;
+  // launch counting and optional per-launch event timing
+  long long launches[DC_PHASE_COUNT] = {};
+  bool profiling = false;
+  struct Timed { int phase; cudaEvent_t a, b; };
+  std::vector<Timed> timed;
+  std::vector<cudaEvent_t> event_pool;
+  double ms[DC_PHASE_COUNT] = {};
+};
+
+namespace {
+
+dc_status fail(dc_cache* h, dc_status s, const std::string& msg) {
+  if (h) h->err = msg; else g_create_error = msg;
+  return s;
+}
+
+dc_status cuda_fail(dc_cache* h, cudaError_t e, const char* what) {
+  std::string m = std::string(what) + ": " + cudaGetErrorString(e);
+  if (h) { h->broken = true; h->err = m; } else g_create_error = m;
+  return DC_ERR_CUDA;
+}
+
+bool valid(const dc_cache* h) { return h && h->magic == kMagic; }
+
+#define DC_CHECK_HANDLE(h)                                                     \
+  do {                                                                         \
+    if (!valid(h)) return DC_ERR_INVALID_ARG;                                  \
+    if ((h)->broken) return DC_ERR_CUDA;                                       \
+  } while (0)
+
+#define DC_CUDA(h, call)                                                       \
+  do {                                                                         \
+    cudaError_t e_ = (call);                                                   \
+    if (e_ != cudaSuccess) return cuda_fail((h), e_, #call);                   \
+  } while (0)
+
+template <class T>
+cudaError_t dalloc(dc_cache* h, T** p, size_t bytes) {
+  void* q = nullptr;
+  cudaError_t e = cudaMalloc(&q, bytes ? bytes : 16);
+  if (e != cudaSuccess) return e;
+  h->allocs.push_back(q);
+  *p = (T*)q;
+  return cudaMemsetAsync(q, 0, bytes ? bytes : 16, h->stream);
+}
+
+void free_all(dc_cache* h) {
+  for (void* p : h->allocs) cudaFree(p);
+  h->allocs.clear();
+}
+
+// Split count and chunk (a multiple of 128 tokens) for n tokens per row.
+void split_plan(const dc_cache* h, int n, int* nsplit, int* chunk) {
+  int want = std::max(1, std::min(h->dev.smax, (n + 127) / 128));
+  int c = (n + want - 1) / want;
+  c = (c + 127) / 128 * 128;
+  if (c < 128) c = 128;
+  *chunk = c;
+  *nsplit = std::max(1, (n + c - 1) / c);
+}
+
+cudaEvent_t take_event(dc_cache* h) {
+  if (!h->event_pool.empty()) {
+    cudaEvent_t e = h->event_pool.back();
+    h->event_pool.pop_back();
+    return e;
+  }
+  cudaEvent_t e = nullptr;
+  cudaEventCreate(&e);
+  return e;
+}
+
+// Brackets the kernels of one phase: counts them and, when profiling, records
+// CUDA events around them on the handle's stream.
+struct Phase {
+  dc_cache* h;
+  int phase;
+  cudaEvent_t a = nullptr;
+  Phase(dc_cache* h_, int ph, int kernels) : h(h_), phase(ph) {
+    h->launches[ph] += kernels;
+    if (h->profiling) {
+      a = take_event(h);
+      cudaEventRecord(a, h->stream);
+    }
+  }
+  ~Phase() {
+    if (a) {
+      cudaEvent_t b = take_event(h);
+      cudaEventRecord(b, h->stream);
+      h->timed.push_back({phase, a, b});
+    }
+  }
+};
+
+dc_status launch_error(dc_cache* h, const char* what) {
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return cuda_fail(h, e, what);
+  return DC_OK;
+}
+
+bool run_split_step(dc_cache* h, const dc::Step& st, const void* q, float* out) {
+  const dc::Dev& p = h->dev;
+  if (!dc::split_supported(p)) return false;
+  { Phase ph(h, DC_PHASE_ATTEND, 1); dc::launch_split_qk(p, st, q, h->stream); }
+  { Phase ph(h, DC_PHASE_STATS, 1); dc::launch_split_stats(p, st, q, h->stream); }
+  { Phase ph(h, DC_PHASE_SCORE, 1); dc::launch_split_v(p, st, h->stream); }
+  { Phase ph(h, DC_PHASE_COMBINE, 1); dc::launch_split_out(p, st, out, h->stream); }
+  return true;
+}
+
+}  // namespace
+
+extern "C" {
+
+dc_status dc_config_default(dc_config* cfg) {
+  if (!cfg) return DC_ERR_INVALID_ARG;
+  std::memset(cfg, 0, sizeof *cfg);
+  cfg->batch = 1;
+  cfg->q_heads = 0;
+  cfg->window = 64;
+  cfg->mlp_hidden = 128;
+  cfg->layernorm = 1;
+  cfg->alpha_mode = 0;
+  cfg->engine = 0;
+  cfg->keep_features = 0;
+  cfg->seed = 0;
+  cfg->stream = nullptr;
+  return DC_OK;
+}
+
+size_t dc_policy_blob_len(int hidden) { return hidden > 0 ? (size_t)9 * hidden + 1 : 0; }
+
+dc_status dc_policy_init(unsigned long long seed, int hidden, float* out, size_t n) {
+  if (hidden <= 0 || !out || n < dc_policy_blob_len(hidden)) return DC_ERR_INVALID_ARG;
+  const int H = hidden;
+  uint64_t key = splitmix64(kTagPolicy);
+  key = splitmix64(key ^ (uint64_t)seed);
+  key = splitmix64(key ^ (uint64_t)H);
+  const float b1 = (float)(1.0 / std::sqrt(5.0));
+  const float b2 = (float)(1.0 / std::sqrt((double)H));
+  auto draw = [&](uint64_t j) {
+    float u = (float)(splitmix64(key + j) >> 40) / 16777216.0f;
+    return 2.0f * u - 1.0f;  // exact: u has 24 bits
+  };
+  uint64_t j = 0;
+  for (int i = 0; i < 5 * H; ++i) out[i] = draw(j++) * b1;            // W1
+  for (int i = 0; i < H; ++i) out[5 * H + i] = draw(j++) * b1;        // b1
+  for (int i = 0; i < H; ++i) out[6 * H + i] = 1.0f;                  // gamma
+  for (int i = 0; i < H; ++i) out[7 * H + i] = 0.0f;                  // beta
+  for (int i = 0; i < H; ++i) out[8 * H + i] = draw(j++) * b2;        // w2
+  out[9 * H] = draw(j++) * b2;                                        // b2
+  return DC_OK;
+}
+
+dc_status dc_cache_create(int layers, int kv_heads, int head_dim, int capacity, int budget,
+                          const dc_config* cfg_in, dc_cache** out) {
+  if (!out) return fail(nullptr, DC_ERR_INVALID_ARG, "out is NULL");
+  *out = nullptr;
+  dc_config cfg;
+  if (cfg_in) cfg = *cfg_in; else dc_config_default(&cfg);
+  if (cfg.q_heads == 0) cfg.q_heads = 4 * kv_heads;
+  if (layers < 1 || kv_heads < 1 || cfg.batch < 1)
+    return fail(nullptr, DC_ERR_INVALID_ARG, "layers, kv_heads and batch must be >= 1");
+  if (head_dim != 64 && head_dim != 128) return fail(nullptr, DC_ERR_INVALID_ARG, "head_dim must be 64 or 128");
+  if (cfg.q_heads % kv_heads) return fail(nullptr, DC_ERR_INVALID_ARG, "q_heads % kv_heads != 0");
+  const int G = cfg.q_heads / kv_heads;
+  if (G != 1 && G != 2 && G != 4 && G != 8) return fail(nullptr, DC_ERR_INVALID_ARG, "group must be 1, 2, 4 or 8");
+  if (budget < 1 || capacity <= budget) return fail(nullptr, DC_ERR_INVALID_ARG, "need 1 <= budget < capacity");
+  if (cfg.window < 1 || cfg.window > 1024) return fail(nullptr, DC_ERR_INVALID_ARG, "window must be in [1, 1024]");
+  if (cfg.mlp_hidden < 1 || cfg.mlp_hidden > 256 || (cfg.mlp_hidden >= 32 && cfg.mlp_hidden % 32))
+    return fail(nullptr, DC_ERR_INVALID_ARG, "mlp_hidden must be in [1, 256], a multiple of 32 when >= 32");
+  if (cfg.alpha_mode != 0 && cfg.alpha_mode != 1) return fail(nullptr, DC_ERR_INVALID_ARG, "alpha_mode must be 0 or 1");
+  if (cfg.engine != 0 && cfg.engine != 1) return fail(nullptr, DC_ERR_INVALID_ARG, "engine must be 0 or 1");
+  const long long R = (long long)layers * cfg.batch * kv_heads;
+  if (R > 65535 || (long long)capacity * R > (1ll << 40))
+    return fail(nullptr, DC_ERR_INVALID_ARG, "cache too large");
+
+  dc_cache* h = new dc_cache();
+  h->layers = layers; h->kv_heads = kv_heads; h->head_dim = head_dim;
+  h->capacity = capacity; h->budget = budget; h->cfg = cfg;
+  h->stream = (cudaStream_t)cfg.stream;
+  h->ring_pnew.assign(cfg.window, -1);
+  int dev_id = 0;
+  cudaError_t e = cudaGetDevice(&dev_id);
+  if (e == cudaSuccess) e = cudaDeviceGetAttribute(&h->num_sms, cudaDevAttrMultiProcessorCount, dev_id);
+  if (e != cudaSuccess) {
+    dc_status s = cuda_fail(nullptr, e, "cudaGetDevice");
+    delete h;
+    return s;
+  }
+  dc::Dev& p = h->dev;
+  p.R = (int)R; p.cap = capacity; p.d = head_dim; p.G = G; p.qh = cfg.q_heads; p.kvh = kv_heads;
+  p.w = cfg.window; p.hidden = cfg.mlp_hidden; p.layernorm = cfg.layernorm ? 1 : 0;
+  p.alpha_mode = cfg.alpha_mode; p.keep_features = cfg.keep_features ? 1 : 0;
+  p.c = (float)(1.4426950408889634 / std::sqrt((double)head_dim));
+  p.smax = (int)std::max(1ll, std::min(64ll, (8ll * h->num_sms + R - 1) / R));
+  const size_t RC = (size_t)R * capacity;
+  const size_t kv = RC * head_dim * sizeof(__nv_bfloat16);
+  const size_t blob = dc_policy_blob_len(cfg.mlp_hidden);
+  cudaError_t ae = cudaSuccess;
+  auto A = [&](auto** ptr, size_t bytes) { if (ae == cudaSuccess) ae = dalloc(h, ptr, bytes); };
+  A(&p.K, kv);
+  A(&p.V, kv);
+  A(&p.pos, RC * sizeof(int));
+  A(&p.S, RC * sizeof(double));
+  A(&p.Z, RC * sizeof(double));
+  if (cfg.alpha_mode == 1) A(&p.acc, RC * sizeof(float));
+  A(&p.score, RC * sizeof(float));
+  if (p.keep_features) A(&p.feat, RC * 5 * sizeof(float));
+  A(&p.hq, (size_t)R * G * sizeof(float));
+  A(&p.ring_q, (size_t)R * cfg.window * G * head_dim * sizeof(__nv_bfloat16));
+  A(&p.ring_stats, (size_t)R * cfg.window * G * 4 * sizeof(float));
+  float* pol = nullptr;
+  A(&pol, blob * sizeof(float));
+  p.policy = pol;
+  A(&p.status, sizeof(unsigned));
+  A(&p.logit, RC * G * sizeof(float));
+  A(&p.dep, RC * 2 * sizeof(float));
+  A(&p.part, (size_t)R * p.smax * G * 4 * sizeof(float));
+  A(&p.opart, (size_t)R * p.smax * G * head_dim * sizeof(float));
+  A(&p.holes, RC * sizeof(int));
+  A(&h->st_q, (size_t)R * G * head_dim * 2);
+  A(&h->st_k, (size_t)R * head_dim * 2);
+  A(&h->st_v, (size_t)R * head_dim * 2);
+  A(&h->st_out, (size_t)R * G * head_dim * sizeof(float));
+  if (ae != cudaSuccess) {
+    cudaGetLastError();
+    free_all(h);
+    std::string m = std::string("device allocation failed: ") + cudaGetErrorString(ae);
+    delete h;
+    return fail(nullptr, ae == cudaErrorMemoryAllocation ? DC_ERR_OOM : DC_ERR_CUDA, m);
+  }
+  std::vector<float> w(blob);
+  dc_policy_init(cfg.seed, cfg.mlp_hidden, w.data(), blob);
+  e = cudaMemcpyAsync(pol, w.data(), blob * sizeof(float), cudaMemcpyHostToDevice, h->stream);
+  if (e == cudaSuccess) e = cudaStreamSynchronize(h->stream);
+  if (e != cudaSuccess) {
+    dc_status s = cuda_fail(nullptr, e, "policy upload");
+    free_all(h);
+    delete h;
+    return s;
+  }
+  *out = h;
+  return DC_OK;
+}
+
+dc_status dc_cache_destroy(dc_cache* h) {
+  if (!h) return DC_OK;
+  if (!valid(h)) return DC_ERR_INVALID_ARG;
+  cudaStreamSynchronize(h->stream);
+  for (auto& t : h->timed) { cudaEventDestroy(t.a); cudaEventDestroy(t.b); }
+  for (auto e : h->event_pool) cudaEventDestroy(e);
+  free_all(h);
+  h->magic = kDead;
+  delete h;
+  return DC_OK;
+}
+
+dc_status dc_policy_set_weights(dc_cache* h, const float* blob, size_t n) {
+  DC_CHECK_HANDLE(h);
+  if (!blob || n != dc_policy_blob_len(h->cfg.mlp_hidden))
+    return fail(h, DC_ERR_INVALID_ARG, "policy blob must hold 9 * mlp_hidden + 1 floats");
+  DC_CUDA(h, cudaMemcpyAsync((void*)h->dev.policy, blob, n * sizeof(float), cudaMemcpyHostToDevice,
+                             h->stream));
+  DC_CUDA(h, cudaStreamSynchronize(h->stream));  // the caller may free the blob on return
+  return DC_OK;
+}
+
+dc_status dc_append(dc_cache* h, const void* k, const void* v, int n_tokens) {
+  DC_CHECK_HANDLE(h);
+  if (n_tokens < 0 || (n_tokens > 0 && (!k || !v))) return fail(h, DC_ERR_INVALID_ARG, "bad append arguments");
+  if (((uintptr_t)k | (uintptr_t)v) & 15) return fail(h, DC_ERR_INVALID_ARG, "k and v must be 16-byte aligned");
+  if (n_tokens == 0) return DC_OK;
+  if ((long long)h->n + n_tokens > h->capacity) return fail(h, DC_ERR_CAPACITY, "append exceeds capacity");
+  if (h->seen + n_tokens > 0x7FFFFFFFll) return fail(h, DC_ERR_CAPACITY, "position counter overflow");
+  {
+    Phase ph(h, DC_PHASE_APPEND, 1);
+    dc::launch_append(h->dev, k, v, n_tokens, h->n, (int)h->seen, h->stream);
+  }
+  dc_status s = launch_error(h, "append");
+  if (s != DC_OK) return s;
+  h->n += n_tokens;
+  h->seen += n_tokens;
+  h->have_scores = false;
+  return DC_OK;
+}
+
+dc_status dc_decode_step(dc_cache* h, const void* q, const void* k_new, const void* v_new, float* out) {
+  DC_CHECK_HANDLE(h);
+  if (!q || !k_new || !v_new || !out) return fail(h, DC_ERR_INVALID_ARG, "NULL pointer");
+  if (((uintptr_t)k_new | (uintptr_t)v_new) & 15) return fail(h, DC_ERR_INVALID_ARG, "k_new and v_new must be 16-byte aligned");
+  if (h->n + 1 > h->capacity) return fail(h, DC_ERR_CAPACITY, "decode step exceeds capacity");
+  if (h->seen + 1 > 0x7FFFFFFFll) return fail(h, DC_ERR_CAPACITY, "position counter overflow");
+  {
+    Phase ph(h, DC_PHASE_APPEND, 1);
+    dc::launch_append(h->dev, k_new, v_new, 1, h->n, (int)h->seen, h->stream);
+  }
+  dc::Step st{};
+  st.n = h->n + 1;
+  st.p_newest = (int)h->seen;
+  st.slot = (int)(h->steps % h->cfg.window);
+  st.has_dep = h->steps >= h->cfg.window ? 1 : 0;
+  st.p_dep = h->ring_pnew[st.slot];
+  split_plan(h, st.n, &st.nsplit, &st.chunk);
+  if (!run_split_step(h, st, q, out)) return fail(h, DC_ERR_INVALID_ARG, "unsupported head_dim / group");
+  dc_status s = launch_error(h, "decode step");
+  if (s != DC_OK) return s;
+  h->n += 1;
+  h->seen += 1;
+  h->ring_pnew[st.slot] = st.p_newest;
+  h->steps += 1;
+  h->have_scores = true;
+  return DC_OK;
+}
+
+dc_status dc_decode_step_host(dc_cache* h, const void* q, const void* k_new, const void* v_new,
+                              float* out) {
+  DC_CHECK_HANDLE(h);
+  if (!q || !k_new || !v_new || !out) return fail(h, DC_ERR_INVALID_ARG, "NULL pointer");
+  const size_t R = h->dev.R, G = h->dev.G, d = h->dev.d;
+  DC_CUDA(h, cudaMemcpyAsync(h->st_q, q, R * G * d * 2, cudaMemcpyHostToDevice, h->stream));
+  DC_CUDA(h, cudaMemcpyAsync(h->st_k, k_new, R * d * 2, cudaMemcpyHostToDevice, h->stream));
+  DC_CUDA(h, cudaMemcpyAsync(h->st_v, v_new, R * d * 2, cudaMemcpyHostToDevice, h->stream));
+  dc_status s = dc_decode_step(h, h->st_q, h->st_k, h->st_v, h->st_out);
+  if (s != DC_OK) return s;
+  DC_CUDA(h, cudaMemcpyAsync(out, h->st_out, R * G * d * sizeof(float), cudaMemcpyDeviceToHost, h->stream));
+  DC_CUDA(h, cudaStreamSynchronize(h->stream));
+  return DC_OK;
+}
+
+dc_status dc_evict(dc_cache* h, int budget) {
+  DC_CHECK_HANDLE(h);
+  if (!h->have_scores) return fail(h, DC_ERR_STATE, "evict needs the scores of a decode step");
+  const int B = budget <= 0 ? h->budget : budget;
+  const int keep = std::min(h->n, B);
+  if (keep < h->n) {
+    Phase ph(h, DC_PHASE_EVICT, 1);
+    dc::launch_evict(h->dev, h->n, keep, h->stream);
+    dc_status s = launch_error(h, "evict");
+    if (s != DC_OK) return s;
+  }
+  h->n = keep;
+  h->have_scores = false;
+  return DC_OK;
+}
+
+dc_status dc_full_decode(dc_cache* h, const void* q, float* out) {
+  DC_CHECK_HANDLE(h);
+  if (!q || !out) return fail(h, DC_ERR_INVALID_ARG, "NULL pointer");
+  if (h->n < 1) return fail(h, DC_ERR_STATE, "the cache is empty");
+  int nsplit, chunk;
+  split_plan(h, h->n, &nsplit, &chunk);
+  bool ok;
+  {
+    Phase ph(h, DC_PHASE_FULL, 2);
+    ok = dc::launch_full_decode(h->dev, h->n, nsplit, chunk, q, out, h->stream);
+  }
+  if (!ok) return fail(h, DC_ERR_INVALID_ARG, "unsupported head_dim / group");
+  return launch_error(h, "full decode");
+}
+
+dc_status dc_get_length(dc_cache* h, int* n, long long* seen) {
+  if (!valid(h)) return DC_ERR_INVALID_ARG;
+  if (n) *n = h->n;
+  if (seen) *seen = h->seen;
+  return DC_OK;
+}
+
+// Base pointer and bytes per row of an internal buffer.
+static char* buffer_ptr(dc_cache* h, dc_buffer which, size_t* row_bytes) {
+  const dc::Dev& p = h->dev;
+  const size_t C = (size_t)p.cap;
+  switch (which) {
+    case DC_BUF_K: *row_bytes = C * p.d * 2; return (char*)p.K;
+    case DC_BUF_V: *row_bytes = C * p.d * 2; return (char*)p.V;
+    case DC_BUF_POS: *row_bytes = C * sizeof(int); return (char*)p.pos;
+    case DC_BUF_S: *row_bytes = C * sizeof(double); return (char*)p.S;
+    case DC_BUF_Z: *row_bytes = C * sizeof(double); return (char*)p.Z;
+    case DC_BUF_ACC: *row_bytes = p.acc ? C * sizeof(float) : 0; return (char*)p.acc;
+    case DC_BUF_SCORE: *row_bytes = C * sizeof(float); return (char*)p.score;
+    case DC_BUF_FEAT: *row_bytes = p.feat ? C * 5 * sizeof(float) : 0; return (char*)p.feat;
+    case DC_BUF_HQ: *row_bytes = (size_t)p.G * sizeof(float); return (char*)p.hq;
+  }
+  *row_bytes = 0;
+  return nullptr;
+}
+
+dc_status dc_buffer_bytes(dc_cache* h, dc_buffer which, size_t* row_bytes) {
+  if (!valid(h) || !row_bytes) return DC_ERR_INVALID_ARG;
+  buffer_ptr(h, which, row_bytes);
+  return DC_OK;
+}
+
+dc_status dc_copy_buffer(dc_cache* h, dc_buffer which, int row0, int nrows, void* dst, size_t bytes) {
+  DC_CHECK_HANDLE(h);
+  size_t rb = 0;
+  char* src = buffer_ptr(h, which, &rb);
+  if (!src || rb == 0 || !dst) return fail(h, DC_ERR_INVALID_ARG, "the cache has no such buffer");
+  if (row0 < 0 || nrows < 0 || row0 + nrows > h->dev.R || bytes != rb * (size_t)nrows)
+    return fail(h, DC_ERR_INVALID_ARG, "row range or size mismatch");
+  if (nrows == 0) return DC_OK;
+  DC_CUDA(h, cudaMemcpyAsync(dst, src + rb * (size_t)row0, bytes, cudaMemcpyDeviceToDevice, h->stream));
+  return DC_OK;
+}
+
+dc_status dc_sync(dc_cache* h) {
+  DC_CHECK_HANDLE(h);
+  DC_CUDA(h, cudaStreamSynchronize(h->stream));
+  unsigned st = 0;
+  DC_CUDA(h, cudaMemcpy(&st, h->dev.status, sizeof st, cudaMemcpyDeviceToHost));
+  if (st) {
+    char buf[96];
+    std::snprintf(buf, sizeof buf, "kernel status word 0x%x", st);
+    return fail(h, DC_ERR_DEVICE, buf);
+  }
+  return DC_OK;
+}
+
+const char* dc_phase_name(int phase) {
+  static const char* names[DC_PHASE_COUNT] = {"append", "attend", "stats", "score", "combine", "evict", "full"};
+  return (phase >= 0 && phase < DC_PHASE_COUNT) ? names[phase] : "";
+}
+
+dc_status dc_profile_enable(dc_cache* h, int on) {
+  DC_CHECK_HANDLE(h);
+  DC_CUDA(h, cudaStreamSynchronize(h->stream));
+  for (auto& t : h->timed) { h->event_pool.push_back(t.a); h->event_pool.push_back(t.b); }
+  h->timed.clear();
+  for (int i = 0; i < DC_PHASE_COUNT; ++i) { h->launches[i] = 0; h->ms[i] = 0.0; }
+  h->profiling = on != 0;
+  return DC_OK;
+}
+
+dc_status dc_profile_read(dc_cache* h, double* ms, long long* launches) {
+  DC_CHECK_HANDLE(h);
+  DC_CUDA(h, cudaStreamSynchronize(h->stream));
+  for (auto& t : h->timed) {
+    float x = 0.f;
+    DC_CUDA(h, cudaEventElapsedTime(&x, t.a, t.b));
+    h->ms[t.phase] += x;
+    h->event_pool.push_back(t.a);
+    h->event_pool.push_back(t.b);
+  }
+  h->timed.clear();
+  for (int i = 0; i < DC_PHASE_COUNT; ++i) {
+    if (ms) ms[i] = h->ms[i];
+    if (launches) launches[i] = h->launches[i];
+  }
+  return DC_OK;
+}
+
+const char* dc_last_error(const dc_cache* h) {
+  if (!h) return g_create_error.c_str();
+  if (!valid(h)) return "invalid handle";
+  return h->err.c_str();
+}
+
+}  // extern "C"

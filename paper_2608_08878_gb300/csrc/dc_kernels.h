@@ -1,0 +1,26 @@
+// dc_kernels.h -- host-side launchers of the decode-step kernels.
+#pragma once
+
+#include <cuda_runtime.h>
+
+#include "dc_common.cuh"
+
+namespace dc {
+
+void launch_append(const Dev& p, const void* k, const void* v, int T, int n0, int seen0,
+                   cudaStream_t s);
+
+// Split engine: attention + features + scores of one decode step (after the
+// append), one launcher per kernel.
+bool split_supported(const Dev& p);
+void launch_split_qk(const Dev& p, const Step& st, const void* q, cudaStream_t s);
+void launch_split_stats(const Dev& p, const Step& st, const void* q, cudaStream_t s);
+void launch_split_v(const Dev& p, const Step& st, cudaStream_t s);
+void launch_split_out(const Dev& p, const Step& st, float* out, cudaStream_t s);
+
+void launch_evict(const Dev& p, int n, int B, cudaStream_t s);
+
+bool launch_full_decode(const Dev& p, int n, int nsplit, int chunk, const void* q, float* out,
+                        cudaStream_t s);
+
+}  // namespace dc

@@ -1,0 +1,230 @@
+"""Python binding of the C ABI in ``include/distillcache.h`` (argument
+marshalling only: every step of the decode path runs in the CUDA library).
+
+Device memory and streams come from PyTorch; tensors are passed to the library
+as raw device pointers. There is no CPU fallback: if ``libdistillcache.so`` is
+missing, opening it raises.
+"""
+
+from __future__ import annotations
+
+import ctypes as C
+import os
+import threading
+
+import numpy as np
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_HERE, "libdistillcache.so")
+
+DC_OK, DC_ERR_INVALID_ARG, DC_ERR_CAPACITY, DC_ERR_OOM, DC_ERR_CUDA, DC_ERR_DEVICE, DC_ERR_STATE = range(7)
+STATUS_NAMES = ["DC_OK", "DC_ERR_INVALID_ARG", "DC_ERR_CAPACITY", "DC_ERR_OOM", "DC_ERR_CUDA",
+                "DC_ERR_DEVICE", "DC_ERR_STATE"]
+
+BUF_K, BUF_V, BUF_POS, BUF_S, BUF_Z, BUF_ACC, BUF_SCORE, BUF_FEAT, BUF_HQ = range(9)
+
+# Every function the header declares (checked by the tests).
+EXPORTS = ["dc_config_default", "dc_cache_create", "dc_cache_destroy", "dc_policy_blob_len",
+           "dc_policy_init", "dc_policy_set_weights", "dc_append", "dc_decode_step",
+           "dc_decode_step_host", "dc_evict", "dc_full_decode", "dc_get_length", "dc_buffer_bytes",
+           "dc_copy_buffer", "dc_sync", "dc_last_error", "dc_phase_name", "dc_profile_enable",
+           "dc_profile_read"]
+PHASES = ["append", "attend", "stats", "score", "combine", "evict", "full"]
+
+
+class dc_config(C.Structure):
+    _fields_ = [("batch", C.c_int), ("q_heads", C.c_int), ("window", C.c_int),
+                ("mlp_hidden", C.c_int), ("layernorm", C.c_int), ("alpha_mode", C.c_int),
+                ("engine", C.c_int), ("keep_features", C.c_int), ("seed", C.c_ulonglong),
+                ("stream", C.c_void_p)]
+
+
+class DCError(RuntimeError):
+    def __init__(self, status: int, msg: str):
+        self.status = status
+        name = STATUS_NAMES[status] if 0 <= status < len(STATUS_NAMES) else str(status)
+        super().__init__(f"{name}: {msg}")
+
+
+_lib = None
+_lock = threading.Lock()
+
+
+def lib():
+    """Opens libdistillcache.so (raises if it has not been built)."""
+    global _lib
+    with _lock:
+        if _lib is None:
+            if not os.path.exists(LIB_PATH):
+                raise OSError(f"{LIB_PATH} is missing: build it with "
+                              "`python -m paper_2608_08878_gb300.build`")
+            L = C.CDLL(LIB_PATH)
+            P, I, S = C.c_void_p, C.c_int, C.c_size_t
+            L.dc_config_default.argtypes = [C.POINTER(dc_config)]
+            L.dc_cache_create.argtypes = [I, I, I, I, I, C.POINTER(dc_config), C.POINTER(P)]
+            L.dc_cache_destroy.argtypes = [P]
+            L.dc_policy_blob_len.argtypes = [I]
+            L.dc_policy_blob_len.restype = S
+            L.dc_policy_init.argtypes = [C.c_ulonglong, I, P, S]
+            L.dc_policy_set_weights.argtypes = [P, P, S]
+            L.dc_append.argtypes = [P, P, P, I]
+            L.dc_decode_step.argtypes = [P, P, P, P, P]
+            L.dc_decode_step_host.argtypes = [P, P, P, P, P]
+            L.dc_evict.argtypes = [P, I]
+            L.dc_full_decode.argtypes = [P, P, P]
+            L.dc_get_length.argtypes = [P, C.POINTER(I), C.POINTER(C.c_longlong)]
+            L.dc_buffer_bytes.argtypes = [P, I, C.POINTER(S)]
+            L.dc_copy_buffer.argtypes = [P, I, I, I, P, S]
+            L.dc_sync.argtypes = [P]
+            L.dc_last_error.argtypes = [P]
+            L.dc_last_error.restype = C.c_char_p
+            L.dc_phase_name.argtypes = [I]
+            L.dc_phase_name.restype = C.c_char_p
+            L.dc_profile_enable.argtypes = [P, I]
+            L.dc_profile_read.argtypes = [P, P, P]
+            for name in EXPORTS:
+                if name not in ("dc_policy_blob_len", "dc_last_error", "dc_phase_name"):
+                    getattr(L, name).restype = I
+            _lib = L
+    return _lib
+
+
+def policy_blob_len(hidden: int) -> int:
+    return int(lib().dc_policy_blob_len(hidden))
+
+
+def policy_init(seed: int, hidden: int) -> np.ndarray:
+    """The library's seeded initial policy weights (host-only, no GPU needed)."""
+    n = policy_blob_len(hidden)
+    out = np.empty(n, dtype=np.float32)
+    st = lib().dc_policy_init(seed, hidden, out.ctypes.data_as(C.c_void_p), n)
+    if st != DC_OK:
+        raise DCError(st, "dc_policy_init rejected its arguments")
+    return out
+
+
+def _ptr(t) -> int:
+    return 0 if t is None else int(t.data_ptr())
+
+
+class DistillCache:
+    """A budgeted KV cache of ``layers x batch x kv_heads`` rows on the current
+    CUDA device, driven through the C ABI on one CUDA stream."""
+
+    def __init__(self, layers: int, kv_heads: int, head_dim: int, capacity: int, budget: int, *,
+                 batch: int = 1, q_heads: int | None = None, window: int = 64,
+                 mlp_hidden: int = 128, layernorm: int = 1, alpha_mode: int = 0, engine: int = 0,
+                 keep_features: bool = False, seed: int = 0, stream=None):
+        import torch
+        L = lib()
+        cfg = dc_config()
+        L.dc_config_default(C.byref(cfg))
+        cfg.batch, cfg.q_heads, cfg.window = batch, q_heads or 4 * kv_heads, window
+        cfg.mlp_hidden, cfg.layernorm, cfg.alpha_mode = mlp_hidden, layernorm, alpha_mode
+        cfg.engine, cfg.keep_features, cfg.seed = engine, int(bool(keep_features)), seed
+        if stream is None:
+            stream = torch.cuda.current_stream()
+        self.stream = stream
+        cfg.stream = stream.cuda_stream
+        h = C.c_void_p()
+        st = L.dc_cache_create(layers, kv_heads, head_dim, capacity, budget, C.byref(cfg), C.byref(h))
+        if st != DC_OK:
+            raise DCError(st, L.dc_last_error(None).decode())
+        self._h = h
+        self.layers, self.kv_heads, self.head_dim = layers, kv_heads, head_dim
+        self.capacity, self.budget, self.batch = capacity, budget, batch
+        self.q_heads = cfg.q_heads
+        self.group = self.q_heads // kv_heads
+        self.rows = layers * batch * kv_heads
+        self.mlp_hidden = mlp_hidden
+
+    # -- lifetime ----------------------------------------------------------
+    def close(self) -> None:
+        if getattr(self, "_h", None):
+            lib().dc_cache_destroy(self._h)
+            self._h = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+    def __enter__(self):
+        return self
+
+    def __exit__(self, *a):
+        self.close()
+
+    def _check(self, st: int) -> None:
+        if st != DC_OK:
+            raise DCError(st, lib().dc_last_error(self._h).decode())
+
+    # -- the ABI -----------------------------------------------------------
+    def set_policy(self, blob: np.ndarray) -> None:
+        blob = np.ascontiguousarray(blob, dtype=np.float32)
+        self._check(lib().dc_policy_set_weights(self._h, blob.ctypes.data_as(C.c_void_p), blob.size))
+
+    def append(self, k, v) -> None:
+        """k, v: bf16 CUDA tensors [layers][batch][kv_heads][T][head_dim]."""
+        T = int(k.shape[-2]) if k.numel() else 0
+        self._check(lib().dc_append(self._h, _ptr(k), _ptr(v), T))
+
+    def decode_step(self, q, k_new, v_new, out=None):
+        import torch
+        if out is None:
+            out = torch.empty(q.shape, dtype=torch.float32, device=q.device)
+        self._check(lib().dc_decode_step(self._h, _ptr(q), _ptr(k_new), _ptr(v_new), _ptr(out)))
+        return out
+
+    def decode_step_host(self, q, k_new, v_new, out) -> None:
+        """Host (preferably pinned) tensors; synchronises before returning."""
+        self._check(lib().dc_decode_step_host(self._h, _ptr(q), _ptr(k_new), _ptr(v_new), _ptr(out)))
+
+    def evict(self, budget: int = 0) -> None:
+        self._check(lib().dc_evict(self._h, budget))
+
+    def full_decode(self, q, out=None):
+        import torch
+        if out is None:
+            out = torch.empty(q.shape, dtype=torch.float32, device=q.device)
+        self._check(lib().dc_full_decode(self._h, _ptr(q), _ptr(out)))
+        return out
+
+    def length(self):
+        n, seen = C.c_int(), C.c_longlong()
+        self._check(lib().dc_get_length(self._h, C.byref(n), C.byref(seen)))
+        return n.value, seen.value
+
+    def profile(self, on: bool = True) -> None:
+        """Zeroes the launch counters; with on=True also times every launch."""
+        self._check(lib().dc_profile_enable(self._h, int(on)))
+
+    def profile_read(self) -> dict:
+        """{phase: (total kernel ms, launches)} since the last profile() call."""
+        ms = (C.c_double * len(PHASES))()
+        n = (C.c_longlong * len(PHASES))()
+        self._check(lib().dc_profile_read(self._h, ms, n))
+        return {PHASES[i]: (ms[i], n[i]) for i in range(len(PHASES))}
+
+    def sync(self) -> None:
+        self._check(lib().dc_sync(self._h))
+
+    def buffer(self, which: int, row0: int = 0, nrows: int | None = None):
+        """A device copy of rows [row0, row0 + nrows) of an internal buffer."""
+        import torch
+        if nrows is None:
+            nrows = self.rows - row0
+        rb = C.c_size_t()
+        self._check(lib().dc_buffer_bytes(self._h, which, C.byref(rb)))
+        cap, d, G = self.capacity, self.head_dim, self.group
+        spec = {BUF_K: (torch.bfloat16, (cap, d)), BUF_V: (torch.bfloat16, (cap, d)),
+                BUF_POS: (torch.int32, (cap,)), BUF_S: (torch.float64, (cap,)),
+                BUF_Z: (torch.float64, (cap,)), BUF_ACC: (torch.float32, (cap,)),
+                BUF_SCORE: (torch.float32, (cap,)), BUF_FEAT: (torch.float32, (cap, 5)),
+                BUF_HQ: (torch.float32, (G,))}[which]
+        if rb.value == 0:
+            raise DCError(DC_ERR_INVALID_ARG, "the cache has no such buffer")
+        out = torch.empty((nrows,) + spec[1], dtype=spec[0], device="cuda")
+        self._check(lib().dc_copy_buffer(self._h, which, row0, nrows, _ptr(out), rb.value * nrows))
+        return out

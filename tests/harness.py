@@ -1,0 +1,165 @@
+"""Lock-step runner: the CUDA path (through the C ABI) and the fp64 oracle on
+the same seeded inputs, compared step by step on a sample of rows."""
+
+from __future__ import annotations
+
+import math
+
+import numpy as np
+
+import oracle
+from paper_2608_08878_gb300 import synth
+
+# Tolerances (bf16 inputs, fp32 accumulation on the GPU, fp64 oracle).
+ATTN_MAX_ABS = 2e-2
+ATTN_REL_L2 = 1e-2
+FEAT_RTOL = 1e-3
+FEAT_FLOOR = 1e-3  # absolute floor as a fraction of the column's RMS over the row
+
+
+def close_rel(gpu, ref, rtol, floor_frac, what):
+    gpu = np.asarray(gpu, dtype=np.float64)
+    ref = np.asarray(ref, dtype=np.float64)
+    assert gpu.shape == ref.shape, (what, gpu.shape, ref.shape)
+    if ref.size == 0:
+        return
+    floor = floor_frac * math.sqrt(float(np.mean(ref ** 2)))
+    err = np.abs(gpu - ref)
+    tol = rtol * np.abs(ref) + floor
+    bad = ~(err <= tol)
+    if bad.any():
+        i = int(np.argmax(np.where(bad, err / np.maximum(tol, 1e-300), 0)))
+        raise AssertionError(f"{what}: {int(bad.sum())}/{bad.size} outside rtol {rtol} + floor {floor:.3g};"
+                             f" worst at {i}: gpu {gpu.flat[i]!r} ref {ref.flat[i]!r}")
+
+
+def check_attention(gpu_o, ref_o, what):
+    gpu_o = np.asarray(gpu_o, dtype=np.float64)
+    ref_o = np.asarray(ref_o, dtype=np.float64)
+    max_abs = float(np.max(np.abs(gpu_o - ref_o))) if ref_o.size else 0.0
+    rel = float(np.linalg.norm(gpu_o - ref_o) / max(np.linalg.norm(ref_o), 1e-30))
+    assert max_abs <= ATTN_MAX_ABS and rel <= ATTN_REL_L2, f"{what}: max-abs {max_abs:.3g} rel-L2 {rel:.3g}"
+    return max_abs, rel
+
+
+class LockStep:
+    """Drives a DistillCache and oracle rows for a sample of its rows."""
+
+    def __init__(self, wl: synth.Workload, rows, *, engine=0, device_inputs=False, capacity=None):
+        import torch
+        from paper_2608_08878_gb300 import dc, synth_device
+        self.torch, self.dc, self.sd = torch, dc, synth_device
+        self.wl = wl
+        self.rows = list(rows)
+        self.device_inputs = device_inputs
+        cap = capacity or wl.capacity
+        self.blob = synth.policy_weights(wl.policy_seed, wl.mlp_hidden)
+        self.cache = dc.DistillCache(wl.layers, wl.kv_heads, wl.head_dim, cap, wl.budget,
+                                     batch=wl.batch, q_heads=wl.q_heads, window=wl.window,
+                                     mlp_hidden=wl.mlp_hidden, layernorm=wl.layernorm,
+                                     alpha_mode=wl.alpha_mode, engine=engine, keep_features=True,
+                                     seed=wl.policy_seed)
+        self.cache.set_policy(self.blob)
+        self.orows = {}
+        for r in self.rows:
+            self.orows[r] = oracle.OracleRow(wl.head_dim, wl.group, wl.window, wl.alpha_mode, cap)
+        self.step_idx = 0
+        self.stats = {"attn_max_abs": 0.0, "attn_rel": 0.0, "steps": 0, "evicted": 0}
+
+    def load_prompt(self, chunk=8192):
+        wl, torch = self.wl, self.torch
+        if self.device_inputs:
+            for t0 in range(0, wl.prompt_len, chunk):
+                T = min(chunk, wl.prompt_len - t0)
+                k, v = self.sd.prompt(wl, t0, T)
+                self.cache.append(k, v)
+                del k, v
+        else:
+            k, v = synth.prompt_all(wl)
+            kt = torch.from_numpy(k.view(np.int16)).view(torch.bfloat16).cuda()
+            vt = torch.from_numpy(v.view(np.int16)).view(torch.bfloat16).cuda()
+            self.cache.append(kt, vt)
+        for r, orow in self.orows.items():
+            layer, b, g = wl.row_coords(r)
+            k, v = synth.prompt_row(wl, layer, b, g)
+            orow.append(k, v)
+
+    def _inputs(self, step):
+        wl, torch = self.wl, self.torch
+        if self.device_inputs:
+            return self.sd.step_inputs(wl, step)
+        q, kn, vn = synth.step_all(wl, step)
+        f = lambda a: torch.from_numpy(a.view(np.int16)).view(torch.bfloat16).cuda()
+        return f(q), f(kn), f(vn)
+
+    def _row_slice(self, which, r, n):
+        return self.cache.buffer(which, r, 1)[0, :n].cpu().numpy()
+
+    def step(self, evict=True, budget=0, check=True):
+        wl, dc = self.wl, self.dc
+        s = self.step_idx
+        q, kn, vn = self._inputs(s)
+        out = self.cache.decode_step(q, kn, vn)
+        n, _ = self.cache.length()
+        out_h = out.cpu().numpy()
+        G = wl.group
+        for r, orow in self.orows.items():
+            layer, b, g = wl.row_coords(r)
+            qb, knb, vnb = synth.step_row(wl, s, layer, b, g)
+            res = orow.step(qb, knb, vnb, self.blob, wl.mlp_hidden, wl.layernorm)
+            if not check:
+                continue
+            o_gpu = out_h[layer, b, g * G:(g + 1) * G]
+            ma, rel = check_attention(o_gpu, res["o"], f"step {s} row {r} attention")
+            self.stats["attn_max_abs"] = max(self.stats["attn_max_abs"], ma)
+            self.stats["attn_rel"] = max(self.stats["attn_rel"], rel)
+            hq = self.cache.buffer(dc.BUF_HQ, r, 1)[0].cpu().numpy()
+            close_rel(hq, res["Hq"], FEAT_RTOL, 0.0, f"step {s} row {r} entropy")
+            pos = self._row_slice(dc.BUF_POS, r, n)
+            order = np.argsort(pos, kind="stable")
+            assert np.array_equal(pos[order], res["pos"]), f"step {s} row {r}: positions differ"
+            feat = self._row_slice(dc.BUF_FEAT, r, n)[order]
+            names = ["alpha", "|v|", "sigma", "H", "pos"]
+            for c in range(5):
+                close_rel(feat[:, c], res["feat"][:, c], FEAT_RTOL, FEAT_FLOOR, f"step {s} row {r} {names[c]}")
+            score = self._row_slice(dc.BUF_SCORE, r, n)[order]
+            close_rel(score, res["score"], FEAT_RTOL, FEAT_FLOOR, f"step {s} row {r} score")
+        if evict:
+            self.evict(budget)
+        self.step_idx += 1
+        self.stats["steps"] += 1
+        return out
+
+    def evict(self, budget=0):
+        dc = self.dc
+        n, _ = self.cache.length()
+        gpu_scores = {}
+        for r in self.orows:
+            pos = self._row_slice(dc.BUF_POS, r, n)
+            sc = self._row_slice(dc.BUF_SCORE, r, n)
+            order = np.argsort(pos, kind="stable")
+            gpu_scores[r] = sc[order]
+        self.cache.evict(budget)
+        B = budget if budget > 0 else self.wl.budget
+        n2, _ = self.cache.length()
+        assert n2 == min(n, B)
+        self.stats["evicted"] += n - n2
+        for r, orow in self.orows.items():
+            orow.evict(B, gpu_scores[r])
+            self.check_row_state(r, n2)
+
+    def check_row_state(self, r, n):
+        dc = self.dc
+        orow = self.orows[r]
+        pos = self._row_slice(dc.BUF_POS, r, n)
+        order = np.argsort(pos, kind="stable")
+        assert np.array_equal(pos[order], orow.positions()), f"row {r}: retained positions differ"
+        K = self.cache.buffer(dc.BUF_K, r, 1)[0, :n].view(self.torch.int16).cpu().numpy().view(np.uint16)
+        V = self.cache.buffer(dc.BUF_V, r, 1)[0, :n].view(self.torch.int16).cpu().numpy().view(np.uint16)
+        ok, ov = orow.kv_bits()
+        assert np.array_equal(K[order], ok) and np.array_equal(V[order], ov), f"row {r}: K/V bytes differ"
+        S = self._row_slice(dc.BUF_S, r, n)[order]
+        Z = self._row_slice(dc.BUF_Z, r, n)[order]
+        oS, oZ, _ = orow.window_sums()
+        close_rel(Z, oZ, FEAT_RTOL, FEAT_FLOOR, f"row {r} window mass Z")
+        close_rel(S, oS, FEAT_RTOL, FEAT_FLOOR, f"row {r} window sum S")

@@ -1,0 +1,87 @@
+"""Host-side checks of the C ABI library (no GPU): it loads, exports every
+function the header declares, validates arguments before touching the device,
+and its seeded policy initialisation matches the input generator bit for bit."""
+
+import ctypes as C
+import os
+import re
+
+import numpy as np
+import pytest
+
+from paper_2608_08878_gb300 import dc, synth
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module", autouse=True)
+def built():
+    from paper_2608_08878_gb300 import build
+    build.build()
+
+
+def header_functions():
+    names = set()
+    inc = os.path.join(ROOT, "include")
+    for f in os.listdir(inc):
+        if f.endswith(".h"):
+            text = open(os.path.join(inc, f)).read()
+            text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+            names |= set(re.findall(r"\b(dc_[a-z_0-9]+)\s*\(", text))
+    return names
+
+
+def test_library_exports_every_declared_function():
+    L = dc.lib()
+    declared = header_functions()
+    assert declared, "no declarations found"
+    for name in sorted(declared):
+        assert hasattr(L, name), f"{name} is declared but not exported"
+    assert declared <= set(dc.EXPORTS) | set(), sorted(declared - set(dc.EXPORTS))
+
+
+def test_policy_init_matches_generator():
+    for seed, H in [(0, 128), (0, 64), (7, 32), (123456789, 256), (1, 5)]:
+        np.testing.assert_array_equal(dc.policy_init(seed, H), synth.policy_weights(seed, H))
+    assert dc.policy_blob_len(128) == 9 * 128 + 1
+
+
+def test_config_defaults():
+    cfg = dc.dc_config()
+    assert dc.lib().dc_config_default(C.byref(cfg)) == dc.DC_OK
+    assert (cfg.batch, cfg.q_heads, cfg.window, cfg.mlp_hidden, cfg.layernorm, cfg.alpha_mode,
+            cfg.engine, cfg.keep_features, cfg.seed) == (1, 0, 64, 128, 1, 0, 0, 0, 0)
+    assert dc.lib().dc_config_default(None) == dc.DC_ERR_INVALID_ARG
+
+
+@pytest.mark.parametrize("args,field", [
+    ((1, 8, 96, 100, 10), "head_dim"),
+    ((1, 8, 128, 10, 10), "budget"),
+    ((1, 8, 128, 10, 0), "budget"),
+    ((0, 8, 128, 100, 10), "layers"),
+])
+def test_create_rejects_bad_shapes_without_touching_the_device(args, field):
+    h = C.c_void_p()
+    st = dc.lib().dc_cache_create(*args, None, C.byref(h))
+    assert st == dc.DC_ERR_INVALID_ARG and not h.value
+    assert field in dc.lib().dc_last_error(None).decode()
+
+
+def test_create_rejects_bad_config():
+    L = dc.lib()
+    for field, value in [("q_heads", 12), ("window", 0), ("mlp_hidden", 100), ("alpha_mode", 2),
+                         ("engine", 5)]:
+        cfg = dc.dc_config()
+        L.dc_config_default(C.byref(cfg))
+        setattr(cfg, field, value)
+        h = C.c_void_p()
+        assert L.dc_cache_create(1, 8, 128, 100, 10, C.byref(cfg), C.byref(h)) == dc.DC_ERR_INVALID_ARG
+
+
+def test_null_handles_are_rejected():
+    L = dc.lib()
+    assert L.dc_cache_destroy(None) == dc.DC_OK
+    assert L.dc_evict(None, 1) == dc.DC_ERR_INVALID_ARG
+    assert L.dc_append(None, None, None, 0) == dc.DC_ERR_INVALID_ARG
+    assert L.dc_sync(None) == dc.DC_ERR_INVALID_ARG
+    assert L.dc_policy_init(0, 0, None, 0) == dc.DC_ERR_INVALID_ARG

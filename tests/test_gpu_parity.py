@@ -1,0 +1,181 @@
+"""CUDA path (through the C ABI) against the fp64 oracle on the same seeded
+inputs: attention output, per-head entropy, the five features, policy scores,
+the retained sets (oracle fed the GPU's scores), compacted K/V bytes and the
+window state. Small cases run every row; the full-size workloads run in the
+benchmark's launch configuration and check a sample of rows."""
+
+import numpy as np
+import pytest
+
+from paper_2608_08878_gb300 import synth
+
+from harness import LockStep, check_attention
+
+pytestmark = pytest.mark.gpu
+
+ENGINES = [0, 1]
+
+
+@pytest.fixture(scope="module", autouse=True)
+def built():
+    from paper_2608_08878_gb300 import build
+    build.build()
+    import torch
+    torch.cuda.init()
+
+
+def _bits(t):
+    import torch
+    return t.view(torch.int16).cpu().numpy().view(np.uint16)
+
+
+def test_device_generator_matches_host():
+    from paper_2608_08878_gb300 import synth_device
+    for wl in (synth.TINY, synth.MISTRAL_1L.with_(prompt_len=300), synth.AGGRESSIVE.with_(layers=2, batch=2)):
+        k, v = synth_device.prompt(wl, 0, min(wl.prompt_len, 300))
+        kb, vb = _bits(k), _bits(v)
+        for r in (0, wl.rows - 1, wl.rows // 2):
+            layer, b, g = wl.row_coords(r)
+            hk, hv = synth.prompt_row(wl, layer, b, g, 0, min(wl.prompt_len, 300))
+            assert np.array_equal(kb[layer, b, g], hk) and np.array_equal(vb[layer, b, g], hv)
+        for step in (0, 17, 40):
+            q, kn, vn = synth_device.step_inputs(wl, step)
+            hq, hk, hv = synth.step_all(wl, step) if wl.rows <= 64 else (None, None, None)
+            if hq is not None:
+                assert np.array_equal(_bits(q), hq) and np.array_equal(_bits(kn), hk)
+                assert np.array_equal(_bits(vn), hv)
+
+
+@pytest.mark.parametrize("engine", ENGINES)
+def test_tiny_all_rows(engine):
+    wl = synth.TINY
+    ls = LockStep(wl, range(wl.rows), engine=engine)
+    ls.load_prompt()
+    for _ in range(wl.steps):
+        ls.step()
+    assert ls.stats["evicted"] == (wl.prompt_len + 1 - wl.budget) + (wl.steps - 1)
+
+
+@pytest.mark.parametrize("engine", ENGINES)
+@pytest.mark.parametrize("alpha_mode", [0, 1])
+def test_window_departure(engine, alpha_mode):
+    wl = synth.TINY.with_(window=4, steps=32, prompt_len=200, budget=60, alpha_mode=alpha_mode)
+    ls = LockStep(wl, range(wl.rows), engine=engine)
+    ls.load_prompt()
+    for _ in range(wl.steps):
+        ls.step()
+
+
+@pytest.mark.parametrize("engine", ENGINES)
+@pytest.mark.parametrize("prompt_len,budget", [(0, 3), (1, 1), (126, 40), (129, 128), (300, 299)])
+def test_ragged_lengths(engine, prompt_len, budget):
+    wl = synth.TINY.with_(prompt_len=prompt_len, budget=budget, steps=6, window=3)
+    ls = LockStep(wl, range(wl.rows), engine=engine, capacity=max(prompt_len, budget) + 8)
+    ls.load_prompt()
+    for _ in range(wl.steps):
+        ls.step()
+
+
+@pytest.mark.parametrize("engine", ENGINES)
+def test_budget_at_least_n_is_full_attention(engine):
+    import torch
+    wl = synth.MISTRAL_1L.with_(prompt_len=500, budget=600, steps=4)
+    ls = LockStep(wl, [0, 5], engine=engine, capacity=700)
+    ls.load_prompt()
+    for s in range(wl.steps):
+        out = ls.step()
+        q, _, _ = ls._inputs(s)
+        full = ls.cache.full_decode(q)
+        torch.cuda.synchronize()
+        assert torch.allclose(out, full, atol=2e-3, rtol=0), float((out - full).abs().max())
+    assert ls.cache.length()[0] == 504
+
+
+@pytest.mark.parametrize("engine", ENGINES)
+def test_mistral_single_layer(engine):
+    wl = synth.MISTRAL_1L.with_(steps=72)  # > w so queries leave the window
+    ls = LockStep(wl, range(wl.rows), engine=engine)
+    ls.load_prompt()
+    for s in range(wl.steps):
+        ls.step(check=(s < 3 or s % 8 == 0 or s >= 64))
+
+
+def test_full_decode_matches_oracle():
+    import torch
+    import oracle
+    from paper_2608_08878_gb300 import dc
+    wl = synth.MISTRAL_1L.with_(prompt_len=3000)
+    k, v = synth.prompt_all(wl)
+    q, _, _ = synth.step_all(wl, 0)
+    f = lambda a: torch.from_numpy(a.view(np.int16)).view(torch.bfloat16).cuda()
+    cache = dc.DistillCache(1, 8, 128, 3001, 100)
+    cache.append(f(k), f(v))
+    out = cache.full_decode(f(q)).cpu().numpy()
+    for g in range(8):
+        o, _ = oracle.attend(q[0, 0, 4 * g:4 * g + 4], k[0, 0, g], v[0, 0, g])
+        check_attention(out[0, 0, 4 * g:4 * g + 4], o, f"full decode row {g}")
+
+
+def test_host_buffer_step_equals_device_step():
+    import torch
+    from paper_2608_08878_gb300 import dc
+    wl = synth.MISTRAL_1L.with_(prompt_len=1000, budget=300)
+    a, b = LockStep(wl, []), LockStep(wl, [])
+    a.load_prompt()
+    b.load_prompt()
+    for s in range(3):
+        q, kn, vn = synth.step_all(wl, s)
+        f = lambda x: torch.from_numpy(x.view(np.int16)).view(torch.bfloat16)
+        out_h = torch.empty(q.shape, dtype=torch.float32).pin_memory()
+        a.cache.decode_step_host(f(q).pin_memory(), f(kn).pin_memory(), f(vn).pin_memory(), out_h)
+        out_d = b.cache.decode_step(f(q).cuda(), f(kn).cuda(), f(vn).cuda())
+        assert torch.equal(out_h, out_d.cpu())
+        a.cache.evict()
+        b.cache.evict()
+        for which in (dc.BUF_POS, dc.BUF_SCORE):
+            assert torch.equal(a.cache.buffer(which), b.cache.buffer(which))
+
+
+def test_errors_leave_the_cache_usable():
+    import torch
+    from paper_2608_08878_gb300 import dc
+    cache = dc.DistillCache(1, 2, 64, 10, 4, q_heads=4)
+    k = torch.zeros((1, 1, 2, 11, 64), dtype=torch.bfloat16, device="cuda")
+    with pytest.raises(dc.DCError) as e:
+        cache.append(k, k)
+    assert e.value.status == dc.DC_ERR_CAPACITY
+    with pytest.raises(dc.DCError) as e:
+        cache.evict()
+    assert e.value.status == dc.DC_ERR_STATE
+    cache.append(k[:, :, :, :9].contiguous(), k[:, :, :, :9].contiguous())
+    q = torch.zeros((1, 1, 4, 64), dtype=torch.bfloat16, device="cuda")
+    kn = torch.zeros((1, 1, 2, 64), dtype=torch.bfloat16, device="cuda")
+    cache.decode_step(q, kn, kn)
+    with pytest.raises(dc.DCError) as e:
+        cache.decode_step(q, kn, kn)
+    assert e.value.status == dc.DC_ERR_CAPACITY
+    cache.evict()
+    assert cache.length() == (4, 10)
+    cache.sync()
+
+
+@pytest.mark.parametrize("engine", ENGINES)
+def test_full_stack_sampled_rows(engine):
+    """Mistral-7B 32 layers, batch 8, 32K context, budget 8192 at full size: the
+    prompt-compression step and steady steps, 3 sampled rows."""
+    wl = synth.MISTRAL_FULL
+    ls = LockStep(wl, [0, 1029, wl.rows - 1], engine=engine, device_inputs=True)
+    ls.load_prompt()
+    for _ in range(3):
+        ls.step()
+    assert ls.cache.length()[0] == wl.budget
+
+
+def test_aggressive_sampled_rows():
+    """32 layers, batch 16, 32K context, budget 3277 (10%), hot sets reshuffled
+    every 16 steps: crosses one reshuffle, 2 sampled rows."""
+    wl = synth.AGGRESSIVE
+    ls = LockStep(wl, [7, wl.rows - 3], engine=0, device_inputs=True)
+    ls.load_prompt()
+    for s in range(18):
+        ls.step(check=(s < 2 or s >= 15))
