@@ -226,15 +226,14 @@ def run_gpu(args):
     # step 0: prompt compression (32769 -> 8192 tokens per row), timed apart
     ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     ev0.record(stream)
-    cache.decode_step(*inputs[0], out=out)
-    cache.evict()
+    cache.step(*inputs[0], out=out)
     ev1.record(stream)
     torch.cuda.synchronize()
     first_ms = ev0.elapsed_time(ev1)
     for s in range(1, 1 + W):
-        cache.decode_step(*inputs[s], out=out)
-        cache.evict()
+        cache.step(*inputs[s], out=out)
     n_steady = cache.length()[0] + 1
+    engine = cache.engine()
     cache.profile(True)
     torch.cuda.synchronize()
     if dist:
@@ -243,8 +242,7 @@ def run_gpu(args):
     with ClockSampler(gpu_index_for_smi(local_rank)) as clk:
         ev0.record(stream)
         for s in range(1 + W, 1 + W + K):
-            cache.decode_step(*inputs[s], out=out)
-            cache.evict()
+            cache.step(*inputs[s], out=out)
         ev1.record(stream)
         torch.cuda.synchronize()
     el_ms = ev0.elapsed_time(ev1)
@@ -264,12 +262,16 @@ def run_gpu(args):
     dom = max((ph for ph in prof if prof[ph][1] > 0), key=lambda ph: prof[ph][0])
     dom_ms, dom_n = prof[dom]
     per_launch_ms = dom_ms / dom_n
-    if dom == "attend" and args.engine == 1:
-        alg = wl.rows * n_steady * (2 * wl.head_dim + 4)  # K read + positions
+    d = wl.head_dim
+    if dom == "attend" and engine == "fused":
+        # the whole step but the append: K/V, positions, window sums, one move per row
+        alg = wl.rows * (row_bytes_per_step(n_steady, d, wl.alpha_mode) + 2 * (4 * d + 20))
+    elif dom == "attend":
+        alg = wl.rows * n_steady * (2 * d + 36)  # K read + positions + window sums R/W
     elif dom == "score":
-        alg = wl.rows * n_steady * (2 * wl.head_dim + 36)  # V read + positions + window sums R/W
+        alg = wl.rows * n_steady * (2 * d + 20)  # V read + positions + window sums read
     else:
-        alg = wl.rows * row_bytes_per_step(n_steady, wl.head_dim, wl.alpha_mode)
+        alg = wl.rows * row_bytes_per_step(n_steady, d, wl.alpha_mode)
     achieved = alg / (per_launch_ms / 1e3) / 1e9
     gpu_launches = int(sum(v[1] for v in prof.values()))
 
@@ -316,7 +318,7 @@ def run_gpu(args):
             "config": {"workload": wl.name, "layers": wl.layers, "batch": wl.batch, "q_heads": wl.q_heads,
                        "kv_heads": wl.kv_heads, "head_dim": wl.head_dim, "context": wl.prompt_len,
                        "budget": wl.budget, "window": wl.window, "policy": f"5-{wl.mlp_hidden}-LN-ReLU-1",
-                       "engine": ["fused", "split"][args.engine], "parallelism": f"replicas x{world}",
+                       "engine": engine, "parallelism": f"replicas x{world}",
                        "l2": f"inputs larger than L2: {bytes_step / 1e9:.2f} GB streamed per step vs 129 MB L2",
                        "steady_tokens_per_row": n_steady},
             "hbm": {"algorithmic_bytes_per_step": bytes_step, "gbs": gbs,
@@ -356,13 +358,11 @@ def run_e2e(wl, args, inputs):
     out = torch.empty((wl.layers, wl.batch, wl.q_heads, wl.head_dim), dtype=torch.float32).pin_memory()
     W, K = args.warmup, args.steps
     for s in range(0, 1 + W):
-        cache.decode_step_host(*host[s], out)
-        cache.evict()
+        cache.step_host(*host[s], out)
     torch.cuda.synchronize()
     t0 = time.perf_counter()
     for s in range(1 + W, 1 + W + K):
-        cache.decode_step_host(*host[s], out)
-        cache.evict()
+        cache.step_host(*host[s], out)
     cache.sync()
     el = time.perf_counter() - t0
     h2d = sum(x.numel() * x.element_size() for x in host[0])
@@ -394,7 +394,7 @@ def main():
     ap.add_argument("--steps", type=int, default=200)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
-    ap.add_argument("--engine", type=int, default=0, help="0 fused, 1 split")
+    ap.add_argument("--engine", type=int, default=0, help="0 auto, 1 split, 2 fused")
     ap.add_argument("--cpu-seconds", type=float, default=12.0)
     ap.add_argument("--no-cpu", action="store_true")
     ap.add_argument("--no-full", action="store_true")

@@ -58,8 +58,11 @@ typedef struct {
   int layernorm;      /* 1: LayerNorm after the first layer (default, App. D) */
   int alpha_mode;     /* 0: alpha_i from the most recent pass (Sec. 3.1.1, default);
                          1: cumulative since insertion */
-  int engine;         /* 0: fused (one kernel streams K/V once per step, default);
-                         1: split (separate attention, feature and scoring kernels) */
+  int engine;         /* 0: auto (default): the fused kernel whenever the step
+                            fits it and the rows fill the GPU, else split;
+                         1: split (separate attention, feature and scoring kernels);
+                         2: fused whenever the step fits it (one CTA per row
+                            streams K/V once and does the whole step) */
   int keep_features;  /* 1: also store x_i [R][capacity][5] fp32 for inspection */
   unsigned long long seed; /* policy weight seed (dc_policy_init) */
   void* stream;       /* cudaStream_t */
@@ -123,6 +126,20 @@ dc_status dc_decode_step(dc_cache* h, const void* q, const void* k_new, const vo
  * returns, so `out_host` is ready. */
 dc_status dc_decode_step_host(dc_cache* h, const void* q_host, const void* k_new_host,
                               const void* v_new_host, float* out_host);
+
+/* One whole step of Algorithm 1: dc_decode_step followed by dc_evict(budget),
+ * as one kernel when the fused engine takes the step (no scores are stored
+ * then; DC_BUF_SCORE is not updated). Same arguments as dc_decode_step. */
+dc_status dc_step(dc_cache* h, const void* q, const void* k_new, const void* v_new, float* out,
+                  int budget);
+
+/* dc_step with HOST buffers (copies on the handle's stream; synchronises). */
+dc_status dc_step_host(dc_cache* h, const void* q_host, const void* k_new_host,
+                       const void* v_new_host, float* out_host, int budget);
+
+/* Which engine a step over n tokens per row would use (n <= 0: the next
+ * decode step): 1 split, 2 fused. */
+dc_status dc_engine(dc_cache* h, int n, int* engine);
 
 /* argtop_B and prune (Algorithm 1): every row keeps its min(n, B) highest-scored
  * tokens (ties: lower position first; -0 equals +0; NaN ranks last) and

@@ -49,6 +49,7 @@ def lib():
             L.dco_row_positions.argtypes = [P, P]
             L.dco_row_kv_bits.argtypes = [P, P, P]
             L.dco_row_window_sums.argtypes = [P, P, P, P]
+            L.dco_row_window_sums_prior.argtypes = [P, P, P]
             L.dco_attend.argtypes = [P, P, P, C.c_int, C.c_int, C.c_int, P, P]
             L.dco_policy.argtypes = [P, C.c_int, P, C.c_int, C.c_int, P]
             _lib = L
@@ -128,6 +129,13 @@ class OracleRow:
         S, Z, acc = np.empty(n), np.empty(n), np.empty(n)
         lib().dco_row_window_sums(self._h, _ptr(S), _ptr(Z), _ptr(acc))
         return S, Z, acc
+
+    def window_sums_prior(self):
+        """Window sums without the most recent step's query."""
+        n = len(self)
+        S, Z = np.empty(n), np.empty(n)
+        lib().dco_row_window_sums_prior(self._h, _ptr(S), _ptr(Z))
+        return S, Z
 
 
 def attend(q_bits, k_bits, v_bits):

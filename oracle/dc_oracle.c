@@ -46,6 +46,7 @@ struct dco_row {
   int64_t* pos;      /* [cap] */
   double* acc;       /* [cap] cumulative alpha (alpha_mode 1) */
   double *S, *Z;     /* [cap] window sums of the last step */
+  double *Sp, *Zp;   /* [cap] the same without the last step's query */
   double* score;     /* [cap] scores of the last step */
   int have_scores;
   win_entry* win;    /* ring of w entries */
@@ -73,9 +74,12 @@ dco_row* dco_row_new(int d, int G, int w, int alpha_mode, int cap) {
   r->acc = (double*)calloc((size_t)cap, sizeof(double));
   r->S = (double*)calloc((size_t)cap, sizeof(double));
   r->Z = (double*)calloc((size_t)cap, sizeof(double));
+  r->Sp = (double*)calloc((size_t)cap, sizeof(double));
+  r->Zp = (double*)calloc((size_t)cap, sizeof(double));
   r->score = (double*)calloc((size_t)cap, sizeof(double));
   r->win = (win_entry*)calloc((size_t)w, sizeof(win_entry));
-  if (!r->kb || !r->vb || !r->k || !r->v || !r->pos || !r->acc || !r->S || !r->Z || !r->score ||
+  if (!r->kb || !r->vb || !r->k || !r->v || !r->pos || !r->acc || !r->S || !r->Z || !r->Sp ||
+      !r->Zp || !r->score ||
       !r->win) {
     dco_row_free(r);
     return NULL;
@@ -93,7 +97,7 @@ void dco_row_free(dco_row* r) {
   if (r->win)
     for (int i = 0; i < r->w; ++i) win_entry_clear(&r->win[i]);
   free(r->win); free(r->kb); free(r->vb); free(r->k); free(r->v); free(r->pos);
-  free(r->acc); free(r->S); free(r->Z); free(r->score);
+  free(r->acc); free(r->S); free(r->Z); free(r->Sp); free(r->Zp); free(r->score);
   free(r);
 }
 
@@ -259,7 +263,8 @@ int dco_row_step(dco_row* r, const uint16_t* q, const uint16_t* k_new, const uin
     for (int c = 0; c < d; ++c) vn += r->v[(size_t)i * d + c] * r->v[(size_t)i * d + c];
     vn = sqrt(vn);
     /* H_i = S_i / Z_i over the window of recent queries. */
-    double S = 0.0, Z = 0.0;
+    double S = 0.0, Z = 0.0, Sp = 0.0, Zp = 0.0;
+    int newest_entry = (r->win_next + r->w - 1) % r->w;
     for (int qi = 0; qi < r->win_count; ++qi) {
       const win_entry* we = &r->win[qi];
       int j = find_pos(we->pos, we->n, r->pos[i]);
@@ -267,10 +272,16 @@ int dco_row_step(dco_row* r, const uint16_t* q, const uint16_t* k_new, const uin
       for (int h = 0; h < G; ++h) {
         Z += we->a[(size_t)j * G + h];
         S += we->a[(size_t)j * G + h] * we->H[h];
+        if (qi != newest_entry) {
+          Zp += we->a[(size_t)j * G + h];
+          Sp += we->a[(size_t)j * G + h] * we->H[h];
+        }
       }
     }
     r->S[i] = S;
     r->Z[i] = Z;
+    r->Sp[i] = Sp;
+    r->Zp[i] = Zp;
     double Hi = Z > 0.0 ? S / Z : 0.0;
     double posn = (double)r->pos[i] / pos_den;
     x[(size_t)i * 5 + 0] = alpha;
@@ -328,6 +339,8 @@ int dco_row_evict(dco_row* r, int budget, const float* scores_f32) {
       r->acc[w] = r->acc[i];
       r->S[w] = r->S[i];
       r->Z[w] = r->Z[i];
+      r->Sp[w] = r->Sp[i];
+      r->Zp[w] = r->Zp[i];
       r->score[w] = r->score[i];
     }
     w++;
@@ -353,4 +366,9 @@ void dco_row_window_sums(const dco_row* r, double* S, double* Z, double* acc) {
   if (S) memcpy(S, r->S, sizeof(double) * (size_t)r->n);
   if (Z) memcpy(Z, r->Z, sizeof(double) * (size_t)r->n);
   if (acc) memcpy(acc, r->acc, sizeof(double) * (size_t)r->n);
+}
+
+void dco_row_window_sums_prior(const dco_row* r, double* S, double* Z) {
+  if (S) memcpy(S, r->Sp, sizeof(double) * (size_t)r->n);
+  if (Z) memcpy(Z, r->Zp, sizeof(double) * (size_t)r->n);
 }

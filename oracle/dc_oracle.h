@@ -69,6 +69,10 @@ void dco_row_kv_bits(const dco_row* r, uint16_t* k, uint16_t* v);
  * and S_i (entropy-weighted mass); cumulative alpha (alpha_mode 1) in acc. */
 void dco_row_window_sums(const dco_row* r, double* S, double* Z, double* acc);
 
+/* The same window sums without the most recent step's query (the window's
+ * earlier min(w, steps) - 1 queries), [n] each. */
+void dco_row_window_sums_prior(const dco_row* r, double* S, double* Z);
+
 /* Plain softmax attention of G query heads over n keys (no state): the
  * full-cache decode comparator. q [G][d], k/v [n][d] bf16 bits, o [G][d]. */
 void dco_attend(const uint16_t* q, const uint16_t* k, const uint16_t* v, int n, int d, int G,

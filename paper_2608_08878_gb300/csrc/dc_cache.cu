@@ -11,6 +11,7 @@
 
 #include "../../include/distillcache.h"
 #include "dc_common.cuh"
+#include "dc_fused.h"
 #include "dc_kernels.h"
 
 namespace {
@@ -50,6 +51,12 @@ struct dc_cache {
   void* st_k = nullptr;
   void* st_v = nullptr;
   float* st_out = nullptr;
+  // fused engine: TMA descriptors of K/V and the folded policy
+  bool fused_ok = false;
+  std::string fused_why;
+  dc::FusedMaps maps{};
+  dc::FusedPolicy fpol{};
+  __nv_bfloat16* wtile = nullptr;
   std::vector<void*> allocs;
   std::string err;
   bool broken = false;
@@ -153,6 +160,47 @@ dc_status launch_error(dc_cache* h, const char* what) {
   return DC_OK;
 }
 
+// Fused engine for this step? (auto: only when the rows fill the GPU)
+bool use_fused(const dc_cache* h, int n) {
+  if (!h->fused_ok || !dc::fused_eligible(h->dev, n)) return false;
+  if (h->cfg.engine == 2) return true;
+  if (h->cfg.engine == 0) return 2 * h->dev.R >= h->num_sms;
+  return false;
+}
+
+cudaError_t upload_fused_policy(dc_cache* h, const float* blob) {
+  std::vector<__nv_bfloat16> wt;
+  dc::prepare_policy(blob, h->cfg.mlp_hidden, h->cfg.layernorm, &h->fpol, &wt);
+  h->fpol.wtile = h->wtile;
+  cudaError_t e = cudaMemcpyAsync(h->wtile, wt.data(), wt.size() * sizeof(__nv_bfloat16), cudaMemcpyHostToDevice,
+                                  h->stream);
+  if (e == cudaSuccess) e = cudaStreamSynchronize(h->stream);
+  return e;
+}
+
+// The step's common part: append the new pair, fill the step arguments.
+dc::Step begin_step(dc_cache* h) {
+  dc::Step st{};
+  st.n = h->n + 1;
+  st.p_newest = (int)h->seen;
+  st.slot = (int)(h->steps % h->cfg.window);
+  st.has_dep = h->steps >= h->cfg.window ? 1 : 0;
+  st.p_dep = h->ring_pnew[st.slot];
+  st.has_prev = h->steps >= 1 ? 1 : 0;
+  st.slot_prev = (int)((h->steps + h->cfg.window - 1) % h->cfg.window);
+  st.p_prev = h->ring_pnew[st.slot_prev];
+  split_plan(h, st.n, &st.nsplit, &st.chunk);
+  return st;
+}
+
+void end_step(dc_cache* h, const dc::Step& st) {
+  h->n += 1;
+  h->seen += 1;
+  h->ring_pnew[st.slot] = st.p_newest;
+  h->steps += 1;
+  h->have_scores = true;
+}
+
 bool run_split_step(dc_cache* h, const dc::Step& st, const void* q, float* out) {
   const dc::Dev& p = h->dev;
   if (!dc::split_supported(p)) return false;
@@ -225,7 +273,7 @@ dc_status dc_cache_create(int layers, int kv_heads, int head_dim, int capacity, 
   if (cfg.mlp_hidden < 1 || cfg.mlp_hidden > 256 || (cfg.mlp_hidden >= 32 && cfg.mlp_hidden % 32))
     return fail(nullptr, DC_ERR_INVALID_ARG, "mlp_hidden must be in [1, 256], a multiple of 32 when >= 32");
   if (cfg.alpha_mode != 0 && cfg.alpha_mode != 1) return fail(nullptr, DC_ERR_INVALID_ARG, "alpha_mode must be 0 or 1");
-  if (cfg.engine != 0 && cfg.engine != 1) return fail(nullptr, DC_ERR_INVALID_ARG, "engine must be 0 or 1");
+  if (cfg.engine < 0 || cfg.engine > 2) return fail(nullptr, DC_ERR_INVALID_ARG, "engine must be 0, 1 or 2");
   const long long R = (long long)layers * cfg.batch * kv_heads;
   if (R > 65535 || (long long)capacity * R > (1ll << 40))
     return fail(nullptr, DC_ERR_INVALID_ARG, "cache too large");
@@ -270,7 +318,6 @@ dc_status dc_cache_create(int layers, int kv_heads, int head_dim, int capacity, 
   p.policy = pol;
   A(&p.status, sizeof(unsigned));
   A(&p.logit, RC * G * sizeof(float));
-  A(&p.dep, RC * 2 * sizeof(float));
   A(&p.part, (size_t)R * p.smax * G * 4 * sizeof(float));
   A(&p.opart, (size_t)R * p.smax * G * head_dim * sizeof(float));
   A(&p.holes, RC * sizeof(int));
@@ -289,6 +336,19 @@ dc_status dc_cache_create(int layers, int kv_heads, int head_dim, int capacity, 
   dc_policy_init(cfg.seed, cfg.mlp_hidden, w.data(), blob);
   e = cudaMemcpyAsync(pol, w.data(), blob * sizeof(float), cudaMemcpyHostToDevice, h->stream);
   if (e == cudaSuccess) e = cudaStreamSynchronize(h->stream);
+  if (e == cudaSuccess && cfg.engine != 1 && dc::fused_eligible(p, 1) && R * (long long)capacity < (1ll << 31)) {
+    const char* why = "";
+    cudaError_t fe = dalloc(h, &h->wtile, 128 * 32 * sizeof(__nv_bfloat16));
+    if (fe == cudaSuccess) fe = dc::make_fused_maps(p, &h->maps, &why);
+    if (fe == cudaSuccess) fe = upload_fused_policy(h, w.data());
+    if (fe == cudaSuccess) {
+      h->fused_ok = true;
+    } else {
+      cudaGetLastError();
+      h->fused_why = why;
+      if (cfg.engine == 2) e = fe;
+    }
+  }
   if (e != cudaSuccess) {
     dc_status s = cuda_fail(nullptr, e, "policy upload");
     free_all(h);
@@ -318,6 +378,7 @@ dc_status dc_policy_set_weights(dc_cache* h, const float* blob, size_t n) {
   DC_CUDA(h, cudaMemcpyAsync((void*)h->dev.policy, blob, n * sizeof(float), cudaMemcpyHostToDevice,
                              h->stream));
   DC_CUDA(h, cudaStreamSynchronize(h->stream));  // the caller may free the blob on return
+  if (h->fused_ok) DC_CUDA(h, upload_fused_policy(h, blob));
   return DC_OK;
 }
 
@@ -343,28 +404,82 @@ dc_status dc_append(dc_cache* h, const void* k, const void* v, int n_tokens) {
 dc_status dc_decode_step(dc_cache* h, const void* q, const void* k_new, const void* v_new, float* out) {
   DC_CHECK_HANDLE(h);
   if (!q || !k_new || !v_new || !out) return fail(h, DC_ERR_INVALID_ARG, "NULL pointer");
-  if (((uintptr_t)k_new | (uintptr_t)v_new) & 15) return fail(h, DC_ERR_INVALID_ARG, "k_new and v_new must be 16-byte aligned");
+  if (((uintptr_t)q | (uintptr_t)k_new | (uintptr_t)v_new) & 15)
+    return fail(h, DC_ERR_INVALID_ARG, "q, k_new and v_new must be 16-byte aligned");
   if (h->n + 1 > h->capacity) return fail(h, DC_ERR_CAPACITY, "decode step exceeds capacity");
   if (h->seen + 1 > 0x7FFFFFFFll) return fail(h, DC_ERR_CAPACITY, "position counter overflow");
   {
     Phase ph(h, DC_PHASE_APPEND, 1);
     dc::launch_append(h->dev, k_new, v_new, 1, h->n, (int)h->seen, h->stream);
   }
-  dc::Step st{};
-  st.n = h->n + 1;
-  st.p_newest = (int)h->seen;
-  st.slot = (int)(h->steps % h->cfg.window);
-  st.has_dep = h->steps >= h->cfg.window ? 1 : 0;
-  st.p_dep = h->ring_pnew[st.slot];
-  split_plan(h, st.n, &st.nsplit, &st.chunk);
-  if (!run_split_step(h, st, q, out)) return fail(h, DC_ERR_INVALID_ARG, "unsupported head_dim / group");
+  const dc::Step st = begin_step(h);
+  if (use_fused(h, st.n)) {
+    dc::FusedStep fs{(const __nv_bfloat16*)q, out, 0, 0, 1};
+    cudaError_t e;
+    {
+      Phase ph(h, DC_PHASE_ATTEND, 1);
+      e = dc::launch_fused_step(h->maps, h->dev, st, fs, h->fpol, h->num_sms, h->stream);
+    }
+    if (e != cudaSuccess) return cuda_fail(h, e, "fused step");
+  } else if (!run_split_step(h, st, q, out)) {
+    return fail(h, DC_ERR_INVALID_ARG, "unsupported head_dim / group");
+  }
   dc_status s = launch_error(h, "decode step");
   if (s != DC_OK) return s;
-  h->n += 1;
-  h->seen += 1;
-  h->ring_pnew[st.slot] = st.p_newest;
-  h->steps += 1;
-  h->have_scores = true;
+  end_step(h, st);
+  return DC_OK;
+}
+
+dc_status dc_step(dc_cache* h, const void* q, const void* k_new, const void* v_new, float* out, int budget) {
+  DC_CHECK_HANDLE(h);
+  if (!q || !k_new || !v_new || !out) return fail(h, DC_ERR_INVALID_ARG, "NULL pointer");
+  if (((uintptr_t)q | (uintptr_t)k_new | (uintptr_t)v_new) & 15)
+    return fail(h, DC_ERR_INVALID_ARG, "q, k_new and v_new must be 16-byte aligned");
+  if (h->n + 1 > h->capacity) return fail(h, DC_ERR_CAPACITY, "decode step exceeds capacity");
+  const int n1 = h->n + 1;
+  if (!use_fused(h, n1)) {
+    dc_status s = dc_decode_step(h, q, k_new, v_new, out);
+    if (s != DC_OK) return s;
+    return dc_evict(h, budget);
+  }
+  if (h->seen + 1 > 0x7FFFFFFFll) return fail(h, DC_ERR_CAPACITY, "position counter overflow");
+  {
+    Phase ph(h, DC_PHASE_APPEND, 1);
+    dc::launch_append(h->dev, k_new, v_new, 1, h->n, (int)h->seen, h->stream);
+  }
+  const dc::Step st = begin_step(h);
+  const int B = budget <= 0 ? h->budget : budget;
+  const int keep = std::min(st.n, B);
+  dc::FusedStep fs{(const __nv_bfloat16*)q, out, keep < st.n ? 1 : 0, keep, 0};
+  cudaError_t e;
+  {
+    Phase ph(h, DC_PHASE_ATTEND, 1);
+    e = dc::launch_fused_step(h->maps, h->dev, st, fs, h->fpol, h->num_sms, h->stream);
+  }
+  if (e != cudaSuccess) return cuda_fail(h, e, "fused step");
+  end_step(h, st);
+  h->n = keep;
+  h->have_scores = false;
+  return DC_OK;
+}
+
+dc_status dc_step_host(dc_cache* h, const void* q, const void* k_new, const void* v_new, float* out, int budget) {
+  DC_CHECK_HANDLE(h);
+  if (!q || !k_new || !v_new || !out) return fail(h, DC_ERR_INVALID_ARG, "NULL pointer");
+  const size_t R = h->dev.R, G = h->dev.G, d = h->dev.d;
+  DC_CUDA(h, cudaMemcpyAsync(h->st_q, q, R * G * d * 2, cudaMemcpyHostToDevice, h->stream));
+  DC_CUDA(h, cudaMemcpyAsync(h->st_k, k_new, R * d * 2, cudaMemcpyHostToDevice, h->stream));
+  DC_CUDA(h, cudaMemcpyAsync(h->st_v, v_new, R * d * 2, cudaMemcpyHostToDevice, h->stream));
+  dc_status s = dc_step(h, h->st_q, h->st_k, h->st_v, h->st_out, budget);
+  if (s != DC_OK) return s;
+  DC_CUDA(h, cudaMemcpyAsync(out, h->st_out, R * G * d * sizeof(float), cudaMemcpyDeviceToHost, h->stream));
+  DC_CUDA(h, cudaStreamSynchronize(h->stream));
+  return DC_OK;
+}
+
+dc_status dc_engine(dc_cache* h, int n, int* engine) {
+  if (!valid(h) || !engine) return DC_ERR_INVALID_ARG;
+  *engine = use_fused(h, n > 0 ? n : h->n + 1) ? 2 : 1;
   return DC_OK;
 }
 

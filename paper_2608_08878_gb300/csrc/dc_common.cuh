@@ -4,7 +4,12 @@
 // Row r = (layer * batch + b) * kv_heads + g owns `cap` slots. Per-slot data:
 //   K, V   bf16 [R][cap][d]      keys / values
 //   pos    int32 [R][cap]        absolute position (tokens seen before it)
-//   S, Z   fp64 [R][cap]         window sums of the entropy feature H_i
+//   S, Z   fp64 [R][cap]         window sums of the entropy feature H_i over
+//                                the window's queries BEFORE the last step
+//                                (the last step's terms are added, and the
+//                                departing query's subtracted, by the next
+//                                step's attention pass; both are recomputed
+//                                by the same code, so they cancel bit for bit)
 //   acc    fp32 [R][cap]         cumulative alpha (alpha_mode 1 only)
 //   score  fp32 [R][cap]         policy score of the last decode step
 // Per-row ring of the last w decode queries (the window of H_i, Sec. 3.1.1):
@@ -42,7 +47,6 @@ struct Dev {
   unsigned* status;
   // scratch of the split engine
   float* logit;   // [R][cap][G]
-  float* dep;     // [R][cap][2]: departing query's (Z, S) terms
   float* part;    // [R][smax][G][4]: per-split (m, l, u2, 0)
   float* opart;   // [R][smax][G][d]
   int* holes;     // [R][cap]
@@ -55,8 +59,11 @@ struct Step {
   int n;          // tokens per row after the append
   int p_newest;   // position of the newest token
   int slot;       // ring slot of this step (= slot of the departing query)
-  int has_dep;    // a query leaves the window this step
+  int has_dep;    // a query leaves the window this step (step t - w)
   int p_dep;      // newest position at the departing query's step
+  int has_prev;   // the previous step's query joins the stored sums (step t - 1)
+  int slot_prev;  // its ring slot
+  int p_prev;     // newest position at the previous step
   int nsplit;     // splits per row (split engine)
   int chunk;      // tokens per split
 };

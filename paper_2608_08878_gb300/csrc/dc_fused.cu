@@ -1,0 +1,721 @@
+// dc_fused.cu -- the fused engine: one persistent kernel streams every row's
+// keys and values from HBM exactly once per decode step and does the whole
+// step of Algorithm 1 for that row: attention (with the exact row softmax
+// statistics), the five token features of Sec. 3.1.1, the policy MLP of
+// Sec. 3.1.2 / App. D, and (dc_step) the top-B select and compaction.
+//
+// One CTA per SM; each CTA takes rows r = blockIdx.x, blockIdx.x + gridDim.x...
+// Warp roles (192 threads):
+//   warp 0     producer: writes the row's query tile (current, previous and
+//              departing queries) and streams K then V tiles of 128 tokens
+//              with TMA (128-byte swizzle) through a 3-stage ring;
+//   warp 1     MMA issuer (one lane): tcgen05.mma, accumulators in TMEM:
+//                S  = K Q^T        [128 tokens x 16]  per K tile
+//                O^T += V^T P^T    [d x 16]           per V tile (P = weights)
+//                Z  = A W^T        [128 tokens x 128] per V tile (policy layer)
+//   warps 2-5  epilogue, one token (TMEM lane) per thread:
+//                K pass: online softmax statistics, window-sum update (the
+//                previous step's query in, the departing one out, both
+//                recomputed from the same S tile), raw logits kept in TMEM;
+//                V pass: weights with the final statistics, features, the
+//                policy's input row, score; then the output and the select.
+//
+// TMEM columns: S tiles [0, 32), O [32, 48), policy layer [64, 192), the
+// logit stash [192, 512) (G columns per tile of 128 tokens).
+#include <cuda.h>
+
+#include "dc_common.cuh"
+#include "dc_fused.h"
+#include "dc_kernels.h"
+#include "dc_select.cuh"
+#include "dc_sm100.cuh"
+
+namespace dc {
+using namespace sm100;
+
+namespace {
+
+constexpr int kStages = 3;
+constexpr int kStageBytes = 32768;
+constexpr int kTok = 128;
+constexpr int kThreads = 192;
+constexpr int kEpi = 128;
+constexpr uint32_t kTmemCols = 512;
+constexpr int kColS = 0, kColO = 32, kColM = 64, kColStash = 192;
+
+constexpr int OFF_STAGE = 0;
+constexpr int OFF_Q = OFF_STAGE + kStages * kStageBytes;  // 2 x 4 KB
+constexpr int OFF_P = OFF_Q + 2 * 4096;                    // 2 x 4 KB
+constexpr int OFF_A = OFF_P + 2 * 4096;                    // 2 x 16 KB
+constexpr int OFF_W = OFF_A + 2 * 16384;                   // 16 KB
+constexpr int OFF_SC = OFF_W + 16384;                      // scores, kFusedMaxTok floats
+constexpr int OFF_MISC = OFF_SC + kFusedMaxTok * 4;
+constexpr int MISC_BYTES = 4096;
+constexpr int kSmemBytes = OFF_MISC + MISC_BYTES + 1024;   // + alignment slack
+
+// barrier indices in the misc area
+enum {
+  B_FULL = 0, B_EMPTY = 3, B_QFULL = 6, B_QEMPTY = 8, B_SFULL = 10, B_SEMPTY = 12, B_PFULL = 14,
+  B_PEMPTY = 16, B_MFULL = 18, B_MEMPTY = 19, B_OFULL = 20, B_OEMPTY = 21, B_DRAIN = 22, B_COUNT = 24
+};
+
+// byte offset of 16-byte chunk `c` (0..7) of row `row` inside a 128-byte
+// swizzled tile (8-row atoms of 1024 bytes)
+__device__ __forceinline__ uint32_t sw128(int row, int c) {
+  return (uint32_t)((row >> 3) * 1024 + (row & 7) * 128 + ((c ^ (row & 7)) << 4));
+}
+
+__device__ __forceinline__ uint32_t pack_bf16(float a, float b) {
+  __nv_bfloat162 v = __floats2bfloat162_rn(a, b);
+  return *reinterpret_cast<uint32_t*>(&v);
+}
+
+template <int G>
+__device__ __forceinline__ void tmem_st_g(uint32_t taddr, const float* v) {
+  if constexpr (G == 4) {
+    asm volatile("tcgen05.st.sync.aligned.32x32b.x4.b32 [%0], {%1,%2,%3,%4};" ::"r"(taddr),
+                 "r"(__float_as_uint(v[0])), "r"(__float_as_uint(v[1])), "r"(__float_as_uint(v[2])),
+                 "r"(__float_as_uint(v[3]))
+                 : "memory");
+  } else if constexpr (G == 2) {
+    asm volatile("tcgen05.st.sync.aligned.32x32b.x2.b32 [%0], {%1,%2};" ::"r"(taddr), "r"(__float_as_uint(v[0])),
+                 "r"(__float_as_uint(v[1]))
+                 : "memory");
+  } else {
+    asm volatile("tcgen05.st.sync.aligned.32x32b.x1.b32 [%0], {%1};" ::"r"(taddr), "r"(__float_as_uint(v[0]))
+                 : "memory");
+  }
+}
+
+template <int G>
+__device__ __forceinline__ void tmem_ld_g(uint32_t taddr, float* v) {
+  if constexpr (G == 4) {
+    float t[4];
+    tmem_ld4(taddr, t);
+#pragma unroll
+    for (int h = 0; h < 4; ++h) v[h] = t[h];
+  } else if constexpr (G == 2) {
+    uint32_t a, b;
+    asm volatile("tcgen05.ld.sync.aligned.32x32b.x2.b32 {%0,%1}, [%2];" : "=r"(a), "=r"(b) : "r"(taddr));
+    v[0] = __uint_as_float(a);
+    v[1] = __uint_as_float(b);
+  } else {
+    uint32_t a;
+    asm volatile("tcgen05.ld.sync.aligned.32x32b.x1.b32 {%0}, [%1];" : "=r"(a) : "r"(taddr));
+    v[0] = __uint_as_float(a);
+  }
+}
+
+__device__ __forceinline__ void online_add(float& m, float& l, float& u, float s, float c) {
+  if (s > m) {
+    if (m == -INFINITY) {
+      l = 1.f;
+      u = 0.f;
+    } else {
+      const float dl = (m - s) * c, f = ex2(dl);
+      u = (u + l * dl) * f;
+      l = fmaf(l, f, 1.f);
+    }
+    m = s;
+  } else {
+    const float x = (s - m) * c, pe = ex2(x);
+    l += pe;
+    u = fmaf(pe, x, u);
+  }
+}
+
+__device__ __forceinline__ void online_merge(float& m, float& l, float& u, float mo, float lo, float uo, float c) {
+  if (mo == -INFINITY) return;
+  if (m == -INFINITY) { m = mo; l = lo; u = uo; return; }
+  const float M = fmaxf(m, mo), da = (m - M) * c, db = (mo - M) * c;
+  const float fa = ex2(da), fb = ex2(db);
+  u = (u + l * da) * fa + (uo + lo * db) * fb;
+  l = l * fa + lo * fb;
+  m = M;
+}
+
+template <int D, int G>
+__global__ void __launch_bounds__(kThreads, 1)
+    fused_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmV, Dev p,
+                 Step st, FusedStep fs, FusedPolicy fp) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  uint64_t* bar = reinterpret_cast<uint64_t*>(smem + OFF_MISC);
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + OFF_MISC + 8 * B_COUNT);
+  volatile int* abort = reinterpret_cast<volatile int*>(smem + OFF_MISC + 8 * B_COUNT + 4);
+  float* red = reinterpret_cast<float*>(smem + OFF_MISC + 256);            // [4][G][3]
+  int* s_hist = reinterpret_cast<int*>(smem + OFF_MISC + 1024);           // [256]
+  int* s_sh = reinterpret_cast<int*>(smem + OFF_MISC + 2048);             // [4]
+  int* s_wsum = reinterpret_cast<int*>(smem + OFF_MISC + 2064);           // [4]
+  unsigned long long* s_best = reinterpret_cast<unsigned long long*>(smem + OFF_MISC + 2112);  // [4]
+  int* s_best_slot = reinterpret_cast<int*>(smem + OFF_MISC + 2176);      // [4]
+  float* sc = reinterpret_cast<float*>(smem + OFF_SC);
+
+  const int warp = threadIdx.x / kWarp, lane = threadIdx.x % kWarp;
+  const int n = st.n, nT = (n + kTok - 1) / kTok;
+  constexpr uint32_t kTileBytes = (uint32_t)D * kTok * 2;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < kStages; ++s) {
+      mbar_init(&bar[B_FULL + s], 1);
+      mbar_init(&bar[B_EMPTY + s], 5);
+    }
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(&bar[B_QFULL + b], 1);
+      mbar_init(&bar[B_QEMPTY + b], 1);
+      mbar_init(&bar[B_SFULL + b], 1);
+      mbar_init(&bar[B_SEMPTY + b], 4);
+      mbar_init(&bar[B_PFULL + b], 4);
+      mbar_init(&bar[B_PEMPTY + b], 1);
+    }
+    mbar_init(&bar[B_MFULL], 1);
+    mbar_init(&bar[B_MEMPTY], 4);
+    mbar_init(&bar[B_OFULL], 1);
+    mbar_init(&bar[B_OEMPTY], 4);
+    mbar_init(&bar[B_DRAIN], 1);
+    *abort = 0;
+    fence_mbar_init();
+  }
+  // zero the query and weight tiles (unused rows stay zero), then write the
+  // policy layer's B operand (128 rows x 64 bf16, swizzled; 32 columns used)
+  for (int e = threadIdx.x; e < (OFF_A - OFF_Q) / 16; e += kThreads)
+    reinterpret_cast<uint4*>(smem + OFF_Q)[e] = make_uint4(0, 0, 0, 0);
+  for (int e = threadIdx.x; e < 128 * 8; e += kThreads) {
+    const int row = e >> 3, c = e & 7;
+    uint4 v = make_uint4(0, 0, 0, 0);
+    if (c < 4) v = reinterpret_cast<const uint4*>(fp.wtile)[row * 4 + c];
+    *reinterpret_cast<uint4*>(smem + OFF_W + sw128(row, c)) = v;
+  }
+  fence_proxy_async();
+  if (warp == 1) {
+    tmem_alloc(tmem_slot, kTmemCols);
+    tmem_relinquish();
+  }
+  if (warp == 0 && lane == 0) {
+    prefetch_tmap(&tmK);
+    prefetch_tmap(&tmV);
+  }
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+
+  if (warp == 0) {
+    // ------------------------------------------------------------ producer
+    const uint64_t pol = l2_evict_first_policy();
+    int g = 0, gr = 0, issued = 0;
+    for (int r = blockIdx.x; r < p.R; r += gridDim.x, ++gr) {
+      if (*abort) break;
+      const int qb = gr & 1;
+      if (!mbar_wait(&bar[B_QEMPTY + qb], ((gr >> 1) & 1) ^ 1, abort)) break;
+      // query tile: rows [0,G) current, [G,2G) previous step, [2G,3G) departing
+      uint8_t* qt = smem + OFF_Q + qb * 4096;
+      const int qo = ((r / p.kvh) * p.qh + (r % p.kvh) * G) * D;
+      const __nv_bfloat16* prev = p.ring_q + ((size_t)r * p.w + st.slot_prev) * G * D;
+      const __nv_bfloat16* dep = p.ring_q + ((size_t)r * p.w + st.slot) * G * D;
+      for (int e = lane; e < 3 * G * (D / 8); e += kWarp) {
+        const int qi = e / (D / 8), kc = e % (D / 8);
+        const int which = qi / G, h = qi % G;
+        uint4 v = make_uint4(0, 0, 0, 0);
+        if (which == 0) v = reinterpret_cast<const uint4*>(fs.q + qo + h * D)[kc];
+        else if (which == 1 && st.has_prev) v = reinterpret_cast<const uint4*>(prev + h * D)[kc];
+        else if (which == 2 && st.has_dep) v = reinterpret_cast<const uint4*>(dep + h * D)[kc];
+        *reinterpret_cast<uint4*>(qt + (kc >> 3) * 2048 + sw128(qi, kc & 7)) = v;
+      }
+      fence_proxy_async();
+      __syncwarp();
+      if (lane == 0) {
+        mbar_arrive(&bar[B_QFULL + qb]);
+        for (int pass = 0; pass < 2 && !*abort; ++pass) {
+          const CUtensorMap* tm = pass ? &tmV : &tmK;
+          for (int j = 0; j < nT; ++j, ++g) {
+            const int s = g % kStages;
+            if (!mbar_wait(&bar[B_EMPTY + s], ((g / kStages) & 1) ^ 1, abort)) break;
+            mbar_expect_tx(&bar[B_FULL + s], kTileBytes);
+            uint8_t* dst = smem + OFF_STAGE + s * kStageBytes;
+            const int y = r * p.cap + j * kTok;
+            tma_load_2d(dst, tm, 0, y, &bar[B_FULL + s], pol);
+            if (D == 128) tma_load_2d(dst + 16384, tm, 64, y, &bar[B_FULL + s], pol);
+            issued = g + 1;
+          }
+        }
+      }
+      g = __shfl_sync(0xffffffffu, g, 0);
+      issued = __shfl_sync(0xffffffffu, issued, 0);
+    }
+    // every issued load must land before the CTA may exit
+    if (lane == 0) {
+      for (int t = issued - kStages < 0 ? 0 : issued - kStages; t < issued; ++t)
+        mbar_wait_drain(&bar[B_FULL + t % kStages], (t / kStages) & 1);
+    }
+  } else if (warp == 1) {
+    // ------------------------------------------------------------ MMA issuer
+    if (lane == 0) {
+      const uint32_t id_qk = idesc_bf16(128, 16, 0, 0);
+      const uint32_t id_pv = idesc_bf16(128, 16, 1, 0);
+      const uint32_t id_m = idesc_bf16(128, 128, 0, 0);
+      int g = 0, gs = 0, gv = 0, gr = 0;
+      for (int r = blockIdx.x; r < p.R; r += gridDim.x, ++gr) {
+        if (*abort) break;
+        const int qb = gr & 1;
+        if (!mbar_wait(&bar[B_QFULL + qb], (gr >> 1) & 1, abort)) break;
+        tc_fence_after();
+        const uint32_t qaddr = smem_u32(smem + OFF_Q + qb * 4096);
+        for (int j = 0; j < nT; ++j, ++g, ++gs) {
+          const int s = g % kStages, b = gs & 1;
+          if (!mbar_wait(&bar[B_FULL + s], (g / kStages) & 1, abort)) break;
+          if (!mbar_wait(&bar[B_SEMPTY + b], ((gs >> 1) & 1) ^ 1, abort)) break;
+          tc_fence_after();
+          const uint32_t kaddr = smem_u32(smem + OFF_STAGE + s * kStageBytes);
+#pragma unroll
+          for (int ks = 0; ks < D / 16; ++ks) {
+            const uint32_t off = (uint32_t)(ks >> 2) * 16384u + (uint32_t)(ks & 3) * 32u;
+            const uint32_t qoff = (uint32_t)(ks >> 2) * 2048u + (uint32_t)(ks & 3) * 32u;
+            mma_bf16(tmem + kColS + b * 16, sdesc_sw128(kaddr + off, 16, 1024), sdesc_sw128(qaddr + qoff, 16, 1024),
+                     id_qk, ks > 0);
+          }
+          mma_commit(&bar[B_SFULL + b]);
+          mma_commit(&bar[B_EMPTY + s]);
+        }
+        mma_commit(&bar[B_QEMPTY + qb]);
+        for (int j = 0; j < nT; ++j, ++g, ++gv) {
+          const int s = g % kStages, pb = gv & 1;
+          if (!mbar_wait(&bar[B_FULL + s], (g / kStages) & 1, abort)) break;
+          if (!mbar_wait(&bar[B_PFULL + pb], (gv >> 1) & 1, abort)) break;
+          if (j == 0 && !mbar_wait(&bar[B_OEMPTY], (gr & 1) ^ 1, abort)) break;
+          if (!mbar_wait(&bar[B_MEMPTY], (gv & 1) ^ 1, abort)) break;
+          tc_fence_after();
+          const uint32_t vaddr = smem_u32(smem + OFF_STAGE + s * kStageBytes);
+          const uint32_t paddr = smem_u32(smem + OFF_P + pb * 4096);
+          const uint32_t aaddr = smem_u32(smem + OFF_A + pb * 16384);
+          const uint32_t waddr = smem_u32(smem + OFF_W);
+          // O^T[d x 16] += V^T[d x 128] P^T: V^T is MN-major (dims contiguous)
+#pragma unroll
+          for (int ks = 0; ks < kTok / 16; ++ks) {
+            const uint32_t poff = (uint32_t)(ks >> 2) * 2048u + (uint32_t)(ks & 3) * 32u;
+            mma_bf16(tmem + kColO, sdesc_sw128(vaddr + ks * 2048u, 16384, 1024),
+                     sdesc_sw128(paddr + poff, 16, 1024), id_pv, (j > 0 || ks > 0) ? 1u : 0u);
+          }
+          // policy layer: Z[128 x 128] = A[128 x 32] W^T
+#pragma unroll
+          for (int ks = 0; ks < 2; ++ks)
+            mma_bf16(tmem + kColM, sdesc_sw128(aaddr + ks * 32u, 16, 1024), sdesc_sw128(waddr + ks * 32u, 16, 1024),
+                     id_m, ks > 0);
+          mma_commit(&bar[B_MFULL]);
+          mma_commit(&bar[B_PEMPTY + pb]);
+          mma_commit(&bar[B_EMPTY + s]);
+          if (j == nT - 1) mma_commit(&bar[B_OFULL]);
+        }
+      }
+      // all issued MMAs complete before TMEM is released
+      mma_commit(&bar[B_DRAIN]);
+      mbar_wait_drain(&bar[B_DRAIN], 0);
+    }
+    __syncwarp();
+  } else {
+    // ------------------------------------------------------------ epilogue
+    const int ew = warp - 2;                    // 0..3
+    const int quad = warp & 3;                  // TMEM lane quarter of this warp
+    const int tok = quad * 32 + lane;           // token (TMEM lane) within a tile
+    const int etid = ew * 32 + lane;            // 0..127
+    const uint32_t lane_addr = tmem + ((uint32_t)(quad * 32) << 16);
+    const float c = p.c;
+    auto sync = [] { named_bar(1, kEpi); };
+    const SelectScratch scr{s_hist, s_sh, s_wsum, s_best, s_best_slot};
+    int g = 0, gs = 0, gv = 0, gr = 0;
+    for (int r = blockIdx.x; r < p.R; r += gridDim.x, ++gr) {
+      if (named_bar_or(1, kEpi, *abort != 0)) break;
+      const size_t rbase = (size_t)r * p.cap;
+      float pm[G], pl[G], pH[G], dm[G], dl[G], dH[G];
+#pragma unroll
+      for (int h = 0; h < G; ++h) {
+        const float* rp = p.ring_stats + (((size_t)r * p.w + st.slot_prev) * G + h) * 4;
+        const float* rd = p.ring_stats + (((size_t)r * p.w + st.slot) * G + h) * 4;
+        pm[h] = rp[0]; pl[h] = rp[1]; pH[h] = rp[2];
+        dm[h] = rd[0]; dl[h] = rd[1]; dH[h] = rd[2];
+      }
+      float m[G], l[G], u[G];
+#pragma unroll
+      for (int h = 0; h < G; ++h) { m[h] = -INFINITY; l[h] = 0.f; u[h] = 0.f; }
+
+      // ---------------- K pass
+      for (int j = 0; j < nT; ++j, ++g, ++gs) {
+        const int s = g % kStages, b = gs & 1;
+        mbar_wait(&bar[B_SFULL + b], (gs >> 1) & 1, abort);
+        __syncwarp();
+        tc_fence_after();
+        float S16[16];
+        tmem_ld16(lane_addr + kColS + b * 16, S16);
+        tmem_ld_wait();
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) {
+          mbar_arrive(&bar[B_SEMPTY + b]);
+          mbar_arrive(&bar[B_EMPTY + s]);
+        }
+        const int i = j * kTok + tok;
+        if (i < n) {
+#pragma unroll
+          for (int h = 0; h < G; ++h) online_add(m[h], l[h], u[h], S16[h], c);
+          if (st.has_prev || st.has_dep) {
+            const int pos = p.pos[rbase + i];
+            float zp = 0.f, sp = 0.f, zd = 0.f, sd = 0.f;
+            if (st.has_prev && pos <= st.p_prev) window_terms<G>(S16 + G, pm, pl, pH, c, zp, sp);
+            if (st.has_dep && pos <= st.p_dep) window_terms<G>(S16 + 2 * G, dm, dl, dH, c, zd, sd);
+            p.Z[rbase + i] = (p.Z[rbase + i] + (double)zp) - (double)zd;
+            p.S[rbase + i] = (p.S[rbase + i] + (double)sp) - (double)sd;
+          }
+        }
+        __syncwarp();
+        tmem_st_g<G>(lane_addr + kColStash + j * G, S16);
+      }
+      tmem_st_wait();
+      // ---------------- row softmax statistics (deterministic merge order)
+#pragma unroll
+      for (int h = 0; h < G; ++h) {
+        float mm = m[h], ll = l[h], uu = u[h];
+#pragma unroll
+        for (int off = 16; off > 0; off >>= 1) {
+          const float mo = __shfl_xor_sync(0xffffffffu, mm, off);
+          const float lo = __shfl_xor_sync(0xffffffffu, ll, off);
+          const float uo = __shfl_xor_sync(0xffffffffu, uu, off);
+          online_merge(mm, ll, uu, mo, lo, uo, c);
+        }
+        if (lane == 0) {
+          red[(ew * G + h) * 3 + 0] = mm;
+          red[(ew * G + h) * 3 + 1] = ll;
+          red[(ew * G + h) * 3 + 2] = uu;
+        }
+      }
+      sync();
+      float M[G], L[G], Hh[G];
+#pragma unroll
+      for (int h = 0; h < G; ++h) {
+        float mm = -INFINITY, ll = 0.f, uu = 0.f;
+        for (int w = 0; w < 4; ++w)
+          online_merge(mm, ll, uu, red[(w * G + h) * 3 + 0], red[(w * G + h) * 3 + 1], red[(w * G + h) * 3 + 2], c);
+        M[h] = mm;
+        L[h] = ll;
+        Hh[h] = logf(ll) - 0.69314718055994531f * (uu / ll);
+      }
+      sync();  // red is rewritten by the next row
+      // push (q, m, l, H) of this step into the ring slot it takes over
+      if (etid < G) {
+        float* rs = p.ring_stats + (((size_t)r * p.w + st.slot) * G + etid) * 4;
+        rs[0] = M[etid]; rs[1] = L[etid]; rs[2] = Hh[etid]; rs[3] = 0.f;
+        p.hq[(size_t)r * G + etid] = Hh[etid];
+      }
+      {
+        const int qo = ((r / p.kvh) * p.qh + (r % p.kvh) * G) * D;
+        uint4* rq = reinterpret_cast<uint4*>(p.ring_q + ((size_t)r * p.w + st.slot) * G * D);
+        const uint4* qs = reinterpret_cast<const uint4*>(fs.q + qo);
+        for (int e = etid; e < G * D / 8; e += kEpi) rq[e] = qs[e];
+      }
+
+      // ---------------- V pass (prep of tile j+1 overlaps the MMAs of tile j)
+      const float pos_den = (float)max(st.p_newest, 1);
+      auto prep = [&](int j) {
+        const int gj = g + j, gvj = gv + j;
+        const int s = gj % kStages, pb = gvj & 1;
+        mbar_wait(&bar[B_FULL + s], (gj / kStages) & 1, abort);
+        mbar_wait(&bar[B_PEMPTY + pb], ((gvj >> 1) & 1) ^ 1, abort);
+        const int i = j * kTok + tok;
+        const bool valid = i < n;
+        float sv[G];
+        __syncwarp();
+        tmem_ld_g<G>(lane_addr + kColStash + j * G, sv);
+        tmem_ld_wait();
+        float a[G], mean = 0.f, zc, scur;
+        window_terms<G>(sv, M, L, Hh, c, zc, scur);
+#pragma unroll
+        for (int h = 0; h < G; ++h) {
+          a[h] = attn_weight(sv[h], M[h], c, L[h]);
+          mean += a[h];
+        }
+        mean /= (float)G;
+        float var = 0.f;
+#pragma unroll
+        for (int h = 0; h < G; ++h) var = fmaf(a[h] - mean, a[h] - mean, var);
+        var /= (float)G;
+        // |v_i| from the swizzled V tile
+        const uint8_t* vt = smem + OFF_STAGE + s * kStageBytes;
+        float vn = 0.f;
+#pragma unroll
+        for (int blk = 0; blk < D / 64; ++blk)
+#pragma unroll
+          for (int cch = 0; cch < 8; ++cch) {
+            const uint4 u4 = *reinterpret_cast<const uint4*>(vt + blk * 16384 + sw128(tok, cch));
+            const uint32_t w4[4] = {u4.x, u4.y, u4.z, u4.w};
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+              const float x0 = bf16lo(w4[e]), x1 = bf16hi(w4[e]);
+              vn = fmaf(x0, x0, vn);
+              vn = fmaf(x1, x1, vn);
+            }
+          }
+        vn = sqrtf(vn);
+        float x[5] = {mean, vn, var, 0.f, 0.f};
+        if (valid) {
+          const size_t slot = rbase + i;
+          const double Zt = p.Z[slot] + (double)zc;
+          const double St = p.S[slot] + (double)scur;
+          x[3] = Zt > 0.0 ? (float)(St / Zt) : 0.f;
+          x[4] = (float)p.pos[slot] / pos_den;
+          if (p.alpha_mode == 1) {
+            x[0] = p.acc[slot] + mean;
+            p.acc[slot] = x[0];
+          }
+          if (p.keep_features)
+#pragma unroll
+            for (int e = 0; e < 5; ++e) p.feat[slot * 5 + e] = x[e];
+        }
+        // the policy layer's input row: [r x, r, 1, 0] (LayerNorm folded into
+        // the weights) or [x, 1, 0, 0], as bf16 hi | lo | hi parts
+        float av[8];
+        if (fp.layernorm) {
+          const float xt[6] = {x[0], x[1], x[2], x[3], x[4], 1.f};
+          float q2 = 0.f;
+          int k = 0;
+#pragma unroll
+          for (int aa = 0; aa < 6; ++aa)
+#pragma unroll
+            for (int bb = aa; bb < 6; ++bb) q2 = fmaf(fp.M[k++] * xt[aa], xt[bb], q2);
+          const float rs = rsqrtf(fmaxf(q2, 0.f) + 1e-5f);
+#pragma unroll
+          for (int e = 0; e < 6; ++e) av[e] = rs * xt[e];
+          av[6] = 1.f;
+          av[7] = 0.f;
+        } else {
+#pragma unroll
+          for (int e = 0; e < 5; ++e) av[e] = x[e];
+          av[5] = 1.f;
+          av[6] = 0.f;
+          av[7] = 0.f;
+        }
+        uint32_t hi[4], lo[4];
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          const __nv_bfloat16 h0 = __float2bfloat16_rn(av[2 * e]), h1 = __float2bfloat16_rn(av[2 * e + 1]);
+          const float r0 = av[2 * e] - __bfloat162float(h0), r1 = av[2 * e + 1] - __bfloat162float(h1);
+          hi[e] = (uint32_t)__bfloat16_as_ushort(h0) | ((uint32_t)__bfloat16_as_ushort(h1) << 16);
+          lo[e] = pack_bf16(r0, r1);
+        }
+        uint8_t* at = smem + OFF_A + pb * 16384;
+        *reinterpret_cast<uint4*>(at + sw128(tok, 0)) = make_uint4(hi[0], hi[1], hi[2], hi[3]);
+        *reinterpret_cast<uint4*>(at + sw128(tok, 1)) = make_uint4(lo[0], lo[1], lo[2], lo[3]);
+        *reinterpret_cast<uint4*>(at + sw128(tok, 2)) = make_uint4(hi[0], hi[1], hi[2], hi[3]);
+        *reinterpret_cast<uint4*>(at + sw128(tok, 3)) = make_uint4(0, 0, 0, 0);
+        // attention weights as the PV operand: row h, column = token
+        uint8_t* pt = smem + OFF_P + pb * 4096 + (tok >> 6) * 2048;
+        const int tc = tok & 63;
+#pragma unroll
+        for (int h = 0; h < G; ++h)
+          *reinterpret_cast<__nv_bfloat16*>(pt + sw128(h, tc >> 3) + (tc & 7) * 2) =
+              __float2bfloat16_rn(valid ? a[h] : 0.f);
+        fence_proxy_async();
+        __syncwarp();
+        if (lane == 0) {
+          mbar_arrive(&bar[B_PFULL + pb]);
+          mbar_arrive(&bar[B_EMPTY + s]);
+        }
+      };
+      auto finish = [&](int j) {
+        const int gvj = gv + j;
+        mbar_wait(&bar[B_MFULL], gvj & 1, abort);
+        __syncwarp();
+        tc_fence_after();
+        float accp = 0.f, accn = 0.f;
+#pragma unroll
+        for (int c4 = 0; c4 < 4; ++c4) {
+          float z[32];
+          tmem_ld32(lane_addr + kColM + c4 * 32, z);
+          tmem_ld_wait();
+#pragma unroll
+          for (int e = 0; e < 32; ++e) {
+            if (c4 * 32 + e < fp.npos) accp += fmaxf(z[e], 0.f);
+            else accn += fminf(z[e], 0.f);
+          }
+        }
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&bar[B_MEMPTY]);
+        const int i = j * kTok + tok;
+        if (i < n) {
+          const float score = fp.b2 + (accp + accn);
+          sc[i] = score;
+          if (fs.write_scores) p.score[rbase + i] = score;
+        }
+      };
+      prep(0);
+      for (int j = 0; j < nT; ++j) {
+        if (j + 1 < nT) prep(j + 1);
+        finish(j);
+      }
+      g += nT;
+      gv += nT;
+      // ---------------- attention output
+      mbar_wait(&bar[B_OFULL], gr & 1, abort);
+      __syncwarp();
+      tc_fence_after();
+      float o4[4];
+      tmem_ld4(lane_addr + kColO, o4);
+      tmem_ld_wait();
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&bar[B_OEMPTY]);
+      if (tok < D) {
+        float* op = fs.out + ((r / p.kvh) * p.qh + (r % p.kvh) * G) * D;
+#pragma unroll
+        for (int h = 0; h < G; ++h) op[h * D + tok] = o4[h];
+      }
+      // ---------------- argtop_B and prune
+      if (fs.do_evict && fs.B < n) {
+        sync();
+        team_select_compact<kEpi>(p, r, n, fs.B, sc, etid, scr, sync);
+      }
+    }
+  }
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem, kTmemCols);
+  }
+  if (threadIdx.x == 0 && *abort) atomicOr(p.status, kStatusTimeout);
+}
+
+}  // namespace
+
+bool fused_eligible(const Dev& p, int n) {
+  return (p.d == 64 || p.d == 128) && (p.G == 1 || p.G == 2 || p.G == 4) && p.hidden <= 128 && n >= 1 &&
+         n <= kFusedMaxTok;
+}
+
+int fused_smem_bytes() { return kSmemBytes; }
+
+template <int D, int G>
+static cudaError_t launch_t(const FusedMaps& maps, const Dev& p, const Step& st, const FusedStep& fs,
+                            const FusedPolicy& fp, int grid, cudaStream_t s) {
+  static bool attr = false;
+  if (!attr) {
+    cudaError_t e = cudaFuncSetAttribute(fused_kernel<D, G>, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes);
+    if (e != cudaSuccess) return e;
+    attr = true;
+  }
+  fused_kernel<D, G><<<grid, kThreads, kSmemBytes, s>>>(maps.k, maps.v, p, st, fs, fp);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_fused_step(const FusedMaps& maps, const Dev& p, const Step& st, const FusedStep& fs,
+                              const FusedPolicy& fp, int num_sms, cudaStream_t s) {
+  const int grid = p.R < num_sms ? p.R : num_sms;
+  if (p.d == 128) {
+    if (p.G == 4) return launch_t<128, 4>(maps, p, st, fs, fp, grid, s);
+    if (p.G == 2) return launch_t<128, 2>(maps, p, st, fs, fp, grid, s);
+    return launch_t<128, 1>(maps, p, st, fs, fp, grid, s);
+  }
+  if (p.G == 4) return launch_t<64, 4>(maps, p, st, fs, fp, grid, s);
+  if (p.G == 2) return launch_t<64, 2>(maps, p, st, fs, fp, grid, s);
+  return launch_t<64, 1>(maps, p, st, fs, fp, grid, s);
+}
+
+}  // namespace dc
+
+// ---------------------------------------------------------------------------
+// Host-side preparation
+// ---------------------------------------------------------------------------
+#include <algorithm>
+#include <cmath>
+#include <numeric>
+
+namespace dc {
+
+typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
+                                  const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
+                                  CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+cudaError_t make_fused_maps(const Dev& p, FusedMaps* maps, const char** why) {
+  static EncodeTiledFn encode = nullptr;
+  if (!encode) {
+    void* fn = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    cudaError_t e = cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault, &q);
+    if (e != cudaSuccess || q != cudaDriverEntryPointSuccess || !fn) {
+      *why = "cuTensorMapEncodeTiled is unavailable";
+      return e != cudaSuccess ? e : cudaErrorNotSupported;
+    }
+    encode = reinterpret_cast<EncodeTiledFn>(fn);
+  }
+  const cuuint64_t dims[2] = {(cuuint64_t)p.d, (cuuint64_t)p.R * (cuuint64_t)p.cap};
+  const cuuint64_t strides[1] = {(cuuint64_t)p.d * 2};
+  const cuuint32_t box[2] = {64, 128};
+  const cuuint32_t estr[2] = {1, 1};
+  for (int which = 0; which < 2; ++which) {
+    CUresult r = encode(which ? &maps->v : &maps->k, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, which ? (void*)p.V : (void*)p.K,
+                        dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                        CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    if (r != CUDA_SUCCESS) {
+      *why = "cuTensorMapEncodeTiled rejected the K/V layout";
+      return cudaErrorInvalidValue;
+    }
+  }
+  return cudaSuccess;
+}
+
+void prepare_policy(const float* blob, int H, int layernorm, FusedPolicy* fp, std::vector<__nv_bfloat16>* wtile) {
+  const float* W1 = blob;
+  const float* b1 = W1 + 5 * H;
+  const float* gamma = b1 + H;
+  const float* beta = gamma + H;
+  const float* w2 = beta + H;
+  const double b2 = w2[H];
+  // rows w_j (8 values) of the folded first layer, in double precision
+  std::vector<double> rows((size_t)H * 8, 0.0);
+  double Mq[6][6] = {};
+  if (layernorm) {
+    double mW[5] = {}, mb = 0.0;
+    for (int j = 0; j < H; ++j) {
+      for (int k = 0; k < 5; ++k) mW[k] += W1[j * 5 + k];
+      mb += b1[j];
+    }
+    for (int k = 0; k < 5; ++k) mW[k] /= H;
+    mb /= H;
+    for (int j = 0; j < H; ++j) {
+      double cj[6];
+      for (int k = 0; k < 5; ++k) cj[k] = (double)W1[j * 5 + k] - mW[k];
+      cj[5] = (double)b1[j] - mb;
+      for (int a = 0; a < 6; ++a)
+        for (int b = 0; b < 6; ++b) Mq[a][b] += cj[a] * cj[b] / H;
+      const double s = (double)w2[j] * (double)gamma[j];
+      for (int k = 0; k < 6; ++k) rows[(size_t)j * 8 + k] = s * cj[k];
+      rows[(size_t)j * 8 + 6] = (double)w2[j] * (double)beta[j];
+    }
+  } else {
+    for (int j = 0; j < H; ++j) {
+      for (int k = 0; k < 5; ++k) rows[(size_t)j * 8 + k] = (double)w2[j] * (double)W1[j * 5 + k];
+      rows[(size_t)j * 8 + 5] = (double)w2[j] * (double)b1[j];
+    }
+  }
+  int k = 0;
+  for (int a = 0; a < 6; ++a)
+    for (int b = a; b < 6; ++b) fp->M[k++] = (float)(a == b ? Mq[a][b] : 2.0 * Mq[a][b]);
+  fp->b2 = (float)b2;
+  fp->layernorm = layernorm ? 1 : 0;
+  // hidden units with w2 >= 0 first (their term is max(z, 0), the rest min(z, 0))
+  std::vector<int> perm(H);
+  std::iota(perm.begin(), perm.end(), 0);
+  std::stable_partition(perm.begin(), perm.end(), [&](int j) { return w2[j] >= 0.f; });
+  fp->npos = (int)std::count_if(w2, w2 + H, [](float x) { return x >= 0.f; });
+  wtile->assign(128 * 32, __float2bfloat16_rn(0.f));
+  for (int jj = 0; jj < H; ++jj) {
+    const double* rj = &rows[(size_t)perm[jj] * 8];
+    for (int e = 0; e < 8; ++e) {
+      const __nv_bfloat16 hi = __float2bfloat16_rn((float)rj[e]);
+      const __nv_bfloat16 lo = __float2bfloat16_rn((float)(rj[e] - (double)__bfloat162float(hi)));
+      (*wtile)[jj * 32 + e] = hi;
+      (*wtile)[jj * 32 + 8 + e] = hi;
+      (*wtile)[jj * 32 + 16 + e] = lo;
+    }
+  }
+  fp->wtile = nullptr;
+}
+
+}  // namespace dc

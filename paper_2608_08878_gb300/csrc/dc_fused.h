@@ -1,0 +1,56 @@
+// dc_fused.h -- host-visible pieces of the fused engine: launch arguments,
+// the policy network in the form the fused kernel consumes, TMA descriptors.
+#pragma once
+
+#include <cuda.h>
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+
+#include <vector>
+
+#include "dc_common.cuh"
+
+namespace dc {
+
+// Most tokens a row may hold for the fused kernel (one CTA per row: the raw
+// logits of the row live in TMEM, the scores in shared memory).
+constexpr int kFusedMaxTok = 10240;
+
+struct FusedMaps {
+  CUtensorMap k, v;  // [R * cap][d] bf16, boxes of 64 dims x 128 tokens, 128-byte swizzle
+};
+
+struct FusedStep {
+  const __nv_bfloat16* q;
+  float* out;
+  int do_evict;      // 1: select and compact in the same kernel
+  int B;             // tokens to keep when do_evict
+  int write_scores;  // 1: also store scores in Dev::score (for dc_evict)
+};
+
+// The policy MLP folded for the tensor cores (see prepare_policy):
+//   z_j = <a, w_j> with a = [r x, r, 1, 0] (LayerNorm) or [x, 1, 0, 0];
+//   score = b2 + sum_{j < npos} max(z_j, 0) + sum_{j >= npos} min(z_j, 0);
+//   r = 1 / sqrt(x~^T M x~ + 1e-5), x~ = [x, 1] (LayerNorm variance).
+struct FusedPolicy {
+  float M[21];                   // upper triangle, off-diagonal terms doubled
+  float b2;
+  int npos;
+  int layernorm;
+  const __nv_bfloat16* wtile;    // device [128][32]: rows w_j as bf16 hi | hi | lo | 0
+};
+
+bool fused_eligible(const Dev& p, int n);
+int fused_smem_bytes();
+
+// Builds the two TMA descriptors of the K and V buffers.
+cudaError_t make_fused_maps(const Dev& p, FusedMaps* maps, const char** why);
+
+// Folds a policy blob [W1 | b1 | gamma | beta | w2 | b2] (hidden H) into
+// FusedPolicy fields and the host copy of the weight tile (128 * 32 bf16).
+void prepare_policy(const float* blob, int H, int layernorm, FusedPolicy* fp, std::vector<__nv_bfloat16>* wtile);
+
+cudaError_t launch_fused_step(const FusedMaps& maps, const Dev& p, const Step& st, const FusedStep& fs,
+                              const FusedPolicy& fp, int num_sms, cudaStream_t s);
+
+}  // namespace dc

@@ -102,29 +102,35 @@ __device__ __forceinline__ int row_q_offset(const Dev& p, int r) {
 
 // ---------------------------------------------------------------------------
 // Pass 1: raw logits of the current queries (to scratch), per-split softmax
-// statistics (m, l, u2) and the departing query's window terms.
+// statistics (m, l, u2) and the window-sum update: the previous step's query
+// joins the stored sums S, Z and the departing one (step t - w) leaves them,
+// both recomputed here from their ring entries.
 // grid (nsplit, R), block kTile.
 // ---------------------------------------------------------------------------
 template <int D, int G>
 __global__ void __launch_bounds__(kTile) split_qk_kernel(Dev p, Step st,
                                                          const __nv_bfloat16* __restrict__ q) {
-  __shared__ float qs[2 * G][D];
+  __shared__ float qs[3 * G][D];  // current, previous, departing
   __shared__ __align__(16) __nv_bfloat16 kt[kTile][D + 8];
-  __shared__ float dep_ml[G][3];
+  __shared__ float ring_ml[2][G][3];  // (m, l, H) of previous / departing
   __shared__ float red[kTile / kWarp][G][3];
   const int r = blockIdx.y, sp = blockIdx.x, tid = threadIdx.x;
   const int c0 = sp * st.chunk, c1 = min(st.n, c0 + st.chunk);
   const int qo = row_q_offset(p, r);
+  const __nv_bfloat16* rq_prev = p.ring_q + ((size_t)r * p.w + st.slot_prev) * G * D;
+  const __nv_bfloat16* rq_dep = p.ring_q + ((size_t)r * p.w + st.slot) * G * D;
   for (int e = tid; e < G * D; e += blockDim.x) {
     qs[e / D][e % D] = __bfloat162float(q[qo + e]);
-    qs[G + e / D][e % D] =
-        st.has_dep ? __bfloat162float(p.ring_q[((size_t)r * p.w + st.slot) * G * D + e]) : 0.f;
+    qs[G + e / D][e % D] = st.has_prev ? __bfloat162float(rq_prev[e]) : 0.f;
+    qs[2 * G + e / D][e % D] = st.has_dep ? __bfloat162float(rq_dep[e]) : 0.f;
   }
-  if (tid < G) {
-    const float* rs = p.ring_stats + (((size_t)r * p.w + st.slot) * G + tid) * 4;
-    dep_ml[tid][0] = rs[0];
-    dep_ml[tid][1] = rs[1];
-    dep_ml[tid][2] = rs[2];
+  if (tid < 2 * G) {
+    const int which = tid / G, h = tid % G;
+    const int slot = which == 0 ? st.slot_prev : st.slot;
+    const float* rs = p.ring_stats + (((size_t)r * p.w + slot) * G + h) * 4;
+    ring_ml[which][h][0] = rs[0];
+    ring_ml[which][h][1] = rs[1];
+    ring_ml[which][h][2] = rs[2];
   }
   float m[G], l[G], u[G];
 #pragma unroll
@@ -136,26 +142,32 @@ __global__ void __launch_bounds__(kTile) split_qk_kernel(Dev p, Step st,
     load_tile<D>(kt, p.K + ((size_t)r * p.cap + base) * D, rows);
     __syncthreads();
     if (tid < rows) {
-      const int i = base + tid;
-      float s[2 * G];
-      if (st.has_dep) dots<D, 2 * G>(&kt[tid][0], qs, s);
-      else dots<D, G>(&kt[tid][0], qs, s);
-      float* lo = p.logit + ((size_t)r * p.cap + i) * G;
+      const size_t slot = (size_t)r * p.cap + base + tid;
+      float s[3 * G];
+      dots<D, 3 * G>(&kt[tid][0], qs, s);
+      float* lo = p.logit + slot * G;
 #pragma unroll
       for (int h = 0; h < G; ++h) {
         lo[h] = s[h];
         online_add(m[h], l[h], u[h], s[h], c);
       }
-      float z = 0.f, sh = 0.f;
-      if (st.has_dep && p.pos[(size_t)r * p.cap + i] <= st.p_dep) {
-        float dm[G], dl[G], dH[G];
+      if (st.has_prev || st.has_dep) {
+        const int pos = p.pos[slot];
+        float zp = 0.f, sp_ = 0.f, zd = 0.f, sd = 0.f;
+        float rm[G], rl[G], rH[G];
+        if (st.has_prev && pos <= st.p_prev) {
 #pragma unroll
-        for (int h = 0; h < G; ++h) { dm[h] = dep_ml[h][0]; dl[h] = dep_ml[h][1]; dH[h] = dep_ml[h][2]; }
-        window_terms<G>(s + G, dm, dl, dH, c, z, sh);
+          for (int h = 0; h < G; ++h) { rm[h] = ring_ml[0][h][0]; rl[h] = ring_ml[0][h][1]; rH[h] = ring_ml[0][h][2]; }
+          window_terms<G>(s + G, rm, rl, rH, c, zp, sp_);
+        }
+        if (st.has_dep && pos <= st.p_dep) {
+#pragma unroll
+          for (int h = 0; h < G; ++h) { rm[h] = ring_ml[1][h][0]; rl[h] = ring_ml[1][h][1]; rH[h] = ring_ml[1][h][2]; }
+          window_terms<G>(s + 2 * G, rm, rl, rH, c, zd, sd);
+        }
+        p.Z[slot] = (p.Z[slot] + (double)zp) - (double)zd;
+        p.S[slot] = (p.S[slot] + (double)sp_) - (double)sd;
       }
-      float* dp = p.dep + ((size_t)r * p.cap + i) * 2;
-      dp[0] = z;
-      dp[1] = sh;
     }
   }
   // Merge the per-thread (m, l, u2) of each head across the CTA.
@@ -276,11 +288,9 @@ __global__ void __launch_bounds__(kTile) split_v_kernel(Dev p, Step st) {
         }
       }
       vn = sqrtf(vn);
-      const float* dp = p.dep + slot * 2;
-      double Z = p.Z[slot] - (double)dp[0] + (double)zc;
-      double S = p.S[slot] - (double)dp[1] + (double)sc;
-      p.Z[slot] = Z;
-      p.S[slot] = S;
+      // H_i over the whole window: stored sums (earlier queries) + this step
+      const double Z = p.Z[slot] + (double)zc;
+      const double S = p.S[slot] + (double)sc;
       float alpha = mean;
       if (p.alpha_mode == 1) {
         alpha = p.acc[slot] + mean;

@@ -28,7 +28,7 @@ EXPORTS = ["dc_config_default", "dc_cache_create", "dc_cache_destroy", "dc_polic
            "dc_policy_init", "dc_policy_set_weights", "dc_append", "dc_decode_step",
            "dc_decode_step_host", "dc_evict", "dc_full_decode", "dc_get_length", "dc_buffer_bytes",
            "dc_copy_buffer", "dc_sync", "dc_last_error", "dc_phase_name", "dc_profile_enable",
-           "dc_profile_read"]
+           "dc_profile_read", "dc_step", "dc_step_host", "dc_engine"]
 PHASES = ["append", "attend", "stats", "score", "combine", "evict", "full"]
 
 
@@ -71,6 +71,9 @@ def lib():
             L.dc_decode_step.argtypes = [P, P, P, P, P]
             L.dc_decode_step_host.argtypes = [P, P, P, P, P]
             L.dc_evict.argtypes = [P, I]
+            L.dc_step.argtypes = [P, P, P, P, P, I]
+            L.dc_step_host.argtypes = [P, P, P, P, P, I]
+            L.dc_engine.argtypes = [P, I, C.POINTER(I)]
             L.dc_full_decode.argtypes = [P, P, P]
             L.dc_get_length.argtypes = [P, C.POINTER(I), C.POINTER(C.c_longlong)]
             L.dc_buffer_bytes.argtypes = [P, I, C.POINTER(S)]
@@ -180,6 +183,22 @@ class DistillCache:
     def decode_step_host(self, q, k_new, v_new, out) -> None:
         """Host (preferably pinned) tensors; synchronises before returning."""
         self._check(lib().dc_decode_step_host(self._h, _ptr(q), _ptr(k_new), _ptr(v_new), _ptr(out)))
+
+    def step(self, q, k_new, v_new, out=None, budget: int = 0):
+        """decode_step + evict (one kernel on the fused engine)."""
+        import torch
+        if out is None:
+            out = torch.empty(q.shape, dtype=torch.float32, device=q.device)
+        self._check(lib().dc_step(self._h, _ptr(q), _ptr(k_new), _ptr(v_new), _ptr(out), budget))
+        return out
+
+    def step_host(self, q, k_new, v_new, out, budget: int = 0) -> None:
+        self._check(lib().dc_step_host(self._h, _ptr(q), _ptr(k_new), _ptr(v_new), _ptr(out), budget))
+
+    def engine(self, n: int = 0) -> str:
+        e = C.c_int()
+        self._check(lib().dc_engine(self._h, n, C.byref(e)))
+        return {1: "split", 2: "fused"}[e.value]
 
     def evict(self, budget: int = 0) -> None:
         self._check(lib().dc_evict(self._h, budget))

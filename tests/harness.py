@@ -158,8 +158,9 @@ class LockStep:
         V = self.cache.buffer(dc.BUF_V, r, 1)[0, :n].view(self.torch.int16).cpu().numpy().view(np.uint16)
         ok, ov = orow.kv_bits()
         assert np.array_equal(K[order], ok) and np.array_equal(V[order], ov), f"row {r}: K/V bytes differ"
+        # the stored sums cover the window's queries before the last step
         S = self._row_slice(dc.BUF_S, r, n)[order]
         Z = self._row_slice(dc.BUF_Z, r, n)[order]
-        oS, oZ, _ = orow.window_sums()
+        oS, oZ = orow.window_sums_prior()
         close_rel(Z, oZ, FEAT_RTOL, FEAT_FLOOR, f"row {r} window mass Z")
         close_rel(S, oS, FEAT_RTOL, FEAT_FLOOR, f"row {r} window sum S")

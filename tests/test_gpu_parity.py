@@ -13,7 +13,7 @@ from harness import LockStep, check_attention
 
 pytestmark = pytest.mark.gpu
 
-ENGINES = [0, 1]
+ENGINES = [1, 2]  # split, fused (forced wherever the step fits it)
 
 
 @pytest.fixture(scope="module", autouse=True)
@@ -100,6 +100,41 @@ def test_mistral_single_layer(engine):
         ls.step(check=(s < 3 or s % 8 == 0 or s >= 64))
 
 
+@pytest.mark.parametrize("engine", ENGINES)
+def test_step_equals_decode_then_evict(engine):
+    """dc_step (one kernel on the fused engine) leaves the cache and output
+    bit-identical to dc_decode_step followed by dc_evict."""
+    import torch
+    from paper_2608_08878_gb300 import dc
+    wl = synth.MISTRAL_1L.with_(prompt_len=700, budget=256, window=5)
+    a, b = LockStep(wl, [], engine=engine), LockStep(wl, [], engine=engine)
+    a.load_prompt()
+    b.load_prompt()
+    for s in range(12):
+        q, kn, vn = a._inputs(s)
+        budget = 200 if s == 6 else 0  # one step with a smaller budget: many evictions
+        oa = a.cache.step(q, kn, vn, budget=budget)
+        ob = b.cache.decode_step(q, kn, vn)
+        b.cache.evict(budget)
+        torch.cuda.synchronize()
+        assert torch.equal(oa, ob), s
+        assert a.cache.length() == b.cache.length()
+        n = a.cache.length()[0]
+        for which in (dc.BUF_K, dc.BUF_V, dc.BUF_POS, dc.BUF_S, dc.BUF_Z):
+            assert torch.equal(a.cache.buffer(which)[:, :n], b.cache.buffer(which)[:, :n]), (s, which)
+
+
+def test_engine_choice():
+    from paper_2608_08878_gb300 import dc
+    big = dc.DistillCache(32, 8, 128, 200, 100, batch=1)
+    assert big.engine() == "fused" and big.engine(20000) == "split"
+    small = dc.DistillCache(1, 2, 64, 200, 100, q_heads=4)
+    assert small.engine() == "split"
+    forced = dc.DistillCache(1, 2, 64, 200, 100, q_heads=4, engine=2)
+    assert forced.engine() == "fused"
+    assert dc.DistillCache(1, 2, 64, 200, 100, q_heads=16, engine=2).engine() == "split"  # group 8
+
+
 def test_full_decode_matches_oracle():
     import torch
     import oracle
@@ -175,7 +210,7 @@ def test_aggressive_sampled_rows():
     """32 layers, batch 16, 32K context, budget 3277 (10%), hot sets reshuffled
     every 16 steps: crosses one reshuffle, 2 sampled rows."""
     wl = synth.AGGRESSIVE
-    ls = LockStep(wl, [7, wl.rows - 3], engine=0, device_inputs=True)
+    ls = LockStep(wl, [7, wl.rows - 3], engine=0, device_inputs=True)  # auto: fused steady steps
     ls.load_prompt()
     for s in range(18):
         ls.step(check=(s < 2 or s >= 15))

@@ -191,7 +191,11 @@ def _bruteforce_run(alpha_mode, w, steps, seed):
         Hq = np.array([scipy.stats.entropy(a[h]) for h in range(G)])
         history.append(({int(p): a[:, i] for i, p in enumerate(pos)}, Hq))
         S_w, Z_w, acc = row.window_sums()
+        S_p, Z_p = row.window_sums_prior()
+        newest = history[-1][0]
         for i, p in enumerate(pos):
+            np.testing.assert_allclose(Z_p[i] + newest[int(p)].sum(), Z_w[i], rtol=1e-12)
+            np.testing.assert_allclose(S_p[i] + (newest[int(p)] * history[-1][1]).sum(), S_w[i], rtol=1e-12)
             Z = S = 0.0
             for amap, Hh in history[-w:]:
                 if int(p) in amap:
