@@ -161,12 +161,14 @@ typedef enum {
   DC_BUF_K = 0,     /* bf16 [R][capacity][head_dim] */
   DC_BUF_V = 1,     /* bf16 [R][capacity][head_dim] */
   DC_BUF_POS = 2,   /* int32 [R][capacity] absolute position of each slot */
-  DC_BUF_S = 3,     /* fp64 [R][capacity] entropy-weighted window mass S_i */
-  DC_BUF_Z = 4,     /* fp64 [R][capacity] window mass Z_i */
+  DC_BUF_S = 3,     /* fp64 [R][capacity] entropy-weighted window mass S_i over the
+                       window's queries before the last step (Sec. 3.1.1, H_i) */
+  DC_BUF_Z = 4,     /* fp64 [R][capacity] window mass Z_i, same queries */
   DC_BUF_ACC = 5,   /* fp32 [R][capacity] cumulative alpha (alpha_mode 1) */
   DC_BUF_SCORE = 6, /* fp32 [R][capacity] policy scores of the last step */
   DC_BUF_FEAT = 7,  /* fp32 [R][capacity][5] features (keep_features only) */
-  DC_BUF_HQ = 8     /* fp32 [R][q_heads / kv_heads] entropy of each head, last step */
+  DC_BUF_HQ = 8,    /* fp32 [R][q_heads / kv_heads] entropy of each head, last step */
+  DC_BUF_VNORM = 9  /* fp32 [R][capacity] |v_i|_2 of each slot */
 } dc_buffer;
 
 /* Size in bytes of one row of an internal buffer (0 if the handle has none of

@@ -275,7 +275,7 @@ dc_status dc_cache_create(int layers, int kv_heads, int head_dim, int capacity, 
   if (cfg.alpha_mode != 0 && cfg.alpha_mode != 1) return fail(nullptr, DC_ERR_INVALID_ARG, "alpha_mode must be 0 or 1");
   if (cfg.engine < 0 || cfg.engine > 2) return fail(nullptr, DC_ERR_INVALID_ARG, "engine must be 0, 1 or 2");
   const long long R = (long long)layers * cfg.batch * kv_heads;
-  if (R > 65535 || (long long)capacity * R > (1ll << 40))
+  if (R > 65535 || (long long)capacity * R > (1ll << 40) || capacity > (1 << 30))
     return fail(nullptr, DC_ERR_INVALID_ARG, "cache too large");
 
   dc_cache* h = new dc_cache();
@@ -292,12 +292,12 @@ dc_status dc_cache_create(int layers, int kv_heads, int head_dim, int capacity, 
     return s;
   }
   dc::Dev& p = h->dev;
-  p.R = (int)R; p.cap = capacity; p.d = head_dim; p.G = G; p.qh = cfg.q_heads; p.kvh = kv_heads;
+  p.R = (int)R; p.cap = capacity; p.stride = (capacity + 127) / 128 * 128; p.d = head_dim; p.G = G; p.qh = cfg.q_heads; p.kvh = kv_heads;
   p.w = cfg.window; p.hidden = cfg.mlp_hidden; p.layernorm = cfg.layernorm ? 1 : 0;
   p.alpha_mode = cfg.alpha_mode; p.keep_features = cfg.keep_features ? 1 : 0;
   p.c = (float)(1.4426950408889634 / std::sqrt((double)head_dim));
   p.smax = (int)std::max(1ll, std::min(64ll, (8ll * h->num_sms + R - 1) / R));
-  const size_t RC = (size_t)R * capacity;
+  const size_t RC = (size_t)R * p.stride;
   const size_t kv = RC * head_dim * sizeof(__nv_bfloat16);
   const size_t blob = dc_policy_blob_len(cfg.mlp_hidden);
   cudaError_t ae = cudaSuccess;
@@ -305,8 +305,8 @@ dc_status dc_cache_create(int layers, int kv_heads, int head_dim, int capacity, 
   A(&p.K, kv);
   A(&p.V, kv);
   A(&p.pos, RC * sizeof(int));
-  A(&p.S, RC * sizeof(double));
-  A(&p.Z, RC * sizeof(double));
+  A(&p.vnorm, RC * sizeof(float));
+  A(&p.SZ, RC * sizeof(float4));
   if (cfg.alpha_mode == 1) A(&p.acc, RC * sizeof(float));
   A(&p.score, RC * sizeof(float));
   if (p.keep_features) A(&p.feat, RC * 5 * sizeof(float));
@@ -336,7 +336,7 @@ dc_status dc_cache_create(int layers, int kv_heads, int head_dim, int capacity, 
   dc_policy_init(cfg.seed, cfg.mlp_hidden, w.data(), blob);
   e = cudaMemcpyAsync(pol, w.data(), blob * sizeof(float), cudaMemcpyHostToDevice, h->stream);
   if (e == cudaSuccess) e = cudaStreamSynchronize(h->stream);
-  if (e == cudaSuccess && cfg.engine != 1 && dc::fused_eligible(p, 1) && R * (long long)capacity < (1ll << 31)) {
+  if (e == cudaSuccess && cfg.engine != 1 && dc::fused_eligible(p, 1) && R * (long long)p.stride < (1ll << 31)) {
     const char* why = "";
     cudaError_t fe = dalloc(h, &h->wtile, 128 * 32 * sizeof(__nv_bfloat16));
     if (fe == cudaSuccess) fe = dc::make_fused_maps(p, &h->maps, &why);
@@ -536,40 +536,60 @@ dc_status dc_get_length(dc_cache* h, int* n, long long* seen) {
   return DC_OK;
 }
 
-// Base pointer and bytes per row of an internal buffer.
-static char* buffer_ptr(dc_cache* h, dc_buffer which, size_t* row_bytes) {
+// Base pointer, element size and elements per slot of an internal buffer
+// (stored with the padded row stride; the ABI view is [R][capacity]).
+static char* buffer_ptr(dc_cache* h, dc_buffer which, size_t* elem, size_t* per_slot) {
   const dc::Dev& p = h->dev;
-  const size_t C = (size_t)p.cap;
+  *per_slot = 1;
   switch (which) {
-    case DC_BUF_K: *row_bytes = C * p.d * 2; return (char*)p.K;
-    case DC_BUF_V: *row_bytes = C * p.d * 2; return (char*)p.V;
-    case DC_BUF_POS: *row_bytes = C * sizeof(int); return (char*)p.pos;
-    case DC_BUF_S: *row_bytes = C * sizeof(double); return (char*)p.S;
-    case DC_BUF_Z: *row_bytes = C * sizeof(double); return (char*)p.Z;
-    case DC_BUF_ACC: *row_bytes = p.acc ? C * sizeof(float) : 0; return (char*)p.acc;
-    case DC_BUF_SCORE: *row_bytes = C * sizeof(float); return (char*)p.score;
-    case DC_BUF_FEAT: *row_bytes = p.feat ? C * 5 * sizeof(float) : 0; return (char*)p.feat;
-    case DC_BUF_HQ: *row_bytes = (size_t)p.G * sizeof(float); return (char*)p.hq;
+    case DC_BUF_K: *elem = 2; *per_slot = p.d; return (char*)p.K;
+    case DC_BUF_V: *elem = 2; *per_slot = p.d; return (char*)p.V;
+    case DC_BUF_POS: *elem = 4; return (char*)p.pos;
+    case DC_BUF_S: *elem = 8; return (char*)p.SZ;
+    case DC_BUF_Z: *elem = 8; return (char*)p.SZ;
+    case DC_BUF_ACC: *elem = 4; return (char*)p.acc;
+    case DC_BUF_SCORE: *elem = 4; return (char*)p.score;
+    case DC_BUF_FEAT: *elem = 4; *per_slot = 5; return (char*)p.feat;
+    case DC_BUF_HQ: *elem = 4; *per_slot = p.G; return (char*)p.hq;
+    case DC_BUF_VNORM: *elem = 4; return (char*)p.vnorm;
   }
-  *row_bytes = 0;
+  *elem = 0;
   return nullptr;
 }
 
-dc_status dc_buffer_bytes(dc_cache* h, dc_buffer which, size_t* row_bytes) {
-  if (!valid(h) || !row_bytes) return DC_ERR_INVALID_ARG;
-  buffer_ptr(h, which, row_bytes);
+static size_t row_bytes(dc_cache* h, dc_buffer which) {
+  size_t elem = 0, per = 0;
+  char* b = buffer_ptr(h, which, &elem, &per);
+  if (!b) return 0;
+  return which == DC_BUF_HQ ? elem * per : elem * per * (size_t)h->capacity;
+}
+
+dc_status dc_buffer_bytes(dc_cache* h, dc_buffer which, size_t* rb) {
+  if (!valid(h) || !rb) return DC_ERR_INVALID_ARG;
+  *rb = row_bytes(h, which);
   return DC_OK;
 }
 
 dc_status dc_copy_buffer(dc_cache* h, dc_buffer which, int row0, int nrows, void* dst, size_t bytes) {
   DC_CHECK_HANDLE(h);
-  size_t rb = 0;
-  char* src = buffer_ptr(h, which, &rb);
+  size_t elem = 0, per = 0;
+  char* src = buffer_ptr(h, which, &elem, &per);
+  const size_t rb = row_bytes(h, which);
   if (!src || rb == 0 || !dst) return fail(h, DC_ERR_INVALID_ARG, "the cache has no such buffer");
   if (row0 < 0 || nrows < 0 || row0 + nrows > h->dev.R || bytes != rb * (size_t)nrows)
     return fail(h, DC_ERR_INVALID_ARG, "row range or size mismatch");
   if (nrows == 0) return DC_OK;
-  DC_CUDA(h, cudaMemcpyAsync(dst, src + rb * (size_t)row0, bytes, cudaMemcpyDeviceToDevice, h->stream));
+  if (which == DC_BUF_S || which == DC_BUF_Z) {
+    dc::launch_convert_sz(h->dev, row0, nrows, which == DC_BUF_S ? 0 : 1, (double*)dst, h->stream);
+    return launch_error(h, "window-sum copy");
+  }
+  if (which == DC_BUF_HQ) {
+    DC_CUDA(h, cudaMemcpyAsync(dst, src + rb * (size_t)row0, bytes, cudaMemcpyDeviceToDevice, h->stream));
+    return DC_OK;
+  }
+  const size_t spitch = elem * per * (size_t)h->dev.stride;
+  DC_CUDA(h, cudaMemcpy2DAsync(dst, rb, src + spitch * (size_t)row0, spitch, rb, (size_t)nrows,
+                               cudaMemcpyDeviceToDevice, h->stream));
   return DC_OK;
 }
 

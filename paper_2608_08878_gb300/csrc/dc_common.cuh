@@ -1,21 +1,25 @@
 // dc_common.cuh -- device-side layout, parameters and shared arithmetic of the
 // DistillCache decode step (sm_103a).
 //
-// Row r = (layer * batch + b) * kv_heads + g owns `cap` slots. Per-slot data:
-//   K, V   bf16 [R][cap][d]      keys / values
-//   pos    int32 [R][cap]        absolute position (tokens seen before it)
-//   S, Z   fp64 [R][cap]         window sums of the entropy feature H_i over
-//                                the window's queries BEFORE the last step
+// Row r = (layer * batch + b) * kv_heads + g owns `cap` slots, laid out with a
+// row stride of `stride` slots (cap rounded up to 128, so that every 128-token
+// tile of a row is 16-byte aligned and stays inside the row). Per-slot data:
+//   K, V   bf16 [R][stride][d]   keys / values
+//   pos    int32 [R][stride]     absolute position (tokens seen before it)
+//   vnorm  fp32 [R][stride]      |v_i|_2, computed once when the token is appended
+//   SZ     fp32x4 [R][stride]    window sums of the entropy feature H_i as
+//                                double-float pairs (S_hi, S_lo, Z_hi, Z_lo),
+//                                over the window's queries BEFORE the last step
 //                                (the last step's terms are added, and the
 //                                departing query's subtracted, by the next
 //                                step's attention pass; both are recomputed
 //                                by the same code, so they cancel bit for bit)
-//   acc    fp32 [R][cap]         cumulative alpha (alpha_mode 1 only)
-//   score  fp32 [R][cap]         policy score of the last decode step
+//   acc    fp32 [R][stride]      cumulative alpha (alpha_mode 1 only)
+//   score  fp32 [R][stride]      policy score of the last decode step
 // Per-row ring of the last w decode queries (the window of H_i, Sec. 3.1.1):
 //   ring_q     bf16 [R][w][G][d] the query vectors
-//   ring_stats fp32 [R][w][G][4] (m, l, H, 0): max raw logit, softmax
-//              denominator 2^((s-m)c) summed, entropy in nats
+//   ring_stats fp32 [R][w][G][4] (m, l, H, nl): max raw logit, softmax
+//              denominator sum of 2^((s-m)c), entropy in nats, -log2(l)
 #pragma once
 
 #include <cuda_bf16.h>
@@ -31,12 +35,12 @@ constexpr unsigned kStatusBadShape = 1u;
 constexpr unsigned kStatusTimeout = 2u;
 
 struct Dev {
-  int R, cap, d, G, qh, kvh, w, hidden, layernorm, alpha_mode, keep_features;
+  int R, cap, stride, d, G, qh, kvh, w, hidden, layernorm, alpha_mode, keep_features;
   __nv_bfloat16* K;
   __nv_bfloat16* V;
   int* pos;
-  double* S;
-  double* Z;
+  float* vnorm;
+  float4* SZ;
   float* acc;
   float* score;
   float* feat;
@@ -46,10 +50,10 @@ struct Dev {
   const float* policy;
   unsigned* status;
   // scratch of the split engine
-  float* logit;   // [R][cap][G]
+  float* logit;   // [R][stride][G]
   float* part;    // [R][smax][G][4]: per-split (m, l, u2, 0)
   float* opart;   // [R][smax][G][d]
-  int* holes;     // [R][cap]
+  int* holes;     // [R][stride]
   int smax;
   float c;        // log2(e) / sqrt(d): raw logit difference -> log2 units
 };
@@ -74,28 +78,50 @@ __device__ __forceinline__ float ex2(float x) {
   return y;
 }
 
-// Attention weight a = 2^((s - m) c) / l of a token with raw logit s under a
-// query whose max raw logit is m and whose denominator is l. Written with
-// explicitly rounded operations so that the value is bit-identical wherever
-// it is evaluated: the term a query adds to Z_i and S_i at its own step is
-// subtracted again, bit for bit, when it leaves the window w steps later.
-__device__ __forceinline__ float attn_weight(float s, float m, float c, float l) {
-  return __fdiv_rn(ex2(__fmul_rn(__fsub_rn(s, m), c)), l);
+// Attention weight a = 2^((s - m) c) / l = 2^((s - m) c + nl), nl = -log2(l),
+// of a token with raw logit s under a query whose max raw logit is m. Written
+// with explicitly rounded operations so that the value is bit-identical
+// wherever it is evaluated: the term a query adds to the window sums one step
+// after its own is subtracted again, bit for bit, when it leaves the window.
+__device__ __forceinline__ float attn_weight(float s, float m, float c, float nl) {
+  return ex2(__fmaf_rn(__fsub_rn(s, m), c, nl));
 }
 
 // (Z, S) terms of one query step for one token: sum over heads of a_h and of
 // a_h * H_h, accumulated in head order with rounded adds (see attn_weight).
 template <int G>
-__device__ __forceinline__ void window_terms(const float* s, const float* m, const float* l,
+__device__ __forceinline__ void window_terms(const float* s, const float* m, const float* nl,
                                              const float* H, float c, float& z, float& sh) {
   z = 0.f;
   sh = 0.f;
 #pragma unroll
   for (int h = 0; h < G; ++h) {
-    float a = attn_weight(s[h], m[h], c, l[h]);
+    float a = attn_weight(s[h], m[h], c, nl[h]);
     z = __fadd_rn(z, a);
     sh = __fadd_rn(sh, __fmul_rn(a, H[h]));
   }
+}
+
+// Double-float accumulation (a value held as an unevaluated sum hi + lo, about
+// 48 significant bits): (hi, lo) += x with Knuth's TwoSum and a renormalising
+// Fast2Sum. The window sums stay exact enough that adding a term and
+// subtracting the same term many steps later leaves no visible residue.
+__device__ __forceinline__ void df_add(float& hi, float& lo, float x) {
+  const float s = __fadd_rn(hi, x);
+  const float bb = __fsub_rn(s, hi);
+  const float e = __fadd_rn(__fsub_rn(hi, __fsub_rn(s, bb)), __fsub_rn(x, bb));
+  const float t = __fadd_rn(e, lo);
+  hi = __fadd_rn(s, t);
+  lo = __fsub_rn(t, __fsub_rn(hi, s));
+}
+
+// Window sums after this step's update: S += sp - sd, Z += zp - zd.
+__device__ __forceinline__ float4 window_update(float4 sz, float sp, float sd, float zp, float zd) {
+  df_add(sz.x, sz.y, sp);
+  df_add(sz.x, sz.y, -sd);
+  df_add(sz.z, sz.w, zp);
+  df_add(sz.z, sz.w, -zd);
+  return sz;
 }
 
 // Order-preserving 32-bit key of a score for the top-B selection: larger key =

@@ -19,7 +19,7 @@ __global__ void __launch_bounds__(kEvictThreads) evict_kernel(Dev p, int n, int 
   const SelectScratch scr{hist, sh, wsum, best, best_slot};
   auto sync = [] { __syncthreads(); };
   const int r = blockIdx.x;
-  team_select_compact<kEvictThreads>(p, r, n, B, p.score + (size_t)r * p.cap, threadIdx.x, scr, sync);
+  team_select_compact<kEvictThreads>(p, r, n, B, p.score + (size_t)r * p.stride, threadIdx.x, scr, sync);
 }
 
 void launch_evict(const Dev& p, int n, int B, cudaStream_t s) {

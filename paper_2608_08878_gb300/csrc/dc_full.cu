@@ -49,7 +49,7 @@ __global__ void __launch_bounds__(kFullTile) full_split_kernel(Dev p, int n, int
   for (int base = c0; base < c1; base += kFullTile) {
     const int rows = min(kFullTile, c1 - base);
     __syncthreads();
-    full_load_tile<D>(kt, p.K + ((size_t)r * p.cap + base) * D, rows);
+    full_load_tile<D>(kt, p.K + ((size_t)r * p.stride + base) * D, rows);
     __syncthreads();
     float s[G];
 #pragma unroll
@@ -105,7 +105,7 @@ __global__ void __launch_bounds__(kFullTile) full_split_kernel(Dev p, int n, int
     }
     // V tile reuses the key buffer
     __syncthreads();
-    full_load_tile<D>(kt, p.V + ((size_t)r * p.cap + base) * D, rows);
+    full_load_tile<D>(kt, p.V + ((size_t)r * p.stride + base) * D, rows);
     __syncthreads();
     if (owns) {
       const float f = scale[oh];

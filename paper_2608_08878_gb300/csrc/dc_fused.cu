@@ -11,7 +11,8 @@
 //              with TMA (128-byte swizzle) through a 3-stage ring;
 //   warp 1     MMA issuer (one lane): tcgen05.mma, accumulators in TMEM:
 //                S  = K Q^T        [128 tokens x 16]  per K tile
-//                O^T += V^T P^T    [d x 16]           per V tile (P = weights)
+//                O^T += V^T P^T    [d x 16]           per V tile (P = weights,
+//                                  bf16 high and low parts in separate columns)
 //                Z  = A W^T        [128 tokens x 128] per V tile (policy layer)
 //   warps 2-5  epilogue, one token (TMEM lane) per thread:
 //                K pass: online softmax statistics, window-sum update (the
@@ -22,6 +23,11 @@
 //
 // TMEM columns: S tiles [0, 32), O [32, 48), policy layer [64, 192), the
 // logit stash [192, 512) (G columns per tile of 128 tokens).
+//
+// Per-token state rides along with the tiles: TMA bulk copies bring the
+// positions and window sums with each K tile and the positions and |v| with
+// each V tile. The K pass writes the updated window sums back; the V pass
+// re-reads them (L2-resident by then) with loads issued two tiles ahead.
 #include <cuda.h>
 
 #include "dc_common.cuh"
@@ -36,7 +42,13 @@ using namespace sm100;
 namespace {
 
 constexpr int kStages = 3;
-constexpr int kStageBytes = 32768;
+// stage: K or V tile (32 KB, two 64-dim column blocks) + the tile's per-token
+// state: positions (512 B), |v| (512 B, V tiles) or window sums (2 KB, K tiles)
+constexpr int kTileRegion = 32768;
+constexpr int kOffPos = kTileRegion;          // int32 [128]
+constexpr int kOffVn = kTileRegion + 512;     // fp32 [128]
+constexpr int kOffSZ = kTileRegion + 1024;    // fp32x4 [128]
+constexpr int kStageBytes = kTileRegion + 3072;
 constexpr int kTok = 128;
 constexpr int kThreads = 192;
 constexpr int kEpi = 128;
@@ -230,11 +242,14 @@ __global__ void __launch_bounds__(kThreads, 1)
           for (int j = 0; j < nT; ++j, ++g) {
             const int s = g % kStages;
             if (!mbar_wait(&bar[B_EMPTY + s], ((g / kStages) & 1) ^ 1, abort)) break;
-            mbar_expect_tx(&bar[B_FULL + s], kTileBytes);
+            mbar_expect_tx(&bar[B_FULL + s], kTileBytes + (pass ? 1024u : 2560u));
             uint8_t* dst = smem + OFF_STAGE + s * kStageBytes;
-            const int y = r * p.cap + j * kTok;
+            const int y = r * p.stride + j * kTok;
             tma_load_2d(dst, tm, 0, y, &bar[B_FULL + s], pol);
             if (D == 128) tma_load_2d(dst + 16384, tm, 64, y, &bar[B_FULL + s], pol);
+            bulk_load(dst + kOffPos, p.pos + y, 512, &bar[B_FULL + s]);
+            if (pass) bulk_load(dst + kOffVn, p.vnorm + y, 512, &bar[B_FULL + s]);
+            else bulk_load(dst + kOffSZ, p.SZ + y, 2048, &bar[B_FULL + s]);
             issued = g + 1;
           }
         }
@@ -324,14 +339,14 @@ __global__ void __launch_bounds__(kThreads, 1)
     int g = 0, gs = 0, gv = 0, gr = 0;
     for (int r = blockIdx.x; r < p.R; r += gridDim.x, ++gr) {
       if (named_bar_or(1, kEpi, *abort != 0)) break;
-      const size_t rbase = (size_t)r * p.cap;
-      float pm[G], pl[G], pH[G], dm[G], dl[G], dH[G];
+      const size_t rbase = (size_t)r * p.stride;
+      float pm[G], pnl[G], pH[G], dm[G], dnl[G], dH[G];
 #pragma unroll
       for (int h = 0; h < G; ++h) {
-        const float* rp = p.ring_stats + (((size_t)r * p.w + st.slot_prev) * G + h) * 4;
-        const float* rd = p.ring_stats + (((size_t)r * p.w + st.slot) * G + h) * 4;
-        pm[h] = rp[0]; pl[h] = rp[1]; pH[h] = rp[2];
-        dm[h] = rd[0]; dl[h] = rd[1]; dH[h] = rd[2];
+        const float4 rp = reinterpret_cast<const float4*>(p.ring_stats)[((size_t)r * p.w + st.slot_prev) * G + h];
+        const float4 rd = reinterpret_cast<const float4*>(p.ring_stats)[((size_t)r * p.w + st.slot) * G + h];
+        pm[h] = rp.x; pnl[h] = rp.w; pH[h] = rp.z;
+        dm[h] = rd.x; dnl[h] = rd.w; dH[h] = rd.z;
       }
       float m[G], l[G], u[G];
 #pragma unroll
@@ -346,6 +361,9 @@ __global__ void __launch_bounds__(kThreads, 1)
         float S16[16];
         tmem_ld16(lane_addr + kColS + b * 16, S16);
         tmem_ld_wait();
+        const uint8_t* stg = smem + OFF_STAGE + s * kStageBytes;
+        const int pos = reinterpret_cast<const int*>(stg + kOffPos)[tok];
+        float4 sz = reinterpret_cast<const float4*>(stg + kOffSZ)[tok];
         tc_fence_before();
         __syncwarp();
         if (lane == 0) {
@@ -357,12 +375,11 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
           for (int h = 0; h < G; ++h) online_add(m[h], l[h], u[h], S16[h], c);
           if (st.has_prev || st.has_dep) {
-            const int pos = p.pos[rbase + i];
             float zp = 0.f, sp = 0.f, zd = 0.f, sd = 0.f;
-            if (st.has_prev && pos <= st.p_prev) window_terms<G>(S16 + G, pm, pl, pH, c, zp, sp);
-            if (st.has_dep && pos <= st.p_dep) window_terms<G>(S16 + 2 * G, dm, dl, dH, c, zd, sd);
-            p.Z[rbase + i] = (p.Z[rbase + i] + (double)zp) - (double)zd;
-            p.S[rbase + i] = (p.S[rbase + i] + (double)sp) - (double)sd;
+            if (st.has_prev && pos <= st.p_prev) window_terms<G>(S16 + G, pm, pnl, pH, c, zp, sp);
+            if (st.has_dep && pos <= st.p_dep) window_terms<G>(S16 + 2 * G, dm, dnl, dH, c, zd, sd);
+            sz = window_update(sz, sp, sd, zp, zd);
+            p.SZ[rbase + i] = sz;
           }
         }
         __syncwarp();
@@ -387,7 +404,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
       }
       sync();
-      float M[G], L[G], Hh[G];
+      float M[G], L[G], NL[G], Hh[G];
 #pragma unroll
       for (int h = 0; h < G; ++h) {
         float mm = -INFINITY, ll = 0.f, uu = 0.f;
@@ -395,13 +412,14 @@ __global__ void __launch_bounds__(kThreads, 1)
           online_merge(mm, ll, uu, red[(w * G + h) * 3 + 0], red[(w * G + h) * 3 + 1], red[(w * G + h) * 3 + 2], c);
         M[h] = mm;
         L[h] = ll;
+        NL[h] = -log2f(ll);
         Hh[h] = logf(ll) - 0.69314718055994531f * (uu / ll);
       }
       sync();  // red is rewritten by the next row
       // push (q, m, l, H) of this step into the ring slot it takes over
       if (etid < G) {
         float* rs = p.ring_stats + (((size_t)r * p.w + st.slot) * G + etid) * 4;
-        rs[0] = M[etid]; rs[1] = L[etid]; rs[2] = Hh[etid]; rs[3] = 0.f;
+        rs[0] = M[etid]; rs[1] = L[etid]; rs[2] = Hh[etid]; rs[3] = NL[etid];
         p.hq[(size_t)r * G + etid] = Hh[etid];
       }
       {
@@ -413,22 +431,32 @@ __global__ void __launch_bounds__(kThreads, 1)
 
       // ---------------- V pass (prep of tile j+1 overlaps the MMAs of tile j)
       const float pos_den = (float)max(st.p_newest, 1);
+      const float4* szrow = p.SZ + rbase + tok;
+      float4 szA = szrow[0];
+      float4 szB = nT > 1 ? szrow[kTok] : make_float4(0.f, 0.f, 0.f, 0.f);
       auto prep = [&](int j) {
         const int gj = g + j, gvj = gv + j;
         const int s = gj % kStages, pb = gvj & 1;
+        // window sums of tile j (loaded two tiles ahead)
+        const float4 sz = szA;
+        szA = szB;
+        if (j + 2 < nT) szB = szrow[(j + 2) * kTok];
         mbar_wait(&bar[B_FULL + s], (gj / kStages) & 1, abort);
         mbar_wait(&bar[B_PEMPTY + pb], ((gvj >> 1) & 1) ^ 1, abort);
         const int i = j * kTok + tok;
         const bool valid = i < n;
+        const uint8_t* stg = smem + OFF_STAGE + s * kStageBytes;
+        const int pos = reinterpret_cast<const int*>(stg + kOffPos)[tok];
+        const float vn = reinterpret_cast<const float*>(stg + kOffVn)[tok];
         float sv[G];
         __syncwarp();
         tmem_ld_g<G>(lane_addr + kColStash + j * G, sv);
         tmem_ld_wait();
         float a[G], mean = 0.f, zc, scur;
-        window_terms<G>(sv, M, L, Hh, c, zc, scur);
+        window_terms<G>(sv, M, NL, Hh, c, zc, scur);
 #pragma unroll
         for (int h = 0; h < G; ++h) {
-          a[h] = attn_weight(sv[h], M[h], c, L[h]);
+          a[h] = attn_weight(sv[h], M[h], c, NL[h]);
           mean += a[h];
         }
         mean /= (float)G;
@@ -436,30 +464,11 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
         for (int h = 0; h < G; ++h) var = fmaf(a[h] - mean, a[h] - mean, var);
         var /= (float)G;
-        // |v_i| from the swizzled V tile
-        const uint8_t* vt = smem + OFF_STAGE + s * kStageBytes;
-        float vn = 0.f;
-#pragma unroll
-        for (int blk = 0; blk < D / 64; ++blk)
-#pragma unroll
-          for (int cch = 0; cch < 8; ++cch) {
-            const uint4 u4 = *reinterpret_cast<const uint4*>(vt + blk * 16384 + sw128(tok, cch));
-            const uint32_t w4[4] = {u4.x, u4.y, u4.z, u4.w};
-#pragma unroll
-            for (int e = 0; e < 4; ++e) {
-              const float x0 = bf16lo(w4[e]), x1 = bf16hi(w4[e]);
-              vn = fmaf(x0, x0, vn);
-              vn = fmaf(x1, x1, vn);
-            }
-          }
-        vn = sqrtf(vn);
-        float x[5] = {mean, vn, var, 0.f, 0.f};
+        const float Zt = __fadd_rn(__fadd_rn(sz.z, zc), sz.w);
+        const float St = __fadd_rn(__fadd_rn(sz.x, scur), sz.y);
+        float x[5] = {mean, vn, var, Zt > 0.f ? St / Zt : 0.f, (float)pos / pos_den};
         if (valid) {
           const size_t slot = rbase + i;
-          const double Zt = p.Z[slot] + (double)zc;
-          const double St = p.S[slot] + (double)scur;
-          x[3] = Zt > 0.0 ? (float)(St / Zt) : 0.f;
-          x[4] = (float)p.pos[slot] / pos_den;
           if (p.alpha_mode == 1) {
             x[0] = p.acc[slot] + mean;
             p.acc[slot] = x[0];
@@ -504,13 +513,19 @@ __global__ void __launch_bounds__(kThreads, 1)
         *reinterpret_cast<uint4*>(at + sw128(tok, 1)) = make_uint4(lo[0], lo[1], lo[2], lo[3]);
         *reinterpret_cast<uint4*>(at + sw128(tok, 2)) = make_uint4(hi[0], hi[1], hi[2], hi[3]);
         *reinterpret_cast<uint4*>(at + sw128(tok, 3)) = make_uint4(0, 0, 0, 0);
-        // attention weights as the PV operand: row h, column = token
+        // attention weights as the PV operand (row = query head, column =
+        // token): bf16 high parts in rows [0, G), the residuals in [G, 2G),
+        // so that O = D[:, h] + D[:, G + h] carries ~16 mantissa bits
         uint8_t* pt = smem + OFF_P + pb * 4096 + (tok >> 6) * 2048;
         const int tc = tok & 63;
 #pragma unroll
-        for (int h = 0; h < G; ++h)
-          *reinterpret_cast<__nv_bfloat16*>(pt + sw128(h, tc >> 3) + (tc & 7) * 2) =
-              __float2bfloat16_rn(valid ? a[h] : 0.f);
+        for (int h = 0; h < G; ++h) {
+          const float ah = valid ? a[h] : 0.f;
+          const __nv_bfloat16 hi = __float2bfloat16_rn(ah);
+          *reinterpret_cast<__nv_bfloat16*>(pt + sw128(h, tc >> 3) + (tc & 7) * 2) = hi;
+          *reinterpret_cast<__nv_bfloat16*>(pt + sw128(G + h, tc >> 3) + (tc & 7) * 2) =
+              __float2bfloat16_rn(ah - __bfloat162float(hi));
+        }
         fence_proxy_async();
         __syncwarp();
         if (lane == 0) {
@@ -529,10 +544,20 @@ __global__ void __launch_bounds__(kThreads, 1)
           float z[32];
           tmem_ld32(lane_addr + kColM + c4 * 32, z);
           tmem_ld_wait();
+          // columns [0, npos) take max(z, 0), the rest min(z, 0); only the
+          // chunk holding npos mixes the two
+          if (c4 * 32 + 32 <= fp.npos) {
 #pragma unroll
-          for (int e = 0; e < 32; ++e) {
-            if (c4 * 32 + e < fp.npos) accp += fmaxf(z[e], 0.f);
-            else accn += fminf(z[e], 0.f);
+            for (int e = 0; e < 32; ++e) accp += fmaxf(z[e], 0.f);
+          } else if (c4 * 32 >= fp.npos) {
+#pragma unroll
+            for (int e = 0; e < 32; ++e) accn += fminf(z[e], 0.f);
+          } else {
+#pragma unroll
+            for (int e = 0; e < 32; ++e) {
+              if (c4 * 32 + e < fp.npos) accp += fmaxf(z[e], 0.f);
+              else accn += fminf(z[e], 0.f);
+            }
           }
         }
         tc_fence_before();
@@ -556,8 +581,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_wait(&bar[B_OFULL], gr & 1, abort);
       __syncwarp();
       tc_fence_after();
-      float o4[4];
-      tmem_ld4(lane_addr + kColO, o4);
+      float o16[16];
+      tmem_ld16(lane_addr + kColO, o16);
       tmem_ld_wait();
       tc_fence_before();
       __syncwarp();
@@ -565,7 +590,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (tok < D) {
         float* op = fs.out + ((r / p.kvh) * p.qh + (r % p.kvh) * G) * D;
 #pragma unroll
-        for (int h = 0; h < G; ++h) op[h * D + tok] = o4[h];
+        for (int h = 0; h < G; ++h) op[h * D + tok] = o16[h] + o16[G + h];
       }
       // ---------------- argtop_B and prune
       if (fs.do_evict && fs.B < n) {
@@ -644,7 +669,7 @@ cudaError_t make_fused_maps(const Dev& p, FusedMaps* maps, const char** why) {
     }
     encode = reinterpret_cast<EncodeTiledFn>(fn);
   }
-  const cuuint64_t dims[2] = {(cuuint64_t)p.d, (cuuint64_t)p.R * (cuuint64_t)p.cap};
+  const cuuint64_t dims[2] = {(cuuint64_t)p.d, (cuuint64_t)p.R * (cuuint64_t)p.stride};
   const cuuint64_t strides[1] = {(cuuint64_t)p.d * 2};
   const cuuint32_t box[2] = {64, 128};
   const cuuint32_t estr[2] = {1, 1};

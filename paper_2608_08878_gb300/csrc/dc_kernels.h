@@ -20,6 +20,10 @@ void launch_split_out(const Dev& p, const Step& st, float* out, cudaStream_t s);
 
 void launch_evict(const Dev& p, int n, int B, cudaStream_t s);
 
+// Window sums S (which 0) or Z (which 1) of rows [row0, row0 + nrows) as fp64
+// [nrows][cap].
+void launch_convert_sz(const Dev& p, int row0, int nrows, int which, double* dst, cudaStream_t s);
+
 bool launch_full_decode(const Dev& p, int n, int nsplit, int chunk, const void* q, float* out,
                         cudaStream_t s);
 

@@ -107,8 +107,8 @@ __device__ __forceinline__ void move_slot(const Dev& p, size_t src, size_t dst, 
   }
   if (l == 0) {
     p.pos[dst] = p.pos[src];
-    p.S[dst] = p.S[src];
-    p.Z[dst] = p.Z[src];
+    p.vnorm[dst] = p.vnorm[src];
+    p.SZ[dst] = p.SZ[src];
     p.score[dst] = p.score[src];
     if (p.acc) p.acc[dst] = p.acc[src];
     if (p.keep_features)
@@ -122,7 +122,7 @@ __device__ __forceinline__ void move_slot(const Dev& p, size_t src, size_t dst, 
 template <int NT, class Sync>
 __device__ void team_select_compact(const Dev& p, int r, int n, int B, const float* score, int tid,
                                     const SelectScratch& s, Sync sync) {
-  const size_t base = (size_t)r * p.cap;
+  const size_t base = (size_t)r * p.stride;
   const int* ps = p.pos + base;
   auto key = [&](int i) { return score_key(score[i]); };
   if (n == B + 1) {

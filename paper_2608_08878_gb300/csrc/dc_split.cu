@@ -1,5 +1,5 @@
 // dc_split.cu -- the split engine: the decode step as separate kernels
-// (append; attention logits + departing-query terms; softmax statistics;
+// (append; attention logits + window-sum update; softmax statistics;
 // attention output + features + policy scores; output combine). Each row's
 // tokens are cut into `nsplit` chunks that run as separate CTAs; logits go
 // through a global scratch buffer between the passes.
@@ -15,20 +15,30 @@ constexpr int kTile = 128;  // tokens per tile = threads per CTA
 
 // ---------------------------------------------------------------------------
 // Append T tokens to every row: slot n0 + t gets k/v[r][t], position
-// seen0 + t, zeroed window sums and cumulative alpha.
+// seen0 + t, |v|_2, zeroed window sums and cumulative alpha.
 // grid (T, R), block d/8 threads (one 16-byte vector each of K and V).
 // ---------------------------------------------------------------------------
 __global__ void append_kernel(Dev p, const uint4* __restrict__ k, const uint4* __restrict__ v,
                               int T, int n0, int seen0) {
   const int t = blockIdx.x, r = blockIdx.y, vpr = p.d / 8;
   const size_t src = ((size_t)r * T + t) * vpr + threadIdx.x;
-  const size_t slot = (size_t)r * p.cap + n0 + t;
-  reinterpret_cast<uint4*>(p.K)[slot * vpr + threadIdx.x] = k[src];
-  reinterpret_cast<uint4*>(p.V)[slot * vpr + threadIdx.x] = v[src];
+  const size_t slot = (size_t)r * p.stride + n0 + t;
+  const uint4 kv = k[src], vv = v[src];
+  reinterpret_cast<uint4*>(p.K)[slot * vpr + threadIdx.x] = kv;
+  reinterpret_cast<uint4*>(p.V)[slot * vpr + threadIdx.x] = vv;
+  const uint32_t w4[4] = {vv.x, vv.y, vv.z, vv.w};
+  float ss = 0.f;
+#pragma unroll
+  for (int e = 0; e < 4; ++e) {
+    const float x0 = bf16lo(w4[e]), x1 = bf16hi(w4[e]);
+    ss = fmaf(x0, x0, ss);
+    ss = fmaf(x1, x1, ss);
+  }
+  for (int off = 1; off < vpr; off <<= 1) ss += __shfl_xor_sync((1u << vpr) - 1u, ss, off);
   if (threadIdx.x == 0) {
     p.pos[slot] = seen0 + t;
-    p.S[slot] = 0.0;
-    p.Z[slot] = 0.0;
+    p.vnorm[slot] = sqrtf(ss);
+    p.SZ[slot] = make_float4(0.f, 0.f, 0.f, 0.f);
     if (p.acc) p.acc[slot] = 0.f;
   }
 }
@@ -112,7 +122,7 @@ __global__ void __launch_bounds__(kTile) split_qk_kernel(Dev p, Step st,
                                                          const __nv_bfloat16* __restrict__ q) {
   __shared__ float qs[3 * G][D];  // current, previous, departing
   __shared__ __align__(16) __nv_bfloat16 kt[kTile][D + 8];
-  __shared__ float ring_ml[2][G][3];  // (m, l, H) of previous / departing
+  __shared__ float ring_ml[2][G][3];  // (m, nl, H) of previous / departing
   __shared__ float red[kTile / kWarp][G][3];
   const int r = blockIdx.y, sp = blockIdx.x, tid = threadIdx.x;
   const int c0 = sp * st.chunk, c1 = min(st.n, c0 + st.chunk);
@@ -129,7 +139,7 @@ __global__ void __launch_bounds__(kTile) split_qk_kernel(Dev p, Step st,
     const int slot = which == 0 ? st.slot_prev : st.slot;
     const float* rs = p.ring_stats + (((size_t)r * p.w + slot) * G + h) * 4;
     ring_ml[which][h][0] = rs[0];
-    ring_ml[which][h][1] = rs[1];
+    ring_ml[which][h][1] = rs[3];
     ring_ml[which][h][2] = rs[2];
   }
   float m[G], l[G], u[G];
@@ -139,10 +149,10 @@ __global__ void __launch_bounds__(kTile) split_qk_kernel(Dev p, Step st,
   for (int base = c0; base < c1; base += kTile) {
     const int rows = min(kTile, c1 - base);
     __syncthreads();
-    load_tile<D>(kt, p.K + ((size_t)r * p.cap + base) * D, rows);
+    load_tile<D>(kt, p.K + ((size_t)r * p.stride + base) * D, rows);
     __syncthreads();
     if (tid < rows) {
-      const size_t slot = (size_t)r * p.cap + base + tid;
+      const size_t slot = (size_t)r * p.stride + base + tid;
       float s[3 * G];
       dots<D, 3 * G>(&kt[tid][0], qs, s);
       float* lo = p.logit + slot * G;
@@ -154,19 +164,18 @@ __global__ void __launch_bounds__(kTile) split_qk_kernel(Dev p, Step st,
       if (st.has_prev || st.has_dep) {
         const int pos = p.pos[slot];
         float zp = 0.f, sp_ = 0.f, zd = 0.f, sd = 0.f;
-        float rm[G], rl[G], rH[G];
+        float rm[G], rnl[G], rH[G];
         if (st.has_prev && pos <= st.p_prev) {
 #pragma unroll
-          for (int h = 0; h < G; ++h) { rm[h] = ring_ml[0][h][0]; rl[h] = ring_ml[0][h][1]; rH[h] = ring_ml[0][h][2]; }
-          window_terms<G>(s + G, rm, rl, rH, c, zp, sp_);
+          for (int h = 0; h < G; ++h) { rm[h] = ring_ml[0][h][0]; rnl[h] = ring_ml[0][h][1]; rH[h] = ring_ml[0][h][2]; }
+          window_terms<G>(s + G, rm, rnl, rH, c, zp, sp_);
         }
         if (st.has_dep && pos <= st.p_dep) {
 #pragma unroll
-          for (int h = 0; h < G; ++h) { rm[h] = ring_ml[1][h][0]; rl[h] = ring_ml[1][h][1]; rH[h] = ring_ml[1][h][2]; }
-          window_terms<G>(s + 2 * G, rm, rl, rH, c, zd, sd);
+          for (int h = 0; h < G; ++h) { rm[h] = ring_ml[1][h][0]; rnl[h] = ring_ml[1][h][1]; rH[h] = ring_ml[1][h][2]; }
+          window_terms<G>(s + 2 * G, rm, rnl, rH, c, zd, sd);
         }
-        p.Z[slot] = (p.Z[slot] + (double)zp) - (double)zd;
-        p.S[slot] = (p.S[slot] + (double)sp_) - (double)sd;
+        p.SZ[slot] = window_update(p.SZ[slot], sp_, sd, zp, zd);
       }
     }
   }
@@ -214,7 +223,7 @@ __global__ void split_stats_kernel(Dev p, Step st, const __nv_bfloat16* __restri
     }
     float H = logf(L) - 0.69314718055994531f * (U / L);
     float* rs = p.ring_stats + (((size_t)r * p.w + st.slot) * G + h) * 4;
-    rs[0] = M; rs[1] = L; rs[2] = H; rs[3] = 0.f;
+    rs[0] = M; rs[1] = L; rs[2] = H; rs[3] = -log2f(L);
     p.hq[(size_t)r * G + h] = H;
   }
 }
@@ -229,14 +238,14 @@ __global__ void __launch_bounds__(kTile) split_v_kernel(Dev p, Step st) {
   extern __shared__ float wsm[];
   __shared__ __align__(16) __nv_bfloat16 vt[kTile][D + 8];
   __shared__ float at[kTile][G];
-  __shared__ float stat[G][3];
+  __shared__ float stat[G][3];  // (m, nl, H)
   const int r = blockIdx.y, sp = blockIdx.x, tid = threadIdx.x;
   const int c0 = sp * st.chunk, c1 = min(st.n, c0 + st.chunk);
   const int H = p.hidden, nblob = 9 * H + 1;
   for (int e = tid; e < nblob; e += blockDim.x) wsm[e] = p.policy[e];
   if (tid < G) {
     const float* rs = p.ring_stats + (((size_t)r * p.w + st.slot) * G + tid) * 4;
-    stat[tid][0] = rs[0]; stat[tid][1] = rs[1]; stat[tid][2] = rs[2];
+    stat[tid][0] = rs[0]; stat[tid][1] = rs[3]; stat[tid][2] = rs[2];
   }
   constexpr int NOUT = G * D;
   constexpr int OPT = NOUT >= kTile ? NOUT / kTile : 1;  // outputs per thread
@@ -251,21 +260,21 @@ __global__ void __launch_bounds__(kTile) split_v_kernel(Dev p, Step st) {
   for (int base = c0; base < c1; base += kTile) {
     const int rows = min(kTile, c1 - base);
     __syncthreads();
-    load_tile<D>(vt, p.V + ((size_t)r * p.cap + base) * D, rows);
+    load_tile<D>(vt, p.V + ((size_t)r * p.stride + base) * D, rows);
     __syncthreads();
     if (tid < rows) {
-      const size_t slot = (size_t)r * p.cap + base + tid;
+      const size_t slot = (size_t)r * p.stride + base + tid;
       const float* lo = p.logit + slot * G;
       float a[G], mean = 0.f;
       float zc = 0.f, sc = 0.f;
       {
-        float s[G], mm[G], ll[G], hh[G];
+        float s[G], mm[G], nl[G], hh[G];
 #pragma unroll
-        for (int h = 0; h < G; ++h) { s[h] = lo[h]; mm[h] = stat[h][0]; ll[h] = stat[h][1]; hh[h] = stat[h][2]; }
-        window_terms<G>(s, mm, ll, hh, c, zc, sc);
+        for (int h = 0; h < G; ++h) { s[h] = lo[h]; mm[h] = stat[h][0]; nl[h] = stat[h][1]; hh[h] = stat[h][2]; }
+        window_terms<G>(s, mm, nl, hh, c, zc, sc);
 #pragma unroll
         for (int h = 0; h < G; ++h) {
-          a[h] = attn_weight(s[h], mm[h], c, ll[h]);
+          a[h] = attn_weight(s[h], mm[h], c, nl[h]);
           at[tid][h] = a[h];
           mean += a[h];
         }
@@ -275,28 +284,17 @@ __global__ void __launch_bounds__(kTile) split_v_kernel(Dev p, Step st) {
 #pragma unroll
       for (int h = 0; h < G; ++h) var = fmaf(a[h] - mean, a[h] - mean, var);
       var /= (float)G;
-      float vn = 0.f;
-#pragma unroll 4
-      for (int c8 = 0; c8 < D / 8; ++c8) {
-        uint4 u4 = *reinterpret_cast<const uint4*>(&vt[tid][c8 * 8]);
-        uint32_t w4[4] = {u4.x, u4.y, u4.z, u4.w};
-#pragma unroll
-        for (int e = 0; e < 4; ++e) {
-          float x0 = bf16lo(w4[e]), x1 = bf16hi(w4[e]);
-          vn = fmaf(x0, x0, vn);
-          vn = fmaf(x1, x1, vn);
-        }
-      }
-      vn = sqrtf(vn);
+      const float vn = p.vnorm[slot];
       // H_i over the whole window: stored sums (earlier queries) + this step
-      const double Z = p.Z[slot] + (double)zc;
-      const double S = p.S[slot] + (double)sc;
+      const float4 sz = p.SZ[slot];
+      const float Zt = __fadd_rn(__fadd_rn(sz.z, zc), sz.w);
+      const float St = __fadd_rn(__fadd_rn(sz.x, sc), sz.y);
       float alpha = mean;
       if (p.alpha_mode == 1) {
         alpha = p.acc[slot] + mean;
         p.acc[slot] = alpha;
       }
-      float Hi = Z > 0.0 ? (float)(S / Z) : 0.f;
+      float Hi = Zt > 0.f ? St / Zt : 0.f;
       float x[5] = {alpha, vn, var, Hi, (float)p.pos[slot] / pos_den};
       if (p.keep_features) {
 #pragma unroll
@@ -341,6 +339,24 @@ __global__ void split_out_kernel(Dev p, Step st, float* __restrict__ out) {
     for (int sp = 0; sp < st.nsplit; ++sp) s += p.opart[(((size_t)r * p.smax + sp) * G) * D + e];
     out[row_q_offset(p, r) + e] = s;
   }
+}
+
+// ---------------------------------------------------------------------------
+// Window sums as fp64 [nrows][cap] (hi + lo of the stored double-float pairs)
+// for inspection. grid-stride over the elements.
+// ---------------------------------------------------------------------------
+__global__ void convert_sz_kernel(Dev p, int row0, int nrows, int which, double* __restrict__ dst) {
+  const long long total = (long long)nrows * p.cap;
+  for (long long e = blockIdx.x * (long long)blockDim.x + threadIdx.x; e < total;
+       e += (long long)gridDim.x * blockDim.x) {
+    const int r = row0 + (int)(e / p.cap), i = (int)(e % p.cap);
+    const float4 v = p.SZ[(size_t)r * p.stride + i];
+    dst[e] = which == 0 ? (double)v.x + (double)v.y : (double)v.z + (double)v.w;
+  }
+}
+
+void launch_convert_sz(const Dev& p, int row0, int nrows, int which, double* dst, cudaStream_t s) {
+  convert_sz_kernel<<<1024, 256, 0, s>>>(p, row0, nrows, which, dst);
 }
 
 // ---------------------------------------------------------------------------

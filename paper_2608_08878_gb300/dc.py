@@ -21,7 +21,7 @@ DC_OK, DC_ERR_INVALID_ARG, DC_ERR_CAPACITY, DC_ERR_OOM, DC_ERR_CUDA, DC_ERR_DEVI
 STATUS_NAMES = ["DC_OK", "DC_ERR_INVALID_ARG", "DC_ERR_CAPACITY", "DC_ERR_OOM", "DC_ERR_CUDA",
                 "DC_ERR_DEVICE", "DC_ERR_STATE"]
 
-BUF_K, BUF_V, BUF_POS, BUF_S, BUF_Z, BUF_ACC, BUF_SCORE, BUF_FEAT, BUF_HQ = range(9)
+BUF_K, BUF_V, BUF_POS, BUF_S, BUF_Z, BUF_ACC, BUF_SCORE, BUF_FEAT, BUF_HQ, BUF_VNORM = range(10)
 
 # Every function the header declares (checked by the tests).
 EXPORTS = ["dc_config_default", "dc_cache_create", "dc_cache_destroy", "dc_policy_blob_len",
@@ -241,7 +241,7 @@ class DistillCache:
                 BUF_POS: (torch.int32, (cap,)), BUF_S: (torch.float64, (cap,)),
                 BUF_Z: (torch.float64, (cap,)), BUF_ACC: (torch.float32, (cap,)),
                 BUF_SCORE: (torch.float32, (cap,)), BUF_FEAT: (torch.float32, (cap, 5)),
-                BUF_HQ: (torch.float32, (G,))}[which]
+                BUF_HQ: (torch.float32, (G,)), BUF_VNORM: (torch.float32, (cap,))}[which]
         if rb.value == 0:
             raise DCError(DC_ERR_INVALID_ARG, "the cache has no such buffer")
         out = torch.empty((nrows,) + spec[1], dtype=spec[0], device="cuda")
