@@ -37,9 +37,18 @@ def measured_peaks():
         return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0}, "fallback"
 
 
+_OVERRIDES = {}
+
+
 def workload():
+    """The benchmark workload (Mistral-7B KV shape, 32 layers, batch 8, 32K
+    context, 25% budget); --layers / --batch shrink it for profiling."""
     from paper_2608_08878_gb300 import synth
-    return synth.MISTRAL_FULL
+    wl = synth.MISTRAL_FULL
+    if _OVERRIDES:
+        wl = wl.with_(**_OVERRIDES)
+        wl = wl.with_(name=f"{wl.name} [reduced: {wl.layers} layers, batch {wl.batch}]")
+    return wl
 
 
 def row_bytes_per_step(n: int, d: int, alpha_mode: int = 0) -> int:
@@ -399,7 +408,13 @@ def main():
     ap.add_argument("--no-cpu", action="store_true")
     ap.add_argument("--no-full", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--layers", type=int, default=None, help="profiling: fewer layers than the workload's 32")
+    ap.add_argument("--batch", type=int, default=None, help="profiling: another batch than the workload's 8")
     args = ap.parse_args()
+    if args.layers:
+        _OVERRIDES["layers"] = args.layers
+    if args.batch:
+        _OVERRIDES["batch"] = args.batch
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")
     if args.impl == "reference":
