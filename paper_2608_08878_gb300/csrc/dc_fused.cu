@@ -5,29 +5,32 @@
 // Sec. 3.1.2 / App. D, and (dc_step) the top-B select and compaction.
 //
 // One CTA per SM; each CTA takes rows r = blockIdx.x, blockIdx.x + gridDim.x...
-// Warp roles (192 threads):
+// Warp roles (320 threads):
 //   warp 0     producer: writes the row's query tile (current, previous and
 //              departing queries) and streams K then V tiles of 128 tokens
-//              with TMA (128-byte swizzle) through a 3-stage ring;
+//              with TMA (128-byte swizzle) through a 3-stage ring, each tile
+//              with its tokens' state (positions, window sums or |v|);
 //   warp 1     MMA issuer (one lane): tcgen05.mma, accumulators in TMEM:
 //                S  = K Q^T        [128 tokens x 16]  per K tile
 //                O^T += V^T P^T    [d x 16]           per V tile (P = weights,
 //                                  bf16 high and low parts in separate columns)
 //                Z  = A W^T        [128 tokens x 128] per V tile (policy layer)
-//   warps 2-5  epilogue, one token (TMEM lane) per thread:
+//   warps 2-9  epilogue: two warpgroups; warpgroup w takes the tiles whose
+//              global index is w mod 2, one token (TMEM lane) per thread:
 //                K pass: online softmax statistics, window-sum update (the
 //                previous step's query in, the departing one out, both
-//                recomputed from the same S tile), raw logits kept in TMEM;
+//                recomputed from the same S tile), raw logits kept for the
+//                V pass (heads 0..G-2 in TMEM, head G-1 in shared memory);
 //                V pass: weights with the final statistics, features, the
 //                policy's input row, score; then the output and the select.
 //
-// TMEM columns: S tiles [0, 32), O [32, 48), policy layer [64, 192), the
-// logit stash [192, 512) (G columns per tile of 128 tokens).
+// TMEM columns: S tiles [0, 32), O [32, 48), policy layer of warpgroup w
+// [128 + 128 w, 256 + 128 w), logit stash [48, 128) and [384, 512).
 //
 // Per-token state rides along with the tiles: TMA bulk copies bring the
 // positions and window sums with each K tile and the positions and |v| with
 // each V tile. The K pass writes the updated window sums back; the V pass
-// re-reads them (L2-resident by then) with loads issued two tiles ahead.
+// re-reads them (L2-resident by then) with loads issued ahead of use.
 #include <cuda.h>
 
 #include "dc_common.cuh"
@@ -50,17 +53,18 @@ constexpr int kOffVn = kTileRegion + 512;     // fp32 [128]
 constexpr int kOffSZ = kTileRegion + 1024;    // fp32x4 [128]
 constexpr int kStageBytes = kTileRegion + 3072;
 constexpr int kTok = 128;
-constexpr int kThreads = 192;
-constexpr int kEpi = 128;
+constexpr int kThreads = 320;
+constexpr int kEpi = 256;                     // two warpgroups
 constexpr uint32_t kTmemCols = 512;
-constexpr int kColS = 0, kColO = 32, kColM = 64, kColStash = 192;
+constexpr int kColS = 0, kColO = 32, kColM = 128;
+constexpr int kStashA = 48, kStashAEnd = 128, kStashB = 384, kStashBEnd = 512;
 
 constexpr int OFF_STAGE = 0;
 constexpr int OFF_Q = OFF_STAGE + kStages * kStageBytes;  // 2 x 4 KB
-constexpr int OFF_P = OFF_Q + 2 * 4096;                    // 2 x 4 KB
-constexpr int OFF_A = OFF_P + 2 * 4096;                    // 2 x 16 KB
+constexpr int OFF_P = OFF_Q + 2 * 4096;                    // 2 x 4 KB (one per warpgroup)
+constexpr int OFF_A = OFF_P + 2 * 4096;                    // 2 x 16 KB (one per warpgroup)
 constexpr int OFF_W = OFF_A + 2 * 16384;                   // 16 KB
-constexpr int OFF_SC = OFF_W + 16384;                      // scores, kFusedMaxTok floats
+constexpr int OFF_SC = OFF_W + 16384;                      // head G-1 logits, then scores
 constexpr int OFF_MISC = OFF_SC + kFusedMaxTok * 4;
 constexpr int MISC_BYTES = 4096;
 constexpr int kSmemBytes = OFF_MISC + MISC_BYTES + 1024;   // + alignment slack
@@ -68,8 +72,15 @@ constexpr int kSmemBytes = OFF_MISC + MISC_BYTES + 1024;   // + alignment slack
 // barrier indices in the misc area
 enum {
   B_FULL = 0, B_EMPTY = 3, B_QFULL = 6, B_QEMPTY = 8, B_SFULL = 10, B_SEMPTY = 12, B_PFULL = 14,
-  B_PEMPTY = 16, B_MFULL = 18, B_MEMPTY = 19, B_OFULL = 20, B_OEMPTY = 21, B_DRAIN = 22, B_COUNT = 24
+  B_PEMPTY = 16, B_MFULL = 18, B_MEMPTY = 20, B_OFULL = 22, B_OEMPTY = 23, B_DRAIN = 24, B_COUNT = 26
 };
+
+// TMEM column of the stashed logits of tile j (GS = G - 1 columns per tile).
+template <int GS>
+__device__ __forceinline__ uint32_t stash_col(int j) {
+  constexpr int TA = GS > 0 ? (kStashAEnd - kStashA) / GS : 0;
+  return j < TA ? (uint32_t)(kStashA + GS * j) : (uint32_t)(kStashB + GS * (j - TA));
+}
 
 // byte offset of 16-byte chunk `c` (0..7) of row `row` inside a 128-byte
 // swizzled tile (8-row atoms of 1024 bytes)
@@ -82,36 +93,31 @@ __device__ __forceinline__ uint32_t pack_bf16(float a, float b) {
   return *reinterpret_cast<uint32_t*>(&v);
 }
 
-template <int G>
-__device__ __forceinline__ void tmem_st_g(uint32_t taddr, const float* v) {
-  if constexpr (G == 4) {
-    asm volatile("tcgen05.st.sync.aligned.32x32b.x4.b32 [%0], {%1,%2,%3,%4};" ::"r"(taddr),
-                 "r"(__float_as_uint(v[0])), "r"(__float_as_uint(v[1])), "r"(__float_as_uint(v[2])),
-                 "r"(__float_as_uint(v[3]))
-                 : "memory");
-  } else if constexpr (G == 2) {
+// Stores / loads the first GS of the G logits of this thread's token.
+template <int GS>
+__device__ __forceinline__ void stash_store(uint32_t taddr, const float* v) {
+  if constexpr (GS == 3) {
     asm volatile("tcgen05.st.sync.aligned.32x32b.x2.b32 [%0], {%1,%2};" ::"r"(taddr), "r"(__float_as_uint(v[0])),
                  "r"(__float_as_uint(v[1]))
                  : "memory");
-  } else {
+    asm volatile("tcgen05.st.sync.aligned.32x32b.x1.b32 [%0], {%1};" ::"r"(taddr + 2), "r"(__float_as_uint(v[2]))
+                 : "memory");
+  } else if constexpr (GS == 1) {
     asm volatile("tcgen05.st.sync.aligned.32x32b.x1.b32 [%0], {%1};" ::"r"(taddr), "r"(__float_as_uint(v[0]))
                  : "memory");
   }
 }
 
-template <int G>
-__device__ __forceinline__ void tmem_ld_g(uint32_t taddr, float* v) {
-  if constexpr (G == 4) {
-    float t[4];
-    tmem_ld4(taddr, t);
-#pragma unroll
-    for (int h = 0; h < 4; ++h) v[h] = t[h];
-  } else if constexpr (G == 2) {
-    uint32_t a, b;
+template <int GS>
+__device__ __forceinline__ void stash_load(uint32_t taddr, float* v) {
+  if constexpr (GS == 3) {
+    uint32_t a, b, c;
     asm volatile("tcgen05.ld.sync.aligned.32x32b.x2.b32 {%0,%1}, [%2];" : "=r"(a), "=r"(b) : "r"(taddr));
+    asm volatile("tcgen05.ld.sync.aligned.32x32b.x1.b32 {%0}, [%1];" : "=r"(c) : "r"(taddr + 2));
     v[0] = __uint_as_float(a);
     v[1] = __uint_as_float(b);
-  } else {
+    v[2] = __uint_as_float(c);
+  } else if constexpr (GS == 1) {
     uint32_t a;
     asm volatile("tcgen05.ld.sync.aligned.32x32b.x1.b32 {%0}, [%1];" : "=r"(a) : "r"(taddr));
     v[0] = __uint_as_float(a);
@@ -150,17 +156,18 @@ template <int D, int G>
 __global__ void __launch_bounds__(kThreads, 1)
     fused_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmV, Dev p,
                  Step st, FusedStep fs, FusedPolicy fp) {
+  constexpr int GS = G - 1;  // heads whose logits wait in TMEM between the passes
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint64_t* bar = reinterpret_cast<uint64_t*>(smem + OFF_MISC);
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + OFF_MISC + 8 * B_COUNT);
   volatile int* abort = reinterpret_cast<volatile int*>(smem + OFF_MISC + 8 * B_COUNT + 4);
-  float* red = reinterpret_cast<float*>(smem + OFF_MISC + 256);            // [4][G][3]
+  float* red = reinterpret_cast<float*>(smem + OFF_MISC + 256);            // [8][G][3]
   int* s_hist = reinterpret_cast<int*>(smem + OFF_MISC + 1024);           // [256]
   int* s_sh = reinterpret_cast<int*>(smem + OFF_MISC + 2048);             // [4]
-  int* s_wsum = reinterpret_cast<int*>(smem + OFF_MISC + 2064);           // [4]
-  unsigned long long* s_best = reinterpret_cast<unsigned long long*>(smem + OFF_MISC + 2112);  // [4]
-  int* s_best_slot = reinterpret_cast<int*>(smem + OFF_MISC + 2176);      // [4]
+  int* s_wsum = reinterpret_cast<int*>(smem + OFF_MISC + 2064);           // [8]
+  unsigned long long* s_best = reinterpret_cast<unsigned long long*>(smem + OFF_MISC + 2112);  // [8]
+  int* s_best_slot = reinterpret_cast<int*>(smem + OFF_MISC + 2176);      // [8]
   float* sc = reinterpret_cast<float*>(smem + OFF_SC);
 
   const int warp = threadIdx.x / kWarp, lane = threadIdx.x % kWarp;
@@ -179,9 +186,9 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_init(&bar[B_SEMPTY + b], 4);
       mbar_init(&bar[B_PFULL + b], 4);
       mbar_init(&bar[B_PEMPTY + b], 1);
+      mbar_init(&bar[B_MFULL + b], 1);
+      mbar_init(&bar[B_MEMPTY + b], 4);
     }
-    mbar_init(&bar[B_MFULL], 1);
-    mbar_init(&bar[B_MEMPTY], 4);
     mbar_init(&bar[B_OFULL], 1);
     mbar_init(&bar[B_OEMPTY], 4);
     mbar_init(&bar[B_DRAIN], 1);
@@ -297,7 +304,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           if (!mbar_wait(&bar[B_FULL + s], (g / kStages) & 1, abort)) break;
           if (!mbar_wait(&bar[B_PFULL + pb], (gv >> 1) & 1, abort)) break;
           if (j == 0 && !mbar_wait(&bar[B_OEMPTY], (gr & 1) ^ 1, abort)) break;
-          if (!mbar_wait(&bar[B_MEMPTY], (gv & 1) ^ 1, abort)) break;
+          if (!mbar_wait(&bar[B_MEMPTY + pb], ((gv >> 1) & 1) ^ 1, abort)) break;
           tc_fence_after();
           const uint32_t vaddr = smem_u32(smem + OFF_STAGE + s * kStageBytes);
           const uint32_t paddr = smem_u32(smem + OFF_P + pb * 4096);
@@ -313,9 +320,9 @@ __global__ void __launch_bounds__(kThreads, 1)
           // policy layer: Z[128 x 128] = A[128 x 32] W^T
 #pragma unroll
           for (int ks = 0; ks < 2; ++ks)
-            mma_bf16(tmem + kColM, sdesc_sw128(aaddr + ks * 32u, 16, 1024), sdesc_sw128(waddr + ks * 32u, 16, 1024),
-                     id_m, ks > 0);
-          mma_commit(&bar[B_MFULL]);
+            mma_bf16(tmem + kColM + pb * 128, sdesc_sw128(aaddr + ks * 32u, 16, 1024),
+                     sdesc_sw128(waddr + ks * 32u, 16, 1024), id_m, ks > 0);
+          mma_commit(&bar[B_MFULL + pb]);
           mma_commit(&bar[B_PEMPTY + pb]);
           mma_commit(&bar[B_EMPTY + s]);
           if (j == nT - 1) mma_commit(&bar[B_OFULL]);
@@ -328,10 +335,11 @@ __global__ void __launch_bounds__(kThreads, 1)
     __syncwarp();
   } else {
     // ------------------------------------------------------------ epilogue
-    const int ew = warp - 2;                    // 0..3
+    const int ew = warp - 2;                    // 0..7
+    const int wg = ew >> 2;                     // warpgroup 0 / 1
     const int quad = warp & 3;                  // TMEM lane quarter of this warp
     const int tok = quad * 32 + lane;           // token (TMEM lane) within a tile
-    const int etid = ew * 32 + lane;            // 0..127
+    const int etid = ew * 32 + lane;            // 0..255
     const uint32_t lane_addr = tmem + ((uint32_t)(quad * 32) << 16);
     const float c = p.c;
     auto sync = [] { named_bar(1, kEpi); };
@@ -352,10 +360,11 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
       for (int h = 0; h < G; ++h) { m[h] = -INFINITY; l[h] = 0.f; u[h] = 0.f; }
 
-      // ---------------- K pass
-      for (int j = 0; j < nT; ++j, ++g, ++gs) {
-        const int s = g % kStages, b = gs & 1;
-        mbar_wait(&bar[B_SFULL + b], (gs >> 1) & 1, abort);
+      // ---------------- K pass: this warpgroup's tiles (global index parity)
+      for (int j = (wg - gs) & 1; j < nT; j += 2) {
+        const int gj = g + j, gsj = gs + j;
+        const int s = gj % kStages, b = gsj & 1;
+        mbar_wait(&bar[B_SFULL + b], (gsj >> 1) & 1, abort);
         __syncwarp();
         tc_fence_after();
         float S16[16];
@@ -382,10 +391,13 @@ __global__ void __launch_bounds__(kThreads, 1)
             p.SZ[rbase + i] = sz;
           }
         }
+        sc[i] = S16[G - 1];
         __syncwarp();
-        tmem_st_g<G>(lane_addr + kColStash + j * G, S16);
+        stash_store<GS>(lane_addr + stash_col<GS>(j), S16);
       }
-      tmem_st_wait();
+      g += nT;
+      gs += nT;
+      if constexpr (GS > 0) tmem_st_wait();
       // ---------------- row softmax statistics (deterministic merge order)
 #pragma unroll
       for (int h = 0; h < G; ++h) {
@@ -404,22 +416,24 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
       }
       sync();
-      float M[G], L[G], NL[G], Hh[G];
+      float M[G], NL[G], Hh[G];
+      float L0 = 0.f;
 #pragma unroll
       for (int h = 0; h < G; ++h) {
         float mm = -INFINITY, ll = 0.f, uu = 0.f;
-        for (int w = 0; w < 4; ++w)
+        for (int w = 0; w < 8; ++w)
           online_merge(mm, ll, uu, red[(w * G + h) * 3 + 0], red[(w * G + h) * 3 + 1], red[(w * G + h) * 3 + 2], c);
         M[h] = mm;
-        L[h] = ll;
         NL[h] = -log2f(ll);
         Hh[h] = logf(ll) - 0.69314718055994531f * (uu / ll);
+        if (etid == h) L0 = ll;
       }
       sync();  // red is rewritten by the next row
-      // push (q, m, l, H) of this step into the ring slot it takes over
+      // push (q, m, l, H, -log2 l) of this step into the ring slot it takes over
       if (etid < G) {
-        float* rs = p.ring_stats + (((size_t)r * p.w + st.slot) * G + etid) * 4;
-        rs[0] = M[etid]; rs[1] = L[etid]; rs[2] = Hh[etid]; rs[3] = NL[etid];
+        float4 v;
+        v.x = M[etid]; v.y = L0; v.z = Hh[etid]; v.w = NL[etid];
+        reinterpret_cast<float4*>(p.ring_stats)[((size_t)r * p.w + st.slot) * G + etid] = v;
         p.hq[(size_t)r * G + etid] = Hh[etid];
       }
       {
@@ -429,18 +443,20 @@ __global__ void __launch_bounds__(kThreads, 1)
         for (int e = etid; e < G * D / 8; e += kEpi) rq[e] = qs[e];
       }
 
-      // ---------------- V pass (prep of tile j+1 overlaps the MMAs of tile j)
+      // ---------------- V pass: this warpgroup's tiles; prep of the next one
+      // overlaps the MMAs of the current one
       const float pos_den = (float)max(st.p_newest, 1);
+      const int j0 = (wg - gv) & 1;
       const float4* szrow = p.SZ + rbase + tok;
-      float4 szA = szrow[0];
-      float4 szB = nT > 1 ? szrow[kTok] : make_float4(0.f, 0.f, 0.f, 0.f);
+      float4 szA = j0 < nT ? szrow[j0 * kTok] : make_float4(0.f, 0.f, 0.f, 0.f);
+      float4 szB = j0 + 2 < nT ? szrow[(j0 + 2) * kTok] : make_float4(0.f, 0.f, 0.f, 0.f);
       auto prep = [&](int j) {
         const int gj = g + j, gvj = gv + j;
         const int s = gj % kStages, pb = gvj & 1;
-        // window sums of tile j (loaded two tiles ahead)
+        // window sums of tile j (loaded two own tiles ahead)
         const float4 sz = szA;
         szA = szB;
-        if (j + 2 < nT) szB = szrow[(j + 2) * kTok];
+        if (j + 4 < nT) szB = szrow[(j + 4) * kTok];
         mbar_wait(&bar[B_FULL + s], (gj / kStages) & 1, abort);
         mbar_wait(&bar[B_PEMPTY + pb], ((gvj >> 1) & 1) ^ 1, abort);
         const int i = j * kTok + tok;
@@ -450,16 +466,17 @@ __global__ void __launch_bounds__(kThreads, 1)
         const float vn = reinterpret_cast<const float*>(stg + kOffVn)[tok];
         float sv[G];
         __syncwarp();
-        tmem_ld_g<G>(lane_addr + kColStash + j * G, sv);
-        tmem_ld_wait();
-        float a[G], mean = 0.f, zc, scur;
-        window_terms<G>(sv, M, NL, Hh, c, zc, scur);
+        stash_load<GS>(lane_addr + stash_col<GS>(j), sv);
+        if constexpr (GS > 0) tmem_ld_wait();
+        sv[G - 1] = sc[i];
+        float a[G], zc = 0.f, scur = 0.f;
 #pragma unroll
         for (int h = 0; h < G; ++h) {
           a[h] = attn_weight(sv[h], M[h], c, NL[h]);
-          mean += a[h];
+          zc += a[h];
+          scur = fmaf(a[h], Hh[h], scur);
         }
-        mean /= (float)G;
+        const float mean = zc / (float)G;
         float var = 0.f;
 #pragma unroll
         for (int h = 0; h < G; ++h) var = fmaf(a[h] - mean, a[h] - mean, var);
@@ -521,10 +538,10 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
         for (int h = 0; h < G; ++h) {
           const float ah = valid ? a[h] : 0.f;
-          const __nv_bfloat16 hi = __float2bfloat16_rn(ah);
-          *reinterpret_cast<__nv_bfloat16*>(pt + sw128(h, tc >> 3) + (tc & 7) * 2) = hi;
+          const __nv_bfloat16 hv = __float2bfloat16_rn(ah);
+          *reinterpret_cast<__nv_bfloat16*>(pt + sw128(h, tc >> 3) + (tc & 7) * 2) = hv;
           *reinterpret_cast<__nv_bfloat16*>(pt + sw128(G + h, tc >> 3) + (tc & 7) * 2) =
-              __float2bfloat16_rn(ah - __bfloat162float(hi));
+              __float2bfloat16_rn(ah - __bfloat162float(hv));
         }
         fence_proxy_async();
         __syncwarp();
@@ -534,15 +551,15 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
       };
       auto finish = [&](int j) {
-        const int gvj = gv + j;
-        mbar_wait(&bar[B_MFULL], gvj & 1, abort);
+        const int gvj = gv + j, pb = gvj & 1;
+        mbar_wait(&bar[B_MFULL + pb], (gvj >> 1) & 1, abort);
         __syncwarp();
         tc_fence_after();
         float accp = 0.f, accn = 0.f;
 #pragma unroll
         for (int c4 = 0; c4 < 4; ++c4) {
           float z[32];
-          tmem_ld32(lane_addr + kColM + c4 * 32, z);
+          tmem_ld32(lane_addr + kColM + pb * 128 + c4 * 32, z);
           tmem_ld_wait();
           // columns [0, npos) take max(z, 0), the rest min(z, 0); only the
           // chunk holding npos mixes the two
@@ -562,7 +579,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         tc_fence_before();
         __syncwarp();
-        if (lane == 0) mbar_arrive(&bar[B_MEMPTY]);
+        if (lane == 0) mbar_arrive(&bar[B_MEMPTY + pb]);
         const int i = j * kTok + tok;
         if (i < n) {
           const float score = fp.b2 + (accp + accn);
@@ -570,27 +587,29 @@ __global__ void __launch_bounds__(kThreads, 1)
           if (fs.write_scores) p.score[rbase + i] = score;
         }
       };
-      prep(0);
-      for (int j = 0; j < nT; ++j) {
-        if (j + 1 < nT) prep(j + 1);
+      if (j0 < nT) prep(j0);
+      for (int j = j0; j < nT; j += 2) {
+        if (j + 2 < nT) prep(j + 2);
         finish(j);
       }
       g += nT;
       gv += nT;
-      // ---------------- attention output
-      mbar_wait(&bar[B_OFULL], gr & 1, abort);
-      __syncwarp();
-      tc_fence_after();
-      float o16[16];
-      tmem_ld16(lane_addr + kColO, o16);
-      tmem_ld_wait();
-      tc_fence_before();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(&bar[B_OEMPTY]);
-      if (tok < D) {
-        float* op = fs.out + ((r / p.kvh) * p.qh + (r % p.kvh) * G) * D;
+      // ---------------- attention output (warpgroup 0)
+      if (wg == 0) {
+        mbar_wait(&bar[B_OFULL], gr & 1, abort);
+        __syncwarp();
+        tc_fence_after();
+        float o16[16];
+        tmem_ld16(lane_addr + kColO, o16);
+        tmem_ld_wait();
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&bar[B_OEMPTY]);
+        if (tok < D) {
+          float* op = fs.out + ((r / p.kvh) * p.qh + (r % p.kvh) * G) * D;
 #pragma unroll
-        for (int h = 0; h < G; ++h) op[h * D + tok] = o16[h] + o16[G + h];
+          for (int h = 0; h < G; ++h) op[h * D + tok] = o16[h] + o16[G + h];
+        }
       }
       // ---------------- argtop_B and prune
       if (fs.do_evict && fs.B < n) {
@@ -609,9 +628,16 @@ __global__ void __launch_bounds__(kThreads, 1)
 
 }  // namespace
 
+int fused_max_tokens(int G) {
+  if (G <= 1) return kFusedMaxTok;
+  const int GS = G - 1;
+  const int tiles = (kStashAEnd - kStashA) / GS + (kStashBEnd - kStashB) / GS;
+  return tiles * kTok < kFusedMaxTok ? tiles * kTok : kFusedMaxTok;
+}
+
 bool fused_eligible(const Dev& p, int n) {
   return (p.d == 64 || p.d == 128) && (p.G == 1 || p.G == 2 || p.G == 4) && p.hidden <= 128 && n >= 1 &&
-         n <= kFusedMaxTok;
+         n <= fused_max_tokens(p.G);
 }
 
 int fused_smem_bytes() { return kSmemBytes; }

@@ -40,6 +40,8 @@ struct FusedPolicy {
   const __nv_bfloat16* wtile;    // device [128][32]: rows w_j as bf16 hi | hi | lo | 0
 };
 
+// Most tokens per row the fused kernel takes for a query group of G heads.
+int fused_max_tokens(int G);
 bool fused_eligible(const Dev& p, int n);
 int fused_smem_bytes();
 
