@@ -72,7 +72,8 @@ constexpr int kSmemBytes = OFF_MISC + MISC_BYTES + 1024;   // + alignment slack
 // barrier indices in the misc area
 enum {
   B_FULL = 0, B_EMPTY = 3, B_QFULL = 6, B_QEMPTY = 8, B_SFULL = 10, B_SEMPTY = 12, B_PFULL = 14,
-  B_PEMPTY = 16, B_MFULL = 18, B_MEMPTY = 20, B_OFULL = 22, B_OEMPTY = 23, B_DRAIN = 24, B_COUNT = 26
+  B_PEMPTY = 16, B_MFULL = 18, B_MEMPTY = 20, B_AFULL = 22, B_AEMPTY = 24, B_OFULL = 26, B_OEMPTY = 27,
+  B_DRAIN = 28, B_COUNT = 30
 };
 
 // TMEM column of the stashed logits of tile j (GS = G - 1 columns per tile).
@@ -188,6 +189,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_init(&bar[B_PEMPTY + b], 1);
       mbar_init(&bar[B_MFULL + b], 1);
       mbar_init(&bar[B_MEMPTY + b], 4);
+      mbar_init(&bar[B_AFULL + b], 4);
+      mbar_init(&bar[B_AEMPTY + b], 1);
     }
     mbar_init(&bar[B_OFULL], 1);
     mbar_init(&bar[B_OEMPTY], 4);
@@ -299,34 +302,60 @@ __global__ void __launch_bounds__(kThreads, 1)
           mma_commit(&bar[B_EMPTY + s]);
         }
         mma_commit(&bar[B_QEMPTY + qb]);
-        for (int j = 0; j < nT; ++j, ++g, ++gv) {
-          const int s = g % kStages, pb = gv & 1;
-          if (!mbar_wait(&bar[B_FULL + s], (g / kStages) & 1, abort)) break;
-          if (!mbar_wait(&bar[B_PFULL + pb], (gv >> 1) & 1, abort)) break;
-          if (j == 0 && !mbar_wait(&bar[B_OEMPTY], (gr & 1) ^ 1, abort)) break;
-          if (!mbar_wait(&bar[B_MEMPTY + pb], ((gv >> 1) & 1) ^ 1, abort)) break;
-          tc_fence_after();
-          const uint32_t vaddr = smem_u32(smem + OFF_STAGE + s * kStageBytes);
-          const uint32_t paddr = smem_u32(smem + OFF_P + pb * 4096);
-          const uint32_t aaddr = smem_u32(smem + OFF_A + pb * 16384);
-          const uint32_t waddr = smem_u32(smem + OFF_W);
-          // O^T[d x 16] += V^T[d x 128] P^T: V^T is MN-major (dims contiguous)
+        // V pass: the PV MMAs (tile order) and the policy-layer MMAs (tile
+        // order, after their tile's PV) are issued as their operands become
+        // ready, so a V stage is released as soon as its weights are in
+        const uint32_t waddr = smem_u32(smem + OFF_W);
+        int jp = 0, jm = 0, idle = 0;
+        uint64_t t0 = globaltimer_ns();
+        while ((jp < nT || jm < nT) && !*abort) {
+          bool did = false;
+          if (jp < nT) {
+            const int gj = g + jp, gvj = gv + jp, s = gj % kStages, pb = gvj & 1;
+            if (mbar_test(&bar[B_FULL + s], (gj / kStages) & 1) && mbar_test(&bar[B_PFULL + pb], (gvj >> 1) & 1) &&
+                (jp > 0 || mbar_test(&bar[B_OEMPTY], (gr & 1) ^ 1))) {
+              tc_fence_after();
+              const uint32_t vaddr = smem_u32(smem + OFF_STAGE + s * kStageBytes);
+              const uint32_t paddr = smem_u32(smem + OFF_P + pb * 4096);
+              // O^T[d x 16] += V^T[d x 128] P^T: V^T is MN-major (dims contiguous)
 #pragma unroll
-          for (int ks = 0; ks < kTok / 16; ++ks) {
-            const uint32_t poff = (uint32_t)(ks >> 2) * 2048u + (uint32_t)(ks & 3) * 32u;
-            mma_bf16(tmem + kColO, sdesc_sw128(vaddr + ks * 2048u, 16384, 1024),
-                     sdesc_sw128(paddr + poff, 16, 1024), id_pv, (j > 0 || ks > 0) ? 1u : 0u);
+              for (int ks = 0; ks < kTok / 16; ++ks) {
+                const uint32_t poff = (uint32_t)(ks >> 2) * 2048u + (uint32_t)(ks & 3) * 32u;
+                mma_bf16(tmem + kColO, sdesc_sw128(vaddr + ks * 2048u, 16384, 1024),
+                         sdesc_sw128(paddr + poff, 16, 1024), id_pv, (jp > 0 || ks > 0) ? 1u : 0u);
+              }
+              mma_commit(&bar[B_PEMPTY + pb]);
+              mma_commit(&bar[B_EMPTY + s]);
+              if (jp == nT - 1) mma_commit(&bar[B_OFULL]);
+              ++jp;
+              did = true;
+            }
           }
-          // policy layer: Z[128 x 128] = A[128 x 32] W^T
+          if (jm < jp) {
+            const int gvj = gv + jm, pb = gvj & 1;
+            if (mbar_test(&bar[B_AFULL + pb], (gvj >> 1) & 1) && mbar_test(&bar[B_MEMPTY + pb], ((gvj >> 1) & 1) ^ 1)) {
+              tc_fence_after();
+              const uint32_t aaddr = smem_u32(smem + OFF_A + pb * 16384);
+              // policy layer: Z[128 x 128] = A[128 x 32] W^T
 #pragma unroll
-          for (int ks = 0; ks < 2; ++ks)
-            mma_bf16(tmem + kColM + pb * 128, sdesc_sw128(aaddr + ks * 32u, 16, 1024),
-                     sdesc_sw128(waddr + ks * 32u, 16, 1024), id_m, ks > 0);
-          mma_commit(&bar[B_MFULL + pb]);
-          mma_commit(&bar[B_PEMPTY + pb]);
-          mma_commit(&bar[B_EMPTY + s]);
-          if (j == nT - 1) mma_commit(&bar[B_OFULL]);
+              for (int ks = 0; ks < 2; ++ks)
+                mma_bf16(tmem + kColM + pb * 128, sdesc_sw128(aaddr + ks * 32u, 16, 1024),
+                         sdesc_sw128(waddr + ks * 32u, 16, 1024), id_m, ks > 0);
+              mma_commit(&bar[B_MFULL + pb]);
+              mma_commit(&bar[B_AEMPTY + pb]);
+              ++jm;
+              did = true;
+            }
+          }
+          if (did) {
+            idle = 0;
+            t0 = globaltimer_ns();
+          } else if ((++idle & 255) == 0 && globaltimer_ns() - t0 > kWaitNs) {
+            *abort = 1;
+          }
         }
+        g += nT;
+        gv += nT;
       }
       // all issued MMAs complete before TMEM is released
       mma_commit(&bar[B_DRAIN]);
@@ -458,14 +487,15 @@ __global__ void __launch_bounds__(kThreads, 1)
         szA = szB;
         if (j + 4 < nT) szB = szrow[(j + 4) * kTok];
         mbar_wait(&bar[B_FULL + s], (gj / kStages) & 1, abort);
-        mbar_wait(&bar[B_PEMPTY + pb], ((gvj >> 1) & 1) ^ 1, abort);
         const int i = j * kTok + tok;
         const bool valid = i < n;
         const uint8_t* stg = smem + OFF_STAGE + s * kStageBytes;
         const int pos = reinterpret_cast<const int*>(stg + kOffPos)[tok];
         const float vn = reinterpret_cast<const float*>(stg + kOffVn)[tok];
-        float sv[G];
         __syncwarp();
+        if (lane == 0) mbar_arrive(&bar[B_EMPTY + s]);  // stage: only the PV MMA still reads it
+        __syncwarp();
+        float sv[G];
         stash_load<GS>(lane_addr + stash_col<GS>(j), sv);
         if constexpr (GS > 0) tmem_ld_wait();
         sv[G - 1] = sc[i];
@@ -475,6 +505,25 @@ __global__ void __launch_bounds__(kThreads, 1)
           a[h] = attn_weight(sv[h], M[h], c, NL[h]);
           zc += a[h];
           scur = fmaf(a[h], Hh[h], scur);
+        }
+        // attention weights as the PV operand (row = query head, column =
+        // token): bf16 high parts in rows [0, G), the residuals in [G, 2G),
+        // so that O = D[:, h] + D[:, G + h] carries ~16 mantissa bits
+        mbar_wait(&bar[B_PEMPTY + pb], ((gvj >> 1) & 1) ^ 1, abort);
+        {
+          uint8_t* pt = smem + OFF_P + pb * 4096 + (tok >> 6) * 2048;
+          const int tc = tok & 63;
+#pragma unroll
+          for (int h = 0; h < G; ++h) {
+            const float ah = valid ? a[h] : 0.f;
+            const __nv_bfloat16 hv = __float2bfloat16_rn(ah);
+            *reinterpret_cast<__nv_bfloat16*>(pt + sw128(h, tc >> 3) + (tc & 7) * 2) = hv;
+            *reinterpret_cast<__nv_bfloat16*>(pt + sw128(G + h, tc >> 3) + (tc & 7) * 2) =
+                __float2bfloat16_rn(ah - __bfloat162float(hv));
+          }
+          fence_proxy_async();
+          __syncwarp();
+          if (lane == 0) mbar_arrive(&bar[B_PFULL + pb]);
         }
         const float mean = zc / (float)G;
         float var = 0.f;
@@ -525,30 +574,15 @@ __global__ void __launch_bounds__(kThreads, 1)
           hi[e] = (uint32_t)__bfloat16_as_ushort(h0) | ((uint32_t)__bfloat16_as_ushort(h1) << 16);
           lo[e] = pack_bf16(r0, r1);
         }
+        mbar_wait(&bar[B_AEMPTY + pb], ((gvj >> 1) & 1) ^ 1, abort);
         uint8_t* at = smem + OFF_A + pb * 16384;
         *reinterpret_cast<uint4*>(at + sw128(tok, 0)) = make_uint4(hi[0], hi[1], hi[2], hi[3]);
         *reinterpret_cast<uint4*>(at + sw128(tok, 1)) = make_uint4(lo[0], lo[1], lo[2], lo[3]);
         *reinterpret_cast<uint4*>(at + sw128(tok, 2)) = make_uint4(hi[0], hi[1], hi[2], hi[3]);
         *reinterpret_cast<uint4*>(at + sw128(tok, 3)) = make_uint4(0, 0, 0, 0);
-        // attention weights as the PV operand (row = query head, column =
-        // token): bf16 high parts in rows [0, G), the residuals in [G, 2G),
-        // so that O = D[:, h] + D[:, G + h] carries ~16 mantissa bits
-        uint8_t* pt = smem + OFF_P + pb * 4096 + (tok >> 6) * 2048;
-        const int tc = tok & 63;
-#pragma unroll
-        for (int h = 0; h < G; ++h) {
-          const float ah = valid ? a[h] : 0.f;
-          const __nv_bfloat16 hv = __float2bfloat16_rn(ah);
-          *reinterpret_cast<__nv_bfloat16*>(pt + sw128(h, tc >> 3) + (tc & 7) * 2) = hv;
-          *reinterpret_cast<__nv_bfloat16*>(pt + sw128(G + h, tc >> 3) + (tc & 7) * 2) =
-              __float2bfloat16_rn(ah - __bfloat162float(hv));
-        }
         fence_proxy_async();
         __syncwarp();
-        if (lane == 0) {
-          mbar_arrive(&bar[B_PFULL + pb]);
-          mbar_arrive(&bar[B_EMPTY + s]);
-        }
+        if (lane == 0) mbar_arrive(&bar[B_AFULL + pb]);
       };
       auto finish = [&](int j) {
         const int gvj = gv + j, pb = gvj & 1;
