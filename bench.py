@@ -255,6 +255,7 @@ def run_gpu(args):
         ev1.record(stream)
         torch.cuda.synchronize()
     el_ms = ev0.elapsed_time(ev1)
+    cache.sync()  # device-side status of every timed step (raises on error)
     prof = cache.profile_read()
     cache.profile(False)
     if dist:

@@ -317,6 +317,7 @@ dc_status dc_cache_create(int layers, int kv_heads, int head_dim, int capacity, 
   A(&pol, blob * sizeof(float));
   p.policy = pol;
   A(&p.status, sizeof(unsigned));
+  A(&p.dbg, 8 * sizeof(unsigned));
   A(&p.logit, RC * G * sizeof(float));
   A(&p.part, (size_t)R * p.smax * G * 4 * sizeof(float));
   A(&p.opart, (size_t)R * p.smax * G * head_dim * sizeof(float));
@@ -596,11 +597,13 @@ dc_status dc_copy_buffer(dc_cache* h, dc_buffer which, int row0, int nrows, void
 dc_status dc_sync(dc_cache* h) {
   DC_CHECK_HANDLE(h);
   DC_CUDA(h, cudaStreamSynchronize(h->stream));
-  unsigned st = 0;
+  unsigned st = 0, dbg[8] = {};
   DC_CUDA(h, cudaMemcpy(&st, h->dev.status, sizeof st, cudaMemcpyDeviceToHost));
+  DC_CUDA(h, cudaMemcpy(dbg, h->dev.dbg, sizeof dbg, cudaMemcpyDeviceToHost));
   if (st) {
-    char buf[96];
-    std::snprintf(buf, sizeof buf, "kernel status word 0x%x", st);
+    char buf[160];
+    std::snprintf(buf, sizeof buf, "kernel status word 0x%x (first wait timeout: site %u block %u parity %u info 0x%x)",
+                  st, dbg[1], dbg[2], dbg[3], dbg[4]);
     return fail(h, DC_ERR_DEVICE, buf);
   }
   return DC_OK;

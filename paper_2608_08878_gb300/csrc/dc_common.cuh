@@ -49,6 +49,7 @@ struct Dev {
   float* ring_stats;
   const float* policy;
   unsigned* status;
+  unsigned* dbg;  // [8]: first wait timeout of a launch (site, block, parity, info)
   // scratch of the split engine
   float* logit;   // [R][stride][G]
   float* part;    // [R][smax][G][4]: per-split (m, l, u2, 0)

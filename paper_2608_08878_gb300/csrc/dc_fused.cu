@@ -228,7 +228,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     for (int r = blockIdx.x; r < p.R; r += gridDim.x, ++gr) {
       if (*abort) break;
       const int qb = gr & 1;
-      if (!mbar_wait(&bar[B_QEMPTY + qb], ((gr >> 1) & 1) ^ 1, abort)) break;
+      if (!mbar_wait(&bar[B_QEMPTY + qb], ((gr >> 1) & 1) ^ 1, abort, p.dbg, 1u, (unsigned)gr)) break;
       // query tile: rows [0,G) current, [G,2G) previous step, [2G,3G) departing
       uint8_t* qt = smem + OFF_Q + qb * 4096;
       const int qo = ((r / p.kvh) * p.qh + (r % p.kvh) * G) * D;
@@ -251,7 +251,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           const CUtensorMap* tm = pass ? &tmV : &tmK;
           for (int j = 0; j < nT; ++j, ++g) {
             const int s = g % kStages;
-            if (!mbar_wait(&bar[B_EMPTY + s], ((g / kStages) & 1) ^ 1, abort)) break;
+            if (!mbar_wait(&bar[B_EMPTY + s], ((g / kStages) & 1) ^ 1, abort, p.dbg, 2u, (unsigned)g)) break;
             mbar_expect_tx(&bar[B_FULL + s], kTileBytes + (pass ? 1024u : 2560u));
             uint8_t* dst = smem + OFF_STAGE + s * kStageBytes;
             const int y = r * p.stride + j * kTok;
@@ -282,13 +282,13 @@ __global__ void __launch_bounds__(kThreads, 1)
       for (int r = blockIdx.x; r < p.R; r += gridDim.x, ++gr) {
         if (*abort) break;
         const int qb = gr & 1;
-        if (!mbar_wait(&bar[B_QFULL + qb], (gr >> 1) & 1, abort)) break;
+        if (!mbar_wait(&bar[B_QFULL + qb], (gr >> 1) & 1, abort, p.dbg, 3u, (unsigned)gr)) break;
         tc_fence_after();
         const uint32_t qaddr = smem_u32(smem + OFF_Q + qb * 4096);
         for (int j = 0; j < nT; ++j, ++g, ++gs) {
           const int s = g % kStages, b = gs & 1;
-          if (!mbar_wait(&bar[B_FULL + s], (g / kStages) & 1, abort)) break;
-          if (!mbar_wait(&bar[B_SEMPTY + b], ((gs >> 1) & 1) ^ 1, abort)) break;
+          if (!mbar_wait(&bar[B_FULL + s], (g / kStages) & 1, abort, p.dbg, 4u, (unsigned)g)) break;
+          if (!mbar_wait(&bar[B_SEMPTY + b], ((gs >> 1) & 1) ^ 1, abort, p.dbg, 5u, (unsigned)gs)) break;
           tc_fence_after();
           const uint32_t kaddr = smem_u32(smem + OFF_STAGE + s * kStageBytes);
 #pragma unroll
@@ -351,6 +351,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             idle = 0;
             t0 = globaltimer_ns();
           } else if ((++idle & 255) == 0 && globaltimer_ns() - t0 > kWaitNs) {
+            record_timeout(p.dbg, 20u + (jp < nT ? 0u : 1u), (unsigned)(jp | (jm << 16)), (unsigned)(gv | (nT << 24)));
             *abort = 1;
           }
         }
@@ -393,7 +394,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       for (int j = (wg - gs) & 1; j < nT; j += 2) {
         const int gj = g + j, gsj = gs + j;
         const int s = gj % kStages, b = gsj & 1;
-        mbar_wait(&bar[B_SFULL + b], (gsj >> 1) & 1, abort);
+        mbar_wait(&bar[B_SFULL + b], (gsj >> 1) & 1, abort, p.dbg, 6u, (unsigned)gsj);
+        mbar_wait(&bar[B_FULL + s], (gj / kStages) & 1, abort, p.dbg, 12u, (unsigned)gj);
         __syncwarp();
         tc_fence_after();
         float S16[16];
@@ -486,7 +488,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         const float4 sz = szA;
         szA = szB;
         if (j + 4 < nT) szB = szrow[(j + 4) * kTok];
-        mbar_wait(&bar[B_FULL + s], (gj / kStages) & 1, abort);
+        mbar_wait(&bar[B_FULL + s], (gj / kStages) & 1, abort, p.dbg, 7u, (unsigned)gj);
         const int i = j * kTok + tok;
         const bool valid = i < n;
         const uint8_t* stg = smem + OFF_STAGE + s * kStageBytes;
@@ -509,7 +511,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         // attention weights as the PV operand (row = query head, column =
         // token): bf16 high parts in rows [0, G), the residuals in [G, 2G),
         // so that O = D[:, h] + D[:, G + h] carries ~16 mantissa bits
-        mbar_wait(&bar[B_PEMPTY + pb], ((gvj >> 1) & 1) ^ 1, abort);
+        mbar_wait(&bar[B_PEMPTY + pb], ((gvj >> 1) & 1) ^ 1, abort, p.dbg, 8u, (unsigned)gvj);
         {
           uint8_t* pt = smem + OFF_P + pb * 4096 + (tok >> 6) * 2048;
           const int tc = tok & 63;
@@ -574,7 +576,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           hi[e] = (uint32_t)__bfloat16_as_ushort(h0) | ((uint32_t)__bfloat16_as_ushort(h1) << 16);
           lo[e] = pack_bf16(r0, r1);
         }
-        mbar_wait(&bar[B_AEMPTY + pb], ((gvj >> 1) & 1) ^ 1, abort);
+        mbar_wait(&bar[B_AEMPTY + pb], ((gvj >> 1) & 1) ^ 1, abort, p.dbg, 9u, (unsigned)gvj);
         uint8_t* at = smem + OFF_A + pb * 16384;
         *reinterpret_cast<uint4*>(at + sw128(tok, 0)) = make_uint4(hi[0], hi[1], hi[2], hi[3]);
         *reinterpret_cast<uint4*>(at + sw128(tok, 1)) = make_uint4(lo[0], lo[1], lo[2], lo[3]);
@@ -586,7 +588,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       };
       auto finish = [&](int j) {
         const int gvj = gv + j, pb = gvj & 1;
-        mbar_wait(&bar[B_MFULL + pb], (gvj >> 1) & 1, abort);
+        mbar_wait(&bar[B_MFULL + pb], (gvj >> 1) & 1, abort, p.dbg, 10u, (unsigned)gvj);
         __syncwarp();
         tc_fence_after();
         float accp = 0.f, accn = 0.f;
@@ -630,7 +632,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       gv += nT;
       // ---------------- attention output (warpgroup 0)
       if (wg == 0) {
-        mbar_wait(&bar[B_OFULL], gr & 1, abort);
+        mbar_wait(&bar[B_OFULL], gr & 1, abort, p.dbg, 11u, (unsigned)gr);
         __syncwarp();
         tc_fence_after();
         float o16[16];

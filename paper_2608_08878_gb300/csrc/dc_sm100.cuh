@@ -68,10 +68,22 @@ __device__ __forceinline__ bool mbar_test(uint64_t* bar, uint32_t parity) {
   return ok != 0;
 }
 
+// Where a wait gave up: the first timeout in a launch records its site, block
+// and the waited parity in dbg[1..4] (dbg[0] is the claim flag).
+__device__ __forceinline__ void record_timeout(unsigned* dbg, unsigned site, unsigned a, unsigned b) {
+  if (dbg && atomicCAS(dbg, 0u, 1u) == 0u) {
+    dbg[1] = site;
+    dbg[2] = blockIdx.x;
+    dbg[3] = a;
+    dbg[4] = b;
+  }
+}
+
 // Waits for the phase of `parity` to complete. Gives up (returns false) when
 // *abort is set by another role, or when the time limit passes, in which case
-// it sets *abort itself so that every role winds down.
-__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, volatile int* abort) {
+// it records the site and sets *abort itself so that every role winds down.
+__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, volatile int* abort,
+                                          unsigned* dbg = nullptr, unsigned site = 0, unsigned info = 0) {
   if (mbar_try_wait(bar, parity)) return true;
   const uint64_t t0 = globaltimer_ns();
   for (uint32_t i = 1; i < kSpinLimit; ++i) {
@@ -79,6 +91,7 @@ __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, volati
     if (*abort) return false;
     if ((i & 255u) == 0 && globaltimer_ns() - t0 > kWaitNs) break;
   }
+  record_timeout(dbg, site, parity, info);
   *abort = 1;
   return false;
 }

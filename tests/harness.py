@@ -100,6 +100,7 @@ class LockStep:
         s = self.step_idx
         q, kn, vn = self._inputs(s)
         out = self.cache.decode_step(q, kn, vn)
+        self.cache.sync()  # raises on any device-side status (e.g. a wait that gave up)
         n, _ = self.cache.length()
         out_h = out.cpu().numpy()
         G = wl.group
@@ -140,6 +141,7 @@ class LockStep:
             order = np.argsort(pos, kind="stable")
             gpu_scores[r] = sc[order]
         self.cache.evict(budget)
+        self.cache.sync()
         B = budget if budget > 0 else self.wl.budget
         n2, _ = self.cache.length()
         assert n2 == min(n, B)
