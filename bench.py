@@ -47,7 +47,8 @@ def workload():
     wl = synth.MISTRAL_FULL
     if _OVERRIDES:
         wl = wl.with_(**_OVERRIDES)
-        wl = wl.with_(name=f"{wl.name} [reduced: {wl.layers} layers, batch {wl.batch}]")
+        wl = wl.with_(name=f"{wl.name} [profiling case: {wl.layers} layers, batch {wl.batch}, "
+                           f"context {wl.prompt_len}, budget {wl.budget}]")
     return wl
 
 
@@ -411,11 +412,17 @@ def main():
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--layers", type=int, default=None, help="profiling: fewer layers than the workload's 32")
     ap.add_argument("--batch", type=int, default=None, help="profiling: another batch than the workload's 8")
+    ap.add_argument("--context", type=int, default=None, help="profiling: another prompt length than 32768")
+    ap.add_argument("--budget", type=int, default=None, help="profiling: another budget than 8192")
     args = ap.parse_args()
     if args.layers:
         _OVERRIDES["layers"] = args.layers
     if args.batch:
         _OVERRIDES["batch"] = args.batch
+    if args.context:
+        _OVERRIDES["prompt_len"] = args.context
+    if args.budget:
+        _OVERRIDES["budget"] = args.budget
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")
     if args.impl == "reference":
