@@ -5,7 +5,7 @@
 // Sec. 3.1.2 / App. D, and (dc_step) the top-B select and compaction.
 //
 // One CTA per SM; each CTA takes rows r = blockIdx.x, blockIdx.x + gridDim.x...
-// Warp roles (320 threads):
+// Warp roles (352 threads):
 //   warp 0     producer: writes the row's query tile (current, previous and
 //              departing queries) and streams K then V tiles of 128 tokens
 //              with TMA (128-byte swizzle) through a 3-stage ring, each tile
@@ -14,7 +14,8 @@
 //                S  = K Q^T        [128 tokens x 16]  per K tile
 //                O^T += V^T P^T    [d x 16]           per V tile (P = weights,
 //                                  bf16 high and low parts in separate columns)
-//                Z  = A W^T        [128 tokens x 128] per V tile (policy layer)
+//   warp 10    policy-layer MMA issuer (one lane):
+//                Z  = A W^T        [128 tokens x 128] per V tile
 //   warps 2-9  epilogue: two warpgroups; warpgroup w takes the tiles whose
 //              global index is w mod 2, one token (TMEM lane) per thread:
 //                K pass: online softmax statistics, window-sum update (the
@@ -53,7 +54,7 @@ constexpr int kOffVn = kTileRegion + 512;     // fp32 [128]
 constexpr int kOffSZ = kTileRegion + 1024;    // fp32x4 [128]
 constexpr int kStageBytes = kTileRegion + 3072;
 constexpr int kTok = 128;
-constexpr int kThreads = 320;
+constexpr int kThreads = 352;
 constexpr int kEpi = 256;                     // two warpgroups
 constexpr uint32_t kTmemCols = 512;
 constexpr int kColS = 0, kColO = 32, kColM = 128;
@@ -73,7 +74,7 @@ constexpr int kSmemBytes = OFF_MISC + MISC_BYTES + 1024;   // + alignment slack
 enum {
   B_FULL = 0, B_EMPTY = 3, B_QFULL = 6, B_QEMPTY = 8, B_SFULL = 10, B_SEMPTY = 12, B_PFULL = 14,
   B_PEMPTY = 16, B_MFULL = 18, B_MEMPTY = 20, B_AFULL = 22, B_AEMPTY = 24, B_OFULL = 26, B_OEMPTY = 27,
-  B_DRAIN = 28, B_COUNT = 30
+  B_DRAIN = 28, B_DRAIN2 = 29, B_COUNT = 30
 };
 
 // TMEM column of the stashed logits of tile j (GS = G - 1 columns per tile).
@@ -195,6 +196,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     mbar_init(&bar[B_OFULL], 1);
     mbar_init(&bar[B_OEMPTY], 4);
     mbar_init(&bar[B_DRAIN], 1);
+    mbar_init(&bar[B_DRAIN2], 1);
     *abort = 0;
     fence_mbar_init();
   }
@@ -277,7 +279,6 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (lane == 0) {
       const uint32_t id_qk = idesc_bf16(128, 16, 0, 0);
       const uint32_t id_pv = idesc_bf16(128, 16, 1, 0);
-      const uint32_t id_m = idesc_bf16(128, 128, 0, 0);
       int g = 0, gs = 0, gv = 0, gr = 0;
       for (int r = blockIdx.x; r < p.R; r += gridDim.x, ++gr) {
         if (*abort) break;
@@ -302,65 +303,58 @@ __global__ void __launch_bounds__(kThreads, 1)
           mma_commit(&bar[B_EMPTY + s]);
         }
         mma_commit(&bar[B_QEMPTY + qb]);
-        // V pass: the PV MMAs (tile order) and the policy-layer MMAs (tile
-        // order, after their tile's PV) are issued as their operands become
-        // ready, so a V stage is released as soon as its weights are in
-        const uint32_t waddr = smem_u32(smem + OFF_W);
-        int jp = 0, jm = 0, idle = 0;
-        uint64_t t0 = globaltimer_ns();
-        while ((jp < nT || jm < nT) && !*abort) {
-          bool did = false;
-          if (jp < nT) {
-            const int gj = g + jp, gvj = gv + jp, s = gj % kStages, pb = gvj & 1;
-            if (mbar_test(&bar[B_FULL + s], (gj / kStages) & 1) && mbar_test(&bar[B_PFULL + pb], (gvj >> 1) & 1) &&
-                (jp > 0 || mbar_test(&bar[B_OEMPTY], (gr & 1) ^ 1))) {
-              tc_fence_after();
-              const uint32_t vaddr = smem_u32(smem + OFF_STAGE + s * kStageBytes);
-              const uint32_t paddr = smem_u32(smem + OFF_P + pb * 4096);
-              // O^T[d x 16] += V^T[d x 128] P^T: V^T is MN-major (dims contiguous)
+        // V pass: PV MMAs in tile order; a V stage is released as soon as its
+        // tile's weights are in (the policy-layer MMAs run on warp 10)
+        for (int j = 0; j < nT; ++j, ++g, ++gv) {
+          const int s = g % kStages, pb = gv & 1;
+          if (!mbar_wait(&bar[B_FULL + s], (g / kStages) & 1, abort, p.dbg, 13u, (unsigned)g)) break;
+          if (!mbar_wait(&bar[B_PFULL + pb], (gv >> 1) & 1, abort, p.dbg, 14u, (unsigned)gv)) break;
+          if (j == 0 && !mbar_wait(&bar[B_OEMPTY], (gr & 1) ^ 1, abort, p.dbg, 15u, (unsigned)gr)) break;
+          tc_fence_after();
+          const uint32_t vaddr = smem_u32(smem + OFF_STAGE + s * kStageBytes);
+          const uint32_t paddr = smem_u32(smem + OFF_P + pb * 4096);
+          // O^T[d x 16] += V^T[d x 128] P^T: V^T is MN-major (dims contiguous)
 #pragma unroll
-              for (int ks = 0; ks < kTok / 16; ++ks) {
-                const uint32_t poff = (uint32_t)(ks >> 2) * 2048u + (uint32_t)(ks & 3) * 32u;
-                mma_bf16(tmem + kColO, sdesc_sw128(vaddr + ks * 2048u, 16384, 1024),
-                         sdesc_sw128(paddr + poff, 16, 1024), id_pv, (jp > 0 || ks > 0) ? 1u : 0u);
-              }
-              mma_commit(&bar[B_PEMPTY + pb]);
-              mma_commit(&bar[B_EMPTY + s]);
-              if (jp == nT - 1) mma_commit(&bar[B_OFULL]);
-              ++jp;
-              did = true;
-            }
+          for (int ks = 0; ks < kTok / 16; ++ks) {
+            const uint32_t poff = (uint32_t)(ks >> 2) * 2048u + (uint32_t)(ks & 3) * 32u;
+            mma_bf16(tmem + kColO, sdesc_sw128(vaddr + ks * 2048u, 16384, 1024),
+                     sdesc_sw128(paddr + poff, 16, 1024), id_pv, (j > 0 || ks > 0) ? 1u : 0u);
           }
-          if (jm < jp) {
-            const int gvj = gv + jm, pb = gvj & 1;
-            if (mbar_test(&bar[B_AFULL + pb], (gvj >> 1) & 1) && mbar_test(&bar[B_MEMPTY + pb], ((gvj >> 1) & 1) ^ 1)) {
-              tc_fence_after();
-              const uint32_t aaddr = smem_u32(smem + OFF_A + pb * 16384);
-              // policy layer: Z[128 x 128] = A[128 x 32] W^T
-#pragma unroll
-              for (int ks = 0; ks < 2; ++ks)
-                mma_bf16(tmem + kColM + pb * 128, sdesc_sw128(aaddr + ks * 32u, 16, 1024),
-                         sdesc_sw128(waddr + ks * 32u, 16, 1024), id_m, ks > 0);
-              mma_commit(&bar[B_MFULL + pb]);
-              mma_commit(&bar[B_AEMPTY + pb]);
-              ++jm;
-              did = true;
-            }
-          }
-          if (did) {
-            idle = 0;
-            t0 = globaltimer_ns();
-          } else if ((++idle & 255) == 0 && globaltimer_ns() - t0 > kWaitNs) {
-            record_timeout(p.dbg, 20u + (jp < nT ? 0u : 1u), (unsigned)(jp | (jm << 16)), (unsigned)(gv | (nT << 24)));
-            *abort = 1;
-          }
+          mma_commit(&bar[B_PEMPTY + pb]);
+          mma_commit(&bar[B_EMPTY + s]);
+          if (j == nT - 1) mma_commit(&bar[B_OFULL]);
         }
-        g += nT;
-        gv += nT;
       }
       // all issued MMAs complete before TMEM is released
       mma_commit(&bar[B_DRAIN]);
       mbar_wait_drain(&bar[B_DRAIN], 0);
+    }
+    __syncwarp();
+  } else if (warp == 10) {
+    // ------------------------------------------------------------ policy-layer MMA issuer
+    if (lane == 0) {
+      const uint32_t id_m = idesc_bf16(128, 128, 0, 0);
+      const uint32_t waddr = smem_u32(smem + OFF_W);
+      int gv = 0;
+      for (int r = blockIdx.x; r < p.R; r += gridDim.x) {
+        if (*abort) break;
+        for (int j = 0; j < nT; ++j, ++gv) {
+          const int pb = gv & 1;
+          if (!mbar_wait(&bar[B_AFULL + pb], (gv >> 1) & 1, abort, p.dbg, 16u, (unsigned)gv)) break;
+          if (!mbar_wait(&bar[B_MEMPTY + pb], ((gv >> 1) & 1) ^ 1, abort, p.dbg, 17u, (unsigned)gv)) break;
+          tc_fence_after();
+          const uint32_t aaddr = smem_u32(smem + OFF_A + pb * 16384);
+          // Z[128 x 128] = A[128 x 32] W^T
+#pragma unroll
+          for (int ks = 0; ks < 2; ++ks)
+            mma_bf16(tmem + kColM + pb * 128, sdesc_sw128(aaddr + ks * 32u, 16, 1024),
+                     sdesc_sw128(waddr + ks * 32u, 16, 1024), id_m, ks > 0);
+          mma_commit(&bar[B_MFULL + pb]);
+          mma_commit(&bar[B_AEMPTY + pb]);
+        }
+      }
+      mma_commit(&bar[B_DRAIN2]);
+      mbar_wait_drain(&bar[B_DRAIN2], 0);
     }
     __syncwarp();
   } else {
@@ -593,23 +587,29 @@ __global__ void __launch_bounds__(kThreads, 1)
         tc_fence_after();
         float accp = 0.f, accn = 0.f;
 #pragma unroll
-        for (int c4 = 0; c4 < 4; ++c4) {
-          float z[32];
-          tmem_ld32(lane_addr + kColM + pb * 128 + c4 * 32, z);
+        for (int c8 = 0; c8 < 2; ++c8) {
+          float z2[2][32];
+          tmem_ld32(lane_addr + kColM + pb * 128 + c8 * 64, z2[0]);
+          tmem_ld32(lane_addr + kColM + pb * 128 + c8 * 64 + 32, z2[1]);
           tmem_ld_wait();
-          // columns [0, npos) take max(z, 0), the rest min(z, 0); only the
-          // chunk holding npos mixes the two
-          if (c4 * 32 + 32 <= fp.npos) {
 #pragma unroll
-            for (int e = 0; e < 32; ++e) accp += fmaxf(z[e], 0.f);
-          } else if (c4 * 32 >= fp.npos) {
+          for (int hh = 0; hh < 2; ++hh) {
+            const int c4 = c8 * 2 + hh;
+            const float* z = z2[hh];
+            // columns [0, npos) take max(z, 0), the rest min(z, 0); only the
+            // chunk holding npos mixes the two
+            if (c4 * 32 + 32 <= fp.npos) {
 #pragma unroll
-            for (int e = 0; e < 32; ++e) accn += fminf(z[e], 0.f);
-          } else {
+              for (int e = 0; e < 32; ++e) accp += fmaxf(z[e], 0.f);
+            } else if (c4 * 32 >= fp.npos) {
 #pragma unroll
-            for (int e = 0; e < 32; ++e) {
-              if (c4 * 32 + e < fp.npos) accp += fmaxf(z[e], 0.f);
-              else accn += fminf(z[e], 0.f);
+              for (int e = 0; e < 32; ++e) accn += fminf(z[e], 0.f);
+            } else {
+#pragma unroll
+              for (int e = 0; e < 32; ++e) {
+                if (c4 * 32 + e < fp.npos) accp += fmaxf(z[e], 0.f);
+                else accn += fminf(z[e], 0.f);
+              }
             }
           }
         }
