@@ -236,14 +236,18 @@ __global__ void __launch_bounds__(kThreads, 1)
       const int qo = ((r / p.kvh) * p.qh + (r % p.kvh) * G) * D;
       const __nv_bfloat16* prev = p.ring_q + ((size_t)r * p.w + st.slot_prev) * G * D;
       const __nv_bfloat16* dep = p.ring_q + ((size_t)r * p.w + st.slot) * G * D;
-      for (int e = lane; e < 3 * G * (D / 8); e += kWarp) {
-        const int qi = e / (D / 8), kc = e % (D / 8);
-        const int which = qi / G, h = qi % G;
-        uint4 v = make_uint4(0, 0, 0, 0);
-        if (which == 0) v = reinterpret_cast<const uint4*>(fs.q + qo + h * D)[kc];
-        else if (which == 1 && st.has_prev) v = reinterpret_cast<const uint4*>(prev + h * D)[kc];
-        else if (which == 2 && st.has_dep) v = reinterpret_cast<const uint4*>(dep + h * D)[kc];
-        *reinterpret_cast<uint4*>(qt + (kc >> 3) * 2048 + sw128(qi, kc & 7)) = v;
+      // The current query also takes over the departing query's ring slot:
+      // each lane reads the departing element before it writes the same one.
+      __nv_bfloat16* ring_slot = p.ring_q + ((size_t)r * p.w + st.slot) * G * D;
+      for (int e = lane; e < G * (D / 8); e += kWarp) {
+        const int h = e / (D / 8), kc = e % (D / 8);
+        const uint4 cur = reinterpret_cast<const uint4*>(fs.q + qo + h * D)[kc];
+        const uint4 pv = st.has_prev ? reinterpret_cast<const uint4*>(prev + h * D)[kc] : make_uint4(0, 0, 0, 0);
+        const uint4 dv = st.has_dep ? reinterpret_cast<const uint4*>(dep + h * D)[kc] : make_uint4(0, 0, 0, 0);
+        *reinterpret_cast<uint4*>(qt + (kc >> 3) * 2048 + sw128(h, kc & 7)) = cur;
+        *reinterpret_cast<uint4*>(qt + (kc >> 3) * 2048 + sw128(G + h, kc & 7)) = pv;
+        *reinterpret_cast<uint4*>(qt + (kc >> 3) * 2048 + sw128(2 * G + h, kc & 7)) = dv;
+        reinterpret_cast<uint4*>(ring_slot + h * D)[kc] = cur;
       }
       fence_proxy_async();
       __syncwarp();
@@ -454,18 +458,13 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (etid == h) L0 = ll;
       }
       sync();  // red is rewritten by the next row
-      // push (q, m, l, H, -log2 l) of this step into the ring slot it takes over
+      // push (m, l, H, -log2 l) of this step into the ring slot it takes over
+      // (the producer already wrote the query there)
       if (etid < G) {
         float4 v;
         v.x = M[etid]; v.y = L0; v.z = Hh[etid]; v.w = NL[etid];
         reinterpret_cast<float4*>(p.ring_stats)[((size_t)r * p.w + st.slot) * G + etid] = v;
         p.hq[(size_t)r * G + etid] = Hh[etid];
-      }
-      {
-        const int qo = ((r / p.kvh) * p.qh + (r % p.kvh) * G) * D;
-        uint4* rq = reinterpret_cast<uint4*>(p.ring_q + ((size_t)r * p.w + st.slot) * G * D);
-        const uint4* qs = reinterpret_cast<const uint4*>(fs.q + qo);
-        for (int e = etid; e < G * D / 8; e += kEpi) rq[e] = qs[e];
       }
 
       // ---------------- V pass: this warpgroup's tiles; prep of the next one

@@ -5,7 +5,7 @@
 // Ranking: score descending, then position ascending (Sec. 3.1.2: inference
 // keeps the top-B tokens deterministically). Scores become order-preserving
 // 32-bit keys (score_key). One eviction (n == B + 1, the steady state) is an
-// argmin over the 64-bit rank key (score key, ~position). Otherwise four 8-bit
+// argmin over (score key, -position). Otherwise four 8-bit
 // MSB-first histogram passes find the threshold key T with
 // #(key > T) < B <= #(key >= T); when keys equal to T outnumber the places
 // left, a second select over their positions keeps the lowest ones.
@@ -126,26 +126,32 @@ __device__ void team_select_compact(const Dev& p, int r, int n, int B, const flo
   const int* ps = p.pos + base;
   auto key = [&](int i) { return score_key(score[i]); };
   if (n == B + 1) {
-    // One eviction: the lowest-ranked token, rank key = (score key, ~pos).
-    unsigned long long bk = ~0ull;
+    // One eviction: the lowest-ranked token (smallest score key; among equal
+    // keys the highest position). Positions are read only to break ties.
+    uint32_t bk = 0xFFFFFFFFu;
     int bs = -1;
     for (int i = tid; i < n; i += NT) {
-      const unsigned long long k = ((unsigned long long)key(i) << 32) | (uint32_t)(~(uint32_t)ps[i]);
-      if (k < bk) { bk = k; bs = i; }
+      const uint32_t k = key(i);
+      if (k < bk || (k == bk && bs >= 0 && ps[i] > ps[bs])) { bk = k; bs = i; }
     }
+    auto better = [&](uint32_t ka, int sa, uint32_t kb, int sb) {  // (kb, sb) ranks lower?
+      if (sb < 0) return false;
+      if (sa < 0) return true;
+      return kb < ka || (kb == ka && ps[sb] > ps[sa]);
+    };
 #pragma unroll
     for (int off = 16; off > 0; off >>= 1) {
-      const unsigned long long ok = __shfl_xor_sync(0xffffffffu, bk, off);
+      const uint32_t ok = __shfl_xor_sync(0xffffffffu, bk, off);
       const int os = __shfl_xor_sync(0xffffffffu, bs, off);
-      if (ok < bk) { bk = ok; bs = os; }
+      if (better(bk, bs, ok, os)) { bk = ok; bs = os; }
     }
     const int lane = tid % kWarp, wid = tid / kWarp;
     if (lane == 0) { s.best[wid] = bk; s.best_slot[wid] = bs; }
     sync();
-    unsigned long long fk = s.best[0];
+    uint32_t fk = (uint32_t)s.best[0];
     int e = s.best_slot[0];
     for (int w = 1; w < NT / kWarp; ++w)
-      if (s.best[w] < fk) { fk = s.best[w]; e = s.best_slot[w]; }
+      if (better(fk, e, (uint32_t)s.best[w], s.best_slot[w])) { fk = (uint32_t)s.best[w]; e = s.best_slot[w]; }
     // slot B (the last) is the only candidate mover; it fills the hole at e
     if (e >= 0 && e < B && tid < kWarp) move_slot(p, base + B, base + e, tid, kWarp);
     sync();
