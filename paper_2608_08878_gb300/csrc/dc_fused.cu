@@ -584,7 +584,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         mbar_wait(&bar[B_MFULL + pb], (gvj >> 1) & 1, abort, p.dbg, 10u, (unsigned)gvj);
         __syncwarp();
         tc_fence_after();
-        float accp = 0.f, accn = 0.f;
+        // score = b2 + sum_j sgn_j max(z_j, 0); eight independent partial sums
+        float acc[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
 #pragma unroll
         for (int c8 = 0; c8 < 2; ++c8) {
           float z2[2][32];
@@ -592,32 +593,16 @@ __global__ void __launch_bounds__(kThreads, 1)
           tmem_ld32(lane_addr + kColM + pb * 128 + c8 * 64 + 32, z2[1]);
           tmem_ld_wait();
 #pragma unroll
-          for (int hh = 0; hh < 2; ++hh) {
-            const int c4 = c8 * 2 + hh;
-            const float* z = z2[hh];
-            // columns [0, npos) take max(z, 0), the rest min(z, 0); only the
-            // chunk holding npos mixes the two
-            if (c4 * 32 + 32 <= fp.npos) {
-#pragma unroll
-              for (int e = 0; e < 32; ++e) accp += fmaxf(z[e], 0.f);
-            } else if (c4 * 32 >= fp.npos) {
-#pragma unroll
-              for (int e = 0; e < 32; ++e) accn += fminf(z[e], 0.f);
-            } else {
-#pragma unroll
-              for (int e = 0; e < 32; ++e) {
-                if (c4 * 32 + e < fp.npos) accp += fmaxf(z[e], 0.f);
-                else accn += fminf(z[e], 0.f);
-              }
-            }
-          }
+          for (int e = 0; e < 64; ++e)
+            acc[e & 7] = fmaf(fp.sgn[c8 * 64 + e], fmaxf(z2[e >> 5][e & 31], 0.f), acc[e & 7]);
         }
+        const float relu_sum = ((acc[0] + acc[1]) + (acc[2] + acc[3])) + ((acc[4] + acc[5]) + (acc[6] + acc[7]));
         tc_fence_before();
         __syncwarp();
         if (lane == 0) mbar_arrive(&bar[B_MEMPTY + pb]);
         const int i = j * kTok + tok;
         if (i < n) {
-          const float score = fp.b2 + (accp + accn);
+          const float score = fp.b2 + relu_sum;
           sc[i] = score;
           if (fs.write_scores) p.score[rbase + i] = score;
         }
@@ -770,14 +755,16 @@ void prepare_policy(const float* blob, int H, int layernorm, FusedPolicy* fp, st
       cj[5] = (double)b1[j] - mb;
       for (int a = 0; a < 6; ++a)
         for (int b = 0; b < 6; ++b) Mq[a][b] += cj[a] * cj[b] / H;
-      const double s = (double)w2[j] * (double)gamma[j];
+      const double aw = std::fabs((double)w2[j]);
+      const double s = aw * (double)gamma[j];
       for (int k = 0; k < 6; ++k) rows[(size_t)j * 8 + k] = s * cj[k];
-      rows[(size_t)j * 8 + 6] = (double)w2[j] * (double)beta[j];
+      rows[(size_t)j * 8 + 6] = aw * (double)beta[j];
     }
   } else {
     for (int j = 0; j < H; ++j) {
-      for (int k = 0; k < 5; ++k) rows[(size_t)j * 8 + k] = (double)w2[j] * (double)W1[j * 5 + k];
-      rows[(size_t)j * 8 + 5] = (double)w2[j] * (double)b1[j];
+      const double aw = std::fabs((double)w2[j]);
+      for (int k = 0; k < 5; ++k) rows[(size_t)j * 8 + k] = aw * (double)W1[j * 5 + k];
+      rows[(size_t)j * 8 + 5] = aw * (double)b1[j];
     }
   }
   int k = 0;
@@ -785,12 +772,13 @@ void prepare_policy(const float* blob, int H, int layernorm, FusedPolicy* fp, st
     for (int b = a; b < 6; ++b) fp->M[k++] = (float)(a == b ? Mq[a][b] : 2.0 * Mq[a][b]);
   fp->b2 = (float)b2;
   fp->layernorm = layernorm ? 1 : 0;
-  // hidden units with w2 >= 0 first (their term is max(z, 0), the rest min(z, 0))
+  // hidden units with w2 >= 0 first (the order is immaterial to the sum)
   std::vector<int> perm(H);
   std::iota(perm.begin(), perm.end(), 0);
   std::stable_partition(perm.begin(), perm.end(), [&](int j) { return w2[j] >= 0.f; });
   fp->npos = (int)std::count_if(w2, w2 + H, [](float x) { return x >= 0.f; });
   wtile->assign(128 * 32, __float2bfloat16_rn(0.f));
+  for (int jj = 0; jj < 128; ++jj) fp->sgn[jj] = jj < H ? (w2[perm[jj]] >= 0.f ? 1.f : -1.f) : 0.f;
   for (int jj = 0; jj < H; ++jj) {
     const double* rj = &rows[(size_t)perm[jj] * 8];
     for (int e = 0; e < 8; ++e) {

@@ -29,8 +29,9 @@ struct FusedStep {
 };
 
 // The policy MLP folded for the tensor cores (see prepare_policy):
-//   z_j = <a, w_j> with a = [r x, r, 1, 0] (LayerNorm) or [x, 1, 0, 0];
-//   score = b2 + sum_{j < npos} max(z_j, 0) + sum_{j >= npos} min(z_j, 0);
+//   z_j = <a, w_j> with a = [r x, r, 1, 0] (LayerNorm) or [x, 1, 0, 0], where
+//   w_j carries |w2_j| (and the LayerNorm gain and shift);
+//   score = b2 + sum_j sgn_j max(z_j, 0), sgn_j = sign(w2_j);
 //   r = 1 / sqrt(x~^T M x~ + 1e-5), x~ = [x, 1] (LayerNorm variance).
 struct FusedPolicy {
   float M[21];                   // upper triangle, off-diagonal terms doubled
@@ -38,6 +39,7 @@ struct FusedPolicy {
   int npos;
   int layernorm;
   const __nv_bfloat16* wtile;    // device [128][32]: rows w_j as bf16 hi | hi | lo | 0
+  float sgn[128];                // +1 / -1 per hidden unit, 0 for unused columns
 };
 
 // Most tokens per row the fused kernel takes for a query group of G heads.
