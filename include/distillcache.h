@@ -208,6 +208,33 @@ dc_status dc_profile_read(dc_cache* h, double* ms, long long* launches);
  * status the kernels raised (DC_ERR_DEVICE). */
 dc_status dc_sync(dc_cache* h);
 
+/* Full-cache decode attention that allocates no device memory, for callers
+ * that cannot allocate: code running while a stream is being captured into a
+ * CUDA graph, runtimes that reserve all device memory up front, and paths that
+ * cannot afford the implicit synchronisation of cudaMalloc/cudaFree. The
+ * paper has no counterpart; it is the dc_full_decode computation on
+ * caller-provided buffers, with no handle.
+ *   q:   bf16 [rows][group][head_dim]; k, v: bf16 [rows][n][head_dim]
+ *        (16-byte aligned); out: fp32 [rows][group][head_dim]; all device.
+ *   stream: cudaStream_t (NULL: legacy default stream).
+ * The split-K partial results go to a 16 MiB file-scope device array that is
+ * reserved on every GPU that loads this library until the process exits.
+ * DC_ERR_CAPACITY if one split of all rows does not fit it, i.e. if
+ * rows * group * (head_dim + 4) * 4 > 16 MiB; DC_ERR_INVALID_ARG for bad
+ * shapes (head_dim 64 or 128, group 1, 2, 4 or 8, 1 <= rows <= 65535, n >= 1).
+ * The first call on a device looks up the array's device address (once per
+ * device, with that device current); make that first call before any stream
+ * capture. Every call shares the array and overwrites the part it uses, so
+ * nothing carries over between calls, but calls that overlap on the GPU (two
+ * streams, or two host threads) race on it and must be serialised by the
+ * caller. Asynchronous on `stream`; dc_noalloc_last_error() describes a
+ * failure. */
+dc_status dc_attend_noalloc(const void* q, const void* k, const void* v, int rows, int n,
+                            int head_dim, int group, float* out, void* stream);
+
+/* Message of the last failed dc_attend_noalloc call on this host thread. */
+const char* dc_noalloc_last_error(void);
+
 /* Message of the last error on the handle (or of the last failed create when
  * h is NULL). Valid until the next call on the handle. */
 const char* dc_last_error(const dc_cache* h);

@@ -28,7 +28,8 @@ EXPORTS = ["dc_config_default", "dc_cache_create", "dc_cache_destroy", "dc_polic
            "dc_policy_init", "dc_policy_set_weights", "dc_append", "dc_decode_step",
            "dc_decode_step_host", "dc_evict", "dc_full_decode", "dc_get_length", "dc_buffer_bytes",
            "dc_copy_buffer", "dc_sync", "dc_last_error", "dc_phase_name", "dc_profile_enable",
-           "dc_profile_read", "dc_step", "dc_step_host", "dc_engine"]
+           "dc_profile_read", "dc_step", "dc_step_host", "dc_engine", "dc_attend_noalloc",
+           "dc_noalloc_last_error"]
 PHASES = ["append", "attend", "stats", "score", "combine", "evict", "full"]
 
 
@@ -74,6 +75,9 @@ def lib():
             L.dc_step.argtypes = [P, P, P, P, P, I]
             L.dc_step_host.argtypes = [P, P, P, P, P, I]
             L.dc_engine.argtypes = [P, I, C.POINTER(I)]
+            L.dc_attend_noalloc.argtypes = [P, P, P, I, I, I, I, P, P]
+            L.dc_noalloc_last_error.argtypes = []
+            L.dc_noalloc_last_error.restype = C.c_char_p
             L.dc_full_decode.argtypes = [P, P, P]
             L.dc_get_length.argtypes = [P, C.POINTER(I), C.POINTER(C.c_longlong)]
             L.dc_buffer_bytes.argtypes = [P, I, C.POINTER(S)]
@@ -86,7 +90,7 @@ def lib():
             L.dc_profile_enable.argtypes = [P, I]
             L.dc_profile_read.argtypes = [P, P, P]
             for name in EXPORTS:
-                if name not in ("dc_policy_blob_len", "dc_last_error", "dc_phase_name"):
+                if name not in ("dc_policy_blob_len", "dc_last_error", "dc_phase_name", "dc_noalloc_last_error"):
                     getattr(L, name).restype = I
             _lib = L
     return _lib
@@ -103,6 +107,21 @@ def policy_init(seed: int, hidden: int) -> np.ndarray:
     st = lib().dc_policy_init(seed, hidden, out.ctypes.data_as(C.c_void_p), n)
     if st != DC_OK:
         raise DCError(st, "dc_policy_init rejected its arguments")
+    return out
+
+
+def attend_noalloc(q, k, v, out=None, stream=None):
+    """Full-cache decode attention with no device allocation by the library:
+    q [rows][group][d], k/v [rows][n][d] bf16 CUDA tensors -> out fp32."""
+    import torch
+    rows, group, d = q.shape
+    n = k.shape[1]
+    if out is None:
+        out = torch.empty((rows, group, d), dtype=torch.float32, device=q.device)
+    s = (stream or torch.cuda.current_stream()).cuda_stream
+    st = lib().dc_attend_noalloc(q.data_ptr(), k.data_ptr(), v.data_ptr(), rows, n, d, group, out.data_ptr(), s)
+    if st != DC_OK:
+        raise DCError(st, lib().dc_noalloc_last_error().decode())
     return out
 
 
