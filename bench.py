@@ -70,6 +70,23 @@ def step_bytes(wl, n: int, moved_per_row: float = 1.0) -> float:
     return wl.rows * per_row
 
 
+def fused_traffic_per_token_row():
+    """DRAM bytes per token-row of the fused kernel from the committed ncu
+    summary, or None if the kernel source changed since it was captured."""
+    import hashlib
+    import re
+    prof = os.path.join(ROOT, "profiles", "fused_kernel_19L_b4_n8193_ncu_full.md")
+    src = os.path.join(ROOT, "paper_2608_08878_gb300", "csrc", "dc_fused.cu")
+    try:
+        text = open(prof).read()
+        t = float(re.search(r"traffic_bytes_per_token_row:\s*([0-9.]+)", text).group(1))
+        sha = re.search(r"kernel_source_sha256_prefix:\s*([0-9a-f]+)", text).group(1)
+        cur = hashlib.sha256(open(src, "rb").read()).hexdigest()[:len(sha)]
+        return t if cur == sha else None
+    except Exception:
+        return None
+
+
 class ClockSampler:
     """nvidia-smi clock/throttle samples while the timed region runs."""
 
@@ -284,6 +301,11 @@ def run_gpu(args):
     else:
         alg = wl.rows * row_bytes_per_step(n_steady, d, wl.alpha_mode)
     achieved = alg / (per_launch_ms / 1e3) / 1e9
+    traffic = None
+    if dom == "attend" and engine == "fused":
+        tpr = fused_traffic_per_token_row()
+        if tpr is not None:
+            traffic = wl.rows * n_steady * tpr  # scaled from the profiled case by token-rows
     gpu_launches = int(sum(v[1] for v in prof.values()))
 
     # full-cache comparator on the same inputs (the uncompressed prompt)
@@ -337,7 +359,7 @@ def run_gpu(args):
                     "frac_of_measured": gbs / peaks["hbm_gbs"], "peak_source": peak_src},
             "first_step_ms": first_ms,
             "roofline": {"bound": "hbm", "kernel": dom, "achieved": achieved, "peak": peaks["hbm_gbs"],
-                         "unit": "GB/s", "frac": achieved / peaks["hbm_gbs"], "traffic": None,
+                         "unit": "GB/s", "frac": achieved / peaks["hbm_gbs"], "traffic": traffic,
                          "peak_source": f"{peak_src} copy bandwidth",
                          "per_launch_ms": per_launch_ms, "algorithmic_bytes_per_launch": alg},
             "phases_ms_per_step": {k: v[0] / K for k, v in prof.items() if v[1]},
