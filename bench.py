@@ -218,6 +218,19 @@ def oracle_sample(wl, seconds: float = 12.0, threads: int | None = None, warm_st
 # GPU leg
 # ---------------------------------------------------------------------------
 
+def job_throughput(el_ms: float, steps: int, dist=None, device="cpu"):
+    """(max elapsed ms over ranks, whole-job decode steps/s): every rank runs
+    `steps` steps of its own replica and the job ends with the slowest rank."""
+    world = 1
+    if dist is not None:
+        import torch
+        world = dist.get_world_size()
+        t = torch.tensor([el_ms], dtype=torch.float64, device=device)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        el_ms = float(t.item())
+    return el_ms, world * steps / (el_ms / 1e3)
+
+
 def run_gpu(args):
     import torch
     from paper_2608_08878_gb300 import build, dc, synth, synth_device
@@ -276,12 +289,8 @@ def run_gpu(args):
     cache.sync()  # device-side status of every timed step (raises on error)
     prof = cache.profile_read()
     cache.profile(False)
-    if dist:
-        t = torch.tensor([el_ms], device="cuda")
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        el_ms = float(t.item())
+    el_ms, value = job_throughput(el_ms, K, dist, device="cuda")
     ms_per_step = el_ms / K
-    value = world * K / (el_ms / 1e3)
     bytes_step = step_bytes(wl, n_steady)
     gbs = bytes_step / (ms_per_step / 1e3) / 1e9
     peaks, peak_src = measured_peaks()

@@ -1,0 +1,53 @@
+"""Multi-rank host logic of the benchmark on CPU (gloo, world size 2): the
+job time is the slowest rank's, the rate counts every rank's replica, and the
+reference arm runs on rank 0 only."""
+
+import os
+import socket
+
+import pytest
+import torch.multiprocessing as mp
+
+
+def _free_port():
+    s = socket.socket()
+    s.bind(("127.0.0.1", 0))
+    port = s.getsockname()[1]
+    s.close()
+    return port
+
+
+def _worker(rank, world, port, q):
+    import torch.distributed as dist
+    import bench
+    os.environ.update(MASTER_ADDR="127.0.0.1", MASTER_PORT=str(port), RANK=str(rank), WORLD_SIZE=str(world))
+    dist.init_process_group("gloo", rank=rank, world_size=world)
+    el, rate = bench.job_throughput(100.0 + 50.0 * rank, 10, dist, device="cpu")
+    ref = bench.run_reference(type("A", (), {"steps": 1, "warmup": 3, "cpu_seconds": 0.01})()) if rank else "skip"
+    q.put((rank, el, rate, ref))
+    dist.barrier()
+    dist.destroy_process_group()
+
+
+def test_job_throughput_takes_slowest_rank_and_counts_all_replicas():
+    ctx = mp.get_context("spawn")
+    q = ctx.Queue()
+    port = _free_port()
+    procs = [ctx.Process(target=_worker, args=(r, 2, port, q)) for r in range(2)]
+    for p in procs:
+        p.start()
+    out = sorted(q.get(timeout=120) for _ in procs)
+    for p in procs:
+        p.join(timeout=60)
+        assert p.exitcode == 0
+    for rank, el, rate, ref in out:
+        assert el == pytest.approx(150.0)
+        assert rate == pytest.approx(2 * 10 / 0.150)
+        if rank == 1:
+            assert ref is None  # the reference arm does no work off rank 0
+
+
+def test_single_rank_throughput():
+    import bench
+    el, rate = bench.job_throughput(200.0, 40)
+    assert el == 200.0 and rate == pytest.approx(200.0)
