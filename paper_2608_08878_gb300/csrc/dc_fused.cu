@@ -126,27 +126,24 @@ __device__ __forceinline__ void stash_load(uint32_t taddr, float* v) {
   }
 }
 
+// Online softmax state of one head in log2 units (m = max raw logit,
+// l = sum 2^x, u = sum 2^x x with x = (s - m) c), updated without branches.
+// The state starts at m = kNoMax, a finite stand-in for -infinity: its first
+// rescale factor underflows to 0.
+constexpr float kNoMax = -1e30f;
+
 __device__ __forceinline__ void online_add(float& m, float& l, float& u, float s, float c) {
-  if (s > m) {
-    if (m == -INFINITY) {
-      l = 1.f;
-      u = 0.f;
-    } else {
-      const float dl = (m - s) * c, f = ex2(dl);
-      u = (u + l * dl) * f;
-      l = fmaf(l, f, 1.f);
-    }
-    m = s;
-  } else {
-    const float x = (s - m) * c, pe = ex2(x);
-    l += pe;
-    u = fmaf(pe, x, u);
-  }
+  const float mn = fmaxf(m, s);
+  const float dm = (m - mn) * c;
+  const float f = ex2(dm);
+  const float x = (s - mn) * c;
+  const float pe = ex2(x);
+  u = fmaf(pe, x, (u + l * dm) * f);
+  l = fmaf(l, f, pe);
+  m = mn;
 }
 
 __device__ __forceinline__ void online_merge(float& m, float& l, float& u, float mo, float lo, float uo, float c) {
-  if (mo == -INFINITY) return;
-  if (m == -INFINITY) { m = mo; l = lo; u = uo; return; }
   const float M = fmaxf(m, mo), da = (m - M) * c, db = (mo - M) * c;
   const float fa = ex2(da), fb = ex2(db);
   u = (u + l * da) * fa + (uo + lo * db) * fb;
@@ -386,7 +383,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
       float m[G], l[G], u[G];
 #pragma unroll
-      for (int h = 0; h < G; ++h) { m[h] = -INFINITY; l[h] = 0.f; u[h] = 0.f; }
+      for (int h = 0; h < G; ++h) { m[h] = kNoMax; l[h] = 0.f; u[h] = 0.f; }
 
       // ---------------- K pass: this warpgroup's tiles (global index parity)
       for (int j = (wg - gs) & 1; j < nT; j += 2) {
@@ -413,10 +410,14 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
           for (int h = 0; h < G; ++h) online_add(m[h], l[h], u[h], S16[h], c);
           if (st.has_prev || st.has_dep) {
-            float zp = 0.f, sp = 0.f, zd = 0.f, sd = 0.f;
-            if (st.has_prev && pos <= st.p_prev) window_terms<G>(S16 + G, pm, pnl, pH, c, zp, sp);
-            if (st.has_dep && pos <= st.p_dep) window_terms<G>(S16 + 2 * G, dm, dnl, dH, c, zd, sd);
-            sz = window_update(sz, sp, sd, zp, zd);
+            // terms of the previous and the departing query, masked (x 1 or x 0,
+            // both exact) where the token was not yet in the cache at that step
+            float zp, sp, zd, sd;
+            window_terms<G>(S16 + G, pm, pnl, pH, c, zp, sp);
+            window_terms<G>(S16 + 2 * G, dm, dnl, dH, c, zd, sd);
+            const float mp = (st.has_prev && pos <= st.p_prev) ? 1.f : 0.f;
+            const float md = (st.has_dep && pos <= st.p_dep) ? 1.f : 0.f;
+            sz = window_update(sz, sp * mp, sd * md, zp * mp, zd * md);
             p.SZ[rbase + i] = sz;
           }
         }
@@ -449,7 +450,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       float L0 = 0.f;
 #pragma unroll
       for (int h = 0; h < G; ++h) {
-        float mm = -INFINITY, ll = 0.f, uu = 0.f;
+        float mm = kNoMax, ll = 0.f, uu = 0.f;
         for (int w = 0; w < 8; ++w)
           online_merge(mm, ll, uu, red[(w * G + h) * 3 + 0], red[(w * G + h) * 3 + 1], red[(w * G + h) * 3 + 2], c);
         M[h] = mm;
