@@ -66,6 +66,12 @@ typedef struct {
   int keep_features;  /* 1: also store x_i [R][capacity][5] fp32 for inspection */
   unsigned long long seed; /* policy weight seed (dc_policy_init) */
   void* stream;       /* cudaStream_t */
+  int tail_split;     /* fused engine, rows not a multiple of the grid: 1 (default)
+                         splits each row of the last, partly filled wave over two
+                         CTAs, which exchange softmax statistics, output and the
+                         eviction candidate through global memory under a
+                         cooperative launch (steps that evict one token or none);
+                         0: whole rows only */
 } dc_config;
 
 /* Fills *cfg with the defaults above (batch 1, q_heads 0 meaning 4 * kv_heads,
@@ -129,7 +135,10 @@ dc_status dc_decode_step_host(dc_cache* h, const void* q_host, const void* k_new
 
 /* One whole step of Algorithm 1: dc_decode_step followed by dc_evict(budget),
  * as one kernel when the fused engine takes the step (no scores are stored
- * then; DC_BUF_SCORE is not updated). Same arguments as dc_decode_step. */
+ * then; DC_BUF_SCORE is not updated). Exception: with split rows (see
+ * tail_split) a step that evicts more than one token runs as the two calls.
+ * The result is bit-identical to the two calls either way. Same arguments as
+ * dc_decode_step. */
 dc_status dc_step(dc_cache* h, const void* q, const void* k_new, const void* v_new, float* out,
                   int budget);
 

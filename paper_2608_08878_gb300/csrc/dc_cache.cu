@@ -57,6 +57,12 @@ struct dc_cache {
   dc::FusedMaps maps{};
   dc::FusedPolicy fpol{};
   __nv_bfloat16* wtile = nullptr;
+  // exchange buffers of the half rows (FusedStep::split_tail)
+  float* xstats = nullptr;
+  float* xo = nullptr;
+  int* xsel = nullptr;
+  unsigned* xflag = nullptr;
+  unsigned epoch = 0;
   std::vector<void*> allocs;
   std::string err;
   bool broken = false;
@@ -228,6 +234,7 @@ dc_status dc_config_default(dc_config* cfg) {
   cfg->keep_features = 0;
   cfg->seed = 0;
   cfg->stream = nullptr;
+  cfg->tail_split = 1;
   return DC_OK;
 }
 
@@ -342,6 +349,16 @@ dc_status dc_cache_create(int layers, int kv_heads, int head_dim, int capacity, 
     cudaError_t fe = dalloc(h, &h->wtile, 128 * 32 * sizeof(__nv_bfloat16));
     if (fe == cudaSuccess) fe = dc::make_fused_maps(p, &h->maps, &why);
     if (fe == cudaSuccess) fe = upload_fused_policy(h, w.data());
+    if (fe == cudaSuccess && cfg.tail_split) {
+      const int grid = (int)std::min<long long>(R, h->num_sms);
+      fe = dalloc(h, &h->xstats, dc::fused_xstats_len(grid, G) * sizeof(float));
+      if (fe == cudaSuccess) fe = dalloc(h, &h->xo, dc::fused_xo_len(grid, G, head_dim) * sizeof(float));
+      if (fe == cudaSuccess) fe = dalloc(h, &h->xsel, dc::fused_xsel_len(grid) * sizeof(int));
+      if (fe == cudaSuccess) fe = dalloc(h, &h->xflag, dc::fused_xflag_len(grid) * sizeof(unsigned));
+      if (fe == cudaSuccess)
+        fe = cudaMemsetAsync(h->xflag, 0, dc::fused_xflag_len(grid) * sizeof(unsigned), h->stream);
+      if (fe == cudaSuccess) fe = cudaStreamSynchronize(h->stream);
+    }
     if (fe == cudaSuccess) {
       h->fused_ok = true;
     } else {
@@ -402,6 +419,44 @@ dc_status dc_append(dc_cache* h, const void* k, const void* v, int n_tokens) {
   return DC_OK;
 }
 
+namespace {
+
+// Arguments of one fused launch; enables the half-row tail split when the
+// handle has exchange buffers and the step qualifies.
+dc::FusedStep fused_args(dc_cache* h, const dc::Step& st, const void* q, float* out, int do_evict, int B,
+                         int write_scores) {
+  dc::FusedStep fs{};
+  fs.q = (const __nv_bfloat16*)q;
+  fs.out = out;
+  fs.do_evict = do_evict;
+  fs.B = B;
+  fs.write_scores = write_scores;
+  fs.xstats = h->xstats;
+  fs.xo = h->xo;
+  fs.xsel = h->xsel;
+  fs.xflag = h->xflag;
+  if (h->xflag && dc::fused_can_split_tail(h->dev, st.n, fs, h->num_sms)) {
+    fs.split_tail = 1;
+    // flags hold epoch * 4 + phase; skip 0 so that a zeroed flag never matches
+    if (++h->epoch == 0) ++h->epoch;
+    fs.epoch = h->epoch;
+  }
+  return fs;
+}
+
+// Whether a decode step over n tokens would split the fused grid's last wave.
+bool tail_split_applies(dc_cache* h, int n) {
+  if (!h->xflag) return false;
+  dc::FusedStep fs{};
+  fs.xstats = h->xstats;
+  fs.xo = h->xo;
+  fs.xsel = h->xsel;
+  fs.xflag = h->xflag;
+  return dc::fused_can_split_tail(h->dev, n, fs, h->num_sms);
+}
+
+}  // namespace
+
 dc_status dc_decode_step(dc_cache* h, const void* q, const void* k_new, const void* v_new, float* out) {
   DC_CHECK_HANDLE(h);
   if (!q || !k_new || !v_new || !out) return fail(h, DC_ERR_INVALID_ARG, "NULL pointer");
@@ -415,7 +470,7 @@ dc_status dc_decode_step(dc_cache* h, const void* q, const void* k_new, const vo
   }
   const dc::Step st = begin_step(h);
   if (use_fused(h, st.n)) {
-    dc::FusedStep fs{(const __nv_bfloat16*)q, out, 0, 0, 1};
+    const dc::FusedStep fs = fused_args(h, st, q, out, 0, 0, 1);
     cudaError_t e;
     {
       Phase ph(h, DC_PHASE_ATTEND, 1);
@@ -443,15 +498,22 @@ dc_status dc_step(dc_cache* h, const void* q, const void* k_new, const void* v_n
     if (s != DC_OK) return s;
     return dc_evict(h, budget);
   }
+  const int B = budget <= 0 ? h->budget : budget;
+  if (B < n1 - 1 && tail_split_applies(h, n1)) {
+    // several evictions need the whole row's scores in one CTA: with half
+    // rows this step runs as the decode kernel plus the eviction kernel
+    dc_status s = dc_decode_step(h, q, k_new, v_new, out);
+    if (s != DC_OK) return s;
+    return dc_evict(h, budget);
+  }
   if (h->seen + 1 > 0x7FFFFFFFll) return fail(h, DC_ERR_CAPACITY, "position counter overflow");
   {
     Phase ph(h, DC_PHASE_APPEND, 1);
     dc::launch_append(h->dev, k_new, v_new, 1, h->n, (int)h->seen, h->stream);
   }
   const dc::Step st = begin_step(h);
-  const int B = budget <= 0 ? h->budget : budget;
   const int keep = std::min(st.n, B);
-  dc::FusedStep fs{(const __nv_bfloat16*)q, out, keep < st.n ? 1 : 0, keep, 0};
+  const dc::FusedStep fs = fused_args(h, st, q, out, keep < st.n ? 1 : 0, keep, 0);
   cudaError_t e;
   {
     Phase ph(h, DC_PHASE_ATTEND, 1);

@@ -28,10 +28,18 @@
 // TMEM columns: S tiles [0, 32), O [32, 48), policy layer of warpgroup w
 // [128 + 128 w, 256 + 128 w), logit stash [48, 128) and [384, 512).
 //
-// Per-token state rides along with the tiles: TMA bulk copies bring the
-// positions and window sums with each K tile and the positions and |v| with
-// each V tile. The K pass writes the updated window sums back; the V pass
-// re-reads them (L2-resident by then) with loads issued ahead of use.
+// Per-token state rides along with the K tiles: TMA bulk copies bring the
+// positions and window sums. The K pass writes the updated window sums back;
+// the V pass re-reads them, with the positions and |v| (L2-resident), in loads
+// issued two tiles ahead of use.
+//
+// Barrier phases: a parity wait is only sound when the waiting thread cannot
+// be two phases ahead of the barrier. Every barrier here has one waiter that
+// waits its phases in order (the producer, the MMA issuer, one warpgroup), or,
+// for the K pass's stage reads, waits after a signal that implies the phase:
+// the tile's S, committed by the MMA issuer after its own in-order wait. The
+// stages alternate between the warpgroups, so the V pass does not wait on
+// them at all.
 #include <cuda.h>
 
 #include "dc_common.cuh"
@@ -46,13 +54,12 @@ using namespace sm100;
 namespace {
 
 constexpr int kStages = 3;
-// stage: K or V tile (32 KB, two 64-dim column blocks) + the tile's per-token
-// state: positions (512 B), |v| (512 B, V tiles) or window sums (2 KB, K tiles)
+// stage: K or V tile (32 KB, two 64-dim column blocks); K tiles also bring the
+// tile's positions (512 B) and window sums (2 KB)
 constexpr int kTileRegion = 32768;
-constexpr int kOffPos = kTileRegion;          // int32 [128]
-constexpr int kOffVn = kTileRegion + 512;     // fp32 [128]
-constexpr int kOffSZ = kTileRegion + 1024;    // fp32x4 [128]
-constexpr int kStageBytes = kTileRegion + 3072;
+constexpr int kOffPos = kTileRegion;          // int32 [128] (K tiles)
+constexpr int kOffSZ = kTileRegion + 1024;    // fp32x4 [128] (K tiles)
+constexpr int kStageBytes = kTileRegion + 3072;  // a multiple of 1024 (swizzle atoms)
 constexpr int kTok = 128;
 constexpr int kThreads = 352;
 constexpr int kEpi = 256;                     // two warpgroups
@@ -151,6 +158,25 @@ __device__ __forceinline__ void online_merge(float& m, float& l, float& u, float
   m = M;
 }
 
+// Work items of a CTA: whole rows r = blockIdx.x + k * gridDim.x, and with a
+// split tail, half of one row of the last wave (half 0: the first ceil(nT/2)
+// tiles, half 1: the rest).
+struct Item {
+  int row, t0, t1, half;  // half -1: the whole row
+};
+
+__device__ __forceinline__ int item_count(const FusedStep& fs, int R) {
+  const int W = gridDim.x, c = blockIdx.x, full = R / W, rem = R % W;
+  return full + (fs.split_tail ? (c < 2 * rem ? 1 : 0) : (c < rem ? 1 : 0));
+}
+
+__device__ __forceinline__ Item item_at(const FusedStep& fs, int R, int nT, int k) {
+  const int W = gridDim.x, c = blockIdx.x, full = R / W;
+  if (k < full || !fs.split_tail) return Item{c + k * W, 0, nT, -1};
+  const int mid = (nT + 1) >> 1, h = c & 1;
+  return Item{full * W + (c >> 1), h ? mid : 0, h ? nT : mid, h};
+}
+
 template <int D, int G>
 __global__ void __launch_bounds__(kThreads, 1)
     fused_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmV, Dev p,
@@ -224,8 +250,11 @@ __global__ void __launch_bounds__(kThreads, 1)
     // ------------------------------------------------------------ producer
     const uint64_t pol = l2_evict_first_policy();
     int g = 0, gr = 0, issued = 0;
-    for (int r = blockIdx.x; r < p.R; r += gridDim.x, ++gr) {
+    const int nitems = item_count(fs, p.R);
+    for (int k = 0; k < nitems; ++k, ++gr) {
       if (*abort) break;
+      const Item it = item_at(fs, p.R, nT, k);
+      const int r = it.row;
       const int qb = gr & 1;
       if (!mbar_wait(&bar[B_QEMPTY + qb], ((gr >> 1) & 1) ^ 1, abort, p.dbg, 1u, (unsigned)gr)) break;
       // query tile: rows [0,G) current, [G,2G) previous step, [2G,3G) departing
@@ -244,7 +273,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         *reinterpret_cast<uint4*>(qt + (kc >> 3) * 2048 + sw128(h, kc & 7)) = cur;
         *reinterpret_cast<uint4*>(qt + (kc >> 3) * 2048 + sw128(G + h, kc & 7)) = pv;
         *reinterpret_cast<uint4*>(qt + (kc >> 3) * 2048 + sw128(2 * G + h, kc & 7)) = dv;
-        reinterpret_cast<uint4*>(ring_slot + h * D)[kc] = cur;
+        if (it.half < 0) reinterpret_cast<uint4*>(ring_slot + h * D)[kc] = cur;  // halves: see the epilogue
       }
       fence_proxy_async();
       __syncwarp();
@@ -252,17 +281,18 @@ __global__ void __launch_bounds__(kThreads, 1)
         mbar_arrive(&bar[B_QFULL + qb]);
         for (int pass = 0; pass < 2 && !*abort; ++pass) {
           const CUtensorMap* tm = pass ? &tmV : &tmK;
-          for (int j = 0; j < nT; ++j, ++g) {
+          for (int j = it.t0; j < it.t1; ++j, ++g) {
             const int s = g % kStages;
             if (!mbar_wait(&bar[B_EMPTY + s], ((g / kStages) & 1) ^ 1, abort, p.dbg, 2u, (unsigned)g)) break;
-            mbar_expect_tx(&bar[B_FULL + s], kTileBytes + (pass ? 1024u : 2560u));
+            mbar_expect_tx(&bar[B_FULL + s], kTileBytes + (pass ? 0u : 2560u));
             uint8_t* dst = smem + OFF_STAGE + s * kStageBytes;
             const int y = r * p.stride + j * kTok;
             tma_load_2d(dst, tm, 0, y, &bar[B_FULL + s], pol);
             if (D == 128) tma_load_2d(dst + 16384, tm, 64, y, &bar[B_FULL + s], pol);
-            bulk_load(dst + kOffPos, p.pos + y, 512, &bar[B_FULL + s]);
-            if (pass) bulk_load(dst + kOffVn, p.vnorm + y, 512, &bar[B_FULL + s]);
-            else bulk_load(dst + kOffSZ, p.SZ + y, 2048, &bar[B_FULL + s]);
+            if (!pass) {
+              bulk_load(dst + kOffPos, p.pos + y, 512, &bar[B_FULL + s]);
+              bulk_load(dst + kOffSZ, p.SZ + y, 2048, &bar[B_FULL + s]);
+            }
             issued = g + 1;
           }
         }
@@ -281,13 +311,15 @@ __global__ void __launch_bounds__(kThreads, 1)
       const uint32_t id_qk = idesc_bf16(128, 16, 0, 0);
       const uint32_t id_pv = idesc_bf16(128, 16, 1, 0);
       int g = 0, gs = 0, gv = 0, gr = 0;
-      for (int r = blockIdx.x; r < p.R; r += gridDim.x, ++gr) {
+      const int nitems = item_count(fs, p.R);
+      for (int k = 0; k < nitems; ++k, ++gr) {
         if (*abort) break;
+        const Item it = item_at(fs, p.R, nT, k);
         const int qb = gr & 1;
         if (!mbar_wait(&bar[B_QFULL + qb], (gr >> 1) & 1, abort, p.dbg, 3u, (unsigned)gr)) break;
         tc_fence_after();
         const uint32_t qaddr = smem_u32(smem + OFF_Q + qb * 4096);
-        for (int j = 0; j < nT; ++j, ++g, ++gs) {
+        for (int j = it.t0; j < it.t1; ++j, ++g, ++gs) {
           const int s = g % kStages, b = gs & 1;
           if (!mbar_wait(&bar[B_FULL + s], (g / kStages) & 1, abort, p.dbg, 4u, (unsigned)g)) break;
           if (!mbar_wait(&bar[B_SEMPTY + b], ((gs >> 1) & 1) ^ 1, abort, p.dbg, 5u, (unsigned)gs)) break;
@@ -306,11 +338,14 @@ __global__ void __launch_bounds__(kThreads, 1)
         mma_commit(&bar[B_QEMPTY + qb]);
         // V pass: PV MMAs in tile order; a V stage is released as soon as its
         // tile's weights are in (the policy-layer MMAs run on warp 10)
-        for (int j = 0; j < nT; ++j, ++g, ++gv) {
+        for (int j = it.t0; j < it.t1; ++j, ++g, ++gv) {
           const int s = g % kStages, pb = gv & 1;
           if (!mbar_wait(&bar[B_FULL + s], (g / kStages) & 1, abort, p.dbg, 13u, (unsigned)g)) break;
+          // only these MMAs read a V stage: the four epilogue arrivals of the
+          // stage's release are made here (its last one is the commit below)
+          mbar_arrive_cnt(&bar[B_EMPTY + s], 4);
           if (!mbar_wait(&bar[B_PFULL + pb], (gv >> 1) & 1, abort, p.dbg, 14u, (unsigned)gv)) break;
-          if (j == 0 && !mbar_wait(&bar[B_OEMPTY], (gr & 1) ^ 1, abort, p.dbg, 15u, (unsigned)gr)) break;
+          if (j == it.t0 && !mbar_wait(&bar[B_OEMPTY], (gr & 1) ^ 1, abort, p.dbg, 15u, (unsigned)gr)) break;
           tc_fence_after();
           const uint32_t vaddr = smem_u32(smem + OFF_STAGE + s * kStageBytes);
           const uint32_t paddr = smem_u32(smem + OFF_P + pb * 4096);
@@ -319,11 +354,11 @@ __global__ void __launch_bounds__(kThreads, 1)
           for (int ks = 0; ks < kTok / 16; ++ks) {
             const uint32_t poff = (uint32_t)(ks >> 2) * 2048u + (uint32_t)(ks & 3) * 32u;
             mma_bf16(tmem + kColO, sdesc_sw128(vaddr + ks * 2048u, 16384, 1024),
-                     sdesc_sw128(paddr + poff, 16, 1024), id_pv, (j > 0 || ks > 0) ? 1u : 0u);
+                     sdesc_sw128(paddr + poff, 16, 1024), id_pv, (j > it.t0 || ks > 0) ? 1u : 0u);
           }
           mma_commit(&bar[B_PEMPTY + pb]);
           mma_commit(&bar[B_EMPTY + s]);
-          if (j == nT - 1) mma_commit(&bar[B_OFULL]);
+          if (j == it.t1 - 1) mma_commit(&bar[B_OFULL]);
         }
       }
       // all issued MMAs complete before TMEM is released
@@ -337,9 +372,11 @@ __global__ void __launch_bounds__(kThreads, 1)
       const uint32_t id_m = idesc_bf16(128, 128, 0, 0);
       const uint32_t waddr = smem_u32(smem + OFF_W);
       int gv = 0;
-      for (int r = blockIdx.x; r < p.R; r += gridDim.x) {
+      const int nitems = item_count(fs, p.R);
+      for (int k = 0; k < nitems; ++k) {
         if (*abort) break;
-        for (int j = 0; j < nT; ++j, ++gv) {
+        const Item it = item_at(fs, p.R, nT, k);
+        for (int j = it.t0; j < it.t1; ++j, ++gv) {
           const int pb = gv & 1;
           if (!mbar_wait(&bar[B_AFULL + pb], (gv >> 1) & 1, abort, p.dbg, 16u, (unsigned)gv)) break;
           if (!mbar_wait(&bar[B_MEMPTY + pb], ((gv >> 1) & 1) ^ 1, abort, p.dbg, 17u, (unsigned)gv)) break;
@@ -370,8 +407,12 @@ __global__ void __launch_bounds__(kThreads, 1)
     auto sync = [] { named_bar(1, kEpi); };
     const SelectScratch scr{s_hist, s_sh, s_wsum, s_best, s_best_slot};
     int g = 0, gs = 0, gv = 0, gr = 0;
-    for (int r = blockIdx.x; r < p.R; r += gridDim.x, ++gr) {
+    const int nitems = item_count(fs, p.R);
+    for (int k = 0; k < nitems; ++k, ++gr) {
       if (named_bar_or(1, kEpi, *abort != 0)) break;
+      const Item it = item_at(fs, p.R, nT, k);
+      const int r = it.row, t0 = it.t0, t1 = it.t1, nTi = it.t1 - it.t0;
+      const int ts = r - (p.R / gridDim.x) * gridDim.x;  // tail slot (half rows only)
       const size_t rbase = (size_t)r * p.stride;
       float pm[G], pnl[G], pH[G], dm[G], dnl[G], dH[G];
 #pragma unroll
@@ -386,8 +427,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       for (int h = 0; h < G; ++h) { m[h] = kNoMax; l[h] = 0.f; u[h] = 0.f; }
 
       // ---------------- K pass: this warpgroup's tiles (global index parity)
-      for (int j = (wg - gs) & 1; j < nT; j += 2) {
-        const int gj = g + j, gsj = gs + j;
+      for (int j = t0 + ((wg - gs) & 1); j < t1; j += 2) {
+        const int gj = g + (j - t0), gsj = gs + (j - t0);
         const int s = gj % kStages, b = gsj & 1;
         mbar_wait(&bar[B_SFULL + b], (gsj >> 1) & 1, abort, p.dbg, 6u, (unsigned)gsj);
         mbar_wait(&bar[B_FULL + s], (gj / kStages) & 1, abort, p.dbg, 12u, (unsigned)gj);
@@ -425,8 +466,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         __syncwarp();
         stash_store<GS>(lane_addr + stash_col<GS>(j), S16);
       }
-      g += nT;
-      gs += nT;
+      g += nTi;
+      gs += nTi;
       if constexpr (GS > 0) tmem_st_wait();
       // ---------------- row softmax statistics (deterministic merge order)
 #pragma unroll
@@ -446,22 +487,66 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
       }
       sync();
-      float M[G], NL[G], Hh[G];
-      float L0 = 0.f;
+      float Mm[G], Ll[G], Uu[G];
 #pragma unroll
       for (int h = 0; h < G; ++h) {
         float mm = kNoMax, ll = 0.f, uu = 0.f;
         for (int w = 0; w < 8; ++w)
           online_merge(mm, ll, uu, red[(w * G + h) * 3 + 0], red[(w * G + h) * 3 + 1], red[(w * G + h) * 3 + 2], c);
-        M[h] = mm;
-        NL[h] = -log2f(ll);
-        Hh[h] = logf(ll) - 0.69314718055994531f * (uu / ll);
-        if (etid == h) L0 = ll;
+        Mm[h] = mm; Ll[h] = ll; Uu[h] = uu;
       }
       sync();  // red is rewritten by the next row
+      const int half = it.half;
+      unsigned* my_flag = half >= 0 ? fs.xflag + 2 * ts + half : nullptr;
+      const unsigned* peer_flag = half >= 0 ? fs.xflag + 2 * ts + (half ^ 1) : nullptr;
+      const unsigned ep = fs.epoch * 4u;
+      if (half >= 0) {
+        // half row: swap the partial statistics with the other half, then
+        // both merge half 0's before half 1's (identical results on both)
+        float4* xs = reinterpret_cast<float4*>(fs.xstats);
+        if (etid < G) {
+          xs[(2 * ts + half) * G + etid] = make_float4(Mm[etid], Ll[etid], Uu[etid], 0.f);
+          __threadfence();
+        }
+        sync();
+        if (etid == 0) {
+          flag_release(my_flag, ep + 1u);
+          flag_wait(peer_flag, ep + 1u, abort, p.dbg, 20u, (unsigned)r);
+        }
+        sync();
+#pragma unroll
+        for (int h = 0; h < G; ++h) {
+          const float4 o = __ldcg(&xs[(2 * ts + (half ^ 1)) * G + h]);
+          float mm = kNoMax, ll = 0.f, uu = 0.f;
+          if (half == 0) {
+            online_merge(mm, ll, uu, Mm[h], Ll[h], Uu[h], c);
+            online_merge(mm, ll, uu, o.x, o.y, o.z, c);
+          } else {
+            online_merge(mm, ll, uu, o.x, o.y, o.z, c);
+            online_merge(mm, ll, uu, Mm[h], Ll[h], Uu[h], c);
+          }
+          Mm[h] = mm; Ll[h] = ll; Uu[h] = uu;
+        }
+        // half 1 has read the departing query and statistics (it published
+        // after its K pass): half 0 may now give their ring slot to this step
+        if (half == 0) {
+          const int qo = ((r / p.kvh) * p.qh + (r % p.kvh) * G) * D;
+          uint4* ring_slot = reinterpret_cast<uint4*>(p.ring_q + ((size_t)r * p.w + st.slot) * G * D);
+          for (int e = etid; e < G * (D / 8); e += kEpi) ring_slot[e] = reinterpret_cast<const uint4*>(fs.q + qo)[e];
+        }
+      }
+      float M[G], NL[G], Hh[G];
+      float L0 = 0.f;
+#pragma unroll
+      for (int h = 0; h < G; ++h) {
+        M[h] = Mm[h];
+        NL[h] = -log2f(Ll[h]);
+        Hh[h] = logf(Ll[h]) - 0.69314718055994531f * (Uu[h] / Ll[h]);
+        if (etid == h) L0 = Ll[h];
+      }
       // push (m, l, H, -log2 l) of this step into the ring slot it takes over
-      // (the producer already wrote the query there)
-      if (etid < G) {
+      // (the producer, or half 0 above, wrote the query there)
+      if (etid < G && half <= 0) {
         float4 v;
         v.x = M[etid]; v.y = L0; v.z = Hh[etid]; v.w = NL[etid];
         reinterpret_cast<float4*>(p.ring_stats)[((size_t)r * p.w + st.slot) * G + etid] = v;
@@ -471,26 +556,34 @@ __global__ void __launch_bounds__(kThreads, 1)
       // ---------------- V pass: this warpgroup's tiles; prep of the next one
       // overlaps the MMAs of the current one
       const float pos_den = (float)max(st.p_newest, 1);
-      const int j0 = (wg - gv) & 1;
+      const int j0 = t0 + ((wg - gv) & 1);
+      // per-token state of this warpgroup's tiles, loaded two own tiles ahead
+      // (window sums written by the K pass, positions, |v|)
       const float4* szrow = p.SZ + rbase + tok;
-      float4 szA = j0 < nT ? szrow[j0 * kTok] : make_float4(0.f, 0.f, 0.f, 0.f);
-      float4 szB = j0 + 2 < nT ? szrow[(j0 + 2) * kTok] : make_float4(0.f, 0.f, 0.f, 0.f);
+      const int* posrow = p.pos + rbase + tok;
+      const float* vnrow = p.vnorm + rbase + tok;
+      const float4 kZero4 = make_float4(0.f, 0.f, 0.f, 0.f);
+      float4 szA = j0 < t1 ? szrow[j0 * kTok] : kZero4;
+      float4 szB = j0 + 2 < t1 ? szrow[(j0 + 2) * kTok] : kZero4;
+      int posA = j0 < t1 ? posrow[j0 * kTok] : 0;
+      int posB = j0 + 2 < t1 ? posrow[(j0 + 2) * kTok] : 0;
+      float vnA = j0 < t1 ? vnrow[j0 * kTok] : 0.f;
+      float vnB = j0 + 2 < t1 ? vnrow[(j0 + 2) * kTok] : 0.f;
       auto prep = [&](int j) {
-        const int gj = g + j, gvj = gv + j;
-        const int s = gj % kStages, pb = gvj & 1;
-        // window sums of tile j (loaded two own tiles ahead)
+        const int gvj = gv + (j - t0), pb = gvj & 1;
         const float4 sz = szA;
+        const int pos = posA;
+        const float vn = vnA;
         szA = szB;
-        if (j + 4 < nT) szB = szrow[(j + 4) * kTok];
-        mbar_wait(&bar[B_FULL + s], (gj / kStages) & 1, abort, p.dbg, 7u, (unsigned)gj);
+        posA = posB;
+        vnA = vnB;
+        if (j + 4 < t1) {
+          szB = szrow[(j + 4) * kTok];
+          posB = posrow[(j + 4) * kTok];
+          vnB = vnrow[(j + 4) * kTok];
+        }
         const int i = j * kTok + tok;
         const bool valid = i < n;
-        const uint8_t* stg = smem + OFF_STAGE + s * kStageBytes;
-        const int pos = reinterpret_cast<const int*>(stg + kOffPos)[tok];
-        const float vn = reinterpret_cast<const float*>(stg + kOffVn)[tok];
-        __syncwarp();
-        if (lane == 0) mbar_arrive(&bar[B_EMPTY + s]);  // stage: only the PV MMA still reads it
-        __syncwarp();
         float sv[G];
         stash_load<GS>(lane_addr + stash_col<GS>(j), sv);
         if constexpr (GS > 0) tmem_ld_wait();
@@ -581,7 +674,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (lane == 0) mbar_arrive(&bar[B_AFULL + pb]);
       };
       auto finish = [&](int j) {
-        const int gvj = gv + j, pb = gvj & 1;
+        const int gvj = gv + (j - t0), pb = gvj & 1;
         mbar_wait(&bar[B_MFULL + pb], (gvj >> 1) & 1, abort, p.dbg, 10u, (unsigned)gvj);
         __syncwarp();
         tc_fence_after();
@@ -608,14 +701,16 @@ __global__ void __launch_bounds__(kThreads, 1)
           if (fs.write_scores) p.score[rbase + i] = score;
         }
       };
-      if (j0 < nT) prep(j0);
-      for (int j = j0; j < nT; j += 2) {
-        if (j + 2 < nT) prep(j + 2);
+      if (j0 < t1) prep(j0);
+      for (int j = j0; j < t1; j += 2) {
+        if (j + 2 < t1) prep(j + 2);
         finish(j);
       }
-      g += nT;
-      gv += nT;
-      // ---------------- attention output (warpgroup 0)
+      g += nTi;
+      gv += nTi;
+      // ---------------- attention output (warpgroup 0); a half row's two
+      // partial sums (weights already normalised by the whole row) add up
+      float ov[G];
       if (wg == 0) {
         mbar_wait(&bar[B_OFULL], gr & 1, abort, p.dbg, 11u, (unsigned)gr);
         __syncwarp();
@@ -626,16 +721,87 @@ __global__ void __launch_bounds__(kThreads, 1)
         tc_fence_before();
         __syncwarp();
         if (lane == 0) mbar_arrive(&bar[B_OEMPTY]);
-        if (tok < D) {
-          float* op = fs.out + ((r / p.kvh) * p.qh + (r % p.kvh) * G) * D;
 #pragma unroll
-          for (int h = 0; h < G; ++h) op[h * D + tok] = o16[h] + o16[G + h];
+        for (int h = 0; h < G; ++h) ov[h] = o16[h] + o16[G + h];
+        if (half == 1 && tok < D) {
+#pragma unroll
+          for (int h = 0; h < G; ++h) fs.xo[((size_t)ts * G + h) * D + tok] = ov[h];
+          __threadfence();
         }
+      }
+      if (half >= 0) {
+        sync();
+        if (etid == 0) {
+          if (half == 1) flag_release(my_flag, ep + 2u);
+          else flag_wait(peer_flag, ep + 2u, abort, p.dbg, 21u, (unsigned)r);
+        }
+        sync();
+      }
+      if (wg == 0 && half <= 0 && tok < D) {
+        float* op = fs.out + ((r / p.kvh) * p.qh + (r % p.kvh) * G) * D;
+#pragma unroll
+        for (int h = 0; h < G; ++h)
+          op[h * D + tok] = half == 0 ? ov[h] + __ldcg(&fs.xo[((size_t)ts * G + h) * D + tok]) : ov[h];
       }
       // ---------------- argtop_B and prune
       if (fs.do_evict && fs.B < n) {
         sync();
-        team_select_compact<kEpi>(p, r, n, fs.B, sc, etid, scr, sync);
+        if (half < 0) {
+          team_select_compact<kEpi>(p, r, n, fs.B, sc, etid, scr, sync);
+        } else {
+          // one eviction (B == n - 1): each half finds its lowest-ranked
+          // token, the halves swap candidates, and half 1, which holds the
+          // last slot B, moves it into the evicted slot
+          const int* ps = p.pos + rbase;
+          const int i0 = t0 * kTok, i1 = min(t1 * kTok, n);
+          uint32_t bk = 0xFFFFFFFFu;
+          int bs = -1, bp = -1;
+          for (int i = i0 + etid; i < i1; i += kEpi) {
+            const uint32_t kk = score_key(sc[i]);
+            if (kk < bk || (kk == bk && bs >= 0 && ps[i] > bp)) { bk = kk; bs = i; bp = ps[i]; }
+          }
+          auto lower = [](uint32_t ka, int sa, int pa, uint32_t kb, int sb, int pb) {  // (kb, sb) ranks lower?
+            if (sb < 0) return false;
+            if (sa < 0) return true;
+            return kb < ka || (kb == ka && pb > pa);
+          };
+#pragma unroll
+          for (int off = 16; off > 0; off >>= 1) {
+            const uint32_t ok = __shfl_xor_sync(0xffffffffu, bk, off);
+            const int os = __shfl_xor_sync(0xffffffffu, bs, off);
+            const int op = __shfl_xor_sync(0xffffffffu, bp, off);
+            if (lower(bk, bs, bp, ok, os, op)) { bk = ok; bs = os; bp = op; }
+          }
+          if (lane == 0) { s_best[ew] = bk; s_best_slot[ew] = bs; s_hist[ew] = bp; }
+          sync();
+          if (etid == 0) {
+            uint32_t fk = (uint32_t)s_best[0];
+            int fe = s_best_slot[0], fpos = s_hist[0];
+            for (int w = 1; w < kEpi / kWarp; ++w)
+              if (lower(fk, fe, fpos, (uint32_t)s_best[w], s_best_slot[w], s_hist[w])) {
+                fk = (uint32_t)s_best[w]; fe = s_best_slot[w]; fpos = s_hist[w];
+              }
+            int* xs = fs.xsel + (2 * ts + half) * 4;
+            xs[0] = (int)fk; xs[1] = fe; xs[2] = fpos;
+            __threadfence();
+            flag_release(my_flag, ep + 3u);
+            if (flag_wait(peer_flag, ep + 3u, abort, p.dbg, 22u, (unsigned)r)) {
+              const int* ys = fs.xsel + (2 * ts + (half ^ 1)) * 4;
+              const uint32_t ok = (uint32_t)__ldcg(&ys[0]);
+              const int oe = __ldcg(&ys[1]), opos = __ldcg(&ys[2]);
+              // the same total order on both halves: lower key, then the later position
+              if (lower(fk, fe, fpos, ok, oe, opos)) fe = oe;
+            } else {
+              fe = -1;
+            }
+            s_sh[0] = fe;
+          }
+          sync();
+          const int e = s_sh[0];
+          if (half == 1 && e >= 0 && e < fs.B && etid < kWarp)
+            move_slot(p, rbase + fs.B, rbase + e, etid, kWarp);
+          sync();
+        }
       }
     }
   }
@@ -672,13 +838,37 @@ static cudaError_t launch_t(const FusedMaps& maps, const Dev& p, const Step& st,
     if (e != cudaSuccess) return e;
     attr = true;
   }
-  fused_kernel<D, G><<<grid, kThreads, kSmemBytes, s>>>(maps.k, maps.v, p, st, fs, fp);
-  return cudaGetLastError();
+  if (!fs.split_tail) {
+    fused_kernel<D, G><<<grid, kThreads, kSmemBytes, s>>>(maps.k, maps.v, p, st, fs, fp);
+    return cudaGetLastError();
+  }
+  // the two CTAs of a half row wait on each other: a cooperative launch
+  // guarantees that the whole grid is resident at once
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(grid);
+  cfg.blockDim = dim3(kThreads);
+  cfg.dynamicSmemBytes = kSmemBytes;
+  cfg.stream = s;
+  cudaLaunchAttribute la[1];
+  la[0].id = cudaLaunchAttributeCooperative;
+  la[0].val.cooperative = 1;
+  cfg.attrs = la;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, fused_kernel<D, G>, maps.k, maps.v, p, st, fs, fp);
+}
+
+static int fused_grid(const Dev& p, int num_sms) { return p.R < num_sms ? p.R : num_sms; }
+
+bool fused_can_split_tail(const Dev& p, int n, const FusedStep& fs, int num_sms) {
+  const int grid = fused_grid(p, num_sms), rem = p.R % grid;
+  const int nT = (n + kTok - 1) / kTok;
+  return fs.xflag && fs.xstats && fs.xo && fs.xsel && rem > 0 && 2 * rem <= grid && nT >= 2 &&
+         (!fs.do_evict || fs.B >= n || fs.B == n - 1);
 }
 
 cudaError_t launch_fused_step(const FusedMaps& maps, const Dev& p, const Step& st, const FusedStep& fs,
                               const FusedPolicy& fp, int num_sms, cudaStream_t s) {
-  const int grid = p.R < num_sms ? p.R : num_sms;
+  const int grid = fused_grid(p, num_sms);
   if (p.d == 128) {
     if (p.G == 4) return launch_t<128, 4>(maps, p, st, fs, fp, grid, s);
     if (p.G == 2) return launch_t<128, 2>(maps, p, st, fs, fp, grid, s);

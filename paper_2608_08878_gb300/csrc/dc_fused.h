@@ -26,7 +26,23 @@ struct FusedStep {
   int do_evict;      // 1: select and compact in the same kernel
   int B;             // tokens to keep when do_evict
   int write_scores;  // 1: also store scores in Dev::score (for dc_evict)
+  // Tail split: the R % grid rows of the last wave are each taken by two CTAs
+  // (halves of the row's tiles) that exchange softmax statistics, the output
+  // and the eviction candidate through global memory. Needs a cooperative
+  // launch (all CTAs resident) and, with do_evict, exactly one eviction.
+  int split_tail;
+  unsigned epoch;    // increases every launch; exchange flags compare against it
+  float* xstats;     // [grid/2][2][G][4]
+  float* xo;         // [grid/2][G][d]
+  int* xsel;         // [grid/2][2][4]
+  unsigned* xflag;   // [grid/2][2]
 };
+
+// Exchange buffer sizes (floats / ints) for a grid of `grid` CTAs.
+inline size_t fused_xstats_len(int grid, int G) { return (size_t)(grid / 2 + 1) * 2 * G * 4; }
+inline size_t fused_xo_len(int grid, int G, int d) { return (size_t)(grid / 2 + 1) * G * d; }
+inline size_t fused_xsel_len(int grid) { return (size_t)(grid / 2 + 1) * 2 * 4; }
+inline size_t fused_xflag_len(int grid) { return (size_t)(grid / 2 + 1) * 2; }
 
 // The policy MLP folded for the tensor cores (see prepare_policy):
 //   z_j = <a, w_j> with a = [r x, r, 1, 0] (LayerNorm) or [x, 1, 0, 0], where
@@ -53,6 +69,9 @@ cudaError_t make_fused_maps(const Dev& p, FusedMaps* maps, const char** why);
 // Folds a policy blob [W1 | b1 | gamma | beta | w2 | b2] (hidden H) into
 // FusedPolicy fields and the host copy of the weight tile (128 * 32 bf16).
 void prepare_policy(const float* blob, int H, int layernorm, FusedPolicy* fp, std::vector<__nv_bfloat16>* wtile);
+
+// Whether the step can split its last wave's rows (see FusedStep).
+bool fused_can_split_tail(const Dev& p, int n, const FusedStep& fs, int num_sms);
 
 cudaError_t launch_fused_step(const FusedMaps& maps, const Dev& p, const Step& st, const FusedStep& fs,
                               const FusedPolicy& fp, int num_sms, cudaStream_t s);

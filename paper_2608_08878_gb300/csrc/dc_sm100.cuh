@@ -37,6 +37,11 @@ __device__ __forceinline__ void mbar_arrive(uint64_t* bar) {
   asm volatile("mbarrier.arrive.release.cta.shared::cta.b64 _, [%0];" ::"r"(smem_u32(bar)) : "memory");
 }
 
+__device__ __forceinline__ void mbar_arrive_cnt(uint64_t* bar, uint32_t count) {
+  asm volatile("mbarrier.arrive.release.cta.shared::cta.b64 _, [%0], %1;" ::"r"(smem_u32(bar)), "r"(count)
+               : "memory");
+}
+
 __device__ __forceinline__ void mbar_expect_tx(uint64_t* bar, uint32_t bytes) {
   asm volatile("mbarrier.arrive.expect_tx.release.cta.shared::cta.b64 _, [%0], %1;" ::"r"(smem_u32(bar)),
                "r"(bytes)
@@ -103,6 +108,36 @@ __device__ __forceinline__ bool mbar_wait_drain(uint64_t* bar, uint32_t parity) 
     if (mbar_try_wait(bar, parity)) return true;
     if ((i & 255u) == 255u && globaltimer_ns() - t0 > kWaitNs) return false;
   }
+  return false;
+}
+
+// ---------------------------------------------------------------- flags between CTAs
+// A flag in global memory that only grows (a launch epoch times a small phase
+// count plus the phase); written with release, read with acquire semantics at
+// GPU scope.
+__device__ __forceinline__ void flag_release(unsigned* f, unsigned v) {
+  asm volatile("st.release.gpu.global.u32 [%0], %1;" ::"l"(f), "r"(v) : "memory");
+}
+
+__device__ __forceinline__ unsigned flag_acquire(const unsigned* f) {
+  unsigned v;
+  asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(f) : "memory");
+  return v;
+}
+
+// Waits until *f has reached `target` (wrap-safe compare). Bounded like
+// mbar_wait: gives up on *abort or after kWaitNs, recording the site.
+__device__ __forceinline__ bool flag_wait(const unsigned* f, unsigned target, volatile int* abort,
+                                          unsigned* dbg, unsigned site, unsigned info) {
+  const uint64_t t0 = globaltimer_ns();
+  for (uint32_t i = 0; i < kSpinLimit; ++i) {
+    if ((int)(flag_acquire(f) - target) >= 0) return true;
+    if (*abort) return false;
+    if ((i & 63u) == 63u && globaltimer_ns() - t0 > kWaitNs) break;
+    __nanosleep(64);
+  }
+  record_timeout(dbg, site, target, info);
+  *abort = 1;
   return false;
 }
 

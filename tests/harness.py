@@ -45,7 +45,8 @@ def check_attention(gpu_o, ref_o, what):
 class LockStep:
     """Drives a DistillCache and oracle rows for a sample of its rows."""
 
-    def __init__(self, wl: synth.Workload, rows, *, engine=0, device_inputs=False, capacity=None):
+    def __init__(self, wl: synth.Workload, rows, *, engine=0, device_inputs=False, capacity=None,
+                 tail_split=True):
         import torch
         from paper_2608_08878_gb300 import dc, synth_device
         self.torch, self.dc, self.sd = torch, dc, synth_device
@@ -58,7 +59,7 @@ class LockStep:
                                      batch=wl.batch, q_heads=wl.q_heads, window=wl.window,
                                      mlp_hidden=wl.mlp_hidden, layernorm=wl.layernorm,
                                      alpha_mode=wl.alpha_mode, engine=engine, keep_features=True,
-                                     seed=wl.policy_seed)
+                                     seed=wl.policy_seed, tail_split=tail_split)
         self.cache.set_policy(self.blob)
         self.orows = {}
         for r in self.rows:

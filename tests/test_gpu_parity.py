@@ -124,6 +124,57 @@ def test_step_equals_decode_then_evict(engine):
             assert torch.equal(a.cache.buffer(which)[:, :n], b.cache.buffer(which)[:, :n]), (s, which)
 
 
+def _tail_workload(**kw):
+    """Mistral-7B head shapes with a few more rows than SMs, so that the fused
+    grid's last wave is partly filled and its rows are split in halves."""
+    import torch
+    sms = torch.cuda.get_device_properties(0).multi_processor_count
+    batch = sms // 8 + 1
+    wl = synth.MISTRAL_1L.with_(batch=batch, **kw)
+    assert 0 < wl.rows - sms <= sms // 2
+    return wl, sms
+
+
+def test_tail_split_rows_match_oracle():
+    """Half rows (two CTAs per row, statistics and output exchanged) against
+    the oracle, across the window's departures."""
+    wl, sms = _tail_workload(prompt_len=1500, budget=600, steps=70)
+    ls = LockStep(wl, [0, sms - 1, sms, sms + 3, wl.rows - 1], engine=2)
+    ls.load_prompt()
+    for s in range(wl.steps):
+        ls.step(check=(s < 3 or s % 16 == 0 or s >= 66))
+
+
+def test_tail_split_step_equals_decode_then_evict():
+    """With half rows, dc_step's in-kernel eviction (candidates exchanged
+    between the halves) leaves the cache bit-identical to dc_decode_step and
+    dc_evict; the output agrees with whole-row CTAs to rounding."""
+    import torch
+    from paper_2608_08878_gb300 import dc
+    wl, _ = _tail_workload(prompt_len=900, budget=400, window=6)
+    a, b = LockStep(wl, [], engine=2), LockStep(wl, [], engine=2)
+    c = LockStep(wl, [], engine=2, tail_split=False)
+    for x in (a, b, c):
+        x.load_prompt()
+    for s in range(10):
+        q, kn, vn = a._inputs(s)
+        oa = a.cache.step(q, kn, vn)
+        ob = b.cache.decode_step(q, kn, vn)
+        b.cache.evict()
+        oc = c.cache.step(q, kn, vn)
+        a.cache.sync()
+        b.cache.sync()
+        c.cache.sync()
+        assert torch.equal(oa, ob), s
+        assert a.cache.length() == b.cache.length()
+        n = a.cache.length()[0]
+        for which in (dc.BUF_K, dc.BUF_V, dc.BUF_POS, dc.BUF_S, dc.BUF_Z, dc.BUF_VNORM):
+            assert torch.equal(a.cache.buffer(which)[:, :n], b.cache.buffer(which)[:, :n]), (s, which)
+        if s == 0:  # before the two caches' evictions could part on near-ties
+            err = float((oa - oc).abs().max())
+            assert err <= 1e-4, err
+
+
 def test_engine_choice():
     from paper_2608_08878_gb300 import dc
     big = dc.DistillCache(32, 8, 128, 200, 100, batch=1)
