@@ -223,9 +223,10 @@ __global__ void __launch_bounds__(kThreads, 1)
     *abort = 0;
     fence_mbar_init();
   }
-  // zero the query and weight tiles (unused rows stay zero), then write the
+  // zero the query, weight and policy-input tiles (unused rows and columns
+  // stay zero), then write the
   // policy layer's B operand (128 rows x 64 bf16, swizzled; 32 columns used)
-  for (int e = threadIdx.x; e < (OFF_A - OFF_Q) / 16; e += kThreads)
+  for (int e = threadIdx.x; e < (OFF_W - OFF_Q) / 16; e += kThreads)
     reinterpret_cast<uint4*>(smem + OFF_Q)[e] = make_uint4(0, 0, 0, 0);
   for (int e = threadIdx.x; e < 128 * 8; e += kThreads) {
     const int row = e >> 3, c = e & 7;
@@ -309,7 +310,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     // ------------------------------------------------------------ MMA issuer
     if (lane == 0) {
       const uint32_t id_qk = idesc_bf16(128, 16, 0, 0);
-      const uint32_t id_pv = idesc_bf16(128, 16, 1, 0);
+      const uint32_t id_pv = idesc_bf16(128, 16, 1, 1);
       int g = 0, gs = 0, gv = 0, gr = 0;
       const int nitems = item_count(fs, p.R);
       for (int k = 0; k < nitems; ++k, ++gr) {
@@ -351,11 +352,9 @@ __global__ void __launch_bounds__(kThreads, 1)
           const uint32_t paddr = smem_u32(smem + OFF_P + pb * 4096);
           // O^T[d x 16] += V^T[d x 128] P^T: V^T is MN-major (dims contiguous)
 #pragma unroll
-          for (int ks = 0; ks < kTok / 16; ++ks) {
-            const uint32_t poff = (uint32_t)(ks >> 2) * 2048u + (uint32_t)(ks & 3) * 32u;
+          for (int ks = 0; ks < kTok / 16; ++ks)
             mma_bf16(tmem + kColO, sdesc_sw128(vaddr + ks * 2048u, 16384, 1024),
-                     sdesc_sw128(paddr + poff, 16, 1024), id_pv, (j > it.t0 || ks > 0) ? 1u : 0u);
-          }
+                     sdesc_sw32(paddr + ks * 512u, 4096, 256), id_pv, (j > it.t0 || ks > 0) ? 1u : 0u);
           mma_commit(&bar[B_PEMPTY + pb]);
           mma_commit(&bar[B_EMPTY + s]);
           if (j == it.t1 - 1) mma_commit(&bar[B_OFULL]);
@@ -469,16 +468,19 @@ __global__ void __launch_bounds__(kThreads, 1)
       g += nTi;
       gs += nTi;
       if constexpr (GS > 0) tmem_st_wait();
-      // ---------------- row softmax statistics (deterministic merge order)
+      // ---------------- row softmax statistics (deterministic merge order):
+      // the maximum first, then every partial (l, u) rescaled to it and summed
 #pragma unroll
       for (int h = 0; h < G; ++h) {
-        float mm = m[h], ll = l[h], uu = u[h];
+        float mm = m[h];
+#pragma unroll
+        for (int off = 16; off > 0; off >>= 1) mm = fmaxf(mm, __shfl_xor_sync(0xffffffffu, mm, off));
+        const float dm = (m[h] - mm) * c, f = ex2(dm);
+        float ll = l[h] * f, uu = (u[h] + l[h] * dm) * f;
 #pragma unroll
         for (int off = 16; off > 0; off >>= 1) {
-          const float mo = __shfl_xor_sync(0xffffffffu, mm, off);
-          const float lo = __shfl_xor_sync(0xffffffffu, ll, off);
-          const float uo = __shfl_xor_sync(0xffffffffu, uu, off);
-          online_merge(mm, ll, uu, mo, lo, uo, c);
+          ll += __shfl_xor_sync(0xffffffffu, ll, off);
+          uu += __shfl_xor_sync(0xffffffffu, uu, off);
         }
         if (lane == 0) {
           red[(ew * G + h) * 3 + 0] = mm;
@@ -490,9 +492,17 @@ __global__ void __launch_bounds__(kThreads, 1)
       float Mm[G], Ll[G], Uu[G];
 #pragma unroll
       for (int h = 0; h < G; ++h) {
-        float mm = kNoMax, ll = 0.f, uu = 0.f;
-        for (int w = 0; w < 8; ++w)
-          online_merge(mm, ll, uu, red[(w * G + h) * 3 + 0], red[(w * G + h) * 3 + 1], red[(w * G + h) * 3 + 2], c);
+        float mm = kNoMax;
+#pragma unroll
+        for (int w = 0; w < 8; ++w) mm = fmaxf(mm, red[(w * G + h) * 3 + 0]);
+        float ll = 0.f, uu = 0.f;
+#pragma unroll
+        for (int w = 0; w < 8; ++w) {
+          const float lw = red[(w * G + h) * 3 + 1];
+          const float dm = (red[(w * G + h) * 3 + 0] - mm) * c, f = ex2(dm);
+          ll = fmaf(lw, f, ll);
+          uu = fmaf(red[(w * G + h) * 3 + 2] + lw * dm, f, uu);
+        }
         Mm[h] = mm; Ll[h] = ll; Uu[h] = uu;
       }
       sync();  // red is rewritten by the next row
@@ -595,21 +605,26 @@ __global__ void __launch_bounds__(kThreads, 1)
           zc += a[h];
           scur = fmaf(a[h], Hh[h], scur);
         }
-        // attention weights as the PV operand (row = query head, column =
-        // token): bf16 high parts in rows [0, G), the residuals in [G, 2G),
-        // so that O = D[:, h] + D[:, G + h] carries ~16 mantissa bits
+        // attention weights as the PV operand, MN-major (one 32-byte row of 16
+        // columns per token, 32-byte swizzle): bf16 high parts in columns
+        // [0, G), the residuals in [G, 2G), so that O = D[:, h] + D[:, G + h]
+        // carries ~16 mantissa bits; columns [8, 16) stay zero
         mbar_wait(&bar[B_PEMPTY + pb], ((gvj >> 1) & 1) ^ 1, abort, p.dbg, 8u, (unsigned)gvj);
         {
-          uint8_t* pt = smem + OFF_P + pb * 4096 + (tok >> 6) * 2048;
-          const int tc = tok & 63;
+          float pw[8];
+#pragma unroll
+          for (int h = 0; h < 8; ++h) pw[h] = 0.f;
 #pragma unroll
           for (int h = 0; h < G; ++h) {
             const float ah = valid ? a[h] : 0.f;
-            const __nv_bfloat16 hv = __float2bfloat16_rn(ah);
-            *reinterpret_cast<__nv_bfloat16*>(pt + sw128(h, tc >> 3) + (tc & 7) * 2) = hv;
-            *reinterpret_cast<__nv_bfloat16*>(pt + sw128(G + h, tc >> 3) + (tc & 7) * 2) =
-                __float2bfloat16_rn(ah - __bfloat162float(hv));
+            const float hv = __bfloat162float(__float2bfloat16_rn(ah));
+            pw[h] = hv;
+            pw[G + h] = ah - hv;
           }
+          const uint4 row = make_uint4(pack_bf16(pw[0], pw[1]), pack_bf16(pw[2], pw[3]), pack_bf16(pw[4], pw[5]),
+                                       pack_bf16(pw[6], pw[7]));
+          *reinterpret_cast<uint4*>(smem + OFF_P + pb * 4096 + (tok >> 3) * 256 + (tok & 7) * 32 +
+                                    (((tok >> 2) & 1) << 4)) = row;
           fence_proxy_async();
           __syncwarp();
           if (lane == 0) mbar_arrive(&bar[B_PFULL + pb]);
@@ -668,17 +683,24 @@ __global__ void __launch_bounds__(kThreads, 1)
         *reinterpret_cast<uint4*>(at + sw128(tok, 0)) = make_uint4(hi[0], hi[1], hi[2], hi[3]);
         *reinterpret_cast<uint4*>(at + sw128(tok, 1)) = make_uint4(lo[0], lo[1], lo[2], lo[3]);
         *reinterpret_cast<uint4*>(at + sw128(tok, 2)) = make_uint4(hi[0], hi[1], hi[2], hi[3]);
-        *reinterpret_cast<uint4*>(at + sw128(tok, 3)) = make_uint4(0, 0, 0, 0);
         fence_proxy_async();
         __syncwarp();
         if (lane == 0) mbar_arrive(&bar[B_AFULL + pb]);
+        // the linear part of the score, sum_j sgn_j z_j, on the CUDA cores
+        float lin = 0.f;
+#pragma unroll
+        for (int e = 0; e < 8; ++e) lin = fmaf(av[e], fp.u[e], lin);
+        return make_float2(lin, __int_as_float(pos));
       };
-      auto finish = [&](int j) {
+      uint32_t ev_key = 0xFFFFFFFFu;
+      int ev_slot = -1, ev_pos = -1;
+      auto finish = [&](int j, float lin, int pos) {
         const int gvj = gv + (j - t0), pb = gvj & 1;
         mbar_wait(&bar[B_MFULL + pb], (gvj >> 1) & 1, abort, p.dbg, 10u, (unsigned)gvj);
         __syncwarp();
         tc_fence_after();
-        // score = b2 + sum_j sgn_j max(z_j, 0); eight independent partial sums
+        // score = b2 + sum_j sgn_j max(z_j, 0) = b2 + (lin + sum_j sgn_j |z_j|) / 2;
+        // eight independent partial sums
         float acc[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
 #pragma unroll
         for (int c8 = 0; c8 < 2; ++c8) {
@@ -688,9 +710,10 @@ __global__ void __launch_bounds__(kThreads, 1)
           tmem_ld_wait();
 #pragma unroll
           for (int e = 0; e < 64; ++e)
-            acc[e & 7] = fmaf(fp.sgn[c8 * 64 + e], fmaxf(z2[e >> 5][e & 31], 0.f), acc[e & 7]);
+            acc[e & 7] = fmaf(fp.sgn[c8 * 64 + e], fabsf(z2[e >> 5][e & 31]), acc[e & 7]);
         }
-        const float relu_sum = ((acc[0] + acc[1]) + (acc[2] + acc[3])) + ((acc[4] + acc[5]) + (acc[6] + acc[7]));
+        const float abs_sum = ((acc[0] + acc[1]) + (acc[2] + acc[3])) + ((acc[4] + acc[5]) + (acc[6] + acc[7]));
+        const float relu_sum = 0.5f * (lin + abs_sum);
         tc_fence_before();
         __syncwarp();
         if (lane == 0) mbar_arrive(&bar[B_MEMPTY + pb]);
@@ -699,12 +722,21 @@ __global__ void __launch_bounds__(kThreads, 1)
           const float score = fp.b2 + relu_sum;
           sc[i] = score;
           if (fs.write_scores) p.score[rbase + i] = score;
+          // this thread's lowest-ranked token so far (lower key, then the later position)
+          const uint32_t kk = score_key(score);
+          if (ev_slot < 0 || kk < ev_key || (kk == ev_key && pos > ev_pos)) {
+            ev_key = kk;
+            ev_slot = i;
+            ev_pos = pos;
+          }
         }
       };
-      if (j0 < t1) prep(j0);
+      // prep(j) returns (the linear score part, the position) for finish(j)
+      float2 pf_cur = j0 < t1 ? prep(j0) : make_float2(0.f, 0.f);
       for (int j = j0; j < t1; j += 2) {
-        if (j + 2 < t1) prep(j + 2);
-        finish(j);
+        const float2 pf_next = j + 2 < t1 ? prep(j + 2) : make_float2(0.f, 0.f);
+        finish(j, pf_cur.x, __float_as_int(pf_cur.y));
+        pf_cur = pf_next;
       }
       g += nTi;
       gv += nTi;
@@ -744,43 +776,39 @@ __global__ void __launch_bounds__(kThreads, 1)
           op[h * D + tok] = half == 0 ? ov[h] + __ldcg(&fs.xo[((size_t)ts * G + h) * D + tok]) : ov[h];
       }
       // ---------------- argtop_B and prune
-      if (fs.do_evict && fs.B < n) {
-        sync();
-        if (half < 0) {
-          team_select_compact<kEpi>(p, r, n, fs.B, sc, etid, scr, sync);
-        } else {
-          // one eviction (B == n - 1): each half finds its lowest-ranked
-          // token, the halves swap candidates, and half 1, which holds the
-          // last slot B, moves it into the evicted slot
-          const int* ps = p.pos + rbase;
-          const int i0 = t0 * kTok, i1 = min(t1 * kTok, n);
-          uint32_t bk = 0xFFFFFFFFu;
-          int bs = -1, bp = -1;
-          for (int i = i0 + etid; i < i1; i += kEpi) {
-            const uint32_t kk = score_key(sc[i]);
-            if (kk < bk || (kk == bk && bs >= 0 && ps[i] > bp)) { bk = kk; bs = i; bp = ps[i]; }
-          }
-          auto lower = [](uint32_t ka, int sa, int pa, uint32_t kb, int sb, int pb) {  // (kb, sb) ranks lower?
-            if (sb < 0) return false;
-            if (sa < 0) return true;
-            return kb < ka || (kb == ka && pb > pa);
-          };
+      if (fs.do_evict && n == fs.B + 1) {
+        // one eviction (the steady state): the lowest-ranked token, from each
+        // thread's running candidate; slot B (the last, held by the whole row
+        // or by half 1) is the only mover and fills the evicted slot. Half
+        // rows swap their candidates first.
+        const bool mover = half != 0;
+        SlotCopy mv{};
+        if (mover && etid < kWarp) mv = slot_load(p, rbase + fs.B, etid);
+        auto lower = [](uint32_t ka, int sa, int pa, uint32_t kb, int sb, int pb) {  // (kb, sb) ranks lower?
+          if (sb < 0) return false;
+          if (sa < 0) return true;
+          return kb < ka || (kb == ka && pb > pa);
+        };
+        uint32_t bk = ev_key;
+        int bs = ev_slot, bp = ev_pos;
 #pragma unroll
-          for (int off = 16; off > 0; off >>= 1) {
-            const uint32_t ok = __shfl_xor_sync(0xffffffffu, bk, off);
-            const int os = __shfl_xor_sync(0xffffffffu, bs, off);
-            const int op = __shfl_xor_sync(0xffffffffu, bp, off);
-            if (lower(bk, bs, bp, ok, os, op)) { bk = ok; bs = os; bp = op; }
-          }
-          if (lane == 0) { s_best[ew] = bk; s_best_slot[ew] = bs; s_hist[ew] = bp; }
-          sync();
-          if (etid == 0) {
-            uint32_t fk = (uint32_t)s_best[0];
-            int fe = s_best_slot[0], fpos = s_hist[0];
-            for (int w = 1; w < kEpi / kWarp; ++w)
-              if (lower(fk, fe, fpos, (uint32_t)s_best[w], s_best_slot[w], s_hist[w])) {
-                fk = (uint32_t)s_best[w]; fe = s_best_slot[w]; fpos = s_hist[w];
-              }
+        for (int off = 16; off > 0; off >>= 1) {
+          const uint32_t ok = __shfl_xor_sync(0xffffffffu, bk, off);
+          const int os = __shfl_xor_sync(0xffffffffu, bs, off);
+          const int op = __shfl_xor_sync(0xffffffffu, bp, off);
+          if (lower(bk, bs, bp, ok, os, op)) { bk = ok; bs = os; bp = op; }
+        }
+        sync();
+        if (lane == 0) { s_best[ew] = bk; s_best_slot[ew] = bs; s_hist[ew] = bp; }
+        sync();
+        if (etid == 0) {
+          uint32_t fk = (uint32_t)s_best[0];
+          int fe = s_best_slot[0], fpos = s_hist[0];
+          for (int w = 1; w < kEpi / kWarp; ++w)
+            if (lower(fk, fe, fpos, (uint32_t)s_best[w], s_best_slot[w], s_hist[w])) {
+              fk = (uint32_t)s_best[w]; fe = s_best_slot[w]; fpos = s_hist[w];
+            }
+          if (half >= 0) {
             int* xs = fs.xsel + (2 * ts + half) * 4;
             xs[0] = (int)fk; xs[1] = fe; xs[2] = fpos;
             __threadfence();
@@ -794,14 +822,17 @@ __global__ void __launch_bounds__(kThreads, 1)
             } else {
               fe = -1;
             }
-            s_sh[0] = fe;
           }
-          sync();
-          const int e = s_sh[0];
-          if (half == 1 && e >= 0 && e < fs.B && etid < kWarp)
-            move_slot(p, rbase + fs.B, rbase + e, etid, kWarp);
-          sync();
+          s_sh[0] = fe;
         }
+        sync();
+        const int e = s_sh[0];
+        if (mover && e >= 0 && e < fs.B && etid < kWarp) slot_store(p, rbase + e, etid, mv);
+        sync();
+      } else if (fs.do_evict && fs.B < n) {
+        // several evictions (whole rows only): radix select over the scores
+        sync();
+        team_select_compact<kEpi>(p, r, n, fs.B, sc, etid, scr, sync);
       }
     }
   }
@@ -970,6 +1001,7 @@ void prepare_policy(const float* blob, int H, int layernorm, FusedPolicy* fp, st
   fp->npos = (int)std::count_if(w2, w2 + H, [](float x) { return x >= 0.f; });
   wtile->assign(128 * 32, __float2bfloat16_rn(0.f));
   for (int jj = 0; jj < 128; ++jj) fp->sgn[jj] = jj < H ? (w2[perm[jj]] >= 0.f ? 1.f : -1.f) : 0.f;
+  double u[8] = {};
   for (int jj = 0; jj < H; ++jj) {
     const double* rj = &rows[(size_t)perm[jj] * 8];
     for (int e = 0; e < 8; ++e) {
@@ -978,8 +1010,10 @@ void prepare_policy(const float* blob, int H, int layernorm, FusedPolicy* fp, st
       (*wtile)[jj * 32 + e] = hi;
       (*wtile)[jj * 32 + 8 + e] = hi;
       (*wtile)[jj * 32 + 16 + e] = lo;
+      u[e] += (double)fp->sgn[jj] * ((double)__bfloat162float(hi) + (double)__bfloat162float(lo));
     }
   }
+  for (int e = 0; e < 8; ++e) fp->u[e] = (float)u[e];
   fp->wtile = nullptr;
 }
 

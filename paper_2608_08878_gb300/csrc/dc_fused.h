@@ -56,6 +56,8 @@ struct FusedPolicy {
   int layernorm;
   const __nv_bfloat16* wtile;    // device [128][32]: rows w_j as bf16 hi | hi | lo | 0
   float sgn[128];                // +1 / -1 per hidden unit, 0 for unused columns
+  float u[8];                    // sum_j sgn_j w_j: the policy input row dotted with
+                                 // it is sum_j sgn_j z_j (relu(z) = (z + |z|) / 2)
 };
 
 // Most tokens per row the fused kernel takes for a query group of G heads.

@@ -93,27 +93,66 @@ __device__ uint32_t team_radix_select(int n, int need, KeyF keyf, Pred pred, int
   return prefix;
 }
 
-// Copies slot `src` of a row to slot `dst` (K, V, position, window state and
-// the per-token extras), using `nl` cooperating lanes starting at lane `l`.
-__device__ __forceinline__ void move_slot(const Dev& p, size_t src, size_t dst, int l, int nl) {
+// One slot's contents held by a warp: lane l keeps 16-byte chunk l of the
+// slot's [K | V] row (d / 4 chunks) and per-token field l: 0 position, 1 |v|,
+// 2 window sums, 3 score, 4 cumulative alpha, 5..9 features. Every lane loads
+// before any stores, so a move costs one memory round trip.
+struct SlotCopy {
+  uint4 kv;
+  uint4 f;
+};
+
+__device__ __forceinline__ SlotCopy slot_load(const Dev& p, size_t src, int lane) {
+  SlotCopy c{};
   const int VPR = p.d / 8;
+  if (lane < VPR) c.kv = reinterpret_cast<const uint4*>(p.K)[src * VPR + lane];
+  else if (lane < 2 * VPR) c.kv = reinterpret_cast<const uint4*>(p.V)[src * VPR + lane - VPR];
+  if (lane == 0) c.f.x = (unsigned)p.pos[src];
+  else if (lane == 1) c.f.x = __float_as_uint(p.vnorm[src]);
+  else if (lane == 2) c.f = *reinterpret_cast<const uint4*>(p.SZ + src);
+  else if (lane == 3) c.f.x = __float_as_uint(p.score[src]);
+  else if (lane == 4 && p.acc) c.f.x = __float_as_uint(p.acc[src]);
+  else if (lane >= 5 && lane < 10 && p.keep_features) c.f.x = __float_as_uint(p.feat[src * 5 + lane - 5]);
+  return c;
+}
+
+__device__ __forceinline__ void slot_store(const Dev& p, size_t dst, int lane, const SlotCopy& c) {
+  const int VPR = p.d / 8;
+  if (lane < VPR) reinterpret_cast<uint4*>(p.K)[dst * VPR + lane] = c.kv;
+  else if (lane < 2 * VPR) reinterpret_cast<uint4*>(p.V)[dst * VPR + lane - VPR] = c.kv;
+  if (lane == 0) p.pos[dst] = (int)c.f.x;
+  else if (lane == 1) p.vnorm[dst] = __uint_as_float(c.f.x);
+  else if (lane == 2) *reinterpret_cast<uint4*>(p.SZ + dst) = c.f;
+  else if (lane == 3) p.score[dst] = __uint_as_float(c.f.x);
+  else if (lane == 4 && p.acc) p.acc[dst] = __uint_as_float(c.f.x);
+  else if (lane >= 5 && lane < 10 && p.keep_features) p.feat[dst * 5 + lane - 5] = __uint_as_float(c.f.x);
+}
+
+// Copies slot `src` of a row to slot `dst` with one thread (loads first).
+__device__ __forceinline__ void move_slot_1(const Dev& p, size_t src, size_t dst) {
+  const int VPR = p.d / 8;
+  const int ps = p.pos[src];
+  const float vn = p.vnorm[src];
+  const float4 sz = p.SZ[src];
+  const float scr = p.score[src];
+  const float ac = p.acc ? p.acc[src] : 0.f;
   const uint4* ks = reinterpret_cast<const uint4*>(p.K) + src * VPR;
   const uint4* vs = reinterpret_cast<const uint4*>(p.V) + src * VPR;
   uint4* kd = reinterpret_cast<uint4*>(p.K) + dst * VPR;
   uint4* vd = reinterpret_cast<uint4*>(p.V) + dst * VPR;
-  for (int e = l; e < 2 * VPR; e += nl) {
-    if (e < VPR) kd[e] = ks[e];
-    else vd[e - VPR] = vs[e - VPR];
+  for (int e = 0; e < VPR; e += 4) {
+    const uint4 k0 = ks[e], k1 = ks[e + 1], k2 = ks[e + 2], k3 = ks[e + 3];
+    const uint4 v0 = vs[e], v1 = vs[e + 1], v2 = vs[e + 2], v3 = vs[e + 3];
+    kd[e] = k0; kd[e + 1] = k1; kd[e + 2] = k2; kd[e + 3] = k3;
+    vd[e] = v0; vd[e + 1] = v1; vd[e + 2] = v2; vd[e + 3] = v3;
   }
-  if (l == 0) {
-    p.pos[dst] = p.pos[src];
-    p.vnorm[dst] = p.vnorm[src];
-    p.SZ[dst] = p.SZ[src];
-    p.score[dst] = p.score[src];
-    if (p.acc) p.acc[dst] = p.acc[src];
-    if (p.keep_features)
-      for (int e = 0; e < 5; ++e) p.feat[dst * 5 + e] = p.feat[src * 5 + e];
-  }
+  p.pos[dst] = ps;
+  p.vnorm[dst] = vn;
+  p.SZ[dst] = sz;
+  p.score[dst] = scr;
+  if (p.acc) p.acc[dst] = ac;
+  if (p.keep_features)
+    for (int e = 0; e < 5; ++e) p.feat[dst * 5 + e] = p.feat[src * 5 + e];
 }
 
 // Keeps the top B of the row's n tokens (scores from `score`, length n) and
@@ -128,11 +167,14 @@ __device__ void team_select_compact(const Dev& p, int r, int n, int B, const flo
   if (n == B + 1) {
     // One eviction: the lowest-ranked token (smallest score key; among equal
     // keys the highest position). Positions are read only to break ties.
+    // Slot B (the last) is the only candidate mover: load it meanwhile.
+    SlotCopy mv{};
+    if (tid < kWarp) mv = slot_load(p, base + B, tid);
     uint32_t bk = 0xFFFFFFFFu;
     int bs = -1;
     for (int i = tid; i < n; i += NT) {
       const uint32_t k = key(i);
-      if (k < bk || (k == bk && bs >= 0 && ps[i] > ps[bs])) { bk = k; bs = i; }
+      if (bs < 0 || k < bk || (k == bk && ps[i] > ps[bs])) { bk = k; bs = i; }
     }
     auto better = [&](uint32_t ka, int sa, uint32_t kb, int sb) {  // (kb, sb) ranks lower?
       if (sb < 0) return false;
@@ -152,8 +194,8 @@ __device__ void team_select_compact(const Dev& p, int r, int n, int B, const flo
     int e = s.best_slot[0];
     for (int w = 1; w < NT / kWarp; ++w)
       if (better(fk, e, (uint32_t)s.best[w], s.best_slot[w])) { fk = (uint32_t)s.best[w]; e = s.best_slot[w]; }
-    // slot B (the last) is the only candidate mover; it fills the hole at e
-    if (e >= 0 && e < B && tid < kWarp) move_slot(p, base + B, base + e, tid, kWarp);
+    // slot B fills the hole at e
+    if (e >= 0 && e < B && tid < kWarp) slot_store(p, base + e, tid, mv);
     sync();
     return;
   }
@@ -193,7 +235,7 @@ __device__ void team_select_compact(const Dev& p, int r, int n, int B, const flo
     const int f = (i < n && keep(i)) ? 1 : 0;
     int tot;
     const int rank = team_exclusive_scan<NT>(f, tid, s.wsum, &tot, sync);
-    if (f && nm + rank < nh) move_slot(p, base + i, base + holes[nm + rank], 0, 1);
+    if (f && nm + rank < nh) move_slot_1(p, base + i, base + holes[nm + rank]);
     nm += tot;
   }
   if (tid == 0 && nm != nh) atomicOr(p.status, kStatusBadShape);

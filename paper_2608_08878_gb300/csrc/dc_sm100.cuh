@@ -234,14 +234,26 @@ __host__ __device__ constexpr uint32_t idesc_bf16(int M, int N, int a_mn, int b_
 
 // Shared-memory matrix descriptor, 128-byte swizzle: start address, leading
 // and stride byte offsets (all in bytes, encoded >> 4).
-__device__ __forceinline__ uint64_t sdesc_sw128(uint32_t saddr, uint32_t lbo, uint32_t sbo) {
+// Swizzle modes (bits 61..63): 2 = 128-byte, 4 = 64-byte, 6 = 32-byte. For a
+// K-major operand the stride offset steps between 8-row groups; for an
+// MN-major one the leading offset steps between swizzle atoms along M/N and
+// the stride offset between 8-row groups along K.
+__device__ __forceinline__ uint64_t sdesc(uint32_t saddr, uint32_t lbo, uint32_t sbo, uint32_t mode) {
   uint64_t d = 0;
   d |= (uint64_t)((saddr >> 4) & 0x3FFF);
   d |= (uint64_t)((lbo >> 4) & 0x3FFF) << 16;
   d |= (uint64_t)((sbo >> 4) & 0x3FFF) << 32;
   d |= (uint64_t)1 << 46;  // descriptor version
-  d |= (uint64_t)2 << 61;  // 128-byte swizzle
+  d |= (uint64_t)(mode & 7) << 61;
   return d;
+}
+
+__device__ __forceinline__ uint64_t sdesc_sw128(uint32_t saddr, uint32_t lbo, uint32_t sbo) {
+  return sdesc(saddr, lbo, sbo, 2);
+}
+
+__device__ __forceinline__ uint64_t sdesc_sw32(uint32_t saddr, uint32_t lbo, uint32_t sbo) {
+  return sdesc(saddr, lbo, sbo, 6);
 }
 
 // TMEM loads/stores, 32 lanes x N columns of 32-bit, this warp's lane quarter.
