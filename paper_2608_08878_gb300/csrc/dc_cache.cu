@@ -57,7 +57,8 @@ struct dc_cache {
   dc::FusedMaps maps{};
   dc::FusedPolicy fpol{};
   __nv_bfloat16* wtile = nullptr;
-  // exchange buffers of the half rows (FusedStep::split_tail)
+  // queue counters and exchange buffers of the half rows (FusedStep)
+  unsigned* work = nullptr;
   float* xstats = nullptr;
   float* xo = nullptr;
   int* xsel = nullptr;
@@ -349,6 +350,8 @@ dc_status dc_cache_create(int layers, int kv_heads, int head_dim, int capacity, 
     cudaError_t fe = dalloc(h, &h->wtile, 128 * 32 * sizeof(__nv_bfloat16));
     if (fe == cudaSuccess) fe = dc::make_fused_maps(p, &h->maps, &why);
     if (fe == cudaSuccess) fe = upload_fused_policy(h, w.data());
+    if (fe == cudaSuccess) fe = dalloc(h, &h->work, 2 * sizeof(unsigned));
+    if (fe == cudaSuccess) fe = cudaMemsetAsync(h->work, 0, 2 * sizeof(unsigned), h->stream);
     if (fe == cudaSuccess && cfg.tail_split) {
       const int grid = (int)std::min<long long>(R, h->num_sms);
       fe = dalloc(h, &h->xstats, dc::fused_xstats_len(grid, G) * sizeof(float));
@@ -435,12 +438,11 @@ dc::FusedStep fused_args(dc_cache* h, const dc::Step& st, const void* q, float* 
   fs.xo = h->xo;
   fs.xsel = h->xsel;
   fs.xflag = h->xflag;
-  if (h->xflag && dc::fused_can_split_tail(h->dev, st.n, fs, h->num_sms)) {
-    fs.split_tail = 1;
-    // flags hold epoch * 4 + phase; skip 0 so that a zeroed flag never matches
-    if (++h->epoch == 0) ++h->epoch;
-    fs.epoch = h->epoch;
-  }
+  fs.work = h->work;
+  fs.half_rows = h->xflag ? dc::fused_half_rows(h->dev, st.n, fs, h->num_sms) : 0;
+  // launch epoch: the queue counter is work[epoch & 1]; exchange flags hold
+  // epoch * 4 + phase (1..3), so a flag left by an earlier launch never matches
+  fs.epoch = ++h->epoch;
   return fs;
 }
 
@@ -452,7 +454,7 @@ bool tail_split_applies(dc_cache* h, int n) {
   fs.xo = h->xo;
   fs.xsel = h->xsel;
   fs.xflag = h->xflag;
-  return dc::fused_can_split_tail(h->dev, n, fs, h->num_sms);
+  return dc::fused_half_rows(h->dev, n, fs, h->num_sms) > 0;
 }
 
 }  // namespace

@@ -4,12 +4,13 @@
 // statistics), the five token features of Sec. 3.1.1, the policy MLP of
 // Sec. 3.1.2 / App. D, and (dc_step) the top-B select and compaction.
 //
-// One CTA per SM; each CTA takes rows r = blockIdx.x, blockIdx.x + gridDim.x...
+// One CTA per SM; the CTAs take rows (and, for a partly filled last wave,
+// half rows) from a shared queue as they become free.
 // Warp roles (352 threads):
-//   warp 0     producer: writes the row's query tile (current, previous and
-//              departing queries) and streams K then V tiles of 128 tokens
-//              with TMA (128-byte swizzle) through a 3-stage ring, each tile
-//              with its tokens' state (positions, window sums or |v|);
+//   warp 0     producer: takes the next row, writes its query tile (current,
+//              previous and departing queries) and streams K then V tiles of
+//              128 tokens with TMA (128-byte swizzle) through a 4-stage ring,
+//              K tiles with their tokens' positions and window sums;
 //   warp 1     MMA issuer (one lane): tcgen05.mma, accumulators in TMEM:
 //                S  = K Q^T        [128 tokens x 16]  per K tile
 //                O^T += V^T P^T    [d x 16]           per V tile (P = weights,
@@ -53,13 +54,14 @@ using namespace sm100;
 
 namespace {
 
-constexpr int kStages = 3;
-// stage: K or V tile (32 KB, two 64-dim column blocks); K tiles also bring the
-// tile's positions (512 B) and window sums (2 KB)
-constexpr int kTileRegion = 32768;
-constexpr int kOffPos = kTileRegion;          // int32 [128] (K tiles)
-constexpr int kOffSZ = kTileRegion + 1024;    // fp32x4 [128] (K tiles)
-constexpr int kStageBytes = kTileRegion + 3072;  // a multiple of 1024 (swizzle atoms)
+constexpr int kStages = 4;
+// stage: K or V tile (32 KB, two 64-dim column blocks, 1024-byte aligned);
+// K tiles also bring the tile's positions (512 B) and window sums (2 KB) into
+// the stage's slot of the per-token area
+constexpr int kStageBytes = 32768;
+constexpr int kAuxBytes = 2560;
+constexpr int kAuxPos = 0;                    // int32 [128] (K tiles)
+constexpr int kAuxSZ = 512;                   // fp32x4 [128] (K tiles)
 constexpr int kTok = 128;
 constexpr int kThreads = 352;
 constexpr int kEpi = 256;                     // two warpgroups
@@ -70,18 +72,21 @@ constexpr int kStashA = 48, kStashAEnd = 128, kStashB = 384, kStashBEnd = 512;
 constexpr int OFF_STAGE = 0;
 constexpr int OFF_Q = OFF_STAGE + kStages * kStageBytes;  // 2 x 4 KB
 constexpr int OFF_P = OFF_Q + 2 * 4096;                    // 2 x 4 KB (one per warpgroup)
-constexpr int OFF_A = OFF_P + 2 * 4096;                    // 2 x 16 KB (one per warpgroup)
-constexpr int OFF_W = OFF_A + 2 * 16384;                   // 16 KB
-constexpr int OFF_SC = OFF_W + 16384;                      // head G-1 logits, then scores
+constexpr int OFF_A = OFF_P + 2 * 4096;                    // 2 x 8 KB (one per warpgroup)
+constexpr int OFF_W = OFF_A + 2 * 8192;                    // 8 KB
+constexpr int OFF_AUX = OFF_W + 8192;                      // kStages x 2560 B
+constexpr int OFF_SC = OFF_AUX + kStages * kAuxBytes;      // head G-1 logits, then scores
 constexpr int OFF_MISC = OFF_SC + kFusedMaxTok * 4;
 constexpr int MISC_BYTES = 4096;
 constexpr int kSmemBytes = OFF_MISC + MISC_BYTES + 1024;   // + alignment slack
+static_assert(kSmemBytes <= 232448, "more shared memory than a CTA may have");
 
 // barrier indices in the misc area
 enum {
-  B_FULL = 0, B_EMPTY = 3, B_QFULL = 6, B_QEMPTY = 8, B_SFULL = 10, B_SEMPTY = 12, B_PFULL = 14,
-  B_PEMPTY = 16, B_MFULL = 18, B_MEMPTY = 20, B_AFULL = 22, B_AEMPTY = 24, B_OFULL = 26, B_OEMPTY = 27,
-  B_DRAIN = 28, B_DRAIN2 = 29, B_COUNT = 30
+  B_FULL = 0, B_EMPTY = kStages, B_QFULL = 2 * kStages, B_QEMPTY = B_QFULL + 2, B_SFULL = B_QFULL + 4,
+  B_SEMPTY = B_QFULL + 6, B_PFULL = B_QFULL + 8, B_PEMPTY = B_QFULL + 10, B_MFULL = B_QFULL + 12,
+  B_MEMPTY = B_QFULL + 14, B_AFULL = B_QFULL + 16, B_AEMPTY = B_QFULL + 18, B_OFULL = B_QFULL + 20,
+  B_OEMPTY = B_QFULL + 21, B_DRAIN = B_QFULL + 22, B_DRAIN2 = B_QFULL + 23, B_COUNT = B_QFULL + 24
 };
 
 // TMEM column of the stashed logits of tile j (GS = G - 1 columns per tile).
@@ -95,6 +100,12 @@ __device__ __forceinline__ uint32_t stash_col(int j) {
 // swizzled tile (8-row atoms of 1024 bytes)
 __device__ __forceinline__ uint32_t sw128(int row, int c) {
   return (uint32_t)((row >> 3) * 1024 + (row & 7) * 128 + ((c ^ (row & 7)) << 4));
+}
+
+// byte offset of 16-byte chunk `c` (0..3) of row `row` inside a 64-byte
+// swizzled tile (8-row atoms of 512 bytes)
+__device__ __forceinline__ uint32_t sw64(int row, int c) {
+  return (uint32_t)((row >> 3) * 512 + (row & 7) * 64 + ((c ^ ((row & 7) >> 1)) << 4));
 }
 
 __device__ __forceinline__ uint32_t pack_bf16(float a, float b) {
@@ -158,23 +169,56 @@ __device__ __forceinline__ void online_merge(float& m, float& l, float& u, float
   m = M;
 }
 
-// Work items of a CTA: whole rows r = blockIdx.x + k * gridDim.x, and with a
-// split tail, half of one row of the last wave (half 0: the first ceil(nT/2)
-// tiles, half 1: the rest).
+// Work items come from a queue shared by all CTAs (an atomic counter): the
+// first R - half_rows rows whole, then both halves of each of the last
+// half_rows rows (half 0: the first ceil(nT/2) tiles, half 1: the rest). A CTA
+// that takes a half row takes nothing after it, so the halves of a row always
+// go to two different CTAs, which then wait on each other (all CTAs are
+// resident under a cooperative launch). Taking rows as CTAs become free keeps
+// their finishing times together however their speeds drift.
 struct Item {
-  int row, t0, t1, half;  // half -1: the whole row
+  int row, t0, t1, half;  // row -1: no more work; half -1: the whole row
 };
 
-__device__ __forceinline__ int item_count(const FusedStep& fs, int R) {
-  const int W = gridDim.x, c = blockIdx.x, full = R / W, rem = R % W;
-  return full + (fs.split_tail ? (c < 2 * rem ? 1 : 0) : (c < rem ? 1 : 0));
+constexpr int kItemRing = 8;  // items published ahead of the slowest role (at most ~3)
+
+__device__ __forceinline__ Item take_item(const FusedStep& fs, int R, int nT) {
+  const unsigned whole = (unsigned)(R - fs.half_rows);
+  const unsigned w = atomicAdd(fs.work + (fs.epoch & 1u), 1u);
+  if (w < whole) return Item{(int)w, 0, nT, -1};
+  const unsigned k = w - whole;
+  if (k >= 2u * (unsigned)fs.half_rows) return Item{-1, 0, 0, 0};
+  const int mid = (nT + 1) >> 1, h = (int)(k & 1u);
+  return Item{(int)(whole + (k >> 1)), h ? mid : 0, h ? nT : mid, h};
 }
 
-__device__ __forceinline__ Item item_at(const FusedStep& fs, int R, int nT, int k) {
-  const int W = gridDim.x, c = blockIdx.x, full = R / W;
-  if (k < full || !fs.split_tail) return Item{c + k * W, 0, nT, -1};
-  const int mid = (nT + 1) >> 1, h = c & 1;
-  return Item{full * W + (c >> 1), h ? mid : 0, h ? nT : mid, h};
+// Producer: item `gr` into the shared ring for the other roles.
+__device__ __forceinline__ void publish_item(volatile int* ring, int gr, const Item& it) {
+  volatile int* e = ring + (gr % kItemRing) * 4;
+  e[0] = it.row;
+  e[1] = it.t0;
+  e[2] = it.t1;
+  e[3] = it.half;
+  __threadfence_block();
+  ring[4 * kItemRing + gr % kItemRing] = gr + 1;  // sequence number
+}
+
+// One thread: item `gr` once published; row -1 when the kernel winds down.
+__device__ __forceinline__ Item read_item(volatile int* ring, int gr, volatile int* abort, unsigned* dbg,
+                                          unsigned site) {
+  const uint64_t t0 = globaltimer_ns();
+  for (uint32_t i = 0;; ++i) {
+    if (ring[4 * kItemRing + gr % kItemRing] == gr + 1) break;
+    if (*abort) return Item{-1, 0, 0, 0};
+    if ((i & 255u) == 255u && globaltimer_ns() - t0 > kWaitNs) {
+      record_timeout(dbg, site, (unsigned)gr, 0u);
+      *abort = 1;
+      return Item{-1, 0, 0, 0};
+    }
+  }
+  __threadfence_block();
+  volatile int* e = ring + (gr % kItemRing) * 4;
+  return Item{e[0], e[1], e[2], e[3]};
 }
 
 template <int D, int G>
@@ -185,15 +229,17 @@ __global__ void __launch_bounds__(kThreads, 1)
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint64_t* bar = reinterpret_cast<uint64_t*>(smem + OFF_MISC);
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + OFF_MISC + 8 * B_COUNT);
-  volatile int* abort = reinterpret_cast<volatile int*>(smem + OFF_MISC + 8 * B_COUNT + 4);
-  float* red = reinterpret_cast<float*>(smem + OFF_MISC + 256);            // [8][G][3]
+  static_assert(8 * B_COUNT <= 384, "barriers overlap the misc fields");
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + OFF_MISC + 384);
+  volatile int* abort = reinterpret_cast<volatile int*>(smem + OFF_MISC + 388);
+  float* red = reinterpret_cast<float*>(smem + OFF_MISC + 512);            // [8][G][3]
   int* s_hist = reinterpret_cast<int*>(smem + OFF_MISC + 1024);           // [256]
   int* s_sh = reinterpret_cast<int*>(smem + OFF_MISC + 2048);             // [4]
   int* s_wsum = reinterpret_cast<int*>(smem + OFF_MISC + 2064);           // [8]
   unsigned long long* s_best = reinterpret_cast<unsigned long long*>(smem + OFF_MISC + 2112);  // [8]
   int* s_best_slot = reinterpret_cast<int*>(smem + OFF_MISC + 2176);      // [8]
   float* sc = reinterpret_cast<float*>(smem + OFF_SC);
+  volatile int* items = reinterpret_cast<volatile int*>(smem + OFF_MISC + 2304);  // [8][4] + seq [8]
 
   const int warp = threadIdx.x / kWarp, lane = threadIdx.x % kWarp;
   const int n = st.n, nT = (n + kTok - 1) / kTok;
@@ -221,18 +267,19 @@ __global__ void __launch_bounds__(kThreads, 1)
     mbar_init(&bar[B_DRAIN], 1);
     mbar_init(&bar[B_DRAIN2], 1);
     *abort = 0;
+    for (int e = 0; e < kItemRing; ++e) items[4 * kItemRing + e] = 0;
+    // the next launch's queue counter (this launch uses the other one)
+    if (blockIdx.x == 0) fs.work[(fs.epoch + 1u) & 1u] = 0u;
     fence_mbar_init();
   }
   // zero the query, weight and policy-input tiles (unused rows and columns
-  // stay zero), then write the
-  // policy layer's B operand (128 rows x 64 bf16, swizzled; 32 columns used)
+  // stay zero), then write the policy layer's B operand (128 rows x 32 bf16,
+  // 64-byte swizzle)
   for (int e = threadIdx.x; e < (OFF_W - OFF_Q) / 16; e += kThreads)
     reinterpret_cast<uint4*>(smem + OFF_Q)[e] = make_uint4(0, 0, 0, 0);
-  for (int e = threadIdx.x; e < 128 * 8; e += kThreads) {
-    const int row = e >> 3, c = e & 7;
-    uint4 v = make_uint4(0, 0, 0, 0);
-    if (c < 4) v = reinterpret_cast<const uint4*>(fp.wtile)[row * 4 + c];
-    *reinterpret_cast<uint4*>(smem + OFF_W + sw128(row, c)) = v;
+  for (int e = threadIdx.x; e < 128 * 4; e += kThreads) {
+    const int row = e >> 2, c = e & 3;
+    *reinterpret_cast<uint4*>(smem + OFF_W + sw64(row, c)) = reinterpret_cast<const uint4*>(fp.wtile)[row * 4 + c];
   }
   fence_proxy_async();
   if (warp == 1) {
@@ -250,14 +297,27 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (warp == 0) {
     // ------------------------------------------------------------ producer
     const uint64_t pol = l2_evict_first_policy();
-    int g = 0, gr = 0, issued = 0;
-    const int nitems = item_count(fs, p.R);
-    for (int k = 0; k < nitems; ++k, ++gr) {
+    int g = 0, issued = 0;
+    bool last = false;  // a half row was taken: nothing more
+    for (int gr = 0;; ++gr) {
       if (*abort) break;
-      const Item it = item_at(fs, p.R, nT, k);
-      const int r = it.row;
       const int qb = gr & 1;
       if (!mbar_wait(&bar[B_QEMPTY + qb], ((gr >> 1) & 1) ^ 1, abort, p.dbg, 1u, (unsigned)gr)) break;
+      // the next item, taken once this CTA's query buffer is free
+      int4 iv = make_int4(-1, 0, 0, 0);
+      if (lane == 0) {
+        const Item t = last ? Item{-1, 0, 0, 0} : take_item(fs, p.R, nT);
+        publish_item(items, gr, t);
+        iv = make_int4(t.row, t.t0, t.t1, t.half);
+      }
+      iv.x = __shfl_sync(0xffffffffu, iv.x, 0);
+      iv.y = __shfl_sync(0xffffffffu, iv.y, 0);
+      iv.z = __shfl_sync(0xffffffffu, iv.z, 0);
+      iv.w = __shfl_sync(0xffffffffu, iv.w, 0);
+      const Item it{iv.x, iv.y, iv.z, iv.w};
+      if (it.row < 0) break;
+      last = it.half >= 0;
+      const int r = it.row;
       // query tile: rows [0,G) current, [G,2G) previous step, [2G,3G) departing
       uint8_t* qt = smem + OFF_Q + qb * 4096;
       const int qo = ((r / p.kvh) * p.qh + (r % p.kvh) * G) * D;
@@ -287,12 +347,13 @@ __global__ void __launch_bounds__(kThreads, 1)
             if (!mbar_wait(&bar[B_EMPTY + s], ((g / kStages) & 1) ^ 1, abort, p.dbg, 2u, (unsigned)g)) break;
             mbar_expect_tx(&bar[B_FULL + s], kTileBytes + (pass ? 0u : 2560u));
             uint8_t* dst = smem + OFF_STAGE + s * kStageBytes;
+            uint8_t* aux = smem + OFF_AUX + s * kAuxBytes;
             const int y = r * p.stride + j * kTok;
             tma_load_2d(dst, tm, 0, y, &bar[B_FULL + s], pol);
             if (D == 128) tma_load_2d(dst + 16384, tm, 64, y, &bar[B_FULL + s], pol);
             if (!pass) {
-              bulk_load(dst + kOffPos, p.pos + y, 512, &bar[B_FULL + s]);
-              bulk_load(dst + kOffSZ, p.SZ + y, 2048, &bar[B_FULL + s]);
+              bulk_load(aux + kAuxPos, p.pos + y, 512, &bar[B_FULL + s]);
+              bulk_load(aux + kAuxSZ, p.SZ + y, 2048, &bar[B_FULL + s]);
             }
             issued = g + 1;
           }
@@ -311,11 +372,10 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (lane == 0) {
       const uint32_t id_qk = idesc_bf16(128, 16, 0, 0);
       const uint32_t id_pv = idesc_bf16(128, 16, 1, 1);
-      int g = 0, gs = 0, gv = 0, gr = 0;
-      const int nitems = item_count(fs, p.R);
-      for (int k = 0; k < nitems; ++k, ++gr) {
-        if (*abort) break;
-        const Item it = item_at(fs, p.R, nT, k);
+      int g = 0, gs = 0, gv = 0;
+      for (int gr = 0;; ++gr) {
+        const Item it = read_item(items, gr, abort, p.dbg, 23u);
+        if (it.row < 0) break;
         const int qb = gr & 1;
         if (!mbar_wait(&bar[B_QFULL + qb], (gr >> 1) & 1, abort, p.dbg, 3u, (unsigned)gr)) break;
         tc_fence_after();
@@ -371,21 +431,20 @@ __global__ void __launch_bounds__(kThreads, 1)
       const uint32_t id_m = idesc_bf16(128, 128, 0, 0);
       const uint32_t waddr = smem_u32(smem + OFF_W);
       int gv = 0;
-      const int nitems = item_count(fs, p.R);
-      for (int k = 0; k < nitems; ++k) {
-        if (*abort) break;
-        const Item it = item_at(fs, p.R, nT, k);
+      for (int gr = 0;; ++gr) {
+        const Item it = read_item(items, gr, abort, p.dbg, 24u);
+        if (it.row < 0) break;
         for (int j = it.t0; j < it.t1; ++j, ++gv) {
           const int pb = gv & 1;
           if (!mbar_wait(&bar[B_AFULL + pb], (gv >> 1) & 1, abort, p.dbg, 16u, (unsigned)gv)) break;
           if (!mbar_wait(&bar[B_MEMPTY + pb], ((gv >> 1) & 1) ^ 1, abort, p.dbg, 17u, (unsigned)gv)) break;
           tc_fence_after();
-          const uint32_t aaddr = smem_u32(smem + OFF_A + pb * 16384);
+          const uint32_t aaddr = smem_u32(smem + OFF_A + pb * 8192);
           // Z[128 x 128] = A[128 x 32] W^T
 #pragma unroll
           for (int ks = 0; ks < 2; ++ks)
-            mma_bf16(tmem + kColM + pb * 128, sdesc_sw128(aaddr + ks * 32u, 16, 1024),
-                     sdesc_sw128(waddr + ks * 32u, 16, 1024), id_m, ks > 0);
+            mma_bf16(tmem + kColM + pb * 128, sdesc_sw64(aaddr + ks * 32u, 16, 512),
+                     sdesc_sw64(waddr + ks * 32u, 16, 512), id_m, ks > 0);
           mma_commit(&bar[B_MFULL + pb]);
           mma_commit(&bar[B_AEMPTY + pb]);
         }
@@ -405,13 +464,21 @@ __global__ void __launch_bounds__(kThreads, 1)
     const float c = p.c;
     auto sync = [] { named_bar(1, kEpi); };
     const SelectScratch scr{s_hist, s_sh, s_wsum, s_best, s_best_slot};
-    int g = 0, gs = 0, gv = 0, gr = 0;
-    const int nitems = item_count(fs, p.R);
-    for (int k = 0; k < nitems; ++k, ++gr) {
-      if (named_bar_or(1, kEpi, *abort != 0)) break;
-      const Item it = item_at(fs, p.R, nT, k);
+    int g = 0, gs = 0, gv = 0;
+    for (int gr = 0;; ++gr) {
+      int4 iv = make_int4(-1, 0, 0, 0);
+      if (lane == 0) {
+        const Item t = read_item(items, gr, abort, p.dbg, 25u);
+        iv = make_int4(t.row, t.t0, t.t1, t.half);
+      }
+      iv.x = __shfl_sync(0xffffffffu, iv.x, 0);
+      iv.y = __shfl_sync(0xffffffffu, iv.y, 0);
+      iv.z = __shfl_sync(0xffffffffu, iv.z, 0);
+      iv.w = __shfl_sync(0xffffffffu, iv.w, 0);
+      if (named_bar_or(1, kEpi, *abort != 0 || iv.x < 0)) break;
+      const Item it{iv.x, iv.y, iv.z, iv.w};
       const int r = it.row, t0 = it.t0, t1 = it.t1, nTi = it.t1 - it.t0;
-      const int ts = r - (p.R / gridDim.x) * gridDim.x;  // tail slot (half rows only)
+      const int ts = r - (p.R - fs.half_rows);  // exchange slot (half rows only)
       const size_t rbase = (size_t)r * p.stride;
       float pm[G], pnl[G], pH[G], dm[G], dnl[G], dH[G];
 #pragma unroll
@@ -436,9 +503,9 @@ __global__ void __launch_bounds__(kThreads, 1)
         float S16[16];
         tmem_ld16(lane_addr + kColS + b * 16, S16);
         tmem_ld_wait();
-        const uint8_t* stg = smem + OFF_STAGE + s * kStageBytes;
-        const int pos = reinterpret_cast<const int*>(stg + kOffPos)[tok];
-        float4 sz = reinterpret_cast<const float4*>(stg + kOffSZ)[tok];
+        const uint8_t* aux = smem + OFF_AUX + s * kAuxBytes;
+        const int pos = reinterpret_cast<const int*>(aux + kAuxPos)[tok];
+        float4 sz = reinterpret_cast<const float4*>(aux + kAuxSZ)[tok];
         tc_fence_before();
         __syncwarp();
         if (lane == 0) {
@@ -679,10 +746,10 @@ __global__ void __launch_bounds__(kThreads, 1)
           lo[e] = pack_bf16(r0, r1);
         }
         mbar_wait(&bar[B_AEMPTY + pb], ((gvj >> 1) & 1) ^ 1, abort, p.dbg, 9u, (unsigned)gvj);
-        uint8_t* at = smem + OFF_A + pb * 16384;
-        *reinterpret_cast<uint4*>(at + sw128(tok, 0)) = make_uint4(hi[0], hi[1], hi[2], hi[3]);
-        *reinterpret_cast<uint4*>(at + sw128(tok, 1)) = make_uint4(lo[0], lo[1], lo[2], lo[3]);
-        *reinterpret_cast<uint4*>(at + sw128(tok, 2)) = make_uint4(hi[0], hi[1], hi[2], hi[3]);
+        uint8_t* at = smem + OFF_A + pb * 8192;
+        *reinterpret_cast<uint4*>(at + sw64(tok, 0)) = make_uint4(hi[0], hi[1], hi[2], hi[3]);
+        *reinterpret_cast<uint4*>(at + sw64(tok, 1)) = make_uint4(lo[0], lo[1], lo[2], lo[3]);
+        *reinterpret_cast<uint4*>(at + sw64(tok, 2)) = make_uint4(hi[0], hi[1], hi[2], hi[3]);
         fence_proxy_async();
         __syncwarp();
         if (lane == 0) mbar_arrive(&bar[B_AFULL + pb]);
@@ -869,7 +936,7 @@ static cudaError_t launch_t(const FusedMaps& maps, const Dev& p, const Step& st,
     if (e != cudaSuccess) return e;
     attr = true;
   }
-  if (!fs.split_tail) {
+  if (fs.half_rows == 0) {
     fused_kernel<D, G><<<grid, kThreads, kSmemBytes, s>>>(maps.k, maps.v, p, st, fs, fp);
     return cudaGetLastError();
   }
@@ -890,11 +957,12 @@ static cudaError_t launch_t(const FusedMaps& maps, const Dev& p, const Step& st,
 
 static int fused_grid(const Dev& p, int num_sms) { return p.R < num_sms ? p.R : num_sms; }
 
-bool fused_can_split_tail(const Dev& p, int n, const FusedStep& fs, int num_sms) {
+int fused_half_rows(const Dev& p, int n, const FusedStep& fs, int num_sms) {
   const int grid = fused_grid(p, num_sms), rem = p.R % grid;
   const int nT = (n + kTok - 1) / kTok;
-  return fs.xflag && fs.xstats && fs.xo && fs.xsel && rem > 0 && 2 * rem <= grid && nT >= 2 &&
-         (!fs.do_evict || fs.B >= n || fs.B == n - 1);
+  const bool ok = fs.xflag && fs.xstats && fs.xo && fs.xsel && rem > 0 && 2 * rem <= grid && nT >= 2 &&
+                  (!fs.do_evict || fs.B >= n || fs.B == n - 1);
+  return ok ? rem : 0;
 }
 
 cudaError_t launch_fused_step(const FusedMaps& maps, const Dev& p, const Step& st, const FusedStep& fs,

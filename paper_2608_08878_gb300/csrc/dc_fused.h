@@ -26,16 +26,18 @@ struct FusedStep {
   int do_evict;      // 1: select and compact in the same kernel
   int B;             // tokens to keep when do_evict
   int write_scores;  // 1: also store scores in Dev::score (for dc_evict)
-  // Tail split: the R % grid rows of the last wave are each taken by two CTAs
-  // (halves of the row's tiles) that exchange softmax statistics, the output
-  // and the eviction candidate through global memory. Needs a cooperative
-  // launch (all CTAs resident) and, with do_evict, exactly one eviction.
-  int split_tail;
-  unsigned epoch;    // increases every launch; exchange flags compare against it
-  float* xstats;     // [grid/2][2][G][4]
-  float* xo;         // [grid/2][G][d]
-  int* xsel;         // [grid/2][2][4]
-  unsigned* xflag;   // [grid/2][2]
+  // Rows are taken from a queue (an atomic counter) as CTAs become free. With
+  // half_rows > 0 the last half_rows rows are each taken as two halves by two
+  // CTAs, which exchange softmax statistics, the output and the eviction
+  // candidate through global memory. Needs a cooperative launch (all CTAs
+  // resident), 2 * half_rows <= grid and, with do_evict, one eviction per row.
+  int half_rows;
+  unsigned epoch;    // increases every launch; queue and exchange flags key on it
+  unsigned* work;    // [2] queue counters, used by alternate launches
+  float* xstats;     // [half_rows][2][G][4]
+  float* xo;         // [half_rows][G][d]
+  int* xsel;         // [half_rows][2][4]
+  unsigned* xflag;   // [half_rows][2]
 };
 
 // Exchange buffer sizes (floats / ints) for a grid of `grid` CTAs.
@@ -72,8 +74,9 @@ cudaError_t make_fused_maps(const Dev& p, FusedMaps* maps, const char** why);
 // FusedPolicy fields and the host copy of the weight tile (128 * 32 bf16).
 void prepare_policy(const float* blob, int H, int layernorm, FusedPolicy* fp, std::vector<__nv_bfloat16>* wtile);
 
-// Whether the step can split its last wave's rows (see FusedStep).
-bool fused_can_split_tail(const Dev& p, int n, const FusedStep& fs, int num_sms);
+// How many rows a step over n tokens splits into halves (see FusedStep): the
+// remainder of R over the grid when it is at most half the grid, else 0.
+int fused_half_rows(const Dev& p, int n, const FusedStep& fs, int num_sms);
 
 cudaError_t launch_fused_step(const FusedMaps& maps, const Dev& p, const Step& st, const FusedStep& fs,
                               const FusedPolicy& fp, int num_sms, cudaStream_t s);
