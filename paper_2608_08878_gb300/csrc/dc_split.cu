@@ -18,24 +18,35 @@ constexpr int kTile = 128;  // tokens per tile = threads per CTA
 // seen0 + t, |v|_2, zeroed window sums and cumulative alpha.
 // grid (T, R), block d/8 threads (one 16-byte vector each of K and V).
 // ---------------------------------------------------------------------------
-__global__ void append_kernel(Dev p, const uint4* __restrict__ k, const uint4* __restrict__ v,
-                              int T, int n0, int seen0) {
-  const int t = blockIdx.x, r = blockIdx.y, vpr = p.d / 8;
-  const size_t src = ((size_t)r * T + t) * vpr + threadIdx.x;
+// One (row, token) pair per group of d/8 lanes (16-byte chunks), 256 threads
+// per block: pair e = r * T + t goes to slot n0 + t of row r.
+__global__ void __launch_bounds__(256) append_kernel(Dev p, const uint4* __restrict__ k,
+                                                     const uint4* __restrict__ v, long long pairs, int T,
+                                                     int n0, int seen0) {
+  const int vpr = p.d / 8;
+  const long long e = ((long long)blockIdx.x * blockDim.x + threadIdx.x) / vpr;
+  const int c = threadIdx.x % vpr;
+  const bool live = e < pairs;
+  const long long ee = live ? e : pairs - 1;
+  const int r = (int)(ee / T), t = (int)(ee % T);
+  const size_t src = (size_t)ee * vpr + c;
   const size_t slot = (size_t)r * p.stride + n0 + t;
   const uint4 kv = k[src], vv = v[src];
-  reinterpret_cast<uint4*>(p.K)[slot * vpr + threadIdx.x] = kv;
-  reinterpret_cast<uint4*>(p.V)[slot * vpr + threadIdx.x] = vv;
+  if (live) {
+    reinterpret_cast<uint4*>(p.K)[slot * vpr + c] = kv;
+    reinterpret_cast<uint4*>(p.V)[slot * vpr + c] = vv;
+  }
   const uint32_t w4[4] = {vv.x, vv.y, vv.z, vv.w};
   float ss = 0.f;
 #pragma unroll
-  for (int e = 0; e < 4; ++e) {
-    const float x0 = bf16lo(w4[e]), x1 = bf16hi(w4[e]);
+  for (int q = 0; q < 4; ++q) {
+    const float x0 = bf16lo(w4[q]), x1 = bf16hi(w4[q]);
     ss = fmaf(x0, x0, ss);
     ss = fmaf(x1, x1, ss);
   }
-  for (int off = 1; off < vpr; off <<= 1) ss += __shfl_xor_sync((1u << vpr) - 1u, ss, off);
-  if (threadIdx.x == 0) {
+  // xor offsets below vpr stay inside the pair's aligned lane group
+  for (int off = 1; off < vpr; off <<= 1) ss += __shfl_xor_sync(0xffffffffu, ss, off);
+  if (live && c == 0) {
     p.pos[slot] = seen0 + t;
     p.vnorm[slot] = sqrtf(ss);
     p.SZ[slot] = make_float4(0.f, 0.f, 0.f, 0.f);
@@ -364,8 +375,11 @@ void launch_convert_sz(const Dev& p, int row0, int nrows, int which, double* dst
 // ---------------------------------------------------------------------------
 void launch_append(const Dev& p, const void* k, const void* v, int T, int n0, int seen0,
                    cudaStream_t s) {
-  dim3 grid(T, p.R);
-  append_kernel<<<grid, p.d / 8, 0, s>>>(p, (const uint4*)k, (const uint4*)v, T, n0, seen0);
+  const long long pairs = (long long)T * p.R;
+  if (pairs == 0) return;
+  const long long per_block = 256 / (p.d / 8);
+  const unsigned blocks = (unsigned)((pairs + per_block - 1) / per_block);
+  append_kernel<<<blocks, 256, 0, s>>>(p, (const uint4*)k, (const uint4*)v, pairs, T, n0, seen0);
 }
 
 #define DC_DISPATCH(EXPR)                                                   \
