@@ -430,6 +430,99 @@ def run_reference(args):
             "e2e": {"value": cb["value"], "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
 
 
+# ---------------------------------------------------------------------------
+# Throughput sweep (batch x context x budget ratio), one JSON line per point
+# ---------------------------------------------------------------------------
+
+SWEEP_BATCH = (1, 4, 16, 64)
+SWEEP_CONTEXT = (4096, 16384, 32768)
+SWEEP_RATIO = (0.10, 0.25, 0.50)
+
+
+def run_sweep(args):
+    """Steady-state decode steps/s per point of the sweep, next to full-cache
+    attention on the same shapes. The steady cache is synthesised at its
+    budget size (B prompt tokens, then decode steps that append one token and
+    evict one), which is what the cache holds after prompt compression; the
+    full-cache comparator attends over context + 1 tokens and is timed on as
+    many layers as fit in 48 GB, scaled to 32 layers (its time is linear in
+    the rows)."""
+    import torch
+    from paper_2608_08878_gb300 import build, dc, synth, synth_device
+    torch.cuda.set_device(0)
+    build.build()
+    peaks, _ = measured_peaks()
+    stream = torch.cuda.current_stream()
+    pts = [(b, c, r) for b in SWEEP_BATCH for c in SWEEP_CONTEXT for r in SWEEP_RATIO]
+    if args.sweep_points:
+        keep = set(args.sweep_points.split(","))
+        pts = [p for p in pts if f"{p[0]}x{p[1]}x{int(round(p[2] * 100))}" in keep]
+    K, W = args.steps, args.warmup
+    for b, c, r in pts:
+        wl = synth.sweep_point(b, c, r)
+        B, d = wl.budget, wl.head_dim
+        cache = dc.DistillCache(wl.layers, wl.kv_heads, d, B + 1, B, batch=b, q_heads=wl.q_heads,
+                                window=wl.window, mlp_hidden=wl.mlp_hidden, layernorm=wl.layernorm,
+                                seed=wl.policy_seed)
+        chunk = max(1, min(B, (1 << 31) // (wl.rows * d * 2)))
+        for t0 in range(0, B, chunk):
+            k, v = synth_device.prompt(wl, t0, min(chunk, B - t0))
+            cache.append(k, v)
+            del k, v
+        inputs = [synth_device.step_inputs(wl, s) for s in range(W + K)]
+        out = torch.empty((wl.layers, b, wl.q_heads, d), dtype=torch.float32, device="cuda")
+        for s in range(W):
+            cache.step(*inputs[s], out=out)
+        engine = cache.engine()
+        torch.cuda.synchronize()
+        ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        with ClockSampler(gpu_index_for_smi(0)) as clk:
+            ev0.record(stream)
+            for s in range(W, W + K):
+                cache.step(*inputs[s], out=out)
+            ev1.record(stream)
+            torch.cuda.synchronize()
+        cache.sync()
+        ms = ev0.elapsed_time(ev1) / K
+        bytes_step = step_bytes(wl, B + 1)
+        del cache, inputs, out
+        torch.cuda.empty_cache()
+        # full-cache comparator on a layer subset
+        per_layer = b * wl.kv_heads * (c + 1) * (4 * d + 20)
+        lf = max(1, min(wl.layers, int(48e9 // per_layer)))
+        wf = wl.with_(layers=lf)
+        full = dc.DistillCache(lf, wl.kv_heads, d, c + 1, c, batch=b, q_heads=wl.q_heads, engine=1)
+        chunk = max(1, min(c + 1, (1 << 31) // (wf.rows * d * 2)))
+        for t0 in range(0, c + 1, chunk):
+            k, v = synth_device.prompt(wf, t0, min(chunk, c + 1 - t0))
+            full.append(k, v)
+            del k, v
+        qf = synth_device.step_inputs(wf, 0)[0]
+        for _ in range(2):
+            full.full_decode(qf)
+        torch.cuda.synchronize()
+        reps = 5
+        ev0.record(stream)
+        for _ in range(reps):
+            full.full_decode(qf)
+        ev1.record(stream)
+        torch.cuda.synchronize()
+        full_ms = ev0.elapsed_time(ev1) / reps * wl.layers / lf
+        del full, qf
+        torch.cuda.empty_cache()
+        gbs = bytes_step / (ms / 1e3) / 1e9
+        print(json.dumps({
+            "sweep_point": f"{b}x{c}x{int(round(r * 100))}", "batch": b, "context": c, "ratio": r,
+            "budget": B, "rows": wl.rows, "engine": engine, "steps": K, "warmup": W,
+            "ms_per_step": ms, "steps_per_s": 1e3 / ms, "gbs": gbs,
+            "frac_of_8tbs": gbs / NOMINAL_HBM_GBS, "frac_of_measured": gbs / peaks["hbm_gbs"],
+            "full_cache_ms_per_step": full_ms, "full_cache_layers_timed": lf,
+            "speedup_vs_full": full_ms / ms,
+            "footprint_steady_gb": wl.rows * (B + 1) * (4 * d + 20) / 1e9,
+            "footprint_prompt_gb": wl.rows * (c + 1) * (4 * d + 20) / 1e9,
+            "clocks": clk.summary(), "data": "synthetic"}), flush=True)
+
+
 def main():
     ap = argparse.ArgumentParser(description=__doc__.splitlines()[0])
     ap.add_argument("--gpus", type=int, default=1)
@@ -445,6 +538,9 @@ def main():
     ap.add_argument("--batch", type=int, default=None, help="profiling: another batch than the workload's 8")
     ap.add_argument("--context", type=int, default=None, help="profiling: another prompt length than 32768")
     ap.add_argument("--budget", type=int, default=None, help="profiling: another budget than 8192")
+    ap.add_argument("--sweep", action="store_true",
+                    help="throughput sweep (batch x context x ratio): one JSON line per point")
+    ap.add_argument("--sweep-points", default=None, help="e.g. 1x4096x10,64x32768x50 (default: all 36)")
     args = ap.parse_args()
     if args.layers:
         _OVERRIDES["layers"] = args.layers
@@ -456,6 +552,9 @@ def main():
         _OVERRIDES["budget"] = args.budget
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")
+    if args.sweep:
+        run_sweep(args)
+        return
     if args.impl == "reference":
         res = run_reference(args)
         if res:

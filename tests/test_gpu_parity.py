@@ -257,6 +257,21 @@ def test_full_stack_sampled_rows(engine):
     assert ls.cache.length()[0] == wl.budget
 
 
+@pytest.mark.parametrize("batch,ctx,ratio", [(1, 4096, 0.10), (64, 4096, 0.25), (4, 16384, 0.50),
+                                              (1, 32768, 0.50)])
+def test_sweep_points_sampled_rows(batch, ctx, ratio):
+    """Points of the throughput sweep (32 layers, Mistral-7B KV heads) at full
+    size in the engine auto-selection the sweep uses: prompt compression and
+    steady steps, 3 sampled rows. The last point's budget (16384) is past the
+    fused kernel's row limit, so it runs on the split engine."""
+    wl = synth.sweep_point(batch, ctx, ratio)
+    ls = LockStep(wl, [0, wl.rows // 2 + 3, wl.rows - 1], engine=0, device_inputs=True)
+    ls.load_prompt()
+    for _ in range(3):
+        ls.step()
+    assert ls.cache.length()[0] == wl.budget
+
+
 def test_aggressive_sampled_rows():
     """32 layers, batch 16, 32K context, budget 3277 (10%), hot sets reshuffled
     every 16 steps: crosses one reshuffle, 2 sampled rows."""
