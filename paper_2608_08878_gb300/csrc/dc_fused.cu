@@ -89,6 +89,35 @@ enum {
   B_OEMPTY = B_QFULL + 21, B_DRAIN = B_QFULL + 22, B_DRAIN2 = B_QFULL + 23, B_COUNT = B_QFULL + 24
 };
 
+// Tiles whose logits stay on chip between the passes (heads 0..G-2 in TMEM,
+// head G-1 in shared memory); later tiles of longer rows keep all G logits in
+// the global scratch [R][stride][G] instead.
+template <int GS>
+constexpr int onchip_tiles() {
+  constexpr int st = GS > 0 ? (kStashAEnd - kStashA) / GS + (kStashBEnd - kStashB) / GS : (1 << 20);
+  return st < kFusedMaxTok / kTok ? st : kFusedMaxTok / kTok;
+}
+
+template <int G>
+__device__ __forceinline__ void store_logits(float* dst, const float* v) {
+  if constexpr (G == 4) *reinterpret_cast<float4*>(dst) = make_float4(v[0], v[1], v[2], v[3]);
+  else if constexpr (G == 2) *reinterpret_cast<float2*>(dst) = make_float2(v[0], v[1]);
+  else dst[0] = v[0];
+}
+
+template <int G>
+__device__ __forceinline__ void load_logits(const float* src, float* v) {
+  if constexpr (G == 4) {
+    const float4 x = *reinterpret_cast<const float4*>(src);
+    v[0] = x.x; v[1] = x.y; v[2] = x.z; v[3] = x.w;
+  } else if constexpr (G == 2) {
+    const float2 x = *reinterpret_cast<const float2*>(src);
+    v[0] = x.x; v[1] = x.y;
+  } else {
+    v[0] = src[0];
+  }
+}
+
 // TMEM column of the stashed logits of tile j (GS = G - 1 columns per tile).
 template <int GS>
 __device__ __forceinline__ uint32_t stash_col(int j) {
@@ -221,7 +250,9 @@ __device__ __forceinline__ Item read_item(volatile int* ring, int gr, volatile i
   return Item{e[0], e[1], e[2], e[3]};
 }
 
-template <int D, int G>
+// LONG: the row may be longer than its on-chip logit capacity (a separate
+// instantiation, so rows that fit run code without the spill branches).
+template <int D, int G, bool LONG>
 __global__ void __launch_bounds__(kThreads, 1)
     fused_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmV, Dev p,
                  Step st, FusedStep fs, FusedPolicy fp) {
@@ -528,9 +559,13 @@ __global__ void __launch_bounds__(kThreads, 1)
             p.SZ[rbase + i] = sz;
           }
         }
-        sc[i] = S16[G - 1];
-        __syncwarp();
-        stash_store<GS>(lane_addr + stash_col<GS>(j), S16);
+        if (!LONG || j < onchip_tiles<GS>()) {
+          sc[i] = S16[G - 1];
+          __syncwarp();
+          stash_store<GS>(lane_addr + stash_col<GS>(j), S16);
+        } else {
+          store_logits<G>(p.logit + (rbase + i) * G, S16);
+        }
       }
       g += nTi;
       gs += nTi;
@@ -662,9 +697,13 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int i = j * kTok + tok;
         const bool valid = i < n;
         float sv[G];
-        stash_load<GS>(lane_addr + stash_col<GS>(j), sv);
-        if constexpr (GS > 0) tmem_ld_wait();
-        sv[G - 1] = sc[i];
+        if (!LONG || j < onchip_tiles<GS>()) {
+          stash_load<GS>(lane_addr + stash_col<GS>(j), sv);
+          if constexpr (GS > 0) tmem_ld_wait();
+          sv[G - 1] = sc[i];
+        } else {
+          load_logits<G>(p.logit + (rbase + i) * G, sv);
+        }
         float a[G], zc = 0.f, scur = 0.f;
 #pragma unroll
         for (int h = 0; h < G; ++h) {
@@ -787,8 +826,14 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int i = j * kTok + tok;
         if (i < n) {
           const float score = fp.b2 + relu_sum;
-          sc[i] = score;
-          if (fs.write_scores) p.score[rbase + i] = score;
+          if constexpr (LONG) {
+            // rows longer than the shared score array keep their scores in HBM
+            if (n > kFusedMaxTok || fs.write_scores) p.score[rbase + i] = score;
+            if (n <= kFusedMaxTok) sc[i] = score;
+          } else {
+            sc[i] = score;
+            if (fs.write_scores) p.score[rbase + i] = score;
+          }
           // this thread's lowest-ranked token so far (lower key, then the later position)
           const uint32_t kk = score_key(score);
           if (ev_slot < 0 || kk < ev_key || (kk == ev_key && pos > ev_pos)) {
@@ -899,7 +944,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       } else if (fs.do_evict && fs.B < n) {
         // several evictions (whole rows only): radix select over the scores
         sync();
-        team_select_compact<kEpi>(p, r, n, fs.B, sc, etid, scr, sync);
+        team_select_compact<kEpi>(p, r, n, fs.B, LONG && n > kFusedMaxTok ? p.score + rbase : sc, etid, scr,
+                                  sync);
       }
     }
   }
@@ -913,31 +959,29 @@ __global__ void __launch_bounds__(kThreads, 1)
 
 }  // namespace
 
-int fused_max_tokens(int G) {
-  if (G <= 1) return kFusedMaxTok;
-  const int GS = G - 1;
-  const int tiles = (kStashAEnd - kStashA) / GS + (kStashBEnd - kStashB) / GS;
-  return tiles * kTok < kFusedMaxTok ? tiles * kTok : kFusedMaxTok;
+int fused_onchip_tokens(int G) {
+  const int t = G == 4 ? onchip_tiles<3>() : G == 2 ? onchip_tiles<1>() : onchip_tiles<0>();
+  return t * kTok;
 }
 
 bool fused_eligible(const Dev& p, int n) {
   return (p.d == 64 || p.d == 128) && (p.G == 1 || p.G == 2 || p.G == 4) && p.hidden <= 128 && n >= 1 &&
-         n <= fused_max_tokens(p.G);
+         p.logit != nullptr && p.score != nullptr;
 }
 
 int fused_smem_bytes() { return kSmemBytes; }
 
-template <int D, int G>
+template <int D, int G, bool LONG>
 static cudaError_t launch_t(const FusedMaps& maps, const Dev& p, const Step& st, const FusedStep& fs,
                             const FusedPolicy& fp, int grid, cudaStream_t s) {
   static bool attr = false;
   if (!attr) {
-    cudaError_t e = cudaFuncSetAttribute(fused_kernel<D, G>, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes);
+    cudaError_t e = cudaFuncSetAttribute(fused_kernel<D, G, LONG>, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes);
     if (e != cudaSuccess) return e;
     attr = true;
   }
   if (fs.half_rows == 0) {
-    fused_kernel<D, G><<<grid, kThreads, kSmemBytes, s>>>(maps.k, maps.v, p, st, fs, fp);
+    fused_kernel<D, G, LONG><<<grid, kThreads, kSmemBytes, s>>>(maps.k, maps.v, p, st, fs, fp);
     return cudaGetLastError();
   }
   // the two CTAs of a half row wait on each other: a cooperative launch
@@ -952,7 +996,7 @@ static cudaError_t launch_t(const FusedMaps& maps, const Dev& p, const Step& st,
   la[0].val.cooperative = 1;
   cfg.attrs = la;
   cfg.numAttrs = 1;
-  return cudaLaunchKernelEx(&cfg, fused_kernel<D, G>, maps.k, maps.v, p, st, fs, fp);
+  return cudaLaunchKernelEx(&cfg, fused_kernel<D, G, LONG>, maps.k, maps.v, p, st, fs, fp);
 }
 
 static int fused_grid(const Dev& p, int num_sms) { return p.R < num_sms ? p.R : num_sms; }
@@ -968,14 +1012,18 @@ int fused_half_rows(const Dev& p, int n, const FusedStep& fs, int num_sms) {
 cudaError_t launch_fused_step(const FusedMaps& maps, const Dev& p, const Step& st, const FusedStep& fs,
                               const FusedPolicy& fp, int num_sms, cudaStream_t s) {
   const int grid = fused_grid(p, num_sms);
+  const bool lg = st.n > fused_onchip_tokens(p.G);
+#define DC_FUSED_LAUNCH(D, G) \
+  return lg ? launch_t<D, G, true>(maps, p, st, fs, fp, grid, s) : launch_t<D, G, false>(maps, p, st, fs, fp, grid, s)
   if (p.d == 128) {
-    if (p.G == 4) return launch_t<128, 4>(maps, p, st, fs, fp, grid, s);
-    if (p.G == 2) return launch_t<128, 2>(maps, p, st, fs, fp, grid, s);
-    return launch_t<128, 1>(maps, p, st, fs, fp, grid, s);
+    if (p.G == 4) DC_FUSED_LAUNCH(128, 4);
+    if (p.G == 2) DC_FUSED_LAUNCH(128, 2);
+    DC_FUSED_LAUNCH(128, 1);
   }
-  if (p.G == 4) return launch_t<64, 4>(maps, p, st, fs, fp, grid, s);
-  if (p.G == 2) return launch_t<64, 2>(maps, p, st, fs, fp, grid, s);
-  return launch_t<64, 1>(maps, p, st, fs, fp, grid, s);
+  if (p.G == 4) DC_FUSED_LAUNCH(64, 4);
+  if (p.G == 2) DC_FUSED_LAUNCH(64, 2);
+  DC_FUSED_LAUNCH(64, 1);
+#undef DC_FUSED_LAUNCH
 }
 
 }  // namespace dc

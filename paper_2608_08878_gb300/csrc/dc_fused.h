@@ -12,8 +12,8 @@
 
 namespace dc {
 
-// Most tokens a row may hold for the fused kernel (one CTA per row: the raw
-// logits of the row live in TMEM, the scores in shared memory).
+// Tokens of a row whose head-(G-1) logits and scores the fused kernel keeps in
+// shared memory; longer rows keep them in HBM (Dev::logit, Dev::score).
 constexpr int kFusedMaxTok = 10240;
 
 struct FusedMaps {
@@ -62,8 +62,11 @@ struct FusedPolicy {
                                  // it is sum_j sgn_j z_j (relu(z) = (z + |z|) / 2)
 };
 
-// Most tokens per row the fused kernel takes for a query group of G heads.
-int fused_max_tokens(int G);
+// Tokens per row whose logits the fused kernel keeps on chip between its two
+// passes (G query heads per KV head); beyond that a row's logits go through
+// the global scratch Dev::logit (16 bytes per token written and read back)
+// and its scores through Dev::score.
+int fused_onchip_tokens(int G);
 bool fused_eligible(const Dev& p, int n);
 int fused_smem_bytes();
 

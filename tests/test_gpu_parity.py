@@ -175,10 +175,25 @@ def test_tail_split_step_equals_decode_then_evict():
             assert err <= 1e-4, err
 
 
+@pytest.mark.parametrize("prompt_len,budget", [(12000, 10000), (16000, 12000)])
+def test_fused_long_rows(prompt_len, budget):
+    """Rows longer than the fused kernel keeps on chip (8704 tokens with four
+    query heads per KV head): later tiles' logits go through HBM, and past
+    10240 tokens the scores too. Prompt compression (many evictions) and
+    steady steps, all 8 rows against the oracle."""
+    wl = synth.MISTRAL_1L.with_(prompt_len=prompt_len, budget=budget, steps=4)
+    ls = LockStep(wl, range(wl.rows), engine=2)
+    assert ls.cache.engine() == "fused"
+    ls.load_prompt()
+    for _ in range(wl.steps):
+        ls.step()
+    assert ls.cache.length()[0] == budget
+
+
 def test_engine_choice():
     from paper_2608_08878_gb300 import dc
     big = dc.DistillCache(32, 8, 128, 200, 100, batch=1)
-    assert big.engine() == "fused" and big.engine(20000) == "split"
+    assert big.engine() == "fused" and big.engine(20000) == "fused"
     small = dc.DistillCache(1, 2, 64, 200, 100, q_heads=4)
     assert small.engine() == "split"
     forced = dc.DistillCache(1, 2, 64, 200, 100, q_heads=4, engine=2)
