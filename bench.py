@@ -491,7 +491,7 @@ def run_sweep(args):
         per_layer = b * wl.kv_heads * (c + 1) * (4 * d + 20)
         lf = max(1, min(wl.layers, int(48e9 // per_layer)))
         wf = wl.with_(layers=lf)
-        full = dc.DistillCache(lf, wl.kv_heads, d, c + 1, c, batch=b, q_heads=wl.q_heads, engine=1)
+        full = dc.DistillCache(lf, wl.kv_heads, d, c + 1, c, batch=b, q_heads=wl.q_heads)
         chunk = max(1, min(c + 1, (1 << 31) // (wf.rows * d * 2)))
         for t0 in range(0, c + 1, chunk):
             k, v = synth_device.prompt(wf, t0, min(chunk, c + 1 - t0))

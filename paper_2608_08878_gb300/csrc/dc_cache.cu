@@ -583,6 +583,19 @@ dc_status dc_full_decode(dc_cache* h, const void* q, float* out) {
   DC_CHECK_HANDLE(h);
   if (!q || !out) return fail(h, DC_ERR_INVALID_ARG, "NULL pointer");
   if (h->n < 1) return fail(h, DC_ERR_STATE, "the cache is empty");
+  if (h->fused_ok && dc::fused_eligible(h->dev, h->n)) {
+    // the fused kernel's attention-only variant (TMA + tensor cores)
+    dc::Step st{};
+    st.n = h->n;
+    const dc::FusedStep fs = fused_args(h, st, q, out, 0, 0, 0);
+    cudaError_t e;
+    {
+      Phase ph(h, DC_PHASE_FULL, 1);
+      e = dc::launch_fused_full(h->maps, h->dev, h->n, fs, h->fpol, h->num_sms, h->stream);
+    }
+    if (e != cudaSuccess) return cuda_fail(h, e, "full decode");
+    return launch_error(h, "full decode");
+  }
   int nsplit, chunk;
   split_plan(h, h->n, &nsplit, &chunk);
   bool ok;

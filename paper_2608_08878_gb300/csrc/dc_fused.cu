@@ -252,7 +252,9 @@ __device__ __forceinline__ Item read_item(volatile int* ring, int gr, volatile i
 
 // LONG: the row may be longer than its on-chip logit capacity (a separate
 // instantiation, so rows that fit run code without the spill branches).
-template <int D, int G, bool LONG>
+// FULL: attention only, over the cache as it is (the full-cache comparator):
+// no window state, features, policy, select, or writes to the cache's state.
+template <int D, int G, bool LONG, bool FULL>
 __global__ void __launch_bounds__(kThreads, 1)
     fused_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmV, Dev p,
                  Step st, FusedStep fs, FusedPolicy fp) {
@@ -365,7 +367,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         *reinterpret_cast<uint4*>(qt + (kc >> 3) * 2048 + sw128(h, kc & 7)) = cur;
         *reinterpret_cast<uint4*>(qt + (kc >> 3) * 2048 + sw128(G + h, kc & 7)) = pv;
         *reinterpret_cast<uint4*>(qt + (kc >> 3) * 2048 + sw128(2 * G + h, kc & 7)) = dv;
-        if (it.half < 0) reinterpret_cast<uint4*>(ring_slot + h * D)[kc] = cur;  // halves: see the epilogue
+        if (!FULL && it.half < 0) reinterpret_cast<uint4*>(ring_slot + h * D)[kc] = cur;  // halves: see the epilogue
       }
       fence_proxy_async();
       __syncwarp();
@@ -376,13 +378,13 @@ __global__ void __launch_bounds__(kThreads, 1)
           for (int j = it.t0; j < it.t1; ++j, ++g) {
             const int s = g % kStages;
             if (!mbar_wait(&bar[B_EMPTY + s], ((g / kStages) & 1) ^ 1, abort, p.dbg, 2u, (unsigned)g)) break;
-            mbar_expect_tx(&bar[B_FULL + s], kTileBytes + (pass ? 0u : 2560u));
+            mbar_expect_tx(&bar[B_FULL + s], kTileBytes + ((pass || FULL) ? 0u : 2560u));
             uint8_t* dst = smem + OFF_STAGE + s * kStageBytes;
             uint8_t* aux = smem + OFF_AUX + s * kAuxBytes;
             const int y = r * p.stride + j * kTok;
             tma_load_2d(dst, tm, 0, y, &bar[B_FULL + s], pol);
             if (D == 128) tma_load_2d(dst + 16384, tm, 64, y, &bar[B_FULL + s], pol);
-            if (!pass) {
+            if (!FULL && !pass) {
               bulk_load(aux + kAuxPos, p.pos + y, 512, &bar[B_FULL + s]);
               bulk_load(aux + kAuxSZ, p.SZ + y, 2048, &bar[B_FULL + s]);
             }
@@ -458,7 +460,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     __syncwarp();
   } else if (warp == 10) {
     // ------------------------------------------------------------ policy-layer MMA issuer
-    if (lane == 0) {
+    if (!FULL && lane == 0) {
       const uint32_t id_m = idesc_bf16(128, 128, 0, 0);
       const uint32_t waddr = smem_u32(smem + OFF_W);
       int gv = 0;
@@ -547,7 +549,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (i < n) {
 #pragma unroll
           for (int h = 0; h < G; ++h) online_add(m[h], l[h], u[h], S16[h], c);
-          if (st.has_prev || st.has_dep) {
+          if (!FULL && (st.has_prev || st.has_dep)) {
             // terms of the previous and the departing query, masked (x 1 or x 0,
             // both exact) where the token was not yet in the cache at that step
             float zp, sp, zd, sd;
@@ -641,7 +643,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         // half 1 has read the departing query and statistics (it published
         // after its K pass): half 0 may now give their ring slot to this step
-        if (half == 0) {
+        if (!FULL && half == 0) {
           const int qo = ((r / p.kvh) * p.qh + (r % p.kvh) * G) * D;
           uint4* ring_slot = reinterpret_cast<uint4*>(p.ring_q + ((size_t)r * p.w + st.slot) * G * D);
           for (int e = etid; e < G * (D / 8); e += kEpi) ring_slot[e] = reinterpret_cast<const uint4*>(fs.q + qo)[e];
@@ -658,7 +660,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
       // push (m, l, H, -log2 l) of this step into the ring slot it takes over
       // (the producer, or half 0 above, wrote the query there)
-      if (etid < G && half <= 0) {
+      if (!FULL && etid < G && half <= 0) {
         float4 v;
         v.x = M[etid]; v.y = L0; v.z = Hh[etid]; v.w = NL[etid];
         reinterpret_cast<float4*>(p.ring_stats)[((size_t)r * p.w + st.slot) * G + etid] = v;
@@ -675,12 +677,17 @@ __global__ void __launch_bounds__(kThreads, 1)
       const int* posrow = p.pos + rbase + tok;
       const float* vnrow = p.vnorm + rbase + tok;
       const float4 kZero4 = make_float4(0.f, 0.f, 0.f, 0.f);
-      float4 szA = j0 < t1 ? szrow[j0 * kTok] : kZero4;
-      float4 szB = j0 + 2 < t1 ? szrow[(j0 + 2) * kTok] : kZero4;
-      int posA = j0 < t1 ? posrow[j0 * kTok] : 0;
-      int posB = j0 + 2 < t1 ? posrow[(j0 + 2) * kTok] : 0;
-      float vnA = j0 < t1 ? vnrow[j0 * kTok] : 0.f;
-      float vnB = j0 + 2 < t1 ? vnrow[(j0 + 2) * kTok] : 0.f;
+      float4 szA = kZero4, szB = kZero4;
+      int posA = 0, posB = 0;
+      float vnA = 0.f, vnB = 0.f;
+      if constexpr (!FULL) {
+        szA = j0 < t1 ? szrow[j0 * kTok] : kZero4;
+        szB = j0 + 2 < t1 ? szrow[(j0 + 2) * kTok] : kZero4;
+        posA = j0 < t1 ? posrow[j0 * kTok] : 0;
+        posB = j0 + 2 < t1 ? posrow[(j0 + 2) * kTok] : 0;
+        vnA = j0 < t1 ? vnrow[j0 * kTok] : 0.f;
+        vnB = j0 + 2 < t1 ? vnrow[(j0 + 2) * kTok] : 0.f;
+      }
       auto prep = [&](int j) {
         const int gvj = gv + (j - t0), pb = gvj & 1;
         const float4 sz = szA;
@@ -689,7 +696,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         szA = szB;
         posA = posB;
         vnA = vnB;
-        if (j + 4 < t1) {
+        if (!FULL && j + 4 < t1) {
           szB = szrow[(j + 4) * kTok];
           posB = posrow[(j + 4) * kTok];
           vnB = vnrow[(j + 4) * kTok];
@@ -735,6 +742,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           __syncwarp();
           if (lane == 0) mbar_arrive(&bar[B_PFULL + pb]);
         }
+        if constexpr (FULL) return make_float2(0.f, 0.f);
         const float mean = zc / (float)G;
         float var = 0.f;
 #pragma unroll
@@ -847,7 +855,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       float2 pf_cur = j0 < t1 ? prep(j0) : make_float2(0.f, 0.f);
       for (int j = j0; j < t1; j += 2) {
         const float2 pf_next = j + 2 < t1 ? prep(j + 2) : make_float2(0.f, 0.f);
-        finish(j, pf_cur.x, __float_as_int(pf_cur.y));
+        if constexpr (!FULL) finish(j, pf_cur.x, __float_as_int(pf_cur.y));
         pf_cur = pf_next;
       }
       g += nTi;
@@ -971,17 +979,17 @@ bool fused_eligible(const Dev& p, int n) {
 
 int fused_smem_bytes() { return kSmemBytes; }
 
-template <int D, int G, bool LONG>
+template <int D, int G, bool LONG, bool FULL = false>
 static cudaError_t launch_t(const FusedMaps& maps, const Dev& p, const Step& st, const FusedStep& fs,
                             const FusedPolicy& fp, int grid, cudaStream_t s) {
   static bool attr = false;
   if (!attr) {
-    cudaError_t e = cudaFuncSetAttribute(fused_kernel<D, G, LONG>, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes);
+    cudaError_t e = cudaFuncSetAttribute(fused_kernel<D, G, LONG, FULL>, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes);
     if (e != cudaSuccess) return e;
     attr = true;
   }
   if (fs.half_rows == 0) {
-    fused_kernel<D, G, LONG><<<grid, kThreads, kSmemBytes, s>>>(maps.k, maps.v, p, st, fs, fp);
+    fused_kernel<D, G, LONG, FULL><<<grid, kThreads, kSmemBytes, s>>>(maps.k, maps.v, p, st, fs, fp);
     return cudaGetLastError();
   }
   // the two CTAs of a half row wait on each other: a cooperative launch
@@ -996,7 +1004,7 @@ static cudaError_t launch_t(const FusedMaps& maps, const Dev& p, const Step& st,
   la[0].val.cooperative = 1;
   cfg.attrs = la;
   cfg.numAttrs = 1;
-  return cudaLaunchKernelEx(&cfg, fused_kernel<D, G, LONG>, maps.k, maps.v, p, st, fs, fp);
+  return cudaLaunchKernelEx(&cfg, fused_kernel<D, G, LONG, FULL>, maps.k, maps.v, p, st, fs, fp);
 }
 
 static int fused_grid(const Dev& p, int num_sms) { return p.R < num_sms ? p.R : num_sms; }
@@ -1024,6 +1032,21 @@ cudaError_t launch_fused_step(const FusedMaps& maps, const Dev& p, const Step& s
   if (p.G == 2) DC_FUSED_LAUNCH(64, 2);
   DC_FUSED_LAUNCH(64, 1);
 #undef DC_FUSED_LAUNCH
+}
+
+cudaError_t launch_fused_full(const FusedMaps& maps, const Dev& p, int n, const FusedStep& fs,
+                              const FusedPolicy& fp, int num_sms, cudaStream_t s) {
+  const int grid = fused_grid(p, num_sms);
+  Step st{};
+  st.n = n;  // no previous or departing query terms: has_prev = has_dep = 0
+  if (p.d == 128) {
+    if (p.G == 4) return launch_t<128, 4, true, true>(maps, p, st, fs, fp, grid, s);
+    if (p.G == 2) return launch_t<128, 2, true, true>(maps, p, st, fs, fp, grid, s);
+    return launch_t<128, 1, true, true>(maps, p, st, fs, fp, grid, s);
+  }
+  if (p.G == 4) return launch_t<64, 4, true, true>(maps, p, st, fs, fp, grid, s);
+  if (p.G == 2) return launch_t<64, 2, true, true>(maps, p, st, fs, fp, grid, s);
+  return launch_t<64, 1, true, true>(maps, p, st, fs, fp, grid, s);
 }
 
 }  // namespace dc

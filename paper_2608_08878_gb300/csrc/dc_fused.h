@@ -84,4 +84,10 @@ int fused_half_rows(const Dev& p, int n, const FusedStep& fs, int num_sms);
 cudaError_t launch_fused_step(const FusedMaps& maps, const Dev& p, const Step& st, const FusedStep& fs,
                               const FusedPolicy& fp, int num_sms, cudaStream_t s);
 
+// Attention only over the first n tokens of every row as they are (the
+// full-cache comparator): writes fs.out, touches no cache state (the logit
+// scratch aside). fs.do_evict and fs.write_scores must be 0.
+cudaError_t launch_fused_full(const FusedMaps& maps, const Dev& p, int n, const FusedStep& fs,
+                              const FusedPolicy& fp, int num_sms, cudaStream_t s);
+
 }  // namespace dc
