@@ -72,6 +72,21 @@ typedef struct {
                          eviction candidate through global memory under a
                          cooperative launch (steps that evict one token or none);
                          0: whole rows only */
+  int scorer;         /* what ranks the tokens for argtop_B:
+                         0: the policy MLP (default, Sec. 3.1.2);
+                         1: H2O, cumulative attention mass since insertion (the
+                            heavy-hitter baseline of Sec. 2 / Sec. 4; implies
+                            alpha_mode 1);
+                         2: StreamingLLM, the first n_sinks positions (attention
+                            sinks) and then the most recent tokens */
+  int n_sinks;        /* sink tokens kept by scorer 2 (default 4) */
+  float budget_ratio; /* > 0: dynamic budget B_t = max(floor(r * L_t), budget_min)
+                         whenever a call passes budget <= 0 (App. D); 0 (default):
+                         the fixed budget given to dc_cache_create */
+  int budget_min;     /* B_min of the dynamic budget (default 32) */
+  int budget_basis;   /* L_t of the dynamic budget: 0 (default) tokens seen so far
+                         (the sequence length), 1 the tokens cached before the
+                         eviction, |C_t| */
 } dc_config;
 
 /* Fills *cfg with the defaults above (batch 1, q_heads 0 meaning 4 * kv_heads,
@@ -154,8 +169,10 @@ dc_status dc_engine(dc_cache* h, int n, int* engine);
  * tokens (ties: lower position first; -0 equals +0; NaN ranks last) and
  * compacts them into its first min(n, B) slots. Survivors below that bound do
  * not move; each survivor above it moves into the lowest free slot, in
- * ascending slot order. budget <= 0 uses the configured budget. Needs the
- * scores of a decode step since the last append/evict (else DC_ERR_STATE). */
+ * ascending slot order. budget <= 0 uses the configured budget: the dynamic
+ * max(floor(budget_ratio * L_t), budget_min) when budget_ratio > 0 (capped at
+ * capacity - 1), else the fixed one. Needs the scores of a decode step since
+ * the last append/evict (else DC_ERR_STATE). */
 dc_status dc_evict(dc_cache* h, int budget);
 
 /* Full-cache comparator: softmax attention of q over the current rows with no

@@ -50,6 +50,7 @@ def lib():
             L.dco_row_kv_bits.argtypes = [P, P, P]
             L.dco_row_window_sums.argtypes = [P, P, P, P]
             L.dco_row_window_sums_prior.argtypes = [P, P, P]
+            L.dco_row_heuristic_scores.argtypes = [P, C.c_int, C.c_int, P]
             L.dco_attend.argtypes = [P, P, P, C.c_int, C.c_int, C.c_int, P, P]
             L.dco_policy.argtypes = [P, C.c_int, P, C.c_int, C.c_int, P]
             _lib = L
@@ -108,6 +109,14 @@ class OracleRow:
         if n < 0:
             raise RuntimeError("no scores to evict with")
         return n
+
+    def heuristic_scores(self, scorer: int, n_sinks: int = 4) -> np.ndarray:
+        """H2O (scorer 1: cumulative attention mass) or StreamingLLM (scorer 2:
+        sinks, then recency) scores of the row's tokens, ascending positions."""
+        out = np.empty(len(self))
+        if lib().dco_row_heuristic_scores(self._h, scorer, n_sinks, _ptr(out)) != 0:
+            raise ValueError("unknown scorer, or H2O without cumulative attention mass")
+        return out
 
     def __len__(self) -> int:
         return lib().dco_row_len(self._h)

@@ -368,6 +368,28 @@ void dco_row_window_sums(const dco_row* r, double* S, double* Z, double* acc) {
   if (acc) memcpy(acc, r->acc, sizeof(double) * (size_t)r->n);
 }
 
+/* Heuristic scorers on the same path (the baselines the paper compares with,
+ * Sec. 2 and Sec. 4): scorer 1, H2O: the cumulative attention mass each token
+ * received since insertion (needs alpha_mode 1); scorer 2, StreamingLLM: the
+ * first n_sinks positions rank first (score 3e38, ties by position), then the
+ * most recent tokens (score = position - newest position). Scores are for the
+ * row as the last decode step left it (ascending positions). Returns 0, or -1
+ * for an unknown scorer or scorer 1 without cumulative mass. */
+int dco_row_heuristic_scores(const dco_row* r, int scorer, int n_sinks, double* score) {
+  if (scorer == 1) {
+    if (r->alpha_mode != 1) return -1;
+    for (int i = 0; i < r->n; ++i) score[i] = r->acc[i];
+    return 0;
+  }
+  if (scorer == 2) {
+    const int64_t newest = r->seen - 1;
+    for (int i = 0; i < r->n; ++i)
+      score[i] = r->pos[i] < (int64_t)n_sinks ? 3.0e38 : (double)(r->pos[i] - newest);
+    return 0;
+  }
+  return -1;
+}
+
 void dco_row_window_sums_prior(const dco_row* r, double* S, double* Z) {
   if (S) memcpy(S, r->Sp, sizeof(double) * (size_t)r->n);
   if (Z) memcpy(Z, r->Zp, sizeof(double) * (size_t)r->n);

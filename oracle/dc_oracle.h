@@ -69,6 +69,11 @@ void dco_row_kv_bits(const dco_row* r, uint16_t* k, uint16_t* v);
  * and S_i (entropy-weighted mass); cumulative alpha (alpha_mode 1) in acc. */
 void dco_row_window_sums(const dco_row* r, double* S, double* Z, double* acc);
 
+/* Heuristic scores of the row's tokens (ascending positions): scorer 1 H2O
+ * (cumulative attention mass; needs alpha_mode 1), scorer 2 StreamingLLM
+ * (n_sinks first positions, then the most recent). Returns 0 or -1. */
+int dco_row_heuristic_scores(const dco_row* r, int scorer, int n_sinks, double* score);
+
 /* The same window sums without the most recent step's query (the window's
  * earlier min(w, steps) - 1 queries), [n] each. */
 void dco_row_window_sums_prior(const dco_row* r, double* S, double* Z);

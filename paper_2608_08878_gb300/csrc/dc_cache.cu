@@ -236,6 +236,11 @@ dc_status dc_config_default(dc_config* cfg) {
   cfg->seed = 0;
   cfg->stream = nullptr;
   cfg->tail_split = 1;
+  cfg->scorer = 0;
+  cfg->n_sinks = 4;
+  cfg->budget_ratio = 0.f;
+  cfg->budget_min = 32;
+  cfg->budget_basis = 0;
   return DC_OK;
 }
 
@@ -281,6 +286,12 @@ dc_status dc_cache_create(int layers, int kv_heads, int head_dim, int capacity, 
   if (cfg.mlp_hidden < 1 || cfg.mlp_hidden > 256 || (cfg.mlp_hidden >= 32 && cfg.mlp_hidden % 32))
     return fail(nullptr, DC_ERR_INVALID_ARG, "mlp_hidden must be in [1, 256], a multiple of 32 when >= 32");
   if (cfg.alpha_mode != 0 && cfg.alpha_mode != 1) return fail(nullptr, DC_ERR_INVALID_ARG, "alpha_mode must be 0 or 1");
+  if (cfg.scorer < 0 || cfg.scorer > 2) return fail(nullptr, DC_ERR_INVALID_ARG, "scorer must be 0, 1 or 2");
+  if (cfg.n_sinks < 0) return fail(nullptr, DC_ERR_INVALID_ARG, "n_sinks must be >= 0");
+  if (!(cfg.budget_ratio >= 0.f && cfg.budget_ratio <= 1.f) || cfg.budget_min < 1 ||
+      (cfg.budget_basis != 0 && cfg.budget_basis != 1))
+    return fail(nullptr, DC_ERR_INVALID_ARG, "need 0 <= budget_ratio <= 1, budget_min >= 1, budget_basis 0 or 1");
+  if (cfg.scorer == 1) cfg.alpha_mode = 1;  // H2O ranks by the cumulative mass
   if (cfg.engine < 0 || cfg.engine > 2) return fail(nullptr, DC_ERR_INVALID_ARG, "engine must be 0, 1 or 2");
   const long long R = (long long)layers * cfg.batch * kv_heads;
   if (R > 65535 || (long long)capacity * R > (1ll << 40) || capacity > (1 << 30))
@@ -303,6 +314,7 @@ dc_status dc_cache_create(int layers, int kv_heads, int head_dim, int capacity, 
   p.R = (int)R; p.cap = capacity; p.stride = (capacity + 127) / 128 * 128; p.d = head_dim; p.G = G; p.qh = cfg.q_heads; p.kvh = kv_heads;
   p.w = cfg.window; p.hidden = cfg.mlp_hidden; p.layernorm = cfg.layernorm ? 1 : 0;
   p.alpha_mode = cfg.alpha_mode; p.keep_features = cfg.keep_features ? 1 : 0;
+  p.scorer = cfg.scorer; p.n_sinks = cfg.n_sinks;
   p.c = (float)(1.4426950408889634 / std::sqrt((double)head_dim));
   p.smax = (int)std::max(1ll, std::min(64ll, (8ll * h->num_sms + R - 1) / R));
   const size_t RC = (size_t)R * p.stride;
@@ -424,6 +436,20 @@ dc_status dc_append(dc_cache* h, const void* k, const void* v, int n_tokens) {
 
 namespace {
 
+// The budget of a step: the caller's if > 0, else the dynamic budget
+// B_t = max(floor(r * L_t), B_min) (App. D) when configured, else the fixed
+// one. L_t: tokens seen (basis 0) or tokens cached before the eviction
+// (basis 1). Kept below the capacity so the next append fits.
+int effective_budget(const dc_cache* h, int budget, int n_cached, long long seen) {
+  if (budget > 0) return budget;
+  if (h->cfg.budget_ratio <= 0.f) return h->budget;
+  const double L = h->cfg.budget_basis == 0 ? (double)seen : (double)n_cached;
+  long long B = (long long)std::floor((double)h->cfg.budget_ratio * L);
+  if (B < h->cfg.budget_min) B = h->cfg.budget_min;
+  if (B > h->capacity - 1) B = h->capacity - 1;
+  return (int)B;
+}
+
 // Arguments of one fused launch; enables the half-row tail split when the
 // handle has exchange buffers and the step qualifies.
 dc::FusedStep fused_args(dc_cache* h, const dc::Step& st, const void* q, float* out, int do_evict, int B,
@@ -500,7 +526,7 @@ dc_status dc_step(dc_cache* h, const void* q, const void* k_new, const void* v_n
     if (s != DC_OK) return s;
     return dc_evict(h, budget);
   }
-  const int B = budget <= 0 ? h->budget : budget;
+  const int B = effective_budget(h, budget, n1, h->seen + 1);
   if (B < n1 - 1 && tail_split_applies(h, n1)) {
     // several evictions need the whole row's scores in one CTA: with half
     // rows this step runs as the decode kernel plus the eviction kernel
@@ -566,7 +592,7 @@ dc_status dc_decode_step_host(dc_cache* h, const void* q, const void* k_new, con
 dc_status dc_evict(dc_cache* h, int budget) {
   DC_CHECK_HANDLE(h);
   if (!h->have_scores) return fail(h, DC_ERR_STATE, "evict needs the scores of a decode step");
-  const int B = budget <= 0 ? h->budget : budget;
+  const int B = effective_budget(h, budget, h->n, h->seen);
   const int keep = std::min(h->n, B);
   if (keep < h->n) {
     Phase ph(h, DC_PHASE_EVICT, 1);

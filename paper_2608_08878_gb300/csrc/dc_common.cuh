@@ -36,6 +36,7 @@ constexpr unsigned kStatusTimeout = 2u;
 
 struct Dev {
   int R, cap, stride, d, G, qh, kvh, w, hidden, layernorm, alpha_mode, keep_features;
+  int scorer, n_sinks;  // 0 policy MLP, 1 H2O (cumulative alpha), 2 StreamingLLM
   __nv_bfloat16* K;
   __nv_bfloat16* V;
   int* pos;
@@ -175,6 +176,15 @@ __device__ __forceinline__ float policy_score(const float* __restrict__ wsm, int
     }
   }
   return out;
+}
+
+// Scores of the heuristic scorers on the same path: H2O ranks by the
+// cumulative attention mass (alpha, accumulated since insertion); StreamingLLM
+// keeps the first n_sinks positions, then the most recent tokens (the score is
+// the position relative to the newest, exact in fp32 for the last 2^24).
+__device__ __forceinline__ float heuristic_score(const Dev& p, float alpha_cum, int pos, int p_newest) {
+  if (p.scorer == 1) return alpha_cum;
+  return pos < p.n_sinks ? 3.0e38f : (float)(pos - p_newest);
 }
 
 }  // namespace dc

@@ -254,7 +254,9 @@ __device__ __forceinline__ Item read_item(volatile int* ring, int gr, volatile i
 // instantiation, so rows that fit run code without the spill branches).
 // FULL: attention only, over the cache as it is (the full-cache comparator):
 // no window state, features, policy, select, or writes to the cache's state.
-template <int D, int G, bool LONG, bool FULL>
+// HEUR: a heuristic scorer (H2O or StreamingLLM, Dev::scorer) ranks the tokens
+// instead of the policy MLP, whose tensor-core layer is then skipped.
+template <int D, int G, bool LONG, bool FULL, bool HEUR>
 __global__ void __launch_bounds__(kThreads, 1)
     fused_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmV, Dev p,
                  Step st, FusedStep fs, FusedPolicy fp) {
@@ -460,7 +462,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     __syncwarp();
   } else if (warp == 10) {
     // ------------------------------------------------------------ policy-layer MMA issuer
-    if (!FULL && lane == 0) {
+    if (!FULL && !HEUR && lane == 0) {
       const uint32_t id_m = idesc_bf16(128, 128, 0, 0);
       const uint32_t waddr = smem_u32(smem + OFF_W);
       int gv = 0;
@@ -761,6 +763,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
             for (int e = 0; e < 5; ++e) p.feat[slot * 5 + e] = x[e];
         }
+        if constexpr (HEUR) return make_float2(heuristic_score(p, x[0], pos, st.p_newest), __int_as_float(pos));
         // the policy layer's input row: [r x, r, 1, 0] (LayerNorm folded into
         // the weights) or [x, 1, 0, 0], as bf16 hi | lo | hi parts
         float av[8];
@@ -851,11 +854,27 @@ __global__ void __launch_bounds__(kThreads, 1)
           }
         }
       };
-      // prep(j) returns (the linear score part, the position) for finish(j)
+      // the score of a heuristic scorer, recorded like finish() records the policy's
+      auto record_h = [&](int j, float score, int pos) {
+        const int i = j * kTok + tok;
+        if (i < n) {
+          if (n > kFusedMaxTok || fs.write_scores) p.score[rbase + i] = score;
+          if (n <= kFusedMaxTok) sc[i] = score;
+          const uint32_t kk = score_key(score);
+          if (ev_slot < 0 || kk < ev_key || (kk == ev_key && pos > ev_pos)) {
+            ev_key = kk;
+            ev_slot = i;
+            ev_pos = pos;
+          }
+        }
+      };
+      // prep(j) returns (the linear score part, or a heuristic score; the
+      // position) for finish(j)
       float2 pf_cur = j0 < t1 ? prep(j0) : make_float2(0.f, 0.f);
       for (int j = j0; j < t1; j += 2) {
         const float2 pf_next = j + 2 < t1 ? prep(j + 2) : make_float2(0.f, 0.f);
-        if constexpr (!FULL) finish(j, pf_cur.x, __float_as_int(pf_cur.y));
+        if constexpr (HEUR) record_h(j, pf_cur.x, __float_as_int(pf_cur.y));
+        else if constexpr (!FULL) finish(j, pf_cur.x, __float_as_int(pf_cur.y));
         pf_cur = pf_next;
       }
       g += nTi;
@@ -979,17 +998,17 @@ bool fused_eligible(const Dev& p, int n) {
 
 int fused_smem_bytes() { return kSmemBytes; }
 
-template <int D, int G, bool LONG, bool FULL = false>
+template <int D, int G, bool LONG, bool FULL = false, bool HEUR = false>
 static cudaError_t launch_t(const FusedMaps& maps, const Dev& p, const Step& st, const FusedStep& fs,
                             const FusedPolicy& fp, int grid, cudaStream_t s) {
   static bool attr = false;
   if (!attr) {
-    cudaError_t e = cudaFuncSetAttribute(fused_kernel<D, G, LONG, FULL>, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes);
+    cudaError_t e = cudaFuncSetAttribute(fused_kernel<D, G, LONG, FULL, HEUR>, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes);
     if (e != cudaSuccess) return e;
     attr = true;
   }
   if (fs.half_rows == 0) {
-    fused_kernel<D, G, LONG, FULL><<<grid, kThreads, kSmemBytes, s>>>(maps.k, maps.v, p, st, fs, fp);
+    fused_kernel<D, G, LONG, FULL, HEUR><<<grid, kThreads, kSmemBytes, s>>>(maps.k, maps.v, p, st, fs, fp);
     return cudaGetLastError();
   }
   // the two CTAs of a half row wait on each other: a cooperative launch
@@ -1004,7 +1023,7 @@ static cudaError_t launch_t(const FusedMaps& maps, const Dev& p, const Step& st,
   la[0].val.cooperative = 1;
   cfg.attrs = la;
   cfg.numAttrs = 1;
-  return cudaLaunchKernelEx(&cfg, fused_kernel<D, G, LONG, FULL>, maps.k, maps.v, p, st, fs, fp);
+  return cudaLaunchKernelEx(&cfg, fused_kernel<D, G, LONG, FULL, HEUR>, maps.k, maps.v, p, st, fs, fp);
 }
 
 static int fused_grid(const Dev& p, int num_sms) { return p.R < num_sms ? p.R : num_sms; }
@@ -1021,8 +1040,11 @@ cudaError_t launch_fused_step(const FusedMaps& maps, const Dev& p, const Step& s
                               const FusedPolicy& fp, int num_sms, cudaStream_t s) {
   const int grid = fused_grid(p, num_sms);
   const bool lg = st.n > fused_onchip_tokens(p.G);
-#define DC_FUSED_LAUNCH(D, G) \
-  return lg ? launch_t<D, G, true>(maps, p, st, fs, fp, grid, s) : launch_t<D, G, false>(maps, p, st, fs, fp, grid, s)
+  // heuristic scorers: one instantiation for any row length
+#define DC_FUSED_LAUNCH(D, G)                                                                 \
+  return p.scorer != 0 ? launch_t<D, G, true, false, true>(maps, p, st, fs, fp, grid, s)      \
+         : lg          ? launch_t<D, G, true>(maps, p, st, fs, fp, grid, s)                   \
+                       : launch_t<D, G, false>(maps, p, st, fs, fp, grid, s)
   if (p.d == 128) {
     if (p.G == 4) DC_FUSED_LAUNCH(128, 4);
     if (p.G == 2) DC_FUSED_LAUNCH(128, 2);

@@ -311,7 +311,8 @@ __global__ void __launch_bounds__(kTile) split_v_kernel(Dev p, Step st) {
 #pragma unroll
         for (int e = 0; e < 5; ++e) p.feat[slot * 5 + e] = x[e];
       }
-      p.score[slot] = policy_score(wsm, H, p.layernorm, x);
+      p.score[slot] = p.scorer == 0 ? policy_score(wsm, H, p.layernorm, x)
+                                    : heuristic_score(p, alpha, p.pos[slot], st.p_newest);
     }
     __syncthreads();
     if (owns) {

@@ -37,7 +37,9 @@ class dc_config(C.Structure):
     _fields_ = [("batch", C.c_int), ("q_heads", C.c_int), ("window", C.c_int),
                 ("mlp_hidden", C.c_int), ("layernorm", C.c_int), ("alpha_mode", C.c_int),
                 ("engine", C.c_int), ("keep_features", C.c_int), ("seed", C.c_ulonglong),
-                ("stream", C.c_void_p), ("tail_split", C.c_int)]
+                ("stream", C.c_void_p), ("tail_split", C.c_int), ("scorer", C.c_int),
+                ("n_sinks", C.c_int), ("budget_ratio", C.c_float), ("budget_min", C.c_int),
+                ("budget_basis", C.c_int)]
 
 
 class DCError(RuntimeError):
@@ -136,7 +138,9 @@ class DistillCache:
     def __init__(self, layers: int, kv_heads: int, head_dim: int, capacity: int, budget: int, *,
                  batch: int = 1, q_heads: int | None = None, window: int = 64,
                  mlp_hidden: int = 128, layernorm: int = 1, alpha_mode: int = 0, engine: int = 0,
-                 keep_features: bool = False, seed: int = 0, stream=None, tail_split: bool = True):
+                 keep_features: bool = False, seed: int = 0, stream=None, tail_split: bool = True,
+                 scorer: int = 0, n_sinks: int = 4, budget_ratio: float = 0.0, budget_min: int = 32,
+                 budget_basis: int = 0):
         import torch
         L = lib()
         cfg = dc_config()
@@ -145,6 +149,8 @@ class DistillCache:
         cfg.mlp_hidden, cfg.layernorm, cfg.alpha_mode = mlp_hidden, layernorm, alpha_mode
         cfg.engine, cfg.keep_features, cfg.seed = engine, int(bool(keep_features)), seed
         cfg.tail_split = int(bool(tail_split))
+        cfg.scorer, cfg.n_sinks = scorer, n_sinks
+        cfg.budget_ratio, cfg.budget_min, cfg.budget_basis = budget_ratio, budget_min, budget_basis
         if stream is None:
             stream = torch.cuda.current_stream()
         self.stream = stream

@@ -46,7 +46,7 @@ class LockStep:
     """Drives a DistillCache and oracle rows for a sample of its rows."""
 
     def __init__(self, wl: synth.Workload, rows, *, engine=0, device_inputs=False, capacity=None,
-                 tail_split=True):
+                 tail_split=True, scorer=0, n_sinks=4, budget_ratio=0.0, budget_min=32, budget_basis=0):
         import torch
         from paper_2608_08878_gb300 import dc, synth_device
         self.torch, self.dc, self.sd = torch, dc, synth_device
@@ -59,11 +59,17 @@ class LockStep:
                                      batch=wl.batch, q_heads=wl.q_heads, window=wl.window,
                                      mlp_hidden=wl.mlp_hidden, layernorm=wl.layernorm,
                                      alpha_mode=wl.alpha_mode, engine=engine, keep_features=True,
-                                     seed=wl.policy_seed, tail_split=tail_split)
+                                     seed=wl.policy_seed, tail_split=tail_split, scorer=scorer,
+                                     n_sinks=n_sinks, budget_ratio=budget_ratio, budget_min=budget_min,
+                                     budget_basis=budget_basis)
+        self.scorer, self.n_sinks = scorer, n_sinks
+        self.budget_ratio, self.budget_min, self.budget_basis = budget_ratio, budget_min, budget_basis
+        self.capacity = cap
         self.cache.set_policy(self.blob)
         self.orows = {}
+        alpha_mode = 1 if scorer == 1 else wl.alpha_mode  # H2O ranks by the cumulative mass
         for r in self.rows:
-            self.orows[r] = oracle.OracleRow(wl.head_dim, wl.group, wl.window, wl.alpha_mode, cap)
+            self.orows[r] = oracle.OracleRow(wl.head_dim, wl.group, wl.window, alpha_mode, cap)
         self.step_idx = 0
         self.stats = {"attn_max_abs": 0.0, "attn_rel": 0.0, "steps": 0, "evicted": 0}
 
@@ -125,7 +131,12 @@ class LockStep:
             for c in range(5):
                 close_rel(feat[:, c], res["feat"][:, c], FEAT_RTOL, FEAT_FLOOR, f"step {s} row {r} {names[c]}")
             score = self._row_slice(dc.BUF_SCORE, r, n)[order]
-            close_rel(score, res["score"], FEAT_RTOL, FEAT_FLOOR, f"step {s} row {r} score")
+            if self.scorer == 2:  # sinks, then positions relative to the newest: exact in fp32
+                ref = orow.heuristic_scores(2, self.n_sinks).astype(np.float32)
+                assert np.array_equal(score.astype(np.float32), ref), f"step {s} row {r} score"
+            else:
+                ref = res["score"] if self.scorer == 0 else orow.heuristic_scores(1)
+                close_rel(score, ref, FEAT_RTOL, FEAT_FLOOR, f"step {s} row {r} score")
         if evict:
             self.evict(budget)
         self.step_idx += 1
@@ -143,13 +154,22 @@ class LockStep:
             gpu_scores[r] = sc[order]
         self.cache.evict(budget)
         self.cache.sync()
-        B = budget if budget > 0 else self.wl.budget
+        B = budget if budget > 0 else self.budget_now(n)
         n2, _ = self.cache.length()
         assert n2 == min(n, B)
         self.stats["evicted"] += n - n2
         for r, orow in self.orows.items():
             orow.evict(B, gpu_scores[r])
             self.check_row_state(r, n2)
+
+    def budget_now(self, n_cached):
+        """The budget of the step that just ran (fixed, or the dynamic one)."""
+        if self.budget_ratio <= 0:
+            return self.wl.budget
+        _, seen = self.cache.length()
+        L = seen if self.budget_basis == 0 else n_cached
+        B = max(int(math.floor(float(np.float32(self.budget_ratio)) * L)), self.budget_min)
+        return min(B, self.capacity - 1)
 
     def check_row_state(self, r, n):
         dc = self.dc

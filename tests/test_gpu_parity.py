@@ -190,6 +190,57 @@ def test_fused_long_rows(prompt_len, budget):
     assert ls.cache.length()[0] == budget
 
 
+@pytest.mark.parametrize("engine", ENGINES)
+@pytest.mark.parametrize("scorer", [1, 2])
+def test_heuristic_scorers(engine, scorer):
+    """H2O (cumulative attention mass) and StreamingLLM (sinks + recent) on the
+    same attention/top-k/compaction path, all rows, past the window; then
+    dc_step bit-identical to dc_decode_step + dc_evict with that scorer."""
+    import torch
+    from paper_2608_08878_gb300 import dc
+    wl = synth.MISTRAL_1L.with_(prompt_len=900, budget=300, steps=70)
+    ls = LockStep(wl, range(wl.rows), engine=engine, scorer=scorer)
+    ls.load_prompt()
+    for s in range(wl.steps):
+        ls.step(check=(s < 3 or s % 16 == 0 or s >= 66))
+    wl2 = wl.with_(window=5)
+    a = LockStep(wl2, [], engine=engine, scorer=scorer)
+    b = LockStep(wl2, [], engine=engine, scorer=scorer)
+    a.load_prompt()
+    b.load_prompt()
+    for s in range(8):
+        q, kn, vn = a._inputs(s)
+        oa = a.cache.step(q, kn, vn)
+        ob = b.cache.decode_step(q, kn, vn)
+        b.cache.evict()
+        torch.cuda.synchronize()
+        assert torch.equal(oa, ob), s
+        n = a.cache.length()[0]
+        for which in (dc.BUF_K, dc.BUF_POS, dc.BUF_S, dc.BUF_Z):
+            assert torch.equal(a.cache.buffer(which)[:, :n], b.cache.buffer(which)[:, :n]), (s, which)
+
+
+@pytest.mark.parametrize("engine", ENGINES)
+@pytest.mark.parametrize("basis", [0, 1])
+def test_dynamic_budget(engine, basis):
+    """B_t = max(floor(r L_t), B_min) with L_t the tokens seen (basis 0: the
+    cache grows with the sequence) or the cached tokens (basis 1: it shrinks to
+    B_min); every step checked against the oracle with that budget."""
+    wl = synth.MISTRAL_1L.with_(prompt_len=700, budget=600, steps=12)
+    cap = wl.prompt_len + wl.steps + 8
+    ls = LockStep(wl, range(wl.rows), engine=engine, capacity=cap, budget_ratio=0.25, budget_min=32,
+                  budget_basis=basis)
+    ls.load_prompt()
+    lengths = []
+    for _ in range(wl.steps):
+        ls.step()
+        lengths.append(ls.cache.length()[0])
+    if basis == 0:
+        assert lengths[-1] == (wl.prompt_len + wl.steps) // 4
+    else:
+        assert lengths[:4] == [175, 44, 32, 32] and lengths[-1] == 32
+
+
 def test_engine_choice():
     from paper_2608_08878_gb300 import dc
     big = dc.DistillCache(32, 8, 128, 200, 100, batch=1)

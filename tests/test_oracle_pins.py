@@ -340,3 +340,56 @@ def test_capacity_overflow_leaves_row_unchanged():
     with pytest.raises(OverflowError):
         row.append(np.zeros((2, 4), np.uint16), np.zeros((2, 4), np.uint16))
     assert len(row) == 4
+
+
+# --------------------------------------------------------------------------
+# Heuristic scorers (H2O, StreamingLLM) on the same path
+# --------------------------------------------------------------------------
+
+def test_h2o_scores_are_cumulative_mass_brute_force():
+    """H2O ranks by the attention mass a token received since it entered the
+    cache: recomputed here from torch softmax over every step's cache."""
+    rng = np.random.default_rng(21)
+    d, G, T, steps, B = 16, 2, 30, 6, 24
+    row = oracle.OracleRow(d, G, 4, 1, T + steps + 2)
+    k0, v0 = rand_bits(rng, T, d), rand_bits(rng, T, d)
+    row.append(k0, v0)
+    keys = {p: k0[p] for p in range(T)}
+    mass = {p: 0.0 for p in range(T)}
+    blob = synth.policy_weights(3, 8)
+    for s in range(steps):
+        q, kn, vn = rand_bits(rng, G, d), rand_bits(rng, 1, d)[0], rand_bits(rng, 1, d)[0]
+        row.step(q, kn, vn, blob, 8, 1)
+        p_new = T + s
+        keys[p_new] = kn
+        mass[p_new] = 0.0
+        pos = row.positions()
+        a = softmax_rows(q, np.stack([keys[p] for p in pos]))  # [G][n]
+        for i, p in enumerate(pos):
+            mass[p] += a[:, i].mean()
+        h = row.heuristic_scores(1)
+        np.testing.assert_allclose(h, [mass[p] for p in pos], rtol=1e-12, atol=1e-15)
+        # evict with the H2O scores: the kept set is the top-B by (mass desc, position asc)
+        want = sorted(pos, key=lambda p: (-mass[p], p))[:B]
+        row.evict(B, h.astype(np.float32))
+        assert sorted(row.positions().tolist()) == sorted(want)
+        for p in set(mass) - set(row.positions().tolist()):
+            mass.pop(p)
+
+
+@pytest.mark.parametrize("n_sinks", [0, 4])
+def test_streamingllm_keeps_sinks_and_most_recent(n_sinks):
+    """StreamingLLM keeps the first n_sinks positions and then the most recent
+    tokens: after every eviction the cache is exactly that set."""
+    rng = np.random.default_rng(22)
+    d, G, T, B = 8, 2, 40, 16
+    row = oracle.OracleRow(d, G, 4, 0, T + 20)
+    row.append(rand_bits(rng, T, d), rand_bits(rng, T, d))
+    blob = synth.policy_weights(3, 8)
+    for s in range(10):
+        row.step(rand_bits(rng, G, d), rand_bits(rng, 1, d)[0], rand_bits(rng, 1, d)[0], blob, 8, 1)
+        h = row.heuristic_scores(2, n_sinks)
+        row.evict(B, h.astype(np.float32))
+        newest = T + s
+        want = list(range(n_sinks)) + list(range(newest - (B - n_sinks) + 1, newest + 1))
+        assert row.positions().tolist() == want
