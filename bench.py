@@ -523,6 +523,39 @@ def run_sweep(args):
             "clocks": clk.summary(), "data": "synthetic"}), flush=True)
 
 
+def run_train(args):
+    """Training-side kernels (App. C) at the paper's training scale (L = 4096
+    tokens, B = 1024): the exact Plackett-Luce log-partition and Gumbel-top-B
+    with log-probabilities, for 64 sequences; one JSON line."""
+    import torch
+    from paper_2608_08878_gb300 import build, dc
+    torch.cuda.set_device(0)
+    build.build()
+    rows, L, B, tau = 64, 4096, 1024, 1.0
+    g = torch.Generator(device="cuda").manual_seed(5)
+    s = torch.randn((rows, L), device="cuda", generator=g) * 3.0
+    u = torch.rand((rows, L), device="cuda", generator=g).clamp_(1e-12, 1.0 - 1e-7)
+    gum = -torch.log(-torch.log(u))
+    stream = torch.cuda.current_stream()
+    out = {}
+    for name, fn in (("log_partition", lambda: dc.pl_log_partition(s, B, tau)),
+                     ("gumbel_top_b_with_logp", lambda: dc.gumbel_top_b(s, gum, B, tau))):
+        for _ in range(3):
+            fn()
+        torch.cuda.synchronize()
+        ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        reps = 10
+        ev0.record(stream)
+        for _ in range(reps):
+            fn()
+        ev1.record(stream)
+        torch.cuda.synchronize()
+        ms = ev0.elapsed_time(ev1) / reps
+        out[name] = {"ms_per_call": ms, "dp_cells_per_s": rows * L * B / (ms / 1e3)}
+    print(json.dumps({"training_kernels": out, "rows": rows, "L": L, "B": B, "tau": tau,
+                      "data": "synthetic"}), flush=True)
+
+
 def main():
     ap = argparse.ArgumentParser(description=__doc__.splitlines()[0])
     ap.add_argument("--gpus", type=int, default=1)
@@ -541,6 +574,7 @@ def main():
     ap.add_argument("--sweep", action="store_true",
                     help="throughput sweep (batch x context x ratio): one JSON line per point")
     ap.add_argument("--sweep-points", default=None, help="e.g. 1x4096x10,64x32768x50 (default: all 36)")
+    ap.add_argument("--train", action="store_true", help="time the training-side kernels (App. C)")
     args = ap.parse_args()
     if args.layers:
         _OVERRIDES["layers"] = args.layers
@@ -554,6 +588,9 @@ def main():
         ap.error("--warmup must be >= 3")
     if args.sweep:
         run_sweep(args)
+        return
+    if args.train:
+        run_train(args)
         return
     if args.impl == "reference":
         res = run_reference(args)

@@ -265,6 +265,37 @@ const char* dc_noalloc_last_error(void);
  * h is NULL). Valid until the next call on the handle. */
 const char* dc_last_error(const dc_cache* h);
 
+/* ---------------------------------------------------------------------------
+ * Training-side kernels (App. C). Handle-free; device pointers, asynchronous on
+ * `stream` (a cudaStream_t, NULL for the default stream).
+ * ------------------------------------------------------------------------- */
+
+/* Exact log-partition function of the Plackett-Luce distribution over size-B
+ * subsets (App. C): out[r] = log sum_{a subset of [L], |a| = B}
+ * exp(sum_{i in a} scores[r][i] / tau), for `rows` independent rows.
+ * scores: fp32 [rows][L]; out: fp32 [rows]. Computed by the O(L B) dynamic
+ * programme over the elementary symmetric polynomials, in base-2 log space,
+ * fp32 with the hardware exp2/log2 (the error grows at most linearly in L:
+ * |error| <= 2 L 2^-24 (|log Z| + max |s| / tau) + L 2^-21). Needs
+ * 1 <= B <= L, rows <= 65535, B <= 25599, tau > 0;
+ * else DC_ERR_INVALID_ARG (message in dc_train_last_error()). */
+dc_status dc_pl_log_partition(const float* scores, int rows, int L, int B, float tau, float* out,
+                              void* stream);
+
+/* Gumbel-top-B sampling (Sec. 3.1.2, App. C): per row, the perturbed scores
+ * scores[r][i] / tau + gumbel[r][i] (each operation rounded to fp32; gumbel
+ * holds caller-drawn Gumbel(0, 1) noise, fp32 [rows][L]); the B largest are
+ * kept (ties: lower index first) and their indices written to idx[r][0..B) in
+ * ascending order (int32 [rows][B]). If logp is not NULL, logp[r] =
+ * sum_{i in a} scores[r][i] / tau - log Z, the log-probability of the sampled
+ * subset under the Plackett-Luce distribution; logz_scratch (fp32 [rows])
+ * receives log Z. Same argument rules as dc_pl_log_partition. */
+dc_status dc_gumbel_top_b(const float* scores, const float* gumbel, int rows, int L, int B, float tau,
+                          int* idx, float* logp, float* logz_scratch, void* stream);
+
+/* Message of the last failed training-side call of this thread. */
+const char* dc_train_last_error(void);
+
 #ifdef __cplusplus
 }
 #endif

@@ -51,6 +51,9 @@ def lib():
             L.dco_row_window_sums.argtypes = [P, P, P, P]
             L.dco_row_window_sums_prior.argtypes = [P, P, P]
             L.dco_row_heuristic_scores.argtypes = [P, C.c_int, C.c_int, P]
+            L.dco_pl_logz.argtypes = [P, C.c_int, C.c_int, C.c_double]
+            L.dco_pl_logz.restype = C.c_double
+            L.dco_gumbel_topb.argtypes = [P, P, C.c_int, C.c_int, C.c_float, P]
             L.dco_attend.argtypes = [P, P, P, C.c_int, C.c_int, C.c_int, P, P]
             L.dco_policy.argtypes = [P, C.c_int, P, C.c_int, C.c_int, P]
             _lib = L
@@ -163,4 +166,20 @@ def policy(x: np.ndarray, mlp: np.ndarray, hidden: int, layernorm: int) -> np.nd
     mlp = np.ascontiguousarray(mlp, dtype=np.float32)
     out = np.empty(x.shape[0])
     lib().dco_policy(_ptr(x), x.shape[0], _ptr(mlp), hidden, layernorm, _ptr(out))
+    return out
+
+
+def pl_logz(scores, B: int, tau: float = 1.0) -> float:
+    """log Z of the Plackett-Luce distribution over size-B subsets (App. C)."""
+    s = np.ascontiguousarray(scores, dtype=np.float64)
+    return lib().dco_pl_logz(_ptr(s), s.shape[0], B, tau)
+
+
+def gumbel_topb(scores, gumbel, B: int, tau: float = 1.0) -> np.ndarray:
+    """Indices (ascending) of the B largest fp32 perturbed scores s/tau + g."""
+    s = np.ascontiguousarray(scores, dtype=np.float32)
+    g = np.ascontiguousarray(gumbel, dtype=np.float32)
+    out = np.empty(B, dtype=np.int32)
+    if lib().dco_gumbel_topb(_ptr(s), _ptr(g), s.shape[0], B, tau, _ptr(out)) != 0:
+        raise ValueError("bad arguments")
     return out

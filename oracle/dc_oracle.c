@@ -394,3 +394,77 @@ void dco_row_window_sums_prior(const dco_row* r, double* S, double* Z) {
   if (S) memcpy(S, r->Sp, sizeof(double) * (size_t)r->n);
   if (Z) memcpy(Z, r->Zp, sizeof(double) * (size_t)r->n);
 }
+
+/* ------------------------------------------------------------------------
+ * Training side (App. C): the Plackett-Luce log-partition over size-B subsets
+ * and Gumbel-top-B selection.
+ * ---------------------------------------------------------------------- */
+
+/* log Z = log sum_{|a| = B} exp(sum_{i in a} s_i / tau), as the log of the
+ * elementary symmetric polynomial e_B(x) of x_i = exp(s_i / tau): items are
+ * added one at a time, e_k <- e_k + x_i e_{k-1} (highest k first), in log
+ * space. Returns -inf when B > L. */
+static double log_add(double a, double b) {
+  if (a == -INFINITY) return b;
+  if (b == -INFINITY) return a;
+  const double m = a > b ? a : b;
+  return m + log1p(exp(-fabs(a - b)));
+}
+
+double dco_pl_logz(const double* s, int L, int B, double tau) {
+  if (B < 0 || L < 0) return NAN;
+  double* e = (double*)malloc(sizeof(double) * (size_t)(B + 1));
+  if (!e) return NAN;
+  e[0] = 0.0;
+  for (int k = 1; k <= B; ++k) e[k] = -INFINITY;
+  for (int i = 0; i < L; ++i) {
+    const double y = s[i] / tau;
+    for (int k = B; k >= 1; --k) e[k] = log_add(e[k], y + e[k - 1]);
+  }
+  const double out = e[B];
+  free(e);
+  return out;
+}
+
+/* Gumbel-top-B: the perturbed scores v_i = fl32(fl32(s_i / tau) + g_i) (each
+ * operation rounded to fp32, as the device computes them), sorted by (value
+ * descending, index ascending); the first B indices, written ascending. A NaN
+ * value ranks below every number. Returns 0, or -1 on bad arguments. */
+typedef struct {
+  float v;
+  int i;
+} gt_item;
+
+static int gt_cmp(const void* pa, const void* pb) {
+  const gt_item* a = (const gt_item*)pa;
+  const gt_item* b = (const gt_item*)pb;
+  const int an = a->v != a->v, bn = b->v != b->v;
+  if (an != bn) return an - bn; /* NaN last */
+  if (!an) {
+    if (a->v > b->v) return -1;
+    if (a->v < b->v) return 1;
+  }
+  return (a->i > b->i) - (a->i < b->i);
+}
+
+static int int_cmp(const void* pa, const void* pb) {
+  const int a = *(const int*)pa, b = *(const int*)pb;
+  return (a > b) - (a < b);
+}
+
+int dco_gumbel_topb(const float* s, const float* g, int L, int B, float tau, int* idx) {
+  if (L < 1 || B < 1 || B > L || !(tau > 0.f)) return -1;
+  gt_item* it = (gt_item*)malloc(sizeof(gt_item) * (size_t)L);
+  if (!it) return -1;
+  for (int i = 0; i < L; ++i) {
+    volatile float y = s[i] / tau; /* fp32 quotient */
+    volatile float v = y + g[i];   /* fp32 sum */
+    it[i].v = v == 0.f ? 0.f : v;  /* -0 ranks as +0 */
+    it[i].i = i;
+  }
+  qsort(it, (size_t)L, sizeof *it, gt_cmp);
+  for (int k = 0; k < B; ++k) idx[k] = it[k].i;
+  qsort(idx, (size_t)B, sizeof(int), int_cmp);
+  free(it);
+  return 0;
+}

@@ -86,6 +86,14 @@ void dco_attend(const uint16_t* q, const uint16_t* k, const uint16_t* v, int n, 
 /* The policy MLP on m feature vectors x [m][5] -> score [m]. */
 void dco_policy(const double* x, int m, const float* mlp, int hidden, int layernorm, double* score);
 
+/* Training side (App. C). log Z of the Plackett-Luce distribution over
+ * size-B subsets of the L scores s at temperature tau (fp64). */
+double dco_pl_logz(const double* s, int L, int B, double tau);
+
+/* Gumbel-top-B: indices (ascending) of the B largest fp32 perturbed scores
+ * s_i / tau + g_i (ties: lower index). Returns 0 or -1. */
+int dco_gumbel_topb(const float* s, const float* g, int L, int B, float tau, int* idx);
+
 #ifdef __cplusplus
 }
 #endif

@@ -23,7 +23,8 @@ INCLUDE = os.path.join(os.path.dirname(HERE), "include")
 LIB_MAIN = os.path.join(HERE, "libdistillcache.so")
 LIB_SYNTH = os.path.join(HERE, "libdc_synth.so")
 
-MAIN_SOURCES = ["dc_cache.cu", "dc_split.cu", "dc_evict.cu", "dc_full.cu", "dc_fused.cu", "dc_noalloc.cu"]
+MAIN_SOURCES = ["dc_cache.cu", "dc_split.cu", "dc_evict.cu", "dc_full.cu", "dc_fused.cu", "dc_noalloc.cu",
+                "dc_train.cu"]
 SYNTH_SOURCES = ["synth.cu"]
 
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]

@@ -29,7 +29,7 @@ EXPORTS = ["dc_config_default", "dc_cache_create", "dc_cache_destroy", "dc_polic
            "dc_decode_step_host", "dc_evict", "dc_full_decode", "dc_get_length", "dc_buffer_bytes",
            "dc_copy_buffer", "dc_sync", "dc_last_error", "dc_phase_name", "dc_profile_enable",
            "dc_profile_read", "dc_step", "dc_step_host", "dc_engine", "dc_attend_noalloc",
-           "dc_noalloc_last_error"]
+           "dc_noalloc_last_error", "dc_pl_log_partition", "dc_gumbel_top_b", "dc_train_last_error"]
 PHASES = ["append", "attend", "stats", "score", "combine", "evict", "full"]
 
 
@@ -81,6 +81,10 @@ def lib():
             L.dc_noalloc_last_error.argtypes = []
             L.dc_noalloc_last_error.restype = C.c_char_p
             L.dc_full_decode.argtypes = [P, P, P]
+            L.dc_pl_log_partition.argtypes = [P, I, I, I, C.c_float, P, P]
+            L.dc_gumbel_top_b.argtypes = [P, P, I, I, I, C.c_float, P, P, P, P]
+            L.dc_train_last_error.argtypes = []
+            L.dc_train_last_error.restype = C.c_char_p
             L.dc_get_length.argtypes = [P, C.POINTER(I), C.POINTER(C.c_longlong)]
             L.dc_buffer_bytes.argtypes = [P, I, C.POINTER(S)]
             L.dc_copy_buffer.argtypes = [P, I, I, I, P, S]
@@ -92,7 +96,8 @@ def lib():
             L.dc_profile_enable.argtypes = [P, I]
             L.dc_profile_read.argtypes = [P, P, P]
             for name in EXPORTS:
-                if name not in ("dc_policy_blob_len", "dc_last_error", "dc_phase_name", "dc_noalloc_last_error"):
+                if name not in ("dc_policy_blob_len", "dc_last_error", "dc_phase_name", "dc_noalloc_last_error",
+                                "dc_train_last_error"):
                     getattr(L, name).restype = I
             _lib = L
     return _lib
@@ -125,6 +130,37 @@ def attend_noalloc(q, k, v, out=None, stream=None):
     if st != DC_OK:
         raise DCError(st, lib().dc_noalloc_last_error().decode())
     return out
+
+
+def pl_log_partition(scores, B: int, tau: float = 1.0, out=None, stream=None):
+    """Exact log Z of the Plackett-Luce distribution over size-B subsets for
+    each row of scores (fp32 CUDA tensor [rows][L]) -> fp32 [rows] (App. C)."""
+    import torch
+    rows, L = scores.shape
+    if out is None:
+        out = torch.empty(rows, dtype=torch.float32, device=scores.device)
+    s = (stream or torch.cuda.current_stream()).cuda_stream
+    st = lib().dc_pl_log_partition(scores.data_ptr(), rows, L, B, tau, out.data_ptr(), s)
+    if st != DC_OK:
+        raise DCError(st, lib().dc_train_last_error().decode())
+    return out
+
+
+def gumbel_top_b(scores, gumbel, B: int, tau: float = 1.0, with_logp: bool = True, stream=None):
+    """Gumbel-top-B sample per row (scores, gumbel: fp32 CUDA tensors [rows][L]):
+    the B kept indices ascending (int32 [rows][B]) and, if with_logp, the
+    subset's Plackett-Luce log-probability (fp32 [rows]) (App. C)."""
+    import torch
+    rows, L = scores.shape
+    idx = torch.empty((rows, B), dtype=torch.int32, device=scores.device)
+    logp = torch.empty(rows, dtype=torch.float32, device=scores.device) if with_logp else None
+    logz = torch.empty(rows, dtype=torch.float32, device=scores.device) if with_logp else None
+    s = (stream or torch.cuda.current_stream()).cuda_stream
+    st = lib().dc_gumbel_top_b(scores.data_ptr(), gumbel.data_ptr(), rows, L, B, tau, idx.data_ptr(),
+                               _ptr(logp), _ptr(logz), s)
+    if st != DC_OK:
+        raise DCError(st, lib().dc_train_last_error().decode())
+    return idx, logp
 
 
 def _ptr(t) -> int:

@@ -51,6 +51,8 @@ def test_config_defaults():
     assert dc.lib().dc_config_default(C.byref(cfg)) == dc.DC_OK
     assert (cfg.batch, cfg.q_heads, cfg.window, cfg.mlp_hidden, cfg.layernorm, cfg.alpha_mode,
             cfg.engine, cfg.keep_features, cfg.seed) == (1, 0, 64, 128, 1, 0, 0, 0, 0)
+    assert (cfg.tail_split, cfg.scorer, cfg.n_sinks, cfg.budget_ratio, cfg.budget_min,
+            cfg.budget_basis) == (1, 0, 4, 0.0, 32, 0)
     assert dc.lib().dc_config_default(None) == dc.DC_ERR_INVALID_ARG
 
 
@@ -70,7 +72,8 @@ def test_create_rejects_bad_shapes_without_touching_the_device(args, field):
 def test_create_rejects_bad_config():
     L = dc.lib()
     for field, value in [("q_heads", 12), ("window", 0), ("mlp_hidden", 100), ("alpha_mode", 2),
-                         ("engine", 5)]:
+                         ("engine", 5), ("scorer", 3), ("n_sinks", -1), ("budget_ratio", 1.5),
+                         ("budget_min", 0), ("budget_basis", 2)]:
         cfg = dc.dc_config()
         L.dc_config_default(C.byref(cfg))
         setattr(cfg, field, value)
@@ -85,3 +88,14 @@ def test_null_handles_are_rejected():
     assert L.dc_append(None, None, None, 0) == dc.DC_ERR_INVALID_ARG
     assert L.dc_sync(None) == dc.DC_ERR_INVALID_ARG
     assert L.dc_policy_init(0, 0, None, 0) == dc.DC_ERR_INVALID_ARG
+
+
+def test_training_kernels_validate_before_touching_the_device():
+    L = dc.lib()
+    for args in [(1, 10, 11, 1.0), (0, 10, 5, 1.0), (1, 10, 5, 0.0), (1, 10, 0, 1.0)]:
+        rows, n, B, tau = args
+        assert L.dc_pl_log_partition(C.c_void_p(16), rows, n, B, tau, C.c_void_p(16), None) == dc.DC_ERR_INVALID_ARG
+        assert L.dc_gumbel_top_b(C.c_void_p(16), C.c_void_p(16), rows, n, B, tau, C.c_void_p(16), None, None,
+                                 None) == dc.DC_ERR_INVALID_ARG
+    assert L.dc_pl_log_partition(None, 1, 10, 5, 1.0, C.c_void_p(16), None) == dc.DC_ERR_INVALID_ARG
+    assert b"B <= L" in L.dc_train_last_error() or b"NULL" in L.dc_train_last_error()

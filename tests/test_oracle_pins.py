@@ -393,3 +393,93 @@ def test_streamingllm_keeps_sinks_and_most_recent(n_sinks):
         newest = T + s
         want = list(range(n_sinks)) + list(range(newest - (B - n_sinks) + 1, newest + 1))
         assert row.positions().tolist() == want
+
+
+# --------------------------------------------------------------------------
+# Training side (App. C): Plackett-Luce log-partition, Gumbel-top-B
+# --------------------------------------------------------------------------
+
+@pytest.mark.parametrize("L", [1, 2, 5, 9])
+def test_pl_logz_brute_force_subsets(L):
+    """log Z is the log-sum-exp over every size-B subset of the subset's score
+    sum / tau: enumerated here for every B."""
+    from scipy.special import logsumexp
+    rng = np.random.default_rng(30 + L)
+    s = rng.standard_normal(L) * 3.0
+    for tau in (1.0, 0.5):
+        for B in range(1, L + 1):
+            sums = [sum(s[list(a)]) / tau for a in itertools.combinations(range(L), B)]
+            assert oracle.pl_logz(s, B, tau) == pytest.approx(logsumexp(sums), rel=1e-12, abs=1e-12)
+
+
+def test_pl_logz_closed_forms():
+    """B = 1: log-sum-exp of s / tau; B = L: sum of s / tau; equal scores c:
+    log C(L, B) + B c / tau."""
+    from scipy.special import logsumexp
+    rng = np.random.default_rng(31)
+    s = rng.standard_normal(1000) * 4.0
+    assert oracle.pl_logz(s, 1, 0.7) == pytest.approx(logsumexp(s / 0.7), rel=1e-12)
+    assert oracle.pl_logz(s, 1000, 0.7) == pytest.approx(s.sum() / 0.7, rel=1e-12)
+    c, L, B = 1.25, 1000, 300
+    want = math.lgamma(L + 1) - math.lgamma(B + 1) - math.lgamma(L - B + 1) + B * c
+    assert oracle.pl_logz(np.full(L, c), B, 1.0) == pytest.approx(want, rel=1e-12)
+
+
+def test_gumbel_topb_matches_lexsort():
+    """The kept set is the B largest fp32 perturbed scores (ties: lower index),
+    with -0 equal to +0: against numpy's lexsort on the same fp32 values."""
+    rng = np.random.default_rng(32)
+    L, B, tau = 500, 123, np.float32(0.5)
+    s = np.round(rng.standard_normal(L) * 4).astype(np.float32)   # many ties
+    g = np.zeros(L, dtype=np.float32)
+    g[::3] = np.round(rng.gumbel(size=len(g[::3]))).astype(np.float32)
+    s[7], g[7], s[8], g[8] = np.float32(-0.0), np.float32(0.0), np.float32(0.0), np.float32(0.0)
+    v = (s / tau + g).astype(np.float32)
+    v[v == 0] = 0.0
+    order = np.lexsort((np.arange(L), -v.astype(np.float64)))
+    want = np.sort(order[:B])
+    assert np.array_equal(oracle.gumbel_topb(s, g, B, float(tau)), want)
+
+
+def _pl_without_replacement_subset_prob(x, a):
+    """Probability that sequential Plackett-Luce draws without replacement
+    (weights x) pick exactly the set a in its first |a| draws: the sum over
+    the orderings of a of prod_j x_j / (weight not yet drawn)."""
+    total, p = float(sum(x)), 0.0
+    for perm in itertools.permutations(a):
+        rem, q = total, 1.0
+        for i in perm:
+            q *= x[i] / rem
+            rem -= x[i]
+        p += q
+    return p
+
+
+def test_gumbel_topb_samples_plackett_luce():
+    """Gumbel-top-B draws the B items of Plackett-Luce sampling without
+    replacement: subset frequencies of 40000 seeded draws against those
+    probabilities. For B = 1 this is exp(s_i / tau - log Z) (App. C); for
+    1 < B < L the subset law differs from exp(sum_a s / tau - log Z) (see the
+    design notes), which the second half checks is a real difference."""
+    rng = np.random.default_rng(33)
+    L, tau, N = 5, 1.0, 40000
+    s = np.array([1.0, 0.2, -0.5, 0.7, -1.2], dtype=np.float32)
+    x = np.exp(s.astype(np.float64) / tau)
+    g = rng.gumbel(size=(N, L)).astype(np.float32)
+    for B in (1, 2):
+        logz = oracle.pl_logz(s.astype(np.float64), B, tau)
+        counts = {}
+        for n in range(N):
+            a = tuple(oracle.gumbel_topb(s, g[n], B, tau).tolist())
+            counts[a] = counts.get(a, 0) + 1
+        for a in itertools.combinations(range(L), B):
+            p = _pl_without_replacement_subset_prob(x, a)
+            sd = math.sqrt(p * (1 - p) / N)
+            assert abs(counts.get(a, 0) / N - p) < 5 * sd + 1e-4, (B, a, counts.get(a, 0) / N, p)
+            p_paper = math.exp(float(s[list(a)].astype(np.float64).sum()) / tau - logz)
+            if B == 1:
+                assert p_paper == pytest.approx(p, rel=1e-12)
+        if B == 2:
+            a = (0, 3)
+            assert abs(_pl_without_replacement_subset_prob(x, a) -
+                       math.exp(float(s[list(a)].astype(np.float64).sum()) / tau - logz)) > 0.02
