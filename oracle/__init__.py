@@ -51,6 +51,16 @@ def lib():
             L.dco_row_window_sums.argtypes = [P, P, P, P]
             L.dco_row_window_sums_prior.argtypes = [P, P, P]
             L.dco_row_heuristic_scores.argtypes = [P, C.c_int, C.c_int, P]
+            L.dco_seq_new.restype = P
+            L.dco_seq_new.argtypes = [C.c_int] * 6
+            L.dco_seq_free.argtypes = [P]
+            L.dco_seq_append.argtypes = [P, P, P, C.c_int]
+            L.dco_seq_step.argtypes = [P, P, P, P, P, C.c_int, C.c_int, P, P, P]
+            L.dco_seq_evict.argtypes = [P, C.c_int, P]
+            L.dco_seq_len.argtypes = [P]
+            L.dco_seq_positions.argtypes = [P, P]
+            L.dco_seq_kv_bits.argtypes = [P, C.c_int, P, P]
+            L.dco_seq_window_sums_prior.argtypes = [P, P, P]
             L.dco_pl_logz.argtypes = [P, C.c_int, C.c_int, C.c_double]
             L.dco_pl_logz.restype = C.c_double
             L.dco_gumbel_topb.argtypes = [P, P, C.c_int, C.c_int, C.c_float, P]
@@ -183,3 +193,69 @@ def gumbel_topb(scores, gumbel, B: int, tau: float = 1.0) -> np.ndarray:
     if lib().dco_gumbel_topb(_ptr(s), _ptr(g), s.shape[0], B, tau, _ptr(out)) != 0:
         raise ValueError("bad arguments")
     return out
+
+
+class OracleSeq:
+    """Global token mode (Sec. 3.1.1): one sequence of R rows (layers x KV
+    heads) sharing its token set; features pooled over all R x G heads, one
+    score and one argtop_B per sequence."""
+
+    def __init__(self, rows: int, head_dim: int, group: int, window: int, alpha_mode: int, capacity: int):
+        self.R, self.d, self.G = rows, head_dim, group
+        self._h = lib().dco_seq_new(rows, head_dim, group, window, alpha_mode, capacity)
+        if not self._h:
+            raise ValueError("dco_seq_new rejected its arguments")
+
+    def __del__(self):
+        h = getattr(self, "_h", None)
+        if h:
+            lib().dco_seq_free(h)
+            self._h = None
+
+    def append(self, k_bits, v_bits) -> None:
+        """k, v: [R][T][d] bf16 bits."""
+        k, v = _u16(k_bits), _u16(v_bits)
+        if lib().dco_seq_append(self._h, _ptr(k), _ptr(v), k.shape[1]) != 0:
+            raise ValueError("capacity exceeded")
+
+    def step(self, q_bits, k_new_bits, v_new_bits, mlp, hidden: int, layernorm: int):
+        """q [R][G][d], k_new/v_new [R][d] -> dict(o [R][G][d], feat, score, pos)."""
+        q, kn, vn = _u16(q_bits), _u16(k_new_bits), _u16(v_new_bits)
+        mlp = np.ascontiguousarray(mlp, dtype=np.float32)
+        n_max = len(self) + 1
+        o = np.empty((self.R, self.G, self.d))
+        feat = np.empty((n_max, 5))
+        score = np.empty(n_max)
+        n = lib().dco_seq_step(self._h, _ptr(q), _ptr(kn), _ptr(vn), _ptr(mlp), hidden, layernorm,
+                               _ptr(o), _ptr(feat), _ptr(score))
+        if n < 0:
+            raise ValueError("capacity exceeded")
+        return {"o": o, "feat": feat[:n], "score": score[:n], "pos": self.positions()}
+
+    def evict(self, budget: int, scores_f32=None) -> int:
+        s = None if scores_f32 is None else np.ascontiguousarray(scores_f32, dtype=np.float32)
+        n = lib().dco_seq_evict(self._h, budget, _ptr(s))
+        if n < 0:
+            raise RuntimeError("no scores to evict with")
+        return n
+
+    def __len__(self) -> int:
+        return lib().dco_seq_len(self._h)
+
+    def positions(self) -> np.ndarray:
+        out = np.empty(len(self), dtype=np.int64)
+        lib().dco_seq_positions(self._h, _ptr(out))
+        return out
+
+    def kv_bits(self, row: int):
+        n = len(self)
+        k = np.empty((n, self.d), dtype=np.uint16)
+        v = np.empty((n, self.d), dtype=np.uint16)
+        lib().dco_seq_kv_bits(self._h, row, _ptr(k), _ptr(v))
+        return k, v
+
+    def window_sums_prior(self):
+        n = len(self)
+        S, Z = np.empty(n), np.empty(n)
+        lib().dco_seq_window_sums_prior(self._h, _ptr(S), _ptr(Z))
+        return S, Z

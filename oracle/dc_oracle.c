@@ -468,3 +468,257 @@ int dco_gumbel_topb(const float* s, const float* g, int L, int B, float tau, int
   free(it);
   return 0;
 }
+
+/* ------------------------------------------------------------------------
+ * Global token mode (Sec. 3.1.1: the features of a token pool all heads and
+ * layers; one policy, one argtop_B per sequence). A sequence is R rows (its
+ * layers x KV heads) sharing one token set: the same positions in the same
+ * order in every row.
+ * ---------------------------------------------------------------------- */
+
+typedef struct {
+  int n;
+  int64_t* pos;  /* [n] ascending */
+  double* za;    /* [n]: sum over the sequence's (row, head) pairs of a */
+  double* sa;    /* [n]: the same sum weighted by each head's entropy */
+} seq_win;
+
+struct dco_seq {
+  int R, d, G, w, alpha_mode, cap;
+  int n;
+  int64_t seen;
+  uint16_t *kb, *vb; /* [R][cap][d] */
+  double *k, *v;     /* [R][cap][d] */
+  int64_t* pos;      /* [cap] */
+  double* acc;       /* [cap] cumulative alpha */
+  double *S, *Z, *Sp, *Zp;
+  double* score;
+  int have_scores;
+  seq_win* win;
+  int win_count, win_next;
+};
+
+static void seq_win_clear(seq_win* e) {
+  free(e->pos); free(e->za); free(e->sa);
+  memset(e, 0, sizeof *e);
+}
+
+void dco_seq_free(dco_seq* s) {
+  if (!s) return;
+  if (s->win)
+    for (int i = 0; i < s->w; ++i) seq_win_clear(&s->win[i]);
+  free(s->win); free(s->kb); free(s->vb); free(s->k); free(s->v); free(s->pos); free(s->acc);
+  free(s->S); free(s->Z); free(s->Sp); free(s->Zp); free(s->score);
+  free(s);
+}
+
+dco_seq* dco_seq_new(int R, int d, int G, int w, int alpha_mode, int cap) {
+  if (R <= 0 || d <= 0 || G <= 0 || w <= 0 || cap <= 0 || (alpha_mode != 0 && alpha_mode != 1)) return NULL;
+  dco_seq* s = (dco_seq*)calloc(1, sizeof *s);
+  if (!s) return NULL;
+  s->R = R; s->d = d; s->G = G; s->w = w; s->alpha_mode = alpha_mode; s->cap = cap;
+  const size_t kv = (size_t)R * cap * d;
+  s->kb = (uint16_t*)calloc(kv, sizeof(uint16_t));
+  s->vb = (uint16_t*)calloc(kv, sizeof(uint16_t));
+  s->k = (double*)calloc(kv, sizeof(double));
+  s->v = (double*)calloc(kv, sizeof(double));
+  s->pos = (int64_t*)calloc((size_t)cap, sizeof(int64_t));
+  s->acc = (double*)calloc((size_t)cap, sizeof(double));
+  s->S = (double*)calloc((size_t)cap, sizeof(double));
+  s->Z = (double*)calloc((size_t)cap, sizeof(double));
+  s->Sp = (double*)calloc((size_t)cap, sizeof(double));
+  s->Zp = (double*)calloc((size_t)cap, sizeof(double));
+  s->score = (double*)calloc((size_t)cap, sizeof(double));
+  s->win = (seq_win*)calloc((size_t)w, sizeof(seq_win));
+  if (!s->kb || !s->vb || !s->k || !s->v || !s->pos || !s->acc || !s->S || !s->Z || !s->Sp || !s->Zp ||
+      !s->score || !s->win) {
+    dco_seq_free(s);
+    return NULL;
+  }
+  return s;
+}
+
+/* The token of row r at slot i. */
+static void seq_put(dco_seq* s, int r, int i, const uint16_t* k, const uint16_t* v) {
+  const size_t o = ((size_t)r * s->cap + i) * s->d;
+  for (int c = 0; c < s->d; ++c) {
+    s->kb[o + c] = k[c];
+    s->vb[o + c] = v[c];
+    s->k[o + c] = bf16_to_double(k[c]);
+    s->v[o + c] = bf16_to_double(v[c]);
+  }
+}
+
+int dco_seq_append(dco_seq* s, const uint16_t* k, const uint16_t* v, int T) {
+  if (T < 0 || s->n + T > s->cap) return -1;
+  for (int t = 0; t < T; ++t) {
+    for (int r = 0; r < s->R; ++r)
+      seq_put(s, r, s->n, k + ((size_t)r * T + t) * s->d, v + ((size_t)r * T + t) * s->d);
+    s->pos[s->n] = s->seen;
+    s->acc[s->n] = 0.0;
+    s->n += 1;
+    s->seen += 1;
+  }
+  s->have_scores = 0;
+  return 0;
+}
+
+int dco_seq_step(dco_seq* s, const uint16_t* q, const uint16_t* k_new, const uint16_t* v_new,
+                 const float* mlp, int hidden, int layernorm, double* o, double* feat, double* score) {
+  const int R = s->R, d = s->d, G = s->G;
+  if (s->n + 1 > s->cap) return -1;
+  /* Algorithm 1: every row's cache already holds the new pair. */
+  for (int r = 0; r < R; ++r) seq_put(s, r, s->n, k_new + (size_t)r * d, v_new + (size_t)r * d);
+  s->pos[s->n] = s->seen;
+  s->acc[s->n] = 0.0;
+  s->n += 1;
+  s->seen += 1;
+  const int n = s->n;
+  const int N = R * G; /* attention heads pooled per token */
+  double* a = (double*)malloc(sizeof(double) * (size_t)R * n * G);
+  double* Hh = (double*)malloc(sizeof(double) * (size_t)R * G);
+  double* qd = (double*)malloc(sizeof(double) * (size_t)G * d);
+  double* oo = (double*)malloc(sizeof(double) * (size_t)G * d);
+  double* Kr = (double*)malloc(sizeof(double) * (size_t)n * d);
+  double* Vr = (double*)malloc(sizeof(double) * (size_t)n * d);
+  for (int r = 0; r < R; ++r) {
+    for (int i = 0; i < G * d; ++i) qd[i] = bf16_to_double(q[(size_t)r * G * d + i]);
+    memcpy(Kr, s->k + (size_t)r * s->cap * d, sizeof(double) * (size_t)n * d);
+    memcpy(Vr, s->v + (size_t)r * s->cap * d, sizeof(double) * (size_t)n * d);
+    attend_rows(qd, Kr, Vr, n, d, G, a + (size_t)r * n * G, oo, Hh + (size_t)r * G);
+    if (o) memcpy(o + (size_t)r * G * d, oo, sizeof(double) * (size_t)G * d);
+  }
+  /* This step's pooled mass and entropy-weighted mass per token, kept (keyed
+   * by position) in the window of the last w steps [Sec. 3.1.1, H_i]. */
+  seq_win* e = &s->win[s->win_next];
+  seq_win_clear(e);
+  e->n = n;
+  e->pos = (int64_t*)malloc(sizeof(int64_t) * (size_t)n);
+  e->za = (double*)calloc((size_t)n, sizeof(double));
+  e->sa = (double*)calloc((size_t)n, sizeof(double));
+  memcpy(e->pos, s->pos, sizeof(int64_t) * (size_t)n);
+  for (int i = 0; i < n; ++i)
+    for (int r = 0; r < R; ++r)
+      for (int h = 0; h < G; ++h) {
+        const double ah = a[((size_t)r * n + i) * G + h];
+        e->za[i] += ah;
+        e->sa[i] += ah * Hh[(size_t)r * G + h];
+      }
+  s->win_next = (s->win_next + 1) % s->w;
+  if (s->win_count < s->w) s->win_count += 1;
+  const int newest_entry = (s->win_next + s->w - 1) % s->w;
+
+  double* x = (double*)malloc(sizeof(double) * (size_t)n * 5);
+  const int64_t newest = s->pos[n - 1];
+  const double pos_den = (double)(newest > 1 ? newest : 1);
+  for (int i = 0; i < n; ++i) {
+    /* alpha_i: mean over every (row, head) pair of the mass token i receives */
+    double mean = 0.0;
+    for (int r = 0; r < R; ++r)
+      for (int h = 0; h < G; ++h) mean += a[((size_t)r * n + i) * G + h];
+    mean /= N;
+    double alpha = mean;
+    if (s->alpha_mode == 1) {
+      s->acc[i] += mean;
+      alpha = s->acc[i];
+    }
+    /* sigma_i: population variance over the same pairs */
+    double var = 0.0;
+    for (int r = 0; r < R; ++r)
+      for (int h = 0; h < G; ++h) {
+        const double dv = a[((size_t)r * n + i) * G + h] - mean;
+        var += dv * dv;
+      }
+    var /= N;
+    /* |v_i|: mean over the rows of the value norm */
+    double vn = 0.0;
+    for (int r = 0; r < R; ++r) {
+      double ss = 0.0;
+      const double* vv = s->v + ((size_t)r * s->cap + i) * d;
+      for (int c = 0; c < d; ++c) ss += vv[c] * vv[c];
+      vn += sqrt(ss);
+    }
+    vn /= R;
+    /* H_i over the window of recent steps, pooled */
+    double S = 0.0, Z = 0.0, Sp = 0.0, Zp = 0.0;
+    for (int qi = 0; qi < s->win_count; ++qi) {
+      const seq_win* we = &s->win[qi];
+      const int j = find_pos(we->pos, we->n, s->pos[i]);
+      if (j < 0) continue;
+      Z += we->za[j];
+      S += we->sa[j];
+      if (qi != newest_entry) {
+        Zp += we->za[j];
+        Sp += we->sa[j];
+      }
+    }
+    s->S[i] = S; s->Z[i] = Z; s->Sp[i] = Sp; s->Zp[i] = Zp;
+    x[(size_t)i * 5 + 0] = alpha;
+    x[(size_t)i * 5 + 1] = vn;
+    x[(size_t)i * 5 + 2] = var;
+    x[(size_t)i * 5 + 3] = Z > 0.0 ? S / Z : 0.0;
+    x[(size_t)i * 5 + 4] = (double)s->pos[i] / pos_den;
+  }
+  dco_policy(x, n, mlp, hidden, layernorm, s->score);
+  s->have_scores = 1;
+  if (feat) memcpy(feat, x, sizeof(double) * (size_t)n * 5);
+  if (score) memcpy(score, s->score, sizeof(double) * (size_t)n);
+  free(a); free(Hh); free(qd); free(oo); free(Kr); free(Vr); free(x);
+  return n;
+}
+
+int dco_seq_evict(dco_seq* s, int budget, const float* scores_f32) {
+  const int n = s->n, d = s->d;
+  if (!scores_f32 && !s->have_scores) return -1;
+  int keep_n = budget < n ? budget : n;
+  if (keep_n < 0) keep_n = 0;
+  rank_item* it = (rank_item*)malloc(sizeof(rank_item) * (size_t)(n > 0 ? n : 1));
+  for (int i = 0; i < n; ++i) {
+    it[i].s = scores_f32 ? (double)scores_f32[i] : s->score[i];
+    it[i].p = s->pos[i];
+    it[i].i = i;
+  }
+  /* one argtop_B for the whole sequence [Algorithm 1] */
+  qsort(it, (size_t)n, sizeof(rank_item), rank_cmp);
+  char* keep = (char*)calloc((size_t)(n > 0 ? n : 1), 1);
+  for (int j = 0; j < keep_n; ++j) keep[it[j].i] = 1;
+  /* prune every row the same way: survivors in ascending position order */
+  int w = 0;
+  for (int i = 0; i < n; ++i) {
+    if (!keep[i]) continue;
+    if (w != i) {
+      for (int r = 0; r < s->R; ++r) {
+        const size_t src = ((size_t)r * s->cap + i) * d, dst = ((size_t)r * s->cap + w) * d;
+        memmove(s->kb + dst, s->kb + src, sizeof(uint16_t) * (size_t)d);
+        memmove(s->vb + dst, s->vb + src, sizeof(uint16_t) * (size_t)d);
+        memmove(s->k + dst, s->k + src, sizeof(double) * (size_t)d);
+        memmove(s->v + dst, s->v + src, sizeof(double) * (size_t)d);
+      }
+      s->pos[w] = s->pos[i];
+      s->acc[w] = s->acc[i];
+      s->S[w] = s->S[i]; s->Z[w] = s->Z[i]; s->Sp[w] = s->Sp[i]; s->Zp[w] = s->Zp[i];
+      s->score[w] = s->score[i];
+    }
+    ++w;
+  }
+  s->n = w;
+  s->have_scores = 0;
+  free(it);
+  free(keep);
+  return w;
+}
+
+int dco_seq_len(const dco_seq* s) { return s->n; }
+
+void dco_seq_positions(const dco_seq* s, int64_t* pos) { memcpy(pos, s->pos, sizeof(int64_t) * (size_t)s->n); }
+
+void dco_seq_kv_bits(const dco_seq* s, int r, uint16_t* k, uint16_t* v) {
+  const size_t o = (size_t)r * s->cap * s->d, m = (size_t)s->n * s->d;
+  memcpy(k, s->kb + o, sizeof(uint16_t) * m);
+  memcpy(v, s->vb + o, sizeof(uint16_t) * m);
+}
+
+void dco_seq_window_sums_prior(const dco_seq* s, double* S, double* Z) {
+  if (S) memcpy(S, s->Sp, sizeof(double) * (size_t)s->n);
+  if (Z) memcpy(Z, s->Zp, sizeof(double) * (size_t)s->n);
+}

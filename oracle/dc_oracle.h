@@ -86,6 +86,26 @@ void dco_attend(const uint16_t* q, const uint16_t* k, const uint16_t* v, int n, 
 /* The policy MLP on m feature vectors x [m][5] -> score [m]. */
 void dco_policy(const double* x, int m, const float* mlp, int hidden, int layernorm, double* score);
 
+/* Global token mode (Sec. 3.1.1, "across all heads and layers"): a sequence of
+ * R rows (its layers x KV heads) sharing one token set. The features of a
+ * token pool all R x G attention heads: alpha (mean mass), sigma (population
+ * variance), H (entropy-weighted window mass over the pooled heads), |v| (mean
+ * over the rows of the value norm) and pos; one policy score and one argtop_B
+ * per sequence; every row pruned the same way. k/v/q arrays are row-major
+ * over the rows: append k [R][T][d]; step q [R][G][d], k_new/v_new [R][d],
+ * o [R][G][d], feat [n][5], score [n]. */
+typedef struct dco_seq dco_seq;
+dco_seq* dco_seq_new(int R, int d, int G, int w, int alpha_mode, int cap);
+void dco_seq_free(dco_seq* s);
+int dco_seq_append(dco_seq* s, const uint16_t* k, const uint16_t* v, int T);
+int dco_seq_step(dco_seq* s, const uint16_t* q, const uint16_t* k_new, const uint16_t* v_new,
+                 const float* mlp, int hidden, int layernorm, double* o, double* feat, double* score);
+int dco_seq_evict(dco_seq* s, int budget, const float* scores_f32);
+int dco_seq_len(const dco_seq* s);
+void dco_seq_positions(const dco_seq* s, int64_t* pos);
+void dco_seq_kv_bits(const dco_seq* s, int r, uint16_t* k, uint16_t* v);
+void dco_seq_window_sums_prior(const dco_seq* s, double* S, double* Z);
+
 /* Training side (App. C). log Z of the Plackett-Luce distribution over
  * size-B subsets of the L scores s at temperature tau (fp64). */
 double dco_pl_logz(const double* s, int L, int B, double tau);

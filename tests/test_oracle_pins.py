@@ -483,3 +483,75 @@ def test_gumbel_topb_samples_plackett_luce():
             a = (0, 3)
             assert abs(_pl_without_replacement_subset_prob(x, a) -
                        math.exp(float(s[list(a)].astype(np.float64).sum()) / tau - logz)) > 0.02
+
+
+# --------------------------------------------------------------------------
+# Global token mode (features over all heads and layers of a sequence)
+# --------------------------------------------------------------------------
+
+def test_global_mode_with_one_row_is_the_row_oracle():
+    """A sequence of one row pools nothing: every step's features, scores,
+    window sums and evictions equal the per-row oracle's."""
+    rng = np.random.default_rng(40)
+    d, G, T, w, cap = 16, 4, 60, 3, 80
+    blob = synth.policy_weights(5, 32)
+    row = oracle.OracleRow(d, G, w, 1, cap)
+    seq = oracle.OracleSeq(1, d, G, w, 1, cap)
+    k, v = rand_bits(rng, T, d), rand_bits(rng, T, d)
+    row.append(k, v)
+    seq.append(k[None], v[None])
+    for s in range(8):
+        q, kn, vn = rand_bits(rng, G, d), rand_bits(rng, 1, d)[0], rand_bits(rng, 1, d)[0]
+        a = row.step(q, kn, vn, blob, 32, 1)
+        b = seq.step(q[None], kn[None], vn[None], blob, 32, 1)
+        np.testing.assert_allclose(b["o"][0], a["o"], rtol=0, atol=0)
+        np.testing.assert_allclose(b["feat"], a["feat"], rtol=1e-13, atol=1e-15)
+        np.testing.assert_allclose(b["score"], a["score"], rtol=1e-13, atol=1e-15)
+        np.testing.assert_allclose(seq.window_sums_prior(), row.window_sums_prior(), rtol=1e-13, atol=1e-15)
+        row.evict(50)
+        seq.evict(50)
+        assert np.array_equal(row.positions(), seq.positions())
+        assert all(np.array_equal(x, y) for x, y in zip(row.kv_bits(), seq.kv_bits(0)))
+
+
+def test_global_mode_pooled_features_brute_force():
+    """alpha, sigma, |v|, H and pos of a 3-row sequence recomputed from torch
+    softmax over every row's heads, stacked, over a 3-step window; every row
+    pruned to the same survivors, which are the sequence's top-B."""
+    rng = np.random.default_rng(41)
+    R, d, G, T, w, B = 3, 16, 2, 25, 3, 20
+    blob = synth.policy_weights(6, 32)
+    seq = oracle.OracleSeq(R, d, G, w, 0, T + 10)
+    K = {r: list(rand_bits(rng, T, d)) for r in range(R)}
+    V = {r: list(rand_bits(rng, T, d)) for r in range(R)}
+    seq.append(np.stack([np.stack(K[r]) for r in range(R)]), np.stack([np.stack(V[r]) for r in range(R)]))
+    pos = list(range(T))
+    hist = []  # per step: {position: (sum a, sum a H)}
+    for s in range(6):
+        q = rand_bits(rng, R, G, d)
+        kn, vn = rand_bits(rng, R, d), rand_bits(rng, R, d)
+        for r in range(R):
+            K[r].append(kn[r]); V[r].append(vn[r])
+        pos.append(T + s)
+        res = seq.step(q, kn, vn, blob, 32, 1)
+        a = np.concatenate([softmax_rows(q[r], np.stack(K[r])) for r in range(R)])  # [R*G][n]
+        Hh = np.array([scipy.stats.entropy(a[j]) for j in range(R * G)])
+        hist.append({p: (a[:, i].sum(), (a[:, i] * Hh).sum()) for i, p in enumerate(pos)})
+        hist = hist[-w:]
+        vnorm = np.mean([np.linalg.norm(widen(np.stack(V[r])), axis=1) for r in range(R)], axis=0)
+        S = np.array([sum(h[p][1] for h in hist if p in h) for p in pos])
+        Z = np.array([sum(h[p][0] for h in hist if p in h) for p in pos])
+        want = np.stack([a.mean(0), vnorm, a.var(0), np.where(Z > 0, S / Z, 0.0),
+                         np.array(pos) / max(pos[-1], 1)], axis=1)
+        np.testing.assert_allclose(res["feat"], want, rtol=1e-11, atol=1e-14)
+        sc = res["score"].astype(np.float32)
+        keep = np.sort(np.lexsort((np.array(pos), -sc.astype(np.float64)))[:B])
+        seq.evict(B, sc)
+        kept_pos = [pos[i] for i in keep]
+        assert seq.positions().tolist() == kept_pos
+        for r in range(R):
+            K[r] = [K[r][i] for i in keep]
+            V[r] = [V[r][i] for i in keep]
+            kb, vb = seq.kv_bits(r)
+            assert np.array_equal(kb, np.stack(K[r])) and np.array_equal(vb, np.stack(V[r]))
+        pos = kept_pos
