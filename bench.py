@@ -254,7 +254,7 @@ def run_gpu(args):
     cache = dc.DistillCache(wl.layers, wl.kv_heads, wl.head_dim, wl.capacity, wl.budget,
                             batch=wl.batch, q_heads=wl.q_heads, window=wl.window,
                             mlp_hidden=wl.mlp_hidden, layernorm=wl.layernorm, engine=args.engine,
-                            seed=wl.policy_seed)
+                            seed=wl.policy_seed, global_tokens=args.global_tokens)
     chunk = 4096
     for t0 in range(0, wl.prompt_len, chunk):
         k, v = synth_device.prompt(wl, t0, min(chunk, wl.prompt_len - t0))
@@ -361,6 +361,8 @@ def run_gpu(args):
                        "kv_heads": wl.kv_heads, "head_dim": wl.head_dim, "context": wl.prompt_len,
                        "budget": wl.budget, "window": wl.window, "policy": f"5-{wl.mlp_hidden}-LN-ReLU-1",
                        "engine": engine, "parallelism": f"replicas x{world}",
+                       "selection": "per sequence (global token mode)" if args.global_tokens else
+                       "per (layer, KV head) row",
                        "l2": f"inputs larger than L2: {bytes_step / 1e9:.2f} GB streamed per step vs 129 MB L2",
                        "steady_tokens_per_row": n_steady},
             "hbm": {"algorithmic_bytes_per_step": bytes_step, "gbs": gbs,
@@ -575,6 +577,8 @@ def main():
                     help="throughput sweep (batch x context x ratio): one JSON line per point")
     ap.add_argument("--sweep-points", default=None, help="e.g. 1x4096x10,64x32768x50 (default: all 36)")
     ap.add_argument("--train", action="store_true", help="time the training-side kernels (App. C)")
+    ap.add_argument("--global-tokens", action="store_true",
+                    help="the global token mode (features over all heads and layers, one selection per sequence)")
     args = ap.parse_args()
     if args.layers:
         _OVERRIDES["layers"] = args.layers

@@ -87,6 +87,14 @@ typedef struct {
   int budget_basis;   /* L_t of the dynamic budget: 0 (default) tokens seen so far
                          (the sequence length), 1 the tokens cached before the
                          eviction, |C_t| */
+  int global_tokens;  /* 1: global token mode (Sec. 3.1.1, "across all heads and
+                         layers"): a token's features pool the attention of every
+                         query head of every layer of its sequence, one policy
+                         score and one argtop_B per sequence, and all rows of a
+                         sequence keep the same tokens. The sequence's window
+                         sums, cumulative alpha, features and scores are kept in
+                         its home row (layer 0, KV head 0). Runs on the split
+                         engine. 0 (default): one selection per row. */
 } dc_config;
 
 /* Fills *cfg with the defaults above (batch 1, q_heads 0 meaning 4 * kv_heads,

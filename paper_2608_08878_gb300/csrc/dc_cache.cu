@@ -169,6 +169,7 @@ dc_status launch_error(dc_cache* h, const char* what) {
 
 // Fused engine for this step? (auto: only when the rows fill the GPU)
 bool use_fused(const dc_cache* h, int n) {
+  if (h->dev.seq_rows) return false;  // the global token mode runs on the split engine
   if (!h->fused_ok || !dc::fused_eligible(h->dev, n)) return false;
   if (h->cfg.engine == 2) return true;
   if (h->cfg.engine == 0) return 2 * h->dev.R >= h->num_sms;
@@ -215,6 +216,11 @@ bool run_split_step(dc_cache* h, const dc::Step& st, const void* q, float* out) 
   { Phase ph(h, DC_PHASE_STATS, 1); dc::launch_split_stats(p, st, q, h->stream); }
   { Phase ph(h, DC_PHASE_SCORE, 1); dc::launch_split_v(p, st, h->stream); }
   { Phase ph(h, DC_PHASE_COMBINE, 1); dc::launch_split_out(p, st, out, h->stream); }
+  if (p.seq_rows) {
+    // global token mode: pool the rows' partial sums per sequence
+    Phase ph(h, DC_PHASE_SCORE, 1);
+    dc::launch_glob_features(p, st, h->stream);
+  }
   return true;
 }
 
@@ -241,6 +247,7 @@ dc_status dc_config_default(dc_config* cfg) {
   cfg->budget_ratio = 0.f;
   cfg->budget_min = 32;
   cfg->budget_basis = 0;
+  cfg->global_tokens = 0;
   return DC_OK;
 }
 
@@ -292,6 +299,8 @@ dc_status dc_cache_create(int layers, int kv_heads, int head_dim, int capacity, 
       (cfg.budget_basis != 0 && cfg.budget_basis != 1))
     return fail(nullptr, DC_ERR_INVALID_ARG, "need 0 <= budget_ratio <= 1, budget_min >= 1, budget_basis 0 or 1");
   if (cfg.scorer == 1) cfg.alpha_mode = 1;  // H2O ranks by the cumulative mass
+  if (cfg.global_tokens != 0 && cfg.global_tokens != 1)
+    return fail(nullptr, DC_ERR_INVALID_ARG, "global_tokens must be 0 or 1");
   if (cfg.engine < 0 || cfg.engine > 2) return fail(nullptr, DC_ERR_INVALID_ARG, "engine must be 0, 1 or 2");
   const long long R = (long long)layers * cfg.batch * kv_heads;
   if (R > 65535 || (long long)capacity * R > (1ll << 40) || capacity > (1 << 30))
@@ -315,6 +324,8 @@ dc_status dc_cache_create(int layers, int kv_heads, int head_dim, int capacity, 
   p.w = cfg.window; p.hidden = cfg.mlp_hidden; p.layernorm = cfg.layernorm ? 1 : 0;
   p.alpha_mode = cfg.alpha_mode; p.keep_features = cfg.keep_features ? 1 : 0;
   p.scorer = cfg.scorer; p.n_sinks = cfg.n_sinks;
+  p.batch = cfg.batch;
+  p.seq_rows = cfg.global_tokens ? layers * kv_heads : 0;
   p.c = (float)(1.4426950408889634 / std::sqrt((double)head_dim));
   p.smax = (int)std::max(1ll, std::min(64ll, (8ll * h->num_sms + R - 1) / R));
   const size_t RC = (size_t)R * p.stride;
@@ -342,6 +353,10 @@ dc_status dc_cache_create(int layers, int kv_heads, int head_dim, int capacity, 
   A(&p.part, (size_t)R * p.smax * G * 4 * sizeof(float));
   A(&p.opart, (size_t)R * p.smax * G * head_dim * sizeof(float));
   A(&p.holes, RC * sizeof(int));
+  if (p.seq_rows) {
+    A(&p.gpart, RC * 2 * sizeof(float4));
+    A(&p.gmoves, (size_t)cfg.batch * (1 + 2 * (size_t)p.stride) * sizeof(int));
+  }
   A(&h->st_q, (size_t)R * G * head_dim * 2);
   A(&h->st_k, (size_t)R * head_dim * 2);
   A(&h->st_v, (size_t)R * head_dim * 2);
@@ -595,8 +610,9 @@ dc_status dc_evict(dc_cache* h, int budget) {
   const int B = effective_budget(h, budget, h->n, h->seen);
   const int keep = std::min(h->n, B);
   if (keep < h->n) {
-    Phase ph(h, DC_PHASE_EVICT, 1);
-    dc::launch_evict(h->dev, h->n, keep, h->stream);
+    Phase ph(h, DC_PHASE_EVICT, h->dev.seq_rows ? 2 : 1);
+    if (h->dev.seq_rows) dc::launch_glob_evict(h->dev, h->n, keep, h->stream);
+    else dc::launch_evict(h->dev, h->n, keep, h->stream);
     dc_status s = launch_error(h, "evict");
     if (s != DC_OK) return s;
   }

@@ -37,6 +37,14 @@ constexpr unsigned kStatusTimeout = 2u;
 struct Dev {
   int R, cap, stride, d, G, qh, kvh, w, hidden, layernorm, alpha_mode, keep_features;
   int scorer, n_sinks;  // 0 policy MLP, 1 H2O (cumulative alpha), 2 StreamingLLM
+  // global token mode: rows per sequence (layers x KV heads), 0 = per-row mode;
+  // batch = sequences. Per-token partial sums of each row ([R][stride][2]:
+  // window terms of the previous/departing queries, then this step's mass,
+  // squared mass, entropy-weighted mass and |v|) and each sequence's move
+  // list ([batch][1 + 2 stride]: count, then hole/mover pairs).
+  int seq_rows, batch;
+  float4* gpart;
+  int* gmoves;
   __nv_bfloat16* K;
   __nv_bfloat16* V;
   int* pos;

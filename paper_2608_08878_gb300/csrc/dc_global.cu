@@ -1,0 +1,141 @@
+// dc_global.cu -- the global token mode (Sec. 3.1.1: a token's features pool
+// every attention head of every layer; one policy score and one argtop_B per
+// sequence). The rows of a sequence (its layers x KV heads) share one token
+// set, slot for slot. The split engine's per-row kernels leave each row's share
+// of the per-token sums in Dev::gpart; here they are pooled per sequence (in a
+// fixed row order, so the window terms of a departing query cancel exactly the
+// sums they once entered), turned into features and scores, and the
+// sequence's selection is applied to every one of its rows.
+//
+// Per-sequence state lives in the sequence's home row (layer 0, KV head 0):
+// window sums, cumulative alpha, features and scores.
+#include "dc_common.cuh"
+#include "dc_kernels.h"
+#include "dc_select.cuh"
+
+namespace dc {
+namespace {
+
+constexpr int kFeatThreads = 256;
+constexpr int kSelThreads = 1024;
+constexpr int kMoveThreads = 256;
+
+__device__ __forceinline__ int seq_row(const Dev& p, int b, int l, int g) { return (l * p.batch + b) * p.kvh + g; }
+
+// grid (ceil(n / 256), batch), block 256; dynamic shared memory: the policy blob.
+__global__ void __launch_bounds__(kFeatThreads) glob_feature_kernel(Dev p, Step st) {
+  extern __shared__ float wsm[];
+  const int b = blockIdx.y, i = blockIdx.x * blockDim.x + threadIdx.x;
+  const int H = p.hidden, nblob = 9 * H + 1;
+  for (int e = threadIdx.x; e < nblob; e += blockDim.x) wsm[e] = p.policy[e];
+  __syncthreads();
+  if (i >= st.n) return;
+  const int layers = p.seq_rows / p.kvh;
+  const bool window = st.has_prev || st.has_dep;
+  float4 W = make_float4(0.f, 0.f, 0.f, 0.f), P = make_float4(0.f, 0.f, 0.f, 0.f);
+  for (int l = 0; l < layers; ++l)
+    for (int g = 0; g < p.kvh; ++g) {
+      const size_t slot = (size_t)seq_row(p, b, l, g) * p.stride + i;
+      if (window) {
+        const float4 w = p.gpart[slot * 2];
+        W.x += w.x; W.y += w.y; W.z += w.z; W.w += w.w;
+      }
+      const float4 q = p.gpart[slot * 2 + 1];
+      P.x += q.x; P.y += q.y; P.z += q.z; P.w += q.w;
+    }
+  const size_t s0 = (size_t)seq_row(p, b, 0, 0) * p.stride + i;
+  float4 sz = p.SZ[s0];
+  if (window) {
+    // the previous step's query joins the stored sums, the departing one leaves
+    sz = window_update(sz, W.y, W.w, W.x, W.z);
+    p.SZ[s0] = sz;
+  }
+  const float N = (float)(p.seq_rows * p.G);
+  const float mean = P.x / N;
+  const float var = fmaxf(P.y / N - mean * mean, 0.f);
+  const float Zt = __fadd_rn(__fadd_rn(sz.z, P.x), sz.w);
+  const float St = __fadd_rn(__fadd_rn(sz.x, P.z), sz.y);
+  float alpha = mean;
+  if (p.alpha_mode == 1) {
+    alpha = p.acc[s0] + mean;
+    p.acc[s0] = alpha;
+  }
+  const float pos_den = (float)max(st.p_newest, 1);
+  const int pos = p.pos[s0];
+  float x[5] = {alpha, P.w / (float)p.seq_rows, var, Zt > 0.f ? St / Zt : 0.f, (float)pos / pos_den};
+  if (p.keep_features)
+#pragma unroll
+    for (int e = 0; e < 5; ++e) p.feat[s0 * 5 + e] = x[e];
+  p.score[s0] = p.scorer == 0 ? policy_score(wsm, H, p.layernorm, x) : heuristic_score(p, alpha, pos, st.p_newest);
+}
+
+// grid (batch), block 1024: the sequence's selection as a move list.
+__global__ void __launch_bounds__(kSelThreads) glob_select_kernel(Dev p, int n, int B) {
+  __shared__ int hist[256];
+  __shared__ int sh[4];
+  __shared__ int wsum[kSelThreads / kWarp];
+  __shared__ unsigned long long best[kSelThreads / kWarp];
+  __shared__ int best_slot[kSelThreads / kWarp];
+  const SelectScratch scr{hist, sh, wsum, best, best_slot};
+  auto sync = [] { __syncthreads(); };
+  const int b = blockIdx.x;
+  const size_t base = (size_t)seq_row(p, b, 0, 0) * p.stride;
+  int* moves = p.gmoves + (size_t)b * (1 + 2 * (size_t)p.stride);
+  team_select_moves<kSelThreads>(p.score + base, p.pos + base, n, B, p.holes + base, moves, threadIdx.x, scr, sync);
+}
+
+// grid (R), block 256: every row applies its sequence's moves (one warp per
+// move); the home row also moves the sequence's state.
+__global__ void __launch_bounds__(kMoveThreads) glob_compact_kernel(Dev p) {
+  const int r = blockIdx.x;
+  const int b = (r / p.kvh) % p.batch;
+  const bool home = r == seq_row(p, b, 0, 0);
+  const int* moves = p.gmoves + (size_t)b * (1 + 2 * (size_t)p.stride);
+  const int count = moves[0];
+  const int lane = threadIdx.x % kWarp, warp = threadIdx.x / kWarp, nwarps = blockDim.x / kWarp;
+  const int VPR = p.d / 8;
+  const size_t base = (size_t)r * p.stride;
+  for (int k = warp; k < count; k += nwarps) {
+    const size_t dst = base + moves[1 + 2 * k], src = base + moves[2 + 2 * k];
+    uint4 kv = make_uint4(0, 0, 0, 0);
+    if (lane < VPR) kv = reinterpret_cast<const uint4*>(p.K)[src * VPR + lane];
+    else if (lane < 2 * VPR) kv = reinterpret_cast<const uint4*>(p.V)[src * VPR + lane - VPR];
+    const int ps = p.pos[src];
+    const float vn = p.vnorm[src];
+    float4 sz = make_float4(0.f, 0.f, 0.f, 0.f);
+    float ac = 0.f, sc = 0.f, ft = 0.f;
+    if (home) {
+      sz = p.SZ[src];
+      sc = p.score[src];
+      if (p.acc) ac = p.acc[src];
+      if (p.keep_features && lane < 5) ft = p.feat[src * 5 + lane];
+    }
+    if (lane < VPR) reinterpret_cast<uint4*>(p.K)[dst * VPR + lane] = kv;
+    else if (lane < 2 * VPR) reinterpret_cast<uint4*>(p.V)[dst * VPR + lane - VPR] = kv;
+    if (lane == 0) {
+      p.pos[dst] = ps;
+      p.vnorm[dst] = vn;
+      if (home) {
+        p.SZ[dst] = sz;
+        p.score[dst] = sc;
+        if (p.acc) p.acc[dst] = ac;
+      }
+    }
+    if (home && p.keep_features && lane < 5) p.feat[dst * 5 + lane] = ft;
+  }
+}
+
+}  // namespace
+
+void launch_glob_features(const Dev& p, const Step& st, cudaStream_t s) {
+  const dim3 grid((st.n + kFeatThreads - 1) / kFeatThreads, p.batch);
+  const size_t smem = (size_t)(9 * p.hidden + 1) * sizeof(float);
+  glob_feature_kernel<<<grid, kFeatThreads, smem, s>>>(p, st);
+}
+
+void launch_glob_evict(const Dev& p, int n, int B, cudaStream_t s) {
+  glob_select_kernel<<<p.batch, kSelThreads, 0, s>>>(p, n, B);
+  glob_compact_kernel<<<p.R, kMoveThreads, 0, s>>>(p);
+}
+
+}  // namespace dc

@@ -20,6 +20,11 @@ void launch_split_out(const Dev& p, const Step& st, float* out, cudaStream_t s);
 
 void launch_evict(const Dev& p, int n, int B, cudaStream_t s);
 
+// Global token mode: pooled per-sequence features and scores after the split
+// engine's per-row pass; the sequence's selection applied to all its rows.
+void launch_glob_features(const Dev& p, const Step& st, cudaStream_t s);
+void launch_glob_evict(const Dev& p, int n, int B, cudaStream_t s);
+
 // Window sums S (which 0) or Z (which 1) of rows [row0, row0 + nrows) as fp64
 // [nrows][cap].
 void launch_convert_sz(const Dev& p, int row0, int nrows, int which, double* dst, cudaStream_t s);

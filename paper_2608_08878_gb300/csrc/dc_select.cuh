@@ -242,4 +242,99 @@ __device__ void team_select_compact(const Dev& p, int r, int n, int B, const flo
   sync();
 }
 
+// The same selection as team_select_compact without moving anything: writes
+// the compaction's (hole, mover) pairs to moves[1 + 2k], moves[2 + 2k] and
+// their count to moves[0] (for sequences whose rows all move alike). `holes`
+// is scratch of n ints. Requires 1 <= B; B >= n gives no moves.
+template <int NT, class Sync>
+__device__ void team_select_moves(const float* score, const int* ps, int n, int B, int* holes, int* moves,
+                                  int tid, const SelectScratch& s, Sync sync) {
+  if (B >= n) {
+    if (tid == 0) moves[0] = 0;
+    sync();
+    return;
+  }
+  auto key = [&](int i) { return score_key(score[i]); };
+  if (n == B + 1) {
+    uint32_t bk = 0xFFFFFFFFu;
+    int bs = -1;
+    for (int i = tid; i < n; i += NT) {
+      const uint32_t k = key(i);
+      if (bs < 0 || k < bk || (k == bk && ps[i] > ps[bs])) { bk = k; bs = i; }
+    }
+    auto better = [&](uint32_t ka, int sa, uint32_t kb, int sb) {
+      if (sb < 0) return false;
+      if (sa < 0) return true;
+      return kb < ka || (kb == ka && ps[sb] > ps[sa]);
+    };
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) {
+      const uint32_t ok = __shfl_xor_sync(0xffffffffu, bk, off);
+      const int os = __shfl_xor_sync(0xffffffffu, bs, off);
+      if (better(bk, bs, ok, os)) { bk = ok; bs = os; }
+    }
+    const int lane = tid % kWarp, wid = tid / kWarp;
+    if (lane == 0) { s.best[wid] = bk; s.best_slot[wid] = bs; }
+    sync();
+    if (tid == 0) {
+      uint32_t fk = (uint32_t)s.best[0];
+      int e = s.best_slot[0];
+      for (int w = 1; w < NT / kWarp; ++w)
+        if (better(fk, e, (uint32_t)s.best[w], s.best_slot[w])) { fk = (uint32_t)s.best[w]; e = s.best_slot[w]; }
+      if (e >= 0 && e < B) {
+        moves[0] = 1;
+        moves[1] = e;
+        moves[2] = B;
+      } else {
+        moves[0] = 0;
+      }
+    }
+    sync();
+    return;
+  }
+  int gt = 0;
+  auto all = [](int) { return true; };
+  const uint32_t T = team_radix_select<NT>(n, B, key, all, tid, s, &gt, sync);
+  const int need_eq = B - gt;
+  int eq_local = 0;
+  for (int i = tid; i < n; i += NT) eq_local += (key(i) == T);
+  int eq_total;
+  (void)team_exclusive_scan<NT>(eq_local, tid, s.wsum, &eq_total, sync);
+  uint32_t P = 0;
+  if (eq_total > need_eq) {
+    auto pkey = [&](int i) { return ~(uint32_t)ps[i]; };
+    auto tied = [&](int i) { return key(i) == T; };
+    int gt2 = 0;
+    P = team_radix_select<NT>(n, need_eq, pkey, tied, tid, s, &gt2, sync);
+  }
+  auto keep = [&](int i) {
+    const uint32_t k = key(i);
+    return k > T || (k == T && ~(uint32_t)ps[i] >= P);
+  };
+  int nh = 0;
+  for (int c0 = 0; c0 < B; c0 += NT) {
+    const int i = c0 + tid;
+    const int f = (i < B && !keep(i)) ? 1 : 0;
+    int tot;
+    const int rank = team_exclusive_scan<NT>(f, tid, s.wsum, &tot, sync);
+    if (f) holes[nh + rank] = i;
+    nh += tot;
+  }
+  sync();
+  int nm = 0;
+  for (int c0 = B; c0 < n; c0 += NT) {
+    const int i = c0 + tid;
+    const int f = (i < n && keep(i)) ? 1 : 0;
+    int tot;
+    const int rank = team_exclusive_scan<NT>(f, tid, s.wsum, &tot, sync);
+    if (f && nm + rank < nh) {
+      moves[1 + 2 * (nm + rank)] = holes[nm + rank];
+      moves[2 + 2 * (nm + rank)] = i;
+    }
+    nm += tot;
+  }
+  if (tid == 0) moves[0] = nm < nh ? nm : nh;
+  sync();
+}
+
 }  // namespace dc

@@ -186,7 +186,8 @@ __global__ void __launch_bounds__(kTile) split_qk_kernel(Dev p, Step st,
           for (int h = 0; h < G; ++h) { rm[h] = ring_ml[1][h][0]; rnl[h] = ring_ml[1][h][1]; rH[h] = ring_ml[1][h][2]; }
           window_terms<G>(s + 2 * G, rm, rnl, rH, c, zd, sd);
         }
-        p.SZ[slot] = window_update(p.SZ[slot], sp_, sd, zp, zd);
+        if (p.seq_rows) p.gpart[slot * 2] = make_float4(zp, sp_, zd, sd);  // pooled per sequence later
+        else p.SZ[slot] = window_update(p.SZ[slot], sp_, sd, zp, zd);
       }
     }
   }
@@ -290,6 +291,13 @@ __global__ void __launch_bounds__(kTile) split_v_kernel(Dev p, Step st) {
           mean += a[h];
         }
       }
+      if (p.seq_rows) {
+        // global token mode: this row's share of the pooled per-token sums
+        float a2 = 0.f;
+#pragma unroll
+        for (int h = 0; h < G; ++h) a2 = fmaf(a[h], a[h], a2);
+        p.gpart[slot * 2 + 1] = make_float4(mean, a2, sc, p.vnorm[slot]);
+      } else {
       mean /= (float)G;
       float var = 0.f;
 #pragma unroll
@@ -313,6 +321,7 @@ __global__ void __launch_bounds__(kTile) split_v_kernel(Dev p, Step st) {
       }
       p.score[slot] = p.scorer == 0 ? policy_score(wsm, H, p.layernorm, x)
                                     : heuristic_score(p, alpha, p.pos[slot], st.p_newest);
+      }
     }
     __syncthreads();
     if (owns) {

@@ -39,7 +39,7 @@ class dc_config(C.Structure):
                 ("engine", C.c_int), ("keep_features", C.c_int), ("seed", C.c_ulonglong),
                 ("stream", C.c_void_p), ("tail_split", C.c_int), ("scorer", C.c_int),
                 ("n_sinks", C.c_int), ("budget_ratio", C.c_float), ("budget_min", C.c_int),
-                ("budget_basis", C.c_int)]
+                ("budget_basis", C.c_int), ("global_tokens", C.c_int)]
 
 
 class DCError(RuntimeError):
@@ -176,7 +176,7 @@ class DistillCache:
                  mlp_hidden: int = 128, layernorm: int = 1, alpha_mode: int = 0, engine: int = 0,
                  keep_features: bool = False, seed: int = 0, stream=None, tail_split: bool = True,
                  scorer: int = 0, n_sinks: int = 4, budget_ratio: float = 0.0, budget_min: int = 32,
-                 budget_basis: int = 0):
+                 budget_basis: int = 0, global_tokens: bool = False):
         import torch
         L = lib()
         cfg = dc_config()
@@ -187,6 +187,7 @@ class DistillCache:
         cfg.tail_split = int(bool(tail_split))
         cfg.scorer, cfg.n_sinks = scorer, n_sinks
         cfg.budget_ratio, cfg.budget_min, cfg.budget_basis = budget_ratio, budget_min, budget_basis
+        cfg.global_tokens = int(bool(global_tokens))
         if stream is None:
             stream = torch.cuda.current_stream()
         self.stream = stream

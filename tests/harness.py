@@ -187,3 +187,108 @@ class LockStep:
         oS, oZ = orow.window_sums_prior()
         close_rel(Z, oZ, FEAT_RTOL, FEAT_FLOOR, f"row {r} window mass Z")
         close_rel(S, oS, FEAT_RTOL, FEAT_FLOOR, f"row {r} window sum S")
+
+
+class SeqLockStep:
+    """Global token mode: drives a DistillCache with global_tokens and one
+    sequence oracle per sampled sequence (rows = layers x KV heads)."""
+
+    def __init__(self, wl: synth.Workload, seqs, *, capacity=None, scorer=0):
+        import torch
+        from paper_2608_08878_gb300 import dc
+        self.torch, self.dc, self.wl = torch, dc, wl
+        self.seqs = list(seqs)
+        cap = capacity or wl.capacity
+        self.blob = synth.policy_weights(wl.policy_seed, wl.mlp_hidden)
+        self.cache = dc.DistillCache(wl.layers, wl.kv_heads, wl.head_dim, cap, wl.budget, batch=wl.batch,
+                                     q_heads=wl.q_heads, window=wl.window, mlp_hidden=wl.mlp_hidden,
+                                     layernorm=wl.layernorm, alpha_mode=wl.alpha_mode, keep_features=True,
+                                     seed=wl.policy_seed, scorer=scorer, global_tokens=True)
+        self.cache.set_policy(self.blob)
+        self.scorer = scorer
+        R = wl.layers * wl.kv_heads
+        alpha_mode = 1 if scorer == 1 else wl.alpha_mode
+        self.oseqs = {b: oracle.OracleSeq(R, wl.head_dim, wl.group, wl.window, alpha_mode, cap) for b in self.seqs}
+        self.step_idx = 0
+        self.stats = {"attn_max_abs": 0.0, "evicted": 0}
+
+    def rows_of(self, b):
+        wl = self.wl
+        return [(l * wl.batch + b) * wl.kv_heads + g for l in range(wl.layers) for g in range(wl.kv_heads)]
+
+    def home(self, b):
+        return b * self.wl.kv_heads
+
+    def _dev(self, a):
+        return self.torch.from_numpy(a.view(np.int16)).view(self.torch.bfloat16).cuda()
+
+    def load_prompt(self):
+        wl = self.wl
+        k, v = synth.prompt_all(wl)
+        self.cache.append(self._dev(k), self._dev(v))
+        R = wl.layers * wl.kv_heads
+        for b, o in self.oseqs.items():
+            o.append(k[:, b].reshape(R, wl.prompt_len, wl.head_dim), v[:, b].reshape(R, wl.prompt_len, wl.head_dim))
+
+    def _slice(self, which, r, n):
+        return self.cache.buffer(which, r, 1)[0, :n].cpu().numpy()
+
+    def step(self, check=True, budget=0):
+        wl, dc = self.wl, self.dc
+        s = self.step_idx
+        q, kn, vn = synth.step_all(wl, s)
+        out = self.cache.decode_step(self._dev(q), self._dev(kn), self._dev(vn)).cpu().numpy()
+        self.cache.sync()
+        n, _ = self.cache.length()
+        R, G, d = wl.layers * wl.kv_heads, wl.group, wl.head_dim
+        gpu_scores = {}
+        for b, o in self.oseqs.items():
+            res = o.step(q[:, b].reshape(R, G, d), kn[:, b].reshape(R, d), vn[:, b].reshape(R, d),
+                         self.blob, wl.mlp_hidden, wl.layernorm)
+            h = self.home(b)
+            pos = self._slice(dc.BUF_POS, h, n)
+            order = np.argsort(pos, kind="stable")
+            assert np.array_equal(pos[order], res["pos"]), f"step {s} seq {b}: positions differ"
+            sc = self._slice(dc.BUF_SCORE, h, n)[order]
+            gpu_scores[b] = sc
+            if not check:
+                continue
+            for j, r in enumerate(self.rows_of(b)):
+                layer, _, g = wl.row_coords(r)
+                ma, _ = check_attention(out[layer, b, g * G:(g + 1) * G], res["o"][j], f"step {s} row {r} attention")
+                self.stats["attn_max_abs"] = max(self.stats["attn_max_abs"], ma)
+            feat = self._slice(dc.BUF_FEAT, h, n)[order]
+            for c, nm in enumerate(["alpha", "|v|", "sigma", "H", "pos"]):
+                close_rel(feat[:, c], res["feat"][:, c], FEAT_RTOL, FEAT_FLOOR, f"step {s} seq {b} {nm}")
+            if self.scorer == 2:  # sinks, then positions relative to the newest
+                newest = res["pos"][-1]
+                ref = np.where(res["pos"] < 4, np.float32(3e38), (res["pos"] - newest).astype(np.float32))
+                assert np.array_equal(sc.astype(np.float32), ref.astype(np.float32)), f"step {s} seq {b} score"
+            else:  # H2O ranks by the cumulative mass, the pooled alpha in cumulative mode
+                ref = res["score"] if self.scorer == 0 else res["feat"][:, 0]
+                close_rel(sc, ref, FEAT_RTOL, FEAT_FLOOR, f"step {s} seq {b} score")
+        self.cache.evict(budget)
+        self.cache.sync()
+        B = budget if budget > 0 else wl.budget
+        n2, _ = self.cache.length()
+        assert n2 == min(n, B)
+        self.stats["evicted"] += n - n2
+        for b, o in self.oseqs.items():
+            o.evict(B, gpu_scores[b])
+            want = o.positions()
+            for j, r in enumerate(self.rows_of(b)):
+                pos = self._slice(dc.BUF_POS, r, n2)
+                order = np.argsort(pos, kind="stable")
+                assert np.array_equal(pos[order], want), f"step {s} row {r}: retained positions differ"
+                K = self.cache.buffer(dc.BUF_K, r, 1)[0, :n2].view(self.torch.int16).cpu().numpy().view(np.uint16)
+                V = self.cache.buffer(dc.BUF_V, r, 1)[0, :n2].view(self.torch.int16).cpu().numpy().view(np.uint16)
+                ok, ov = o.kv_bits(j)
+                assert np.array_equal(K[order], ok) and np.array_equal(V[order], ov), f"row {r}: K/V bytes differ"
+            h = self.home(b)
+            pos = self._slice(dc.BUF_POS, h, n2)
+            order = np.argsort(pos, kind="stable")
+            oS, oZ = o.window_sums_prior()
+            close_rel(self._slice(dc.BUF_Z, h, n2)[order], oZ, FEAT_RTOL, FEAT_FLOOR, f"seq {b} window mass Z")
+            close_rel(self._slice(dc.BUF_S, h, n2)[order], oS, FEAT_RTOL, FEAT_FLOOR, f"seq {b} window sum S")
+        self.step_idx += 1
+        return out

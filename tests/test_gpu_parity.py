@@ -9,7 +9,7 @@ import pytest
 
 from paper_2608_08878_gb300 import synth
 
-from harness import LockStep, check_attention
+from harness import LockStep, SeqLockStep, check_attention
 
 pytestmark = pytest.mark.gpu
 
@@ -346,3 +346,27 @@ def test_aggressive_sampled_rows():
     ls.load_prompt()
     for s in range(18):
         ls.step(check=(s < 2 or s >= 15))
+
+
+@pytest.mark.parametrize("scorer", [0, 1, 2])
+def test_global_token_mode(scorer):
+    """Global token mode: features pooled over all heads and layers of each
+    sequence, one score and one selection per sequence, every row pruned
+    alike; prompt compression and steps past the window, all sequences."""
+    wl = synth.MISTRAL_1L.with_(layers=3, batch=2, kv_heads=2, q_heads=8, prompt_len=400, budget=150,
+                                steps=70, window=6)
+    ls = SeqLockStep(wl, range(wl.batch), scorer=scorer)
+    ls.load_prompt()
+    for s in range(wl.steps):
+        ls.step(check=(s < 3 or s % 16 == 0 or s >= 66))
+    assert ls.cache.length()[0] == wl.budget
+
+
+def test_global_token_mode_full_shape_sampled():
+    """The same at the Mistral-7B shape (32 layers x 8 KV heads = 256 rows per
+    sequence), a 2K prompt compressed to 512, then a steady step."""
+    wl = synth.MISTRAL_1L.with_(layers=32, batch=1, prompt_len=2048, budget=512, steps=2)
+    ls = SeqLockStep(wl, [0])
+    ls.load_prompt()
+    for _ in range(wl.steps):
+        ls.step()
