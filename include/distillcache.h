@@ -93,8 +93,9 @@ typedef struct {
                          score and one argtop_B per sequence, and all rows of a
                          sequence keep the same tokens. The sequence's window
                          sums, cumulative alpha, features and scores are kept in
-                         its home row (layer 0, KV head 0). Runs on the split
-                         engine. 0 (default): one selection per row. */
+                         its home row (layer 0, KV head 0). dc_step runs as
+                         dc_decode_step + dc_evict. 0 (default): one selection
+                         per row. */
 } dc_config;
 
 /* Fills *cfg with the defaults above (batch 1, q_heads 0 meaning 4 * kv_heads,

@@ -169,7 +169,6 @@ dc_status launch_error(dc_cache* h, const char* what) {
 
 // Fused engine for this step? (auto: only when the rows fill the GPU)
 bool use_fused(const dc_cache* h, int n) {
-  if (h->dev.seq_rows) return false;  // the global token mode runs on the split engine
   if (!h->fused_ok || !dc::fused_eligible(h->dev, n)) return false;
   if (h->cfg.engine == 2) return true;
   if (h->cfg.engine == 0) return 2 * h->dev.R >= h->num_sms;
@@ -513,13 +512,18 @@ dc_status dc_decode_step(dc_cache* h, const void* q, const void* k_new, const vo
   }
   const dc::Step st = begin_step(h);
   if (use_fused(h, st.n)) {
-    const dc::FusedStep fs = fused_args(h, st, q, out, 0, 0, 1);
+    const dc::FusedStep fs = fused_args(h, st, q, out, 0, 0, h->dev.seq_rows ? 0 : 1);
     cudaError_t e;
     {
       Phase ph(h, DC_PHASE_ATTEND, 1);
       e = dc::launch_fused_step(h->maps, h->dev, st, fs, h->fpol, h->num_sms, h->stream);
     }
     if (e != cudaSuccess) return cuda_fail(h, e, "fused step");
+    if (h->dev.seq_rows) {
+      // global token mode: pool the rows' partial sums per sequence
+      Phase ph(h, DC_PHASE_SCORE, 1);
+      dc::launch_glob_features(h->dev, st, h->stream);
+    }
   } else if (!run_split_step(h, st, q, out)) {
     return fail(h, DC_ERR_INVALID_ARG, "unsupported head_dim / group");
   }
@@ -536,7 +540,7 @@ dc_status dc_step(dc_cache* h, const void* q, const void* k_new, const void* v_n
     return fail(h, DC_ERR_INVALID_ARG, "q, k_new and v_new must be 16-byte aligned");
   if (h->n + 1 > h->capacity) return fail(h, DC_ERR_CAPACITY, "decode step exceeds capacity");
   const int n1 = h->n + 1;
-  if (!use_fused(h, n1)) {
+  if (!use_fused(h, n1) || h->dev.seq_rows) {  // global mode: per-sequence selection after the rows
     dc_status s = dc_decode_step(h, q, k_new, v_new, out);
     if (s != DC_OK) return s;
     return dc_evict(h, budget);

@@ -256,7 +256,11 @@ __device__ __forceinline__ Item read_item(volatile int* ring, int gr, volatile i
 // no window state, features, policy, select, or writes to the cache's state.
 // HEUR: a heuristic scorer (H2O or StreamingLLM, Dev::scorer) ranks the tokens
 // instead of the policy MLP, whose tensor-core layer is then skipped.
-template <int D, int G, bool LONG, bool FULL, bool HEUR>
+// GLOB: global token mode: each row leaves its share of the per-token sums in
+// Dev::gpart (window terms in the K pass; mass, squared mass, entropy-weighted
+// mass and |v| in the V pass); features, scores and the selection are made
+// per sequence afterwards.
+template <int D, int G, bool LONG, bool FULL, bool HEUR, bool GLOB>
 __global__ void __launch_bounds__(kThreads, 1)
     fused_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmV, Dev p,
                  Step st, FusedStep fs, FusedPolicy fp) {
@@ -380,7 +384,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           for (int j = it.t0; j < it.t1; ++j, ++g) {
             const int s = g % kStages;
             if (!mbar_wait(&bar[B_EMPTY + s], ((g / kStages) & 1) ^ 1, abort, p.dbg, 2u, (unsigned)g)) break;
-            mbar_expect_tx(&bar[B_FULL + s], kTileBytes + ((pass || FULL) ? 0u : 2560u));
+            mbar_expect_tx(&bar[B_FULL + s], kTileBytes + ((pass || FULL) ? 0u : GLOB ? 512u : 2560u));
             uint8_t* dst = smem + OFF_STAGE + s * kStageBytes;
             uint8_t* aux = smem + OFF_AUX + s * kAuxBytes;
             const int y = r * p.stride + j * kTok;
@@ -388,7 +392,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             if (D == 128) tma_load_2d(dst + 16384, tm, 64, y, &bar[B_FULL + s], pol);
             if (!FULL && !pass) {
               bulk_load(aux + kAuxPos, p.pos + y, 512, &bar[B_FULL + s]);
-              bulk_load(aux + kAuxSZ, p.SZ + y, 2048, &bar[B_FULL + s]);
+              if (!GLOB) bulk_load(aux + kAuxSZ, p.SZ + y, 2048, &bar[B_FULL + s]);
             }
             issued = g + 1;
           }
@@ -462,7 +466,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     __syncwarp();
   } else if (warp == 10) {
     // ------------------------------------------------------------ policy-layer MMA issuer
-    if (!FULL && !HEUR && lane == 0) {
+    if (!FULL && !HEUR && !GLOB && lane == 0) {
       const uint32_t id_m = idesc_bf16(128, 128, 0, 0);
       const uint32_t waddr = smem_u32(smem + OFF_W);
       int gv = 0;
@@ -559,8 +563,12 @@ __global__ void __launch_bounds__(kThreads, 1)
             window_terms<G>(S16 + 2 * G, dm, dnl, dH, c, zd, sd);
             const float mp = (st.has_prev && pos <= st.p_prev) ? 1.f : 0.f;
             const float md = (st.has_dep && pos <= st.p_dep) ? 1.f : 0.f;
-            sz = window_update(sz, sp * mp, sd * md, zp * mp, zd * md);
-            p.SZ[rbase + i] = sz;
+            if constexpr (GLOB) {
+              p.gpart[(rbase + i) * 2] = make_float4(zp * mp, sp * mp, zd * md, sd * md);
+            } else {
+              sz = window_update(sz, sp * mp, sd * md, zp * mp, zd * md);
+              p.SZ[rbase + i] = sz;
+            }
           }
         }
         if (!LONG || j < onchip_tiles<GS>()) {
@@ -682,11 +690,13 @@ __global__ void __launch_bounds__(kThreads, 1)
       float4 szA = kZero4, szB = kZero4;
       int posA = 0, posB = 0;
       float vnA = 0.f, vnB = 0.f;
-      if constexpr (!FULL) {
+      if constexpr (!FULL && !GLOB) {
         szA = j0 < t1 ? szrow[j0 * kTok] : kZero4;
         szB = j0 + 2 < t1 ? szrow[(j0 + 2) * kTok] : kZero4;
         posA = j0 < t1 ? posrow[j0 * kTok] : 0;
         posB = j0 + 2 < t1 ? posrow[(j0 + 2) * kTok] : 0;
+      }
+      if constexpr (!FULL) {
         vnA = j0 < t1 ? vnrow[j0 * kTok] : 0.f;
         vnB = j0 + 2 < t1 ? vnrow[(j0 + 2) * kTok] : 0.f;
       }
@@ -699,8 +709,10 @@ __global__ void __launch_bounds__(kThreads, 1)
         posA = posB;
         vnA = vnB;
         if (!FULL && j + 4 < t1) {
-          szB = szrow[(j + 4) * kTok];
-          posB = posrow[(j + 4) * kTok];
+          if constexpr (!GLOB) {
+            szB = szrow[(j + 4) * kTok];
+            posB = posrow[(j + 4) * kTok];
+          }
           vnB = vnrow[(j + 4) * kTok];
         }
         const int i = j * kTok + tok;
@@ -745,6 +757,16 @@ __global__ void __launch_bounds__(kThreads, 1)
           if (lane == 0) mbar_arrive(&bar[B_PFULL + pb]);
         }
         if constexpr (FULL) return make_float2(0.f, 0.f);
+        if constexpr (GLOB) {
+          // this row's share of the token's pooled sums
+          if (valid) {
+            float a2 = 0.f;
+#pragma unroll
+            for (int h = 0; h < G; ++h) a2 = fmaf(a[h], a[h], a2);
+            p.gpart[(rbase + i) * 2 + 1] = make_float4(zc, a2, scur, vn);
+          }
+          return make_float2(0.f, 0.f);
+        }
         const float mean = zc / (float)G;
         float var = 0.f;
 #pragma unroll
@@ -874,7 +896,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       for (int j = j0; j < t1; j += 2) {
         const float2 pf_next = j + 2 < t1 ? prep(j + 2) : make_float2(0.f, 0.f);
         if constexpr (HEUR) record_h(j, pf_cur.x, __float_as_int(pf_cur.y));
-        else if constexpr (!FULL) finish(j, pf_cur.x, __float_as_int(pf_cur.y));
+        else if constexpr (!FULL && !GLOB) finish(j, pf_cur.x, __float_as_int(pf_cur.y));
         pf_cur = pf_next;
       }
       g += nTi;
@@ -998,17 +1020,17 @@ bool fused_eligible(const Dev& p, int n) {
 
 int fused_smem_bytes() { return kSmemBytes; }
 
-template <int D, int G, bool LONG, bool FULL = false, bool HEUR = false>
+template <int D, int G, bool LONG, bool FULL = false, bool HEUR = false, bool GLOB = false>
 static cudaError_t launch_t(const FusedMaps& maps, const Dev& p, const Step& st, const FusedStep& fs,
                             const FusedPolicy& fp, int grid, cudaStream_t s) {
   static bool attr = false;
   if (!attr) {
-    cudaError_t e = cudaFuncSetAttribute(fused_kernel<D, G, LONG, FULL, HEUR>, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes);
+    cudaError_t e = cudaFuncSetAttribute(fused_kernel<D, G, LONG, FULL, HEUR, GLOB>, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes);
     if (e != cudaSuccess) return e;
     attr = true;
   }
   if (fs.half_rows == 0) {
-    fused_kernel<D, G, LONG, FULL, HEUR><<<grid, kThreads, kSmemBytes, s>>>(maps.k, maps.v, p, st, fs, fp);
+    fused_kernel<D, G, LONG, FULL, HEUR, GLOB><<<grid, kThreads, kSmemBytes, s>>>(maps.k, maps.v, p, st, fs, fp);
     return cudaGetLastError();
   }
   // the two CTAs of a half row wait on each other: a cooperative launch
@@ -1023,7 +1045,7 @@ static cudaError_t launch_t(const FusedMaps& maps, const Dev& p, const Step& st,
   la[0].val.cooperative = 1;
   cfg.attrs = la;
   cfg.numAttrs = 1;
-  return cudaLaunchKernelEx(&cfg, fused_kernel<D, G, LONG, FULL, HEUR>, maps.k, maps.v, p, st, fs, fp);
+  return cudaLaunchKernelEx(&cfg, fused_kernel<D, G, LONG, FULL, HEUR, GLOB>, maps.k, maps.v, p, st, fs, fp);
 }
 
 static int fused_grid(const Dev& p, int num_sms) { return p.R < num_sms ? p.R : num_sms; }
@@ -1042,7 +1064,8 @@ cudaError_t launch_fused_step(const FusedMaps& maps, const Dev& p, const Step& s
   const bool lg = st.n > fused_onchip_tokens(p.G);
   // heuristic scorers: one instantiation for any row length
 #define DC_FUSED_LAUNCH(D, G)                                                                 \
-  return p.scorer != 0 ? launch_t<D, G, true, false, true>(maps, p, st, fs, fp, grid, s)      \
+  return p.seq_rows    ? launch_t<D, G, true, false, false, true>(maps, p, st, fs, fp, grid, s) \
+         : p.scorer != 0 ? launch_t<D, G, true, false, true>(maps, p, st, fs, fp, grid, s)      \
          : lg          ? launch_t<D, G, true>(maps, p, st, fs, fp, grid, s)                   \
                        : launch_t<D, G, false>(maps, p, st, fs, fp, grid, s)
   if (p.d == 128) {

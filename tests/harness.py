@@ -193,7 +193,7 @@ class SeqLockStep:
     """Global token mode: drives a DistillCache with global_tokens and one
     sequence oracle per sampled sequence (rows = layers x KV heads)."""
 
-    def __init__(self, wl: synth.Workload, seqs, *, capacity=None, scorer=0):
+    def __init__(self, wl: synth.Workload, seqs, *, capacity=None, scorer=0, engine=0):
         import torch
         from paper_2608_08878_gb300 import dc
         self.torch, self.dc, self.wl = torch, dc, wl
@@ -203,7 +203,7 @@ class SeqLockStep:
         self.cache = dc.DistillCache(wl.layers, wl.kv_heads, wl.head_dim, cap, wl.budget, batch=wl.batch,
                                      q_heads=wl.q_heads, window=wl.window, mlp_hidden=wl.mlp_hidden,
                                      layernorm=wl.layernorm, alpha_mode=wl.alpha_mode, keep_features=True,
-                                     seed=wl.policy_seed, scorer=scorer, global_tokens=True)
+                                     seed=wl.policy_seed, scorer=scorer, global_tokens=True, engine=engine)
         self.cache.set_policy(self.blob)
         self.scorer = scorer
         R = wl.layers * wl.kv_heads

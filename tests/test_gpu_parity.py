@@ -348,14 +348,16 @@ def test_aggressive_sampled_rows():
         ls.step(check=(s < 2 or s >= 15))
 
 
+@pytest.mark.parametrize("engine", ENGINES)
 @pytest.mark.parametrize("scorer", [0, 1, 2])
-def test_global_token_mode(scorer):
+def test_global_token_mode(engine, scorer):
     """Global token mode: features pooled over all heads and layers of each
     sequence, one score and one selection per sequence, every row pruned
     alike; prompt compression and steps past the window, all sequences."""
     wl = synth.MISTRAL_1L.with_(layers=3, batch=2, kv_heads=2, q_heads=8, prompt_len=400, budget=150,
                                 steps=70, window=6)
-    ls = SeqLockStep(wl, range(wl.batch), scorer=scorer)
+    ls = SeqLockStep(wl, range(wl.batch), scorer=scorer, engine=engine)
+    assert ls.cache.engine() == ("fused" if engine == 2 else "split")
     ls.load_prompt()
     for s in range(wl.steps):
         ls.step(check=(s < 3 or s % 16 == 0 or s >= 66))
@@ -367,6 +369,7 @@ def test_global_token_mode_full_shape_sampled():
     sequence), a 2K prompt compressed to 512, then a steady step."""
     wl = synth.MISTRAL_1L.with_(layers=32, batch=1, prompt_len=2048, budget=512, steps=2)
     ls = SeqLockStep(wl, [0])
+    assert ls.cache.engine() == "fused"
     ls.load_prompt()
     for _ in range(wl.steps):
         ls.step()
