@@ -251,10 +251,18 @@ def run_gpu(args):
     wl = wl.with_(seed=wl.seed + 1000 * rank)
     K, W = args.steps, args.warmup
     stream = torch.cuda.current_stream()
-    cache = dc.DistillCache(wl.layers, wl.kv_heads, wl.head_dim, wl.capacity, wl.budget,
+    cap = wl.capacity
+    if args.hybrid:  # full-cache rows grow by one token per step
+        cap = wl.prompt_len + 2 + args.warmup + args.steps
+    cache = dc.DistillCache(wl.layers, wl.kv_heads, wl.head_dim, cap, wl.budget,
                             batch=wl.batch, q_heads=wl.q_heads, window=wl.window,
                             mlp_hidden=wl.mlp_hidden, layernorm=wl.layernorm, engine=args.engine,
                             seed=wl.policy_seed, global_tokens=args.global_tokens)
+    if args.hybrid:
+        # head-level hybrid (Sec. 5): every fifth row (20% of the heads) keeps its
+        # full cache, the others share the rest of a 25% overall budget
+        cache.set_row_budgets(dc.head_level_hybrid_budgets(wl.rows, wl.prompt_len,
+                                                           range(0, wl.rows, 5), 0.25))
     chunk = 4096
     for t0 in range(0, wl.prompt_len, chunk):
         k, v = synth_device.prompt(wl, t0, min(chunk, wl.prompt_len - t0))
@@ -273,6 +281,8 @@ def run_gpu(args):
     for s in range(1, 1 + W):
         cache.step(*inputs[s], out=out)
     n_steady = cache.length()[0] + 1
+    if args.hybrid:  # mean row length after the next append
+        n_steady = float(cache.row_lengths().mean()) + 1
     engine = cache.engine()
     cache.profile(True)
     torch.cuda.synchronize()
@@ -362,7 +372,7 @@ def run_gpu(args):
                        "budget": wl.budget, "window": wl.window, "policy": f"5-{wl.mlp_hidden}-LN-ReLU-1",
                        "engine": engine, "parallelism": f"replicas x{world}",
                        "selection": "per sequence (global token mode)" if args.global_tokens else
-                       "per (layer, KV head) row",
+                       "per (layer, KV head) row" + (", head-level hybrid budgets" if args.hybrid else ""),
                        "l2": f"inputs larger than L2: {bytes_step / 1e9:.2f} GB streamed per step vs 129 MB L2",
                        "steady_tokens_per_row": n_steady},
             "hbm": {"algorithmic_bytes_per_step": bytes_step, "gbs": gbs,
@@ -577,6 +587,8 @@ def main():
                     help="throughput sweep (batch x context x ratio): one JSON line per point")
     ap.add_argument("--sweep-points", default=None, help="e.g. 1x4096x10,64x32768x50 (default: all 36)")
     ap.add_argument("--train", action="store_true", help="time the training-side kernels (App. C)")
+    ap.add_argument("--hybrid", action="store_true",
+                    help="head-level hybrid: 20%% of the rows keep the full cache, the rest share a 25%% budget")
     ap.add_argument("--global-tokens", action="store_true",
                     help="the global token mode (features over all heads and layers, one selection per sequence)")
     args = ap.parse_args()

@@ -170,6 +170,23 @@ dc_status dc_step(dc_cache* h, const void* q, const void* k_new, const void* v_n
 dc_status dc_step_host(dc_cache* h, const void* q_host, const void* k_new_host,
                        const void* v_new_host, float* out_host, int budget);
 
+/* Per-row budgets, the head-level hybrid of Sec. 5 (Table tab:hybrid: the most
+ * important heads keep the full cache, token selection in the others):
+ * budgets[r] for every row r = (layer * batch + b) * kv_heads + g (host array of
+ * n = rows ints, each >= 1). dc_evict / dc_step calls with budget <= 0 then keep
+ * min(n_r, budgets[r]) tokens in row r (a budget >= capacity keeps the row's full
+ * cache up to its capacity); a positive budget argument still applies to every
+ * row; per-row budgets take precedence over budget_ratio. Rows then hold
+ * different lengths (dc_get_row_lengths; dc_get_length reports the longest) and
+ * steps run on the split engine; dc_full_decode needs equal lengths (else
+ * DC_ERR_STATE). budgets == NULL returns to one budget when every row has the
+ * same length (else DC_ERR_STATE). Not with global_tokens (DC_ERR_STATE).
+ * Synchronises the handle's stream. */
+dc_status dc_set_row_budgets(dc_cache* h, const int* budgets_host, int n);
+
+/* Every row's current length (host array of n = rows ints). */
+dc_status dc_get_row_lengths(dc_cache* h, int* lengths_host, int n);
+
 /* Which engine a step over n tokens per row would use (n <= 0: the next
  * decode step): 1 split, 2 fused. */
 dc_status dc_engine(dc_cache* h, int n, int* engine);

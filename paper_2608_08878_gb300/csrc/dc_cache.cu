@@ -3,6 +3,7 @@
 // sequence of each call.
 #include <cuda_runtime.h>
 
+#include <algorithm>
 #include <cmath>
 #include <cstdio>
 #include <cstring>
@@ -64,6 +65,12 @@ struct dc_cache {
   int* xsel = nullptr;
   unsigned* xflag = nullptr;
   unsigned epoch = 0;
+  int* rowlen_dev = nullptr;
+  int* rowbudget_dev = nullptr;
+  // per-row budgets (head-level hybrid): host mirror of every row's length
+  // (kept in step with Dev::rowlen) and the budgets; n is then the longest row
+  bool per_row = false;
+  std::vector<int> hlen, hbudget;
   std::vector<void*> allocs;
   std::string err;
   bool broken = false;
@@ -169,6 +176,7 @@ dc_status launch_error(dc_cache* h, const char* what) {
 
 // Fused engine for this step? (auto: only when the rows fill the GPU)
 bool use_fused(const dc_cache* h, int n) {
+  if (h->per_row) return false;  // rows of different lengths run on the split engine
   if (!h->fused_ok || !dc::fused_eligible(h->dev, n)) return false;
   if (h->cfg.engine == 2) return true;
   if (h->cfg.engine == 0) return 2 * h->dev.R >= h->num_sms;
@@ -202,6 +210,7 @@ dc::Step begin_step(dc_cache* h) {
 
 void end_step(dc_cache* h, const dc::Step& st) {
   h->n += 1;
+  for (int& x : h->hlen) x += 1;
   h->seen += 1;
   h->ring_pnew[st.slot] = st.p_newest;
   h->steps += 1;
@@ -437,12 +446,14 @@ dc_status dc_append(dc_cache* h, const void* k, const void* v, int n_tokens) {
   if ((long long)h->n + n_tokens > h->capacity) return fail(h, DC_ERR_CAPACITY, "append exceeds capacity");
   if (h->seen + n_tokens > 0x7FFFFFFFll) return fail(h, DC_ERR_CAPACITY, "position counter overflow");
   {
-    Phase ph(h, DC_PHASE_APPEND, 1);
+    Phase ph(h, DC_PHASE_APPEND, h->per_row ? 2 : 1);
     dc::launch_append(h->dev, k, v, n_tokens, h->n, (int)h->seen, h->stream);
+    if (h->per_row) dc::launch_rowlen_add(h->dev, n_tokens, h->stream);
   }
   dc_status s = launch_error(h, "append");
   if (s != DC_OK) return s;
   h->n += n_tokens;
+  for (int& x : h->hlen) x += n_tokens;
   h->seen += n_tokens;
   h->have_scores = false;
   return DC_OK;
@@ -507,8 +518,9 @@ dc_status dc_decode_step(dc_cache* h, const void* q, const void* k_new, const vo
   if (h->n + 1 > h->capacity) return fail(h, DC_ERR_CAPACITY, "decode step exceeds capacity");
   if (h->seen + 1 > 0x7FFFFFFFll) return fail(h, DC_ERR_CAPACITY, "position counter overflow");
   {
-    Phase ph(h, DC_PHASE_APPEND, 1);
+    Phase ph(h, DC_PHASE_APPEND, h->per_row ? 2 : 1);
     dc::launch_append(h->dev, k_new, v_new, 1, h->n, (int)h->seen, h->stream);
+    if (h->per_row) dc::launch_rowlen_add(h->dev, 1, h->stream);
   }
   const dc::Step st = begin_step(h);
   if (use_fused(h, st.n)) {
@@ -611,6 +623,23 @@ dc_status dc_decode_step_host(dc_cache* h, const void* q, const void* k_new, con
 dc_status dc_evict(dc_cache* h, int budget) {
   DC_CHECK_HANDLE(h);
   if (!h->have_scores) return fail(h, DC_ERR_STATE, "evict needs the scores of a decode step");
+  if (h->per_row) {
+    // every row to its own budget (or all to `budget` when > 0)
+    {
+      Phase ph(h, DC_PHASE_EVICT, 1);
+      dc::launch_evict(h->dev, h->n, budget > 0 ? budget : 0, h->stream);
+    }
+    dc_status s = launch_error(h, "evict");
+    if (s != DC_OK) return s;
+    int mx = 0;
+    for (size_t r = 0; r < h->hlen.size(); ++r) {
+      h->hlen[r] = std::min(h->hlen[r], budget > 0 ? budget : h->hbudget[r]);
+      mx = std::max(mx, h->hlen[r]);
+    }
+    h->n = mx;
+    h->have_scores = false;
+    return DC_OK;
+  }
   const int B = effective_budget(h, budget, h->n, h->seen);
   const int keep = std::min(h->n, B);
   if (keep < h->n) {
@@ -629,6 +658,8 @@ dc_status dc_full_decode(dc_cache* h, const void* q, float* out) {
   DC_CHECK_HANDLE(h);
   if (!q || !out) return fail(h, DC_ERR_INVALID_ARG, "NULL pointer");
   if (h->n < 1) return fail(h, DC_ERR_STATE, "the cache is empty");
+  if (h->per_row && std::any_of(h->hlen.begin(), h->hlen.end(), [&](int x) { return x != h->n; }))
+    return fail(h, DC_ERR_STATE, "full decode needs rows of equal length (per-row budgets differ)");
   if (h->fused_ok && dc::fused_eligible(h->dev, h->n)) {
     // the fused kernel's attention-only variant (TMA + tensor cores)
     dc::Step st{};
@@ -651,6 +682,48 @@ dc_status dc_full_decode(dc_cache* h, const void* q, float* out) {
   }
   if (!ok) return fail(h, DC_ERR_INVALID_ARG, "unsupported head_dim / group");
   return launch_error(h, "full decode");
+}
+
+dc_status dc_set_row_budgets(dc_cache* h, const int* budgets, int n) {
+  DC_CHECK_HANDLE(h);
+  dc::Dev& p = h->dev;
+  if (!budgets) {
+    if (!h->per_row) return DC_OK;
+    for (int x : h->hlen)
+      if (x != h->n) return fail(h, DC_ERR_STATE, "rows hold different lengths: per-row budgets stay on");
+    h->per_row = false;
+    h->hlen.clear();
+    p.rowlen = nullptr;
+    p.rowbudget = nullptr;
+    return DC_OK;
+  }
+  if (n != p.R) return fail(h, DC_ERR_INVALID_ARG, "one budget per row (layers x batch x kv_heads)");
+  if (p.seq_rows) return fail(h, DC_ERR_STATE, "per-row budgets do not apply to the global token mode");
+  for (int r = 0; r < n; ++r)
+    if (budgets[r] < 1) return fail(h, DC_ERR_INVALID_ARG, "budgets must be >= 1");
+  if (!h->rowlen_dev) {
+    DC_CUDA(h, dalloc(h, &h->rowlen_dev, (size_t)n * sizeof(int)));
+    DC_CUDA(h, dalloc(h, &h->rowbudget_dev, (size_t)n * sizeof(int)));
+  }
+  if (!h->per_row) {
+    h->hlen.assign(n, h->n);
+    DC_CUDA(h, cudaMemcpyAsync(h->rowlen_dev, h->hlen.data(), (size_t)n * sizeof(int), cudaMemcpyHostToDevice,
+                               h->stream));
+  }
+  h->hbudget.assign(budgets, budgets + n);
+  DC_CUDA(h, cudaMemcpyAsync(h->rowbudget_dev, budgets, (size_t)n * sizeof(int), cudaMemcpyHostToDevice, h->stream));
+  DC_CUDA(h, cudaStreamSynchronize(h->stream));  // the caller may free `budgets` on return
+  p.rowlen = h->rowlen_dev;
+  p.rowbudget = h->rowbudget_dev;
+  h->per_row = true;
+  return DC_OK;
+}
+
+dc_status dc_get_row_lengths(dc_cache* h, int* lengths, int n) {
+  DC_CHECK_HANDLE(h);
+  if (!lengths || n != h->dev.R) return fail(h, DC_ERR_INVALID_ARG, "one length per row");
+  for (int r = 0; r < n; ++r) lengths[r] = h->per_row ? h->hlen[r] : h->n;
+  return DC_OK;
 }
 
 dc_status dc_get_length(dc_cache* h, int* n, long long* seen) {

@@ -45,6 +45,10 @@ struct Dev {
   int seq_rows, batch;
   float4* gpart;
   int* gmoves;
+  // per-row budgets (head-level hybrid): each row's length and budget on the
+  // device ([R] each); null when every row has the same length
+  int* rowlen;
+  int* rowbudget;
   __nv_bfloat16* K;
   __nv_bfloat16* V;
   int* pos;

@@ -19,6 +19,15 @@ __global__ void __launch_bounds__(kEvictThreads) evict_kernel(Dev p, int n, int 
   const SelectScratch scr{hist, sh, wsum, best, best_slot};
   auto sync = [] { __syncthreads(); };
   const int r = blockIdx.x;
+  if (p.rowlen) {
+    // per-row lengths and budgets (B > 0 overrides every row's budget)
+    const int nr = p.rowlen[r], Br = B > 0 ? B : p.rowbudget[r];
+    const int keep = nr < Br ? nr : Br;
+    if (keep < nr)
+      team_select_compact<kEvictThreads>(p, r, nr, keep, p.score + (size_t)r * p.stride, threadIdx.x, scr, sync);
+    if (threadIdx.x == 0) p.rowlen[r] = keep;
+    return;
+  }
   team_select_compact<kEvictThreads>(p, r, n, B, p.score + (size_t)r * p.stride, threadIdx.x, scr, sync);
 }
 

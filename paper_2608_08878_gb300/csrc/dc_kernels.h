@@ -9,6 +9,8 @@ namespace dc {
 
 void launch_append(const Dev& p, const void* k, const void* v, int T, int n0, int seen0,
                    cudaStream_t s);
+// Per-row lengths (Dev::rowlen): add T to every row's length after an append.
+void launch_rowlen_add(const Dev& p, int T, cudaStream_t s);
 
 // Split engine: attention + features + scores of one decode step (after the
 // append), one launcher per kernel.

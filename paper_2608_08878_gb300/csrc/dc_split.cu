@@ -30,7 +30,7 @@ __global__ void __launch_bounds__(256) append_kernel(Dev p, const uint4* __restr
   const long long ee = live ? e : pairs - 1;
   const int r = (int)(ee / T), t = (int)(ee % T);
   const size_t src = (size_t)ee * vpr + c;
-  const size_t slot = (size_t)r * p.stride + n0 + t;
+  const size_t slot = (size_t)r * p.stride + (p.rowlen ? p.rowlen[r] : n0) + t;
   const uint4 kv = k[src], vv = v[src];
   if (live) {
     reinterpret_cast<uint4*>(p.K)[slot * vpr + c] = kv;
@@ -136,7 +136,7 @@ __global__ void __launch_bounds__(kTile) split_qk_kernel(Dev p, Step st,
   __shared__ float ring_ml[2][G][3];  // (m, nl, H) of previous / departing
   __shared__ float red[kTile / kWarp][G][3];
   const int r = blockIdx.y, sp = blockIdx.x, tid = threadIdx.x;
-  const int c0 = sp * st.chunk, c1 = min(st.n, c0 + st.chunk);
+  const int c0 = sp * st.chunk, c1 = min(p.rowlen ? p.rowlen[r] : st.n, c0 + st.chunk);
   const int qo = row_q_offset(p, r);
   const __nv_bfloat16* rq_prev = p.ring_q + ((size_t)r * p.w + st.slot_prev) * G * D;
   const __nv_bfloat16* rq_dep = p.ring_q + ((size_t)r * p.w + st.slot) * G * D;
@@ -252,7 +252,7 @@ __global__ void __launch_bounds__(kTile) split_v_kernel(Dev p, Step st) {
   __shared__ float at[kTile][G];
   __shared__ float stat[G][3];  // (m, nl, H)
   const int r = blockIdx.y, sp = blockIdx.x, tid = threadIdx.x;
-  const int c0 = sp * st.chunk, c1 = min(st.n, c0 + st.chunk);
+  const int c0 = sp * st.chunk, c1 = min(p.rowlen ? p.rowlen[r] : st.n, c0 + st.chunk);
   const int H = p.hidden, nblob = 9 * H + 1;
   for (int e = tid; e < nblob; e += blockDim.x) wsm[e] = p.policy[e];
   if (tid < G) {
@@ -383,6 +383,16 @@ void launch_convert_sz(const Dev& p, int row0, int nrows, int which, double* dst
 // ---------------------------------------------------------------------------
 // Host launchers
 // ---------------------------------------------------------------------------
+// Per-row lengths: every row grew by T tokens.
+__global__ void rowlen_add_kernel(Dev p, int T) {
+  const int r = blockIdx.x * blockDim.x + threadIdx.x;
+  if (r < p.R) p.rowlen[r] += T;
+}
+
+void launch_rowlen_add(const Dev& p, int T, cudaStream_t s) {
+  rowlen_add_kernel<<<(p.R + 255) / 256, 256, 0, s>>>(p, T);
+}
+
 void launch_append(const Dev& p, const void* k, const void* v, int T, int n0, int seen0,
                    cudaStream_t s) {
   const long long pairs = (long long)T * p.R;

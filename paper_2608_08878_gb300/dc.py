@@ -29,7 +29,8 @@ EXPORTS = ["dc_config_default", "dc_cache_create", "dc_cache_destroy", "dc_polic
            "dc_decode_step_host", "dc_evict", "dc_full_decode", "dc_get_length", "dc_buffer_bytes",
            "dc_copy_buffer", "dc_sync", "dc_last_error", "dc_phase_name", "dc_profile_enable",
            "dc_profile_read", "dc_step", "dc_step_host", "dc_engine", "dc_attend_noalloc",
-           "dc_noalloc_last_error", "dc_pl_log_partition", "dc_gumbel_top_b", "dc_train_last_error"]
+           "dc_noalloc_last_error", "dc_pl_log_partition", "dc_gumbel_top_b", "dc_train_last_error",
+           "dc_set_row_budgets", "dc_get_row_lengths"]
 PHASES = ["append", "attend", "stats", "score", "combine", "evict", "full"]
 
 
@@ -81,6 +82,8 @@ def lib():
             L.dc_noalloc_last_error.argtypes = []
             L.dc_noalloc_last_error.restype = C.c_char_p
             L.dc_full_decode.argtypes = [P, P, P]
+            L.dc_set_row_budgets.argtypes = [P, P, I]
+            L.dc_get_row_lengths.argtypes = [P, P, I]
             L.dc_pl_log_partition.argtypes = [P, I, I, I, C.c_float, P, P]
             L.dc_gumbel_top_b.argtypes = [P, P, I, I, I, C.c_float, P, P, P, P]
             L.dc_train_last_error.argtypes = []
@@ -161,6 +164,19 @@ def gumbel_top_b(scores, gumbel, B: int, tau: float = 1.0, with_logp: bool = Tru
     if st != DC_OK:
         raise DCError(st, lib().dc_train_last_error().decode())
     return idx, logp
+
+
+def head_level_hybrid_budgets(rows: int, context: int, full_rows, overall_ratio: float = 0.25):
+    """Per-row budgets of the head-level hybrid (Sec. 5): the rows in
+    `full_rows` keep the whole context, the others share what is left of an
+    overall budget of overall_ratio x context per row, equally (at least 1)."""
+    import numpy as np
+    full = np.zeros(rows, dtype=bool)
+    full[list(full_rows)] = True
+    nf = int(full.sum())
+    total = overall_ratio * context * rows
+    rest = max(1, int((total - nf * context) // max(rows - nf, 1)))
+    return np.where(full, context, rest).astype(np.int32)
 
 
 def _ptr(t) -> int:
@@ -271,6 +287,21 @@ class DistillCache:
         if out is None:
             out = torch.empty(q.shape, dtype=torch.float32, device=q.device)
         self._check(lib().dc_full_decode(self._h, _ptr(q), _ptr(out)))
+        return out
+
+    def set_row_budgets(self, budgets) -> None:
+        """Per-row budgets (head-level hybrid); None returns to one budget."""
+        import numpy as np
+        if budgets is None:
+            self._check(lib().dc_set_row_budgets(self._h, None, 0))
+            return
+        b = np.ascontiguousarray(budgets, dtype=np.int32)
+        self._check(lib().dc_set_row_budgets(self._h, b.ctypes.data_as(C.c_void_p), b.size))
+
+    def row_lengths(self):
+        import numpy as np
+        out = np.empty(self.rows, dtype=np.int32)
+        self._check(lib().dc_get_row_lengths(self._h, out.ctypes.data_as(C.c_void_p), out.size))
         return out
 
     def length(self):

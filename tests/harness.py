@@ -46,7 +46,8 @@ class LockStep:
     """Drives a DistillCache and oracle rows for a sample of its rows."""
 
     def __init__(self, wl: synth.Workload, rows, *, engine=0, device_inputs=False, capacity=None,
-                 tail_split=True, scorer=0, n_sinks=4, budget_ratio=0.0, budget_min=32, budget_basis=0):
+                 tail_split=True, scorer=0, n_sinks=4, budget_ratio=0.0, budget_min=32, budget_basis=0,
+                 row_budgets=None):
         import torch
         from paper_2608_08878_gb300 import dc, synth_device
         self.torch, self.dc, self.sd = torch, dc, synth_device
@@ -66,6 +67,9 @@ class LockStep:
         self.budget_ratio, self.budget_min, self.budget_basis = budget_ratio, budget_min, budget_basis
         self.capacity = cap
         self.cache.set_policy(self.blob)
+        self.row_budgets = None if row_budgets is None else np.asarray(row_budgets, dtype=np.int32)
+        if self.row_budgets is not None:
+            self.cache.set_row_budgets(self.row_budgets)
         self.orows = {}
         alpha_mode = 1 if scorer == 1 else wl.alpha_mode  # H2O ranks by the cumulative mass
         for r in self.rows:
@@ -108,7 +112,7 @@ class LockStep:
         q, kn, vn = self._inputs(s)
         out = self.cache.decode_step(q, kn, vn)
         self.cache.sync()  # raises on any device-side status (e.g. a wait that gave up)
-        n, _ = self.cache.length()
+        lens = self.cache.row_lengths()
         out_h = out.cpu().numpy()
         G = wl.group
         for r, orow in self.orows.items():
@@ -117,6 +121,7 @@ class LockStep:
             res = orow.step(qb, knb, vnb, self.blob, wl.mlp_hidden, wl.layernorm)
             if not check:
                 continue
+            n = int(lens[r])
             o_gpu = out_h[layer, b, g * G:(g + 1) * G]
             ma, rel = check_attention(o_gpu, res["o"], f"step {s} row {r} attention")
             self.stats["attn_max_abs"] = max(self.stats["attn_max_abs"], ma)
@@ -145,22 +150,28 @@ class LockStep:
 
     def evict(self, budget=0):
         dc = self.dc
+        lens = self.cache.row_lengths()
         n, _ = self.cache.length()
         gpu_scores = {}
         for r in self.orows:
-            pos = self._row_slice(dc.BUF_POS, r, n)
-            sc = self._row_slice(dc.BUF_SCORE, r, n)
+            pos = self._row_slice(dc.BUF_POS, r, int(lens[r]))
+            sc = self._row_slice(dc.BUF_SCORE, r, int(lens[r]))
             order = np.argsort(pos, kind="stable")
             gpu_scores[r] = sc[order]
         self.cache.evict(budget)
         self.cache.sync()
-        B = budget if budget > 0 else self.budget_now(n)
-        n2, _ = self.cache.length()
-        assert n2 == min(n, B)
-        self.stats["evicted"] += n - n2
+        lens2 = self.cache.row_lengths()
+        self.stats["evicted"] += int(max((lens[r] - lens2[r] for r in self.orows), default=0))
         for r, orow in self.orows.items():
+            if budget > 0:
+                B = budget
+            elif self.row_budgets is not None:
+                B = int(self.row_budgets[r])
+            else:
+                B = self.budget_now(n)
+            assert lens2[r] == min(lens[r], B), (r, lens2[r], lens[r], B)
             orow.evict(B, gpu_scores[r])
-            self.check_row_state(r, n2)
+            self.check_row_state(r, int(lens2[r]))
 
     def budget_now(self, n_cached):
         """The budget of the step that just ran (fixed, or the dynamic one)."""

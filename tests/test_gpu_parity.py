@@ -241,6 +241,28 @@ def test_dynamic_budget(engine, basis):
         assert lengths[:4] == [175, 44, 32, 32] and lengths[-1] == 32
 
 
+def test_per_row_budgets_head_level_hybrid():
+    """Per-row budgets (head-level hybrid, Sec. 5): 2 of 8 KV heads keep the
+    full cache, the rest share a 25% overall budget; every row against the
+    oracle with its own budget, through prompt compression and steady steps."""
+    from paper_2608_08878_gb300 import dc
+    wl = synth.MISTRAL_1L.with_(prompt_len=1200, budget=300, steps=20)
+    cap = wl.prompt_len + wl.steps + 8
+    budgets = dc.head_level_hybrid_budgets(wl.rows, cap, full_rows=[1, 6], overall_ratio=0.25)
+    assert budgets[1] == cap and budgets[6] == cap and budgets[0] < cap
+    ls = LockStep(wl, range(wl.rows), capacity=cap, row_budgets=budgets)
+    assert ls.cache.engine() == "split"
+    ls.load_prompt()
+    for s in range(wl.steps):
+        ls.step(check=(s < 3 or s >= 17))
+    lens = ls.cache.row_lengths()
+    assert lens[1] == wl.prompt_len + wl.steps and lens[0] == budgets[0]
+    with pytest.raises(dc.DCError):
+        ls.cache.full_decode(ls._inputs(0)[0])
+    with pytest.raises(dc.DCError):
+        ls.cache.set_row_budgets(None)  # rows differ in length
+
+
 def test_engine_choice():
     from paper_2608_08878_gb300 import dc
     big = dc.DistillCache(32, 8, 128, 200, 100, batch=1)
