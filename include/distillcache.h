@@ -177,8 +177,9 @@ dc_status dc_step_host(dc_cache* h, const void* q_host, const void* k_new_host,
  * min(n_r, budgets[r]) tokens in row r (a budget >= capacity keeps the row's full
  * cache up to its capacity); a positive budget argument still applies to every
  * row; per-row budgets take precedence over budget_ratio. Rows then hold
- * different lengths (dc_get_row_lengths; dc_get_length reports the longest) and
- * steps run on the split engine; dc_full_decode needs equal lengths (else
+ * different lengths (dc_get_row_lengths; dc_get_length reports the longest);
+ * the fused engine takes them with the policy scorer (heuristic scorers run
+ * on the split engine); dc_full_decode needs equal lengths (else
  * DC_ERR_STATE). budgets == NULL returns to one budget when every row has the
  * same length (else DC_ERR_STATE). Not with global_tokens (DC_ERR_STATE).
  * Synchronises the handle's stream. */

@@ -176,7 +176,8 @@ dc_status launch_error(dc_cache* h, const char* what) {
 
 // Fused engine for this step? (auto: only when the rows fill the GPU)
 bool use_fused(const dc_cache* h, int n) {
-  if (h->per_row) return false;  // rows of different lengths run on the split engine
+  // rows of different lengths: the fused kernel ranks them with the policy only
+  if (h->per_row && h->dev.scorer != 0) return false;
   if (!h->fused_ok || !dc::fused_eligible(h->dev, n)) return false;
   if (h->cfg.engine == 2) return true;
   if (h->cfg.engine == 0) return 2 * h->dev.R >= h->num_sms;
@@ -490,7 +491,7 @@ dc::FusedStep fused_args(dc_cache* h, const dc::Step& st, const void* q, float* 
   fs.xsel = h->xsel;
   fs.xflag = h->xflag;
   fs.work = h->work;
-  fs.half_rows = h->xflag ? dc::fused_half_rows(h->dev, st.n, fs, h->num_sms) : 0;
+  fs.half_rows = (h->xflag && !h->per_row) ? dc::fused_half_rows(h->dev, st.n, fs, h->num_sms) : 0;
   // launch epoch: the queue counter is work[epoch & 1]; exchange flags hold
   // epoch * 4 + phase (1..3), so a flag left by an earlier launch never matches
   fs.epoch = ++h->epoch;
@@ -558,7 +559,7 @@ dc_status dc_step(dc_cache* h, const void* q, const void* k_new, const void* v_n
     return dc_evict(h, budget);
   }
   const int B = effective_budget(h, budget, n1, h->seen + 1);
-  if (B < n1 - 1 && tail_split_applies(h, n1)) {
+  if (!h->per_row && B < n1 - 1 && tail_split_applies(h, n1)) {
     // several evictions need the whole row's scores in one CTA: with half
     // rows this step runs as the decode kernel plus the eviction kernel
     dc_status s = dc_decode_step(h, q, k_new, v_new, out);
@@ -567,10 +568,31 @@ dc_status dc_step(dc_cache* h, const void* q, const void* k_new, const void* v_n
   }
   if (h->seen + 1 > 0x7FFFFFFFll) return fail(h, DC_ERR_CAPACITY, "position counter overflow");
   {
-    Phase ph(h, DC_PHASE_APPEND, 1);
+    Phase ph(h, DC_PHASE_APPEND, h->per_row ? 2 : 1);
     dc::launch_append(h->dev, k_new, v_new, 1, h->n, (int)h->seen, h->stream);
+    if (h->per_row) dc::launch_rowlen_add(h->dev, 1, h->stream);
   }
   const dc::Step st = begin_step(h);
+  if (h->per_row) {
+    // every row to its own budget (B = 0), or all to `budget` when > 0; the
+    // kernel writes the new lengths, the host mirrors them
+    const dc::FusedStep fs = fused_args(h, st, q, out, 1, budget > 0 ? budget : 0, 0);
+    cudaError_t e;
+    {
+      Phase ph(h, DC_PHASE_ATTEND, 1);
+      e = dc::launch_fused_step(h->maps, h->dev, st, fs, h->fpol, h->num_sms, h->stream);
+    }
+    if (e != cudaSuccess) return cuda_fail(h, e, "fused step");
+    end_step(h, st);
+    int mx = 0;
+    for (size_t r = 0; r < h->hlen.size(); ++r) {
+      h->hlen[r] = std::min(h->hlen[r], budget > 0 ? budget : h->hbudget[r]);
+      mx = std::max(mx, h->hlen[r]);
+    }
+    h->n = mx;
+    h->have_scores = false;
+    return DC_OK;
+  }
   const int keep = std::min(st.n, B);
   const dc::FusedStep fs = fused_args(h, st, q, out, keep < st.n ? 1 : 0, keep, 0);
   cudaError_t e;

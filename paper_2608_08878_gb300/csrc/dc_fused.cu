@@ -211,10 +211,11 @@ struct Item {
 
 constexpr int kItemRing = 8;  // items published ahead of the slowest role (at most ~3)
 
-__device__ __forceinline__ Item take_item(const FusedStep& fs, int R, int nT) {
-  const unsigned whole = (unsigned)(R - fs.half_rows);
+template <bool PERROW>
+__device__ __forceinline__ Item take_item(const FusedStep& fs, const Dev& p, int nT) {
+  const unsigned whole = (unsigned)(p.R - fs.half_rows);
   const unsigned w = atomicAdd(fs.work + (fs.epoch & 1u), 1u);
-  if (w < whole) return Item{(int)w, 0, nT, -1};
+  if (w < whole) return Item{(int)w, 0, PERROW ? (p.rowlen[w] + kTok - 1) / kTok : nT, -1};
   const unsigned k = w - whole;
   if (k >= 2u * (unsigned)fs.half_rows) return Item{-1, 0, 0, 0};
   const int mid = (nT + 1) >> 1, h = (int)(k & 1u);
@@ -260,7 +261,10 @@ __device__ __forceinline__ Item read_item(volatile int* ring, int gr, volatile i
 // Dev::gpart (window terms in the K pass; mass, squared mass, entropy-weighted
 // mass and |v| in the V pass); features, scores and the selection are made
 // per sequence afterwards.
-template <int D, int G, bool LONG, bool FULL, bool HEUR, bool GLOB>
+// PERROW: rows of different lengths and budgets (Dev::rowlen, Dev::rowbudget;
+// FusedStep::B > 0 overrides every row's budget); the kernel writes each
+// row's new length after its selection. No half rows.
+template <int D, int G, bool LONG, bool FULL, bool HEUR, bool GLOB, bool PERROW>
 __global__ void __launch_bounds__(kThreads, 1)
     fused_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmV, Dev p,
                  Step st, FusedStep fs, FusedPolicy fp) {
@@ -281,7 +285,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   volatile int* items = reinterpret_cast<volatile int*>(smem + OFF_MISC + 2304);  // [8][4] + seq [8]
 
   const int warp = threadIdx.x / kWarp, lane = threadIdx.x % kWarp;
-  const int n = st.n, nT = (n + kTok - 1) / kTok;
+  const int n_step = st.n, nT = (n_step + kTok - 1) / kTok;
   constexpr uint32_t kTileBytes = (uint32_t)D * kTok * 2;
 
   if (threadIdx.x == 0) {
@@ -345,7 +349,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       // the next item, taken once this CTA's query buffer is free
       int4 iv = make_int4(-1, 0, 0, 0);
       if (lane == 0) {
-        const Item t = last ? Item{-1, 0, 0, 0} : take_item(fs, p.R, nT);
+        const Item t = last ? Item{-1, 0, 0, 0} : take_item<PERROW>(fs, p, nT);
         publish_item(items, gr, t);
         iv = make_int4(t.row, t.t0, t.t1, t.half);
       }
@@ -517,6 +521,9 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (named_bar_or(1, kEpi, *abort != 0 || iv.x < 0)) break;
       const Item it{iv.x, iv.y, iv.z, iv.w};
       const int r = it.row, t0 = it.t0, t1 = it.t1, nTi = it.t1 - it.t0;
+      // this row's length (after the append) and budget
+      const int n = PERROW ? p.rowlen[r] : n_step;
+      const int Bsel = PERROW ? (fs.B > 0 ? fs.B : p.rowbudget[r]) : fs.B;
       const int ts = r - (p.R - fs.half_rows);  // exchange slot (half rows only)
       const size_t rbase = (size_t)r * p.stride;
       float pm[G], pnl[G], pH[G], dm[G], dnl[G], dH[G];
@@ -937,14 +944,14 @@ __global__ void __launch_bounds__(kThreads, 1)
           op[h * D + tok] = half == 0 ? ov[h] + __ldcg(&fs.xo[((size_t)ts * G + h) * D + tok]) : ov[h];
       }
       // ---------------- argtop_B and prune
-      if (fs.do_evict && n == fs.B + 1) {
+      if (fs.do_evict && n == Bsel + 1) {
         // one eviction (the steady state): the lowest-ranked token, from each
         // thread's running candidate; slot B (the last, held by the whole row
         // or by half 1) is the only mover and fills the evicted slot. Half
         // rows swap their candidates first.
         const bool mover = half != 0;
         SlotCopy mv{};
-        if (mover && etid < kWarp) mv = slot_load(p, rbase + fs.B, etid);
+        if (mover && etid < kWarp) mv = slot_load(p, rbase + Bsel, etid);
         auto lower = [](uint32_t ka, int sa, int pa, uint32_t kb, int sb, int pb) {  // (kb, sb) ranks lower?
           if (sb < 0) return false;
           if (sa < 0) return true;
@@ -988,14 +995,15 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         sync();
         const int e = s_sh[0];
-        if (mover && e >= 0 && e < fs.B && etid < kWarp) slot_store(p, rbase + e, etid, mv);
+        if (mover && e >= 0 && e < Bsel && etid < kWarp) slot_store(p, rbase + e, etid, mv);
         sync();
-      } else if (fs.do_evict && fs.B < n) {
+      } else if (fs.do_evict && Bsel < n) {
         // several evictions (whole rows only): radix select over the scores
         sync();
-        team_select_compact<kEpi>(p, r, n, fs.B, LONG && n > kFusedMaxTok ? p.score + rbase : sc, etid, scr,
+        team_select_compact<kEpi>(p, r, n, Bsel, LONG && n > kFusedMaxTok ? p.score + rbase : sc, etid, scr,
                                   sync);
       }
+      if (PERROW && fs.do_evict && etid == 0) p.rowlen[r] = n < Bsel ? n : Bsel;
     }
   }
   __syncthreads();
@@ -1020,17 +1028,17 @@ bool fused_eligible(const Dev& p, int n) {
 
 int fused_smem_bytes() { return kSmemBytes; }
 
-template <int D, int G, bool LONG, bool FULL = false, bool HEUR = false, bool GLOB = false>
+template <int D, int G, bool LONG, bool FULL = false, bool HEUR = false, bool GLOB = false, bool PERROW = false>
 static cudaError_t launch_t(const FusedMaps& maps, const Dev& p, const Step& st, const FusedStep& fs,
                             const FusedPolicy& fp, int grid, cudaStream_t s) {
   static bool attr = false;
   if (!attr) {
-    cudaError_t e = cudaFuncSetAttribute(fused_kernel<D, G, LONG, FULL, HEUR, GLOB>, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes);
+    cudaError_t e = cudaFuncSetAttribute(fused_kernel<D, G, LONG, FULL, HEUR, GLOB, PERROW>, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes);
     if (e != cudaSuccess) return e;
     attr = true;
   }
   if (fs.half_rows == 0) {
-    fused_kernel<D, G, LONG, FULL, HEUR, GLOB><<<grid, kThreads, kSmemBytes, s>>>(maps.k, maps.v, p, st, fs, fp);
+    fused_kernel<D, G, LONG, FULL, HEUR, GLOB, PERROW><<<grid, kThreads, kSmemBytes, s>>>(maps.k, maps.v, p, st, fs, fp);
     return cudaGetLastError();
   }
   // the two CTAs of a half row wait on each other: a cooperative launch
@@ -1045,7 +1053,7 @@ static cudaError_t launch_t(const FusedMaps& maps, const Dev& p, const Step& st,
   la[0].val.cooperative = 1;
   cfg.attrs = la;
   cfg.numAttrs = 1;
-  return cudaLaunchKernelEx(&cfg, fused_kernel<D, G, LONG, FULL, HEUR, GLOB>, maps.k, maps.v, p, st, fs, fp);
+  return cudaLaunchKernelEx(&cfg, fused_kernel<D, G, LONG, FULL, HEUR, GLOB, PERROW>, maps.k, maps.v, p, st, fs, fp);
 }
 
 static int fused_grid(const Dev& p, int num_sms) { return p.R < num_sms ? p.R : num_sms; }
@@ -1064,7 +1072,8 @@ cudaError_t launch_fused_step(const FusedMaps& maps, const Dev& p, const Step& s
   const bool lg = st.n > fused_onchip_tokens(p.G);
   // heuristic scorers: one instantiation for any row length
 #define DC_FUSED_LAUNCH(D, G)                                                                 \
-  return p.seq_rows    ? launch_t<D, G, true, false, false, true>(maps, p, st, fs, fp, grid, s) \
+  return p.rowlen      ? launch_t<D, G, true, false, false, false, true>(maps, p, st, fs, fp, grid, s) \
+         : p.seq_rows  ? launch_t<D, G, true, false, false, true>(maps, p, st, fs, fp, grid, s) \
          : p.scorer != 0 ? launch_t<D, G, true, false, true>(maps, p, st, fs, fp, grid, s)      \
          : lg          ? launch_t<D, G, true>(maps, p, st, fs, fp, grid, s)                   \
                        : launch_t<D, G, false>(maps, p, st, fs, fp, grid, s)

@@ -241,17 +241,37 @@ def test_dynamic_budget(engine, basis):
         assert lengths[:4] == [175, 44, 32, 32] and lengths[-1] == 32
 
 
-def test_per_row_budgets_head_level_hybrid():
+@pytest.mark.parametrize("engine", ENGINES)
+def test_per_row_budgets_head_level_hybrid(engine):
     """Per-row budgets (head-level hybrid, Sec. 5): 2 of 8 KV heads keep the
     full cache, the rest share a 25% overall budget; every row against the
-    oracle with its own budget, through prompt compression and steady steps."""
+    oracle with its own budget, through prompt compression and steady steps;
+    then dc_step (the fused kernel's in-kernel selection per row) against
+    dc_decode_step + dc_evict."""
+    import torch
     from paper_2608_08878_gb300 import dc
     wl = synth.MISTRAL_1L.with_(prompt_len=1200, budget=300, steps=20)
     cap = wl.prompt_len + wl.steps + 8
     budgets = dc.head_level_hybrid_budgets(wl.rows, cap, full_rows=[1, 6], overall_ratio=0.25)
     assert budgets[1] == cap and budgets[6] == cap and budgets[0] < cap
-    ls = LockStep(wl, range(wl.rows), capacity=cap, row_budgets=budgets)
-    assert ls.cache.engine() == "split"
+    a = LockStep(wl, [], engine=engine, capacity=cap, row_budgets=budgets)
+    b = LockStep(wl, [], engine=engine, capacity=cap, row_budgets=budgets)
+    a.load_prompt()
+    b.load_prompt()
+    for s in range(6):
+        q, kn, vn = a._inputs(s)
+        oa = a.cache.step(q, kn, vn)
+        ob = b.cache.decode_step(q, kn, vn)
+        b.cache.evict()
+        torch.cuda.synchronize()
+        assert torch.equal(oa, ob), s
+        assert np.array_equal(a.cache.row_lengths(), b.cache.row_lengths())
+        for r in range(wl.rows):
+            n = int(a.cache.row_lengths()[r])
+            for which in (dc.BUF_K, dc.BUF_POS, dc.BUF_S, dc.BUF_Z):
+                assert torch.equal(a.cache.buffer(which, r, 1)[:, :n], b.cache.buffer(which, r, 1)[:, :n]), (s, r)
+    ls = LockStep(wl, range(wl.rows), engine=engine, capacity=cap, row_budgets=budgets)
+    assert ls.cache.engine() == ("fused" if engine == 2 else "split")
     ls.load_prompt()
     for s in range(wl.steps):
         ls.step(check=(s < 3 or s >= 17))
