@@ -415,3 +415,36 @@ def test_global_token_mode_full_shape_sampled():
     ls.load_prompt()
     for _ in range(wl.steps):
         ls.step()
+
+
+def test_full_decode_with_split_rows_matches_oracle():
+    """The full-cache comparator (the fused kernel's attention-only variant)
+    with the last wave's rows split over CTA pairs: sampled rows, split and
+    whole, against the oracle's plain attention."""
+    import oracle
+    wl, sms = _tail_workload(prompt_len=2500)
+    ls = LockStep(wl, [], engine=2)
+    ls.load_prompt()
+    q, _, _ = ls._inputs(0)
+    out = ls.cache.full_decode(q).cpu().numpy()
+    qh = q.view(__import__("torch").int16).cpu().numpy().view(np.uint16)
+    for r in (0, sms - 1, sms, wl.rows - 1):
+        layer, b, g = wl.row_coords(r)
+        k, v = synth.prompt_row(wl, layer, b, g)
+        G = wl.group
+        o, _ = oracle.attend(qh[layer, b, g * G:(g + 1) * G], k, v)
+        check_attention(out[layer, b, g * G:(g + 1) * G], o, f"full decode row {r}")
+
+
+def test_global_token_mode_with_split_rows():
+    """Global token mode on the fused engine with more rows than SMs, so the
+    last wave's rows are split over CTA pairs: one 160-row sequence."""
+    import torch
+    sms = torch.cuda.get_device_properties(0).multi_processor_count
+    layers = sms // 8 + 1
+    wl = synth.MISTRAL_1L.with_(layers=layers, batch=1, prompt_len=600, budget=250, steps=4, window=3)
+    assert 0 < wl.rows - sms <= sms // 2
+    ls = SeqLockStep(wl, [0], engine=2)
+    ls.load_prompt()
+    for _ in range(wl.steps):
+        ls.step()
