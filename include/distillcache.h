@@ -170,6 +170,16 @@ dc_status dc_step(dc_cache* h, const void* q, const void* k_new, const void* v_n
 dc_status dc_step_host(dc_cache* h, const void* q_host, const void* k_new_host,
                        const void* v_new_host, float* out_host, int budget);
 
+/* dc_step_host without the final synchronisation. The input copies run on a
+ * copy stream of the handle's own, the step on the handle's stream, the output
+ * copy on a second copy stream, with two device staging sets used in turn: the
+ * inputs of step s + 1 and the output of step s move while kernels run. The
+ * call returns at once; out_host holds the output after dc_sync (which also
+ * waits for the copy streams), and every host buffer must stay untouched until
+ * then. Pinned host memory keeps the copies asynchronous. */
+dc_status dc_step_host_async(dc_cache* h, const void* q_host, const void* k_new_host,
+                             const void* v_new_host, float* out_host, int budget);
+
 /* Per-row budgets, the head-level hybrid of Sec. 5 (Table tab:hybrid: the most
  * important heads keep the full cache, token selection in the others):
  * budgets[r] for every row r = (layer * batch + b) * kv_heads + g (host array of
@@ -257,8 +267,9 @@ dc_status dc_profile_enable(dc_cache* h, int on);
  * ms and launches each hold DC_PHASE_COUNT values (either may be NULL). */
 dc_status dc_profile_read(dc_cache* h, double* ms, long long* launches);
 
-/* Waits for all work enqueued on the handle's stream; reports any device
- * status the kernels raised (DC_ERR_DEVICE). */
+/* Waits for all work enqueued on the handle's stream (and on the copy streams
+ * of dc_step_host_async); reports any device status the kernels raised
+ * (DC_ERR_DEVICE). */
 dc_status dc_sync(dc_cache* h);
 
 /* Full-cache decode attention that allocates no device memory, for callers

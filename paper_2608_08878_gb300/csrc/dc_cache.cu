@@ -52,6 +52,15 @@ struct dc_cache {
   void* st_k = nullptr;
   void* st_v = nullptr;
   float* st_out = nullptr;
+  // dc_step_host_async: a second staging set, copy streams and events, so that
+  // step s + 1's input copy and step s's output copy overlap the kernels
+  void* st2_q = nullptr;
+  void* st2_k = nullptr;
+  void* st2_v = nullptr;
+  float* st2_out = nullptr;
+  cudaStream_t h2d = nullptr, d2h = nullptr;
+  cudaEvent_t ev_in[2] = {}, ev_done[2] = {}, ev_out[2] = {};
+  long long host_seq = 0;
   // fused engine: TMA descriptors of K/V and the folded policy
   bool fused_ok = false;
   std::string fused_why;
@@ -420,6 +429,17 @@ dc_status dc_cache_destroy(dc_cache* h) {
   if (!h) return DC_OK;
   if (!valid(h)) return DC_ERR_INVALID_ARG;
   cudaStreamSynchronize(h->stream);
+  if (h->h2d) {
+    cudaStreamSynchronize(h->h2d);
+    cudaStreamSynchronize(h->d2h);
+    for (int i = 0; i < 2; ++i) {
+      cudaEventDestroy(h->ev_in[i]);
+      cudaEventDestroy(h->ev_done[i]);
+      cudaEventDestroy(h->ev_out[i]);
+    }
+    cudaStreamDestroy(h->h2d);
+    cudaStreamDestroy(h->d2h);
+  }
   for (auto& t : h->timed) { cudaEventDestroy(t.a); cudaEventDestroy(t.b); }
   for (auto e : h->event_pool) cudaEventDestroy(e);
   free_all(h);
@@ -607,17 +627,89 @@ dc_status dc_step(dc_cache* h, const void* q, const void* k_new, const void* v_n
   return DC_OK;
 }
 
-dc_status dc_step_host(dc_cache* h, const void* q, const void* k_new, const void* v_new, float* out, int budget) {
+namespace {
+
+// The first staging set is shared with the asynchronous path, whose output
+// copies run on their own stream: the handle's stream waits for them.
+dc_status wait_async_copies(dc_cache* h) {
+  if (h->h2d)
+    for (int i = 0; i < 2; ++i) DC_CUDA(h, cudaStreamWaitEvent(h->stream, h->ev_out[i], 0));
+  return DC_OK;
+}
+
+// dc_step with host buffers: inputs copied into the device staging buffers,
+// the step, the output copied back, all in the handle's stream order (so the
+// staging buffers are reused safely by the next call).
+dc_status step_host(dc_cache* h, const void* q, const void* k_new, const void* v_new, float* out, int budget,
+                    bool synchronise) {
   DC_CHECK_HANDLE(h);
   if (!q || !k_new || !v_new || !out) return fail(h, DC_ERR_INVALID_ARG, "NULL pointer");
   const size_t R = h->dev.R, G = h->dev.G, d = h->dev.d;
+  if (dc_status w = wait_async_copies(h); w != DC_OK) return w;
   DC_CUDA(h, cudaMemcpyAsync(h->st_q, q, R * G * d * 2, cudaMemcpyHostToDevice, h->stream));
   DC_CUDA(h, cudaMemcpyAsync(h->st_k, k_new, R * d * 2, cudaMemcpyHostToDevice, h->stream));
   DC_CUDA(h, cudaMemcpyAsync(h->st_v, v_new, R * d * 2, cudaMemcpyHostToDevice, h->stream));
   dc_status s = dc_step(h, h->st_q, h->st_k, h->st_v, h->st_out, budget);
   if (s != DC_OK) return s;
   DC_CUDA(h, cudaMemcpyAsync(out, h->st_out, R * G * d * sizeof(float), cudaMemcpyDeviceToHost, h->stream));
-  DC_CUDA(h, cudaStreamSynchronize(h->stream));
+  if (synchronise) DC_CUDA(h, cudaStreamSynchronize(h->stream));
+  return DC_OK;
+}
+
+}  // namespace
+
+dc_status dc_step_host(dc_cache* h, const void* q, const void* k_new, const void* v_new, float* out, int budget) {
+  return step_host(h, q, k_new, v_new, out, budget, true);
+}
+
+// Two staging sets used in turn; the input copies of step s + 1 and the output
+// copy of step s run on copy streams while step s (or s + 1) computes.
+
+dc_status dc_step_host_async(dc_cache* h, const void* q, const void* k_new, const void* v_new, float* out,
+                             int budget) {
+  DC_CHECK_HANDLE(h);
+  if (!q || !k_new || !v_new || !out) return fail(h, DC_ERR_INVALID_ARG, "NULL pointer");
+  const size_t R = h->dev.R, G = h->dev.G, d = h->dev.d;
+  if (!h->h2d) {
+    DC_CUDA(h, dalloc(h, &h->st2_q, R * G * d * 2));
+    DC_CUDA(h, dalloc(h, &h->st2_k, R * d * 2));
+    DC_CUDA(h, dalloc(h, &h->st2_v, R * d * 2));
+    DC_CUDA(h, dalloc(h, &h->st2_out, R * G * d * sizeof(float)));
+    DC_CUDA(h, cudaStreamCreateWithFlags(&h->h2d, cudaStreamNonBlocking));
+    DC_CUDA(h, cudaStreamCreateWithFlags(&h->d2h, cudaStreamNonBlocking));
+    for (int i = 0; i < 2; ++i) {
+      DC_CUDA(h, cudaEventCreateWithFlags(&h->ev_in[i], cudaEventDisableTiming));
+      DC_CUDA(h, cudaEventCreateWithFlags(&h->ev_done[i], cudaEventDisableTiming));
+      DC_CUDA(h, cudaEventCreateWithFlags(&h->ev_out[i], cudaEventDisableTiming));
+    }
+    // the first uses of each buffer wait on events that have completed
+    for (int i = 0; i < 2; ++i) {
+      DC_CUDA(h, cudaEventRecord(h->ev_done[i], h->stream));
+      DC_CUDA(h, cudaEventRecord(h->ev_out[i], h->stream));
+    }
+  }
+  const int b = (int)(h->host_seq & 1);
+  void* sq = b ? h->st2_q : h->st_q;
+  void* sk = b ? h->st2_k : h->st_k;
+  void* sv = b ? h->st2_v : h->st_v;
+  float* so = b ? h->st2_out : h->st_out;
+  // inputs: once the step two calls back has read this staging set
+  DC_CUDA(h, cudaStreamWaitEvent(h->h2d, h->ev_done[b], 0));
+  DC_CUDA(h, cudaMemcpyAsync(sq, q, R * G * d * 2, cudaMemcpyHostToDevice, h->h2d));
+  DC_CUDA(h, cudaMemcpyAsync(sk, k_new, R * d * 2, cudaMemcpyHostToDevice, h->h2d));
+  DC_CUDA(h, cudaMemcpyAsync(sv, v_new, R * d * 2, cudaMemcpyHostToDevice, h->h2d));
+  DC_CUDA(h, cudaEventRecord(h->ev_in[b], h->h2d));
+  // the step: after its inputs, and after the output of two calls back has left
+  DC_CUDA(h, cudaStreamWaitEvent(h->stream, h->ev_in[b], 0));
+  DC_CUDA(h, cudaStreamWaitEvent(h->stream, h->ev_out[b], 0));
+  dc_status s = dc_step(h, sq, sk, sv, so, budget);
+  if (s != DC_OK) return s;
+  DC_CUDA(h, cudaEventRecord(h->ev_done[b], h->stream));
+  // the output, on its own stream
+  DC_CUDA(h, cudaStreamWaitEvent(h->d2h, h->ev_done[b], 0));
+  DC_CUDA(h, cudaMemcpyAsync(out, so, R * G * d * sizeof(float), cudaMemcpyDeviceToHost, h->d2h));
+  DC_CUDA(h, cudaEventRecord(h->ev_out[b], h->d2h));
+  h->host_seq += 1;
   return DC_OK;
 }
 
@@ -632,6 +724,7 @@ dc_status dc_decode_step_host(dc_cache* h, const void* q, const void* k_new, con
   DC_CHECK_HANDLE(h);
   if (!q || !k_new || !v_new || !out) return fail(h, DC_ERR_INVALID_ARG, "NULL pointer");
   const size_t R = h->dev.R, G = h->dev.G, d = h->dev.d;
+  if (dc_status w = wait_async_copies(h); w != DC_OK) return w;
   DC_CUDA(h, cudaMemcpyAsync(h->st_q, q, R * G * d * 2, cudaMemcpyHostToDevice, h->stream));
   DC_CUDA(h, cudaMemcpyAsync(h->st_k, k_new, R * d * 2, cudaMemcpyHostToDevice, h->stream));
   DC_CUDA(h, cudaMemcpyAsync(h->st_v, v_new, R * d * 2, cudaMemcpyHostToDevice, h->stream));
@@ -815,6 +908,10 @@ dc_status dc_copy_buffer(dc_cache* h, dc_buffer which, int row0, int nrows, void
 dc_status dc_sync(dc_cache* h) {
   DC_CHECK_HANDLE(h);
   DC_CUDA(h, cudaStreamSynchronize(h->stream));
+  if (h->h2d) {
+    DC_CUDA(h, cudaStreamSynchronize(h->h2d));
+    DC_CUDA(h, cudaStreamSynchronize(h->d2h));
+  }
   unsigned st = 0, dbg[8] = {};
   DC_CUDA(h, cudaMemcpy(&st, h->dev.status, sizeof st, cudaMemcpyDeviceToHost));
   DC_CUDA(h, cudaMemcpy(dbg, h->dev.dbg, sizeof dbg, cudaMemcpyDeviceToHost));

@@ -84,6 +84,14 @@ int fused_half_rows(const Dev& p, int n, const FusedStep& fs, int num_sms);
 cudaError_t launch_fused_step(const FusedMaps& maps, const Dev& p, const Step& st, const FusedStep& fs,
                               const FusedPolicy& fp, int num_sms, cudaStream_t s);
 
+// The variants with a heuristic scorer or per-row budgets (dc_fused_modes.cu)
+// and with the global token mode (dc_fused_glob.cu); launch_fused_step
+// dispatches to them.
+cudaError_t launch_fused_heur_perrow(const FusedMaps& maps, const Dev& p, const Step& st, const FusedStep& fs,
+                                     const FusedPolicy& fp, int num_sms, cudaStream_t s);
+cudaError_t launch_fused_glob(const FusedMaps& maps, const Dev& p, const Step& st, const FusedStep& fs,
+                              const FusedPolicy& fp, int num_sms, cudaStream_t s);
+
 // Attention only over the first n tokens of every row as they are (the
 // full-cache comparator): writes fs.out, touches no cache state (the logit
 // scratch aside). fs.do_evict and fs.write_scores must be 0.

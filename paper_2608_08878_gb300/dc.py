@@ -28,7 +28,7 @@ EXPORTS = ["dc_config_default", "dc_cache_create", "dc_cache_destroy", "dc_polic
            "dc_policy_init", "dc_policy_set_weights", "dc_append", "dc_decode_step",
            "dc_decode_step_host", "dc_evict", "dc_full_decode", "dc_get_length", "dc_buffer_bytes",
            "dc_copy_buffer", "dc_sync", "dc_last_error", "dc_phase_name", "dc_profile_enable",
-           "dc_profile_read", "dc_step", "dc_step_host", "dc_engine", "dc_attend_noalloc",
+           "dc_profile_read", "dc_step", "dc_step_host", "dc_step_host_async", "dc_engine", "dc_attend_noalloc",
            "dc_noalloc_last_error", "dc_pl_log_partition", "dc_gumbel_top_b", "dc_train_last_error",
            "dc_set_row_budgets", "dc_get_row_lengths"]
 PHASES = ["append", "attend", "stats", "score", "combine", "evict", "full"]
@@ -77,6 +77,7 @@ def lib():
             L.dc_evict.argtypes = [P, I]
             L.dc_step.argtypes = [P, P, P, P, P, I]
             L.dc_step_host.argtypes = [P, P, P, P, P, I]
+            L.dc_step_host_async.argtypes = [P, P, P, P, P, I]
             L.dc_engine.argtypes = [P, I, C.POINTER(I)]
             L.dc_attend_noalloc.argtypes = [P, P, P, I, I, I, I, P, P]
             L.dc_noalloc_last_error.argtypes = []
@@ -273,6 +274,11 @@ class DistillCache:
 
     def step_host(self, q, k_new, v_new, out, budget: int = 0) -> None:
         self._check(lib().dc_step_host(self._h, _ptr(q), _ptr(k_new), _ptr(v_new), _ptr(out), budget))
+
+    def step_host_async(self, q, k_new, v_new, out, budget: int = 0) -> None:
+        """step_host without the final synchronisation (pinned host tensors;
+        `out` is valid after sync())."""
+        self._check(lib().dc_step_host_async(self._h, _ptr(q), _ptr(k_new), _ptr(v_new), _ptr(out), budget))
 
     def engine(self, n: int = 0) -> str:
         e = C.c_int()

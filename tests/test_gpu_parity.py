@@ -448,3 +448,34 @@ def test_global_token_mode_with_split_rows():
     ls.load_prompt()
     for _ in range(wl.steps):
         ls.step()
+
+
+def test_async_host_steps_equal_device_steps():
+    """dc_step_host_async queued back to back (one sync at the end) gives the
+    same outputs and cache as dc_step on device buffers."""
+    import torch
+    from paper_2608_08878_gb300 import dc
+    wl = synth.MISTRAL_1L.with_(prompt_len=1000, budget=300)
+    a, b = LockStep(wl, [], engine=2), LockStep(wl, [], engine=2)
+    a.load_prompt()
+    b.load_prompt()
+    f = lambda x: torch.from_numpy(x.view(np.int16)).view(torch.bfloat16)
+    outs, refs, keep = [], [], []
+    for s in range(8):
+        q, kn, vn = synth.step_all(wl, s)
+        hq, hk, hv = f(q).pin_memory(), f(kn).pin_memory(), f(vn).pin_memory()
+        keep.append((hq, hk, hv))
+        out_h = torch.empty(q.shape, dtype=torch.float32).pin_memory()
+        if s == 5:
+            # the synchronous call shares the first staging set with copies
+            # of the asynchronous ones still in flight
+            a.cache.step_host(hq, hk, hv, out_h)
+        else:
+            a.cache.step_host_async(hq, hk, hv, out_h)
+        outs.append(out_h)
+        refs.append(b.cache.step(f(q).cuda(), f(kn).cuda(), f(vn).cuda()).cpu())
+    a.cache.sync()
+    for s in range(8):
+        assert torch.equal(outs[s], refs[s]), s
+    for which in (dc.BUF_K, dc.BUF_POS, dc.BUF_S):
+        assert torch.equal(a.cache.buffer(which), b.cache.buffer(which))
