@@ -251,23 +251,10 @@ def run_gpu(args):
     wl = wl.with_(seed=wl.seed + 1000 * rank)
     K, W = args.steps, args.warmup
     stream = torch.cuda.current_stream()
-    cap = wl.capacity
-    if args.hybrid:  # full-cache rows grow by one token per step
-        cap = wl.prompt_len + 2 + args.warmup + args.steps
-    cache = dc.DistillCache(wl.layers, wl.kv_heads, wl.head_dim, cap, wl.budget,
-                            batch=wl.batch, q_heads=wl.q_heads, window=wl.window,
-                            mlp_hidden=wl.mlp_hidden, layernorm=wl.layernorm, engine=args.engine,
-                            seed=wl.policy_seed, global_tokens=args.global_tokens)
-    if args.hybrid:
-        # head-level hybrid (Sec. 5): every fifth row (20% of the heads) keeps its
-        # full cache, the others share the rest of a 25% overall budget
-        cache.set_row_budgets(dc.head_level_hybrid_budgets(wl.rows, wl.prompt_len,
-                                                           range(0, wl.rows, 5), 0.25))
+    cache = make_cache(wl, args)
+    if args.scorer == 1:  # H2O ranks by cumulative attention (alpha_mode 1 state)
+        wl = wl.with_(alpha_mode=1)
     chunk = 4096
-    for t0 in range(0, wl.prompt_len, chunk):
-        k, v = synth_device.prompt(wl, t0, min(chunk, wl.prompt_len - t0))
-        cache.append(k, v)
-        del k, v
     # all step inputs resident in HBM before timing
     inputs = [synth_device.step_inputs(wl, s) for s in range(1 + W + K)]
     out = torch.empty((wl.layers, wl.batch, wl.q_heads, wl.head_dim), dtype=torch.float32, device="cuda")
@@ -281,7 +268,7 @@ def run_gpu(args):
     for s in range(1, 1 + W):
         cache.step(*inputs[s], out=out)
     n_steady = cache.length()[0] + 1
-    if args.hybrid:  # mean row length after the next append
+    if args.hybrid or args.budget_ratio > 0:  # mean row length after the next append
         n_steady = float(cache.row_lengths().mean()) + 1
     engine = cache.engine()
     cache.profile(True)
@@ -373,6 +360,9 @@ def run_gpu(args):
                        "engine": engine, "parallelism": f"replicas x{world}",
                        "selection": "per sequence (global token mode)" if args.global_tokens else
                        "per (layer, KV head) row" + (", head-level hybrid budgets" if args.hybrid else ""),
+                       "scorer": ["policy MLP", "H2O (cumulative attention)", "StreamingLLM (sinks + recent)"][args.scorer],
+                       "budget_rule": (f"dynamic: max(floor({args.budget_ratio} x tokens seen), 32)"
+                                       if args.budget_ratio > 0 else "fixed"),
                        "l2": f"inputs larger than L2: {bytes_step / 1e9:.2f} GB streamed per step vs 129 MB L2",
                        "steady_tokens_per_row": n_steady},
             "hbm": {"algorithmic_bytes_per_step": bytes_step, "gbs": gbs,
@@ -395,21 +385,38 @@ def run_gpu(args):
     return res
 
 
+def make_cache(wl, args):
+    """The cache of the timed run, with the mode the flags select, holding the
+    workload's prompt."""
+    from paper_2608_08878_gb300 import dc, synth_device
+    cap = wl.capacity
+    if args.hybrid:  # full-cache rows grow by one token per step
+        cap = wl.prompt_len + 2 + args.warmup + args.steps
+    cache = dc.DistillCache(wl.layers, wl.kv_heads, wl.head_dim, cap, wl.budget,
+                            batch=wl.batch, q_heads=wl.q_heads, window=wl.window,
+                            mlp_hidden=wl.mlp_hidden, layernorm=wl.layernorm, engine=args.engine,
+                            seed=wl.policy_seed, global_tokens=args.global_tokens, scorer=args.scorer,
+                            budget_ratio=args.budget_ratio)
+    if args.hybrid:
+        # head-level hybrid (Sec. 5): every fifth row (20% of the heads) keeps its
+        # full cache, the others share the rest of a 25% overall budget
+        cache.set_row_budgets(dc.head_level_hybrid_budgets(wl.rows, wl.prompt_len,
+                                                           range(0, wl.rows, 5), 0.25))
+    chunk = 4096
+    for t0 in range(0, wl.prompt_len, chunk):
+        k, v = synth_device.prompt(wl, t0, min(chunk, wl.prompt_len - t0))
+        cache.append(k, v)
+        del k, v
+    return cache
+
+
 def run_e2e(wl, args, inputs):
     """The same steps through the host-buffer API: every step copies its pinned
     host inputs in and the attention output out (dc_step_host_async, in the
     handle's stream order; one synchronisation at the end of the timed region,
     which therefore holds every copy)."""
     import torch
-    from paper_2608_08878_gb300 import dc, synth_device
-    cache = dc.DistillCache(wl.layers, wl.kv_heads, wl.head_dim, wl.capacity, wl.budget,
-                            batch=wl.batch, q_heads=wl.q_heads, window=wl.window, engine=args.engine,
-                            seed=wl.policy_seed)
-    chunk = 4096
-    for t0 in range(0, wl.prompt_len, chunk):
-        k, v = synth_device.prompt(wl, t0, min(chunk, wl.prompt_len - t0))
-        cache.append(k, v)
-        del k, v
+    cache = make_cache(wl, args)
     host = [tuple(x.cpu().pin_memory() for x in inp) for inp in inputs]
     out = torch.empty((wl.layers, wl.batch, wl.q_heads, wl.head_dim), dtype=torch.float32).pin_memory()
     W, K = args.warmup, args.steps
@@ -591,6 +598,10 @@ def main():
     ap.add_argument("--train", action="store_true", help="time the training-side kernels (App. C)")
     ap.add_argument("--hybrid", action="store_true",
                     help="head-level hybrid: 20%% of the rows keep the full cache, the rest share a 25%% budget")
+    ap.add_argument("--scorer", type=int, choices=[0, 1, 2], default=0,
+                    help="0 policy MLP, 1 H2O, 2 StreamingLLM (the heuristic scorers on the same path)")
+    ap.add_argument("--budget-ratio", type=float, default=0.0,
+                    help="> 0: dynamic budget B_t = max(floor(r x tokens seen), 32) instead of the fixed 8192")
     ap.add_argument("--global-tokens", action="store_true",
                     help="the global token mode (features over all heads and layers, one selection per sequence)")
     args = ap.parse_args()

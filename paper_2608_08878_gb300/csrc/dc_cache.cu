@@ -80,6 +80,12 @@ struct dc_cache {
   // (kept in step with Dev::rowlen) and the budgets; n is then the longest row
   bool per_row = false;
   std::vector<int> hlen, hbudget;
+  // the fused queue's row order in per-row mode (longest rows first): pinned
+  // host copy, device copy, and the event of its last upload
+  int* horder = nullptr;
+  int* roworder_dev = nullptr;
+  cudaEvent_t ev_order = nullptr;
+  bool order_valid = false;
   std::vector<void*> allocs;
   std::string err;
   bool broken = false;
@@ -442,6 +448,8 @@ dc_status dc_cache_destroy(dc_cache* h) {
   }
   for (auto& t : h->timed) { cudaEventDestroy(t.a); cudaEventDestroy(t.b); }
   for (auto e : h->event_pool) cudaEventDestroy(e);
+  if (h->ev_order) cudaEventDestroy(h->ev_order);
+  if (h->horder) cudaFreeHost(h->horder);
   free_all(h);
   h->magic = kDead;
   delete h;
@@ -566,6 +574,40 @@ dc_status dc_decode_step(dc_cache* h, const void* q, const void* k_new, const vo
   return DC_OK;
 }
 
+namespace {
+
+// Per-row mode: rows of many tiles first in the fused engine's queue, so that
+// the CTAs finish together (a long row taken last would run alone). The order
+// is rebuilt only when a row's tile count overtakes the one before it, and
+// uploaded from a pinned buffer (the previous upload has finished before the
+// buffer is rewritten).
+dc_status update_row_order(dc_cache* h) {
+  const int R = h->dev.R;
+  auto tiles = [&](int r) { return (h->hlen[r] + 1 + 127) / 128; };  // after the step's append
+  if (h->order_valid) {
+    bool sorted = true;
+    for (int i = 0; i + 1 < R && sorted; ++i) sorted = tiles(h->horder[i]) >= tiles(h->horder[i + 1]);
+    if (sorted) return DC_OK;
+  }
+  if (!h->horder) {
+    DC_CUDA(h, cudaHostAlloc(reinterpret_cast<void**>(&h->horder), (size_t)R * sizeof(int), cudaHostAllocDefault));
+    DC_CUDA(h, dalloc(h, &h->roworder_dev, (size_t)R * sizeof(int)));
+    DC_CUDA(h, cudaEventCreateWithFlags(&h->ev_order, cudaEventDisableTiming));
+  } else {
+    DC_CUDA(h, cudaEventSynchronize(h->ev_order));
+  }
+  for (int r = 0; r < R; ++r) h->horder[r] = r;
+  std::stable_sort(h->horder, h->horder + R, [&](int a, int b) { return tiles(a) > tiles(b); });
+  DC_CUDA(h, cudaMemcpyAsync(h->roworder_dev, h->horder, (size_t)R * sizeof(int), cudaMemcpyHostToDevice,
+                             h->stream));
+  DC_CUDA(h, cudaEventRecord(h->ev_order, h->stream));
+  h->dev.roworder = h->roworder_dev;
+  h->order_valid = true;
+  return DC_OK;
+}
+
+}  // namespace
+
 dc_status dc_step(dc_cache* h, const void* q, const void* k_new, const void* v_new, float* out, int budget) {
   DC_CHECK_HANDLE(h);
   if (!q || !k_new || !v_new || !out) return fail(h, DC_ERR_INVALID_ARG, "NULL pointer");
@@ -591,6 +633,9 @@ dc_status dc_step(dc_cache* h, const void* q, const void* k_new, const void* v_n
     Phase ph(h, DC_PHASE_APPEND, h->per_row ? 2 : 1);
     dc::launch_append(h->dev, k_new, v_new, 1, h->n, (int)h->seen, h->stream);
     if (h->per_row) dc::launch_rowlen_add(h->dev, 1, h->stream);
+  }
+  if (h->per_row) {
+    if (dc_status o = update_row_order(h); o != DC_OK) return o;
   }
   const dc::Step st = begin_step(h);
   if (h->per_row) {
@@ -810,6 +855,8 @@ dc_status dc_set_row_budgets(dc_cache* h, const int* budgets, int n) {
     h->hlen.clear();
     p.rowlen = nullptr;
     p.rowbudget = nullptr;
+    p.roworder = nullptr;
+    h->order_valid = false;
     return DC_OK;
   }
   if (n != p.R) return fail(h, DC_ERR_INVALID_ARG, "one budget per row (layers x batch x kv_heads)");

@@ -49,6 +49,9 @@ struct Dev {
   // device ([R] each); null when every row has the same length
   int* rowlen;
   int* rowbudget;
+  // per-row mode: the order in which the fused engine's queue hands out rows
+  // (longest first, so that no long row starts last); null: row order
+  const int* roworder;
   __nv_bfloat16* K;
   __nv_bfloat16* V;
   int* pos;

@@ -221,7 +221,11 @@ template <bool PERROW>
 __device__ __forceinline__ Item take_item(const FusedStep& fs, const Dev& p, int nT) {
   const unsigned whole = (unsigned)(p.R - fs.half_rows);
   const unsigned w = atomicAdd(fs.work + (fs.epoch & 1u), 1u);
-  if (w < whole) return Item{(int)w, 0, PERROW ? (p.rowlen[w] + kTok - 1) / kTok : nT, -1};
+  if (w < whole) {
+    if (!PERROW) return Item{(int)w, 0, nT, -1};
+    const int r = p.roworder ? p.roworder[w] : (int)w;
+    return Item{r, 0, (p.rowlen[r] + kTok - 1) / kTok, -1};
+  }
   const unsigned k = w - whole;
   if (k >= 2u * (unsigned)fs.half_rows) return Item{-1, 0, 0, 0};
   const int mid = (nT + 1) >> 1, h = (int)(k & 1u);
@@ -532,6 +536,9 @@ __global__ void __launch_bounds__(kThreads, 1)
       const int Bsel = PERROW ? (fs.B > 0 ? fs.B : p.rowbudget[r]) : fs.B;
       const int ts = r - (p.R - fs.half_rows);  // exchange slot (half rows only)
       const size_t rbase = (size_t)r * p.stride;
+      // a row longer than the shared score array keeps its scores in HBM when
+      // the radix select reads them (several evictions), or when asked to
+      const bool spill_scores = LONG && n > kFusedMaxTok && fs.do_evict && Bsel < n - 1;
       float pm[G], pnl[G], pH[G], dm[G], dnl[G], dH[G];
 #pragma unroll
       for (int h = 0; h < G; ++h) {
@@ -873,8 +880,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (i < n) {
           const float score = fp.b2 + relu_sum;
           if constexpr (LONG) {
-            // rows longer than the shared score array keep their scores in HBM
-            if (n > kFusedMaxTok || fs.write_scores) p.score[rbase + i] = score;
+            if (spill_scores || fs.write_scores) p.score[rbase + i] = score;
             if (n <= kFusedMaxTok) sc[i] = score;
           } else {
             sc[i] = score;
@@ -893,7 +899,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       auto record_h = [&](int j, float score, int pos) {
         const int i = j * kTok + tok;
         if (i < n) {
-          if (n > kFusedMaxTok || fs.write_scores) p.score[rbase + i] = score;
+          if (spill_scores || fs.write_scores) p.score[rbase + i] = score;
           if (n <= kFusedMaxTok) sc[i] = score;
           const uint32_t kk = score_key(score);
           if (ev_slot < 0 || kk < ev_key || (kk == ev_key && pos > ev_pos)) {
