@@ -601,6 +601,28 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
       g += nTi;
       gs += nTi;
+      // per-token state of this warpgroup's V-pass tiles (the same tiles as its
+      // K pass), loaded two own tiles ahead: window sums (this thread wrote
+      // them in the K pass), positions, |v|; the first two issued here, so that
+      // their latency overlaps the statistics merge
+      const int j0 = t0 + ((wg - gv) & 1);
+      const float4* szrow = p.SZ + rbase + tok;
+      const int* posrow = p.pos + rbase + tok;
+      const float* vnrow = p.vnorm + rbase + tok;
+      const float4 kZero4 = make_float4(0.f, 0.f, 0.f, 0.f);
+      float4 szA = kZero4, szB = kZero4;
+      int posA = 0, posB = 0;
+      float vnA = 0.f, vnB = 0.f;
+      if constexpr (!FULL && !GLOB) {
+        szA = j0 < t1 ? szrow[j0 * kTok] : kZero4;
+        szB = j0 + 2 < t1 ? szrow[(j0 + 2) * kTok] : kZero4;
+        posA = j0 < t1 ? posrow[j0 * kTok] : 0;
+        posB = j0 + 2 < t1 ? posrow[(j0 + 2) * kTok] : 0;
+      }
+      if constexpr (!FULL) {
+        vnA = j0 < t1 ? vnrow[j0 * kTok] : 0.f;
+        vnB = j0 + 2 < t1 ? vnrow[(j0 + 2) * kTok] : 0.f;
+      }
       if constexpr (GS > 0) tmem_st_wait();
       // ---------------- row softmax statistics (deterministic merge order):
       // the maximum first, then every partial (l, u) rescaled to it and summed
@@ -697,29 +719,17 @@ __global__ void __launch_bounds__(kThreads, 1)
         p.hq[(size_t)r * G + etid] = Hh[etid];
       }
 
+      // One eviction (the steady state): slot B, the only mover, is loaded now
+      // (its window sums were written before the merge barrier), so that the
+      // select does not wait on it; what the V pass may still write is loaded
+      // at the select.
+      const bool single_evict = fs.do_evict && n == Bsel + 1;
+      SlotCopy mv{};
+      if (single_evict && half != 0 && etid < kWarp) slot_load_settled(p, rbase + Bsel, etid, fs.write_scores, mv);
+
       // ---------------- V pass: this warpgroup's tiles; prep of the next one
       // overlaps the MMAs of the current one
       const float pos_den = (float)max(st.p_newest, 1);
-      const int j0 = t0 + ((wg - gv) & 1);
-      // per-token state of this warpgroup's tiles, loaded two own tiles ahead
-      // (window sums written by the K pass, positions, |v|)
-      const float4* szrow = p.SZ + rbase + tok;
-      const int* posrow = p.pos + rbase + tok;
-      const float* vnrow = p.vnorm + rbase + tok;
-      const float4 kZero4 = make_float4(0.f, 0.f, 0.f, 0.f);
-      float4 szA = kZero4, szB = kZero4;
-      int posA = 0, posB = 0;
-      float vnA = 0.f, vnB = 0.f;
-      if constexpr (!FULL && !GLOB) {
-        szA = j0 < t1 ? szrow[j0 * kTok] : kZero4;
-        szB = j0 + 2 < t1 ? szrow[(j0 + 2) * kTok] : kZero4;
-        posA = j0 < t1 ? posrow[j0 * kTok] : 0;
-        posB = j0 + 2 < t1 ? posrow[(j0 + 2) * kTok] : 0;
-      }
-      if constexpr (!FULL) {
-        vnA = j0 < t1 ? vnrow[j0 * kTok] : 0.f;
-        vnB = j0 + 2 < t1 ? vnrow[(j0 + 2) * kTok] : 0.f;
-      }
       auto prep = [&](int j) {
         const int gvj = gv + (j - t0), pb = gvj & 1;
         const float4 sz = szA;
@@ -956,14 +966,13 @@ __global__ void __launch_bounds__(kThreads, 1)
           op[h * D + tok] = half == 0 ? ov[h] + __ldcg(&fs.xo[((size_t)ts * G + h) * D + tok]) : ov[h];
       }
       // ---------------- argtop_B and prune
-      if (fs.do_evict && n == Bsel + 1) {
+      if (single_evict) {
         // one eviction (the steady state): the lowest-ranked token, from each
         // thread's running candidate; slot B (the last, held by the whole row
         // or by half 1) is the only mover and fills the evicted slot. Half
         // rows swap their candidates first.
         const bool mover = half != 0;
-        SlotCopy mv{};
-        if (mover && etid < kWarp) mv = slot_load(p, rbase + Bsel, etid);
+        if (mover && etid < kWarp) slot_load_late(p, rbase + Bsel, etid, fs.write_scores, mv);
         auto lower = [](uint32_t ka, int sa, int pa, uint32_t kb, int sb, int pb) {  // (kb, sb) ranks lower?
           if (sb < 0) return false;
           if (sa < 0) return true;

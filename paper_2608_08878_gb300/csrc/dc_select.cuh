@@ -116,6 +116,26 @@ __device__ __forceinline__ SlotCopy slot_load(const Dev& p, size_t src, int lane
   return c;
 }
 
+// slot_load in two parts, for a caller that loads a slot early, while the
+// slot's score, cumulative alpha and features may still be written:
+// slot_load_settled takes K, V, position, |v|, window sums (and the score when
+// `score_late` is false); slot_load_late takes the rest.
+__device__ __forceinline__ void slot_load_settled(const Dev& p, size_t src, int lane, bool score_late, SlotCopy& c) {
+  const int VPR = p.d / 8;
+  if (lane < VPR) c.kv = reinterpret_cast<const uint4*>(p.K)[src * VPR + lane];
+  else if (lane < 2 * VPR) c.kv = reinterpret_cast<const uint4*>(p.V)[src * VPR + lane - VPR];
+  if (lane == 0) c.f.x = (unsigned)p.pos[src];
+  else if (lane == 1) c.f.x = __float_as_uint(p.vnorm[src]);
+  else if (lane == 2) c.f = *reinterpret_cast<const uint4*>(p.SZ + src);
+  else if (lane == 3 && !score_late) c.f.x = __float_as_uint(p.score[src]);
+}
+
+__device__ __forceinline__ void slot_load_late(const Dev& p, size_t src, int lane, bool score_late, SlotCopy& c) {
+  if (lane == 3 && score_late) c.f.x = __float_as_uint(p.score[src]);
+  else if (lane == 4 && p.acc) c.f.x = __float_as_uint(p.acc[src]);
+  else if (lane >= 5 && lane < 10 && p.keep_features) c.f.x = __float_as_uint(p.feat[src * 5 + lane - 5]);
+}
+
 __device__ __forceinline__ void slot_store(const Dev& p, size_t dst, int lane, const SlotCopy& c) {
   const int VPR = p.d / 8;
   if (lane < VPR) reinterpret_cast<uint4*>(p.K)[dst * VPR + lane] = c.kv;
