@@ -70,6 +70,19 @@ def step_bytes(wl, n: int, moved_per_row: float = 1.0) -> float:
     return wl.rows * per_row
 
 
+def step_bytes_global(wl, n: int, moved_per_seq: float = 1.0) -> float:
+    """Whole-step algorithmic bytes of the global token mode: every row's K, V
+    and positions read once (4d + 4 bytes per token-row); per sequence and
+    token, the window sums read and written (32), the ring's previous and
+    departing query terms read and this query's written (24), cumulative alpha
+    in alpha_mode 1 (8); the append; each sequence's moves, on every row. The
+    rows' partial sums are the implementation's exchange, not counted."""
+    d = wl.head_dim
+    per_seq_tok = 32 + 24 + (8 if wl.alpha_mode else 0)
+    return (wl.rows * n * (4 * d + 4) + wl.batch * n * per_seq_tok + wl.rows * (4 * d + 20)
+            + moved_per_seq * wl.rows * 2 * (4 * d + 20))
+
+
 def fused_traffic_per_token_row():
     """DRAM bytes per token-row of the fused kernel from the committed ncu
     summary, or None if the kernel source changed since it was captured."""
@@ -288,7 +301,7 @@ def run_gpu(args):
     cache.profile(False)
     el_ms, value = job_throughput(el_ms, K, dist, device="cuda")
     ms_per_step = el_ms / K
-    bytes_step = step_bytes(wl, n_steady)
+    bytes_step = step_bytes_global(wl, n_steady) if args.global_tokens else step_bytes(wl, n_steady)
     gbs = bytes_step / (ms_per_step / 1e3) / 1e9
     peaks, peak_src = measured_peaks()
 
@@ -297,7 +310,10 @@ def run_gpu(args):
     dom_ms, dom_n = prof[dom]
     per_launch_ms = dom_ms / dom_n
     d = wl.head_dim
-    if dom == "attend" and engine == "fused":
+    if dom == "attend" and engine == "fused" and args.global_tokens:
+        # the rows' pass: K/V and positions (the window state is per sequence)
+        alg = wl.rows * n_steady * (4 * d + 4)
+    elif dom == "attend" and engine == "fused":
         # the whole step but the append: K/V, positions, window sums, one move per row
         alg = wl.rows * (row_bytes_per_step(n_steady, d, wl.alpha_mode) + 2 * (4 * d + 20))
     elif dom == "attend":
@@ -308,7 +324,7 @@ def run_gpu(args):
         alg = wl.rows * row_bytes_per_step(n_steady, d, wl.alpha_mode)
     achieved = alg / (per_launch_ms / 1e3) / 1e9
     traffic = None
-    if dom == "attend" and engine == "fused":
+    if dom == "attend" and engine == "fused" and not (args.global_tokens or args.hybrid or args.scorer):
         tpr = fused_traffic_per_token_row()
         if tpr is not None:
             traffic = wl.rows * n_steady * tpr  # scaled from the profiled case by token-rows

@@ -378,7 +378,8 @@ dc_status dc_cache_create(int layers, int kv_heads, int head_dim, int capacity, 
   A(&p.opart, (size_t)R * p.smax * G * head_dim * sizeof(float));
   A(&p.holes, RC * sizeof(int));
   if (p.seq_rows) {
-    A(&p.gpart, RC * 2 * sizeof(float4));
+    A(&p.gpart, RC * sizeof(float4));
+    A(&p.gring, (size_t)cfg.batch * cfg.window * p.stride * sizeof(float2));
     A(&p.gmoves, (size_t)cfg.batch * (1 + 2 * (size_t)p.stride) * sizeof(int));
   }
   A(&h->st_q, (size_t)R * G * head_dim * 2);

@@ -38,12 +38,17 @@ struct Dev {
   int R, cap, stride, d, G, qh, kvh, w, hidden, layernorm, alpha_mode, keep_features;
   int scorer, n_sinks;  // 0 policy MLP, 1 H2O (cumulative alpha), 2 StreamingLLM
   // global token mode: rows per sequence (layers x KV heads), 0 = per-row mode;
-  // batch = sequences. Per-token partial sums of each row ([R][stride][2]:
-  // window terms of the previous/departing queries, then this step's mass,
-  // squared mass, entropy-weighted mass and |v|) and each sequence's move
-  // list ([batch][1 + 2 stride]: count, then hole/mover pairs).
+  // batch = sequences. Per-token partial sums of each row ([R][stride]
+  // float4: this step's attention mass, squared mass, entropy-weighted mass
+  // and |v|); per sequence, the pooled contribution (mass, entropy-weighted
+  // mass) of each of the last w queries to every token ([batch][w][stride]
+  // float2, ring slot = step mod w, zero for a token not yet cached at that
+  // step), from which the window sums gain the previous query's terms and lose
+  // the departing query's exactly; and each sequence's move list
+  // ([batch][1 + 2 stride]: count, then hole/mover pairs).
   int seq_rows, batch;
   float4* gpart;
+  float2* gring;
   int* gmoves;
   // per-row budgets (head-level hybrid): each row's length and budget on the
   // device ([R] each); null when every row has the same length
@@ -74,6 +79,11 @@ struct Dev {
   int smax;
   float c;        // log2(e) / sqrt(d): raw logit difference -> log2 units
 };
+
+// Ring entry (ring slot k, token slot i) of sequence b.
+__host__ __device__ inline float2* gring_at(const Dev& p, int b, int k, size_t i) {
+  return p.gring + ((size_t)b * p.w + k) * p.stride + i;
+}
 
 // Arguments that change every step.
 struct Step {

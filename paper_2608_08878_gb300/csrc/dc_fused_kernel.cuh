@@ -268,9 +268,9 @@ __device__ __forceinline__ Item read_item(volatile int* ring, int gr, volatile i
 // HEUR: a heuristic scorer (H2O or StreamingLLM, Dev::scorer) ranks the tokens
 // instead of the policy MLP, whose tensor-core layer is then skipped.
 // GLOB: global token mode: each row leaves its share of the per-token sums in
-// Dev::gpart (window terms in the K pass; mass, squared mass, entropy-weighted
-// mass and |v| in the V pass); features, scores and the selection are made
-// per sequence afterwards.
+// Dev::gpart (mass, squared mass, entropy-weighted mass and |v|, in the V
+// pass; the window sums come from the sequence's ring of pooled query terms);
+// features, scores and the selection are made per sequence afterwards.
 // PERROW: rows of different lengths and budgets (Dev::rowlen, Dev::rowbudget;
 // FusedStep::B > 0 overrides every row's budget); the kernel writes each
 // row's new length after its selection. No half rows.
@@ -575,7 +575,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (i < n) {
 #pragma unroll
           for (int h = 0; h < G; ++h) online_add(m[h], l[h], u[h], S16[h], c);
-          if (!FULL && (st.has_prev || st.has_dep)) {
+          if (!FULL && !GLOB && (st.has_prev || st.has_dep)) {
             // terms of the previous and the departing query, masked (x 1 or x 0,
             // both exact) where the token was not yet in the cache at that step
             float zp, sp, zd, sd;
@@ -583,12 +583,8 @@ __global__ void __launch_bounds__(kThreads, 1)
             window_terms<G>(S16 + 2 * G, dm, dnl, dH, c, zd, sd);
             const float mp = (st.has_prev && pos <= st.p_prev) ? 1.f : 0.f;
             const float md = (st.has_dep && pos <= st.p_dep) ? 1.f : 0.f;
-            if constexpr (GLOB) {
-              p.gpart[(rbase + i) * 2] = make_float4(zp * mp, sp * mp, zd * md, sd * md);
-            } else {
-              sz = window_update(sz, sp * mp, sd * md, zp * mp, zd * md);
-              p.SZ[rbase + i] = sz;
-            }
+            sz = window_update(sz, sp * mp, sd * md, zp * mp, zd * md);
+            p.SZ[rbase + i] = sz;
           }
         }
         if (!LONG || j < onchip_tiles<GS>()) {
@@ -793,7 +789,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             float a2 = 0.f;
 #pragma unroll
             for (int h = 0; h < G; ++h) a2 = fmaf(a[h], a[h], a2);
-            p.gpart[(rbase + i) * 2 + 1] = make_float4(zc, a2, scur, vn);
+            p.gpart[rbase + i] = make_float4(zc, a2, scur, vn);
           }
           return make_float2(0.f, 0.f);
         }

@@ -1,14 +1,15 @@
 // dc_global.cu -- the global token mode (Sec. 3.1.1: a token's features pool
 // every attention head of every layer; one policy score and one argtop_B per
 // sequence). The rows of a sequence (its layers x KV heads) share one token
-// set, slot for slot. The split engine's per-row kernels leave each row's share
-// of the per-token sums in Dev::gpart; here they are pooled per sequence (in a
-// fixed row order, so the window terms of a departing query cancel exactly the
-// sums they once entered), turned into features and scores, and the
-// sequence's selection is applied to every one of its rows.
+// set, slot for slot. The per-row kernels (fused or split engine) leave each
+// row's share of the per-token sums in Dev::gpart; here they are pooled per
+// sequence, turned into features and scores, and the sequence's selection is
+// applied to every one of its rows.
 //
 // Per-sequence state lives in the sequence's home row (layer 0, KV head 0):
-// window sums, cumulative alpha, features and scores.
+// window sums, cumulative alpha, features and scores; beside it, the ring of
+// the last w queries' pooled terms per token (Dev::gring), which moves with
+// the tokens.
 #include "dc_common.cuh"
 #include "dc_kernels.h"
 #include "dc_select.cuh"
@@ -16,40 +17,56 @@
 namespace dc {
 namespace {
 
-constexpr int kFeatThreads = 256;
+constexpr int kFeatTok = 64;     // tokens per block
+constexpr int kFeatGroups = 4;   // threads per token, each summing a quarter of the rows
+constexpr int kFeatThreads = kFeatTok * kFeatGroups;
 constexpr int kSelThreads = 1024;
 constexpr int kMoveThreads = 256;
 
 __device__ __forceinline__ int seq_row(const Dev& p, int b, int l, int g) { return (l * p.batch + b) * p.kvh + g; }
 
-// grid (ceil(n / 256), batch), block 256; dynamic shared memory: the policy blob.
+// grid (ceil(n / 64), batch), block 256 = 64 tokens x 4 row groups; dynamic
+// shared memory: the policy blob, then the groups' partial sums.
+// The rows of a sequence are taken in a fixed order (layer-major, then KV
+// head): group q sums rows [q S / 4, (q + 1) S / 4) in that order, and the four
+// partials are added in group order.
 __global__ void __launch_bounds__(kFeatThreads) glob_feature_kernel(Dev p, Step st) {
   extern __shared__ float wsm[];
-  const int b = blockIdx.y, i = blockIdx.x * blockDim.x + threadIdx.x;
   const int H = p.hidden, nblob = 9 * H + 1;
+  float4* part = reinterpret_cast<float4*>(wsm + ((nblob + 3) & ~3));  // [groups][kFeatTok]
+  const int b = blockIdx.y, t = threadIdx.x % kFeatTok, grp = threadIdx.x / kFeatTok;
+  const int i = blockIdx.x * kFeatTok + t;
   for (int e = threadIdx.x; e < nblob; e += blockDim.x) wsm[e] = p.policy[e];
-  __syncthreads();
-  if (i >= st.n) return;
-  const int layers = p.seq_rows / p.kvh;
-  const bool window = st.has_prev || st.has_dep;
-  float4 W = make_float4(0.f, 0.f, 0.f, 0.f), P = make_float4(0.f, 0.f, 0.f, 0.f);
-  for (int l = 0; l < layers; ++l)
-    for (int g = 0; g < p.kvh; ++g) {
-      const size_t slot = (size_t)seq_row(p, b, l, g) * p.stride + i;
-      if (window) {
-        const float4 w = p.gpart[slot * 2];
-        W.x += w.x; W.y += w.y; W.z += w.z; W.w += w.w;
-      }
-      const float4 q = p.gpart[slot * 2 + 1];
+  float4 P = make_float4(0.f, 0.f, 0.f, 0.f);
+  if (i < st.n) {
+    const int S = p.seq_rows, r0 = grp * S / kFeatGroups, r1 = (grp + 1) * S / kFeatGroups;
+    int l = r0 / p.kvh, g = r0 % p.kvh;
+    for (int rr = r0; rr < r1; ++rr) {
+      const float4 q = p.gpart[(size_t)seq_row(p, b, l, g) * p.stride + i];
       P.x += q.x; P.y += q.y; P.z += q.z; P.w += q.w;
+      if (++g == p.kvh) { g = 0; ++l; }
     }
+  }
+  part[grp * kFeatTok + t] = P;
+  __syncthreads();
+  if (grp != 0 || i >= st.n) return;
+  for (int q = 1; q < kFeatGroups; ++q) {
+    const float4 pp = part[q * kFeatTok + t];
+    P.x += pp.x; P.y += pp.y; P.z += pp.z; P.w += pp.w;
+  }
   const size_t s0 = (size_t)seq_row(p, b, 0, 0) * p.stride + i;
   float4 sz = p.SZ[s0];
-  if (window) {
-    // the previous step's query joins the stored sums, the departing one leaves
-    sz = window_update(sz, W.y, W.w, W.x, W.z);
+  if (st.has_prev || st.has_dep) {
+    // the previous step's query joins the stored sums, the departing one
+    // (whose ring slot this step's query takes) leaves them: both read from
+    // the ring, so the departing terms are exactly those once added
+    const float2 pv = st.has_prev ? *gring_at(p, b, st.slot_prev, i) : make_float2(0.f, 0.f);
+    const float2 dp = st.has_dep ? *gring_at(p, b, st.slot, i) : make_float2(0.f, 0.f);
+    sz = window_update(sz, pv.y, dp.y, pv.x, dp.x);
     p.SZ[s0] = sz;
   }
+  // this step's query: total mass and entropy-weighted mass over every head
+  *gring_at(p, b, st.slot, i) = make_float2(P.x, P.z);
   const float N = (float)(p.seq_rows * p.G);
   const float mean = P.x / N;
   const float var = fmaxf(P.y / N - mean * mean, 0.f);
@@ -122,14 +139,18 @@ __global__ void __launch_bounds__(kMoveThreads) glob_compact_kernel(Dev p) {
       }
     }
     if (home && p.keep_features && lane < 5) p.feat[dst * 5 + lane] = ft;
+    if (home) {
+      const size_t id = dst - base, is = src - base;
+      for (int e = lane; e < p.w; e += kWarp) *gring_at(p, b, e, id) = *gring_at(p, b, e, is);
+    }
   }
 }
 
 }  // namespace
 
 void launch_glob_features(const Dev& p, const Step& st, cudaStream_t s) {
-  const dim3 grid((st.n + kFeatThreads - 1) / kFeatThreads, p.batch);
-  const size_t smem = (size_t)(9 * p.hidden + 1) * sizeof(float);
+  const dim3 grid((st.n + kFeatTok - 1) / kFeatTok, p.batch);
+  const size_t smem = (size_t)((9 * p.hidden + 1 + 3) & ~3) * sizeof(float) + kFeatGroups * kFeatTok * sizeof(float4);
   glob_feature_kernel<<<grid, kFeatThreads, smem, s>>>(p, st);
 }
 

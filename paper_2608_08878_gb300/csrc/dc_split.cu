@@ -51,6 +51,12 @@ __global__ void __launch_bounds__(256) append_kernel(Dev p, const uint4* __restr
     p.vnorm[slot] = sqrtf(ss);
     p.SZ[slot] = make_float4(0.f, 0.f, 0.f, 0.f);
     if (p.acc) p.acc[slot] = 0.f;
+    if (p.seq_rows && r < p.batch * p.kvh && r % p.kvh == 0) {
+      // global token mode, the sequence's home row: no past query saw this token
+      const int b = r / p.kvh;
+      const size_t i = slot - (size_t)r * p.stride;
+      for (int k = 0; k < p.w; ++k) *gring_at(p, b, k, i) = make_float2(0.f, 0.f);
+    }
   }
 }
 
@@ -172,7 +178,8 @@ __global__ void __launch_bounds__(kTile) split_qk_kernel(Dev p, Step st,
         lo[h] = s[h];
         online_add(m[h], l[h], u[h], s[h], c);
       }
-      if (st.has_prev || st.has_dep) {
+      // global token mode: the window sums come from the sequence's ring
+      if (!p.seq_rows && (st.has_prev || st.has_dep)) {
         const int pos = p.pos[slot];
         float zp = 0.f, sp_ = 0.f, zd = 0.f, sd = 0.f;
         float rm[G], rnl[G], rH[G];
@@ -186,8 +193,7 @@ __global__ void __launch_bounds__(kTile) split_qk_kernel(Dev p, Step st,
           for (int h = 0; h < G; ++h) { rm[h] = ring_ml[1][h][0]; rnl[h] = ring_ml[1][h][1]; rH[h] = ring_ml[1][h][2]; }
           window_terms<G>(s + 2 * G, rm, rnl, rH, c, zd, sd);
         }
-        if (p.seq_rows) p.gpart[slot * 2] = make_float4(zp, sp_, zd, sd);  // pooled per sequence later
-        else p.SZ[slot] = window_update(p.SZ[slot], sp_, sd, zp, zd);
+        p.SZ[slot] = window_update(p.SZ[slot], sp_, sd, zp, zd);
       }
     }
   }
@@ -296,7 +302,7 @@ __global__ void __launch_bounds__(kTile) split_v_kernel(Dev p, Step st) {
         float a2 = 0.f;
 #pragma unroll
         for (int h = 0; h < G; ++h) a2 = fmaf(a[h], a[h], a2);
-        p.gpart[slot * 2 + 1] = make_float4(mean, a2, sc, p.vnorm[slot]);
+        p.gpart[slot] = make_float4(mean, a2, sc, p.vnorm[slot]);
       } else {
       mean /= (float)G;
       float var = 0.f;
