@@ -93,11 +93,16 @@ def test_budget_at_least_n_is_full_attention(engine):
 
 @pytest.mark.parametrize("engine", ENGINES)
 def test_mistral_single_layer(engine):
-    wl = synth.MISTRAL_1L.with_(steps=72)  # > w so queries leave the window
+    """The Mistral-7B single-layer workload as specified: all 8 rows, 8192-token
+    prompt compressed to 2048, 128 decode steps each evicting one token (queries
+    leave the 64-step window from step 64 on)."""
+    wl = synth.MISTRAL_1L
+    assert wl.steps == 128
     ls = LockStep(wl, range(wl.rows), engine=engine)
     ls.load_prompt()
     for s in range(wl.steps):
-        ls.step(check=(s < 3 or s % 8 == 0 or s >= 64))
+        ls.step(check=(s < 3 or s % 8 == 0 or s >= 124))
+    assert ls.cache.length()[0] == wl.budget
 
 
 @pytest.mark.parametrize("engine", ENGINES)
