@@ -500,7 +500,7 @@ def run_sweep(args):
         B, d = wl.budget, wl.head_dim
         cache = dc.DistillCache(wl.layers, wl.kv_heads, d, B + 1, B, batch=b, q_heads=wl.q_heads,
                                 window=wl.window, mlp_hidden=wl.mlp_hidden, layernorm=wl.layernorm,
-                                seed=wl.policy_seed)
+                                seed=wl.policy_seed, engine=args.engine)
         chunk = max(1, min(B, (1 << 31) // (wl.rows * d * 2)))
         for t0 in range(0, B, chunk):
             k, v = synth_device.prompt(wl, t0, min(chunk, B - t0))
