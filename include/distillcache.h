@@ -199,7 +199,9 @@ dc_status dc_set_row_budgets(dc_cache* h, const int* budgets_host, int n);
 dc_status dc_get_row_lengths(dc_cache* h, int* lengths_host, int n);
 
 /* Which engine a step over n tokens per row would use (n <= 0: the next
- * decode step): 1 split, 2 fused. */
+ * decode step): 1 split, 2 fused (one CTA per row), 3 fused on row pairs (each
+ * warpgroup of a CTA on a row of its own; short rows, more rows than SMs, when
+ * that schedule is expected to be faster). */
 dc_status dc_engine(dc_cache* h, int n, int* engine);
 
 /* argtop_B and prune (Algorithm 1): every row keeps its min(n, B) highest-scored

@@ -761,7 +761,8 @@ dc_status dc_step_host_async(dc_cache* h, const void* q, const void* k_new, cons
 
 dc_status dc_engine(dc_cache* h, int n, int* engine) {
   if (!valid(h) || !engine) return DC_ERR_INVALID_ARG;
-  *engine = use_fused(h, n > 0 ? n : h->n + 1) ? 2 : 1;
+  const int nn = n > 0 ? n : h->n + 1;
+  *engine = !use_fused(h, nn) ? 1 : dc::fused_pairs(h->dev, nn, h->num_sms) ? 3 : 2;
   return DC_OK;
 }
 

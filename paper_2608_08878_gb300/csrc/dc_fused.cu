@@ -15,9 +15,26 @@ bool fused_eligible(const Dev& p, int n) {
          p.logit != nullptr && p.score != nullptr;
 }
 
-int fused_smem_bytes() { return kSmemBytes; }
+int fused_smem_bytes() { return Smem<false>::BYTES; }
+
+bool fused_pairs(const Dev& p, int n, int num_sms) {
+  const int nT = (n + kTok - 1) / kTok;
+  if (!(p.seq_rows == 0 && p.rowlen == nullptr && p.scorer == 0 && p.R % 2 == 0 && p.R > num_sms && nT >= 1 &&
+        nT <= kPairTiles))
+    return false;
+  // Critical path of a CTA in units of one token's streaming time at an SM's
+  // share of the bandwidth (measured with per-row timestamps): a row costs its
+  // n tokens plus ~350 of serial epilogue (statistics merge, output, select), a
+  // pair 2n plus ~410. Pairs halve the serial part per row but make the last
+  // wave coarser: the cheaper schedule wins.
+  const int rem = p.R % num_sms;
+  const double waves1 = p.R / num_sms + (rem == 0 ? 0.0 : 2 * rem <= num_sms ? 0.5 : 1.0);
+  const double waves2 = (p.R / 2 + num_sms - 1) / num_sms;
+  return waves2 * (2.0 * n + 410.0) < waves1 * (n + 350.0);
+}
 
 int fused_half_rows(const Dev& p, int n, const FusedStep& fs, int num_sms) {
+  if (fused_pairs(p, n, num_sms)) return 0;
   const int grid = fused_grid(p, num_sms), rem = p.R % grid;
   const int nT = (n + kTok - 1) / kTok;
   const bool ok = fs.xflag && fs.xstats && fs.xo && fs.xsel && rem > 0 && 2 * rem <= grid && nT >= 2 &&
@@ -30,6 +47,7 @@ cudaError_t launch_fused_step(const FusedMaps& maps, const Dev& p, const Step& s
   // the other variants are instantiated in their own translation units
   if (p.seq_rows) return launch_fused_glob(maps, p, st, fs, fp, num_sms, s);
   if (p.rowlen || p.scorer != 0) return launch_fused_heur_perrow(maps, p, st, fs, fp, num_sms, s);
+  if (fs.half_rows == 0 && fused_pairs(p, st.n, num_sms)) return launch_fused_pair(maps, p, st, fs, fp, num_sms, s);
   const int grid = fused_grid(p, num_sms);
   const bool lg = st.n > fused_onchip_tokens(p.G);
 #define DC_FUSED_LAUNCH(D, G) \

@@ -77,8 +77,15 @@ cudaError_t make_fused_maps(const Dev& p, FusedMaps* maps, const char** why);
 // FusedPolicy fields and the host copy of the weight tile (128 * 32 bf16).
 void prepare_policy(const float* blob, int H, int layernorm, FusedPolicy* fp, std::vector<__nv_bfloat16>* wtile);
 
+// Whether a step over n tokens runs on row pairs (each warpgroup of a CTA on
+// its own row): short rows (at most kPairTiles tiles), more rows than SMs, an
+// even row count, the plain step (policy scorer, equal lengths, per-row
+// selection).
+bool fused_pairs(const Dev& p, int n, int num_sms);
+
 // How many rows a step over n tokens splits into halves (see FusedStep): the
-// remainder of R over the grid when it is at most half the grid, else 0.
+// remainder of R over the grid when it is at most half the grid, else 0 (and
+// 0 on row pairs).
 int fused_half_rows(const Dev& p, int n, const FusedStep& fs, int num_sms);
 
 cudaError_t launch_fused_step(const FusedMaps& maps, const Dev& p, const Step& st, const FusedStep& fs,
@@ -90,6 +97,9 @@ cudaError_t launch_fused_step(const FusedMaps& maps, const Dev& p, const Step& s
 cudaError_t launch_fused_heur_perrow(const FusedMaps& maps, const Dev& p, const Step& st, const FusedStep& fs,
                                      const FusedPolicy& fp, int num_sms, cudaStream_t s);
 cudaError_t launch_fused_glob(const FusedMaps& maps, const Dev& p, const Step& st, const FusedStep& fs,
+                              const FusedPolicy& fp, int num_sms, cudaStream_t s);
+// Row pairs (dc_fused_pair.cu).
+cudaError_t launch_fused_pair(const FusedMaps& maps, const Dev& p, const Step& st, const FusedStep& fs,
                               const FusedPolicy& fp, int num_sms, cudaStream_t s);
 
 // Attention only over the first n tokens of every row as they are (the

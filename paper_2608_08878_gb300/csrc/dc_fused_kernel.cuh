@@ -75,17 +75,29 @@ constexpr uint32_t kTmemCols = 512;
 constexpr int kColS = 0, kColO = 32, kColM = 128;
 constexpr int kStashA = 48, kStashAEnd = 128, kStashB = 384, kStashBEnd = 512;
 
-constexpr int OFF_STAGE = 0;
-constexpr int OFF_Q = OFF_STAGE + kStages * kStageBytes;  // 2 x 4 KB
-constexpr int OFF_P = OFF_Q + 2 * 4096;                    // 2 x 4 KB (one per warpgroup)
-constexpr int OFF_A = OFF_P + 2 * 4096;                    // 2 x 8 KB (one per warpgroup)
-constexpr int OFF_W = OFF_A + 2 * 8192;                    // 8 KB
-constexpr int OFF_AUX = OFF_W + 8192;                      // kStages x 2560 B
-constexpr int OFF_SC = OFF_AUX + kStages * kAuxBytes;      // head G-1 logits, then scores
-constexpr int OFF_MISC = OFF_SC + kFusedMaxTok * 4;
+// Row pairs (PAIR): an item is two rows of at most kPairTiles tiles, one per
+// warpgroup; their K and V tiles alternate in the stage ring.
+constexpr int kPairTiles = 21;
+constexpr int kPairTok = kPairTiles * kTok;
+constexpr int kColOB = 48;                                 // the second row's O (PAIR)
+constexpr int kPairStashA = 64;                            // the first row's logit stash (PAIR)
+
+// Shared memory layout; PAIR keeps four query tiles (two per item, double
+// buffered) and a smaller logit/score array per row.
+template <bool PAIR>
+struct Smem {
+  static constexpr int STAGE = 0;
+  static constexpr int Q = STAGE + kStages * kStageBytes;   // (2 or 4) x 4 KB
+  static constexpr int P = Q + (PAIR ? 4 : 2) * 4096;       // 2 x 4 KB (one per warpgroup)
+  static constexpr int A = P + 2 * 4096;                    // 2 x 8 KB (one per warpgroup)
+  static constexpr int W = A + 2 * 8192;                    // 8 KB
+  static constexpr int AUX = W + 8192;                      // kStages x 2560 B
+  static constexpr int SC = AUX + kStages * kAuxBytes;      // head G-1 logits, then scores
+  static constexpr int MISC = SC + (PAIR ? 2 * kPairTok : kFusedMaxTok) * 4;
+  static constexpr int BYTES = MISC + 4096 + 1024;          // misc area + alignment slack
+  static_assert(BYTES <= 232448, "more shared memory than a CTA may have");
+};
 constexpr int MISC_BYTES = 4096;
-constexpr int kSmemBytes = OFF_MISC + MISC_BYTES + 1024;   // + alignment slack
-static_assert(kSmemBytes <= 232448, "more shared memory than a CTA may have");
 
 // barrier indices in the misc area
 enum {
@@ -217,10 +229,11 @@ struct Item {
 
 constexpr int kItemRing = 8;  // items published ahead of the slowest role (at most ~3)
 
-template <bool PERROW>
+template <bool PERROW, bool PAIR>
 __device__ __forceinline__ Item take_item(const FusedStep& fs, const Dev& p, int nT) {
-  const unsigned whole = (unsigned)(p.R - fs.half_rows);
   const unsigned w = atomicAdd(fs.work + (fs.epoch & 1u), 1u);
+  if constexpr (PAIR) return w < (unsigned)(p.R / 2) ? Item{(int)(2 * w), 0, nT, -1} : Item{-1, 0, 0, 0};
+  const unsigned whole = (unsigned)(p.R - fs.half_rows);
   if (w < whole) {
     if (!PERROW) return Item{(int)w, 0, nT, -1};
     const int r = p.roworder ? p.roworder[w] : (int)w;
@@ -271,14 +284,22 @@ __device__ __forceinline__ Item read_item(volatile int* ring, int gr, volatile i
 // Dev::gpart (mass, squared mass, entropy-weighted mass and |v|, in the V
 // pass; the window sums come from the sequence's ring of pooled query terms);
 // features, scores and the selection are made per sequence afterwards.
+// PAIR: items are row pairs (rows 2w and 2w + 1) of at most kPairTiles tiles,
+// warpgroup w doing the whole of row 2w + w (its K and V tiles alternate with
+// the other row's in the ring), so that one row's merge, output and select
+// overlap the other's; policy scorer, whole rows, equal lengths only.
 // PERROW: rows of different lengths and budgets (Dev::rowlen, Dev::rowbudget;
 // FusedStep::B > 0 overrides every row's budget); the kernel writes each
 // row's new length after its selection. No half rows.
-template <int D, int G, bool LONG, bool FULL, bool HEUR, bool GLOB, bool PERROW>
+template <int D, int G, bool LONG, bool FULL, bool HEUR, bool GLOB, bool PERROW, bool PAIR>
 __global__ void __launch_bounds__(kThreads, 1)
     fused_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmV, Dev p,
                  Step st, FusedStep fs, FusedPolicy fp) {
   constexpr int GS = G - 1;  // heads whose logits wait in TMEM between the passes
+  static_assert(!PAIR || (!LONG && !FULL && !HEUR && !GLOB && !PERROW), "row pairs: the plain step only");
+  using L = Smem<PAIR>;
+  constexpr int OFF_STAGE = L::STAGE, OFF_Q = L::Q, OFF_P = L::P, OFF_A = L::A, OFF_W = L::W, OFF_AUX = L::AUX,
+                OFF_SC = L::SC, OFF_MISC = L::MISC;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint64_t* bar = reinterpret_cast<uint64_t*>(smem + OFF_MISC);
@@ -293,6 +314,12 @@ __global__ void __launch_bounds__(kThreads, 1)
   int* s_best_slot = reinterpret_cast<int*>(smem + OFF_MISC + 2176);      // [8]
   float* sc = reinterpret_cast<float*>(smem + OFF_SC);
   volatile int* items = reinterpret_cast<volatile int*>(smem + OFF_MISC + 2304);  // [8][4] + seq [8]
+  // PAIR: the second warpgroup's select scratch
+  int* s_hist2 = reinterpret_cast<int*>(smem + OFF_MISC + 2560);          // [256]
+  int* s_sh2 = reinterpret_cast<int*>(smem + OFF_MISC + 3584);            // [4]
+  int* s_wsum2 = reinterpret_cast<int*>(smem + OFF_MISC + 3600);          // [4]
+  unsigned long long* s_best2 = reinterpret_cast<unsigned long long*>(smem + OFF_MISC + 3616);  // [4]
+  int* s_best_slot2 = reinterpret_cast<int*>(smem + OFF_MISC + 3648);     // [4]
 
   const int warp = threadIdx.x / kWarp, lane = threadIdx.x % kWarp;
   const int n_step = st.n, nT = (n_step + kTok - 1) / kTok;
@@ -316,7 +343,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_init(&bar[B_AEMPTY + b], 1);
     }
     mbar_init(&bar[B_OFULL], 1);
-    mbar_init(&bar[B_OEMPTY], 4);
+    mbar_init(&bar[B_OEMPTY], PAIR ? 8 : 4);
     mbar_init(&bar[B_DRAIN], 1);
     mbar_init(&bar[B_DRAIN2], 1);
     *abort = 0;
@@ -359,7 +386,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       // the next item, taken once this CTA's query buffer is free
       int4 iv = make_int4(-1, 0, 0, 0);
       if (lane == 0) {
-        const Item t = last ? Item{-1, 0, 0, 0} : take_item<PERROW>(fs, p, nT);
+        const Item t = last ? Item{-1, 0, 0, 0} : take_item<PERROW, PAIR>(fs, p, nT);
         publish_item(items, gr, t);
         iv = make_int4(t.row, t.t0, t.t1, t.half);
       }
@@ -371,37 +398,44 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (it.row < 0) break;
       last = it.half >= 0;
       const int r = it.row;
-      // query tile: rows [0,G) current, [G,2G) previous step, [2G,3G) departing
-      uint8_t* qt = smem + OFF_Q + qb * 4096;
-      const int qo = ((r / p.kvh) * p.qh + (r % p.kvh) * G) * D;
-      const __nv_bfloat16* prev = p.ring_q + ((size_t)r * p.w + st.slot_prev) * G * D;
-      const __nv_bfloat16* dep = p.ring_q + ((size_t)r * p.w + st.slot) * G * D;
-      // The current query also takes over the departing query's ring slot:
-      // each lane reads the departing element before it writes the same one.
-      __nv_bfloat16* ring_slot = p.ring_q + ((size_t)r * p.w + st.slot) * G * D;
-      for (int e = lane; e < G * (D / 8); e += kWarp) {
-        const int h = e / (D / 8), kc = e % (D / 8);
-        const uint4 cur = reinterpret_cast<const uint4*>(fs.q + qo + h * D)[kc];
-        const uint4 pv = st.has_prev ? reinterpret_cast<const uint4*>(prev + h * D)[kc] : make_uint4(0, 0, 0, 0);
-        const uint4 dv = st.has_dep ? reinterpret_cast<const uint4*>(dep + h * D)[kc] : make_uint4(0, 0, 0, 0);
-        *reinterpret_cast<uint4*>(qt + (kc >> 3) * 2048 + sw128(h, kc & 7)) = cur;
-        *reinterpret_cast<uint4*>(qt + (kc >> 3) * 2048 + sw128(G + h, kc & 7)) = pv;
-        *reinterpret_cast<uint4*>(qt + (kc >> 3) * 2048 + sw128(2 * G + h, kc & 7)) = dv;
-        if (!FULL && it.half < 0) reinterpret_cast<uint4*>(ring_slot + h * D)[kc] = cur;  // halves: see the epilogue
+      // query tile (PAIR: one per row): rows [0,G) current, [G,2G) previous
+      // step, [2G,3G) departing
+      for (int qi = 0; qi < (PAIR ? 2 : 1); ++qi) {
+        const int rq = r + qi;
+        uint8_t* qt = smem + OFF_Q + (PAIR ? 2 * qb + qi : qb) * 4096;
+        const int qo = ((rq / p.kvh) * p.qh + (rq % p.kvh) * G) * D;
+        const __nv_bfloat16* prev = p.ring_q + ((size_t)rq * p.w + st.slot_prev) * G * D;
+        const __nv_bfloat16* dep = p.ring_q + ((size_t)rq * p.w + st.slot) * G * D;
+        // The current query also takes over the departing query's ring slot:
+        // each lane reads the departing element before it writes the same one.
+        __nv_bfloat16* ring_slot = p.ring_q + ((size_t)rq * p.w + st.slot) * G * D;
+        for (int e = lane; e < G * (D / 8); e += kWarp) {
+          const int h = e / (D / 8), kc = e % (D / 8);
+          const uint4 cur = reinterpret_cast<const uint4*>(fs.q + qo + h * D)[kc];
+          const uint4 pv = st.has_prev ? reinterpret_cast<const uint4*>(prev + h * D)[kc] : make_uint4(0, 0, 0, 0);
+          const uint4 dv = st.has_dep ? reinterpret_cast<const uint4*>(dep + h * D)[kc] : make_uint4(0, 0, 0, 0);
+          *reinterpret_cast<uint4*>(qt + (kc >> 3) * 2048 + sw128(h, kc & 7)) = cur;
+          *reinterpret_cast<uint4*>(qt + (kc >> 3) * 2048 + sw128(G + h, kc & 7)) = pv;
+          *reinterpret_cast<uint4*>(qt + (kc >> 3) * 2048 + sw128(2 * G + h, kc & 7)) = dv;
+          if (!FULL && it.half < 0) reinterpret_cast<uint4*>(ring_slot + h * D)[kc] = cur;  // halves: see the epilogue
+        }
       }
       fence_proxy_async();
       __syncwarp();
       if (lane == 0) {
         mbar_arrive(&bar[B_QFULL + qb]);
+        // PAIR: the two rows' tiles alternate (x even: the first row)
+        const int nx = (PAIR ? 2 : 1) * (it.t1 - it.t0);
         for (int pass = 0; pass < 2 && !*abort; ++pass) {
           const CUtensorMap* tm = pass ? &tmV : &tmK;
-          for (int j = it.t0; j < it.t1; ++j, ++g) {
+          for (int x = 0; x < nx; ++x, ++g) {
+            const int j = it.t0 + (PAIR ? x >> 1 : x), rt = r + (PAIR ? x & 1 : 0);
             const int s = g % kStages;
             if (!mbar_wait(&bar[B_EMPTY + s], ((g / kStages) & 1) ^ 1, abort, p.dbg, 2u, (unsigned)g)) break;
             mbar_expect_tx(&bar[B_FULL + s], kTileBytes + ((pass || FULL) ? 0u : GLOB ? 512u : 2560u));
             uint8_t* dst = smem + OFF_STAGE + s * kStageBytes;
             uint8_t* aux = smem + OFF_AUX + s * kAuxBytes;
-            const int y = r * p.stride + j * kTok;
+            const int y = rt * p.stride + j * kTok;
             tma_load_2d(dst, tm, 0, y, &bar[B_FULL + s], pol);
             if (D == 128) tma_load_2d(dst + 16384, tm, 64, y, &bar[B_FULL + s], pol);
             if (!FULL && !pass) {
@@ -432,8 +466,9 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int qb = gr & 1;
         if (!mbar_wait(&bar[B_QFULL + qb], (gr >> 1) & 1, abort, p.dbg, 3u, (unsigned)gr)) break;
         tc_fence_after();
-        const uint32_t qaddr = smem_u32(smem + OFF_Q + qb * 4096);
-        for (int j = it.t0; j < it.t1; ++j, ++g, ++gs) {
+        const int nx = (PAIR ? 2 : 1) * (it.t1 - it.t0);  // PAIR: the rows' tiles alternate
+        for (int x = 0; x < nx; ++x, ++g, ++gs) {
+          const uint32_t qaddr = smem_u32(smem + OFF_Q + (PAIR ? 2 * qb + (x & 1) : qb) * 4096);
           const int s = g % kStages, b = gs & 1;
           if (!mbar_wait(&bar[B_FULL + s], (g / kStages) & 1, abort, p.dbg, 4u, (unsigned)g)) break;
           if (!mbar_wait(&bar[B_SEMPTY + b], ((gs >> 1) & 1) ^ 1, abort, p.dbg, 5u, (unsigned)gs)) break;
@@ -452,25 +487,28 @@ __global__ void __launch_bounds__(kThreads, 1)
         mma_commit(&bar[B_QEMPTY + qb]);
         // V pass: PV MMAs in tile order; a V stage is released as soon as its
         // tile's weights are in (the policy-layer MMAs run on warp 10)
-        for (int j = it.t0; j < it.t1; ++j, ++g, ++gv) {
+        for (int x = 0; x < nx; ++x, ++g, ++gv) {
           const int s = g % kStages, pb = gv & 1;
+          // the first tile of each row starts its accumulator
+          const bool first = PAIR ? x < 2 : x == 0;
+          const uint32_t ocol = kColO + (PAIR && (x & 1) ? (uint32_t)(kColOB - kColO) : 0u);
           if (!mbar_wait(&bar[B_FULL + s], (g / kStages) & 1, abort, p.dbg, 13u, (unsigned)g)) break;
           // only these MMAs read a V stage: the four epilogue arrivals of the
           // stage's release are made here (its last one is the commit below)
           mbar_arrive_cnt(&bar[B_EMPTY + s], 4);
           if (!mbar_wait(&bar[B_PFULL + pb], (gv >> 1) & 1, abort, p.dbg, 14u, (unsigned)gv)) break;
-          if (j == it.t0 && !mbar_wait(&bar[B_OEMPTY], (gr & 1) ^ 1, abort, p.dbg, 15u, (unsigned)gr)) break;
+          if (x == 0 && !mbar_wait(&bar[B_OEMPTY], (gr & 1) ^ 1, abort, p.dbg, 15u, (unsigned)gr)) break;
           tc_fence_after();
           const uint32_t vaddr = smem_u32(smem + OFF_STAGE + s * kStageBytes);
           const uint32_t paddr = smem_u32(smem + OFF_P + pb * 4096);
           // O^T[d x 16] += V^T[d x 128] P^T: V^T is MN-major (dims contiguous)
 #pragma unroll
           for (int ks = 0; ks < kTok / 16; ++ks)
-            mma_bf16(tmem + kColO, sdesc_sw128(vaddr + ks * 2048u, 16384, 1024),
-                     sdesc_sw32(paddr + ks * 512u, 4096, 256), id_pv, (j > it.t0 || ks > 0) ? 1u : 0u);
+            mma_bf16(tmem + ocol, sdesc_sw128(vaddr + ks * 2048u, 16384, 1024),
+                     sdesc_sw32(paddr + ks * 512u, 4096, 256), id_pv, (!first || ks > 0) ? 1u : 0u);
           mma_commit(&bar[B_PEMPTY + pb]);
           mma_commit(&bar[B_EMPTY + s]);
-          if (j == it.t1 - 1) mma_commit(&bar[B_OFULL]);
+          if (x == nx - 1) mma_commit(&bar[B_OFULL]);
         }
       }
       // all issued MMAs complete before TMEM is released
@@ -487,7 +525,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       for (int gr = 0;; ++gr) {
         const Item it = read_item(items, gr, abort, p.dbg, 24u);
         if (it.row < 0) break;
-        for (int j = it.t0; j < it.t1; ++j, ++gv) {
+        const int nx = (PAIR ? 2 : 1) * (it.t1 - it.t0);
+        for (int x = 0; x < nx; ++x, ++gv) {
           const int pb = gv & 1;
           if (!mbar_wait(&bar[B_AFULL + pb], (gv >> 1) & 1, abort, p.dbg, 16u, (unsigned)gv)) break;
           if (!mbar_wait(&bar[B_MEMPTY + pb], ((gv >> 1) & 1) ^ 1, abort, p.dbg, 17u, (unsigned)gv)) break;
@@ -515,8 +554,26 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int etid = ew * 32 + lane;            // 0..255
     const uint32_t lane_addr = tmem + ((uint32_t)(quad * 32) << 16);
     const float c = p.c;
-    auto sync = [] { named_bar(1, kEpi); };
-    const SelectScratch scr{s_hist, s_sh, s_wsum, s_best, s_best_slot};
+    // the team that works on one row: both warpgroups, or (PAIR) one each
+    constexpr int kTeam = PAIR ? kEpi / 2 : kEpi;
+    const int tid = PAIR ? etid % kTeam : etid;    // thread within the team
+    const int w0 = PAIR ? wg * (kTeam / kWarp) : 0;  // the team's first epilogue warp
+    auto sync = [wg] {
+      if constexpr (PAIR) named_bar(2 + wg, kTeam);
+      else named_bar(1, kEpi);
+    };
+    const SelectScratch scr = (PAIR && wg == 1) ? SelectScratch{s_hist2, s_sh2, s_wsum2, s_best2, s_best_slot2}
+                                                : SelectScratch{s_hist, s_sh, s_wsum, s_best, s_best_slot};
+    // PAIR: this team's logits of head G-1, then scores
+    float* const scw = sc + (PAIR ? wg * kPairTok : 0);
+    // TMEM column of the stashed logits of this team's tile j
+    auto stash_at = [wg](int j) -> uint32_t {
+      if constexpr (PAIR) return (uint32_t)((wg ? kStashB : kPairStashA) + GS * j);
+      else return stash_col<GS>(j);
+    };
+    // position of this team's tile j in the item's tile sequence
+    auto tpos = [wg](int j, int t0) { return PAIR ? 2 * j + wg : j - t0; };
+    constexpr int JS = PAIR ? 1 : 2;  // step between a team's tiles
     int g = 0, gs = 0, gv = 0;
     for (int gr = 0;; ++gr) {
       int4 iv = make_int4(-1, 0, 0, 0);
@@ -530,7 +587,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       iv.w = __shfl_sync(0xffffffffu, iv.w, 0);
       if (named_bar_or(1, kEpi, *abort != 0 || iv.x < 0)) break;
       const Item it{iv.x, iv.y, iv.z, iv.w};
-      const int r = it.row, t0 = it.t0, t1 = it.t1, nTi = it.t1 - it.t0;
+      const int r = it.row + (PAIR ? wg : 0), t0 = it.t0, t1 = it.t1, nTi = it.t1 - it.t0;
+      const int nItem = (PAIR ? 2 : 1) * nTi;  // tiles of the item
       // this row's length (after the append) and budget
       const int n = PERROW ? p.rowlen[r] : n_step;
       const int Bsel = PERROW ? (fs.B > 0 ? fs.B : p.rowbudget[r]) : fs.B;
@@ -552,8 +610,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       for (int h = 0; h < G; ++h) { m[h] = kNoMax; l[h] = 0.f; u[h] = 0.f; }
 
       // ---------------- K pass: this warpgroup's tiles (global index parity)
-      for (int j = t0 + ((wg - gs) & 1); j < t1; j += 2) {
-        const int gj = g + (j - t0), gsj = gs + (j - t0);
+      for (int j = PAIR ? t0 : t0 + ((wg - gs) & 1); j < t1; j += JS) {
+        const int gj = g + tpos(j, t0), gsj = gs + tpos(j, t0);
         const int s = gj % kStages, b = gsj & 1;
         mbar_wait(&bar[B_SFULL + b], (gsj >> 1) & 1, abort, p.dbg, 6u, (unsigned)gsj);
         mbar_wait(&bar[B_FULL + s], (gj / kStages) & 1, abort, p.dbg, 12u, (unsigned)gj);
@@ -588,20 +646,20 @@ __global__ void __launch_bounds__(kThreads, 1)
           }
         }
         if (!LONG || j < onchip_tiles<GS>()) {
-          sc[i] = S16[G - 1];
+          scw[i] = S16[G - 1];
           __syncwarp();
-          stash_store<GS>(lane_addr + stash_col<GS>(j), S16);
+          stash_store<GS>(lane_addr + stash_at(j), S16);
         } else {
           store_logits<G>(p.logit + (rbase + i) * G, S16);
         }
       }
-      g += nTi;
-      gs += nTi;
+      g += nItem;
+      gs += nItem;
       // per-token state of this warpgroup's V-pass tiles (the same tiles as its
       // K pass), loaded two own tiles ahead: window sums (this thread wrote
       // them in the K pass), positions, |v|; the first two issued here, so that
       // their latency overlaps the statistics merge
-      const int j0 = t0 + ((wg - gv) & 1);
+      const int j0 = PAIR ? t0 : t0 + ((wg - gv) & 1);
       const float4* szrow = p.SZ + rbase + tok;
       const int* posrow = p.pos + rbase + tok;
       const float* vnrow = p.vnorm + rbase + tok;
@@ -611,13 +669,13 @@ __global__ void __launch_bounds__(kThreads, 1)
       float vnA = 0.f, vnB = 0.f;
       if constexpr (!FULL && !GLOB) {
         szA = j0 < t1 ? szrow[j0 * kTok] : kZero4;
-        szB = j0 + 2 < t1 ? szrow[(j0 + 2) * kTok] : kZero4;
+        szB = j0 + JS < t1 ? szrow[(j0 + JS) * kTok] : kZero4;
         posA = j0 < t1 ? posrow[j0 * kTok] : 0;
-        posB = j0 + 2 < t1 ? posrow[(j0 + 2) * kTok] : 0;
+        posB = j0 + JS < t1 ? posrow[(j0 + JS) * kTok] : 0;
       }
       if constexpr (!FULL) {
         vnA = j0 < t1 ? vnrow[j0 * kTok] : 0.f;
-        vnB = j0 + 2 < t1 ? vnrow[(j0 + 2) * kTok] : 0.f;
+        vnB = j0 + JS < t1 ? vnrow[(j0 + JS) * kTok] : 0.f;
       }
       if constexpr (GS > 0) tmem_st_wait();
       // ---------------- row softmax statistics (deterministic merge order):
@@ -646,10 +704,10 @@ __global__ void __launch_bounds__(kThreads, 1)
       for (int h = 0; h < G; ++h) {
         float mm = kNoMax;
 #pragma unroll
-        for (int w = 0; w < 8; ++w) mm = fmaxf(mm, red[(w * G + h) * 3 + 0]);
+        for (int w = w0; w < w0 + kTeam / kWarp; ++w) mm = fmaxf(mm, red[(w * G + h) * 3 + 0]);
         float ll = 0.f, uu = 0.f;
 #pragma unroll
-        for (int w = 0; w < 8; ++w) {
+        for (int w = w0; w < w0 + kTeam / kWarp; ++w) {
           const float lw = red[(w * G + h) * 3 + 1];
           const float dm = (red[(w * G + h) * 3 + 0] - mm) * c, f = ex2(dm);
           ll = fmaf(lw, f, ll);
@@ -704,15 +762,15 @@ __global__ void __launch_bounds__(kThreads, 1)
         M[h] = Mm[h];
         NL[h] = -log2f(Ll[h]);
         Hh[h] = logf(Ll[h]) - 0.69314718055994531f * (Uu[h] / Ll[h]);
-        if (etid == h) L0 = Ll[h];
+        if (tid == h) L0 = Ll[h];
       }
       // push (m, l, H, -log2 l) of this step into the ring slot it takes over
       // (the producer, or half 0 above, wrote the query there)
-      if (!FULL && etid < G && half <= 0) {
+      if (!FULL && tid < G && half <= 0) {
         float4 v;
-        v.x = M[etid]; v.y = L0; v.z = Hh[etid]; v.w = NL[etid];
-        reinterpret_cast<float4*>(p.ring_stats)[((size_t)r * p.w + st.slot) * G + etid] = v;
-        p.hq[(size_t)r * G + etid] = Hh[etid];
+        v.x = M[tid]; v.y = L0; v.z = Hh[tid]; v.w = NL[tid];
+        reinterpret_cast<float4*>(p.ring_stats)[((size_t)r * p.w + st.slot) * G + tid] = v;
+        p.hq[(size_t)r * G + tid] = Hh[tid];
       }
 
       // One eviction (the steady state): slot B, the only mover, is loaded now
@@ -721,33 +779,33 @@ __global__ void __launch_bounds__(kThreads, 1)
       // at the select.
       const bool single_evict = fs.do_evict && n == Bsel + 1;
       SlotCopy mv{};
-      if (single_evict && half != 0 && etid < kWarp) slot_load_settled(p, rbase + Bsel, etid, fs.write_scores, mv);
+      if (single_evict && half != 0 && tid < kWarp) slot_load_settled(p, rbase + Bsel, tid, fs.write_scores, mv);
 
       // ---------------- V pass: this warpgroup's tiles; prep of the next one
       // overlaps the MMAs of the current one
       const float pos_den = (float)max(st.p_newest, 1);
       auto prep = [&](int j) {
-        const int gvj = gv + (j - t0), pb = gvj & 1;
+        const int gvj = gv + tpos(j, t0), pb = gvj & 1;
         const float4 sz = szA;
         const int pos = posA;
         const float vn = vnA;
         szA = szB;
         posA = posB;
         vnA = vnB;
-        if (!FULL && j + 4 < t1) {
+        if (!FULL && j + 2 * JS < t1) {
           if constexpr (!GLOB) {
-            szB = szrow[(j + 4) * kTok];
-            posB = posrow[(j + 4) * kTok];
+            szB = szrow[(j + 2 * JS) * kTok];
+            posB = posrow[(j + 2 * JS) * kTok];
           }
-          vnB = vnrow[(j + 4) * kTok];
+          vnB = vnrow[(j + 2 * JS) * kTok];
         }
         const int i = j * kTok + tok;
         const bool valid = i < n;
         float sv[G];
         if (!LONG || j < onchip_tiles<GS>()) {
-          stash_load<GS>(lane_addr + stash_col<GS>(j), sv);
+          stash_load<GS>(lane_addr + stash_at(j), sv);
           if constexpr (GS > 0) tmem_ld_wait();
-          sv[G - 1] = sc[i];
+          sv[G - 1] = scw[i];
         } else {
           load_logits<G>(p.logit + (rbase + i) * G, sv);
         }
@@ -860,7 +918,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       uint32_t ev_key = 0xFFFFFFFFu;
       int ev_slot = -1, ev_pos = -1;
       auto finish = [&](int j, float lin, int pos) {
-        const int gvj = gv + (j - t0), pb = gvj & 1;
+        const int gvj = gv + tpos(j, t0), pb = gvj & 1;
         mbar_wait(&bar[B_MFULL + pb], (gvj >> 1) & 1, abort, p.dbg, 10u, (unsigned)gvj);
         __syncwarp();
         tc_fence_after();
@@ -887,9 +945,9 @@ __global__ void __launch_bounds__(kThreads, 1)
           const float score = fp.b2 + relu_sum;
           if constexpr (LONG) {
             if (spill_scores || fs.write_scores) p.score[rbase + i] = score;
-            if (n <= kFusedMaxTok) sc[i] = score;
+            if (n <= kFusedMaxTok) scw[i] = score;
           } else {
-            sc[i] = score;
+            scw[i] = score;
             if (fs.write_scores) p.score[rbase + i] = score;
           }
           // this thread's lowest-ranked token so far (lower key, then the later position)
@@ -906,7 +964,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int i = j * kTok + tok;
         if (i < n) {
           if (spill_scores || fs.write_scores) p.score[rbase + i] = score;
-          if (n <= kFusedMaxTok) sc[i] = score;
+          if (n <= kFusedMaxTok) scw[i] = score;
           const uint32_t kk = score_key(score);
           if (ev_slot < 0 || kk < ev_key || (kk == ev_key && pos > ev_pos)) {
             ev_key = kk;
@@ -918,23 +976,23 @@ __global__ void __launch_bounds__(kThreads, 1)
       // prep(j) returns (the linear score part, or a heuristic score; the
       // position) for finish(j)
       float2 pf_cur = j0 < t1 ? prep(j0) : make_float2(0.f, 0.f);
-      for (int j = j0; j < t1; j += 2) {
-        const float2 pf_next = j + 2 < t1 ? prep(j + 2) : make_float2(0.f, 0.f);
+      for (int j = j0; j < t1; j += JS) {
+        const float2 pf_next = j + JS < t1 ? prep(j + JS) : make_float2(0.f, 0.f);
         if constexpr (HEUR) record_h(j, pf_cur.x, __float_as_int(pf_cur.y));
         else if constexpr (!FULL && !GLOB) finish(j, pf_cur.x, __float_as_int(pf_cur.y));
         pf_cur = pf_next;
       }
-      g += nTi;
-      gv += nTi;
+      g += nItem;
+      gv += nItem;
       // ---------------- attention output (warpgroup 0); a half row's two
       // partial sums (weights already normalised by the whole row) add up
       float ov[G];
-      if (wg == 0) {
+      if (PAIR || wg == 0) {
         mbar_wait(&bar[B_OFULL], gr & 1, abort, p.dbg, 11u, (unsigned)gr);
         __syncwarp();
         tc_fence_after();
         float o16[16];
-        tmem_ld16(lane_addr + kColO, o16);
+        tmem_ld16(lane_addr + (PAIR && wg ? kColOB : kColO), o16);
         tmem_ld_wait();
         tc_fence_before();
         __syncwarp();
@@ -955,7 +1013,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         sync();
       }
-      if (wg == 0 && half <= 0 && tok < D) {
+      if ((PAIR || wg == 0) && half <= 0 && tok < D) {
         float* op = fs.out + ((r / p.kvh) * p.qh + (r % p.kvh) * G) * D;
 #pragma unroll
         for (int h = 0; h < G; ++h)
@@ -968,7 +1026,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         // or by half 1) is the only mover and fills the evicted slot. Half
         // rows swap their candidates first.
         const bool mover = half != 0;
-        if (mover && etid < kWarp) slot_load_late(p, rbase + Bsel, etid, fs.write_scores, mv);
+        if (mover && tid < kWarp) slot_load_late(p, rbase + Bsel, tid, fs.write_scores, mv);
         auto lower = [](uint32_t ka, int sa, int pa, uint32_t kb, int sb, int pb) {  // (kb, sb) ranks lower?
           if (sb < 0) return false;
           if (sa < 0) return true;
@@ -984,14 +1042,15 @@ __global__ void __launch_bounds__(kThreads, 1)
           if (lower(bk, bs, bp, ok, os, op)) { bk = ok; bs = os; bp = op; }
         }
         sync();
-        if (lane == 0) { s_best[ew] = bk; s_best_slot[ew] = bs; s_hist[ew] = bp; }
+        const int tw = tid / kWarp;  // warp within the team
+        if (lane == 0) { scr.best[tw] = bk; scr.best_slot[tw] = bs; scr.hist[tw] = bp; }
         sync();
-        if (etid == 0) {
-          uint32_t fk = (uint32_t)s_best[0];
-          int fe = s_best_slot[0], fpos = s_hist[0];
-          for (int w = 1; w < kEpi / kWarp; ++w)
-            if (lower(fk, fe, fpos, (uint32_t)s_best[w], s_best_slot[w], s_hist[w])) {
-              fk = (uint32_t)s_best[w]; fe = s_best_slot[w]; fpos = s_hist[w];
+        if (tid == 0) {
+          uint32_t fk = (uint32_t)scr.best[0];
+          int fe = scr.best_slot[0], fpos = scr.hist[0];
+          for (int w = 1; w < kTeam / kWarp; ++w)
+            if (lower(fk, fe, fpos, (uint32_t)scr.best[w], scr.best_slot[w], scr.hist[w])) {
+              fk = (uint32_t)scr.best[w]; fe = scr.best_slot[w]; fpos = scr.hist[w];
             }
           if (half >= 0) {
             int* xs = fs.xsel + (2 * ts + half) * 4;
@@ -1008,19 +1067,19 @@ __global__ void __launch_bounds__(kThreads, 1)
               fe = -1;
             }
           }
-          s_sh[0] = fe;
+          scr.sh[0] = fe;
         }
         sync();
-        const int e = s_sh[0];
-        if (mover && e >= 0 && e < Bsel && etid < kWarp) slot_store(p, rbase + e, etid, mv);
+        const int e = scr.sh[0];
+        if (mover && e >= 0 && e < Bsel && tid < kWarp) slot_store(p, rbase + e, tid, mv);
         sync();
       } else if (fs.do_evict && Bsel < n) {
         // several evictions (whole rows only): radix select over the scores
         sync();
-        team_select_compact<kEpi>(p, r, n, Bsel, LONG && n > kFusedMaxTok ? p.score + rbase : sc, etid, scr,
-                                  sync);
+        team_select_compact<kTeam>(p, r, n, Bsel, LONG && n > kFusedMaxTok ? p.score + rbase : scw, tid, scr,
+                                   sync);
       }
-      if (PERROW && fs.do_evict && etid == 0) p.rowlen[r] = n < Bsel ? n : Bsel;
+      if (PERROW && fs.do_evict && tid == 0) p.rowlen[r] = n < Bsel ? n : Bsel;
     }
   }
   __syncthreads();
@@ -1032,17 +1091,21 @@ __global__ void __launch_bounds__(kThreads, 1)
 }
 
 
-template <int D, int G, bool LONG, bool FULL = false, bool HEUR = false, bool GLOB = false, bool PERROW = false>
+template <int D, int G, bool LONG, bool FULL = false, bool HEUR = false, bool GLOB = false, bool PERROW = false,
+          bool PAIR = false>
 static cudaError_t launch_t(const FusedMaps& maps, const Dev& p, const Step& st, const FusedStep& fs,
                             const FusedPolicy& fp, int grid, cudaStream_t s) {
+  constexpr int kSmemBytes = Smem<PAIR>::BYTES;
   static bool attr = false;
   if (!attr) {
-    cudaError_t e = cudaFuncSetAttribute(fused_kernel<D, G, LONG, FULL, HEUR, GLOB, PERROW>, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes);
+    cudaError_t e = cudaFuncSetAttribute(fused_kernel<D, G, LONG, FULL, HEUR, GLOB, PERROW, PAIR>,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes);
     if (e != cudaSuccess) return e;
     attr = true;
   }
   if (fs.half_rows == 0) {
-    fused_kernel<D, G, LONG, FULL, HEUR, GLOB, PERROW><<<grid, kThreads, kSmemBytes, s>>>(maps.k, maps.v, p, st, fs, fp);
+    fused_kernel<D, G, LONG, FULL, HEUR, GLOB, PERROW, PAIR>
+        <<<grid, kThreads, kSmemBytes, s>>>(maps.k, maps.v, p, st, fs, fp);
     return cudaGetLastError();
   }
   // the two CTAs of a half row wait on each other: a cooperative launch
@@ -1057,7 +1120,8 @@ static cudaError_t launch_t(const FusedMaps& maps, const Dev& p, const Step& st,
   la[0].val.cooperative = 1;
   cfg.attrs = la;
   cfg.numAttrs = 1;
-  return cudaLaunchKernelEx(&cfg, fused_kernel<D, G, LONG, FULL, HEUR, GLOB, PERROW>, maps.k, maps.v, p, st, fs, fp);
+  return cudaLaunchKernelEx(&cfg, fused_kernel<D, G, LONG, FULL, HEUR, GLOB, PERROW, PAIR>, maps.k, maps.v, p, st, fs,
+                            fp);
 }
 
 inline int fused_grid(const Dev& p, int num_sms) { return p.R < num_sms ? p.R : num_sms; }

@@ -283,7 +283,7 @@ class DistillCache:
     def engine(self, n: int = 0) -> str:
         e = C.c_int()
         self._check(lib().dc_engine(self._h, n, C.byref(e)))
-        return {1: "split", 2: "fused"}[e.value]
+        return {1: "split", 2: "fused", 3: "fused-pairs"}[e.value]
 
     def evict(self, budget: int = 0) -> None:
         self._check(lib().dc_evict(self._h, budget))

@@ -142,8 +142,9 @@ def _tail_workload(**kw):
 
 def test_tail_split_rows_match_oracle():
     """Half rows (two CTAs per row, statistics and output exchanged) against
-    the oracle, across the window's departures."""
-    wl, sms = _tail_workload(prompt_len=1500, budget=600, steps=70)
+    the oracle, across the window's departures. Rows of 3001 tokens (24
+    tiles): longer than row pairs take."""
+    wl, sms = _tail_workload(prompt_len=4000, budget=3000, steps=70)
     ls = LockStep(wl, [0, sms - 1, sms, sms + 3, wl.rows - 1], engine=2)
     ls.load_prompt()
     for s in range(wl.steps):
@@ -156,7 +157,7 @@ def test_tail_split_step_equals_decode_then_evict():
     dc_evict; the output agrees with whole-row CTAs to rounding."""
     import torch
     from paper_2608_08878_gb300 import dc
-    wl, _ = _tail_workload(prompt_len=900, budget=400, window=6)
+    wl, _ = _tail_workload(prompt_len=3500, budget=2800, window=6)  # 22 tiles: no row pairs
     a, b = LockStep(wl, [], engine=2), LockStep(wl, [], engine=2)
     c = LockStep(wl, [], engine=2, tail_split=False)
     for x in (a, b, c):
@@ -178,6 +179,55 @@ def test_tail_split_step_equals_decode_then_evict():
         if s == 0:  # before the two caches' evictions could part on near-ties
             err = float((oa - oc).abs().max())
             assert err <= 1e-4, err
+
+
+@pytest.mark.parametrize("group,head_dim,steps", [(4, 128, 70), (2, 128, 12), (1, 64, 12)])
+def test_row_pairs_match_oracle(group, head_dim, steps):
+    """Row pairs (more rows than SMs, rows of at most 21 tiles: each
+    warpgroup of a CTA does one row of the pair, their tiles alternating in
+    the stage ring) against the oracle: both rows of the first and last
+    pairs and of pairs on either side of the first wave, prompt compression
+    (many evictions, one radix select per warpgroup) and steady steps across
+    the window's departures."""
+    import torch
+    sms = torch.cuda.get_device_properties(0).multi_processor_count
+    # four rows per SM: two pairs per CTA
+    wl = synth.MISTRAL_1L.with_(batch=sms // 2, prompt_len=1500, budget=600, steps=steps, q_heads=8 * group,
+                                head_dim=head_dim)
+    assert wl.rows == 4 * sms
+    ls = LockStep(wl, [0, 1, 2 * sms - 2, 2 * sms - 1, wl.rows - 2, wl.rows - 1], engine=2)
+    assert ls.cache.engine(wl.prompt_len + 1) == "fused-pairs" and ls.cache.engine(wl.budget + 1) == "fused-pairs"
+    ls.load_prompt()
+    for s in range(wl.steps):
+        ls.step(check=(s < 3 or s % 16 == 0 or s >= wl.steps - 4))
+    assert ls.cache.length()[0] == wl.budget
+
+
+def test_row_pairs_step_equals_decode_then_evict():
+    """On row pairs, dc_step's in-kernel eviction (a radix select per
+    warpgroup on the prompt compression, then one eviction per step) leaves
+    the cache bit-identical to dc_decode_step and dc_evict, with the same
+    output."""
+    import torch
+    from paper_2608_08878_gb300 import dc
+    sms = torch.cuda.get_device_properties(0).multi_processor_count
+    wl = synth.MISTRAL_1L.with_(batch=sms // 2, prompt_len=2000, budget=500, window=6)
+    a, b = LockStep(wl, [], engine=2), LockStep(wl, [], engine=2)
+    assert a.cache.engine(wl.prompt_len + 1) == "fused-pairs" and a.cache.engine(wl.budget + 1) == "fused-pairs"
+    for x in (a, b):
+        x.load_prompt()
+    for s in range(10):
+        q, kn, vn = a._inputs(s)
+        oa = a.cache.step(q, kn, vn)
+        ob = b.cache.decode_step(q, kn, vn)
+        b.cache.evict()
+        a.cache.sync()
+        b.cache.sync()
+        assert torch.equal(oa, ob), s
+        assert a.cache.length() == b.cache.length()
+        n = a.cache.length()[0]
+        for which in (dc.BUF_K, dc.BUF_V, dc.BUF_POS, dc.BUF_S, dc.BUF_Z, dc.BUF_VNORM):
+            assert torch.equal(a.cache.buffer(which)[:, :n], b.cache.buffer(which)[:, :n]), (s, which)
 
 
 @pytest.mark.parametrize("prompt_len,budget", [(12000, 10000), (16000, 12000)])
@@ -291,7 +341,9 @@ def test_per_row_budgets_head_level_hybrid(engine):
 def test_engine_choice():
     from paper_2608_08878_gb300 import dc
     big = dc.DistillCache(32, 8, 128, 200, 100, batch=1)
-    assert big.engine() == "fused" and big.engine(20000) == "fused"
+    # 256 rows on the GPU's SMs: short rows go in pairs, long ones one per CTA
+    assert big.engine() == "fused-pairs" and big.engine(400) == "fused-pairs"
+    assert big.engine(3000) == "fused" and big.engine(20000) == "fused"
     small = dc.DistillCache(1, 2, 64, 200, 100, q_heads=4)
     assert small.engine() == "split"
     forced = dc.DistillCache(1, 2, 64, 200, 100, q_heads=4, engine=2)
