@@ -59,7 +59,8 @@ typedef struct {
   int alpha_mode;     /* 0: alpha_i from the most recent pass (Sec. 3.1.1, default);
                          1: cumulative since insertion */
   int engine;         /* 0: auto (default): the fused kernel whenever the step
-                            fits it and the rows fill the GPU, else split;
+                            fits it, unless a few long rows run faster on the
+                            split engine (a latency model of the two);
                          1: split (separate attention, feature and scoring kernels);
                          2: fused whenever the step fits it (one CTA per row
                             streams K/V once and does the whole step) */

@@ -344,8 +344,9 @@ def test_engine_choice():
     # 256 rows on the GPU's SMs: short rows go in pairs, long ones one per CTA
     assert big.engine() == "fused-pairs" and big.engine(400) == "fused-pairs"
     assert big.engine(3000) == "fused" and big.engine(20000) == "fused"
-    small = dc.DistillCache(1, 2, 64, 200, 100, q_heads=4)
-    assert small.engine() == "split"
+    # two rows: short ones on the fused kernel, long ones spread by the split engine
+    small = dc.DistillCache(1, 2, 64, 30000, 100, q_heads=4)
+    assert small.engine() == "fused" and small.engine(20000) == "split"
     forced = dc.DistillCache(1, 2, 64, 200, 100, q_heads=4, engine=2)
     assert forced.engine() == "fused"
     assert dc.DistillCache(1, 2, 64, 200, 100, q_heads=16, engine=2).engine() == "split"  # group 8
@@ -427,8 +428,9 @@ def test_full_stack_sampled_rows(engine):
 def test_sweep_points_sampled_rows(batch, ctx, ratio):
     """Points of the throughput sweep (32 layers, Mistral-7B KV heads) at full
     size in the engine auto-selection the sweep uses: prompt compression and
-    steady steps, 3 sampled rows. The last point's budget (16384) is past the
-    fused kernel's row limit, so it runs on the split engine."""
+    steady steps, 3 sampled rows. The first two points run on row pairs; the
+    last point's budget (16384) is past the on-chip logit capacity, so its
+    logits and scores go through HBM."""
     wl = synth.sweep_point(batch, ctx, ratio)
     ls = LockStep(wl, [0, wl.rows // 2 + 3, wl.rows - 1], engine=0, device_inputs=True)
     ls.load_prompt()
