@@ -181,8 +181,8 @@ def test_tail_split_step_equals_decode_then_evict():
             assert err <= 1e-4, err
 
 
-@pytest.mark.parametrize("group,head_dim,steps", [(4, 128, 70), (2, 128, 12), (1, 64, 12)])
-def test_row_pairs_match_oracle(group, head_dim, steps):
+@pytest.mark.parametrize("group,head_dim,steps,alpha_mode", [(4, 128, 70, 0), (2, 128, 12, 1), (1, 64, 12, 0)])
+def test_row_pairs_match_oracle(group, head_dim, steps, alpha_mode):
     """Row pairs (more rows than SMs, rows of at most 21 tiles: each
     warpgroup of a CTA does one row of the pair, their tiles alternating in
     the stage ring) against the oracle: both rows of the first and last
@@ -193,7 +193,7 @@ def test_row_pairs_match_oracle(group, head_dim, steps):
     sms = torch.cuda.get_device_properties(0).multi_processor_count
     # four rows per SM: two pairs per CTA
     wl = synth.MISTRAL_1L.with_(batch=sms // 2, prompt_len=1500, budget=600, steps=steps, q_heads=8 * group,
-                                head_dim=head_dim)
+                                head_dim=head_dim, alpha_mode=alpha_mode)
     assert wl.rows == 4 * sms
     ls = LockStep(wl, [0, 1, 2 * sms - 2, 2 * sms - 1, wl.rows - 2, wl.rows - 1], engine=2)
     assert ls.cache.engine(wl.prompt_len + 1) == "fused-pairs" and ls.cache.engine(wl.budget + 1) == "fused-pairs"
