@@ -412,7 +412,9 @@ dc_status dc_cache_create(int layers, int kv_heads, int head_dim, int capacity, 
     if (fe == cudaSuccess) fe = dalloc(h, &h->work, 2 * sizeof(unsigned));
     if (fe == cudaSuccess) fe = cudaMemsetAsync(h->work, 0, 2 * sizeof(unsigned), h->stream);
     if (fe == cudaSuccess && cfg.tail_split) {
-      const int grid = (int)std::min<long long>(R, h->num_sms);
+      // exchange slots: the last wave's half rows, or every row when rows are
+      // at most half the SMs (fused_*_len(x) has x / 2 + 1 slots)
+      const int grid = 2 * (int)std::min<long long>(R, h->num_sms);
       fe = dalloc(h, &h->xstats, dc::fused_xstats_len(grid, G) * sizeof(float));
       if (fe == cudaSuccess) fe = dalloc(h, &h->xo, dc::fused_xo_len(grid, G, head_dim) * sizeof(float));
       if (fe == cudaSuccess) fe = dalloc(h, &h->xsel, dc::fused_xsel_len(grid) * sizeof(int));

@@ -35,11 +35,16 @@ bool fused_pairs(const Dev& p, int n, int num_sms) {
 
 int fused_half_rows(const Dev& p, int n, const FusedStep& fs, int num_sms) {
   if (fused_pairs(p, n, num_sms)) return 0;
-  const int grid = fused_grid(p, num_sms), rem = p.R % grid;
+  const int grid = p.R < num_sms ? p.R : num_sms, rem = p.R % grid;
   const int nT = (n + kTok - 1) / kTok;
-  const bool ok = fs.xflag && fs.xstats && fs.xo && fs.xsel && rem > 0 && 2 * rem <= grid && nT >= 2 &&
-                  (!fs.do_evict || fs.B >= n || fs.B == n - 1);
-  return ok ? rem : 0;
+  const bool ok = fs.xflag && fs.xstats && fs.xo && fs.xsel && nT >= 2 && (!fs.do_evict || fs.B >= n || fs.B == n - 1);
+  if (!ok) return 0;
+  // at most half as many rows as SMs: every row of 12 tiles or more over two
+  // CTAs (shorter halves cost more in exchanges than they save: 129-token
+  // rows measured 25 us per step whole, 30 us halved; 2049-token rows 44 and
+  // 41 us, 4097-token rows 64 and 51 us)
+  if (2 * p.R <= num_sms) return nT >= 12 ? p.R : 0;
+  return rem > 0 && 2 * rem <= grid ? rem : 0;
 }
 
 cudaError_t launch_fused_step(const FusedMaps& maps, const Dev& p, const Step& st, const FusedStep& fs,
@@ -48,7 +53,7 @@ cudaError_t launch_fused_step(const FusedMaps& maps, const Dev& p, const Step& s
   if (p.seq_rows) return launch_fused_glob(maps, p, st, fs, fp, num_sms, s);
   if (p.rowlen || p.scorer != 0) return launch_fused_heur_perrow(maps, p, st, fs, fp, num_sms, s);
   if (fs.half_rows == 0 && fused_pairs(p, st.n, num_sms)) return launch_fused_pair(maps, p, st, fs, fp, num_sms, s);
-  const int grid = fused_grid(p, num_sms);
+  const int grid = fused_grid(p, fs, num_sms);
   const bool lg = st.n > fused_onchip_tokens(p.G);
 #define DC_FUSED_LAUNCH(D, G) \
   return lg ? launch_t<D, G, true>(maps, p, st, fs, fp, grid, s) : launch_t<D, G, false>(maps, p, st, fs, fp, grid, s)

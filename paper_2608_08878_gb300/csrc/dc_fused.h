@@ -83,9 +83,10 @@ void prepare_policy(const float* blob, int H, int layernorm, FusedPolicy* fp, st
 // selection).
 bool fused_pairs(const Dev& p, int n, int num_sms);
 
-// How many rows a step over n tokens splits into halves (see FusedStep): the
-// remainder of R over the grid when it is at most half the grid, else 0 (and
-// 0 on row pairs).
+// How many rows a step over n tokens splits into halves (see FusedStep): every
+// row when rows are at most half the SMs and at least 12 tiles long, else the
+// remainder of R over the grid when it is at most half the grid, else 0 (and 0
+// on row pairs).
 int fused_half_rows(const Dev& p, int n, const FusedStep& fs, int num_sms);
 
 cudaError_t launch_fused_step(const FusedMaps& maps, const Dev& p, const Step& st, const FusedStep& fs,

@@ -7,7 +7,7 @@ namespace dc {
 
 cudaError_t launch_fused_glob(const FusedMaps& maps, const Dev& p, const Step& st, const FusedStep& fs,
                               const FusedPolicy& fp, int num_sms, cudaStream_t s) {
-  const int grid = fused_grid(p, num_sms);
+  const int grid = fused_grid(p, fs, num_sms);
   if (p.d == 128) {
     if (p.G == 4) return launch_t<128, 4, true, false, false, true>(maps, p, st, fs, fp, grid, s);
     if (p.G == 2) return launch_t<128, 2, true, false, false, true>(maps, p, st, fs, fp, grid, s);
@@ -20,7 +20,7 @@ cudaError_t launch_fused_glob(const FusedMaps& maps, const Dev& p, const Step& s
 
 cudaError_t launch_fused_full(const FusedMaps& maps, const Dev& p, int n, const FusedStep& fs,
                               const FusedPolicy& fp, int num_sms, cudaStream_t s) {
-  const int grid = fused_grid(p, num_sms);
+  const int grid = fused_grid(p, fs, num_sms);
   Step st{};
   st.n = n;  // no previous or departing query terms: has_prev = has_dep = 0
   if (p.d == 128) {

@@ -1124,7 +1124,12 @@ static cudaError_t launch_t(const FusedMaps& maps, const Dev& p, const Step& st,
                             fp);
 }
 
-inline int fused_grid(const Dev& p, int num_sms) { return p.R < num_sms ? p.R : num_sms; }
+// One CTA per SM, or per row when rows are fewer; two per row when every row
+// is split in halves (at most half as many rows as SMs).
+inline int fused_grid(const Dev& p, const FusedStep& fs, int num_sms) {
+  if (fs.half_rows > 0 && fs.half_rows == p.R && 2 * p.R <= num_sms) return 2 * p.R;
+  return p.R < num_sms ? p.R : num_sms;
+}
 
 }  // namespace
 }  // namespace dc

@@ -7,7 +7,7 @@ namespace dc {
 
 cudaError_t launch_fused_heur_perrow(const FusedMaps& maps, const Dev& p, const Step& st, const FusedStep& fs,
                                      const FusedPolicy& fp, int num_sms, cudaStream_t s) {
-  const int grid = fused_grid(p, num_sms);
+  const int grid = fused_grid(p, fs, num_sms);
   // per-row budgets rank with the policy (the host keeps heuristic scorers with
   // per-row budgets on the split engine); both variants take any row length
 #define DC_FUSED_LAUNCH(D, G)                                                               \
