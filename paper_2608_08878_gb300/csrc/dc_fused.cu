@@ -97,10 +97,11 @@ cudaError_t make_fused_maps(const Dev& p, FusedMaps* maps, const char** why) {
   }
   const cuuint64_t dims[2] = {(cuuint64_t)p.d, (cuuint64_t)p.R * (cuuint64_t)p.stride};
   const cuuint64_t strides[1] = {(cuuint64_t)p.d * 2};
-  const cuuint32_t box[2] = {64, 128};
   const cuuint32_t estr[2] = {1, 1};
-  for (int which = 0; which < 2; ++which) {
-    CUresult r = encode(which ? &maps->v : &maps->k, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, which ? (void*)p.V : (void*)p.K,
+  CUtensorMap* const out[4] = {&maps->k, &maps->v, &maps->k16, &maps->v16};
+  for (int which = 0; which < 4; ++which) {
+    const cuuint32_t box[2] = {64, which < 2 ? 128u : 16u};
+    CUresult r = encode(out[which], CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, (which & 1) ? (void*)p.V : (void*)p.K,
                         dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
                         CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
     if (r != CUDA_SUCCESS) {

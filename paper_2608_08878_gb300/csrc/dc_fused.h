@@ -17,7 +17,8 @@ namespace dc {
 constexpr int kFusedMaxTok = 10240;
 
 struct FusedMaps {
-  CUtensorMap k, v;  // [R * cap][d] bf16, boxes of 64 dims x 128 tokens, 128-byte swizzle
+  CUtensorMap k, v;      // [R * cap][d] bf16, boxes of 64 dims x 128 tokens, 128-byte swizzle
+  CUtensorMap k16, v16;  // the same with boxes of 64 dims x 16 tokens (a row's ragged last tile)
 };
 
 struct FusedStep {

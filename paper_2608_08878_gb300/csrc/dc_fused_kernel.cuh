@@ -293,7 +293,8 @@ __device__ __forceinline__ Item read_item(volatile int* ring, int gr, volatile i
 // row's new length after its selection. No half rows.
 template <int D, int G, bool LONG, bool FULL, bool HEUR, bool GLOB, bool PERROW, bool PAIR>
 __global__ void __launch_bounds__(kThreads, 1)
-    fused_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmV, Dev p,
+    fused_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmV,
+                 const __grid_constant__ CUtensorMap tmK16, const __grid_constant__ CUtensorMap tmV16, Dev p,
                  Step st, FusedStep fs, FusedPolicy fp) {
   constexpr int GS = G - 1;  // heads whose logits wait in TMEM between the passes
   static_assert(!PAIR || (!LONG && !FULL && !HEUR && !GLOB && !PERROW), "row pairs: the plain step only");
@@ -352,11 +353,15 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (blockIdx.x == 0) fs.work[(fs.epoch + 1u) & 1u] = 0u;
     fence_mbar_init();
   }
-  // zero the query, weight and policy-input tiles (unused rows and columns
-  // stay zero), then write the policy layer's B operand (128 rows x 32 bf16,
-  // 64-byte swizzle)
-  for (int e = threadIdx.x; e < (OFF_W - OFF_Q) / 16; e += kThreads)
-    reinterpret_cast<uint4*>(smem + OFF_Q)[e] = make_uint4(0, 0, 0, 0);
+  // zero the stages and their per-token areas (a row's ragged last tile loads
+  // only its tokens: the rows past them then hold earlier tiles' finite data,
+  // whose attention weights are zero), the query, weight and policy-input
+  // tiles (unused rows and columns stay zero), then write the policy layer's
+  // B operand (128 rows x 32 bf16, 64-byte swizzle)
+  for (int e = threadIdx.x; e < (OFF_W - OFF_STAGE) / 16; e += kThreads)
+    reinterpret_cast<uint4*>(smem + OFF_STAGE)[e] = make_uint4(0, 0, 0, 0);
+  for (int e = threadIdx.x; e < kStages * kAuxBytes / 16; e += kThreads)
+    reinterpret_cast<uint4*>(smem + OFF_AUX)[e] = make_uint4(0, 0, 0, 0);
   for (int e = threadIdx.x; e < 128 * 4; e += kThreads) {
     const int row = e >> 2, c = e & 3;
     *reinterpret_cast<uint4*>(smem + OFF_W + sw64(row, c)) = reinterpret_cast<const uint4*>(fp.wtile)[row * 4 + c];
@@ -369,6 +374,8 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (warp == 0 && lane == 0) {
     prefetch_tmap(&tmK);
     prefetch_tmap(&tmV);
+    prefetch_tmap(&tmK16);
+    prefetch_tmap(&tmV16);
   }
   __syncthreads();
   tc_fence_after();
@@ -432,15 +439,33 @@ __global__ void __launch_bounds__(kThreads, 1)
             const int j = it.t0 + (PAIR ? x >> 1 : x), rt = r + (PAIR ? x & 1 : 0);
             const int s = g % kStages;
             if (!mbar_wait(&bar[B_EMPTY + s], ((g / kStages) & 1) ^ 1, abort, p.dbg, 2u, (unsigned)g)) break;
-            mbar_expect_tx(&bar[B_FULL + s], kTileBytes + ((pass || FULL) ? 0u : GLOB ? 512u : 2560u));
+            // the tile's tokens: all 128, or the row's ragged last tile, loaded
+            // in boxes of 16 tokens
+            const int nrow = PERROW ? p.rowlen[rt] : n_step;
+            const int valid = nrow - j * kTok < kTok ? nrow - j * kTok : kTok;
+            const int nbox = valid < kTok ? (valid + 15) >> 4 : 0;
+            const uint32_t kv_bytes = nbox ? (uint32_t)nbox * 16u * (uint32_t)D * 2u : kTileBytes;
+            const uint32_t pos_bytes = ((uint32_t)valid * 4u + 15u) & ~15u, sz_bytes = (uint32_t)valid * 16u;
+            const uint32_t aux_bytes = (pass || FULL) ? 0u : pos_bytes + (GLOB ? 0u : sz_bytes);
+            mbar_expect_tx(&bar[B_FULL + s], kv_bytes + aux_bytes);
             uint8_t* dst = smem + OFF_STAGE + s * kStageBytes;
             uint8_t* aux = smem + OFF_AUX + s * kAuxBytes;
             const int y = rt * p.stride + j * kTok;
-            tma_load_2d(dst, tm, 0, y, &bar[B_FULL + s], pol);
-            if (D == 128) tma_load_2d(dst + 16384, tm, 64, y, &bar[B_FULL + s], pol);
+            if (nbox == 0) {
+              tma_load_2d(dst, tm, 0, y, &bar[B_FULL + s], pol);
+              if (D == 128) tma_load_2d(dst + 16384, tm, 64, y, &bar[B_FULL + s], pol);
+            } else {
+              // a 16-token box fills 2 KB (two 1 KB swizzle atoms) of each
+              // 64-dim half, where the whole tile's load would put those rows
+              const CUtensorMap* tm16 = pass ? &tmV16 : &tmK16;
+              for (int b = 0; b < nbox; ++b) {
+                tma_load_2d(dst + b * 2048, tm16, 0, y + 16 * b, &bar[B_FULL + s], pol);
+                if (D == 128) tma_load_2d(dst + 16384 + b * 2048, tm16, 64, y + 16 * b, &bar[B_FULL + s], pol);
+              }
+            }
             if (!FULL && !pass) {
-              bulk_load(aux + kAuxPos, p.pos + y, 512, &bar[B_FULL + s]);
-              if (!GLOB) bulk_load(aux + kAuxSZ, p.SZ + y, 2048, &bar[B_FULL + s]);
+              bulk_load(aux + kAuxPos, p.pos + y, pos_bytes, &bar[B_FULL + s]);
+              if (!GLOB) bulk_load(aux + kAuxSZ, p.SZ + y, sz_bytes, &bar[B_FULL + s]);
             }
             issued = g + 1;
           }
@@ -1105,7 +1130,7 @@ static cudaError_t launch_t(const FusedMaps& maps, const Dev& p, const Step& st,
   }
   if (fs.half_rows == 0) {
     fused_kernel<D, G, LONG, FULL, HEUR, GLOB, PERROW, PAIR>
-        <<<grid, kThreads, kSmemBytes, s>>>(maps.k, maps.v, p, st, fs, fp);
+        <<<grid, kThreads, kSmemBytes, s>>>(maps.k, maps.v, maps.k16, maps.v16, p, st, fs, fp);
     return cudaGetLastError();
   }
   // the two CTAs of a half row wait on each other: a cooperative launch
@@ -1120,8 +1145,8 @@ static cudaError_t launch_t(const FusedMaps& maps, const Dev& p, const Step& st,
   la[0].val.cooperative = 1;
   cfg.attrs = la;
   cfg.numAttrs = 1;
-  return cudaLaunchKernelEx(&cfg, fused_kernel<D, G, LONG, FULL, HEUR, GLOB, PERROW, PAIR>, maps.k, maps.v, p, st, fs,
-                            fp);
+  return cudaLaunchKernelEx(&cfg, fused_kernel<D, G, LONG, FULL, HEUR, GLOB, PERROW, PAIR>, maps.k, maps.v, maps.k16,
+                            maps.v16, p, st, fs, fp);
 }
 
 // One CTA per SM, or per row when rows are fewer; two per row when every row

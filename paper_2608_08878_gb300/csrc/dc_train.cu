@@ -5,10 +5,13 @@
 // log Z(s, B, tau) = log sum over subsets a of [L], |a| = B, of
 // exp(sum_{i in a} s_i / tau): the log of the elementary symmetric polynomial
 // e_B of x_i = exp(s_i / tau). With E_i[k] = e_k(x_1..x_i), adding item i
-// gives E_i[k] = E_{i-1}[k] + x_i E_{i-1}[k-1] (E[0] = 1): L sequential steps,
-// each an independent update of k = 1..B -- O(L B) work in O(B) memory, one
-// CTA per row with the B + 1 terms in shared memory, kept in log space
-// (logaddexp), fp32.
+// gives E_i[k] = E_{i-1}[k] + x_i E_{i-1}[k-1] (E[0] = 1). Items are added in
+// chunks of 31: the generating polynomial prod_i (1 + x_i t) of a chunk has
+// coefficients c_m = e_m(chunk), and E_{i+31}[k] = sum_m E_i[k-m] c_m (the
+// product of the two polynomials). One warp builds a chunk's c_m by the
+// item-by-item recurrence (lane m holds c_m); the CTA then convolves, one
+// barrier per chunk instead of per item. O(L B) work in O(B) memory, one CTA
+// per row, in log space (log-sum-exp), fp32.
 //
 // Gumbel-top-B: perturbed scores s_i / tau + g_i (g_i ~ Gumbel(0, 1), given by
 // the caller), the B largest kept (ties: lower index), their indices written
@@ -41,38 +44,61 @@ __device__ __forceinline__ float log2_add_exp2(float a, float b) {
   return m + lg2(1.f + ex2(fminf(a, b) - m));
 }
 
-// One CTA per row, kLzThreads threads (each owns the terms k = tid, tid +
-// kLzThreads, ...), E = log2 e_k in shared memory, double-buffered ([2][B + 1]).
+constexpr int kChunk = 31;        // items per chunk: c_0..c_31 in one warp's lanes
+constexpr int kChunkBatch = 64;   // chunks whose polynomials are built per pass
+
+// One CTA per row, up to kLzThreads threads (each owns the terms k = tid, tid
+// + blockDim, ...). Shared memory: E = log2 e_k, double-buffered ([2][B + 1]),
+// then the polynomials of a batch of chunks ([kChunkBatch][32], log2 c_m).
 __global__ void __launch_bounds__(kLzThreads) pl_logz_kernel(const float* __restrict__ scores, int L, int B,
                                                              float tau, float* __restrict__ out) {
   extern __shared__ float E[];
   constexpr float kLog2e = 1.4426950408889634f, kLn2 = 0.6931471805599453f;
-  const int row = blockIdx.x;
+  const int row = blockIdx.x, tid = threadIdx.x, lane = tid % kWarp, warp = tid / kWarp;
+  const int nwarps = blockDim.x / kWarp;
   const float* s = scores + (size_t)row * L;
   float* cur = E;
   float* nxt = E + (B + 1);
-  for (int k = threadIdx.x; k <= B; k += blockDim.x) cur[k] = k == 0 ? 0.f : -INFINITY;
-  __syncthreads();
-  const int lane = threadIdx.x % kWarp;
-  for (int i0 = 0; i0 < L; i0 += kWarp) {
-    // the next 32 items' s_i / tau in log2 units, one per lane, broadcast
-    // per step by shuffle (off the step's dependency chain)
-    const float yl = i0 + lane < L ? __fmul_rn(__fdiv_rn(s[i0 + lane], tau), kLog2e) : 0.f;
-    const int cnt = min(kWarp, L - i0);
-    for (int j = 0; j < cnt; ++j) {
-      const float y = __shfl_sync(0xffffffffu, yl, j);
-      const int i = i0 + j;
-      // after item i (0-based) only E[0..i+1] can be finite
-      const int kmax = min(B, i + 1);
-      for (int k = threadIdx.x; k <= B; k += blockDim.x)
-        nxt[k] = (k == 0 || k > kmax) ? cur[k] : log2_add_exp2(cur[k], y + cur[k - 1]);
+  float* C = E + 2 * (B + 1);
+  for (int k = tid; k <= B; k += blockDim.x) cur[k] = k == 0 ? 0.f : -INFINITY;
+  const int nchunks = (L + kChunk - 1) / kChunk;
+  for (int c0 = 0; c0 < nchunks; c0 += kChunkBatch) {
+    const int cb = min(kChunkBatch, nchunks - c0);
+    // each warp: the polynomials of its chunks, item by item (lane m: c_m;
+    // all lanes read c_{m-1} before any writes, through the shuffle)
+    for (int ci = warp; ci < cb; ci += nwarps) {
+      const int i0 = (c0 + ci) * kChunk, cnt = min(kChunk, L - i0);
+      // the chunk's s_i / tau in log2 units, one per lane
+      const float yl = lane < cnt ? __fmul_rn(__fdiv_rn(s[i0 + lane], tau), kLog2e) : 0.f;
+      float e = lane == 0 ? 0.f : -INFINITY;
+      for (int j = 0; j < cnt; ++j) {
+        const float y = __shfl_sync(0xffffffffu, yl, j);
+        const float below = __shfl_up_sync(0xffffffffu, e, 1);
+        if (lane >= 1 && lane <= j + 1) e = log2_add_exp2(e, y + below);
+      }
+      C[ci * kWarp + lane] = e;
+    }
+    __syncthreads();
+    // E <- E * c, chunk by chunk: E'[k] = log2 sum_m 2^(E[k-m] + c_m)
+    for (int ci = 0; ci < cb; ++ci) {
+      const float* c = C + ci * kWarp;
+      const int cnt = min(kChunk, L - (c0 + ci) * kChunk);
+      for (int k = tid; k <= B; k += blockDim.x) {
+        const int mmax = min(k, cnt);
+        float mx = -INFINITY;
+        for (int m = 0; m <= mmax; ++m) mx = fmaxf(mx, cur[k - m] + c[m]);
+        float acc = 0.f;
+        if (mx != -INFINITY)
+          for (int m = 0; m <= mmax; ++m) acc += ex2(cur[k - m] + c[m] - mx);
+        nxt[k] = mx == -INFINITY ? -INFINITY : mx + lg2(acc);
+      }
       __syncthreads();
       float* t = cur;
       cur = nxt;
       nxt = t;
     }
   }
-  if (threadIdx.x == 0) out[row] = cur[B] * kLn2;
+  if (tid == 0) out[row] = cur[B] * kLn2;
 }
 
 // One CTA per row: top-B of the perturbed scores by (value desc, index asc),
@@ -158,8 +184,8 @@ extern "C" dc_status dc_pl_log_partition(const float* scores, int rows, int L, i
   if (!scores || !out) return train_fail(DC_ERR_INVALID_ARG, "NULL pointer");
   if (rows < 1 || rows > 65535 || L < 1 || B < 1 || B > L || !(tau > 0.f))
     return train_fail(DC_ERR_INVALID_ARG, "need 1 <= rows <= 65535, 1 <= B <= L and tau > 0");
-  const size_t smem = 2 * (size_t)(B + 1) * sizeof(float);
-  if (smem > 200 * 1024) return train_fail(DC_ERR_INVALID_ARG, "B too large (at most 25599)");
+  const size_t smem = (2 * (size_t)(B + 1) + kChunkBatch * kWarp) * sizeof(float);
+  if (2 * (size_t)(B + 1) * sizeof(float) > 200 * 1024) return train_fail(DC_ERR_INVALID_ARG, "B too large (at most 25599)");
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   if (smem > 48 * 1024) {
     cudaError_t e = cudaFuncSetAttribute(pl_logz_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
