@@ -47,9 +47,10 @@ __device__ __forceinline__ float log2_add_exp2(float a, float b) {
 constexpr int kChunk = 31;        // items per chunk: c_0..c_31 in one warp's lanes
 constexpr int kChunkBatch = 64;   // chunks whose polynomials are built per pass
 
-// One CTA per row, up to kLzThreads threads (each owns the terms k = tid, tid
-// + blockDim, ...). Shared memory: E = log2 e_k, double-buffered ([2][B + 1]),
-// then the polynomials of a batch of chunks ([kChunkBatch][32], log2 c_m).
+// One CTA per row, up to kLzThreads threads (each owns the terms k = 1 + tid,
+// 1 + tid + blockDim, ...; e_0 = 1 never changes, so B = 1024 takes one term
+// per thread). Shared memory: E = log2 e_k, double-buffered ([2][B + 1]), then
+// the polynomials of a batch of chunks ([kChunkBatch][32], log2 c_m).
 __global__ void __launch_bounds__(kLzThreads) pl_logz_kernel(const float* __restrict__ scores, int L, int B,
                                                              float tau, float* __restrict__ out) {
   extern __shared__ float E[];
@@ -60,7 +61,7 @@ __global__ void __launch_bounds__(kLzThreads) pl_logz_kernel(const float* __rest
   float* cur = E;
   float* nxt = E + (B + 1);
   float* C = E + 2 * (B + 1);
-  for (int k = tid; k <= B; k += blockDim.x) cur[k] = k == 0 ? 0.f : -INFINITY;
+  for (int k = tid; k <= B; k += blockDim.x) cur[k] = nxt[k] = k == 0 ? 0.f : -INFINITY;
   const int nchunks = (L + kChunk - 1) / kChunk;
   for (int c0 = 0; c0 < nchunks; c0 += kChunkBatch) {
     const int cb = min(kChunkBatch, nchunks - c0);
@@ -83,13 +84,19 @@ __global__ void __launch_bounds__(kLzThreads) pl_logz_kernel(const float* __rest
     for (int ci = 0; ci < cb; ++ci) {
       const float* c = C + ci * kWarp;
       const int cnt = min(kChunk, L - (c0 + ci) * kChunk);
-      for (int k = tid; k <= B; k += blockDim.x) {
+      for (int k = 1 + tid; k <= B; k += blockDim.x) {
         const int mmax = min(k, cnt);
+        // the terms in registers: shared memory is read once
+        float t[kChunk + 1];
         float mx = -INFINITY;
-        for (int m = 0; m <= mmax; ++m) mx = fmaxf(mx, cur[k - m] + c[m]);
+#pragma unroll
+        for (int m = 0; m <= kChunk; ++m) {
+          t[m] = m <= mmax ? cur[k - m] + c[m] : -INFINITY;
+          mx = fmaxf(mx, t[m]);
+        }
         float acc = 0.f;
-        if (mx != -INFINITY)
-          for (int m = 0; m <= mmax; ++m) acc += ex2(cur[k - m] + c[m] - mx);
+#pragma unroll
+        for (int m = 0; m <= kChunk; ++m) acc += ex2(t[m] - mx);
         nxt[k] = mx == -INFINITY ? -INFINITY : mx + lg2(acc);
       }
       __syncthreads();
@@ -191,7 +198,7 @@ extern "C" dc_status dc_pl_log_partition(const float* scores, int rows, int L, i
     cudaError_t e = cudaFuncSetAttribute(pl_logz_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return train_fail(DC_ERR_CUDA, cudaGetErrorString(e));
   }
-  const int threads = B + 1 < kLzThreads ? (B + 1 + 31) / 32 * 32 : kLzThreads;
+  const int threads = B < kLzThreads ? (B + 31) / 32 * 32 : kLzThreads;
   pl_logz_kernel<<<rows, threads, smem, s>>>(scores, L, B, tau, out);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return train_fail(DC_ERR_CUDA, cudaGetErrorString(e));
