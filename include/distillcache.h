@@ -27,6 +27,13 @@
  *     dc_last_error() gives the message. Invalid arguments leave the cache
  *     unchanged.
  *   - Calls on one handle must not run concurrently from several host threads.
+ *   - The handle keeps the step's host-side state (row lengths, the window
+ *     slot, the launch epoch that keys the fused kernel's work queue and
+ *     exchange flags) and advances it on every call; the launches it enqueues
+ *     carry that step's values. A stream capture of a call therefore records
+ *     one particular step: replaying the captured graph repeats that step's
+ *     arguments and is not a later decode step. (dc_attend_noalloc keeps no
+ *     state and may be captured and replayed.)
  */
 #ifndef DISTILLCACHE_H
 #define DISTILLCACHE_H
