@@ -189,7 +189,8 @@ dc_status launch_error(dc_cache* h, const char* what) {
   return DC_OK;
 }
 
-// Fused engine for this step? (auto: only when the rows fill the GPU)
+// Fused engine for a step over n tokens per row? (auto: whenever the rows fill
+// at least half the SMs, else by the latency estimates below)
 bool use_fused(const dc_cache* h, int n) {
   // rows of different lengths: the fused kernel ranks them with the policy only
   if (h->per_row && h->dev.scorer != 0) return false;

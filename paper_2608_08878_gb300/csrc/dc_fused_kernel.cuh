@@ -10,8 +10,11 @@
 // statistics), the five token features of Sec. 3.1.1, the policy MLP of
 // Sec. 3.1.2 / App. D, and (dc_step) the top-B select and compaction.
 //
-// One CTA per SM; the CTAs take rows (and, for a partly filled last wave,
-// half rows) from a shared queue as they become free.
+// One CTA per SM (or per row, or two per row: rows of 12 tiles or more are
+// split in halves when there are at most half as many rows as SMs); the CTAs
+// take rows, half rows (also for a partly filled last wave) or, on short rows,
+// row pairs (PAIR) from a shared queue as they become free. A row's ragged
+// last tile is loaded in boxes of 16 tokens.
 // Warp roles (352 threads):
 //   warp 0     producer: takes the next row, writes its query tile (current,
 //              previous and departing queries) and streams K then V tiles of
