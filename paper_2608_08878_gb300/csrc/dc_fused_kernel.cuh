@@ -695,6 +695,14 @@ __global__ void __launch_bounds__(kThreads, 1)
       float4 szA = kZero4, szB = kZero4;
       int posA = 0, posB = 0;
       float vnA = 0.f, vnB = 0.f;
+      // HEUR: cumulative alpha (H2O's score) loaded ahead the same way
+      const bool ac_ahead = HEUR && p.alpha_mode == 1;
+      const float* acrow = ac_ahead ? p.acc + rbase + tok : nullptr;
+      float acA = 0.f, acB = 0.f;
+      if (ac_ahead) {
+        acA = j0 < t1 ? acrow[j0 * kTok] : 0.f;
+        acB = j0 + JS < t1 ? acrow[(j0 + JS) * kTok] : 0.f;
+      }
       if constexpr (!FULL && !GLOB) {
         szA = j0 < t1 ? szrow[j0 * kTok] : kZero4;
         szB = j0 + JS < t1 ? szrow[(j0 + JS) * kTok] : kZero4;
@@ -816,16 +824,18 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int gvj = gv + tpos(j, t0), pb = gvj & 1;
         const float4 sz = szA;
         const int pos = posA;
-        const float vn = vnA;
+        const float vn = vnA, ac = acA;
         szA = szB;
         posA = posB;
         vnA = vnB;
+        acA = acB;
         if (!FULL && j + 2 * JS < t1) {
           if constexpr (!GLOB) {
             szB = szrow[(j + 2 * JS) * kTok];
             posB = posrow[(j + 2 * JS) * kTok];
           }
           vnB = vnrow[(j + 2 * JS) * kTok];
+          if (ac_ahead) acB = acrow[(j + 2 * JS) * kTok];
         }
         const int i = j * kTok + tok;
         const bool valid = i < n;
@@ -890,7 +900,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (valid) {
           const size_t slot = rbase + i;
           if (p.alpha_mode == 1) {
-            x[0] = p.acc[slot] + mean;
+            x[0] = (ac_ahead ? ac : p.acc[slot]) + mean;
             p.acc[slot] = x[0];
           }
           if (p.keep_features)
