@@ -221,10 +221,19 @@ def oracle_sample(wl, seconds: float = 12.0, threads: int | None = None, warm_st
     el = time.perf_counter() - t0
     row_steps = sum(counts.values())
     steps_per_s = row_steps / wl.rows / el
+    # the same on one host thread: one sampled row for a third of the time
+    r1 = sample_rows[0]
+    counts = {r1: 0}
+    t1 = time.perf_counter()
+    deadline[0] = t1 + seconds / 3
+    run(r1)
+    el1 = time.perf_counter() - t1
     return {"value": steps_per_s, "unit": UNIT, "cores": len(sample_rows), "kind": "oracle",
             "sample": (f"{len(sample_rows)} rows (of {wl.rows}) at the steady state n={wl.budget + 1}, "
                        f"full w={wl.window} window, {row_steps} row-steps in {el:.1f}s on "
-                       f"{len(sample_rows)} host threads; value = row-steps / rows / s")}
+                       f"{len(sample_rows)} host threads; value = row-steps / rows / s"),
+            "single_thread": {"value": counts[r1] / wl.rows / el1, "unit": UNIT, "cores": 1,
+                              "sample": f"row {r1}, {counts[r1]} row-steps in {el1:.1f}s on one host thread"}}
 
 
 # ---------------------------------------------------------------------------
