@@ -538,3 +538,52 @@ def test_async_host_steps_equal_device_steps():
         assert torch.equal(outs[s], refs[s]), s
     for which in (dc.BUF_K, dc.BUF_POS, dc.BUF_S):
         assert torch.equal(a.cache.buffer(which), b.cache.buffer(which))
+
+
+def _boundary_workload(kind, budget):
+    import torch
+    sms = torch.cuda.get_device_properties(0).multi_processor_count
+    batch = {"few": 1, "pairs": sms // 2}[kind]  # 8 rows, or 4 rows per SM
+    # prompt = budget: every step appends one token and evicts one, n = budget + 1
+    return synth.MISTRAL_1L.with_(batch=batch, prompt_len=budget, budget=budget, steps=3, window=4)
+
+
+@pytest.mark.parametrize("kind,budget,engine", [
+    ("few", 1535, "fused"),         # 12 whole tiles: every row in halves, no ragged tile
+    ("few", 1536, "fused"),         # 13 tiles in halves, half 1 ends on a 1-token tile
+    ("few", 127, "fused"),          # one whole tile
+    ("few", 16, "fused"),           # one tile of 17 tokens: two 16-token boxes
+    ("pairs", 2687, "fused-pairs"),  # 21 whole tiles, the longest row pairs take
+    ("pairs", 15, "fused-pairs"),    # one tile of 16 tokens: one box
+    ("pairs", 2688, "fused"),        # 22 tiles: whole rows, a 1-token ragged tile
+])
+def test_work_item_boundaries(kind, budget, engine):
+    """The fused engine's work items at their boundaries (halves for few rows
+    from 12 tiles, row pairs up to 21 tiles, a row's ragged last tile loaded in
+    16-token boxes): sampled rows against the oracle over steps past the
+    window, and dc_step's in-kernel eviction bit-identical to dc_decode_step
+    and dc_evict."""
+    import torch
+    from paper_2608_08878_gb300 import dc
+    wl = _boundary_workload(kind, budget)
+    rows = [0, wl.rows // 2 + 1, wl.rows - 1]
+    ls = LockStep(wl, rows, engine=0, device_inputs=True)
+    assert ls.cache.engine(budget + 1) == engine
+    ls.load_prompt()
+    for _ in range(wl.steps):
+        ls.step()
+    a, b = LockStep(wl, [], engine=0, device_inputs=True), LockStep(wl, [], engine=0, device_inputs=True)
+    for x in (a, b):
+        x.load_prompt()
+    for s in range(wl.steps + 4):
+        q, kn, vn = a._inputs(s)
+        oa = a.cache.step(q, kn, vn)
+        ob = b.cache.decode_step(q, kn, vn)
+        b.cache.evict()
+        a.cache.sync()
+        b.cache.sync()
+        assert torch.equal(oa, ob), s
+        n = a.cache.length()[0]
+        assert n == b.cache.length()[0] == budget
+        for which in (dc.BUF_K, dc.BUF_V, dc.BUF_POS, dc.BUF_S, dc.BUF_Z, dc.BUF_VNORM):
+            assert torch.equal(a.cache.buffer(which)[:, :n], b.cache.buffer(which)[:, :n]), (s, which)
