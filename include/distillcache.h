@@ -309,6 +309,20 @@ dc_status dc_attend_noalloc(const void* q, const void* k, const void* v, int row
 /* Message of the last failed dc_attend_noalloc call on this host thread. */
 const char* dc_noalloc_last_error(void);
 
+/* Self-test of the bounded waits every kernel relies on (a wait that cannot be
+ * satisfied gives up after its time limit, records where and lets the kernel
+ * return an error status instead of hanging): one thread waits limit_ns on a
+ * flag in global memory that nothing sets, then limit_ns on an mbarrier that
+ * nothing arrives on. result (host, 7 values): [0] bit 0 the flag wait gave
+ * up, bit 1 the mbarrier wait gave up (3 = both, as they must); [1..4] the first
+ * timeout's record (claim flag, site 901 for the flag, block, waited value);
+ * [5], [6] each wait's duration in microseconds. limit_ns within [1 ms, 1 s].
+ * Synchronises the stream; the CUDA context stays usable. */
+dc_status dc_wait_selftest(unsigned long long limit_ns, unsigned* result, void* stream);
+
+/* Message of the last failed dc_wait_selftest call on this host thread. */
+const char* dc_selftest_last_error(void);
+
 /* Message of the last error on the handle (or of the last failed create when
  * h is NULL). Valid until the next call on the handle. */
 const char* dc_last_error(const dc_cache* h);

@@ -88,13 +88,14 @@ __device__ __forceinline__ void record_timeout(unsigned* dbg, unsigned site, uns
 // *abort is set by another role, or when the time limit passes, in which case
 // it records the site and sets *abort itself so that every role winds down.
 __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, volatile int* abort,
-                                          unsigned* dbg = nullptr, unsigned site = 0, unsigned info = 0) {
+                                          unsigned* dbg = nullptr, unsigned site = 0, unsigned info = 0,
+                                          uint64_t limit_ns = kWaitNs) {
   if (mbar_try_wait(bar, parity)) return true;
   const uint64_t t0 = globaltimer_ns();
   for (uint32_t i = 1; i < kSpinLimit; ++i) {
     if (mbar_try_wait(bar, parity)) return true;
     if (*abort) return false;
-    if ((i & 255u) == 0 && globaltimer_ns() - t0 > kWaitNs) break;
+    if ((i & 255u) == 0 && globaltimer_ns() - t0 > limit_ns) break;
   }
   record_timeout(dbg, site, parity, info);
   *abort = 1;
@@ -128,12 +129,13 @@ __device__ __forceinline__ unsigned flag_acquire(const unsigned* f) {
 // Waits until *f has reached `target` (wrap-safe compare). Bounded like
 // mbar_wait: gives up on *abort or after kWaitNs, recording the site.
 __device__ __forceinline__ bool flag_wait(const unsigned* f, unsigned target, volatile int* abort,
-                                          unsigned* dbg, unsigned site, unsigned info) {
+                                          unsigned* dbg, unsigned site, unsigned info,
+                                          uint64_t limit_ns = kWaitNs) {
   const uint64_t t0 = globaltimer_ns();
   for (uint32_t i = 0; i < kSpinLimit; ++i) {
     if ((int)(flag_acquire(f) - target) >= 0) return true;
     if (*abort) return false;
-    if ((i & 63u) == 63u && globaltimer_ns() - t0 > kWaitNs) break;
+    if ((i & 63u) == 63u && globaltimer_ns() - t0 > limit_ns) break;
     __nanosleep(64);
   }
   record_timeout(dbg, site, target, info);

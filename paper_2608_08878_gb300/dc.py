@@ -30,7 +30,7 @@ EXPORTS = ["dc_config_default", "dc_cache_create", "dc_cache_destroy", "dc_polic
            "dc_copy_buffer", "dc_sync", "dc_last_error", "dc_phase_name", "dc_profile_enable",
            "dc_profile_read", "dc_step", "dc_step_host", "dc_step_host_async", "dc_engine", "dc_attend_noalloc",
            "dc_noalloc_last_error", "dc_pl_log_partition", "dc_gumbel_top_b", "dc_train_last_error",
-           "dc_set_row_budgets", "dc_get_row_lengths"]
+           "dc_set_row_budgets", "dc_get_row_lengths", "dc_wait_selftest", "dc_selftest_last_error"]
 PHASES = ["append", "attend", "stats", "score", "combine", "evict", "full"]
 
 
@@ -89,6 +89,9 @@ def lib():
             L.dc_gumbel_top_b.argtypes = [P, P, I, I, I, C.c_float, P, P, P, P]
             L.dc_train_last_error.argtypes = []
             L.dc_train_last_error.restype = C.c_char_p
+            L.dc_wait_selftest.argtypes = [C.c_ulonglong, P, P]
+            L.dc_selftest_last_error.argtypes = []
+            L.dc_selftest_last_error.restype = C.c_char_p
             L.dc_get_length.argtypes = [P, C.POINTER(I), C.POINTER(C.c_longlong)]
             L.dc_buffer_bytes.argtypes = [P, I, C.POINTER(S)]
             L.dc_copy_buffer.argtypes = [P, I, I, I, P, S]
@@ -101,7 +104,7 @@ def lib():
             L.dc_profile_read.argtypes = [P, P, P]
             for name in EXPORTS:
                 if name not in ("dc_policy_blob_len", "dc_last_error", "dc_phase_name", "dc_noalloc_last_error",
-                                "dc_train_last_error"):
+                                "dc_train_last_error", "dc_selftest_last_error"):
                     getattr(L, name).restype = I
             _lib = L
     return _lib
@@ -134,6 +137,20 @@ def attend_noalloc(q, k, v, out=None, stream=None):
     if st != DC_OK:
         raise DCError(st, lib().dc_noalloc_last_error().decode())
     return out
+
+
+def wait_selftest(limit_ms: float = 50.0, stream=None) -> dict:
+    """Runs the bounded-wait self-test (a flag nothing sets, an mbarrier
+    nothing arrives on, each waited for limit_ms) and returns what the kernel
+    recorded."""
+    import torch
+    res = np.zeros(7, dtype=np.uint32)
+    s = (stream or torch.cuda.current_stream()).cuda_stream
+    st = lib().dc_wait_selftest(C.c_ulonglong(int(limit_ms * 1e6)), res.ctypes.data_as(C.c_void_p), s)
+    if st != DC_OK:
+        raise DCError(st, lib().dc_selftest_last_error().decode())
+    return {"flag_gave_up": bool(res[0] & 1), "barrier_gave_up": bool(res[0] & 2), "site": int(res[2]),
+            "flag_wait_us": int(res[5]), "barrier_wait_us": int(res[6])}
 
 
 def pl_log_partition(scores, B: int, tau: float = 1.0, out=None, stream=None):

@@ -587,3 +587,21 @@ def test_work_item_boundaries(kind, budget, engine):
         assert n == b.cache.length()[0] == budget
         for which in (dc.BUF_K, dc.BUF_V, dc.BUF_POS, dc.BUF_S, dc.BUF_Z, dc.BUF_VNORM):
             assert torch.equal(a.cache.buffer(which)[:, :n], b.cache.buffer(which)[:, :n]), (s, which)
+
+
+def test_bounded_waits_give_up_and_leave_the_context_usable():
+    """A wait that nothing will satisfy (a flag nothing sets, an mbarrier
+    nothing arrives on) gives up after its limit, records where, and the
+    kernel returns; the CUDA context and a cache built afterwards still work."""
+    import torch
+    from paper_2608_08878_gb300 import dc
+    res = dc.wait_selftest(limit_ms=20)
+    assert res["flag_gave_up"] and res["barrier_gave_up"], res
+    assert res["site"] == 901, res  # the first timeout of the launch: the flag wait
+    assert res["flag_wait_us"] >= 20000 and res["barrier_wait_us"] >= 20000, res
+    assert res["flag_wait_us"] < 2000000 and res["barrier_wait_us"] < 2000000, res
+    wl = synth.TINY.with_(steps=2)
+    ls = LockStep(wl, range(wl.rows), engine=2)
+    ls.load_prompt()
+    for _ in range(wl.steps):
+        ls.step()
