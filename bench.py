@@ -83,19 +83,31 @@ def step_bytes_global(wl, n: int, moved_per_seq: float = 1.0) -> float:
             + moved_per_seq * wl.rows * 2 * (4 * d + 20))
 
 
+# The fused kernel's source: the kernel template and every header it includes.
+FUSED_KERNEL_SOURCES = ["dc_fused_kernel.cuh", "dc_common.cuh", "dc_fused.h", "dc_kernels.h", "dc_select.cuh",
+                        "dc_sm100.cuh"]
+
+
+def fused_kernel_source_sha() -> str:
+    """sha256 of the fused kernel's source files, concatenated in the order above."""
+    import hashlib
+    h = hashlib.sha256()
+    for f in FUSED_KERNEL_SOURCES:
+        with open(os.path.join(ROOT, "paper_2608_08878_gb300", "csrc", f), "rb") as fh:
+            h.update(fh.read())
+    return h.hexdigest()
+
+
 def fused_traffic_per_token_row():
     """DRAM bytes per token-row of the fused kernel from the committed ncu
     summary, or None if the kernel source changed since it was captured."""
-    import hashlib
     import re
     prof = os.path.join(ROOT, "profiles", "fused_kernel_19L_b4_n8193_ncu_full.md")
-    src = os.path.join(ROOT, "paper_2608_08878_gb300", "csrc", "dc_fused_kernel.cuh")
     try:
         text = open(prof).read()
         t = float(re.search(r"traffic_bytes_per_token_row:\s*([0-9.]+)", text).group(1))
         sha = re.search(r"kernel_source_sha256_prefix:\s*([0-9a-f]+)", text).group(1)
-        cur = hashlib.sha256(open(src, "rb").read()).hexdigest()[:len(sha)]
-        return t if cur == sha else None
+        return t if fused_kernel_source_sha()[:len(sha)] == sha else None
     except Exception:
         return None
 
