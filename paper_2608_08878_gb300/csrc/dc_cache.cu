@@ -199,12 +199,16 @@ bool use_fused(const dc_cache* h, int n) {
   if (h->cfg.engine != 0) return false;
   if (2 * h->dev.R >= h->num_sms) return true;
   // Few rows: the fused kernel gives each its own CTA, which streams a tile in
-  // ~0.75 us after ~11 us of fixed cost (K and V: 1.5 us per 128 tokens); the
-  // split engine spreads the rows over the GPU but costs ~57 us of launches
-  // plus ~0.55 ns per token-row (both measured on Mistral-7B head shapes). The
-  // split engine wins only for a few long rows.
+  // ~0.75 us after ~11 us of fixed cost (K and V: 1.5 us per 128 tokens), or
+  // two CTAs (rows of 12 tiles or more, at most half as many rows as SMs: ~16
+  // us with the exchange, 0.75 us per 128 tokens); the split engine spreads
+  // the rows over the GPU but costs ~57 us of launches plus ~0.55 ns per
+  // token-row (all measured on Mistral-7B head shapes). The split engine wins
+  // only for a few very long rows.
   const double nT = (double)((n + 127) / 128);
-  return 11.0 + 1.5 * nT < 57.0 + 0.00055 * (double)h->dev.R * (double)n;
+  const bool halves = h->xflag != nullptr && 2 * h->dev.R <= h->num_sms && nT >= 12;
+  const double fused_us = halves ? 16.0 + 0.75 * nT : 11.0 + 1.5 * nT;
+  return fused_us < 57.0 + 0.00055 * (double)h->dev.R * (double)n;
 }
 
 cudaError_t upload_fused_policy(dc_cache* h, const float* blob) {
