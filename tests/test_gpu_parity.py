@@ -605,3 +605,41 @@ def test_bounded_waits_give_up_and_leave_the_context_usable():
     ls.load_prompt()
     for _ in range(wl.steps):
         ls.step()
+
+
+def _random_shapes(count=24, seed=2026):
+    """Seeded shapes over the engines' parameters (group, head size, window,
+    alpha mode, engine, rows from a few to several waves, lengths from one
+    token to past the row-pair limit)."""
+    rng = np.random.default_rng(seed)
+    out = []
+    for _ in range(count):
+        group = int(rng.choice([1, 2, 4]))
+        head_dim = int(rng.choice([64, 128]))
+        kv_heads = int(rng.choice([1, 2, 8]))
+        layers = int(rng.integers(1, 5))
+        batch = int(rng.integers(1, 640 // (layers * kv_heads) + 1))
+        prompt = int(rng.integers(1, 3000))
+        budget = int(rng.integers(1, prompt + 40))
+        out.append(dict(group=group, head_dim=head_dim, kv_heads=kv_heads, layers=layers, batch=batch,
+                        prompt_len=prompt, budget=budget, window=int(rng.choice([1, 2, 4, 8])),
+                        alpha_mode=int(rng.integers(0, 2)), engine=int(rng.choice([0, 1, 2])),
+                        steps=int(rng.integers(3, 7))))
+    return out
+
+
+@pytest.mark.parametrize("shape", _random_shapes(), ids=lambda s: "L{layers}b{batch}h{kv_heads}g{group}d{head_dim}"
+                         "p{prompt_len}B{budget}w{window}a{alpha_mode}e{engine}".format(**s))
+def test_random_shapes_match_oracle(shape):
+    """Seeded random shapes against the oracle on sampled rows: whatever
+    schedule the engine picks (split, whole rows, halves, row pairs, ragged
+    tiles), the step's outputs, features, scores and kept sets agree."""
+    sh = dict(shape)
+    engine, group = sh.pop("engine"), sh.pop("group")
+    wl = synth.MISTRAL_1L.with_(q_heads=sh["kv_heads"] * group, **sh)
+    rows = sorted({0, wl.rows // 2, wl.rows - 1})
+    ls = LockStep(wl, rows, engine=engine, device_inputs=True, capacity=max(wl.prompt_len, wl.budget) + 16)
+    ls.load_prompt()
+    for _ in range(wl.steps):
+        ls.step()
+    assert ls.cache.length()[0] == min(wl.prompt_len + wl.steps, wl.budget)
