@@ -643,3 +643,33 @@ def test_random_shapes_match_oracle(shape):
     for _ in range(wl.steps):
         ls.step()
     assert ls.cache.length()[0] == min(wl.prompt_len + wl.steps, wl.budget)
+
+
+@pytest.mark.parametrize("shape", _random_shapes(count=12, seed=7), ids=lambda s: "L{layers}b{batch}h{kv_heads}g{group}"
+                         "d{head_dim}p{prompt_len}B{budget}w{window}a{alpha_mode}e{engine}".format(**s))
+def test_random_shapes_step_equals_decode_then_evict(shape):
+    """Seeded random shapes: dc_step (the fused engine's in-kernel select and
+    compaction wherever it applies) leaves the same output and cache, bit for
+    bit, as dc_decode_step followed by dc_evict."""
+    import torch
+    from paper_2608_08878_gb300 import dc
+    sh = dict(shape)
+    engine, group = sh.pop("engine"), sh.pop("group")
+    wl = synth.MISTRAL_1L.with_(q_heads=sh["kv_heads"] * group, **sh)
+    cap = max(wl.prompt_len, wl.budget) + 16
+    a = LockStep(wl, [], engine=engine, device_inputs=True, capacity=cap)
+    b = LockStep(wl, [], engine=engine, device_inputs=True, capacity=cap)
+    for x in (a, b):
+        x.load_prompt()
+    for s in range(wl.steps):
+        q, kn, vn = a._inputs(s)
+        oa = a.cache.step(q, kn, vn)
+        ob = b.cache.decode_step(q, kn, vn)
+        b.cache.evict()
+        a.cache.sync()
+        b.cache.sync()
+        assert torch.equal(oa, ob), s
+        n = a.cache.length()[0]
+        assert n == b.cache.length()[0]
+        for which in (dc.BUF_K, dc.BUF_V, dc.BUF_POS, dc.BUF_S, dc.BUF_Z, dc.BUF_VNORM):
+            assert torch.equal(a.cache.buffer(which)[:, :n], b.cache.buffer(which)[:, :n]), (s, which)
