@@ -99,3 +99,35 @@ def test_training_kernels_validate_before_touching_the_device():
                                  None) == dc.DC_ERR_INVALID_ARG
     assert L.dc_pl_log_partition(None, 1, 10, 5, 1.0, C.c_void_p(16), None) == dc.DC_ERR_INVALID_ARG
     assert b"B <= L" in L.dc_train_last_error() or b"NULL" in L.dc_train_last_error()
+
+
+def test_header_compiles_as_c_and_matches_the_binding(tmp_path):
+    """A C11 program includes the header, links the library and calls its
+    host-only entry points; the header's dc_config layout (size and every
+    field's offset) is the binding's."""
+    import shutil
+    import subprocess
+    cc = shutil.which("gcc") or shutil.which("cc")
+    if cc is None:
+        pytest.skip("no C compiler")
+    fields = [f for f, _ in dc.dc_config._fields_]
+    src = tmp_path / "abi.c"
+    src.write_text(
+        "#include <stddef.h>\n#include <stdio.h>\n#include \"distillcache.h\"\n"
+        "int main(void) {\n"
+        "  dc_config cfg;\n"
+        "  if (dc_config_default(&cfg) != DC_OK) return 1;\n"
+        "  dc_cache* h = 0;\n"
+        "  if (dc_cache_create(1, 8, 96, 100, 10, &cfg, &h) != DC_ERR_INVALID_ARG || h) return 2;\n"
+        "  printf(\"%zu %zu %d %d\\n\", sizeof(dc_config), dc_policy_blob_len(128), cfg.window, cfg.mlp_hidden);\n"
+        + "".join(f"  printf(\"%zu\\n\", offsetof(dc_config, {f}));\n" for f in fields)
+        + "  return 0;\n}\n")
+    exe = tmp_path / "abi"
+    lib_dir = os.path.dirname(dc.LIB_PATH)
+    subprocess.run([cc, "-std=c11", "-Wall", "-Wextra", "-Werror", "-I", os.path.join(ROOT, "include"), str(src),
+                    "-o", str(exe), "-L", lib_dir, "-ldistillcache", "-Wl,-rpath," + lib_dir], check=True,
+                   capture_output=True, text=True)
+    out = subprocess.run([str(exe)], check=True, capture_output=True, text=True).stdout.split()
+    size, blob, window, hidden = (int(x) for x in out[:4])
+    assert (size, blob, window, hidden) == (C.sizeof(dc.dc_config), 9 * 128 + 1, 64, 128)
+    assert [int(x) for x in out[4:]] == [getattr(dc.dc_config, f).offset for f in fields]
