@@ -31,9 +31,10 @@
  *     slot, the launch epoch that keys the fused kernel's work queue and
  *     exchange flags) and advances it on every call; the launches it enqueues
  *     carry that step's values. A stream capture of a call therefore records
- *     one particular step: replaying the captured graph repeats that step's
- *     arguments and is not a later decode step. (dc_attend_noalloc keeps no
- *     state and may be captured and replayed.)
+ *     one particular step: replaying it repeats that step's arguments. In
+ *     graph mode (dc_set_graph_mode) dc_step counts steps on the device
+ *     instead, and a captured dc_step replays as the following decode steps.
+ *     (dc_attend_noalloc keeps no state and may be captured and replayed.)
  */
 #ifndef DISTILLCACHE_H
 #define DISTILLCACHE_H
@@ -187,6 +188,21 @@ dc_status dc_step_host(dc_cache* h, const void* q_host, const void* k_new_host,
  * then. Pinned host memory keeps the copies asynchronous. */
 dc_status dc_step_host_async(dc_cache* h, const void* q_host, const void* k_new_host,
                              const void* v_new_host, float* out_host, int budget);
+
+/* Graph mode (enable = 1): dc_step (and dc_step_host, dc_step_host_async)
+ * counts its steps in device memory: the kernels advance positions, window
+ * slots and the launch epoch by that count, so the same enqueued work -- a
+ * CUDA graph captured from one dc_step call -- performs the following decode
+ * steps when replayed, with the inputs the captured buffers hold at each
+ * replay. Needs the steady state of the fused engine: the policy scorer, the
+ * fixed budget, every row at the budget (one eviction per step), at least a
+ * window of consecutive decode steps taken, no per-row budgets or global
+ * token mode (DC_ERR_STATE otherwise). Other calls that change the cache
+ * return DC_ERR_STATE while the mode is on; dc_get_length reports the tokens
+ * seen as of entering the mode. enable = 0 synchronises the stream, reads the
+ * count and brings the handle's state up to date; then every call works as
+ * before. */
+dc_status dc_set_graph_mode(dc_cache* h, int enable);
 
 /* Per-row budgets, the head-level hybrid of Sec. 5 (Table tab:hybrid: the most
  * important heads keep the full cache, token selection in the others):

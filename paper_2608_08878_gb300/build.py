@@ -25,7 +25,7 @@ LIB_SYNTH = os.path.join(HERE, "libdc_synth.so")
 
 MAIN_SOURCES = ["dc_cache.cu", "dc_split.cu", "dc_evict.cu", "dc_full.cu", "dc_fused.cu", "dc_noalloc.cu",
                 "dc_train.cu", "dc_global.cu", "dc_fused_modes.cu", "dc_fused_glob.cu",
-                "dc_fused_pair.cu", "dc_selftest.cu"]
+                "dc_fused_pair.cu", "dc_selftest.cu", "dc_fused_graph.cu"]
 SYNTH_SOURCES = ["synth.cu"]
 
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]

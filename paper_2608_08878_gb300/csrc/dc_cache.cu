@@ -86,6 +86,12 @@ struct dc_cache {
   int* roworder_dev = nullptr;
   cudaEvent_t ev_order = nullptr;
   bool order_valid = false;
+  // device-counted steps (dc_set_graph_mode): the base step arguments and
+  // epoch that the kernels advance by the device's step count
+  bool graph = false;
+  dc::Step gstep{};
+  unsigned gepoch = 0;
+  int* gcount_dev = nullptr;
   std::vector<void*> allocs;
   std::string err;
   bool broken = false;
@@ -473,6 +479,7 @@ dc_status dc_cache_destroy(dc_cache* h) {
 
 dc_status dc_policy_set_weights(dc_cache* h, const float* blob, size_t n) {
   DC_CHECK_HANDLE(h);
+  if (h->graph) return fail(h, DC_ERR_STATE, "graph mode: only dc_step and its host forms until dc_set_graph_mode(h, 0)");
   if (!blob || n != dc_policy_blob_len(h->cfg.mlp_hidden))
     return fail(h, DC_ERR_INVALID_ARG, "policy blob must hold 9 * mlp_hidden + 1 floats");
   DC_CUDA(h, cudaMemcpyAsync((void*)h->dev.policy, blob, n * sizeof(float), cudaMemcpyHostToDevice,
@@ -484,6 +491,7 @@ dc_status dc_policy_set_weights(dc_cache* h, const float* blob, size_t n) {
 
 dc_status dc_append(dc_cache* h, const void* k, const void* v, int n_tokens) {
   DC_CHECK_HANDLE(h);
+  if (h->graph) return fail(h, DC_ERR_STATE, "graph mode: only dc_step and its host forms until dc_set_graph_mode(h, 0)");
   if (n_tokens < 0 || (n_tokens > 0 && (!k || !v))) return fail(h, DC_ERR_INVALID_ARG, "bad append arguments");
   if (((uintptr_t)k | (uintptr_t)v) & 15) return fail(h, DC_ERR_INVALID_ARG, "k and v must be 16-byte aligned");
   if (n_tokens == 0) return DC_OK;
@@ -541,6 +549,36 @@ dc::FusedStep fused_args(dc_cache* h, const dc::Step& st, const void* q, float* 
   return fs;
 }
 
+// One device-counted step (graph mode): the append and the fused step with the
+// base arguments, which the kernels advance by the device's step count; the
+// host's mirror of the step state stays at the base until the mode ends.
+dc_status graph_step(dc_cache* h, const void* q, const void* k_new, const void* v_new, float* out, int budget) {
+  if (budget > 0 && budget != h->budget) return fail(h, DC_ERR_INVALID_ARG, "graph mode keeps the configured budget");
+  {
+    Phase ph(h, DC_PHASE_APPEND, 1);
+    dc::launch_append(h->dev, k_new, v_new, 1, h->n, h->gstep.p_newest, h->stream);
+  }
+  dc::FusedStep fs{};
+  fs.q = (const __nv_bfloat16*)q;
+  fs.out = out;
+  fs.do_evict = 1;
+  fs.B = h->budget;
+  fs.xstats = h->xstats;
+  fs.xo = h->xo;
+  fs.xsel = h->xsel;
+  fs.xflag = h->xflag;
+  fs.work = h->work;
+  fs.half_rows = h->xflag ? dc::fused_half_rows(h->dev, h->gstep.n, fs, h->num_sms, false) : 0;
+  fs.epoch = h->gepoch;
+  cudaError_t e;
+  {
+    Phase ph(h, DC_PHASE_ATTEND, 1);
+    e = dc::launch_fused_graph(h->maps, h->dev, h->gstep, fs, h->fpol, h->num_sms, h->stream);
+  }
+  if (e != cudaSuccess) return cuda_fail(h, e, "fused step (graph mode)");
+  return DC_OK;
+}
+
 // Whether a decode step over n tokens would split the fused grid's last wave.
 bool tail_split_applies(dc_cache* h, int n) {
   if (!h->xflag) return false;
@@ -556,6 +594,7 @@ bool tail_split_applies(dc_cache* h, int n) {
 
 dc_status dc_decode_step(dc_cache* h, const void* q, const void* k_new, const void* v_new, float* out) {
   DC_CHECK_HANDLE(h);
+  if (h->graph) return fail(h, DC_ERR_STATE, "graph mode: only dc_step and its host forms until dc_set_graph_mode(h, 0)");
   if (!q || !k_new || !v_new || !out) return fail(h, DC_ERR_INVALID_ARG, "NULL pointer");
   if (((uintptr_t)q | (uintptr_t)k_new | (uintptr_t)v_new) & 15)
     return fail(h, DC_ERR_INVALID_ARG, "q, k_new and v_new must be 16-byte aligned");
@@ -629,6 +668,7 @@ dc_status dc_step(dc_cache* h, const void* q, const void* k_new, const void* v_n
   if (((uintptr_t)q | (uintptr_t)k_new | (uintptr_t)v_new) & 15)
     return fail(h, DC_ERR_INVALID_ARG, "q, k_new and v_new must be 16-byte aligned");
   if (h->n + 1 > h->capacity) return fail(h, DC_ERR_CAPACITY, "decode step exceeds capacity");
+  if (h->graph) return graph_step(h, q, k_new, v_new, out, budget);
   const int n1 = h->n + 1;
   if (!use_fused(h, n1) || h->dev.seq_rows) {  // global mode: per-sequence selection after the rows
     dc_status s = dc_decode_step(h, q, k_new, v_new, out);
@@ -783,6 +823,7 @@ dc_status dc_engine(dc_cache* h, int n, int* engine) {
 dc_status dc_decode_step_host(dc_cache* h, const void* q, const void* k_new, const void* v_new,
                               float* out) {
   DC_CHECK_HANDLE(h);
+  if (h->graph) return fail(h, DC_ERR_STATE, "graph mode: only dc_step and its host forms until dc_set_graph_mode(h, 0)");
   if (!q || !k_new || !v_new || !out) return fail(h, DC_ERR_INVALID_ARG, "NULL pointer");
   const size_t R = h->dev.R, G = h->dev.G, d = h->dev.d;
   if (dc_status w = wait_async_copies(h); w != DC_OK) return w;
@@ -798,6 +839,7 @@ dc_status dc_decode_step_host(dc_cache* h, const void* q, const void* k_new, con
 
 dc_status dc_evict(dc_cache* h, int budget) {
   DC_CHECK_HANDLE(h);
+  if (h->graph) return fail(h, DC_ERR_STATE, "graph mode: only dc_step and its host forms until dc_set_graph_mode(h, 0)");
   if (!h->have_scores) return fail(h, DC_ERR_STATE, "evict needs the scores of a decode step");
   if (h->per_row) {
     // every row to its own budget (or all to `budget` when > 0)
@@ -832,6 +874,7 @@ dc_status dc_evict(dc_cache* h, int budget) {
 
 dc_status dc_full_decode(dc_cache* h, const void* q, float* out) {
   DC_CHECK_HANDLE(h);
+  if (h->graph) return fail(h, DC_ERR_STATE, "graph mode: only dc_step and its host forms until dc_set_graph_mode(h, 0)");
   if (!q || !out) return fail(h, DC_ERR_INVALID_ARG, "NULL pointer");
   if (h->n < 1) return fail(h, DC_ERR_STATE, "the cache is empty");
   if (h->per_row && std::any_of(h->hlen.begin(), h->hlen.end(), [&](int x) { return x != h->n; }))
@@ -862,6 +905,7 @@ dc_status dc_full_decode(dc_cache* h, const void* q, float* out) {
 
 dc_status dc_set_row_budgets(dc_cache* h, const int* budgets, int n) {
   DC_CHECK_HANDLE(h);
+  if (h->graph) return fail(h, DC_ERR_STATE, "graph mode: only dc_step and its host forms until dc_set_graph_mode(h, 0)");
   dc::Dev& p = h->dev;
   if (!budgets) {
     if (!h->per_row) return DC_OK;
@@ -894,6 +938,46 @@ dc_status dc_set_row_budgets(dc_cache* h, const int* budgets, int n) {
   p.rowlen = h->rowlen_dev;
   p.rowbudget = h->rowbudget_dev;
   h->per_row = true;
+  return DC_OK;
+}
+
+dc_status dc_set_graph_mode(dc_cache* h, int enable) {
+  DC_CHECK_HANDLE(h);
+  const int w = h->cfg.window;
+  if (enable) {
+    if (h->graph) return DC_OK;
+    if (h->per_row || h->dev.seq_rows || h->dev.scorer != 0 || h->cfg.budget_ratio > 0.f)
+      return fail(h, DC_ERR_STATE, "graph mode needs the policy scorer, one fixed budget for every row, per-row selection");
+    if (h->n != h->budget || h->n + 1 > h->capacity)
+      return fail(h, DC_ERR_STATE, "graph mode needs the steady state: the cache at its budget, one eviction per step");
+    if (h->steps < w) return fail(h, DC_ERR_STATE, "graph mode needs a full window of decode steps first");
+    // the window's queries of consecutive steps (no appends in between)
+    for (int k = 1; k <= w; ++k)
+      if (h->ring_pnew[(size_t)((h->steps - k) % w)] != (int)(h->seen - k))
+        return fail(h, DC_ERR_STATE, "graph mode needs the window's last steps to be consecutive decode steps");
+    if (!use_fused(h, h->n + 1)) return fail(h, DC_ERR_STATE, "graph mode runs on the fused engine only");
+    if (h->seen + (1ll << 30) > 0x7FFFFFFFll) return fail(h, DC_ERR_CAPACITY, "position counter too close to its limit");
+    if (!h->gcount_dev) DC_CUDA(h, dalloc(h, &h->gcount_dev, 2 * sizeof(int)));
+    DC_CUDA(h, cudaMemsetAsync(h->gcount_dev, 0, 2 * sizeof(int), h->stream));
+    h->gstep = begin_step(h);
+    h->gepoch = h->epoch + 1;
+    h->dev.gcount = h->gcount_dev;
+    h->graph = true;
+    return DC_OK;
+  }
+  if (!h->graph) return DC_OK;
+  int t = 0;
+  DC_CUDA(h, cudaStreamSynchronize(h->stream));
+  DC_CUDA(h, cudaMemcpy(&t, h->gcount_dev, sizeof t, cudaMemcpyDeviceToHost));
+  // the host mirror takes the t steps the device counted
+  const long long steps0 = h->steps, seen0 = h->seen;
+  for (long long k = (t > w ? t - w : 0); k < t; ++k) h->ring_pnew[(size_t)((steps0 + k) % w)] = (int)(seen0 + k);
+  h->seen += t;
+  h->steps += t;
+  h->epoch = h->gepoch + (unsigned)t - 1u;
+  h->have_scores = false;
+  h->dev.gcount = nullptr;
+  h->graph = false;
   return DC_OK;
 }
 

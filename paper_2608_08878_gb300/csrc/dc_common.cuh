@@ -57,6 +57,11 @@ struct Dev {
   // per-row mode: the order in which the fused engine's queue hands out rows
   // (longest first, so that no long row starts last); null: row order
   const int* roworder;
+  // device-counted steps (CUDA-graph replay): [0] steps taken since the mode
+  // was entered, added by the append and fused kernels to the host's base
+  // step arguments; [1] CTAs of the current fused launch that have finished
+  // (the last one advances [0]); null outside the mode
+  int* gcount;
   __nv_bfloat16* K;
   __nv_bfloat16* V;
   int* pos;

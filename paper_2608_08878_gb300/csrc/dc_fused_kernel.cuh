@@ -287,6 +287,9 @@ __device__ __forceinline__ Item read_item(volatile int* ring, int gr, volatile i
 // Dev::gpart (mass, squared mass, entropy-weighted mass and |v|, in the V
 // pass; the window sums come from the sequence's ring of pooled query terms);
 // features, scores and the selection are made per sequence afterwards.
+// GRAPH: device-counted steps: the step arguments are the host's base values
+// plus the number of steps taken since (Dev::gcount[0], advanced by the last
+// CTA to finish), so that a captured launch replays as the following steps.
 // PAIR: items are row pairs (rows 2w and 2w + 1) of at most kPairTiles tiles,
 // warpgroup w doing the whole of row 2w + w (its K and V tiles alternate with
 // the other row's in the ring), so that one row's merge, output and select
@@ -294,13 +297,26 @@ __device__ __forceinline__ Item read_item(volatile int* ring, int gr, volatile i
 // PERROW: rows of different lengths and budgets (Dev::rowlen, Dev::rowbudget;
 // FusedStep::B > 0 overrides every row's budget); the kernel writes each
 // row's new length after its selection. No half rows.
-template <int D, int G, bool LONG, bool FULL, bool HEUR, bool GLOB, bool PERROW, bool PAIR>
+template <int D, int G, bool LONG, bool FULL, bool HEUR, bool GLOB, bool PERROW, bool PAIR, bool GRAPH>
 __global__ void __launch_bounds__(kThreads, 1)
     fused_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmV,
                  const __grid_constant__ CUtensorMap tmK16, const __grid_constant__ CUtensorMap tmV16, Dev p,
                  Step st, FusedStep fs, FusedPolicy fp) {
   constexpr int GS = G - 1;  // heads whose logits wait in TMEM between the passes
   static_assert(!PAIR || (!LONG && !FULL && !HEUR && !GLOB && !PERROW), "row pairs: the plain step only");
+  static_assert(!GRAPH || (!FULL && !HEUR && !GLOB && !PERROW && !PAIR), "device-counted steps: the plain step");
+  if constexpr (GRAPH) {
+    // this launch's step: the base arguments advanced by the steps taken (in
+    // the steady state a step appends one token, so positions, window slots
+    // and the launch epoch all advance by one per step)
+    const int t = *reinterpret_cast<volatile int*>(p.gcount);
+    st.p_newest += t;
+    st.p_prev += t;
+    st.p_dep += t;
+    st.slot = (st.slot + t) % p.w;
+    st.slot_prev = (st.slot_prev + t) % p.w;
+    fs.epoch += (unsigned)t;
+  }
   using L = Smem<PAIR>;
   constexpr int OFF_STAGE = L::STAGE, OFF_Q = L::Q, OFF_P = L::P, OFF_A = L::A, OFF_W = L::W, OFF_AUX = L::AUX,
                 OFF_SC = L::SC, OFF_MISC = L::MISC;
@@ -1126,23 +1142,32 @@ __global__ void __launch_bounds__(kThreads, 1)
     tmem_dealloc(tmem, kTmemCols);
   }
   if (threadIdx.x == 0 && *abort) atomicOr(p.status, kStatusTimeout);
+  if constexpr (GRAPH) {
+    // the last CTA to finish (every CTA has read the counter by then)
+    // advances the step count for the next launch
+    if (threadIdx.x == 0 && atomicAdd(p.gcount + 1, 1) == (int)gridDim.x - 1) {
+      p.gcount[1] = 0;
+      __threadfence();
+      atomicAdd(p.gcount, 1);
+    }
+  }
 }
 
 
 template <int D, int G, bool LONG, bool FULL = false, bool HEUR = false, bool GLOB = false, bool PERROW = false,
-          bool PAIR = false>
+          bool PAIR = false, bool GRAPH = false>
 static cudaError_t launch_t(const FusedMaps& maps, const Dev& p, const Step& st, const FusedStep& fs,
                             const FusedPolicy& fp, int grid, cudaStream_t s) {
   constexpr int kSmemBytes = Smem<PAIR>::BYTES;
   static bool attr = false;
   if (!attr) {
-    cudaError_t e = cudaFuncSetAttribute(fused_kernel<D, G, LONG, FULL, HEUR, GLOB, PERROW, PAIR>,
+    cudaError_t e = cudaFuncSetAttribute(fused_kernel<D, G, LONG, FULL, HEUR, GLOB, PERROW, PAIR, GRAPH>,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes);
     if (e != cudaSuccess) return e;
     attr = true;
   }
   if (fs.half_rows == 0) {
-    fused_kernel<D, G, LONG, FULL, HEUR, GLOB, PERROW, PAIR>
+    fused_kernel<D, G, LONG, FULL, HEUR, GLOB, PERROW, PAIR, GRAPH>
         <<<grid, kThreads, kSmemBytes, s>>>(maps.k, maps.v, maps.k16, maps.v16, p, st, fs, fp);
     return cudaGetLastError();
   }
@@ -1158,8 +1183,8 @@ static cudaError_t launch_t(const FusedMaps& maps, const Dev& p, const Step& st,
   la[0].val.cooperative = 1;
   cfg.attrs = la;
   cfg.numAttrs = 1;
-  return cudaLaunchKernelEx(&cfg, fused_kernel<D, G, LONG, FULL, HEUR, GLOB, PERROW, PAIR>, maps.k, maps.v, maps.k16,
-                            maps.v16, p, st, fs, fp);
+  return cudaLaunchKernelEx(&cfg, fused_kernel<D, G, LONG, FULL, HEUR, GLOB, PERROW, PAIR, GRAPH>, maps.k, maps.v,
+                            maps.k16, maps.v16, p, st, fs, fp);
 }
 
 // One CTA per SM, or per row when rows are fewer; two per row when every row

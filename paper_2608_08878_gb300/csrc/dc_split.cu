@@ -47,7 +47,8 @@ __global__ void __launch_bounds__(256) append_kernel(Dev p, const uint4* __restr
   // xor offsets below vpr stay inside the pair's aligned lane group
   for (int off = 1; off < vpr; off <<= 1) ss += __shfl_xor_sync(0xffffffffu, ss, off);
   if (live && c == 0) {
-    p.pos[slot] = seen0 + t;
+    // device-counted steps: positions continue from the steps taken since
+    p.pos[slot] = seen0 + t + (p.gcount ? *reinterpret_cast<volatile int*>(p.gcount) : 0);
     p.vnorm[slot] = sqrtf(ss);
     p.SZ[slot] = make_float4(0.f, 0.f, 0.f, 0.f);
     if (p.acc) p.acc[slot] = 0.f;

@@ -30,7 +30,8 @@ EXPORTS = ["dc_config_default", "dc_cache_create", "dc_cache_destroy", "dc_polic
            "dc_copy_buffer", "dc_sync", "dc_last_error", "dc_phase_name", "dc_profile_enable",
            "dc_profile_read", "dc_step", "dc_step_host", "dc_step_host_async", "dc_engine", "dc_attend_noalloc",
            "dc_noalloc_last_error", "dc_pl_log_partition", "dc_gumbel_top_b", "dc_train_last_error",
-           "dc_set_row_budgets", "dc_get_row_lengths", "dc_wait_selftest", "dc_selftest_last_error"]
+           "dc_set_row_budgets", "dc_get_row_lengths", "dc_wait_selftest", "dc_selftest_last_error",
+           "dc_set_graph_mode"]
 PHASES = ["append", "attend", "stats", "score", "combine", "evict", "full"]
 
 
@@ -84,6 +85,7 @@ def lib():
             L.dc_noalloc_last_error.restype = C.c_char_p
             L.dc_full_decode.argtypes = [P, P, P]
             L.dc_set_row_budgets.argtypes = [P, P, I]
+            L.dc_set_graph_mode.argtypes = [P, I]
             L.dc_get_row_lengths.argtypes = [P, P, I]
             L.dc_pl_log_partition.argtypes = [P, I, I, I, C.c_float, P, P]
             L.dc_gumbel_top_b.argtypes = [P, P, I, I, I, C.c_float, P, P, P, P]
@@ -296,6 +298,11 @@ class DistillCache:
         """step_host without the final synchronisation (pinned host tensors;
         `out` is valid after sync())."""
         self._check(lib().dc_step_host_async(self._h, _ptr(q), _ptr(k_new), _ptr(v_new), _ptr(out), budget))
+
+    def set_graph_mode(self, enable: bool = True) -> None:
+        """Device-counted steps: a CUDA graph captured from one step() replays
+        as the following steps (see dc_set_graph_mode)."""
+        self._check(lib().dc_set_graph_mode(self._h, int(bool(enable))))
 
     def engine(self, n: int = 0) -> str:
         e = C.c_int()
