@@ -88,6 +88,11 @@ def test_null_handles_are_rejected():
     assert L.dc_append(None, None, None, 0) == dc.DC_ERR_INVALID_ARG
     assert L.dc_sync(None) == dc.DC_ERR_INVALID_ARG
     assert L.dc_policy_init(0, 0, None, 0) == dc.DC_ERR_INVALID_ARG
+    assert L.dc_set_graph_mode(None, 1) == dc.DC_ERR_INVALID_ARG
+    assert L.dc_step_host_async(None, None, None, None, None, 0) == dc.DC_ERR_INVALID_ARG
+    assert L.dc_set_row_budgets(None, None, 0) == dc.DC_ERR_INVALID_ARG
+    assert L.dc_wait_selftest(1000000, None, None) == dc.DC_ERR_INVALID_ARG
+    assert L.dc_wait_selftest(10, None, None) == dc.DC_ERR_INVALID_ARG
 
 
 def test_training_kernels_validate_before_touching_the_device():
