@@ -568,7 +568,7 @@ dc_status graph_step(dc_cache* h, const void* q, const void* k_new, const void* 
   fs.xsel = h->xsel;
   fs.xflag = h->xflag;
   fs.work = h->work;
-  fs.half_rows = h->xflag ? dc::fused_half_rows(h->dev, h->gstep.n, fs, h->num_sms, false) : 0;
+  fs.half_rows = h->xflag ? dc::fused_half_rows(h->dev, h->gstep.n, fs, h->num_sms) : 0;
   fs.epoch = h->gepoch;
   cudaError_t e;
   {

@@ -33,8 +33,8 @@ bool fused_pairs(const Dev& p, int n, int num_sms) {
   return waves2 * (2.0 * n + 410.0) < waves1 * (n + 350.0);
 }
 
-int fused_half_rows(const Dev& p, int n, const FusedStep& fs, int num_sms, bool allow_pairs) {
-  if (allow_pairs && fused_pairs(p, n, num_sms)) return 0;
+int fused_half_rows(const Dev& p, int n, const FusedStep& fs, int num_sms) {
+  if (fused_pairs(p, n, num_sms)) return 0;
   const int grid = p.R < num_sms ? p.R : num_sms, rem = p.R % grid;
   const int nT = (n + kTok - 1) / kTok;
   const bool ok = fs.xflag && fs.xstats && fs.xo && fs.xsel && nT >= 2 && (!fs.do_evict || fs.B >= n || fs.B == n - 1);

@@ -88,7 +88,7 @@ bool fused_pairs(const Dev& p, int n, int num_sms);
 // row when rows are at most half the SMs and at least 12 tiles long, else the
 // remainder of R over the grid when it is at most half the grid, else 0 (and 0
 // on row pairs).
-int fused_half_rows(const Dev& p, int n, const FusedStep& fs, int num_sms, bool allow_pairs = true);
+int fused_half_rows(const Dev& p, int n, const FusedStep& fs, int num_sms);
 
 cudaError_t launch_fused_step(const FusedMaps& maps, const Dev& p, const Step& st, const FusedStep& fs,
                               const FusedPolicy& fp, int num_sms, cudaStream_t s);
@@ -104,8 +104,8 @@ cudaError_t launch_fused_glob(const FusedMaps& maps, const Dev& p, const Step& s
 cudaError_t launch_fused_pair(const FusedMaps& maps, const Dev& p, const Step& st, const FusedStep& fs,
                               const FusedPolicy& fp, int num_sms, cudaStream_t s);
 // Device-counted steps (dc_fused_graph.cu): st and fs.epoch are base values
-// that the kernel advances by Dev::gcount[0]; whole rows or halves, policy
-// scorer, one eviction per step.
+// that the kernel advances by Dev::gcount[0]; whole rows, halves or row pairs
+// (as the plain step would take them), policy scorer, one eviction per step.
 cudaError_t launch_fused_graph(const FusedMaps& maps, const Dev& p, const Step& st, const FusedStep& fs,
                                const FusedPolicy& fp, int num_sms, cudaStream_t s);
 

@@ -8,11 +8,14 @@ namespace dc {
 
 cudaError_t launch_fused_graph(const FusedMaps& maps, const Dev& p, const Step& st, const FusedStep& fs,
                                const FusedPolicy& fp, int num_sms, cudaStream_t s) {
-  const int grid = fused_grid(p, fs, num_sms);
+  // row pairs where the plain step would take them (never with half rows)
+  const bool pairs = fs.half_rows == 0 && fused_pairs(p, st.n, num_sms);
+  const int grid = pairs ? (p.R / 2 < num_sms ? p.R / 2 : num_sms) : fused_grid(p, fs, num_sms);
   const bool lg = st.n > fused_onchip_tokens(p.G);
-#define DC_FUSED_LAUNCH(D, G)                                                                                \
-  return lg ? launch_t<D, G, true, false, false, false, false, false, true>(maps, p, st, fs, fp, grid, s)  \
-            : launch_t<D, G, false, false, false, false, false, false, true>(maps, p, st, fs, fp, grid, s)
+#define DC_FUSED_LAUNCH(D, G)                                                                                 \
+  return pairs ? launch_t<D, G, false, false, false, false, false, true, true>(maps, p, st, fs, fp, grid, s) \
+         : lg  ? launch_t<D, G, true, false, false, false, false, false, true>(maps, p, st, fs, fp, grid, s) \
+               : launch_t<D, G, false, false, false, false, false, false, true>(maps, p, st, fs, fp, grid, s)
   if (p.d == 128) {
     if (p.G == 4) DC_FUSED_LAUNCH(128, 4);
     if (p.G == 2) DC_FUSED_LAUNCH(128, 2);

@@ -304,7 +304,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                  Step st, FusedStep fs, FusedPolicy fp) {
   constexpr int GS = G - 1;  // heads whose logits wait in TMEM between the passes
   static_assert(!PAIR || (!LONG && !FULL && !HEUR && !GLOB && !PERROW), "row pairs: the plain step only");
-  static_assert(!GRAPH || (!FULL && !HEUR && !GLOB && !PERROW && !PAIR), "device-counted steps: the plain step");
+  static_assert(!GRAPH || (!FULL && !HEUR && !GLOB && !PERROW), "device-counted steps: the plain step");
   if constexpr (GRAPH) {
     // this launch's step: the base arguments advanced by the steps taken (in
     // the steady state a step appends one token, so positions, window slots

@@ -50,14 +50,17 @@ def _rows_for_sms(per_sm_times, extra):
     return (per_sm_times * sms + extra) // 8
 
 
-@pytest.mark.parametrize("case", ["few rows", "few rows in halves", "last wave in halves", "long rows"])
+@pytest.mark.parametrize("case", ["few rows", "few rows in halves", "last wave in halves", "long rows", "row pairs"])
 def test_graph_mode_steps_equal_ordinary_steps(case):
     import torch
     from paper_2608_08878_gb300 import synth_device
     batch, prompt = {"few rows": (1, 600), "few rows in halves": (1, 2000),
-                     "last wave in halves": (_rows_for_sms(1, 8), 600), "long rows": (1, 9000)}[case]
+                     "last wave in halves": (_rows_for_sms(1, 8), 600), "long rows": (1, 9000),
+                     "row pairs": (_rows_for_sms(4, 0), 600)}[case]
     wl = synth.MISTRAL_1L.with_(batch=batch, prompt_len=prompt, budget=prompt, window=4)
     a, b = _pair(wl)
+    if case == "row pairs":
+        assert a.engine(prompt + 1) == "fused-pairs"
     s = 0
     for _ in range(wl.window + 1):  # a full window of decode steps first
         q, kn, vn = synth_device.step_inputs(wl, s)
@@ -85,11 +88,12 @@ def test_graph_mode_steps_equal_ordinary_steps(case):
     _same_cache(a, b)
 
 
-@pytest.mark.parametrize("prompt", [700, 2000])  # whole rows; rows in halves (a cooperative launch)
-def test_graph_mode_replays_a_captured_step_as_the_next_steps(prompt):
+@pytest.mark.parametrize("rows_per_sm,prompt", [(0, 700), (0, 2000), (4, 700)])  # whole rows; halves
+def test_graph_mode_replays_a_captured_step_as_the_next_steps(rows_per_sm, prompt):  # (cooperative); pairs
     import torch
     from paper_2608_08878_gb300 import synth_device
-    wl = synth.MISTRAL_1L.with_(prompt_len=prompt, budget=prompt, window=4)
+    batch = _rows_for_sms(rows_per_sm, 0) if rows_per_sm else 1
+    wl = synth.MISTRAL_1L.with_(batch=batch, prompt_len=prompt, budget=prompt, window=4)
     stream = torch.cuda.Stream()
     with torch.cuda.stream(stream):
         a, b = _pair(wl, stream=stream)
