@@ -555,3 +555,53 @@ def test_global_mode_pooled_features_brute_force():
             kb, vb = seq.kv_bits(r)
             assert np.array_equal(kb, np.stack(K[r])) and np.array_equal(vb, np.stack(V[r]))
         pos = kept_pos
+
+
+# --------------------------------------------------------------------------
+# Invariants on random rows (property-based)
+# --------------------------------------------------------------------------
+
+def test_step_invariants_on_random_rows():
+    """Invariants that hold for any input, checked on random small rows over
+    several steps with evictions: each step's alpha sums to 1 (alpha_mode 0);
+    sigma lies in [0, alpha (1 - alpha)] (the variance of values in [0, 1] with
+    that mean, population form); H_i lies in [0, ln of the longest row the
+    window saw]; pos_i in [0, 1]; every output coordinate lies within the value
+    rows' range (a convex combination); cumulative alpha (mode 1) is
+    non-negative and sums to at most the number of steps."""
+    hyp = pytest.importorskip("hypothesis")
+    st = pytest.importorskip("hypothesis.strategies")
+
+    @hyp.settings(max_examples=60, deadline=None)
+    @hyp.given(n=st.integers(1, 160), G=st.sampled_from([1, 2, 4]), w=st.integers(1, 6), steps=st.integers(1, 7),
+               alpha_mode=st.integers(0, 1), seed=st.integers(0, 2 ** 31 - 1), data=st.data())
+    def run(n, G, w, steps, alpha_mode, seed, data):
+        rng = np.random.default_rng(seed)
+        d = 64
+        B = data.draw(st.integers(1, n + steps))
+        row = oracle.OracleRow(d, G, w, alpha_mode, n + steps + 1)
+        k = rand_bits(rng, n, d, scale=2.0)
+        v = rand_bits(rng, n, d)
+        row.append(k, v)
+        blob = synth.policy_weights(0, 32)
+        longest = n
+        for s in range(steps):
+            q = rand_bits(rng, G, d, scale=1.5)
+            kn, vn = rand_bits(rng, 1, d, scale=2.0)[0], rand_bits(rng, 1, d)[0]
+            vrows = np.concatenate([widen(row.kv_bits()[1]), widen(vn)[None]], axis=0) if len(row) else widen(vn)[None]
+            res = row.step(q, kn, vn, blob, 32, 1)
+            m = len(res["pos"])
+            longest = max(longest, m)
+            alpha, sigma, H, pos = res["feat"][:, 0], res["feat"][:, 2], res["feat"][:, 3], res["feat"][:, 4]
+            if alpha_mode == 0:
+                assert abs(alpha.sum() - 1.0) < 1e-12
+                assert np.all(sigma >= -1e-15) and np.all(sigma <= alpha * (1 - alpha) + 1e-12)
+            else:
+                assert np.all(alpha >= -1e-15) and alpha.sum() <= s + 1 + 1e-9
+            assert np.all(H >= -1e-12) and np.all(H <= math.log(longest) + 1e-12)
+            assert np.all(pos >= 0) and np.all(pos <= 1)
+            lo, hi = vrows.min(axis=0), vrows.max(axis=0)
+            assert np.all(res["o"] >= lo - 1e-12) and np.all(res["o"] <= hi + 1e-12)
+            row.evict(B)
+
+    run()
