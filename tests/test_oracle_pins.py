@@ -605,3 +605,43 @@ def test_step_invariants_on_random_rows():
             row.evict(B)
 
     run()
+
+
+def test_global_mode_invariants_on_random_sequences():
+    """The same invariants in the global token mode, where a token's alpha,
+    sigma and H pool every (row, head) pair of the sequence: alpha sums to 1,
+    sigma in [0, alpha (1 - alpha)], 0 <= H <= ln n, pos in [0, 1], |v| the
+    mean of the rows' value norms, each row's output inside its value range."""
+    hyp = pytest.importorskip("hypothesis")
+    st = pytest.importorskip("hypothesis.strategies")
+
+    @hyp.settings(max_examples=30, deadline=None)
+    @hyp.given(R=st.integers(1, 4), n=st.integers(1, 80), G=st.sampled_from([1, 2, 4]), w=st.integers(1, 4),
+               steps=st.integers(1, 5), seed=st.integers(0, 2 ** 31 - 1), data=st.data())
+    def run(R, n, G, w, steps, seed, data):
+        rng = np.random.default_rng(seed)
+        d = 64
+        B = data.draw(st.integers(1, n + steps))
+        seq = oracle.OracleSeq(R, d, G, w, 0, n + steps + 1)
+        seq.append(rand_bits(rng, R, n, d, scale=2.0), rand_bits(rng, R, n, d))
+        blob = synth.policy_weights(0, 32)
+        longest = n
+        for _ in range(steps):
+            q = rand_bits(rng, R, G, d, scale=1.5)
+            kn, vn = rand_bits(rng, R, d, scale=2.0), rand_bits(rng, R, d)
+            vrows = [np.concatenate([widen(seq.kv_bits(r)[1]), widen(vn[r])[None]], axis=0) for r in range(R)]
+            res = seq.step(q, kn, vn, blob, 32, 1)
+            longest = max(longest, len(res["pos"]))
+            alpha, vnorm, sigma, H, pos = (res["feat"][:, c] for c in range(5))
+            assert abs(alpha.sum() - 1.0) < 1e-12
+            assert np.all(sigma >= -1e-15) and np.all(sigma <= alpha * (1 - alpha) + 1e-12)
+            assert np.all(H >= -1e-12) and np.all(H <= math.log(longest) + 1e-12)
+            assert np.all(pos >= 0) and np.all(pos <= 1)
+            np.testing.assert_allclose(vnorm, np.mean([np.linalg.norm(vr, axis=1) for vr in vrows], axis=0),
+                                       rtol=1e-12)
+            for r in range(R):
+                lo, hi = vrows[r].min(axis=0), vrows[r].max(axis=0)
+                assert np.all(res["o"][r] >= lo - 1e-12) and np.all(res["o"][r] <= hi + 1e-12)
+            seq.evict(B)
+
+    run()
