@@ -34,7 +34,6 @@
  *     one particular step: replaying it repeats that step's arguments. In
  *     graph mode (dc_set_graph_mode) dc_step counts steps on the device
  *     instead, and a captured dc_step replays as the following decode steps.
- *     (dc_attend_noalloc keeps no state and may be captured and replayed.)
  */
 #ifndef DISTILLCACHE_H
 #define DISTILLCACHE_H
@@ -299,11 +298,12 @@ dc_status dc_profile_read(dc_cache* h, double* ms, long long* launches);
 dc_status dc_sync(dc_cache* h);
 
 /* Full-cache decode attention that allocates no device memory, for callers
- * that cannot allocate: code running while a stream is being captured into a
- * CUDA graph, runtimes that reserve all device memory up front, and paths that
- * cannot afford the implicit synchronisation of cudaMalloc/cudaFree. The
- * paper has no counterpart; it is the dc_full_decode computation on
- * caller-provided buffers, with no handle.
+ * that cannot call cudaMalloc: runtimes that reserve all device memory up
+ * front and allow no allocation afterwards (a fixed-footprint serving
+ * process), and paths that cannot afford the implicit device synchronisation
+ * of cudaMalloc/cudaFree. The handle-based calls do not suit them, because
+ * dc_cache_create allocates. The paper has no counterpart; this is the
+ * dc_full_decode computation on caller-provided buffers, with no handle.
  *   q:   bf16 [rows][group][head_dim]; k, v: bf16 [rows][n][head_dim]
  *        (16-byte aligned); out: fp32 [rows][group][head_dim]; all device.
  *   stream: cudaStream_t (NULL: legacy default stream).
@@ -314,10 +314,11 @@ dc_status dc_sync(dc_cache* h);
  * shapes (head_dim 64 or 128, group 1, 2, 4 or 8, 1 <= rows <= 65535, n >= 1).
  * The first call on a device looks up the array's device address (once per
  * device, with that device current); make that first call before any stream
- * capture. Every call shares the array and overwrites the part it uses, so
- * nothing carries over between calls, but calls that overlap on the GPU (two
- * streams, or two host threads) race on it and must be serialised by the
- * caller. Asynchronous on `stream`; dc_noalloc_last_error() describes a
+ * capture. Every call shares the array, which keeps the last call's
+ * contents; nothing in it has to start at zero, because each call writes every
+ * partial result before it reads it. Calls that overlap on the GPU (two
+ * streams, or two host threads) race on the array and must be serialised by
+ * the caller. Asynchronous on `stream`; dc_noalloc_last_error() describes a
  * failure. */
 dc_status dc_attend_noalloc(const void* q, const void* k, const void* v, int rows, int n,
                             int head_dim, int group, float* out, void* stream);

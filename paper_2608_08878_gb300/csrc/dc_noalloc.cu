@@ -2,9 +2,7 @@
 // allocate device memory: the split-K partial results live in a fixed,
 // file-scope device array instead of buffers allocated by the library.
 //
-// Which callers cannot allocate: code that runs while a CUDA stream is being
-// captured into a graph (cudaMalloc is not a stream operation and is not
-// permitted during capture), runtimes that reserve all device memory up
+// Which callers cannot allocate: runtimes that reserve all device memory up
 // front and forbid further allocation (fixed-footprint serving processes),
 // and latency-critical paths where an implicit device synchronisation from
 // cudaMalloc/cudaFree is not acceptable. None of the handle-based calls fit
