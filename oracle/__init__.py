@@ -17,12 +17,17 @@ import numpy as np
 _HERE = os.path.dirname(os.path.abspath(__file__))
 _SRC = os.path.join(_HERE, "dc_oracle.c")
 _LIB_PATH = os.path.join(_HERE, "libdc_oracle.so")
+# A separately compiled copy of the oracle to load instead (the mutation tests
+# load copies with a planted mistake); never set outside the tests.
+_LIB_OVERRIDE = os.environ.get("DC_ORACLE_LIB")
 _lib = None
 _lock = threading.Lock()
 
 
 def build(force: bool = False) -> str:
     """Compiles the oracle with gcc (plain C11, -O2, no fast-math)."""
+    if _LIB_OVERRIDE:
+        return _LIB_OVERRIDE
     if force or not os.path.exists(_LIB_PATH) or os.path.getmtime(_LIB_PATH) < max(
             os.path.getmtime(_SRC), os.path.getmtime(os.path.join(_HERE, "dc_oracle.h"))):
         tmp = _LIB_PATH + f".tmp{os.getpid()}"
@@ -36,8 +41,7 @@ def lib():
     global _lib
     with _lock:
         if _lib is None:
-            build()
-            L = C.CDLL(_LIB_PATH)
+            L = C.CDLL(build())
             P = C.c_void_p
             L.dco_row_new.restype = P
             L.dco_row_new.argtypes = [C.c_int] * 5

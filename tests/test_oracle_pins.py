@@ -73,6 +73,15 @@ def test_entropy_uniform_and_one_hot():
     o, Hq2 = oracle.attend(q, bits(k2), v)
     assert np.all(Hq2 < 1e-20)
     np.testing.assert_allclose(o[0], widen(v[7]), rtol=1e-20, atol=1e-20)
+    # logit 800 above the rest: the other weights underflow to exactly 0 in
+    # fp64, and their terms 0 ln 0 count as 0 (the limit), so H is exactly 0
+    k3 = np.zeros((n, d), dtype=np.float32)
+    k3[7] = 100.0
+    a3 = softmax_rows(q, bits(k3))
+    assert np.count_nonzero(a3[0]) == 1
+    _, Hq3 = oracle.attend(q, bits(k3), v)
+    np.testing.assert_array_equal(Hq3, [scipy.stats.entropy(a3[h]) for h in range(2)])
+    np.testing.assert_array_equal(Hq3, 0.0)
 
 
 # --------------------------------------------------------------------------
@@ -107,6 +116,49 @@ def test_step_features_against_libraries():
     np.testing.assert_allclose(f[:, 3], (a * Hq[:, None]).sum(0) / a.sum(0), rtol=1e-10)
     np.testing.assert_allclose(f[:, 4], np.arange(T + 1) / T, rtol=1e-15)                   # pos
     np.testing.assert_array_equal(r["pos"], np.arange(T + 1))
+
+
+def test_step_after_eviction_against_libraries():
+    """A step after an eviction that removed tokens from the middle of the row:
+    the survivors are a set the test picks (through the scores it passes), so
+    every expected value is computed here from the test's own key/value arrays,
+    never from the oracle's bookkeeping. Attention runs over the survivors plus
+    the new token; pos_i divides the absolute position (tokens seen) by the
+    newest one; with w = 2 the window sums pool the step before the eviction
+    (over all T + 1 tokens) and this one, matched by position."""
+    rng = np.random.default_rng(17)
+    d, G, T = 32, 4, 30
+    row = oracle.OracleRow(d, G, window=2, alpha_mode=0, capacity=64)
+    kp, vp = rand_bits(rng, T, d), rand_bits(rng, T, d)
+    row.append(kp, vp)
+    mlp, H, ln = _mlp()
+    q1, k1, v1 = rand_bits(rng, G, d), rand_bits(rng, d), rand_bits(rng, d)
+    row.step(q1, k1, v1, mlp, H, ln)
+    K1, V1 = np.concatenate([kp, k1[None]]), np.concatenate([vp, v1[None]])   # positions 0..T
+    keep = np.sort(rng.choice(T + 1, size=11, replace=False))
+    scores = np.full(T + 1, -1.0, dtype=np.float32)
+    scores[keep] = 1.0 + np.arange(keep.size, dtype=np.float32)
+    assert row.evict(keep.size, scores) == keep.size
+    q2, k2, v2 = rand_bits(rng, G, d), rand_bits(rng, d), rand_bits(rng, d)
+    r = row.step(q2, k2, v2, mlp, H, ln)
+    pos = np.append(keep, T + 1)
+    np.testing.assert_array_equal(r["pos"], pos)
+    K2, V2 = np.concatenate([K1[keep], k2[None]]), np.concatenate([V1[keep], v2[None]])
+    np.testing.assert_allclose(r["o"], sdpa_gqa(q2, K2, V2), rtol=1e-12, atol=1e-12)
+    a1, a2 = softmax_rows(q1, K1), softmax_rows(q2, K2)                      # [G][T+1], [G][n]
+    H1 = np.array([scipy.stats.entropy(a1[h]) for h in range(G)])
+    H2 = np.array([scipy.stats.entropy(a2[h]) for h in range(G)])
+    f = r["feat"]
+    at = torch.from_numpy(a2)
+    np.testing.assert_allclose(f[:, 0], at.mean(0).numpy(), rtol=1e-12)                    # alpha
+    np.testing.assert_allclose(f[:, 1], np.linalg.norm(widen(V2), axis=1), rtol=1e-13)    # |v|
+    np.testing.assert_allclose(f[:, 2], at.var(0, unbiased=False).numpy(), rtol=1e-9, atol=1e-20)
+    Z = a2.sum(0)
+    S = (a2 * H2[:, None]).sum(0)
+    Z[:-1] += a1[:, keep].sum(0)                                # the survivors were attended before
+    S[:-1] += (a1[:, keep] * H1[:, None]).sum(0)
+    np.testing.assert_allclose(f[:, 3], S / Z, rtol=1e-10)                                  # H_i
+    np.testing.assert_allclose(f[:, 4], pos / (T + 1), rtol=1e-15)                           # pos
 
 
 def test_mlp_equals_torch_sequential():
@@ -514,14 +566,18 @@ def test_global_mode_with_one_row_is_the_row_oracle():
         assert all(np.array_equal(x, y) for x, y in zip(row.kv_bits(), seq.kv_bits(0)))
 
 
-def test_global_mode_pooled_features_brute_force():
+@pytest.mark.parametrize("alpha_mode", [0, 1])
+def test_global_mode_pooled_features_brute_force(alpha_mode):
     """alpha, sigma, |v|, H and pos of a 3-row sequence recomputed from torch
-    softmax over every row's heads, stacked, over a 3-step window; every row
-    pruned to the same survivors, which are the sequence's top-B."""
+    softmax over every row's heads, stacked, over a 3-step window, and the
+    window sums without the latest step; in alpha_mode 1 alpha is the pooled
+    mass summed over the steps since the token's insertion. Every row pruned to
+    the same survivors, which are the sequence's top-B."""
     rng = np.random.default_rng(41)
     R, d, G, T, w, B = 3, 16, 2, 25, 3, 20
     blob = synth.policy_weights(6, 32)
-    seq = oracle.OracleSeq(R, d, G, w, 0, T + 10)
+    seq = oracle.OracleSeq(R, d, G, w, alpha_mode, T + 10)
+    acc = {}  # position -> pooled mass summed over the steps since insertion
     K = {r: list(rand_bits(rng, T, d)) for r in range(R)}
     V = {r: list(rand_bits(rng, T, d)) for r in range(R)}
     seq.append(np.stack([np.stack(K[r]) for r in range(R)]), np.stack([np.stack(V[r]) for r in range(R)]))
@@ -541,9 +597,17 @@ def test_global_mode_pooled_features_brute_force():
         vnorm = np.mean([np.linalg.norm(widen(np.stack(V[r])), axis=1) for r in range(R)], axis=0)
         S = np.array([sum(h[p][1] for h in hist if p in h) for p in pos])
         Z = np.array([sum(h[p][0] for h in hist if p in h) for p in pos])
-        want = np.stack([a.mean(0), vnorm, a.var(0), np.where(Z > 0, S / Z, 0.0),
+        for i, p in enumerate(pos):
+            acc[p] = acc.get(p, 0.0) + a[:, i].mean()
+        alpha = np.array([acc[p] for p in pos]) if alpha_mode else a.mean(0)
+        want = np.stack([alpha, vnorm, a.var(0), np.where(Z > 0, S / Z, 0.0),
                          np.array(pos) / max(pos[-1], 1)], axis=1)
         np.testing.assert_allclose(res["feat"], want, rtol=1e-11, atol=1e-14)
+        Sp, Zp = seq.window_sums_prior()
+        np.testing.assert_allclose(Sp, [sum(h[p][1] for h in hist[:-1] if p in h) for p in pos], rtol=1e-12,
+                                   atol=1e-15)
+        np.testing.assert_allclose(Zp, [sum(h[p][0] for h in hist[:-1] if p in h) for p in pos], rtol=1e-12,
+                                   atol=1e-15)
         sc = res["score"].astype(np.float32)
         keep = np.sort(np.lexsort((np.array(pos), -sc.astype(np.float64)))[:B])
         seq.evict(B, sc)
