@@ -130,12 +130,21 @@ def attend_noalloc(q, k, v, out=None, stream=None):
     """Full-cache decode attention with no device allocation by the library:
     q [rows][group][d], k/v [rows][n][d] bf16 CUDA tensors -> out fp32."""
     import torch
+    if not isinstance(q, torch.Tensor) or q.dim() != 3 or not isinstance(k, torch.Tensor) or k.dim() != 3:
+        raise DCError(DC_ERR_INVALID_ARG, "q must be [rows][group][head_dim] and k, v [rows][n][head_dim]")
     rows, group, d = q.shape
     n = k.shape[1]
+    if k.shape[0] != rows or k.shape[2] != d:
+        raise DCError(DC_ERR_INVALID_ARG, f"k has shape {tuple(k.shape)}, expected ({rows}, n, {d})")
+    dev = q.device.index if q.is_cuda else None
+    pq = _arg(q, "q", torch.bfloat16, rows * group * d, device=dev)
+    pk = _arg(k, "k", torch.bfloat16, rows * n * d, device=dev)
+    pv = _arg(v, "v", torch.bfloat16, rows * n * d, device=dev)
     if out is None:
         out = torch.empty((rows, group, d), dtype=torch.float32, device=q.device)
+    po = _arg(out, "out", torch.float32, rows * group * d, device=dev)
     s = (stream or torch.cuda.current_stream()).cuda_stream
-    st = lib().dc_attend_noalloc(q.data_ptr(), k.data_ptr(), v.data_ptr(), rows, n, d, group, out.data_ptr(), s)
+    st = lib().dc_attend_noalloc(pq, pk, pv, rows, n, d, group, po, s)
     if st != DC_OK:
         raise DCError(st, lib().dc_noalloc_last_error().decode())
     return out
@@ -159,11 +168,16 @@ def pl_log_partition(scores, B: int, tau: float = 1.0, out=None, stream=None):
     """Exact log Z of the Plackett-Luce distribution over size-B subsets for
     each row of scores (fp32 CUDA tensor [rows][L]) -> fp32 [rows] (App. C)."""
     import torch
+    if not isinstance(scores, torch.Tensor) or scores.dim() != 2:
+        raise DCError(DC_ERR_INVALID_ARG, "scores must be a [rows][L] tensor")
     rows, L = scores.shape
+    dev = scores.device.index if scores.is_cuda else None
+    ps = _arg(scores, "scores", torch.float32, rows * L, device=dev)
     if out is None:
         out = torch.empty(rows, dtype=torch.float32, device=scores.device)
+    po = _arg(out, "out", torch.float32, rows, device=dev)
     s = (stream or torch.cuda.current_stream()).cuda_stream
-    st = lib().dc_pl_log_partition(scores.data_ptr(), rows, L, B, tau, out.data_ptr(), s)
+    st = lib().dc_pl_log_partition(ps, rows, L, B, tau, po, s)
     if st != DC_OK:
         raise DCError(st, lib().dc_train_last_error().decode())
     return out
@@ -174,7 +188,14 @@ def gumbel_top_b(scores, gumbel, B: int, tau: float = 1.0, with_logp: bool = Tru
     the B kept indices ascending (int32 [rows][B]) and, if with_logp, the
     subset's Plackett-Luce log-probability (fp32 [rows]) (App. C)."""
     import torch
+    if not isinstance(scores, torch.Tensor) or scores.dim() != 2:
+        raise DCError(DC_ERR_INVALID_ARG, "scores must be a [rows][L] tensor")
     rows, L = scores.shape
+    dev = scores.device.index if scores.is_cuda else None
+    _arg(scores, "scores", torch.float32, rows * L, device=dev)
+    _arg(gumbel, "gumbel", torch.float32, rows * L, device=dev)
+    if B < 1:
+        raise DCError(DC_ERR_INVALID_ARG, "B must be >= 1")
     idx = torch.empty((rows, B), dtype=torch.int32, device=scores.device)
     logp = torch.empty(rows, dtype=torch.float32, device=scores.device) if with_logp else None
     logz = torch.empty(rows, dtype=torch.float32, device=scores.device) if with_logp else None
@@ -201,6 +222,29 @@ def head_level_hybrid_budgets(rows: int, context: int, full_rows, overall_ratio:
 
 def _ptr(t) -> int:
     return 0 if t is None else int(t.data_ptr())
+
+
+def _arg(t, name: str, dtype, numel: int, cuda: bool = True, device: int | None = None) -> int:
+    """The address of tensor argument `name` after checking what the C ABI
+    assumes of it: device memory (or host memory for the *_host calls) on the
+    expected device, the element type, a dense row-major layout and the element
+    count. The library sees only the pointer, so a tensor that fails one of
+    these would be read or written out of bounds (on the GPU: a memory fault).
+    Raises DCError(DC_ERR_INVALID_ARG) before anything is enqueued."""
+    import torch
+    if not isinstance(t, torch.Tensor):
+        raise DCError(DC_ERR_INVALID_ARG, f"{name} must be a torch tensor")
+    if t.is_cuda != cuda:
+        raise DCError(DC_ERR_INVALID_ARG, f"{name} must be a {'CUDA' if cuda else 'host (CPU)'} tensor")
+    if cuda and device is not None and t.device.index != device:
+        raise DCError(DC_ERR_INVALID_ARG, f"{name} is on cuda:{t.device.index}, expected cuda:{device}")
+    if t.dtype != dtype:
+        raise DCError(DC_ERR_INVALID_ARG, f"{name} must be {dtype}, got {t.dtype}")
+    if not t.is_contiguous():
+        raise DCError(DC_ERR_INVALID_ARG, f"{name} must be contiguous (dense row-major)")
+    if t.numel() != numel:
+        raise DCError(DC_ERR_INVALID_ARG, f"{name} has {t.numel()} elements, expected {numel}")
+    return int(t.data_ptr())
 
 
 class DistillCache:
@@ -239,6 +283,7 @@ class DistillCache:
         self.group = self.q_heads // kv_heads
         self.rows = layers * batch * kv_heads
         self.mlp_hidden = mlp_hidden
+        self.device = torch.cuda.current_device()
 
     # -- lifetime ----------------------------------------------------------
     def close(self) -> None:
@@ -267,37 +312,54 @@ class DistillCache:
         blob = np.ascontiguousarray(blob, dtype=np.float32)
         self._check(lib().dc_policy_set_weights(self._h, blob.ctypes.data_as(C.c_void_p), blob.size))
 
+    def _step_args(self, q, k_new, v_new, out, cuda: bool = True):
+        """Addresses of one decode step's tensors: q bf16 [layers][batch][q_heads][d],
+        k_new, v_new bf16 [layers][batch][kv_heads][d], out fp32 like q."""
+        import torch
+        nq, nkv = self.layers * self.batch * self.q_heads * self.head_dim, self.rows * self.head_dim
+        dev = self.device if cuda else None
+        return (_arg(q, "q", torch.bfloat16, nq, cuda, dev), _arg(k_new, "k_new", torch.bfloat16, nkv, cuda, dev),
+                _arg(v_new, "v_new", torch.bfloat16, nkv, cuda, dev), _arg(out, "out", torch.float32, nq, cuda, dev))
+
+    def _out_like(self, q, out):
+        import torch
+        if out is None and isinstance(q, torch.Tensor):
+            out = torch.empty(q.shape, dtype=torch.float32, device=q.device)
+        return out
+
     def append(self, k, v) -> None:
         """k, v: bf16 CUDA tensors [layers][batch][kv_heads][T][head_dim]."""
+        import torch
+        if not isinstance(k, torch.Tensor) or not isinstance(v, torch.Tensor) or k.shape != v.shape:
+            raise DCError(DC_ERR_INVALID_ARG, "k and v must be tensors of the same shape")
         T = int(k.shape[-2]) if k.numel() else 0
-        self._check(lib().dc_append(self._h, _ptr(k), _ptr(v), T))
+        n = self.rows * T * self.head_dim
+        pk = _arg(k, "k", torch.bfloat16, n, device=self.device)
+        pv = _arg(v, "v", torch.bfloat16, n, device=self.device)
+        self._check(lib().dc_append(self._h, pk, pv, T))
 
     def decode_step(self, q, k_new, v_new, out=None):
-        import torch
-        if out is None:
-            out = torch.empty(q.shape, dtype=torch.float32, device=q.device)
-        self._check(lib().dc_decode_step(self._h, _ptr(q), _ptr(k_new), _ptr(v_new), _ptr(out)))
+        out = self._out_like(q, out)
+        self._check(lib().dc_decode_step(self._h, *self._step_args(q, k_new, v_new, out)))
         return out
 
     def decode_step_host(self, q, k_new, v_new, out) -> None:
         """Host (preferably pinned) tensors; synchronises before returning."""
-        self._check(lib().dc_decode_step_host(self._h, _ptr(q), _ptr(k_new), _ptr(v_new), _ptr(out)))
+        self._check(lib().dc_decode_step_host(self._h, *self._step_args(q, k_new, v_new, out, cuda=False)))
 
     def step(self, q, k_new, v_new, out=None, budget: int = 0):
         """decode_step + evict (one kernel on the fused engine)."""
-        import torch
-        if out is None:
-            out = torch.empty(q.shape, dtype=torch.float32, device=q.device)
-        self._check(lib().dc_step(self._h, _ptr(q), _ptr(k_new), _ptr(v_new), _ptr(out), budget))
+        out = self._out_like(q, out)
+        self._check(lib().dc_step(self._h, *self._step_args(q, k_new, v_new, out), budget))
         return out
 
     def step_host(self, q, k_new, v_new, out, budget: int = 0) -> None:
-        self._check(lib().dc_step_host(self._h, _ptr(q), _ptr(k_new), _ptr(v_new), _ptr(out), budget))
+        self._check(lib().dc_step_host(self._h, *self._step_args(q, k_new, v_new, out, cuda=False), budget))
 
     def step_host_async(self, q, k_new, v_new, out, budget: int = 0) -> None:
         """step_host without the final synchronisation (pinned host tensors;
         `out` is valid after sync())."""
-        self._check(lib().dc_step_host_async(self._h, _ptr(q), _ptr(k_new), _ptr(v_new), _ptr(out), budget))
+        self._check(lib().dc_step_host_async(self._h, *self._step_args(q, k_new, v_new, out, cuda=False), budget))
 
     def set_graph_mode(self, enable: bool = True) -> None:
         """Device-counted steps: a CUDA graph captured from one step() replays
@@ -314,9 +376,11 @@ class DistillCache:
 
     def full_decode(self, q, out=None):
         import torch
-        if out is None:
-            out = torch.empty(q.shape, dtype=torch.float32, device=q.device)
-        self._check(lib().dc_full_decode(self._h, _ptr(q), _ptr(out)))
+        out = self._out_like(q, out)
+        nq = self.layers * self.batch * self.q_heads * self.head_dim
+        pq = _arg(q, "q", torch.bfloat16, nq, device=self.device)
+        po = _arg(out, "out", torch.float32, nq, device=self.device)
+        self._check(lib().dc_full_decode(self._h, pq, po))
         return out
 
     def set_row_budgets(self, budgets) -> None:

@@ -136,3 +136,73 @@ def test_header_compiles_as_c_and_matches_the_binding(tmp_path):
     size, blob, window, hidden = (int(x) for x in out[:4])
     assert (size, blob, window, hidden) == (C.sizeof(dc.dc_config), 9 * 128 + 1, 64, 128)
     assert [int(x) for x in out[4:]] == [getattr(dc.dc_config, f).offset for f in fields]
+
+
+def _unopened_cache(layers=2, batch=1, kv_heads=2, q_heads=4, head_dim=64):
+    """A DistillCache object with the shape bookkeeping of a real one but no
+    library handle: the binding's argument checks run before any library call,
+    so they can be exercised without a GPU."""
+    c = object.__new__(dc.DistillCache)
+    c._h = None
+    c.layers, c.batch, c.kv_heads, c.q_heads, c.head_dim = layers, batch, kv_heads, q_heads, head_dim
+    c.group, c.rows, c.device = q_heads // kv_heads, layers * batch * kv_heads, 0
+    return c
+
+
+def test_binding_rejects_tensors_that_do_not_match_the_abi():
+    """Tensors passed by pointer are checked for device or host memory, element
+    type, dense layout and element count, with DC_ERR_INVALID_ARG, before the
+    library is called (a wrong one would be read or written out of bounds)."""
+    import torch
+    c = _unopened_cache()
+    q = torch.zeros((2, 1, 4, 64), dtype=torch.bfloat16)
+    kn = torch.zeros((2, 1, 2, 64), dtype=torch.bfloat16)
+    out = torch.zeros((2, 1, 4, 64), dtype=torch.float32)
+    bad = {
+        "host tensors for a device call": lambda: c.step(q, kn, kn, out),
+        "host tensors for full-cache attention": lambda: c.full_decode(q, out),
+        "host tensors for append": lambda: c.append(kn[..., None, :], kn[..., None, :]),
+        "q of the wrong type": lambda: c.step_host(q.float(), kn, kn, out),
+        "out of the wrong type": lambda: c.step_host(q, kn, kn, out.bfloat16()),
+        "k_new one head short": lambda: c.step_host(q, kn[:, :, :1], kn, out),
+        "q with a group too few": lambda: c.decode_step_host(q[:, :, :2].contiguous(), kn, kn, out),
+        "non-contiguous out": lambda: c.step_host_async(q, kn, kn, out.transpose(2, 3)),
+        "not a tensor": lambda: c.step_host(q.float().numpy(), kn, kn, out),
+        "k and v of different shapes": lambda: c.append(kn[..., None, :], kn[:1, ..., None, :]),
+        "attention q not 3-D": lambda: dc.attend_noalloc(q, kn, kn),
+        "attention on host tensors": lambda: dc.attend_noalloc(q[0, 0, :, None], kn[0, 0, :, None], kn[0, 0, :, None]),
+        "attention k of another head size": lambda: dc.attend_noalloc(
+            torch.zeros((2, 2, 64), dtype=torch.bfloat16), torch.zeros((2, 5, 128), dtype=torch.bfloat16),
+            torch.zeros((2, 5, 128), dtype=torch.bfloat16)),
+        "log Z scores on the host": lambda: dc.pl_log_partition(torch.zeros((2, 10)), 3),
+        "log Z scores not 2-D": lambda: dc.pl_log_partition(torch.zeros(10), 3),
+        "Gumbel-top-B on the host": lambda: dc.gumbel_top_b(torch.zeros((2, 10)), torch.zeros((2, 10)), 3),
+    }
+    for what, call in bad.items():
+        with pytest.raises(dc.DCError) as e:
+            call()
+        assert e.value.status == dc.DC_ERR_INVALID_ARG, what
+
+
+def test_binding_accepts_host_tensors_of_the_abi_shapes(monkeypatch):
+    """The host-buffer calls take CPU tensors of exactly the declared sizes in
+    any shape; a well-formed call reaches the library with the tensors' own
+    addresses (a stand-in library records the call)."""
+    import torch
+    calls = []
+
+    class FakeLib:
+        def __getattr__(self, name):
+            return lambda *a: calls.append((name, a)) or dc.DC_OK
+
+    monkeypatch.setattr(dc, "lib", lambda: FakeLib())
+    c = _unopened_cache()
+    q = torch.zeros((2, 1, 4, 64), dtype=torch.bfloat16)
+    kn = torch.zeros((2, 1, 2, 64), dtype=torch.bfloat16)
+    out = torch.zeros((2, 1, 4, 64), dtype=torch.float32)
+    c.step_host(q, kn, kn, out, budget=3)
+    c.decode_step_host(q.view(8, 64), kn, kn, out)
+    c.step_host_async(q, kn.view(4, 64), kn, out)
+    ptrs = (q.data_ptr(), kn.data_ptr(), kn.data_ptr(), out.data_ptr())
+    assert calls == [("dc_step_host", (None,) + ptrs + (3,)), ("dc_decode_step_host", (None,) + ptrs),
+                     ("dc_step_host_async", (None,) + ptrs + (0,))]
