@@ -164,6 +164,14 @@ MUTANTS = [
      "x[(size_t)i * 5 + 4] = (double)s->pos[i] / pos_den;", "x[(size_t)i * 5 + 4] = (double)i / pos_den;", 1),
     ("global cumulative alpha not accumulated",
      "s->acc[i] += mean;", "s->acc[i] = mean;", 1),
+    ("global append reads the tokens as [T][R] instead of [R][T]",
+     "seq_put(s, r, s->n, k + ((size_t)r * T + t) * s->d, v + ((size_t)r * T + t) * s->d);",
+     "seq_put(s, r, s->n, k + ((size_t)t * s->R + r) * s->d, v + ((size_t)t * s->R + r) * s->d);", 1),
+    ("global step gives every row the first row's query",
+     "qd[i] = bf16_to_double(q[(size_t)r * G * d + i]);", "qd[i] = bf16_to_double(q[i]);", 1),
+    ("global step gives every row the first row's new key",
+     "seq_put(s, r, s->n, k_new + (size_t)r * d, v_new + (size_t)r * d);",
+     "seq_put(s, r, s->n, k_new, v_new + (size_t)r * d);", 1),
     ("global prune moves row 0 only",
      "      for (int r = 0; r < s->R; ++r) {\n        const size_t src",
      "      for (int r = 0; r < 1; ++r) {\n        const size_t src", 1),
