@@ -36,6 +36,7 @@ def close_rel(gpu, ref, rtol, floor_frac, what):
 def check_attention(gpu_o, ref_o, what):
     gpu_o = np.asarray(gpu_o, dtype=np.float64)
     ref_o = np.asarray(ref_o, dtype=np.float64)
+    assert gpu_o.shape == ref_o.shape, (what, gpu_o.shape, ref_o.shape)
     max_abs = float(np.max(np.abs(gpu_o - ref_o))) if ref_o.size else 0.0
     rel = float(np.linalg.norm(gpu_o - ref_o) / max(np.linalg.norm(ref_o), 1e-30))
     assert max_abs <= ATTN_MAX_ABS and rel <= ATTN_REL_L2, f"{what}: max-abs {max_abs:.3g} rel-L2 {rel:.3g}"
