@@ -51,3 +51,21 @@ def test_single_rank_throughput():
     import bench
     el, rate = bench.job_throughput(200.0, 40)
     assert el == 200.0 and rate == pytest.approx(200.0)
+
+
+def test_algorithmic_bytes_are_the_documented_per_unit_figures():
+    """The roofline's numerator: 548 B per token-row of a steady step (K and V
+    read, 4d = 512 B at d = 128; position read, 4 B; window sums read and
+    written, 32 B; cumulative alpha read and written, 8 B more, in alpha_mode 1),
+    plus per row the append (4d + 20 B) and one compaction move (2 x (4d + 20) B).
+    At the benchmark shape (2048 rows of 8193 tokens) that is 9.198 GB a step."""
+    import bench
+    from paper_2608_08878_gb300 import synth
+    assert bench.row_bytes_per_step(1, 128) == 548
+    assert bench.row_bytes_per_step(1, 128, alpha_mode=1) == 556
+    assert bench.row_bytes_per_step(1, 64) == 292
+    wl = synth.MISTRAL_FULL
+    assert (wl.rows, wl.head_dim, wl.alpha_mode) == (2048, 128, 0)
+    assert bench.step_bytes(wl, 8193) == 2048 * (8193 * 548 + 532 + 2 * 532)
+    assert round(bench.step_bytes(wl, 8193) / 1e9, 3) == 9.198
+    assert bench.step_bytes(wl, 8193, moved_per_row=0) == 2048 * (8193 * 548 + 532)
