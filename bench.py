@@ -119,18 +119,25 @@ class ClockSampler:
               "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
               "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
 
+    PERIOD_MS = 20
+
     def __init__(self, index: str):
         self.index = index
         self.proc = None
         self.lines = []
+        self.ready = threading.Event()
 
     def __enter__(self):
         try:
             self.proc = subprocess.Popen(["nvidia-smi", "-i", self.index, f"--query-gpu={self.FIELDS}",
-                                          "--format=csv,noheader,nounits", "-lms", "200"],
+                                          "--format=csv,noheader,nounits", "-lms", str(self.PERIOD_MS)],
                                          stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
             self.thread = threading.Thread(target=self._read, daemon=True)
             self.thread.start()
+            # the timed region starts once nvidia-smi is sampling (its start-up
+            # takes longer than a short timed region)
+            self.ready.wait(timeout=5.0)
+            self.lines.clear()
         except Exception:
             self.proc = None
         return self
@@ -138,6 +145,7 @@ class ClockSampler:
     def _read(self):
         for line in self.proc.stdout:
             self.lines.append(line.strip())
+            self.ready.set()
 
     def __exit__(self, *a):
         if self.proc:
@@ -164,7 +172,7 @@ class ClockSampler:
                 if val.lower().startswith("active"):
                     reasons.add(nm)
         return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": mx,
-                "reasons": sorted(reasons), "samples": len(sm)}
+                "reasons": sorted(reasons), "samples": len(sm), "period_ms": self.PERIOD_MS}
 
 
 def gpu_index_for_smi(local_rank: int) -> str:
@@ -240,17 +248,40 @@ def oracle_sample(wl, seconds: float = 12.0, threads: int | None = None, warm_st
     deadline[0] = t1 + seconds / 3
     run(r1)
     el1 = time.perf_counter() - t1
-    return {"value": steps_per_s, "unit": UNIT, "cores": len(sample_rows), "kind": "oracle",
+    return {"value": steps_per_s, "unit": UNIT, "cores": len(sample_rows), "host_cores": cores,
+            "kind": "oracle", "extrapolated": True, "row_steps_run": row_steps, "seconds": el,
             "sample": (f"{len(sample_rows)} rows (of {wl.rows}) at the steady state n={wl.budget + 1}, "
                        f"full w={wl.window} window, {row_steps} row-steps in {el:.1f}s on "
-                       f"{len(sample_rows)} host threads; value = row-steps / rows / s"),
+                       f"{len(sample_rows)} host threads (of {cores} host cores); whole decode steps/s "
+                       f"extrapolated as row-steps / rows / s (rows are independent)"),
             "single_thread": {"value": counts[r1] / wl.rows / el1, "unit": UNIT, "cores": 1,
+                              "host_cores": cores, "extrapolated": True, "row_steps_run": counts[r1],
                               "sample": f"row {r1}, {counts[r1]} row-steps in {el1:.1f}s on one host thread"}}
 
 
 # ---------------------------------------------------------------------------
 # GPU leg
 # ---------------------------------------------------------------------------
+
+def bench_config(wl, args, world: int) -> dict:
+    """The workload description both arms print (the same dict for the same
+    flags): shape, budget rule, selection mode and scorer."""
+    n_steady = wl.budget + 1
+    bytes_step = step_bytes_global(wl, n_steady) if args.global_tokens else step_bytes(wl, n_steady)
+    return {"workload": wl.name, "layers": wl.layers, "batch": wl.batch, "q_heads": wl.q_heads,
+            "kv_heads": wl.kv_heads, "head_dim": wl.head_dim, "context": wl.prompt_len,
+            "budget": wl.budget, "window": wl.window, "policy": f"5-{wl.mlp_hidden}-LN-ReLU-1",
+            "parallelism": f"replicas x{world}",
+            "selection": "per sequence (global token mode)" if args.global_tokens else
+            "per (layer, KV head) row" + (", head-level hybrid budgets" if args.hybrid else ""),
+            "scorer": ["policy MLP", "H2O (cumulative attention)", "StreamingLLM (sinks + recent)"][args.scorer],
+            "budget_rule": (f"dynamic: max(floor({args.budget_ratio} x tokens seen), 32)"
+                            if args.budget_ratio > 0 else "fixed"),
+            "timed_state": (f"after the prompt compression and {wl.window} + warm-up decode steps: "
+                            f"a full w = {wl.window} entropy window, every step subtracts a departing query"),
+            "l2": f"inputs larger than L2: {bytes_step / 1e9:.2f} GB streamed per step vs 129 MB L2",
+            "steady_tokens_per_row": n_steady}
+
 
 def job_throughput(el_ms: float, steps: int, dist=None, device="cpu"):
     """(max elapsed ms over ranks, whole-job decode steps/s): every rank runs
@@ -263,6 +294,43 @@ def job_throughput(el_ms: float, steps: int, dist=None, device="cpu"):
         dist.all_reduce(t, op=dist.ReduceOp.MAX)
         el_ms = float(t.item())
     return el_ms, world * steps / (el_ms / 1e3)
+
+
+def roofline_of(prof, wl, n_steady, engine, global_tokens=False):
+    """(dominant phase, per-launch ms, algorithmic bytes per launch, launches)
+    from the library's per-launch CUDA events: the fused kernel's bytes are
+    the whole step's but the append (K/V, positions, window sums, one move
+    per row); the split engine's kernels count their own reads and writes."""
+    dom = max((ph for ph in prof if prof[ph][1] > 0), key=lambda ph: prof[ph][0])
+    dom_ms, dom_n = prof[dom]
+    d = wl.head_dim
+    if dom == "attend" and engine.startswith("fused") and global_tokens:
+        alg = wl.rows * n_steady * (4 * d + 4)  # the rows' pass: K/V and positions
+    elif dom == "attend" and engine.startswith("fused"):
+        alg = wl.rows * (row_bytes_per_step(n_steady, d, wl.alpha_mode) + 2 * (4 * d + 20))
+    elif dom == "attend":
+        alg = wl.rows * n_steady * (2 * d + 36)  # K read + positions + window sums R/W
+    elif dom == "score":
+        alg = wl.rows * n_steady * (2 * d + 20)  # V read + positions + window sums read
+    else:
+        alg = wl.rows * row_bytes_per_step(n_steady, d, wl.alpha_mode)
+    return dom, dom_ms / dom_n, alg, dom_n
+
+
+def timed_steps(cache, inputs, s0, K, out, stream, index):
+    """K dc_step calls from inputs[s0], CUDA events on the launching stream,
+    clocks sampled meanwhile: (ms per step, clocks summary)."""
+    import torch
+    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    torch.cuda.synchronize()
+    with ClockSampler(index) as clk:
+        ev0.record(stream)
+        for s in range(s0, s0 + K):
+            cache.step(*inputs[s], out=out)
+        ev1.record(stream)
+        torch.cuda.synchronize()
+    cache.sync()  # device-side status of every timed step (raises on error)
+    return ev0.elapsed_time(ev1) / K, clk.summary()
 
 
 def run_gpu(args):
@@ -281,76 +349,76 @@ def run_gpu(args):
         build.build()
     if dist:
         dist.barrier()
-    wl = workload()
-    wl = wl.with_(seed=wl.seed + 1000 * rank)
+    wl0 = workload()
+    wl = wl0.with_(seed=wl0.seed + 1000 * rank)
     K, W = args.steps, args.warmup
+    # untimed decode steps after the prompt compression, so that the entropy
+    # window is full: every timed step adds the previous query's window terms
+    # and subtracts a departing query's
+    F = wl.window
     stream = torch.cuda.current_stream()
     cache = make_cache(wl, args)
     if args.scorer == 1:  # H2O ranks by cumulative attention (alpha_mode 1 state)
         wl = wl.with_(alpha_mode=1)
     chunk = 4096
     # all step inputs resident in HBM before timing
-    inputs = [synth_device.step_inputs(wl, s) for s in range(1 + W + K)]
+    inputs = [synth_device.step_inputs(wl, s) for s in range(1 + F + W + K)]
     out = torch.empty((wl.layers, wl.batch, wl.q_heads, wl.head_dim), dtype=torch.float32, device="cuda")
     # step 0: prompt compression (32769 -> 8192 tokens per row), timed apart
     ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    cache.profile(True)
     ev0.record(stream)
     cache.step(*inputs[0], out=out)
     ev1.record(stream)
     torch.cuda.synchronize()
     first_ms = ev0.elapsed_time(ev1)
-    for s in range(1, 1 + W):
+    first_prof = cache.profile_read()
+    cache.profile(False)
+    # the prompt compression (first step): per-phase kernel time, and the
+    # slot moves of its many-eviction compaction (a slot below the budget
+    # holds a position at or above it only if a survivor moved there)
+    first = {"ms": first_ms, "phases_ms": {k: v[0] for k, v in first_prof.items() if v[1]}}
+    if not (args.hybrid or args.budget_ratio > 0 or args.global_tokens):
+        pos = cache.buffer(dc.BUF_POS)[:, :wl.budget]
+        moved = int((pos >= wl.budget).sum().item())
+        del pos
+        mv_bytes = moved * 2 * (4 * wl.head_dim + 20)
+        first["moved_slots"] = moved
+        first["move_bytes"] = mv_bytes
+        if "evict" in first["phases_ms"]:
+            first["evict_move_gbs"] = mv_bytes / (first["phases_ms"]["evict"] / 1e3) / 1e9
+        torch.cuda.empty_cache()
+
+    for s in range(1, 1 + F + W):
         cache.step(*inputs[s], out=out)
     n_steady = cache.length()[0] + 1
     if args.hybrid or args.budget_ratio > 0:  # mean row length after the next append
         n_steady = float(cache.row_lengths().mean()) + 1
     engine = cache.engine()
+    # steps taken so far >= w: the next (first timed) step has a departing query
+    window_full = cache.length()[1] - wl.prompt_len >= wl.window
     cache.profile(True)
     torch.cuda.synchronize()
     if dist:
         dist.barrier()
-    torch.cuda.synchronize()
-    with ClockSampler(gpu_index_for_smi(local_rank)) as clk:
-        ev0.record(stream)
-        for s in range(1 + W, 1 + W + K):
-            cache.step(*inputs[s], out=out)
-        ev1.record(stream)
-        torch.cuda.synchronize()
-    el_ms = ev0.elapsed_time(ev1)
-    cache.sync()  # device-side status of every timed step (raises on error)
+    ms_per_step, clocks = timed_steps(cache, inputs, 1 + F + W, K, out, stream, gpu_index_for_smi(local_rank))
     prof = cache.profile_read()
     cache.profile(False)
-    el_ms, value = job_throughput(el_ms, K, dist, device="cuda")
+    el_ms, value = job_throughput(ms_per_step * K, K, dist, device="cuda")
     ms_per_step = el_ms / K
     bytes_step = step_bytes_global(wl, n_steady) if args.global_tokens else step_bytes(wl, n_steady)
     gbs = bytes_step / (ms_per_step / 1e3) / 1e9
     peaks, peak_src = measured_peaks()
 
     # dominant kernel: roofline from the live per-launch events
-    dom = max((ph for ph in prof if prof[ph][1] > 0), key=lambda ph: prof[ph][0])
-    dom_ms, dom_n = prof[dom]
-    per_launch_ms = dom_ms / dom_n
-    d = wl.head_dim
-    if dom == "attend" and engine == "fused" and args.global_tokens:
-        # the rows' pass: K/V and positions (the window state is per sequence)
-        alg = wl.rows * n_steady * (4 * d + 4)
-    elif dom == "attend" and engine == "fused":
-        # the whole step but the append: K/V, positions, window sums, one move per row
-        alg = wl.rows * (row_bytes_per_step(n_steady, d, wl.alpha_mode) + 2 * (4 * d + 20))
-    elif dom == "attend":
-        alg = wl.rows * n_steady * (2 * d + 36)  # K read + positions + window sums R/W
-    elif dom == "score":
-        alg = wl.rows * n_steady * (2 * d + 20)  # V read + positions + window sums read
-    else:
-        alg = wl.rows * row_bytes_per_step(n_steady, d, wl.alpha_mode)
+    dom, per_launch_ms, alg, _ = roofline_of(prof, wl, n_steady, engine, args.global_tokens)
     achieved = alg / (per_launch_ms / 1e3) / 1e9
     traffic = None
-    if dom == "attend" and engine == "fused" and not (args.global_tokens or args.hybrid or args.scorer):
+    if dom == "attend" and engine.startswith("fused") and not (args.global_tokens or args.hybrid or args.scorer):
         tpr = fused_traffic_per_token_row()
         if tpr is not None:
             traffic = wl.rows * n_steady * tpr  # scaled from the profiled case by token-rows
     gpu_launches = int(sum(v[1] for v in prof.values()))
-
     # full-cache comparator on the same inputs (the uncompressed prompt)
     full = None
     if not args.no_full and rank == 0:
@@ -368,7 +436,7 @@ def run_gpu(args):
         torch.cuda.synchronize()
         ev0.record(stream)
         for s in range(kf):
-            fc.full_decode(inputs[1 + W + s][0], out=out)
+            fc.full_decode(inputs[1 + F + W + s][0], out=out)
         ev1.record(stream)
         torch.cuda.synchronize()
         fms = ev0.elapsed_time(ev1) / kf
@@ -379,43 +447,48 @@ def run_gpu(args):
         torch.cuda.empty_cache()
         cache = None
 
-    # end to end through the public API with host buffers (rank 0 does it too
-    # on every rank: each rank its own replica)
+    # end to end through the public API with host buffers (every rank its own
+    # replica)
     e2e = None
     if not args.no_e2e:
-        e2e = run_e2e(wl, args, inputs)
+        e2e = run_e2e(wl, args, inputs, F)
+    del inputs
+    torch.cuda.empty_cache()
+
+    # the other workloads, each in the bench's launch configuration (rank 0 of
+    # a one-GPU run)
+    extra = {}
+    if not args.no_extra and rank == 0 and world == 1 and not _OVERRIDES:
+        extra = run_extra_workloads(args, peaks, stream, gpu_index_for_smi(local_rank))
 
     res = None
     if rank == 0:
+        cfg = bench_config(wl0, args, world)
+        cfg["steady_tokens_per_row"] = n_steady
         res = {
             "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": K, "warmup": W,
             "ms_per_step": ms_per_step, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
             "dtype": "bf16", "data": "synthetic",
-            "config": {"workload": wl.name, "layers": wl.layers, "batch": wl.batch, "q_heads": wl.q_heads,
-                       "kv_heads": wl.kv_heads, "head_dim": wl.head_dim, "context": wl.prompt_len,
-                       "budget": wl.budget, "window": wl.window, "policy": f"5-{wl.mlp_hidden}-LN-ReLU-1",
-                       "engine": engine, "parallelism": f"replicas x{world}",
-                       "selection": "per sequence (global token mode)" if args.global_tokens else
-                       "per (layer, KV head) row" + (", head-level hybrid budgets" if args.hybrid else ""),
-                       "scorer": ["policy MLP", "H2O (cumulative attention)", "StreamingLLM (sinks + recent)"][args.scorer],
-                       "budget_rule": (f"dynamic: max(floor({args.budget_ratio} x tokens seen), 32)"
-                                       if args.budget_ratio > 0 else "fixed"),
-                       "l2": f"inputs larger than L2: {bytes_step / 1e9:.2f} GB streamed per step vs 129 MB L2",
-                       "steady_tokens_per_row": n_steady},
+            "config": cfg,
+            "engine": engine,
+            "window_full": bool(window_full),
+            "untimed_steps_before_warmup": 1 + F,
             "hbm": {"algorithmic_bytes_per_step": bytes_step, "gbs": gbs,
                     "frac_of_8tbs": gbs / NOMINAL_HBM_GBS,
                     "frac_of_measured": gbs / peaks["hbm_gbs"], "peak_source": peak_src},
             "first_step_ms": first_ms,
+            "first_step": first,
             "roofline": {"bound": "hbm", "kernel": dom, "achieved": achieved, "peak": peaks["hbm_gbs"],
                          "unit": "GB/s", "frac": achieved / peaks["hbm_gbs"], "traffic": traffic,
                          "peak_source": f"{peak_src} copy bandwidth",
                          "per_launch_ms": per_launch_ms, "algorithmic_bytes_per_launch": alg},
             "phases_ms_per_step": {k: v[0] / K for k, v in prof.items() if v[1]},
             "gpu_launches": gpu_launches,
-            "clocks": clk.summary(),
+            "clocks": clocks,
             "full_cache": full,
             "e2e": e2e,
         }
+        res.update(extra)
     if dist:
         dist.barrier()
         dist.destroy_process_group()
@@ -447,21 +520,21 @@ def make_cache(wl, args):
     return cache
 
 
-def run_e2e(wl, args, inputs):
+def run_e2e(wl, args, inputs, F):
     """The same steps through the host-buffer API: every step copies its pinned
     host inputs in and the attention output out (dc_step_host_async, in the
     handle's stream order; one synchronisation at the end of the timed region,
-    which therefore holds every copy)."""
+    which therefore holds every copy). The same untimed steps come first."""
     import torch
     cache = make_cache(wl, args)
     host = [tuple(x.cpu().pin_memory() for x in inp) for inp in inputs]
     out = torch.empty((wl.layers, wl.batch, wl.q_heads, wl.head_dim), dtype=torch.float32).pin_memory()
     W, K = args.warmup, args.steps
-    for s in range(0, 1 + W):
+    for s in range(0, 1 + F + W):
         cache.step_host(*host[s], out)
     torch.cuda.synchronize()
     t0 = time.perf_counter()
-    for s in range(1 + W, 1 + W + K):
+    for s in range(1 + F + W, 1 + F + W + K):
         cache.step_host_async(*host[s], out)
     cache.sync()
     el = time.perf_counter() - t0
@@ -478,12 +551,16 @@ def run_reference(args):
         return None
     wl = workload()
     cb = oracle_sample(wl, seconds=args.cpu_seconds)
+    world = int(os.environ.get("WORLD_SIZE", "1"))
     return {"impl": "reference", "metric": METRIC, "value": cb["value"], "unit": UNIT,
-            "n_gpus": int(os.environ.get("WORLD_SIZE", "1")), "steps": args.steps, "warmup": args.warmup,
+            "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
             "ms_per_step": 1e3 / cb["value"], "higher_is_better": True, "scaling": "weak",
             "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-            "config": {"workload": wl.name, "layers": wl.layers, "batch": wl.batch,
-                       "context": wl.prompt_len, "budget": wl.budget},
+            "extrapolated": True,
+            "timing_note": (f"not {args.steps} whole steps: {cb['row_steps_run']} row-steps of {wl.rows}-row "
+                            f"decode steps in {cb['seconds']:.1f}s on {cb['cores']} host threads, "
+                            f"extrapolated to whole steps (rows are independent)"),
+            "config": bench_config(wl, args, world),
             "cpu_baseline": cb,
             "e2e": {"value": cb["value"], "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
 
@@ -497,16 +574,153 @@ SWEEP_CONTEXT = (4096, 16384, 32768)
 SWEEP_RATIO = (0.10, 0.25, 0.50)
 
 
-def run_sweep(args):
-    """Steady-state decode steps/s per point of the sweep, next to full-cache
-    attention on the same shapes. The steady cache is synthesised at its
-    budget size (B prompt tokens, then decode steps that append one token and
-    evict one), which is what the cache holds after prompt compression; the
-    full-cache comparator attends over context + 1 tokens and is timed on as
-    many layers as fit in 48 GB, scaled to 32 layers (its time is linear in
-    the rows)."""
+def sweep_point_run(b, c, r, K, W, engine_flag, peaks, stream, index, with_full=True):
+    """One sweep point: the steady cache (B prompt tokens, then steps that
+    append one token and evict one, the state after prompt compression), W
+    warm-up and K timed dc_step calls, roofline of the dominant kernel from
+    the library's per-launch events, and (with_full) full-cache attention over
+    context + 1 tokens, timed on as many layers as fit in 48 GB and scaled to
+    32 layers (its time is linear in the rows)."""
     import torch
-    from paper_2608_08878_gb300 import build, dc, synth, synth_device
+    from paper_2608_08878_gb300 import dc, synth, synth_device
+    wl = synth.sweep_point(b, c, r)
+    B, d = wl.budget, wl.head_dim
+    cache = dc.DistillCache(wl.layers, wl.kv_heads, d, B + 1, B, batch=b, q_heads=wl.q_heads,
+                            window=wl.window, mlp_hidden=wl.mlp_hidden, layernorm=wl.layernorm,
+                            seed=wl.policy_seed, engine=engine_flag)
+    chunk = max(1, min(B, (1 << 31) // (wl.rows * d * 2)))
+    for t0 in range(0, B, chunk):
+        k, v = synth_device.prompt(wl, t0, min(chunk, B - t0))
+        cache.append(k, v)
+        del k, v
+    inputs = [synth_device.step_inputs(wl, s) for s in range(W + K)]
+    out = torch.empty((wl.layers, b, wl.q_heads, d), dtype=torch.float32, device="cuda")
+    for s in range(W):
+        cache.step(*inputs[s], out=out)
+    engine = cache.engine()
+    cache.profile(True)
+    ms, clocks = timed_steps(cache, inputs, W, K, out, stream, index)
+    prof = cache.profile_read()
+    dom, per_launch_ms, alg, _ = roofline_of(prof, wl, B + 1, engine)
+    achieved = alg / (per_launch_ms / 1e3) / 1e9
+    bytes_step = step_bytes(wl, B + 1)
+    del cache, inputs, out
+    torch.cuda.empty_cache()
+    gbs = bytes_step / (ms / 1e3) / 1e9
+    res = {"sweep_point": f"{b}x{c}x{int(round(r * 100))}", "workload": wl.name, "batch": b, "context": c,
+           "ratio": r, "budget": B, "rows": wl.rows, "engine": engine, "steps": K, "warmup": W,
+           "ms_per_step": ms, "steps_per_s": 1e3 / ms, "gbs": gbs,
+           "frac_of_8tbs": gbs / NOMINAL_HBM_GBS, "frac_of_measured": gbs / peaks["hbm_gbs"],
+           "roofline": {"bound": "hbm", "kernel": dom, "achieved": achieved, "peak": peaks["hbm_gbs"],
+                        "unit": "GB/s", "frac": achieved / peaks["hbm_gbs"], "per_launch_ms": per_launch_ms,
+                        "algorithmic_bytes_per_launch": alg},
+           "footprint_steady_gb": wl.rows * (B + 1) * (4 * d + 20) / 1e9,
+           "footprint_prompt_gb": wl.rows * (c + 1) * (4 * d + 20) / 1e9,
+           "clocks": clocks, "data": "synthetic"}
+    if not with_full:
+        return res
+    per_layer = b * wl.kv_heads * (c + 1) * (4 * d + 20)
+    lf = max(1, min(wl.layers, int(48e9 // per_layer)))
+    wf = wl.with_(layers=lf)
+    full = dc.DistillCache(lf, wl.kv_heads, d, c + 1, c, batch=b, q_heads=wl.q_heads)
+    chunk = max(1, min(c + 1, (1 << 31) // (wf.rows * d * 2)))
+    for t0 in range(0, c + 1, chunk):
+        k, v = synth_device.prompt(wf, t0, min(chunk, c + 1 - t0))
+        full.append(k, v)
+        del k, v
+    qf = synth_device.step_inputs(wf, 0)[0]
+    for _ in range(2):
+        full.full_decode(qf)
+    torch.cuda.synchronize()
+    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    reps = 5
+    ev0.record(stream)
+    for _ in range(reps):
+        full.full_decode(qf)
+    ev1.record(stream)
+    torch.cuda.synchronize()
+    full_ms = ev0.elapsed_time(ev1) / reps * wl.layers / lf
+    del full, qf
+    torch.cuda.empty_cache()
+    res.update({"full_cache_ms_per_step": full_ms, "full_cache_layers_timed": lf,
+                "speedup_vs_full": full_ms / ms})
+    return res
+
+
+def workload_run(wl, steps_total, W, engine_flag, peaks, stream, index):
+    """A workload as its configuration states it: the prompt, then
+    `steps_total` decode steps (dc_step) of which the first is the prompt
+    compression (timed apart), the next W warm-up and the rest timed; roofline
+    of the dominant kernel from the library's per-launch events."""
+    import torch
+    from paper_2608_08878_gb300 import dc, synth_device
+    cache = dc.DistillCache(wl.layers, wl.kv_heads, wl.head_dim, wl.capacity, wl.budget, batch=wl.batch,
+                            q_heads=wl.q_heads, window=wl.window, mlp_hidden=wl.mlp_hidden,
+                            layernorm=wl.layernorm, seed=wl.policy_seed, engine=engine_flag)
+    chunk = max(1, min(wl.prompt_len, (1 << 31) // (wl.rows * wl.head_dim * 2)))
+    for t0 in range(0, wl.prompt_len, chunk):
+        k, v = synth_device.prompt(wl, t0, min(chunk, wl.prompt_len - t0))
+        cache.append(k, v)
+        del k, v
+    inputs = [synth_device.step_inputs(wl, s) for s in range(steps_total)]
+    out = torch.empty((wl.layers, wl.batch, wl.q_heads, wl.head_dim), dtype=torch.float32, device="cuda")
+    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    ev0.record(stream)
+    cache.step(*inputs[0], out=out)
+    ev1.record(stream)
+    torch.cuda.synchronize()
+    first_ms = ev0.elapsed_time(ev1)
+    for s in range(1, 1 + W):
+        cache.step(*inputs[s], out=out)
+    engine = cache.engine()
+    K = steps_total - 1 - W
+    cache.profile(True)
+    ms, clocks = timed_steps(cache, inputs, 1 + W, K, out, stream, index)
+    prof = cache.profile_read()
+    n = wl.budget + 1
+    dom, per_launch_ms, alg, _ = roofline_of(prof, wl, n, engine)
+    achieved = alg / (per_launch_ms / 1e3) / 1e9
+    bytes_step = step_bytes(wl, n)
+    del cache, inputs, out
+    torch.cuda.empty_cache()
+    gbs = bytes_step / (ms / 1e3) / 1e9
+    return {"workload": wl.name, "rows": wl.rows, "tokens_per_row": n, "engine": engine,
+            "decode_steps": steps_total, "first_step_ms": first_ms, "warmup": W, "steps": K,
+            "ms_per_step": ms, "us_per_step": ms * 1e3, "steps_per_s": 1e3 / ms,
+            "hbm": {"algorithmic_bytes_per_step": bytes_step, "gbs": gbs,
+                    "frac_of_measured": gbs / peaks["hbm_gbs"]},
+            "roofline": {"bound": "hbm", "kernel": dom, "achieved": achieved, "peak": peaks["hbm_gbs"],
+                         "unit": "GB/s", "frac": achieved / peaks["hbm_gbs"], "per_launch_ms": per_launch_ms,
+                         "algorithmic_bytes_per_launch": alg},
+            "clocks": clocks, "data": "synthetic"}
+
+
+SWEEP_WORST = ((1, 4096, 0.10), (4, 4096, 0.10), (64, 4096, 0.10), (1, 32768, 0.50))
+
+
+def run_extra_workloads(args, peaks, stream, index):
+    """The other configurations next to the headline, each timed the same
+    way: the Mistral-7B single layer (8 rows of 2049 tokens, 128 decode
+    steps, latency-bound), the aggressive 10% workload (32 layers, batch 16,
+    hot sets reshuffled every 16 steps, 64 decode steps) and the sweep's
+    slowest points (short rows at 10%, one 32K row set at 50%)."""
+    from paper_2608_08878_gb300 import synth
+    W = args.warmup
+    out = {"config2": workload_run(synth.MISTRAL_1L, synth.MISTRAL_1L.steps, W, args.engine, peaks, stream, index)}
+    out["config2"]["note"] = ("9 MB of algorithmic traffic per step: bound by launch and per-row latency, "
+                              "not HBM; the roofline fraction is reported for completeness")
+    out["config4"] = workload_run(synth.AGGRESSIVE, synth.AGGRESSIVE.steps, W, args.engine, peaks, stream, index)
+    out["sweep_worst"] = [sweep_point_run(b, c, r, 32, W, args.engine, peaks, stream, index, with_full=False)
+                          for b, c, r in SWEEP_WORST]
+    return out
+
+
+def run_sweep(args):
+    """Steady-state decode steps/s per point of the sweep (batch x context x
+    budget ratio), one JSON line each, next to full-cache attention on the
+    same shapes."""
+    import torch
+    from paper_2608_08878_gb300 import build
     torch.cuda.set_device(0)
     build.build()
     peaks, _ = measured_peaks()
@@ -515,70 +729,9 @@ def run_sweep(args):
     if args.sweep_points:
         keep = set(args.sweep_points.split(","))
         pts = [p for p in pts if f"{p[0]}x{p[1]}x{int(round(p[2] * 100))}" in keep]
-    K, W = args.steps, args.warmup
     for b, c, r in pts:
-        wl = synth.sweep_point(b, c, r)
-        B, d = wl.budget, wl.head_dim
-        cache = dc.DistillCache(wl.layers, wl.kv_heads, d, B + 1, B, batch=b, q_heads=wl.q_heads,
-                                window=wl.window, mlp_hidden=wl.mlp_hidden, layernorm=wl.layernorm,
-                                seed=wl.policy_seed, engine=args.engine)
-        chunk = max(1, min(B, (1 << 31) // (wl.rows * d * 2)))
-        for t0 in range(0, B, chunk):
-            k, v = synth_device.prompt(wl, t0, min(chunk, B - t0))
-            cache.append(k, v)
-            del k, v
-        inputs = [synth_device.step_inputs(wl, s) for s in range(W + K)]
-        out = torch.empty((wl.layers, b, wl.q_heads, d), dtype=torch.float32, device="cuda")
-        for s in range(W):
-            cache.step(*inputs[s], out=out)
-        engine = cache.engine()
-        torch.cuda.synchronize()
-        ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-        with ClockSampler(gpu_index_for_smi(0)) as clk:
-            ev0.record(stream)
-            for s in range(W, W + K):
-                cache.step(*inputs[s], out=out)
-            ev1.record(stream)
-            torch.cuda.synchronize()
-        cache.sync()
-        ms = ev0.elapsed_time(ev1) / K
-        bytes_step = step_bytes(wl, B + 1)
-        del cache, inputs, out
-        torch.cuda.empty_cache()
-        # full-cache comparator on a layer subset
-        per_layer = b * wl.kv_heads * (c + 1) * (4 * d + 20)
-        lf = max(1, min(wl.layers, int(48e9 // per_layer)))
-        wf = wl.with_(layers=lf)
-        full = dc.DistillCache(lf, wl.kv_heads, d, c + 1, c, batch=b, q_heads=wl.q_heads)
-        chunk = max(1, min(c + 1, (1 << 31) // (wf.rows * d * 2)))
-        for t0 in range(0, c + 1, chunk):
-            k, v = synth_device.prompt(wf, t0, min(chunk, c + 1 - t0))
-            full.append(k, v)
-            del k, v
-        qf = synth_device.step_inputs(wf, 0)[0]
-        for _ in range(2):
-            full.full_decode(qf)
-        torch.cuda.synchronize()
-        reps = 5
-        ev0.record(stream)
-        for _ in range(reps):
-            full.full_decode(qf)
-        ev1.record(stream)
-        torch.cuda.synchronize()
-        full_ms = ev0.elapsed_time(ev1) / reps * wl.layers / lf
-        del full, qf
-        torch.cuda.empty_cache()
-        gbs = bytes_step / (ms / 1e3) / 1e9
-        print(json.dumps({
-            "sweep_point": f"{b}x{c}x{int(round(r * 100))}", "batch": b, "context": c, "ratio": r,
-            "budget": B, "rows": wl.rows, "engine": engine, "steps": K, "warmup": W,
-            "ms_per_step": ms, "steps_per_s": 1e3 / ms, "gbs": gbs,
-            "frac_of_8tbs": gbs / NOMINAL_HBM_GBS, "frac_of_measured": gbs / peaks["hbm_gbs"],
-            "full_cache_ms_per_step": full_ms, "full_cache_layers_timed": lf,
-            "speedup_vs_full": full_ms / ms,
-            "footprint_steady_gb": wl.rows * (B + 1) * (4 * d + 20) / 1e9,
-            "footprint_prompt_gb": wl.rows * (c + 1) * (4 * d + 20) / 1e9,
-            "clocks": clk.summary(), "data": "synthetic"}), flush=True)
+        print(json.dumps(sweep_point_run(b, c, r, args.steps, args.warmup, args.engine, peaks, stream,
+                                         gpu_index_for_smi(0))), flush=True)
 
 
 def run_train(args):
@@ -625,6 +778,8 @@ def main():
     ap.add_argument("--no-cpu", action="store_true")
     ap.add_argument("--no-full", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-extra", action="store_true",
+                    help="skip the other workloads (single layer, aggressive 10%%, the sweep's slowest points)")
     ap.add_argument("--layers", type=int, default=None, help="profiling: fewer layers than the workload's 32")
     ap.add_argument("--batch", type=int, default=None, help="profiling: another batch than the workload's 8")
     ap.add_argument("--context", type=int, default=None, help="profiling: another prompt length than 32768")

@@ -137,10 +137,16 @@ size_t dc_policy_blob_len(int hidden);
 dc_status dc_policy_init(unsigned long long seed, int hidden, float* host_out, size_t n);
 
 /* Replaces the policy weights with a host fp32 blob of dc_policy_blob_len(H)
- * floats (H = cfg->mlp_hidden). The blob is copied before the call returns. */
+ * floats (H = cfg->mlp_hidden): the network f_phi of Sec. 3.1.2 (Action Space,
+ * scores s_i = f_phi(x_i)) with the two-layer, LayerNorm, ReLU shape of App. D
+ * (Training Details), e.g. trained weights. The blob is copied before the call
+ * returns; DC_ERR_INVALID_ARG if n differs from dc_policy_blob_len(H). */
 dc_status dc_policy_set_weights(dc_cache* h, const float* host_blob, size_t n);
 
 /* Appends n_tokens tokens to every row without queries (prompt loading).
+ * Algorithm 1 takes the prompt as the cache at t = 0; later decode steps add
+ * one pair each (C_t includes the new key/value pair before the forward pass,
+ * Sec. 3.1, Problem Formulation).
  * k, v: bf16 [layers][batch][kv_heads][n_tokens][head_dim]. Positions continue
  * from the number of tokens seen. DC_ERR_CAPACITY (cache unchanged) if the
  * rows would exceed capacity. */
@@ -307,8 +313,13 @@ dc_status dc_sync(dc_cache* h);
  *   q:   bf16 [rows][group][head_dim]; k, v: bf16 [rows][n][head_dim]
  *        (16-byte aligned); out: fp32 [rows][group][head_dim]; all device.
  *   stream: cudaStream_t (NULL: legacy default stream).
- * The split-K partial results go to a 16 MiB file-scope device array that is
- * reserved on every GPU that loads this library until the process exits.
+ * The split-K partial results go to a 16 MiB file-scope device array that
+ * stays reserved, on every GPU where this library's device code is loaded,
+ * until the process exits. With CUDA's lazy module loading (the default since
+ * CUDA 12.2) that code, and so the array, is loaded on a device at the first
+ * call there: a caller that reserves the rest of device memory up front must
+ * make one call (a warm-up) on each device before it does, or that first call
+ * can fail with DC_ERR_CUDA (out of memory while loading the module).
  * DC_ERR_CAPACITY if one split of all rows does not fit it, i.e. if
  * rows * group * (head_dim + 4) * 4 > 16 MiB; DC_ERR_INVALID_ARG for bad
  * shapes (head_dim 64 or 128, group 1, 2, 4 or 8, 1 <= rows <= 65535, n >= 1).

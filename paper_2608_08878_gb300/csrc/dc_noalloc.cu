@@ -8,8 +8,11 @@
 // cudaMalloc/cudaFree is not acceptable. None of the handle-based calls fit
 // them, because dc_cache_create allocates.
 //
-// The scratch array is reserved once per device when this library's device
-// code is loaded there, and stays reserved until the process exits.
+// The scratch array is reserved on a device when this library's device code
+// is loaded there, and stays reserved until the process exits. Under lazy
+// module loading (CUDA's default) that happens at the first call on the
+// device, inside cudaGetSymbolAddress below: a caller that reserves the rest
+// of device memory must make its first call before doing so.
 #include <cuda_runtime.h>
 
 #include <cmath>

@@ -128,23 +128,34 @@ def policy_init(seed: int, hidden: int) -> np.ndarray:
 
 def attend_noalloc(q, k, v, out=None, stream=None):
     """Full-cache decode attention with no device allocation by the library:
-    q [rows][group][d], k/v [rows][n][d] bf16 CUDA tensors -> out fp32."""
+    q [rows][group][d], k/v [rows][n][d] bf16 CUDA tensors -> out fp32.
+
+    The library takes the device from the current CUDA device, so the call
+    runs with q's device made current, on `stream` (which must belong to that
+    device) or that device's current stream."""
     import torch
     if not isinstance(q, torch.Tensor) or q.dim() != 3 or not isinstance(k, torch.Tensor) or k.dim() != 3:
         raise DCError(DC_ERR_INVALID_ARG, "q must be [rows][group][head_dim] and k, v [rows][n][head_dim]")
+    if not isinstance(v, torch.Tensor) or tuple(v.shape) != tuple(k.shape):
+        raise DCError(DC_ERR_INVALID_ARG, f"v must have k's shape {tuple(k.shape)}")
+    if not q.is_cuda:
+        raise DCError(DC_ERR_INVALID_ARG, "q must be a CUDA tensor")
     rows, group, d = q.shape
     n = k.shape[1]
     if k.shape[0] != rows or k.shape[2] != d:
         raise DCError(DC_ERR_INVALID_ARG, f"k has shape {tuple(k.shape)}, expected ({rows}, n, {d})")
-    dev = q.device.index if q.is_cuda else None
+    dev = q.device.index
     pq = _arg(q, "q", torch.bfloat16, rows * group * d, device=dev)
     pk = _arg(k, "k", torch.bfloat16, rows * n * d, device=dev)
     pv = _arg(v, "v", torch.bfloat16, rows * n * d, device=dev)
     if out is None:
         out = torch.empty((rows, group, d), dtype=torch.float32, device=q.device)
     po = _arg(out, "out", torch.float32, rows * group * d, device=dev)
-    s = (stream or torch.cuda.current_stream()).cuda_stream
-    st = lib().dc_attend_noalloc(pq, pk, pv, rows, n, d, group, po, s)
+    if stream is not None and stream.device != q.device:
+        raise DCError(DC_ERR_INVALID_ARG, f"stream is on {stream.device}, the tensors on {q.device}")
+    with torch.cuda.device(q.device):
+        s = (stream or torch.cuda.current_stream(q.device)).cuda_stream
+        st = lib().dc_attend_noalloc(pq, pk, pv, rows, n, d, group, po, s)
     if st != DC_OK:
         raise DCError(st, lib().dc_noalloc_last_error().decode())
     return out

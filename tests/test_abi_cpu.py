@@ -174,6 +174,9 @@ def test_binding_rejects_tensors_that_do_not_match_the_abi():
         "attention k of another head size": lambda: dc.attend_noalloc(
             torch.zeros((2, 2, 64), dtype=torch.bfloat16), torch.zeros((2, 5, 128), dtype=torch.bfloat16),
             torch.zeros((2, 5, 128), dtype=torch.bfloat16)),
+        "attention v of another shape than k (same element count)": lambda: dc.attend_noalloc(
+            torch.zeros((2, 2, 64), dtype=torch.bfloat16), torch.zeros((2, 5, 64), dtype=torch.bfloat16),
+            torch.zeros((5, 2, 64), dtype=torch.bfloat16)),
         "log Z scores on the host": lambda: dc.pl_log_partition(torch.zeros((2, 10)), 3),
         "log Z scores not 2-D": lambda: dc.pl_log_partition(torch.zeros(10), 3),
         "Gumbel-top-B on the host": lambda: dc.gumbel_top_b(torch.zeros((2, 10)), torch.zeros((2, 10)), 3),

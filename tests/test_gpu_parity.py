@@ -414,12 +414,16 @@ def test_errors_leave_the_cache_usable():
 @pytest.mark.parametrize("engine", ENGINES)
 def test_full_stack_sampled_rows(engine):
     """Mistral-7B 32 layers, batch 8, 32K context, budget 8192 at full size: the
-    prompt-compression step and steady steps, 3 sampled rows."""
+    prompt-compression step and 71 steady steps, 3 sampled rows (among them the
+    last row, which falls in the fused grid's split last wave). Queries leave
+    the w = 64 window from step 64 on; every step from 62 on is checked, so the
+    departing-query subtraction is compared with the oracle at this shape."""
     wl = synth.MISTRAL_FULL
+    assert wl.window == 64
     ls = LockStep(wl, [0, 1029, wl.rows - 1], engine=engine, device_inputs=True)
     ls.load_prompt()
-    for _ in range(3):
-        ls.step()
+    for s in range(72):
+        ls.step(check=(s < 3 or s % 16 == 0 or s >= 62))
     assert ls.cache.length()[0] == wl.budget
 
 
@@ -441,12 +445,16 @@ def test_sweep_points_sampled_rows(batch, ctx, ratio):
 
 def test_aggressive_sampled_rows():
     """32 layers, batch 16, 32K context, budget 3277 (10%), hot sets reshuffled
-    every 16 steps: crosses one reshuffle, 2 sampled rows."""
+    every 16 steps: 72 steps cross four reshuffles and the w = 64 window's
+    departures; 2 sampled rows, checked around each reshuffle and at every
+    step from 62 on."""
     wl = synth.AGGRESSIVE
+    assert wl.epoch_len == 16 and wl.window == 64
     ls = LockStep(wl, [7, wl.rows - 3], engine=0, device_inputs=True)  # auto: fused steady steps
     ls.load_prompt()
-    for s in range(18):
-        ls.step(check=(s < 2 or s >= 15))
+    for s in range(72):
+        ls.step(check=(s < 2 or s % 16 in (0, 1, 15) or s >= 62))
+    assert ls.cache.length()[0] == wl.budget
 
 
 @pytest.mark.parametrize("engine", ENGINES)

@@ -12,6 +12,7 @@ import pytest
 
 from paper_2608_08878_gb300 import synth
 
+import oracle
 from harness import check_attention
 
 pytestmark = pytest.mark.gpu
@@ -46,6 +47,32 @@ def test_noalloc_attention_matches_full_decode_on_consecutive_calls():
         out = dc.attend_noalloc(qt.reshape(rows, G, d), kr, vr)
         torch.cuda.synchronize()
         check_attention(out.reshape(ref.shape).cpu().numpy(), ref.cpu().numpy(), f"call {step}")
+
+
+@pytest.mark.parametrize("head_dim", [64, 128])
+@pytest.mark.parametrize("group", [1, 2, 4, 8])
+@pytest.mark.parametrize("n", [1, 100, 257])
+def test_noalloc_attention_matches_oracle(head_dim, group, n):
+    """Every <head_dim, group> variant the entry point dispatches to, on rows of
+    one token, of less than one 128-token tile and of a ragged third tile,
+    against the fp64 oracle's softmax attention, twice in a row (the second
+    call finds the first one's partials in the shared scratch array)."""
+    import torch
+    from paper_2608_08878_gb300 import dc
+    rows = 3
+    wl = synth.TINY.with_(kv_heads=rows, q_heads=rows * group, head_dim=head_dim, prompt_len=n,
+                          seed=100 + n + group)
+    k, v = synth.prompt_all(wl)                          # [1][1][rows][n][d]
+    kr, vr = _bf16(torch, k).reshape(rows, n, head_dim), _bf16(torch, v).reshape(rows, n, head_dim)
+    for step in (0, 1):
+        q, _, _ = synth.step_all(wl, step)               # [1][1][rows * group][d]
+        qh = q.reshape(rows, group, head_dim)
+        out = dc.attend_noalloc(_bf16(torch, qh), kr, vr)
+        torch.cuda.synchronize()
+        got = out.cpu().numpy()
+        for r in range(rows):
+            ref, _ = oracle.attend(qh[r], k[0, 0, r], v[0, 0, r])
+            check_attention(got[r], ref, f"d {head_dim} G {group} n {n} row {r} call {step}")
 
 
 def test_noalloc_rejects_oversized_and_bad_shapes():
