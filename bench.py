@@ -48,7 +48,7 @@ def workload():
     if _OVERRIDES:
         wl = wl.with_(**_OVERRIDES)
         wl = wl.with_(name=f"{wl.name} [profiling case: {wl.layers} layers, batch {wl.batch}, "
-                           f"context {wl.prompt_len}, budget {wl.budget}]")
+                           f"{wl.q_heads}q/{wl.kv_heads}kv heads, context {wl.prompt_len}, budget {wl.budget}]")
     return wl
 
 
@@ -784,6 +784,8 @@ def main():
     ap.add_argument("--batch", type=int, default=None, help="profiling: another batch than the workload's 8")
     ap.add_argument("--context", type=int, default=None, help="profiling: another prompt length than 32768")
     ap.add_argument("--budget", type=int, default=None, help="profiling: another budget than 8192")
+    ap.add_argument("--q-heads", type=int, default=None, help="profiling: query heads per layer (32)")
+    ap.add_argument("--kv-heads", type=int, default=None, help="profiling: KV heads per layer (8)")
     ap.add_argument("--sweep", action="store_true",
                     help="throughput sweep (batch x context x ratio): one JSON line per point")
     ap.add_argument("--sweep-points", default=None, help="e.g. 1x4096x10,64x32768x50 (default: all 36)")
@@ -805,6 +807,10 @@ def main():
         _OVERRIDES["prompt_len"] = args.context
     if args.budget:
         _OVERRIDES["budget"] = args.budget
+    if args.q_heads:
+        _OVERRIDES["q_heads"] = args.q_heads
+    if args.kv_heads:
+        _OVERRIDES["kv_heads"] = args.kv_heads
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")
     if args.sweep:

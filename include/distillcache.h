@@ -351,6 +351,41 @@ dc_status dc_wait_selftest(unsigned long long limit_ns, unsigned* result, void* 
 /* Message of the last failed dc_wait_selftest call on this host thread. */
 const char* dc_selftest_last_error(void);
 
+/* ---------------------------------------------------------------------------
+ * Testing hooks: for the library's own tests, not for production use. None
+ * of them can make a kernel fault.
+ * ------------------------------------------------------------------------- */
+
+/* Allocation-failure injection: the device allocation with index nth, counted
+ * from this call over every allocation the library makes for a handle
+ * (dc_cache_create and the buffers some calls add later), fails as if the
+ * device were out of memory, once; nth < 0 disarms. Host-only; DC_OK. A
+ * create that meets the failure returns DC_ERR_OOM after freeing what it
+ * took; a later call that needs a new buffer returns DC_ERR_OOM and leaves
+ * the handle usable and unchanged. */
+dc_status dc_debug_fail_alloc(long long nth);
+
+/* 1 if this library is a debug build (compiled with DC_DEBUG_BOUNDS), else 0.
+ * A debug build checks computed global-memory indices in its kernels before
+ * each access (a failed check raises a status bit that dc_sync reports as
+ * DC_ERR_DEVICE, records the first site, index and limit, and skips the
+ * access), and puts a guard region before and after every device buffer of
+ * a handle, which dc_sync checks. */
+int dc_debug_checks(void);
+
+/* Debug builds: one kernel checks an index one past its limit; result (host,
+ * 5 values): [0] the status word it raised (bit 2: a failed index check),
+ * [1] the site recorded (903), [2] the index, [3] the limit, [4] 1 if the
+ * access was skipped. Synchronises the stream. Release builds: DC_ERR_STATE
+ * (message in dc_selftest_last_error()). */
+dc_status dc_debug_bounds_selftest(unsigned* result, void* stream);
+
+/* Debug builds: overwrites one byte of the guard region after the handle's
+ * first buffer (memory the handle owns, outside every buffer) on its stream,
+ * so that the next dc_sync reports DC_ERR_DEVICE. Release builds:
+ * DC_ERR_STATE. */
+dc_status dc_debug_corrupt_guard(dc_cache* h);
+
 /* Message of the last error on the handle (or of the last failed create when
  * h is NULL). Valid until the next call on the handle. */
 const char* dc_last_error(const dc_cache* h);

@@ -22,6 +22,11 @@ INCLUDE = os.path.join(os.path.dirname(HERE), "include")
 
 LIB_MAIN = os.path.join(HERE, "libdistillcache.so")
 LIB_SYNTH = os.path.join(HERE, "libdc_synth.so")
+# the same library with device-side index checks and guard regions around the
+# handle's buffers (DC_DEBUG_BOUNDS), for tests; the binding loads it when
+# DC_LIBRARY=debug
+LIB_DEBUG = os.path.join(HERE, "libdistillcache_debug.so")
+BUILD_DEBUG = os.path.join(HERE, "_build_debug")
 
 MAIN_SOURCES = ["dc_cache.cu", "dc_split.cu", "dc_evict.cu", "dc_full.cu", "dc_fused.cu", "dc_noalloc.cu",
                 "dc_train.cu", "dc_global.cu", "dc_fused_modes.cu", "dc_fused_glob.cu",
@@ -56,8 +61,8 @@ def _stale(target: str, inputs: list[str]) -> bool:
     return any(os.path.getmtime(i) > t for i in inputs)
 
 
-def _compile(src: str, extra: list[str], verbose: bool) -> str:
-    obj = os.path.join(BUILD, os.path.basename(src).replace(".cu", ".o"))
+def _compile(src: str, extra: list[str], verbose: bool, build_dir: str = BUILD) -> str:
+    obj = os.path.join(build_dir, os.path.basename(src).replace(".cu", ".o"))
     if _stale(obj, _deps()):
         cmd = [nvcc()] + NVCC_FLAGS + extra + ["-c", os.path.join(CSRC, src), "-o", obj]
         if verbose:
@@ -80,6 +85,16 @@ def _link(objs: list[str], target: str, libs: list[str]) -> None:
         os.replace(tmp, target)
 
 
+def build_debug(verbose: bool = False) -> str:
+    """libdistillcache_debug.so: every kernel with its index checks compiled
+    in (DC_DEBUG_BOUNDS) and guard regions around the handle's buffers."""
+    os.makedirs(BUILD_DEBUG, exist_ok=True)
+    with cf.ThreadPoolExecutor(max_workers=min(8, len(MAIN_SOURCES))) as ex:
+        objs = list(ex.map(lambda s: _compile(s, ["-DDC_DEBUG_BOUNDS"], verbose, BUILD_DEBUG), MAIN_SOURCES))
+    _link(objs, LIB_DEBUG, [])
+    return LIB_DEBUG
+
+
 def build(verbose: bool = False) -> tuple[str, str]:
     os.makedirs(BUILD, exist_ok=True)
     srcs = MAIN_SOURCES + SYNTH_SOURCES
@@ -91,4 +106,4 @@ def build(verbose: bool = False) -> tuple[str, str]:
 
 
 if __name__ == "__main__":
-    print(build(verbose="-v" in sys.argv))
+    print(build_debug(verbose="-v" in sys.argv) if "--debug" in sys.argv else build(verbose="-v" in sys.argv))

@@ -3,6 +3,8 @@
 // sequence of each call.
 #include <cuda_runtime.h>
 
+#include <atomic>
+
 #include <algorithm>
 #include <cmath>
 #include <cstdio>
@@ -92,7 +94,11 @@ struct dc_cache {
   dc::Step gstep{};
   unsigned gepoch = 0;
   int* gcount_dev = nullptr;
-  std::vector<void*> allocs;
+  struct Alloc {
+    void* base;    // what cudaMalloc returned (guard regions included in debug builds)
+    size_t bytes;  // the buffer's own size
+  };
+  std::vector<Alloc> allocs;
   std::string err;
   bool broken = false;
   // launch counting and optional per-launch event timing
@@ -131,19 +137,68 @@ bool valid(const dc_cache* h) { return h && h->magic == kMagic; }
     if (e_ != cudaSuccess) return cuda_fail((h), e_, #call);                   \
   } while (0)
 
+// Allocation-failure injection (dc_debug_fail_alloc): the allocation with this
+// index, counted from when the hook was armed, fails as if the device were out
+// of memory; -1: disarmed. Host-only.
+std::atomic<long long> g_fail_alloc_at{-1};
+std::atomic<long long> g_alloc_index{0};
+
+// Debug builds put a guard region of kGuardBytes before and after every device
+// buffer of a handle, filled with kGuardByte; dc_sync checks that both are intact.
+#ifdef DC_DEBUG_BOUNDS
+constexpr size_t kGuardBytes = 256;
+#else
+constexpr size_t kGuardBytes = 0;
+#endif
+constexpr unsigned char kGuardByte = 0xA5;
+
 template <class T>
 cudaError_t dalloc(dc_cache* h, T** p, size_t bytes) {
+  if (g_fail_alloc_at.load() >= 0 && g_alloc_index.fetch_add(1) == g_fail_alloc_at.load()) {
+    g_fail_alloc_at.store(-1);  // one-shot
+    return cudaErrorMemoryAllocation;
+  }
+  const size_t nb = bytes ? bytes : 16;
   void* q = nullptr;
-  cudaError_t e = cudaMalloc(&q, bytes ? bytes : 16);
+  cudaError_t e = cudaMalloc(&q, nb + 2 * kGuardBytes);
   if (e != cudaSuccess) return e;
-  h->allocs.push_back(q);
-  *p = (T*)q;
-  return cudaMemsetAsync(q, 0, bytes ? bytes : 16, h->stream);
+  h->allocs.push_back(dc_cache::Alloc{q, nb});
+  if (kGuardBytes) {
+    e = cudaMemsetAsync(q, kGuardByte, kGuardBytes, h->stream);
+    if (e == cudaSuccess) e = cudaMemsetAsync((char*)q + kGuardBytes + nb, kGuardByte, kGuardBytes, h->stream);
+    if (e != cudaSuccess) return e;
+  }
+  *p = (T*)((char*)q + kGuardBytes);
+  return cudaMemsetAsync(*p, 0, nb, h->stream);
+}
+
+// Frees one buffer of the handle (nullptr: nothing) and clears the pointer.
+template <class T>
+void dfree(dc_cache* h, T** p) {
+  if (!*p) return;
+  char* base = (char*)*p - kGuardBytes;
+  for (size_t i = 0; i < h->allocs.size(); ++i)
+    if (h->allocs[i].base == base) {
+      cudaFree(base);
+      h->allocs.erase(h->allocs.begin() + (long)i);
+      break;
+    }
+  *p = nullptr;
 }
 
 void free_all(dc_cache* h) {
-  for (void* p : h->allocs) cudaFree(p);
+  for (const auto& a : h->allocs) cudaFree(a.base);
   h->allocs.clear();
+}
+
+// A failed allocation after creation: DC_ERR_OOM (the handle stays usable and
+// unchanged), any other CUDA error as usual.
+dc_status alloc_fail(dc_cache* h, cudaError_t e, const char* what) {
+  if (e == cudaErrorMemoryAllocation) {
+    cudaGetLastError();
+    return fail(h, DC_ERR_OOM, std::string(what) + ": device allocation failed: " + cudaGetErrorString(e));
+  }
+  return cuda_fail(h, e, what);
 }
 
 // Split count and chunk (a multiple of 128 tokens) for n tokens per row.
@@ -406,6 +461,7 @@ dc_status dc_cache_create(int layers, int kv_heads, int head_dim, int capacity, 
   A(&h->st_out, (size_t)R * G * head_dim * sizeof(float));
   if (ae != cudaSuccess) {
     cudaGetLastError();
+    cudaStreamSynchronize(h->stream);  // the zeroing of what was taken
     free_all(h);
     std::string m = std::string("device allocation failed: ") + cudaGetErrorString(ae);
     delete h;
@@ -439,11 +495,18 @@ dc_status dc_cache_create(int layers, int kv_heads, int head_dim, int capacity, 
     } else {
       cudaGetLastError();
       h->fused_why = why;
-      if (cfg.engine == 2) e = fe;
+      // out of memory is reported as such; another failure (e.g. a tensor
+      // map the driver rejects) leaves the split engine, unless the fused
+      // engine was asked for
+      if (cfg.engine == 2 || fe == cudaErrorMemoryAllocation) e = fe;
     }
   }
   if (e != cudaSuccess) {
-    dc_status s = cuda_fail(nullptr, e, "policy upload");
+    const bool oom = e == cudaErrorMemoryAllocation;
+    dc_status s = oom ? fail(nullptr, DC_ERR_OOM, std::string("device allocation failed: ") + cudaGetErrorString(e))
+                      : cuda_fail(nullptr, e, "policy upload");
+    cudaGetLastError();
+    cudaStreamSynchronize(h->stream);
     free_all(h);
     delete h;
     return s;
@@ -541,6 +604,7 @@ dc::FusedStep fused_args(dc_cache* h, const dc::Step& st, const void* q, float* 
   fs.xo = h->xo;
   fs.xsel = h->xsel;
   fs.xflag = h->xflag;
+  fs.xslots = h->xflag ? (int)std::min<long long>(h->dev.R, h->num_sms) + 1 : 0;
   fs.work = h->work;
   fs.half_rows = (h->xflag && !h->per_row) ? dc::fused_half_rows(h->dev, st.n, fs, h->num_sms) : 0;
   // launch epoch: the queue counter is work[epoch & 1]; exchange flags hold
@@ -567,6 +631,7 @@ dc_status graph_step(dc_cache* h, const void* q, const void* k_new, const void* 
   fs.xo = h->xo;
   fs.xsel = h->xsel;
   fs.xflag = h->xflag;
+  fs.xslots = h->xflag ? (int)std::min<long long>(h->dev.R, h->num_sms) + 1 : 0;
   fs.work = h->work;
   fs.half_rows = h->xflag ? dc::fused_half_rows(h->dev, h->gstep.n, fs, h->num_sms) : 0;
   fs.epoch = h->gepoch;
@@ -643,13 +708,8 @@ dc_status update_row_order(dc_cache* h) {
     for (int i = 0; i + 1 < R && sorted; ++i) sorted = tiles(h->horder[i]) >= tiles(h->horder[i + 1]);
     if (sorted) return DC_OK;
   }
-  if (!h->horder) {
-    DC_CUDA(h, cudaHostAlloc(reinterpret_cast<void**>(&h->horder), (size_t)R * sizeof(int), cudaHostAllocDefault));
-    DC_CUDA(h, dalloc(h, &h->roworder_dev, (size_t)R * sizeof(int)));
-    DC_CUDA(h, cudaEventCreateWithFlags(&h->ev_order, cudaEventDisableTiming));
-  } else {
-    DC_CUDA(h, cudaEventSynchronize(h->ev_order));
-  }
+  // the buffers come with the per-row budgets (dc_set_row_budgets)
+  DC_CUDA(h, cudaEventSynchronize(h->ev_order));
   for (int r = 0; r < R; ++r) h->horder[r] = r;
   std::stable_sort(h->horder, h->horder + R, [&](int a, int b) { return tiles(a) > tiles(b); });
   DC_CUDA(h, cudaMemcpyAsync(h->roworder_dev, h->horder, (size_t)R * sizeof(int), cudaMemcpyHostToDevice,
@@ -771,10 +831,18 @@ dc_status dc_step_host_async(dc_cache* h, const void* q, const void* k_new, cons
   if (!q || !k_new || !v_new || !out) return fail(h, DC_ERR_INVALID_ARG, "NULL pointer");
   const size_t R = h->dev.R, G = h->dev.G, d = h->dev.d;
   if (!h->h2d) {
-    DC_CUDA(h, dalloc(h, &h->st2_q, R * G * d * 2));
-    DC_CUDA(h, dalloc(h, &h->st2_k, R * d * 2));
-    DC_CUDA(h, dalloc(h, &h->st2_v, R * d * 2));
-    DC_CUDA(h, dalloc(h, &h->st2_out, R * G * d * sizeof(float)));
+    cudaError_t ae = dalloc(h, &h->st2_q, R * G * d * 2);
+    if (ae == cudaSuccess) ae = dalloc(h, &h->st2_k, R * d * 2);
+    if (ae == cudaSuccess) ae = dalloc(h, &h->st2_v, R * d * 2);
+    if (ae == cudaSuccess) ae = dalloc(h, &h->st2_out, R * G * d * sizeof(float));
+    if (ae != cudaSuccess) {
+      cudaStreamSynchronize(h->stream);
+      dfree(h, &h->st2_q);
+      dfree(h, &h->st2_k);
+      dfree(h, &h->st2_v);
+      dfree(h, &h->st2_out);
+      return alloc_fail(h, ae, "second staging set");
+    }
     DC_CUDA(h, cudaStreamCreateWithFlags(&h->h2d, cudaStreamNonBlocking));
     DC_CUDA(h, cudaStreamCreateWithFlags(&h->d2h, cudaStreamNonBlocking));
     for (int i = 0; i < 2; ++i) {
@@ -924,8 +992,21 @@ dc_status dc_set_row_budgets(dc_cache* h, const int* budgets, int n) {
   for (int r = 0; r < n; ++r)
     if (budgets[r] < 1) return fail(h, DC_ERR_INVALID_ARG, "budgets must be >= 1");
   if (!h->rowlen_dev) {
-    DC_CUDA(h, dalloc(h, &h->rowlen_dev, (size_t)n * sizeof(int)));
-    DC_CUDA(h, dalloc(h, &h->rowbudget_dev, (size_t)n * sizeof(int)));
+    // row lengths, budgets and the fused queue's row order (device), with the
+    // order's pinned host copy and the event of its last upload
+    cudaError_t ae = dalloc(h, &h->rowlen_dev, (size_t)n * sizeof(int));
+    if (ae == cudaSuccess) ae = dalloc(h, &h->rowbudget_dev, (size_t)n * sizeof(int));
+    if (ae == cudaSuccess) ae = dalloc(h, &h->roworder_dev, (size_t)n * sizeof(int));
+    if (ae != cudaSuccess) {
+      cudaStreamSynchronize(h->stream);
+      dfree(h, &h->rowlen_dev);
+      dfree(h, &h->rowbudget_dev);
+      dfree(h, &h->roworder_dev);
+      return alloc_fail(h, ae, "per-row budgets");
+    }
+    DC_CUDA(h, cudaHostAlloc(reinterpret_cast<void**>(&h->horder), (size_t)n * sizeof(int), cudaHostAllocDefault));
+    DC_CUDA(h, cudaEventCreateWithFlags(&h->ev_order, cudaEventDisableTiming));
+    DC_CUDA(h, cudaEventRecord(h->ev_order, h->stream));
   }
   if (!h->per_row) {
     h->hlen.assign(n, h->n);
@@ -957,7 +1038,14 @@ dc_status dc_set_graph_mode(dc_cache* h, int enable) {
         return fail(h, DC_ERR_STATE, "graph mode needs the window's last steps to be consecutive decode steps");
     if (!use_fused(h, h->n + 1)) return fail(h, DC_ERR_STATE, "graph mode runs on the fused engine only");
     if (h->seen + (1ll << 30) > 0x7FFFFFFFll) return fail(h, DC_ERR_CAPACITY, "position counter too close to its limit");
-    if (!h->gcount_dev) DC_CUDA(h, dalloc(h, &h->gcount_dev, 2 * sizeof(int)));
+    if (!h->gcount_dev) {
+      cudaError_t ae = dalloc(h, &h->gcount_dev, 2 * sizeof(int));
+      if (ae != cudaSuccess) {
+        cudaStreamSynchronize(h->stream);
+        dfree(h, &h->gcount_dev);
+        return alloc_fail(h, ae, "graph mode step counter");
+      }
+    }
     DC_CUDA(h, cudaMemsetAsync(h->gcount_dev, 0, 2 * sizeof(int), h->stream));
     h->gstep = begin_step(h);
     h->gepoch = h->epoch + 1;
@@ -1063,11 +1151,48 @@ dc_status dc_sync(dc_cache* h) {
   DC_CUDA(h, cudaMemcpy(&st, h->dev.status, sizeof st, cudaMemcpyDeviceToHost));
   DC_CUDA(h, cudaMemcpy(dbg, h->dev.dbg, sizeof dbg, cudaMemcpyDeviceToHost));
   if (st) {
-    char buf[160];
-    std::snprintf(buf, sizeof buf, "kernel status word 0x%x (first wait timeout: site %u block %u parity %u info 0x%x)",
-                  st, dbg[1], dbg[2], dbg[3], dbg[4]);
+    char buf[256];
+    std::snprintf(buf, sizeof buf,
+                  "kernel status word 0x%x (first wait timeout: site %u block %u parity %u info 0x%x; "
+                  "first failed index check: site %u index %u limit %u)",
+                  st, dbg[1], dbg[2], dbg[3], dbg[4], dbg[5], dbg[6], dbg[7]);
     return fail(h, DC_ERR_DEVICE, buf);
   }
+  if (kGuardBytes) {
+    // debug builds: the guard regions around every buffer are intact
+    std::vector<unsigned char> g(kGuardBytes);
+    for (size_t a = 0; a < h->allocs.size(); ++a) {
+      for (int side = 0; side < 2; ++side) {
+        const char* at = (const char*)h->allocs[a].base + (side ? kGuardBytes + h->allocs[a].bytes : 0);
+        DC_CUDA(h, cudaMemcpy(g.data(), at, kGuardBytes, cudaMemcpyDeviceToHost));
+        for (size_t i = 0; i < kGuardBytes; ++i)
+          if (g[i] != kGuardByte) {
+            char buf[160];
+            std::snprintf(buf, sizeof buf, "guard region %s buffer %zu (%zu bytes) overwritten at byte %zu",
+                          side ? "after" : "before", a, h->allocs[a].bytes, i);
+            return fail(h, DC_ERR_DEVICE, buf);
+          }
+      }
+    }
+  }
+  return DC_OK;
+}
+
+dc_status dc_debug_fail_alloc(long long nth) {
+  g_alloc_index.store(0);
+  g_fail_alloc_at.store(nth < 0 ? -1 : nth);
+  return DC_OK;
+}
+
+int dc_debug_checks(void) { return kGuardBytes ? 1 : 0; }
+
+dc_status dc_debug_corrupt_guard(dc_cache* h) {
+  DC_CHECK_HANDLE(h);
+  if (!kGuardBytes || h->allocs.empty()) return fail(h, DC_ERR_STATE, "not a debug build (DC_DEBUG_BOUNDS)");
+  // the first byte of the guard region after the first buffer (K): memory the
+  // handle owns, outside every buffer
+  char* at = (char*)h->allocs[0].base + kGuardBytes + h->allocs[0].bytes;
+  DC_CUDA(h, cudaMemsetAsync(at, (unsigned char)~kGuardByte, 1, h->stream));
   return DC_OK;
 }
 

@@ -33,6 +33,28 @@ constexpr int kWarp = 32;
 // Device status word bits (read back by dc_sync).
 constexpr unsigned kStatusBadShape = 1u;
 constexpr unsigned kStatusTimeout = 2u;
+constexpr unsigned kStatusBounds = 4u;  // debug builds: an index check failed
+
+// Debug builds (DC_DEBUG_BOUNDS) check computed global-memory indices before
+// the access: DC_INB(p, i, lim, site) is false when i is outside [0, lim),
+// after raising kStatusBounds and recording the first failure (site, low 32
+// bits of the index, limit) in dbg[5..7]; the caller then skips the access.
+// Release builds compile it to `true`.
+#ifdef DC_DEBUG_BOUNDS
+__device__ __forceinline__ bool in_bounds(long long i, long long lim, unsigned* status, unsigned* dbg,
+                                          unsigned site) {
+  if (i >= 0 && i < lim) return true;
+  if (status) atomicOr(status, kStatusBounds);
+  if (dbg && atomicCAS(dbg + 5, 0u, site) == 0u) {
+    dbg[6] = (unsigned)i;
+    dbg[7] = (unsigned)lim;
+  }
+  return false;
+}
+#define DC_INB(p, i, lim, site) ::dc::in_bounds((long long)(i), (long long)(lim), (p).status, (p).dbg, (site))
+#else
+#define DC_INB(p, i, lim, site) true
+#endif
 
 struct Dev {
   int R, cap, stride, d, G, qh, kvh, w, hidden, layernorm, alpha_mode, keep_features;

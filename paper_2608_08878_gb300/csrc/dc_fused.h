@@ -39,6 +39,7 @@ struct FusedStep {
   float* xo;         // [half_rows][G][d]
   int* xsel;         // [half_rows][2][4]
   unsigned* xflag;   // [half_rows][2]
+  int xslots;        // exchange slots allocated (bounds of the four above)
 };
 
 // Exchange buffer sizes (floats / ints) for a grid of `grid` CTAs.

@@ -435,7 +435,10 @@ __global__ void __launch_bounds__(kThreads, 1)
         // The current query also takes over the departing query's ring slot:
         // each lane reads the departing element before it writes the same one.
         __nv_bfloat16* ring_slot = p.ring_q + ((size_t)rq * p.w + st.slot) * G * D;
-        for (int e = lane; e < G * (D / 8); e += kWarp) {
+        const bool q_ok = DC_INB(p, qo + G * D - 1, (long long)(p.R / p.kvh) * p.qh * D, 101) &&
+                          DC_INB(p, ((long long)rq * p.w + st.slot) * G * D + G * D - 1, (long long)p.R * p.w * G * D, 102) &&
+                          DC_INB(p, ((long long)rq * p.w + st.slot_prev) * G * D, (long long)p.R * p.w * G * D, 103);
+        for (int e = lane; q_ok && e < G * (D / 8); e += kWarp) {
           const int h = e / (D / 8), kc = e % (D / 8);
           const uint4 cur = reinterpret_cast<const uint4*>(fs.q + qo + h * D)[kc];
           const uint4 pv = st.has_prev ? reinterpret_cast<const uint4*>(prev + h * D)[kc] : make_uint4(0, 0, 0, 0);
@@ -466,10 +469,17 @@ __global__ void __launch_bounds__(kThreads, 1)
             const uint32_t kv_bytes = nbox ? (uint32_t)nbox * 16u * (uint32_t)D * 2u : kTileBytes;
             const uint32_t pos_bytes = ((uint32_t)valid * 4u + 15u) & ~15u, sz_bytes = (uint32_t)valid * 16u;
             const uint32_t aux_bytes = (pass || FULL) ? 0u : pos_bytes + (GLOB ? 0u : sz_bytes);
-            mbar_expect_tx(&bar[B_FULL + s], kv_bytes + aux_bytes);
             uint8_t* dst = smem + OFF_STAGE + s * kStageBytes;
             uint8_t* aux = smem + OFF_AUX + s * kAuxBytes;
             const int y = rt * p.stride + j * kTok;
+            if (!DC_INB(p, (long long)y + kTok - 1, (long long)p.R * p.stride, 104)) {
+              // (debug builds) the tile lies outside the buffers: no copy; a
+              // plain arrival completes the stage's phase with stale contents
+              mbar_arrive(&bar[B_FULL + s]);
+              issued = g + 1;
+              continue;
+            }
+            mbar_expect_tx(&bar[B_FULL + s], kv_bytes + aux_bytes);
             if (nbox == 0) {
               tma_load_2d(dst, tm, 0, y, &bar[B_FULL + s], pol);
               if (D == 128) tma_load_2d(dst + 16384, tm, 64, y, &bar[B_FULL + s], pol);
@@ -638,6 +648,13 @@ __global__ void __launch_bounds__(kThreads, 1)
       const int Bsel = PERROW ? (fs.B > 0 ? fs.B : p.rowbudget[r]) : fs.B;
       const int ts = r - (p.R - fs.half_rows);  // exchange slot (half rows only)
       const size_t rbase = (size_t)r * p.stride;
+      // (debug builds) slot i of this row inside the row and the buffers
+      const long long RS = (long long)p.R * p.stride;
+      auto slot_ok = [&](long long i, unsigned site) {
+        return DC_INB(p, i, p.stride, site) && DC_INB(p, (long long)rbase + i, RS, site);
+      };
+      (void)RS;
+      const bool x_ok = it.half < 0 || (DC_INB(p, ts, fs.xslots, 110) && DC_INB(p, ts, fs.half_rows, 110));
       // a row longer than the shared score array keeps its scores in HBM when
       // the radix select reads them (several evictions), or when asked to
       const bool spill_scores = LONG && n > kFusedMaxTok && fs.do_evict && Bsel < n - 1;
@@ -686,14 +703,14 @@ __global__ void __launch_bounds__(kThreads, 1)
             const float mp = (st.has_prev && pos <= st.p_prev) ? 1.f : 0.f;
             const float md = (st.has_dep && pos <= st.p_dep) ? 1.f : 0.f;
             sz = window_update(sz, sp * mp, sd * md, zp * mp, zd * md);
-            p.SZ[rbase + i] = sz;
+            if (slot_ok(i, 105)) p.SZ[rbase + i] = sz;
           }
         }
         if (!LONG || j < onchip_tiles<GS>()) {
           scw[i] = S16[G - 1];
           __syncwarp();
           stash_store<GS>(lane_addr + stash_at(j), S16);
-        } else {
+        } else if (slot_ok(i, 106)) {
           store_logits<G>(p.logit + (rbase + i) * G, S16);
         }
       }
@@ -772,7 +789,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       unsigned* my_flag = half >= 0 ? fs.xflag + 2 * ts + half : nullptr;
       const unsigned* peer_flag = half >= 0 ? fs.xflag + 2 * ts + (half ^ 1) : nullptr;
       const unsigned ep = fs.epoch * 4u;
-      if (half >= 0) {
+      if (half >= 0 && x_ok) {
         // half row: swap the partial statistics with the other half, then
         // both merge half 0's before half 1's (identical results on both)
         float4* xs = reinterpret_cast<float4*>(fs.xstats);
@@ -801,7 +818,10 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         // half 1 has read the departing query and statistics (it published
         // after its K pass): half 0 may now give their ring slot to this step
-        if (!FULL && half == 0) {
+        if (!FULL && half == 0 && DC_INB(p, ((long long)r * p.w + st.slot) * G * D + G * D - 1,
+                                         (long long)p.R * p.w * G * D, 119) &&
+            DC_INB(p, (long long)((r / p.kvh) * p.qh + (r % p.kvh) * G) * D + G * D - 1,
+                   (long long)(p.R / p.kvh) * p.qh * D, 119)) {
           const int qo = ((r / p.kvh) * p.qh + (r % p.kvh) * G) * D;
           uint4* ring_slot = reinterpret_cast<uint4*>(p.ring_q + ((size_t)r * p.w + st.slot) * G * D);
           for (int e = etid; e < G * (D / 8); e += kEpi) ring_slot[e] = reinterpret_cast<const uint4*>(fs.q + qo)[e];
@@ -818,7 +838,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
       // push (m, l, H, -log2 l) of this step into the ring slot it takes over
       // (the producer, or half 0 above, wrote the query there)
-      if (!FULL && tid < G && half <= 0) {
+      if (!FULL && tid < G && half <= 0 && DC_INB(p, (long long)r * p.w + st.slot, (long long)p.R * p.w, 109)) {
         float4 v;
         v.x = M[tid]; v.y = L0; v.z = Hh[tid]; v.w = NL[tid];
         reinterpret_cast<float4*>(p.ring_stats)[((size_t)r * p.w + st.slot) * G + tid] = v;
@@ -829,7 +849,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       // (its window sums were written before the merge barrier), so that the
       // select does not wait on it; what the V pass may still write is loaded
       // at the select.
-      const bool single_evict = fs.do_evict && n == Bsel + 1;
+      const bool single_evict = fs.do_evict && n == Bsel + 1 && slot_ok(Bsel, 116);
       SlotCopy mv{};
       if (single_evict && half != 0 && tid < kWarp) slot_load_settled(p, rbase + Bsel, tid, fs.write_scores, mv);
 
@@ -845,7 +865,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         posA = posB;
         vnA = vnB;
         acA = acB;
-        if (!FULL && j + 2 * JS < t1) {
+        if (!FULL && j + 2 * JS < t1 && slot_ok((j + 2 * JS) * kTok + tok, 107)) {
           if constexpr (!GLOB) {
             szB = szrow[(j + 2 * JS) * kTok];
             posB = posrow[(j + 2 * JS) * kTok];
@@ -860,7 +880,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           stash_load<GS>(lane_addr + stash_at(j), sv);
           if constexpr (GS > 0) tmem_ld_wait();
           sv[G - 1] = scw[i];
-        } else {
+        } else if (slot_ok(i, 108)) {
           load_logits<G>(p.logit + (rbase + i) * G, sv);
         }
         float a[G], zc = 0.f, scur = 0.f;
@@ -897,7 +917,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         if constexpr (FULL) return make_float2(0.f, 0.f);
         if constexpr (GLOB) {
           // this row's share of the token's pooled sums
-          if (valid) {
+          if (valid && slot_ok(i, 111)) {
             float a2 = 0.f;
 #pragma unroll
             for (int h = 0; h < G; ++h) a2 = fmaf(a[h], a[h], a2);
@@ -913,7 +933,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         const float Zt = __fadd_rn(__fadd_rn(sz.z, zc), sz.w);
         const float St = __fadd_rn(__fadd_rn(sz.x, scur), sz.y);
         float x[5] = {mean, vn, var, Zt > 0.f ? St / Zt : 0.f, (float)pos / pos_den};
-        if (valid) {
+        if (valid && slot_ok(i, 112)) {
           const size_t slot = rbase + i;
           if (p.alpha_mode == 1) {
             x[0] = (ac_ahead ? ac : p.acc[slot]) + mean;
@@ -995,7 +1015,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         __syncwarp();
         if (lane == 0) mbar_arrive(&bar[B_MEMPTY + pb]);
         const int i = j * kTok + tok;
-        if (i < n) {
+        if (i < n && slot_ok(i, 113)) {
           const float score = fp.b2 + relu_sum;
           if constexpr (LONG) {
             if (spill_scores || fs.write_scores) p.score[rbase + i] = score;
@@ -1016,7 +1036,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       // the score of a heuristic scorer, recorded like finish() records the policy's
       auto record_h = [&](int j, float score, int pos) {
         const int i = j * kTok + tok;
-        if (i < n) {
+        if (i < n && slot_ok(i, 114)) {
           if (spill_scores || fs.write_scores) p.score[rbase + i] = score;
           if (n <= kFusedMaxTok) scw[i] = score;
           const uint32_t kk = score_key(score);
@@ -1053,13 +1073,13 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (lane == 0) mbar_arrive(&bar[B_OEMPTY]);
 #pragma unroll
         for (int h = 0; h < G; ++h) ov[h] = o16[h] + o16[G + h];
-        if (half == 1 && tok < D) {
+        if (half == 1 && tok < D && x_ok) {
 #pragma unroll
           for (int h = 0; h < G; ++h) fs.xo[((size_t)ts * G + h) * D + tok] = ov[h];
           __threadfence();
         }
       }
-      if (half >= 0) {
+      if (half >= 0 && x_ok) {
         sync();
         if (etid == 0) {
           if (half == 1) flag_release(my_flag, ep + 2u);
@@ -1067,7 +1087,9 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         sync();
       }
-      if ((PAIR || wg == 0) && half <= 0 && tok < D) {
+      if ((PAIR || wg == 0) && half <= 0 && tok < D && x_ok &&
+          DC_INB(p, (long long)((r / p.kvh) * p.qh + (r % p.kvh) * G) * D + (G - 1) * D + tok,
+                 (long long)(p.R / p.kvh) * p.qh * D, 115)) {
         float* op = fs.out + ((r / p.kvh) * p.qh + (r % p.kvh) * G) * D;
 #pragma unroll
         for (int h = 0; h < G; ++h)
@@ -1106,7 +1128,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             if (lower(fk, fe, fpos, (uint32_t)scr.best[w], scr.best_slot[w], scr.hist[w])) {
               fk = (uint32_t)scr.best[w]; fe = scr.best_slot[w]; fpos = scr.hist[w];
             }
-          if (half >= 0) {
+          if (half >= 0 && x_ok) {
             int* xs = fs.xsel + (2 * ts + half) * 4;
             xs[0] = (int)fk; xs[1] = fe; xs[2] = fpos;
             __threadfence();
@@ -1125,7 +1147,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         sync();
         const int e = scr.sh[0];
-        if (mover && e >= 0 && e < Bsel && tid < kWarp) slot_store(p, rbase + e, tid, mv);
+        if (mover && e >= 0 && e < Bsel && tid < kWarp && slot_ok(e, 117)) slot_store(p, rbase + e, tid, mv);
         sync();
       } else if (fs.do_evict && Bsel < n) {
         // several evictions (whole rows only): radix select over the scores
@@ -1133,7 +1155,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         team_select_compact<kTeam>(p, r, n, Bsel, LONG && n > kFusedMaxTok ? p.score + rbase : scw, tid, scr,
                                    sync);
       }
-      if (PERROW && fs.do_evict && tid == 0) p.rowlen[r] = n < Bsel ? n : Bsel;
+      if (PERROW && fs.do_evict && tid == 0 && DC_INB(p, r, p.R, 118)) p.rowlen[r] = n < Bsel ? n : Bsel;
     }
   }
   __syncthreads();

@@ -17,19 +17,33 @@
 namespace dc {
 namespace {
 
-constexpr int kFeatTok = 64;     // tokens per block
-constexpr int kFeatGroups = 4;   // threads per token, each summing a quarter of the rows
+// The pooling is bound by the latency of each thread's chain of loads (one
+// per row it sums), so every token gets 16 threads, each summing 1/16 of the
+// sequence's rows (16 of 256 at the Mistral-7B shape).
+constexpr int kFeatTok = 32;     // tokens per block
+constexpr int kFeatGroups = 16;  // threads per token, each summing 1/16 of the rows
 constexpr int kFeatThreads = kFeatTok * kFeatGroups;
+constexpr int kPoolBatch = 8;    // rows whose partial sums a thread loads at once
 constexpr int kSelThreads = 1024;
 constexpr int kMoveThreads = 256;
 
+// A streaming 16-byte load (evict-first: read once) that the compiler keeps
+// in program order with the other loads of its batch.
+__device__ __forceinline__ float4 ld_stream(const float4* a) {
+  float4 v;
+  asm volatile("ld.global.cs.v4.f32 {%0, %1, %2, %3}, [%4];"
+               : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w)
+               : "l"(a));
+  return v;
+}
+
 __device__ __forceinline__ int seq_row(const Dev& p, int b, int l, int g) { return (l * p.batch + b) * p.kvh + g; }
 
-// grid (ceil(n / 64), batch), block 256 = 64 tokens x 4 row groups; dynamic
-// shared memory: the policy blob, then the groups' partial sums.
-// The rows of a sequence are taken in a fixed order (layer-major, then KV
-// head): group q sums rows [q S / 4, (q + 1) S / 4) in that order, and the four
-// partials are added in group order.
+// grid (ceil(n / kFeatTok), batch), block kFeatTok tokens x kFeatGroups row
+// groups; dynamic shared memory: the policy blob, then the groups' partial
+// sums. The rows of a sequence are taken in a fixed order (layer-major, then
+// KV head): group q sums rows [q S / kFeatGroups, (q + 1) S / kFeatGroups) in
+// that order, and the partials are added in group order.
 __global__ void __launch_bounds__(kFeatThreads) glob_feature_kernel(Dev p, Step st) {
   extern __shared__ float wsm[];
   const int H = p.hidden, nblob = 9 * H + 1;
@@ -41,8 +55,28 @@ __global__ void __launch_bounds__(kFeatThreads) glob_feature_kernel(Dev p, Step 
   if (i < st.n) {
     const int S = p.seq_rows, r0 = grp * S / kFeatGroups, r1 = (grp + 1) * S / kFeatGroups;
     int l = r0 / p.kvh, g = r0 % p.kvh;
-    for (int rr = r0; rr < r1; ++rr) {
-      const float4 q = p.gpart[(size_t)seq_row(p, b, l, g) * p.stride + i];
+    // the partial sums of kPoolBatch rows are loaded before any is added (the
+    // loads are independent; only the adds are ordered), so that a thread
+    // keeps that many loads in flight
+    int rr = r0;
+    for (; rr + kPoolBatch <= r1; rr += kPoolBatch) {
+      float4 q[kPoolBatch];
+#pragma unroll
+      for (int u = 0; u < kPoolBatch; ++u) {
+        q[u] = ld_stream(&p.gpart[(size_t)seq_row(p, b, l, g) * p.stride + i]);
+        // the next row without a branch, so that the batch's loads can issue
+        // back to back
+        const int wrap = (g + 1 == p.kvh) ? 1 : 0;
+        g = wrap ? 0 : g + 1;
+        l += wrap;
+      }
+#pragma unroll
+      for (int u = 0; u < kPoolBatch; ++u) {
+        P.x += q[u].x; P.y += q[u].y; P.z += q[u].z; P.w += q[u].w;
+      }
+    }
+    for (; rr < r1; ++rr) {
+      const float4 q = __ldcs(&p.gpart[(size_t)seq_row(p, b, l, g) * p.stride + i]);
       P.x += q.x; P.y += q.y; P.z += q.z; P.w += q.w;
       if (++g == p.kvh) { g = 0; ++l; }
     }

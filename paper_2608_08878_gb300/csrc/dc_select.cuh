@@ -93,6 +93,82 @@ __device__ uint32_t team_radix_select(int n, int need, KeyF keyf, Pred pred, int
   return prefix;
 }
 
+// team_radix_select for large teams over keys in shared memory (the eviction
+// kernel): the lanes of a warp that share a histogram bin add to it once, and
+// one warp finds the digit with a prefix sum over its lanes instead of one
+// thread walking the 256 bins. Needs whole warps (every lane of every team
+// warp calls it) and 1 <= need <= the number of elements with pred. (The
+// fused kernel keeps the plain form: this one needs more registers.)
+template <int NT, class KeyF, class Pred, class Sync>
+__device__ uint32_t team_radix_select_wide(int n, int need, KeyF keyf, Pred pred, int tid,
+                                      const SelectScratch& s, int* gt, Sync sync) {
+  uint32_t prefix = 0, mask = 0;
+  int above = 0;
+  const int lane = tid % kWarp;
+  for (int shift = 24; shift >= 0; shift -= 8) {
+    for (int b = tid; b < 256; b += NT) s.hist[b] = 0;
+    sync();
+    // histogram of the next digit among the keys that match the prefix; the
+    // lanes of a warp that share a bin add to it once (scores cluster in a
+    // few bins, where one atomic per lane would serialise)
+    for (int i0 = 0; i0 < n; i0 += NT) {
+      const int i = i0 + tid;
+      unsigned bin = 256u;
+      if (i < n && pred(i)) {
+        const uint32_t k = keyf(i);
+        if ((k & mask) == prefix) bin = (k >> shift) & 255u;
+      }
+      const unsigned peers = __match_any_sync(0xffffffffu, bin);
+      if (bin < 256u && lane == __ffs(peers) - 1) atomicAdd(&s.hist[bin], __popc(peers));
+    }
+    sync();
+    if (tid < kWarp) {
+      // the digit: the highest bin where the count of larger-or-equal keys
+      // reaches `need`. Lane L holds bins 255 - 8L - j (j = 0..7, descending);
+      // a prefix sum over the lanes finds the lane, the lane finds the bin.
+      int c[8], tot = 0;
+#pragma unroll
+      for (int j = 0; j < 8; ++j) {
+        c[j] = s.hist[255 - 8 * lane - j];
+        tot += c[j];
+      }
+      int inc = tot;
+#pragma unroll
+      for (int off = 1; off < kWarp; off <<= 1) {
+        const int y = __shfl_up_sync(0xffffffffu, inc, off);
+        if (lane >= off) inc += y;
+      }
+      const unsigned hit = __ballot_sync(0xffffffffu, above + inc >= need);
+      const int all = __shfl_sync(0xffffffffu, inc, kWarp - 1);
+      if (hit == 0u) {
+        if (lane == 0) {  // fewer keys than `need` (not reached for valid arguments)
+          s.sh[0] = 0;
+          s.sh[1] = above + all;
+        }
+      } else if (lane == __ffs(hit) - 1) {
+        int cum = above + inc - tot, dgt = 255 - 8 * lane - 7;
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+          if (cum + c[j] >= need) {
+            dgt = 255 - 8 * lane - j;
+            break;
+          }
+          cum += c[j];
+        }
+        s.sh[0] = dgt;
+        s.sh[1] = cum;
+      }
+    }
+    sync();
+    prefix |= (uint32_t)s.sh[0] << shift;
+    mask |= 255u << shift;
+    above = s.sh[1];
+    sync();
+  }
+  *gt = above;
+  return prefix;
+}
+
 // One slot's contents held by a warp: lane l keeps 16-byte chunk l of the
 // slot's [K | V] row (d / 4 chunks) and per-token field l: 0 position, 1 |v|,
 // 2 window sums, 3 score, 4 cumulative alpha, 5..9 features. Every lane loads
@@ -175,15 +251,21 @@ __device__ __forceinline__ void move_slot_1(const Dev& p, size_t src, size_t dst
     for (int e = 0; e < 5; ++e) p.feat[dst * 5 + e] = p.feat[src * 5 + e];
 }
 
-// Keeps the top B of the row's n tokens (scores from `score`, length n) and
+// K/V rows a warp of the list-based compaction loads before it stores them.
+constexpr int kMoveUnroll = 6;
+
+// Keeps the top B of the row's n tokens (order keys keyf(i), i < n) and
 // compacts them into slots [0, B). Requires 1 <= B < n. All NT threads of the
-// team call it.
-template <int NT, class Sync>
-__device__ void team_select_compact(const Dev& p, int r, int n, int B, const float* score, int tid,
-                                    const SelectScratch& s, Sync sync) {
+// team call it. Two compactions: WARP_MOVES (the eviction kernel, many moves):
+// hole and mover lists built with ballots, then each warp copies several
+// slots at a time; otherwise (the fused kernel's epilogue, where registers
+// are scarce) chunks of NT candidate slots are ranked with a team scan and
+// each mover thread copies its slot.
+template <int NT, bool WARP_MOVES, class KeyF, class Sync>
+__device__ void team_select_compact_k(const Dev& p, int r, int n, int B, KeyF key, int tid,
+                                      const SelectScratch& s, Sync sync) {
   const size_t base = (size_t)r * p.stride;
   const int* ps = p.pos + base;
-  auto key = [&](int i) { return score_key(score[i]); };
   if (n == B + 1) {
     // One eviction: the lowest-ranked token (smallest score key; among equal
     // keys the highest position). Positions are read only to break ties.
@@ -221,7 +303,11 @@ __device__ void team_select_compact(const Dev& p, int r, int n, int B, const flo
   }
   int gt = 0;
   auto all = [](int) { return true; };
-  const uint32_t T = team_radix_select<NT>(n, B, key, all, tid, s, &gt, sync);
+  auto radix = [&](int nn, int need, auto kf, auto pr, int* g) {
+    if constexpr (WARP_MOVES) return team_radix_select_wide<NT>(nn, need, kf, pr, tid, s, g, sync);
+    else return team_radix_select<NT>(nn, need, kf, pr, tid, s, g, sync);
+  };
+  const uint32_t T = radix(n, B, key, all, &gt);
   const int need_eq = B - gt;
   int eq_local = 0;
   for (int i = tid; i < n; i += NT) eq_local += (key(i) == T);
@@ -232,34 +318,139 @@ __device__ void team_select_compact(const Dev& p, int r, int n, int B, const flo
     auto pkey = [&](int i) { return ~(uint32_t)ps[i]; };
     auto tied = [&](int i) { return key(i) == T; };
     int gt2 = 0;
-    P = team_radix_select<NT>(n, need_eq, pkey, tied, tid, s, &gt2, sync);
+    P = radix(n, need_eq, pkey, tied, &gt2);
   }
   auto keep = [&](int i) {
     const uint32_t k = key(i);
     return k > T || (k == T && ~(uint32_t)ps[i] >= P);
   };
-  int* holes = p.holes + base;
-  int nh = 0;
-  for (int c0 = 0; c0 < B; c0 += NT) {
-    const int i = c0 + tid;
-    const int f = (i < B && !keep(i)) ? 1 : 0;
-    int tot;
-    const int rank = team_exclusive_scan<NT>(f, tid, s.wsum, &tot, sync);
-    if (f) holes[nh + rank] = i;
-    nh += tot;
+  if constexpr (!WARP_MOVES) {
+    int* holes = p.holes + base;
+    int nh = 0;
+    for (int c0 = 0; c0 < B; c0 += NT) {
+      const int i = c0 + tid;
+      const int f = (i < B && !keep(i)) ? 1 : 0;
+      int tot;
+      const int rank = team_exclusive_scan<NT>(f, tid, s.wsum, &tot, sync);
+      if (f && DC_INB(p, nh + rank, B, 201)) holes[nh + rank] = i;
+      nh += tot;
+    }
+    sync();
+    int nm = 0;
+    for (int c0 = B; c0 < n; c0 += NT) {
+      const int i = c0 + tid;
+      const int f = (i < n && keep(i)) ? 1 : 0;
+      int tot;
+      const int rank = team_exclusive_scan<NT>(f, tid, s.wsum, &tot, sync);
+      if (f && nm + rank < nh && DC_INB(p, holes[nm + rank], B, 204)) move_slot_1(p, base + i, base + holes[nm + rank]);
+      nm += tot;
+    }
+    if (tid == 0 && nm != nh) atomicOr(p.status, kStatusBadShape);
+    sync();
+  } else {
+    // Hole and mover lists in ascending slot order: holes (evicted slots below
+    // B) in holes[0, nh), movers (survivors at or above B) in holes[B, B + nm)
+    // (the row's scratch has n >= B + nm entries). Each warp takes a contiguous
+    // run of 32-slot groups: it counts its flags with ballots, the warps' counts
+    // are prefix-summed once, and a second walk writes the indices.
+    int* holes = p.holes + base;
+    int* movers = holes + B;
+    constexpr int NW = NT / kWarp;
+    const int lane = tid % kWarp, wid = tid / kWarp;
+    const int ng = (n + kWarp - 1) / kWarp;
+    const int g0 = (int)((long long)ng * wid / NW), g1 = (int)((long long)ng * (wid + 1) / NW);
+    int ch = 0, cm = 0;
+    for (int gi = g0; gi < g1; ++gi) {
+      const int i = gi * kWarp + lane;
+      const bool kp = i < n && keep(i);
+      ch += __popc(__ballot_sync(0xffffffffu, i < B && !kp));
+      cm += __popc(__ballot_sync(0xffffffffu, i >= B && kp));
+    }
+    if (lane == 0) s.best[wid] = ((unsigned long long)(unsigned)cm << 32) | (unsigned)ch;
+    sync();
+    int hb = 0, mb = 0, nh = 0, nm = 0;
+    for (int w = 0; w < NW; ++w) {
+      const unsigned long long v = s.best[w];
+      const int vh = (int)(unsigned)(v & 0xFFFFFFFFull), vm = (int)(unsigned)(v >> 32);
+      if (w < wid) {
+        hb += vh;
+        mb += vm;
+      }
+      nh += vh;
+      nm += vm;
+    }
+    const unsigned lt = (1u << lane) - 1u;
+    for (int gi = g0; gi < g1; ++gi) {
+      const int i = gi * kWarp + lane;
+      const bool kp = i < n && keep(i);
+      const bool fh = i < B && !kp, fm = i >= B && kp;
+      const unsigned bh = __ballot_sync(0xffffffffu, fh), bm = __ballot_sync(0xffffffffu, fm);
+      if (fh && DC_INB(p, hb + __popc(bh & lt), B, 201)) holes[hb + __popc(bh & lt)] = i;
+      if (fm && DC_INB(p, B + mb + __popc(bm & lt), p.stride, 202)) movers[mb + __popc(bm & lt)] = i;
+      hb += __popc(bh);
+      mb += __popc(bm);
+    }
+    if (tid == 0 && nm != nh) atomicOr(p.status, kStatusBadShape);
+    sync();
+    // The k-th mover fills the k-th hole. Sources are >= B and destinations < B,
+    // so the moves are independent. A warp takes 32 moves at a time: lane l
+    // copies the per-token fields of move l (uniform code, one slot per lane),
+    // then the warp copies the K and V rows, each lane one 16-byte chunk, eight
+    // rows' loads in flight before their stores.
+    const int nmv = nm < nh ? nm : nh;
+    const int VPR = p.d / 8;              // 16-byte chunks per K (or V) row
+    const int rows_per = kWarp / (2 * VPR);  // slots copied per warp instruction
+    const int sub = lane / (2 * VPR), chunk = lane % (2 * VPR);
+    for (int k0 = wid * kWarp; k0 < nmv; k0 += NW * kWarp) {
+      const int k = k0 + lane;
+      const bool live = k < nmv;
+      int src = live ? movers[k] : 0, dst = live ? holes[k] : 0;
+      if (live && !(DC_INB(p, src, p.stride, 203) && DC_INB(p, dst, p.stride, 204))) src = dst = -1;
+      if (live && src >= 0) {
+        const size_t fs = base + src, fd = base + dst;
+        const int ps_ = p.pos[fs];
+        const float vn = p.vnorm[fs];
+        const float4 sz = p.SZ[fs];
+        const float sc = p.score[fs];
+        const float ac = p.acc ? p.acc[fs] : 0.f;
+        p.pos[fd] = ps_;
+        p.vnorm[fd] = vn;
+        p.SZ[fd] = sz;
+        p.score[fd] = sc;
+        if (p.acc) p.acc[fd] = ac;
+        if (p.keep_features)
+          for (int e = 0; e < 5; ++e) p.feat[fd * 5 + e] = p.feat[fs * 5 + e];
+      }
+      const int cnt = nmv - k0 < kWarp ? nmv - k0 : kWarp;
+      const uint4* gk = reinterpret_cast<const uint4*>(chunk < VPR ? p.K : p.V);
+      uint4* gkw = reinterpret_cast<uint4*>(chunk < VPR ? p.K : p.V);
+      const int c = chunk < VPR ? chunk : chunk - VPR;
+      for (int j0 = 0; j0 < cnt; j0 += kMoveUnroll * rows_per) {
+        uint4 v[kMoveUnroll];
+        int d_[kMoveUnroll];
+#pragma unroll
+        for (int u = 0; u < kMoveUnroll; ++u) {
+          const int j = j0 + u * rows_per + sub;
+          const int sj = __shfl_sync(0xffffffffu, src, j & (kWarp - 1));
+          d_[u] = __shfl_sync(0xffffffffu, dst, j & (kWarp - 1));
+          if (j >= cnt || sj < 0) d_[u] = -1;
+          if (d_[u] >= 0) v[u] = gk[(base + sj) * VPR + c];
+        }
+#pragma unroll
+        for (int u = 0; u < kMoveUnroll; ++u)
+          if (d_[u] >= 0) gkw[(base + d_[u]) * VPR + c] = v[u];
+      }
+    }
+    sync();
   }
-  sync();
-  int nm = 0;
-  for (int c0 = B; c0 < n; c0 += NT) {
-    const int i = c0 + tid;
-    const int f = (i < n && keep(i)) ? 1 : 0;
-    int tot;
-    const int rank = team_exclusive_scan<NT>(f, tid, s.wsum, &tot, sync);
-    if (f && nm + rank < nh) move_slot_1(p, base + i, base + holes[nm + rank]);
-    nm += tot;
-  }
-  if (tid == 0 && nm != nh) atomicOr(p.status, kStatusBadShape);
-  sync();
+}
+
+// team_select_compact_k over a score array (shared or global memory), with
+// the per-thread compaction.
+template <int NT, class Sync>
+__device__ void team_select_compact(const Dev& p, int r, int n, int B, const float* score, int tid,
+                                    const SelectScratch& s, Sync sync) {
+  team_select_compact_k<NT, false>(p, r, n, B, [&](int i) { return score_key(score[i]); }, tid, s, sync);
 }
 
 // The same selection as team_select_compact without moving anything: writes

@@ -44,10 +44,62 @@ __global__ void wait_selftest_kernel(const unsigned* never_set, unsigned* out, u
   out[6] = (unsigned)((t2 - t1) / 1000u);
 }
 
+// The index check of debug builds (DC_INB): thread 0 writes buf[i] for an i
+// one past the checked limit `lim`; the check must fail, raise the status bit,
+// record site 903 and skip the write. buf holds lim + 1 elements, so even a
+// check that let the write through would stay inside the allocation.
+__global__ void bounds_selftest_kernel(unsigned* buf, int lim, unsigned* status, unsigned* dbg) {
+  if (threadIdx.x != 0) return;
+  Dev p{};
+  p.status = status;
+  p.dbg = dbg;
+  const int i = lim;
+  if (DC_INB(p, i, lim, 903)) buf[i] = 0xBADu;
+  (void)p;
+}
+
 thread_local std::string g_selftest_error;
 
 }  // namespace
 }  // namespace dc
+
+extern "C" dc_status dc_debug_bounds_selftest(unsigned* result, void* stream) {
+  using namespace dc;
+  if (!result) {
+    g_selftest_error = "NULL pointer";
+    return DC_ERR_INVALID_ARG;
+  }
+#ifndef DC_DEBUG_BOUNDS
+  (void)stream;
+  g_selftest_error = "not a debug build (DC_DEBUG_BOUNDS): the index checks are compiled out";
+  return DC_ERR_STATE;
+#else
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  constexpr int kLim = 64;
+  unsigned* d = nullptr;  // [0, kLim] the buffer, then the status word and dbg[8]
+  cudaError_t e = cudaMalloc(&d, (kLim + 1 + 1 + 8) * sizeof(unsigned));
+  if (e == cudaSuccess) e = cudaMemsetAsync(d, 0, (kLim + 1 + 1 + 8) * sizeof(unsigned), s);
+  if (e == cudaSuccess) {
+    bounds_selftest_kernel<<<1, 32, 0, s>>>(d, kLim, d + kLim + 1, d + kLim + 2);
+    e = cudaGetLastError();
+  }
+  unsigned h[kLim + 1 + 1 + 8] = {};
+  if (e == cudaSuccess) e = cudaMemcpyAsync(h, d, sizeof h, cudaMemcpyDeviceToHost, s);
+  if (e == cudaSuccess) e = cudaStreamSynchronize(s);
+  if (d) cudaFree(d);
+  if (e != cudaSuccess) {
+    g_selftest_error = cudaGetErrorString(e);
+    return DC_ERR_CUDA;
+  }
+  const unsigned* dbg = h + kLim + 2;
+  result[0] = h[kLim + 1];                // status word
+  result[1] = dbg[5];                     // site of the first failed check
+  result[2] = dbg[6];                     // its index
+  result[3] = dbg[7];                     // its limit
+  result[4] = h[kLim] == 0u ? 1u : 0u;    // the write was skipped
+  return DC_OK;
+#endif
+}
 
 extern "C" const char* dc_selftest_last_error(void) { return dc::g_selftest_error.c_str(); }
 

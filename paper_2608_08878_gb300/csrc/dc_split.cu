@@ -30,9 +30,10 @@ __global__ void __launch_bounds__(256) append_kernel(Dev p, const uint4* __restr
   const long long ee = live ? e : pairs - 1;
   const int r = (int)(ee / T), t = (int)(ee % T);
   const size_t src = (size_t)ee * vpr + c;
-  const size_t slot = (size_t)r * p.stride + (p.rowlen ? p.rowlen[r] : n0) + t;
+  const int col = (p.rowlen ? p.rowlen[r] : n0) + t;
+  const size_t slot = (size_t)r * p.stride + col;
   const uint4 kv = k[src], vv = v[src];
-  if (live) {
+  if (live && DC_INB(p, col, p.cap, 301) && DC_INB(p, r, p.R, 301)) {
     reinterpret_cast<uint4*>(p.K)[slot * vpr + c] = kv;
     reinterpret_cast<uint4*>(p.V)[slot * vpr + c] = vv;
   }
@@ -46,7 +47,7 @@ __global__ void __launch_bounds__(256) append_kernel(Dev p, const uint4* __restr
   }
   // xor offsets below vpr stay inside the pair's aligned lane group
   for (int off = 1; off < vpr; off <<= 1) ss += __shfl_xor_sync(0xffffffffu, ss, off);
-  if (live && c == 0) {
+  if (live && c == 0 && DC_INB(p, col, p.cap, 302)) {
     // device-counted steps: positions continue from the steps taken since
     p.pos[slot] = seen0 + t + (p.gcount ? *reinterpret_cast<volatile int*>(p.gcount) : 0);
     p.vnorm[slot] = sqrtf(ss);
@@ -169,7 +170,7 @@ __global__ void __launch_bounds__(kTile) split_qk_kernel(Dev p, Step st,
     __syncthreads();
     load_tile<D>(kt, p.K + ((size_t)r * p.stride + base) * D, rows);
     __syncthreads();
-    if (tid < rows) {
+    if (tid < rows && DC_INB(p, base + tid, p.stride, 311) && DC_INB(p, r, p.R, 311)) {
       const size_t slot = (size_t)r * p.stride + base + tid;
       float s[3 * G];
       dots<D, 3 * G>(&kt[tid][0], qs, s);
@@ -217,7 +218,7 @@ __global__ void __launch_bounds__(kTile) split_qk_kernel(Dev p, Step st,
     float M = -INFINITY, L = 0.f, U = 0.f;
     for (int wv = 0; wv < kTile / kWarp; ++wv) online_merge(M, L, U, red[wv][h][0], red[wv][h][1], red[wv][h][2], c);
     float* pp = p.part + (((size_t)r * p.smax + sp) * G + h) * 4;
-    pp[0] = M; pp[1] = L; pp[2] = U; pp[3] = 0.f;
+    if (DC_INB(p, sp, p.smax, 312)) { pp[0] = M; pp[1] = L; pp[2] = U; pp[3] = 0.f; }
   }
 }
 
@@ -231,6 +232,9 @@ __global__ void split_stats_kernel(Dev p, Step st, const __nv_bfloat16* __restri
   const int r = blockIdx.x, tid = threadIdx.x;
   const int qo = row_q_offset(p, r);
   __nv_bfloat16* rq = p.ring_q + ((size_t)r * p.w + st.slot) * G * D;
+  if (!(DC_INB(p, (long long)r * p.w + st.slot, (long long)p.R * p.w, 316) &&
+        DC_INB(p, (long long)qo + G * D - 1, (long long)(p.R / p.kvh) * p.qh * D, 316)))
+    return;
   for (int e = tid; e < G * D; e += blockDim.x) rq[e] = q[qo + e];
   if (tid < G) {
     const int h = tid;
@@ -281,7 +285,7 @@ __global__ void __launch_bounds__(kTile) split_v_kernel(Dev p, Step st) {
     __syncthreads();
     load_tile<D>(vt, p.V + ((size_t)r * p.stride + base) * D, rows);
     __syncthreads();
-    if (tid < rows) {
+    if (tid < rows && DC_INB(p, base + tid, p.stride, 313) && DC_INB(p, r, p.R, 313)) {
       const size_t slot = (size_t)r * p.stride + base + tid;
       const float* lo = p.logit + slot * G;
       float a[G], mean = 0.f;
@@ -348,7 +352,7 @@ __global__ void __launch_bounds__(kTile) split_v_kernel(Dev p, Step st) {
       }
     }
   }
-  if (owns) {
+  if (owns && DC_INB(p, sp, p.smax, 314)) {
     float* op = p.opart + (((size_t)r * p.smax + sp) * G) * D + o0;
 #pragma unroll
     for (int e = 0; e < OPT; ++e) op[e] = oacc[e];
@@ -365,7 +369,7 @@ __global__ void split_out_kernel(Dev p, Step st, float* __restrict__ out) {
   for (int e = threadIdx.x; e < G * D; e += blockDim.x) {
     float s = 0.f;
     for (int sp = 0; sp < st.nsplit; ++sp) s += p.opart[(((size_t)r * p.smax + sp) * G) * D + e];
-    out[row_q_offset(p, r) + e] = s;
+    if (DC_INB(p, row_q_offset(p, r) + e, (long long)(p.R / p.kvh) * p.qh * D, 315)) out[row_q_offset(p, r) + e] = s;
   }
 }
 

@@ -15,7 +15,10 @@ import threading
 import numpy as np
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
-LIB_PATH = os.path.join(_HERE, "libdistillcache.so")
+# DC_LIBRARY=debug selects the build with device-side index checks and guard
+# regions (build.build_debug); the default is the release library.
+LIB_PATH = os.path.join(_HERE, "libdistillcache_debug.so" if os.environ.get("DC_LIBRARY") == "debug"
+                        else "libdistillcache.so")
 
 DC_OK, DC_ERR_INVALID_ARG, DC_ERR_CAPACITY, DC_ERR_OOM, DC_ERR_CUDA, DC_ERR_DEVICE, DC_ERR_STATE = range(7)
 STATUS_NAMES = ["DC_OK", "DC_ERR_INVALID_ARG", "DC_ERR_CAPACITY", "DC_ERR_OOM", "DC_ERR_CUDA",
@@ -31,7 +34,8 @@ EXPORTS = ["dc_config_default", "dc_cache_create", "dc_cache_destroy", "dc_polic
            "dc_profile_read", "dc_step", "dc_step_host", "dc_step_host_async", "dc_engine", "dc_attend_noalloc",
            "dc_noalloc_last_error", "dc_pl_log_partition", "dc_gumbel_top_b", "dc_train_last_error",
            "dc_set_row_budgets", "dc_get_row_lengths", "dc_wait_selftest", "dc_selftest_last_error",
-           "dc_set_graph_mode"]
+           "dc_set_graph_mode", "dc_debug_fail_alloc", "dc_debug_checks", "dc_debug_bounds_selftest",
+           "dc_debug_corrupt_guard"]
 PHASES = ["append", "attend", "stats", "score", "combine", "evict", "full"]
 
 
@@ -92,6 +96,10 @@ def lib():
             L.dc_train_last_error.argtypes = []
             L.dc_train_last_error.restype = C.c_char_p
             L.dc_wait_selftest.argtypes = [C.c_ulonglong, P, P]
+            L.dc_debug_fail_alloc.argtypes = [C.c_longlong]
+            L.dc_debug_checks.argtypes = []
+            L.dc_debug_bounds_selftest.argtypes = [P, P]
+            L.dc_debug_corrupt_guard.argtypes = [P]
             L.dc_selftest_last_error.argtypes = []
             L.dc_selftest_last_error.restype = C.c_char_p
             L.dc_get_length.argtypes = [P, C.POINTER(I), C.POINTER(C.c_longlong)]
@@ -159,6 +167,30 @@ def attend_noalloc(q, k, v, out=None, stream=None):
     if st != DC_OK:
         raise DCError(st, lib().dc_noalloc_last_error().decode())
     return out
+
+
+def debug_fail_alloc(nth: int) -> None:
+    """Testing hook: the nth device allocation from now on fails as if the
+    device were out of memory (once); nth < 0 disarms."""
+    lib().dc_debug_fail_alloc(int(nth))
+
+
+def debug_checks() -> bool:
+    """Whether the loaded library is the debug build (index checks, guards)."""
+    return bool(lib().dc_debug_checks())
+
+
+def debug_bounds_selftest(stream=None) -> dict:
+    """Debug builds: an index one past its limit must fail its check, raise
+    the status bit, record site 903 and skip the access."""
+    import torch
+    res = np.zeros(5, dtype=np.uint32)
+    s = (stream or torch.cuda.current_stream()).cuda_stream
+    st = lib().dc_debug_bounds_selftest(res.ctypes.data_as(C.c_void_p), s)
+    if st != DC_OK:
+        raise DCError(st, lib().dc_selftest_last_error().decode())
+    return {"status": int(res[0]), "site": int(res[1]), "index": int(res[2]), "limit": int(res[3]),
+            "skipped": bool(res[4])}
 
 
 def wait_selftest(limit_ms: float = 50.0, stream=None) -> dict:
@@ -371,6 +403,10 @@ class DistillCache:
         """step_host without the final synchronisation (pinned host tensors;
         `out` is valid after sync())."""
         self._check(lib().dc_step_host_async(self._h, *self._step_args(q, k_new, v_new, out, cuda=False), budget))
+
+    def debug_corrupt_guard(self) -> None:
+        """Debug builds: damages a guard region so the next sync() must fail."""
+        self._check(lib().dc_debug_corrupt_guard(self._h))
 
     def set_graph_mode(self, enable: bool = True) -> None:
         """Device-counted steps: a CUDA graph captured from one step() replays
