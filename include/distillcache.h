@@ -173,10 +173,11 @@ dc_status dc_decode_step_host(dc_cache* h, const void* q_host, const void* k_new
 
 /* One whole step of Algorithm 1: dc_decode_step followed by dc_evict(budget),
  * as one kernel when the fused engine takes the step (no scores are stored
- * then; DC_BUF_SCORE is not updated). Exception: with split rows (see
- * tail_split) a step that evicts more than one token runs as the two calls.
- * The result is bit-identical to the two calls either way. Same arguments as
- * dc_decode_step. */
+ * then; DC_BUF_SCORE is not updated). Exceptions, which run as the two
+ * calls: with split rows (see tail_split) a step that evicts more than one
+ * token per row, and a step that evicts more than 1024 tokens per row (a
+ * prompt compression). The result is bit-identical to the two calls either
+ * way. Same arguments as dc_decode_step. */
 dc_status dc_step(dc_cache* h, const void* q, const void* k_new, const void* v_new, float* out,
                   int budget);
 

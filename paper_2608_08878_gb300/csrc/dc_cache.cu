@@ -20,6 +20,9 @@
 namespace {
 
 constexpr unsigned kMagic = 0x44434331u;  // "DCC1"
+// dc_step evicts more tokens per row than this with the eviction kernel (a
+// separate launch after the decode kernel) rather than in the fused kernel.
+constexpr int kFusedEvictMax = 1024;
 constexpr unsigned kDead = 0xDEADDEADu;
 
 thread_local std::string g_create_error;
@@ -736,9 +739,12 @@ dc_status dc_step(dc_cache* h, const void* q, const void* k_new, const void* v_n
     return dc_evict(h, budget);
   }
   const int B = effective_budget(h, budget, n1, h->seen + 1);
-  if (!h->per_row && B < n1 - 1 && tail_split_applies(h, n1)) {
+  if (!h->per_row && B < n1 - 1 && (tail_split_applies(h, n1) || n1 - B > kFusedEvictMax)) {
     // several evictions need the whole row's scores in one CTA: with half
-    // rows this step runs as the decode kernel plus the eviction kernel
+    // rows this step runs as the decode kernel plus the eviction kernel; so
+    // does a step with many evictions (a prompt compression), whose moves the
+    // eviction kernel makes with many more bytes in flight than the fused
+    // kernel's epilogue
     dc_status s = dc_decode_step(h, q, k_new, v_new, out);
     if (s != DC_OK) return s;
     return dc_evict(h, budget);

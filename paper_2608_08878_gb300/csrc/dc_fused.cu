@@ -6,21 +6,21 @@
 namespace dc {
 
 int fused_onchip_tokens(int G) {
-  const int t = G == 4 ? onchip_tiles<3>() : G == 2 ? onchip_tiles<1>() : onchip_tiles<0>();
+  const int t = G == 8 ? onchip_tiles<8>() : G == 4 ? onchip_tiles<4>() : G == 2 ? onchip_tiles<2>() : onchip_tiles<1>();
   return t * kTok;
 }
 
 bool fused_eligible(const Dev& p, int n) {
-  return (p.d == 64 || p.d == 128) && (p.G == 1 || p.G == 2 || p.G == 4) && p.hidden <= 128 && n >= 1 &&
+  return (p.d == 64 || p.d == 128) && (p.G == 1 || p.G == 2 || p.G == 4 || p.G == 8) && p.hidden <= 128 && n >= 1 &&
          p.logit != nullptr && p.score != nullptr;
 }
 
-int fused_smem_bytes() { return Smem<false>::BYTES; }
+int fused_smem_bytes() { return Smem<false, 4>::BYTES; }
 
 bool fused_pairs(const Dev& p, int n, int num_sms) {
   const int nT = (n + kTok - 1) / kTok;
-  if (!(p.seq_rows == 0 && p.rowlen == nullptr && p.scorer == 0 && p.R % 2 == 0 && p.R > num_sms && nT >= 1 &&
-        nT <= kPairTiles))
+  if (!(p.seq_rows == 0 && p.rowlen == nullptr && p.scorer == 0 && p.G <= 4 && p.R % 2 == 0 && p.R > num_sms &&
+        nT >= 1 && nT <= kPairTiles))
     return false;
   // Critical path of a CTA in units of one token's streaming time at an SM's
   // share of the bandwidth (measured with per-row timestamps): a row costs its
@@ -58,10 +58,12 @@ cudaError_t launch_fused_step(const FusedMaps& maps, const Dev& p, const Step& s
 #define DC_FUSED_LAUNCH(D, G) \
   return lg ? launch_t<D, G, true>(maps, p, st, fs, fp, grid, s) : launch_t<D, G, false>(maps, p, st, fs, fp, grid, s)
   if (p.d == 128) {
+    if (p.G == 8) DC_FUSED_LAUNCH(128, 8);
     if (p.G == 4) DC_FUSED_LAUNCH(128, 4);
     if (p.G == 2) DC_FUSED_LAUNCH(128, 2);
     DC_FUSED_LAUNCH(128, 1);
   }
+  if (p.G == 8) DC_FUSED_LAUNCH(64, 8);
   if (p.G == 4) DC_FUSED_LAUNCH(64, 4);
   if (p.G == 2) DC_FUSED_LAUNCH(64, 2);
   DC_FUSED_LAUNCH(64, 1);

@@ -16,15 +16,22 @@ cudaError_t launch_fused_graph(const FusedMaps& maps, const Dev& p, const Step& 
   return pairs ? launch_t<D, G, false, false, false, false, false, true, true>(maps, p, st, fs, fp, grid, s) \
          : lg  ? launch_t<D, G, true, false, false, false, false, false, true>(maps, p, st, fs, fp, grid, s) \
                : launch_t<D, G, false, false, false, false, false, false, true>(maps, p, st, fs, fp, grid, s)
+  // eight query heads per KV head: never on row pairs
+#define DC_FUSED_LAUNCH8(D)                                                                                   \
+  return lg ? launch_t<D, 8, true, false, false, false, false, false, true>(maps, p, st, fs, fp, grid, s)    \
+            : launch_t<D, 8, false, false, false, false, false, false, true>(maps, p, st, fs, fp, grid, s)
   if (p.d == 128) {
+    if (p.G == 8) DC_FUSED_LAUNCH8(128);
     if (p.G == 4) DC_FUSED_LAUNCH(128, 4);
     if (p.G == 2) DC_FUSED_LAUNCH(128, 2);
     DC_FUSED_LAUNCH(128, 1);
   }
+  if (p.G == 8) DC_FUSED_LAUNCH8(64);
   if (p.G == 4) DC_FUSED_LAUNCH(64, 4);
   if (p.G == 2) DC_FUSED_LAUNCH(64, 2);
   DC_FUSED_LAUNCH(64, 1);
 #undef DC_FUSED_LAUNCH
+#undef DC_FUSED_LAUNCH8
 }
 
 }  // namespace dc

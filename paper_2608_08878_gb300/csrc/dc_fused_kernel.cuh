@@ -75,8 +75,31 @@ constexpr int kTok = 128;
 constexpr int kThreads = 352;
 constexpr int kEpi = 256;                     // two warpgroups
 constexpr uint32_t kTmemCols = 512;
-constexpr int kColS = 0, kColO = 32, kColM = 128;
-constexpr int kStashA = 48, kStashAEnd = 128, kStashB = 384, kStashBEnd = 512;
+constexpr int kColS = 0, kColM = 128;
+constexpr int kStashAEnd = 128, kStashB = 384, kStashBEnd = 512;
+
+// The query tile holds the current, previous-step and departing queries (3G
+// rows) padded to the QK MMA's N: 16 rows, or 32 for eight query heads per KV
+// head. The S tiles (two buffers of N columns) come first in TMEM, then O (16
+// columns), then the first logit stash area.
+template <int G>
+constexpr int q_rows() {
+  return G == 8 ? 32 : 16;
+}
+template <int G>
+constexpr int col_o() {
+  return kColS + 2 * q_rows<G>();
+}
+template <int G>
+constexpr int stash_a() {
+  return col_o<G>() + 16;
+}
+// Tokens whose head-(G-1) logits, then scores, the fused kernel keeps in
+// shared memory (a G = 8 row's larger query tiles take 8 KB of it).
+template <int G>
+constexpr int max_tok() {
+  return G == 8 ? 8192 : kFusedMaxTok;
+}
 
 // Row pairs (PAIR): an item is two rows of at most kPairTiles tiles, one per
 // warpgroup; their K and V tiles alternate in the stage ring.
@@ -87,16 +110,17 @@ constexpr int kPairStashA = 64;                            // the first row's lo
 
 // Shared memory layout; PAIR keeps four query tiles (two per item, double
 // buffered) and a smaller logit/score array per row.
-template <bool PAIR>
+template <bool PAIR, int G>
 struct Smem {
+  static constexpr int QBYTES = q_rows<G>() * 256;         // one query tile: two 64-dim blocks
   static constexpr int STAGE = 0;
-  static constexpr int Q = STAGE + kStages * kStageBytes;   // (2 or 4) x 4 KB
-  static constexpr int P = Q + (PAIR ? 4 : 2) * 4096;       // 2 x 4 KB (one per warpgroup)
+  static constexpr int Q = STAGE + kStages * kStageBytes;   // (2 or 4) query tiles
+  static constexpr int P = Q + (PAIR ? 4 : 2) * QBYTES;     // 2 x 4 KB (one per warpgroup)
   static constexpr int A = P + 2 * 4096;                    // 2 x 8 KB (one per warpgroup)
   static constexpr int W = A + 2 * 8192;                    // 8 KB
   static constexpr int AUX = W + 8192;                      // kStages x 2560 B
   static constexpr int SC = AUX + kStages * kAuxBytes;      // head G-1 logits, then scores
-  static constexpr int MISC = SC + (PAIR ? 2 * kPairTok : kFusedMaxTok) * 4;
+  static constexpr int MISC = SC + (PAIR ? 2 * kPairTok : max_tok<G>()) * 4;
   static constexpr int BYTES = MISC + 4096 + 1024;          // misc area + alignment slack
   static_assert(BYTES <= 232448, "more shared memory than a CTA may have");
 };
@@ -113,22 +137,30 @@ enum {
 // Tiles whose logits stay on chip between the passes (heads 0..G-2 in TMEM,
 // head G-1 in shared memory); later tiles of longer rows keep all G logits in
 // the global scratch [R][stride][G] instead.
-template <int GS>
+template <int G>
 constexpr int onchip_tiles() {
-  constexpr int st = GS > 0 ? (kStashAEnd - kStashA) / GS + (kStashBEnd - kStashB) / GS : (1 << 20);
-  return st < kFusedMaxTok / kTok ? st : kFusedMaxTok / kTok;
+  constexpr int GS = G - 1;
+  constexpr int st = GS > 0 ? (kStashAEnd - stash_a<G>()) / GS + (kStashBEnd - kStashB) / GS : (1 << 20);
+  return st < max_tok<G>() / kTok ? st : max_tok<G>() / kTok;
 }
 
 template <int G>
 __device__ __forceinline__ void store_logits(float* dst, const float* v) {
-  if constexpr (G == 4) *reinterpret_cast<float4*>(dst) = make_float4(v[0], v[1], v[2], v[3]);
+  if constexpr (G == 8) {
+    reinterpret_cast<float4*>(dst)[0] = make_float4(v[0], v[1], v[2], v[3]);
+    reinterpret_cast<float4*>(dst)[1] = make_float4(v[4], v[5], v[6], v[7]);
+  } else if constexpr (G == 4) *reinterpret_cast<float4*>(dst) = make_float4(v[0], v[1], v[2], v[3]);
   else if constexpr (G == 2) *reinterpret_cast<float2*>(dst) = make_float2(v[0], v[1]);
   else dst[0] = v[0];
 }
 
 template <int G>
 __device__ __forceinline__ void load_logits(const float* src, float* v) {
-  if constexpr (G == 4) {
+  if constexpr (G == 8) {
+    const float4 x = reinterpret_cast<const float4*>(src)[0], y = reinterpret_cast<const float4*>(src)[1];
+    v[0] = x.x; v[1] = x.y; v[2] = x.z; v[3] = x.w;
+    v[4] = y.x; v[5] = y.y; v[6] = y.z; v[7] = y.w;
+  } else if constexpr (G == 4) {
     const float4 x = *reinterpret_cast<const float4*>(src);
     v[0] = x.x; v[1] = x.y; v[2] = x.z; v[3] = x.w;
   } else if constexpr (G == 2) {
@@ -140,10 +172,11 @@ __device__ __forceinline__ void load_logits(const float* src, float* v) {
 }
 
 // TMEM column of the stashed logits of tile j (GS = G - 1 columns per tile).
-template <int GS>
+template <int G>
 __device__ __forceinline__ uint32_t stash_col(int j) {
-  constexpr int TA = GS > 0 ? (kStashAEnd - kStashA) / GS : 0;
-  return j < TA ? (uint32_t)(kStashA + GS * j) : (uint32_t)(kStashB + GS * (j - TA));
+  constexpr int GS = G - 1;
+  constexpr int TA = GS > 0 ? (kStashAEnd - stash_a<G>()) / GS : 0;
+  return j < TA ? (uint32_t)(stash_a<G>() + GS * j) : (uint32_t)(kStashB + GS * (j - TA));
 }
 
 // byte offset of 16-byte chunk `c` (0..7) of row `row` inside a 128-byte
@@ -166,7 +199,17 @@ __device__ __forceinline__ uint32_t pack_bf16(float a, float b) {
 // Stores / loads the first GS of the G logits of this thread's token.
 template <int GS>
 __device__ __forceinline__ void stash_store(uint32_t taddr, const float* v) {
-  if constexpr (GS == 3) {
+  if constexpr (GS == 7) {
+    asm volatile("tcgen05.st.sync.aligned.32x32b.x4.b32 [%0], {%1,%2,%3,%4};" ::"r"(taddr),
+                 "r"(__float_as_uint(v[0])), "r"(__float_as_uint(v[1])), "r"(__float_as_uint(v[2])),
+                 "r"(__float_as_uint(v[3]))
+                 : "memory");
+    asm volatile("tcgen05.st.sync.aligned.32x32b.x2.b32 [%0], {%1,%2};" ::"r"(taddr + 4), "r"(__float_as_uint(v[4])),
+                 "r"(__float_as_uint(v[5]))
+                 : "memory");
+    asm volatile("tcgen05.st.sync.aligned.32x32b.x1.b32 [%0], {%1};" ::"r"(taddr + 6), "r"(__float_as_uint(v[6]))
+                 : "memory");
+  } else if constexpr (GS == 3) {
     asm volatile("tcgen05.st.sync.aligned.32x32b.x2.b32 [%0], {%1,%2};" ::"r"(taddr), "r"(__float_as_uint(v[0])),
                  "r"(__float_as_uint(v[1]))
                  : "memory");
@@ -180,7 +223,21 @@ __device__ __forceinline__ void stash_store(uint32_t taddr, const float* v) {
 
 template <int GS>
 __device__ __forceinline__ void stash_load(uint32_t taddr, float* v) {
-  if constexpr (GS == 3) {
+  if constexpr (GS == 7) {
+    uint32_t a, b, c, d, e, f, g;
+    asm volatile("tcgen05.ld.sync.aligned.32x32b.x4.b32 {%0,%1,%2,%3}, [%4];"
+                 : "=r"(a), "=r"(b), "=r"(c), "=r"(d)
+                 : "r"(taddr));
+    asm volatile("tcgen05.ld.sync.aligned.32x32b.x2.b32 {%0,%1}, [%2];" : "=r"(e), "=r"(f) : "r"(taddr + 4));
+    asm volatile("tcgen05.ld.sync.aligned.32x32b.x1.b32 {%0}, [%1];" : "=r"(g) : "r"(taddr + 6));
+    v[0] = __uint_as_float(a);
+    v[1] = __uint_as_float(b);
+    v[2] = __uint_as_float(c);
+    v[3] = __uint_as_float(d);
+    v[4] = __uint_as_float(e);
+    v[5] = __uint_as_float(f);
+    v[6] = __uint_as_float(g);
+  } else if constexpr (GS == 3) {
     uint32_t a, b, c;
     asm volatile("tcgen05.ld.sync.aligned.32x32b.x2.b32 {%0,%1}, [%2];" : "=r"(a), "=r"(b) : "r"(taddr));
     asm volatile("tcgen05.ld.sync.aligned.32x32b.x1.b32 {%0}, [%1];" : "=r"(c) : "r"(taddr + 2));
@@ -304,6 +361,12 @@ __global__ void __launch_bounds__(kThreads, 1)
                  Step st, FusedStep fs, FusedPolicy fp) {
   constexpr int GS = G - 1;  // heads whose logits wait in TMEM between the passes
   static_assert(!PAIR || (!LONG && !FULL && !HEUR && !GLOB && !PERROW), "row pairs: the plain step only");
+  static_assert(!PAIR || G <= 4, "row pairs: up to four query heads per KV head");
+  constexpr int NQ = q_rows<G>();   // query-tile rows, S-tile columns
+  constexpr int kColO = col_o<G>();
+  // G = 8: the per-row statistics of the window's queries (the K pass) sit in
+  // shared memory rather than in 6 x 8 registers per thread
+  constexpr bool kWqSmem = G == 8;
   static_assert(!GRAPH || (!FULL && !HEUR && !GLOB && !PERROW), "device-counted steps: the plain step");
   if constexpr (GRAPH) {
     // this launch's step: the base arguments advanced by the steps taken (in
@@ -317,7 +380,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     st.slot_prev = (st.slot_prev + t) % p.w;
     fs.epoch += (unsigned)t;
   }
-  using L = Smem<PAIR>;
+  using L = Smem<PAIR, G>;
   constexpr int OFF_STAGE = L::STAGE, OFF_Q = L::Q, OFF_P = L::P, OFF_A = L::A, OFF_W = L::W, OFF_AUX = L::AUX,
                 OFF_SC = L::SC, OFF_MISC = L::MISC;
   extern __shared__ uint8_t smem_raw[];
@@ -326,7 +389,11 @@ __global__ void __launch_bounds__(kThreads, 1)
   static_assert(8 * B_COUNT <= 384, "barriers overlap the misc fields");
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + OFF_MISC + 384);
   volatile int* abort = reinterpret_cast<volatile int*>(smem + OFF_MISC + 388);
-  float* red = reinterpret_cast<float*>(smem + OFF_MISC + 512);            // [8][G][3]
+  // [8][G][3]; with G = 8 in the area the row pairs' scratch takes otherwise
+  float* red = reinterpret_cast<float*>(smem + OFF_MISC + (G == 8 ? 2560 : 512));
+  float* s_wq = reinterpret_cast<float*>(smem + OFF_MISC + 3328);          // G = 8: [6][8], then [3][8]
+  static_assert(G != 8 || (!PAIR && 2560 + 8 * G * 3 * 4 <= 3328 && 3328 + 9 * 8 * 4 <= MISC_BYTES),
+                "misc area layout");
   int* s_hist = reinterpret_cast<int*>(smem + OFF_MISC + 1024);           // [256]
   int* s_sh = reinterpret_cast<int*>(smem + OFF_MISC + 2048);             // [4]
   int* s_wsum = reinterpret_cast<int*>(smem + OFF_MISC + 2064);           // [8]
@@ -428,7 +495,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       // step, [2G,3G) departing
       for (int qi = 0; qi < (PAIR ? 2 : 1); ++qi) {
         const int rq = r + qi;
-        uint8_t* qt = smem + OFF_Q + (PAIR ? 2 * qb + qi : qb) * 4096;
+        uint8_t* qt = smem + OFF_Q + (PAIR ? 2 * qb + qi : qb) * L::QBYTES;
         const int qo = ((rq / p.kvh) * p.qh + (rq % p.kvh) * G) * D;
         const __nv_bfloat16* prev = p.ring_q + ((size_t)rq * p.w + st.slot_prev) * G * D;
         const __nv_bfloat16* dep = p.ring_q + ((size_t)rq * p.w + st.slot) * G * D;
@@ -443,9 +510,9 @@ __global__ void __launch_bounds__(kThreads, 1)
           const uint4 cur = reinterpret_cast<const uint4*>(fs.q + qo + h * D)[kc];
           const uint4 pv = st.has_prev ? reinterpret_cast<const uint4*>(prev + h * D)[kc] : make_uint4(0, 0, 0, 0);
           const uint4 dv = st.has_dep ? reinterpret_cast<const uint4*>(dep + h * D)[kc] : make_uint4(0, 0, 0, 0);
-          *reinterpret_cast<uint4*>(qt + (kc >> 3) * 2048 + sw128(h, kc & 7)) = cur;
-          *reinterpret_cast<uint4*>(qt + (kc >> 3) * 2048 + sw128(G + h, kc & 7)) = pv;
-          *reinterpret_cast<uint4*>(qt + (kc >> 3) * 2048 + sw128(2 * G + h, kc & 7)) = dv;
+          *reinterpret_cast<uint4*>(qt + (kc >> 3) * (NQ * 128) + sw128(h, kc & 7)) = cur;
+          *reinterpret_cast<uint4*>(qt + (kc >> 3) * (NQ * 128) + sw128(G + h, kc & 7)) = pv;
+          *reinterpret_cast<uint4*>(qt + (kc >> 3) * (NQ * 128) + sw128(2 * G + h, kc & 7)) = dv;
           if (!FULL && it.half < 0) reinterpret_cast<uint4*>(ring_slot + h * D)[kc] = cur;  // halves: see the epilogue
         }
       }
@@ -511,7 +578,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   } else if (warp == 1) {
     // ------------------------------------------------------------ MMA issuer
     if (lane == 0) {
-      const uint32_t id_qk = idesc_bf16(128, 16, 0, 0);
+      const uint32_t id_qk = idesc_bf16(128, NQ, 0, 0);
       const uint32_t id_pv = idesc_bf16(128, 16, 1, 1);
       int g = 0, gs = 0, gv = 0;
       for (int gr = 0;; ++gr) {
@@ -522,7 +589,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         tc_fence_after();
         const int nx = (PAIR ? 2 : 1) * (it.t1 - it.t0);  // PAIR: the rows' tiles alternate
         for (int x = 0; x < nx; ++x, ++g, ++gs) {
-          const uint32_t qaddr = smem_u32(smem + OFF_Q + (PAIR ? 2 * qb + (x & 1) : qb) * 4096);
+          const uint32_t qaddr = smem_u32(smem + OFF_Q + (PAIR ? 2 * qb + (x & 1) : qb) * L::QBYTES);
           const int s = g % kStages, b = gs & 1;
           if (!mbar_wait(&bar[B_FULL + s], (g / kStages) & 1, abort, p.dbg, 4u, (unsigned)g)) break;
           if (!mbar_wait(&bar[B_SEMPTY + b], ((gs >> 1) & 1) ^ 1, abort, p.dbg, 5u, (unsigned)gs)) break;
@@ -531,8 +598,8 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
           for (int ks = 0; ks < D / 16; ++ks) {
             const uint32_t off = (uint32_t)(ks >> 2) * 16384u + (uint32_t)(ks & 3) * 32u;
-            const uint32_t qoff = (uint32_t)(ks >> 2) * 2048u + (uint32_t)(ks & 3) * 32u;
-            mma_bf16(tmem + kColS + b * 16, sdesc_sw128(kaddr + off, 16, 1024), sdesc_sw128(qaddr + qoff, 16, 1024),
+            const uint32_t qoff = (uint32_t)(ks >> 2) * (uint32_t)(NQ * 128) + (uint32_t)(ks & 3) * 32u;
+            mma_bf16(tmem + kColS + b * NQ, sdesc_sw128(kaddr + off, 16, 1024), sdesc_sw128(qaddr + qoff, 16, 1024),
                      id_qk, ks > 0);
           }
           mma_commit(&bar[B_SFULL + b]);
@@ -623,7 +690,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     // TMEM column of the stashed logits of this team's tile j
     auto stash_at = [wg](int j) -> uint32_t {
       if constexpr (PAIR) return (uint32_t)((wg ? kStashB : kPairStashA) + GS * j);
-      else return stash_col<GS>(j);
+      else return stash_col<G>(j);
     };
     // position of this team's tile j in the item's tile sequence
     auto tpos = [wg](int j, int t0) { return PAIR ? 2 * j + wg : j - t0; };
@@ -657,14 +724,31 @@ __global__ void __launch_bounds__(kThreads, 1)
       const bool x_ok = it.half < 0 || (DC_INB(p, ts, fs.xslots, 110) && DC_INB(p, ts, fs.half_rows, 110));
       // a row longer than the shared score array keeps its scores in HBM when
       // the radix select reads them (several evictions), or when asked to
-      const bool spill_scores = LONG && n > kFusedMaxTok && fs.do_evict && Bsel < n - 1;
-      float pm[G], pnl[G], pH[G], dm[G], dnl[G], dH[G];
+      const bool spill_scores = LONG && n > max_tok<G>() && fs.do_evict && Bsel < n - 1;
+      // statistics (m, -log2 l, H) of the previous and the departing query
+      constexpr int GR = kWqSmem ? 1 : G;
+      float pm[GR], pnl[GR], pH[GR], dm[GR], dnl[GR], dH[GR];
+      if constexpr (kWqSmem) {
+        // one thread per (query, head) loads them into shared memory; the
+        // team's barrier publishes them (the previous item's K pass, their
+        // last reader, ended before that item's statistics merge)
+        if (tid < 2 * G) {
+          const int h = tid % G, dep = tid / G;
+          const float4 rs =
+              reinterpret_cast<const float4*>(p.ring_stats)[((size_t)r * p.w + (dep ? st.slot : st.slot_prev)) * G + h];
+          s_wq[(3 * dep + 0) * G + h] = rs.x;
+          s_wq[(3 * dep + 1) * G + h] = rs.w;
+          s_wq[(3 * dep + 2) * G + h] = rs.z;
+        }
+        sync();
+      } else {
 #pragma unroll
-      for (int h = 0; h < G; ++h) {
-        const float4 rp = reinterpret_cast<const float4*>(p.ring_stats)[((size_t)r * p.w + st.slot_prev) * G + h];
-        const float4 rd = reinterpret_cast<const float4*>(p.ring_stats)[((size_t)r * p.w + st.slot) * G + h];
-        pm[h] = rp.x; pnl[h] = rp.w; pH[h] = rp.z;
-        dm[h] = rd.x; dnl[h] = rd.w; dH[h] = rd.z;
+        for (int h = 0; h < G; ++h) {
+          const float4 rp = reinterpret_cast<const float4*>(p.ring_stats)[((size_t)r * p.w + st.slot_prev) * G + h];
+          const float4 rd = reinterpret_cast<const float4*>(p.ring_stats)[((size_t)r * p.w + st.slot) * G + h];
+          pm[h] = rp.x; pnl[h] = rp.w; pH[h] = rp.z;
+          dm[h] = rd.x; dnl[h] = rd.w; dH[h] = rd.z;
+        }
       }
       float m[G], l[G], u[G];
 #pragma unroll
@@ -678,8 +762,9 @@ __global__ void __launch_bounds__(kThreads, 1)
         mbar_wait(&bar[B_FULL + s], (gj / kStages) & 1, abort, p.dbg, 12u, (unsigned)gj);
         __syncwarp();
         tc_fence_after();
-        float S16[16];
-        tmem_ld16(lane_addr + kColS + b * 16, S16);
+        float S16[NQ];  // the current, previous and departing queries' logits
+        if constexpr (NQ == 32) tmem_ld32(lane_addr + kColS + b * NQ, S16);
+        else tmem_ld16(lane_addr + kColS + b * NQ, S16);
         tmem_ld_wait();
         const uint8_t* aux = smem + OFF_AUX + s * kAuxBytes;
         const int pos = reinterpret_cast<const int*>(aux + kAuxPos)[tok];
@@ -698,15 +783,20 @@ __global__ void __launch_bounds__(kThreads, 1)
             // terms of the previous and the departing query, masked (x 1 or x 0,
             // both exact) where the token was not yet in the cache at that step
             float zp, sp, zd, sd;
-            window_terms<G>(S16 + G, pm, pnl, pH, c, zp, sp);
-            window_terms<G>(S16 + 2 * G, dm, dnl, dH, c, zd, sd);
+            if constexpr (kWqSmem) {
+              window_terms<G>(S16 + G, s_wq, s_wq + G, s_wq + 2 * G, c, zp, sp);
+              window_terms<G>(S16 + 2 * G, s_wq + 3 * G, s_wq + 4 * G, s_wq + 5 * G, c, zd, sd);
+            } else {
+              window_terms<G>(S16 + G, pm, pnl, pH, c, zp, sp);
+              window_terms<G>(S16 + 2 * G, dm, dnl, dH, c, zd, sd);
+            }
             const float mp = (st.has_prev && pos <= st.p_prev) ? 1.f : 0.f;
             const float md = (st.has_dep && pos <= st.p_dep) ? 1.f : 0.f;
             sz = window_update(sz, sp * mp, sd * md, zp * mp, zd * md);
             if (slot_ok(i, 105)) p.SZ[rbase + i] = sz;
           }
         }
-        if (!LONG || j < onchip_tiles<GS>()) {
+        if (!LONG || j < onchip_tiles<G>()) {
           scw[i] = S16[G - 1];
           __syncwarp();
           stash_store<GS>(lane_addr + stash_at(j), S16);
@@ -836,6 +926,19 @@ __global__ void __launch_bounds__(kThreads, 1)
         Hh[h] = logf(Ll[h]) - 0.69314718055994531f * (Uu[h] / Ll[h]);
         if (tid == h) L0 = Ll[h];
       }
+      // G = 8: the V pass reads the row's final statistics from shared memory
+      float* s_st = s_wq + 6 * 8;  // [3][8]: M, -log2 l, H
+      if constexpr (kWqSmem) {
+        if (tid == 0) {
+#pragma unroll
+          for (int h = 0; h < G; ++h) {
+            s_st[h] = M[h];
+            s_st[G + h] = NL[h];
+            s_st[2 * G + h] = Hh[h];
+          }
+        }
+        sync();
+      }
       // push (m, l, H, -log2 l) of this step into the ring slot it takes over
       // (the producer, or half 0 above, wrote the query there)
       if (!FULL && tid < G && half <= 0 && DC_INB(p, (long long)r * p.w + st.slot, (long long)p.R * p.w, 109)) {
@@ -876,7 +979,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int i = j * kTok + tok;
         const bool valid = i < n;
         float sv[G];
-        if (!LONG || j < onchip_tiles<GS>()) {
+        if (!LONG || j < onchip_tiles<G>()) {
           stash_load<GS>(lane_addr + stash_at(j), sv);
           if constexpr (GS > 0) tmem_ld_wait();
           sv[G - 1] = scw[i];
@@ -886,19 +989,20 @@ __global__ void __launch_bounds__(kThreads, 1)
         float a[G], zc = 0.f, scur = 0.f;
 #pragma unroll
         for (int h = 0; h < G; ++h) {
-          a[h] = attn_weight(sv[h], M[h], c, NL[h]);
+          a[h] = kWqSmem ? attn_weight(sv[h], s_st[h], c, s_st[G + h]) : attn_weight(sv[h], M[h], c, NL[h]);
           zc += a[h];
-          scur = fmaf(a[h], Hh[h], scur);
+          scur = fmaf(a[h], kWqSmem ? s_st[2 * G + h] : Hh[h], scur);
         }
         // attention weights as the PV operand, MN-major (one 32-byte row of 16
         // columns per token, 32-byte swizzle): bf16 high parts in columns
         // [0, G), the residuals in [G, 2G), so that O = D[:, h] + D[:, G + h]
-        // carries ~16 mantissa bits; columns [8, 16) stay zero
+        // carries ~16 mantissa bits; columns [2G, 16) stay zero
         mbar_wait(&bar[B_PEMPTY + pb], ((gvj >> 1) & 1) ^ 1, abort, p.dbg, 8u, (unsigned)gvj);
         {
-          float pw[8];
+          constexpr int NP = G == 8 ? 16 : 8;  // columns written: one or both 16-byte chunks
+          float pw[NP];
 #pragma unroll
-          for (int h = 0; h < 8; ++h) pw[h] = 0.f;
+          for (int h = 0; h < NP; ++h) pw[h] = 0.f;
 #pragma unroll
           for (int h = 0; h < G; ++h) {
             const float ah = valid ? a[h] : 0.f;
@@ -906,10 +1010,12 @@ __global__ void __launch_bounds__(kThreads, 1)
             pw[h] = hv;
             pw[G + h] = ah - hv;
           }
-          const uint4 row = make_uint4(pack_bf16(pw[0], pw[1]), pack_bf16(pw[2], pw[3]), pack_bf16(pw[4], pw[5]),
-                                       pack_bf16(pw[6], pw[7]));
-          *reinterpret_cast<uint4*>(smem + OFF_P + pb * 4096 + (tok >> 3) * 256 + (tok & 7) * 32 +
-                                    (((tok >> 2) & 1) << 4)) = row;
+          uint8_t* prow = smem + OFF_P + pb * 4096 + (tok >> 3) * 256 + (tok & 7) * 32;
+#pragma unroll
+          for (int ck = 0; ck < NP / 8; ++ck)
+            *reinterpret_cast<uint4*>(prow + ((ck ^ ((tok >> 2) & 1)) << 4)) =
+                make_uint4(pack_bf16(pw[8 * ck + 0], pw[8 * ck + 1]), pack_bf16(pw[8 * ck + 2], pw[8 * ck + 3]),
+                           pack_bf16(pw[8 * ck + 4], pw[8 * ck + 5]), pack_bf16(pw[8 * ck + 6], pw[8 * ck + 7]));
           fence_proxy_async();
           __syncwarp();
           if (lane == 0) mbar_arrive(&bar[B_PFULL + pb]);
@@ -1019,7 +1125,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           const float score = fp.b2 + relu_sum;
           if constexpr (LONG) {
             if (spill_scores || fs.write_scores) p.score[rbase + i] = score;
-            if (n <= kFusedMaxTok) scw[i] = score;
+            if (n <= max_tok<G>()) scw[i] = score;
           } else {
             scw[i] = score;
             if (fs.write_scores) p.score[rbase + i] = score;
@@ -1038,7 +1144,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int i = j * kTok + tok;
         if (i < n && slot_ok(i, 114)) {
           if (spill_scores || fs.write_scores) p.score[rbase + i] = score;
-          if (n <= kFusedMaxTok) scw[i] = score;
+          if (n <= max_tok<G>()) scw[i] = score;
           const uint32_t kk = score_key(score);
           if (ev_slot < 0 || kk < ev_key || (kk == ev_key && pos > ev_pos)) {
             ev_key = kk;
@@ -1152,7 +1258,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       } else if (fs.do_evict && Bsel < n) {
         // several evictions (whole rows only): radix select over the scores
         sync();
-        team_select_compact<kTeam>(p, r, n, Bsel, LONG && n > kFusedMaxTok ? p.score + rbase : scw, tid, scr,
+        team_select_compact<kTeam>(p, r, n, Bsel, LONG && n > max_tok<G>() ? p.score + rbase : scw, tid, scr,
                                    sync);
       }
       if (PERROW && fs.do_evict && tid == 0 && DC_INB(p, r, p.R, 118)) p.rowlen[r] = n < Bsel ? n : Bsel;
@@ -1180,7 +1286,7 @@ template <int D, int G, bool LONG, bool FULL = false, bool HEUR = false, bool GL
           bool PAIR = false, bool GRAPH = false>
 static cudaError_t launch_t(const FusedMaps& maps, const Dev& p, const Step& st, const FusedStep& fs,
                             const FusedPolicy& fp, int grid, cudaStream_t s) {
-  constexpr int kSmemBytes = Smem<PAIR>::BYTES;
+  constexpr int kSmemBytes = Smem<PAIR, G>::BYTES;
   static bool attr = false;
   if (!attr) {
     cudaError_t e = cudaFuncSetAttribute(fused_kernel<D, G, LONG, FULL, HEUR, GLOB, PERROW, PAIR, GRAPH>,

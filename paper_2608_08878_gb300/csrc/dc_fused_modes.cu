@@ -14,10 +14,12 @@ cudaError_t launch_fused_heur_perrow(const FusedMaps& maps, const Dev& p, const 
   return p.rowlen ? launch_t<D, G, true, false, false, false, true>(maps, p, st, fs, fp, grid, s) \
                   : launch_t<D, G, true, false, true>(maps, p, st, fs, fp, grid, s)
   if (p.d == 128) {
+    if (p.G == 8) DC_FUSED_LAUNCH(128, 8);
     if (p.G == 4) DC_FUSED_LAUNCH(128, 4);
     if (p.G == 2) DC_FUSED_LAUNCH(128, 2);
     DC_FUSED_LAUNCH(128, 1);
   }
+  if (p.G == 8) DC_FUSED_LAUNCH(64, 8);
   if (p.G == 4) DC_FUSED_LAUNCH(64, 4);
   if (p.G == 2) DC_FUSED_LAUNCH(64, 2);
   DC_FUSED_LAUNCH(64, 1);

@@ -349,7 +349,9 @@ def test_engine_choice():
     assert small.engine() == "fused" and small.engine(20000) == "split"
     forced = dc.DistillCache(1, 2, 64, 200, 100, q_heads=4, engine=2)
     assert forced.engine() == "fused"
-    assert dc.DistillCache(1, 2, 64, 200, 100, q_heads=16, engine=2).engine() == "split"  # group 8
+    assert dc.DistillCache(1, 2, 64, 200, 100, q_heads=16, engine=2).engine() == "fused"  # group 8
+    # a policy wider than the fused kernel's 128 hidden units stays on the split engine
+    assert dc.DistillCache(1, 2, 64, 200, 100, q_heads=4, mlp_hidden=256, engine=2).engine() == "split"
 
 
 def test_full_decode_matches_oracle():
@@ -425,6 +427,27 @@ def test_full_stack_sampled_rows(engine):
     for s in range(72):
         ls.step(check=(s < 3 or s % 16 == 0 or s >= 62))
     assert ls.cache.length()[0] == wl.budget
+
+
+@pytest.mark.parametrize("layers,batch,kv_heads,prompt_len,budget", [
+    (1, 1, 4, 8192, 2048),     # few rows: halves over two CTAs each
+    (5, 8, 4, 8192, 8192),     # 160 rows: the split last wave; rows past the on-chip logits
+    (2, 10, 8, 3000, 1000),    # 160 rows within the on-chip logits, many-eviction first step
+])
+def test_group8_rows_match_oracle(layers, batch, kv_heads, prompt_len, budget):
+    """Eight query heads per KV head on the fused engine: a 32-row query tile,
+    seven TMEM logit columns per tile (24 tiles on chip, then all eight
+    logits through HBM), both 16-byte halves of the PV operand; the prompt
+    compression and steps past a small window, sampled rows."""
+    wl = synth.MISTRAL_1L.with_(layers=layers, batch=batch, kv_heads=kv_heads, q_heads=8 * kv_heads,
+                                prompt_len=prompt_len, budget=budget, window=4, steps=8)
+    rows = sorted({0, wl.rows // 2, wl.rows - 1})
+    ls = LockStep(wl, rows, engine=2, device_inputs=True)
+    assert ls.cache.engine() == "fused"
+    ls.load_prompt()
+    for _ in range(wl.steps):
+        ls.step()
+    assert ls.cache.length()[0] == min(wl.prompt_len + wl.steps, wl.budget)
 
 
 @pytest.mark.parametrize("batch,ctx,ratio", [(1, 4096, 0.10), (64, 4096, 0.25), (4, 16384, 0.50),
@@ -615,14 +638,14 @@ def test_bounded_waits_give_up_and_leave_the_context_usable():
         ls.step()
 
 
-def _random_shapes(count=24, seed=2026):
+def _random_shapes(count=24, seed=2026, groups=(1, 2, 4)):
     """Seeded shapes over the engines' parameters (group, head size, window,
     alpha mode, engine, rows from a few to several waves, lengths from one
     token to past the row-pair limit)."""
     rng = np.random.default_rng(seed)
     out = []
     for _ in range(count):
-        group = int(rng.choice([1, 2, 4]))
+        group = int(rng.choice(list(groups)))
         head_dim = int(rng.choice([64, 128]))
         kv_heads = int(rng.choice([1, 2, 8]))
         layers = int(rng.integers(1, 5))
@@ -636,7 +659,8 @@ def _random_shapes(count=24, seed=2026):
     return out
 
 
-@pytest.mark.parametrize("shape", _random_shapes(), ids=lambda s: "L{layers}b{batch}h{kv_heads}g{group}d{head_dim}"
+@pytest.mark.parametrize("shape", _random_shapes() + _random_shapes(count=12, seed=88, groups=(8,)),
+                         ids=lambda s: "L{layers}b{batch}h{kv_heads}g{group}d{head_dim}"
                          "p{prompt_len}B{budget}w{window}a{alpha_mode}e{engine}".format(**s))
 def test_random_shapes_match_oracle(shape):
     """Seeded random shapes against the oracle on sampled rows: whatever
@@ -653,7 +677,8 @@ def test_random_shapes_match_oracle(shape):
     assert ls.cache.length()[0] == min(wl.prompt_len + wl.steps, wl.budget)
 
 
-@pytest.mark.parametrize("shape", _random_shapes(count=12, seed=7), ids=lambda s: "L{layers}b{batch}h{kv_heads}g{group}"
+@pytest.mark.parametrize("shape", _random_shapes(count=12, seed=7) + _random_shapes(count=6, seed=89, groups=(8,)),
+                         ids=lambda s: "L{layers}b{batch}h{kv_heads}g{group}"
                          "d{head_dim}p{prompt_len}B{budget}w{window}a{alpha_mode}e{engine}".format(**s))
 def test_random_shapes_step_equals_decode_then_evict(shape):
     """Seeded random shapes: dc_step (the fused engine's in-kernel select and
