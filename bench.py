@@ -99,10 +99,11 @@ def fused_kernel_source_sha() -> str:
 
 
 def fused_traffic_per_token_row():
-    """DRAM bytes per token-row of the fused kernel from the committed ncu
-    summary, or None if the kernel source changed since it was captured."""
+    """DRAM bytes per token-row of the fused kernel from the committed one-pass
+    ncu capture of the benchmark workload at full size, or None if the kernel
+    source changed since it was captured."""
     import re
-    prof = os.path.join(ROOT, "profiles", "fused_kernel_19L_b4_n8193_ncu_full.md")
+    prof = os.path.join(ROOT, "profiles", "fused_kernel_mistral7b_32L_b8_ctx32k_dram_traffic.md")
     try:
         text = open(prof).read()
         t = float(re.search(r"traffic_bytes_per_token_row:\s*([0-9.]+)", text).group(1))
@@ -333,6 +334,43 @@ def timed_steps(cache, inputs, s0, K, out, stream, index):
     return ev0.elapsed_time(ev1) / K, clk.summary()
 
 
+def timed_then_profiled(cache, inputs, s0, K, out, stream, index):
+    """For steps of tens of microseconds, where the library's per-launch
+    events would add to the step time: K steps timed with launch counting
+    only, then the same K inputs again with per-launch events (for the
+    roofline). Returns (ms per step, clocks, per-launch profile)."""
+    cache.profile(False)  # counts launches, records no events
+    ms, clocks = timed_steps(cache, inputs, s0, K, out, stream, index)
+    cache.profile(True)
+    for s in range(s0, s0 + K):
+        cache.step(*inputs[s], out=out)
+    prof = cache.profile_read()
+    cache.profile(False)
+    return ms, clocks, prof
+
+
+def warm_modules(wl, args):
+    """Runs the prompt compression's kernels once on a small cache of the
+    workload's head shape (one layer, one sequence, a prompt past the on-chip
+    logit capacity), so that the timed first step does not include the lazy
+    loading of their modules."""
+    import torch
+    from paper_2608_08878_gb300 import dc, synth_device
+    small = wl.with_(layers=1, batch=1, prompt_len=12000, budget=3000)
+    c = dc.DistillCache(1, wl.kv_heads, wl.head_dim, small.prompt_len + 8, small.budget, batch=1,
+                        q_heads=wl.q_heads, window=wl.window, mlp_hidden=wl.mlp_hidden, layernorm=wl.layernorm,
+                        engine=args.engine)
+    k, v = synth_device.prompt(small, 0, small.prompt_len)
+    c.append(k, v)
+    q, kn, vn = synth_device.step_inputs(small, 0)
+    c.decode_step(q, kn, vn)
+    c.evict()
+    c.step(*synth_device.step_inputs(small, 1))
+    c.sync()
+    c.close()
+    torch.cuda.synchronize()
+
+
 def run_gpu(args):
     import torch
     from paper_2608_08878_gb300 import build, dc, synth, synth_device
@@ -364,7 +402,10 @@ def run_gpu(args):
     # all step inputs resident in HBM before timing
     inputs = [synth_device.step_inputs(wl, s) for s in range(1 + F + W + K)]
     out = torch.empty((wl.layers, wl.batch, wl.q_heads, wl.head_dim), dtype=torch.float32, device="cuda")
-    # step 0: prompt compression (32769 -> 8192 tokens per row), timed apart
+    # step 0: prompt compression (32769 -> 8192 tokens per row), timed apart,
+    # after the kernels it runs are loaded (CUDA loads a module at the first
+    # launch of one of its kernels, inside the launch call)
+    warm_modules(wl, args)
     ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     cache.profile(True)
     ev0.record(stream)
@@ -417,7 +458,7 @@ def run_gpu(args):
     if dom == "attend" and engine.startswith("fused") and not (args.global_tokens or args.hybrid or args.scorer):
         tpr = fused_traffic_per_token_row()
         if tpr is not None:
-            traffic = wl.rows * n_steady * tpr  # scaled from the profiled case by token-rows
+            traffic = wl.rows * n_steady * tpr  # the full-size capture's bytes per token-row
     gpu_launches = int(sum(v[1] for v in prof.values()))
     # full-cache comparator on the same inputs (the uncompressed prompt)
     full = None
@@ -598,9 +639,7 @@ def sweep_point_run(b, c, r, K, W, engine_flag, peaks, stream, index, with_full=
     for s in range(W):
         cache.step(*inputs[s], out=out)
     engine = cache.engine()
-    cache.profile(True)
-    ms, clocks = timed_steps(cache, inputs, W, K, out, stream, index)
-    prof = cache.profile_read()
+    ms, clocks, prof = timed_then_profiled(cache, inputs, W, K, out, stream, index)
     dom, per_launch_ms, alg, _ = roofline_of(prof, wl, B + 1, engine)
     achieved = alg / (per_launch_ms / 1e3) / 1e9
     bytes_step = step_bytes(wl, B + 1)
@@ -674,9 +713,7 @@ def workload_run(wl, steps_total, W, engine_flag, peaks, stream, index):
         cache.step(*inputs[s], out=out)
     engine = cache.engine()
     K = steps_total - 1 - W
-    cache.profile(True)
-    ms, clocks = timed_steps(cache, inputs, 1 + W, K, out, stream, index)
-    prof = cache.profile_read()
+    ms, clocks, prof = timed_then_profiled(cache, inputs, 1 + W, K, out, stream, index)
     n = wl.budget + 1
     dom, per_launch_ms, alg, _ = roofline_of(prof, wl, n, engine)
     achieved = alg / (per_launch_ms / 1e3) / 1e9

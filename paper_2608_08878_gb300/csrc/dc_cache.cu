@@ -453,6 +453,7 @@ dc_status dc_cache_create(int layers, int kv_heads, int head_dim, int capacity, 
   A(&p.part, (size_t)R * p.smax * G * 4 * sizeof(float));
   A(&p.opart, (size_t)R * p.smax * G * head_dim * sizeof(float));
   A(&p.holes, RC * sizeof(int));
+  A(&p.nmoves, (size_t)R * 2 * sizeof(int));
   if (p.seq_rows) {
     A(&p.gpart, RC * sizeof(float4));
     A(&p.gring, (size_t)cfg.batch * cfg.window * p.stride * sizeof(float2));
@@ -918,7 +919,7 @@ dc_status dc_evict(dc_cache* h, int budget) {
   if (h->per_row) {
     // every row to its own budget (or all to `budget` when > 0)
     {
-      Phase ph(h, DC_PHASE_EVICT, 1);
+      Phase ph(h, DC_PHASE_EVICT, dc::evict_kernel_count(h->n, budget > 0 ? budget : 0));
       dc::launch_evict(h->dev, h->n, budget > 0 ? budget : 0, h->stream);
     }
     dc_status s = launch_error(h, "evict");
@@ -935,7 +936,7 @@ dc_status dc_evict(dc_cache* h, int budget) {
   const int B = effective_budget(h, budget, h->n, h->seen);
   const int keep = std::min(h->n, B);
   if (keep < h->n) {
-    Phase ph(h, DC_PHASE_EVICT, h->dev.seq_rows ? 2 : 1);
+    Phase ph(h, DC_PHASE_EVICT, h->dev.seq_rows ? 2 : dc::evict_kernel_count(h->n, keep));
     if (h->dev.seq_rows) dc::launch_glob_evict(h->dev, h->n, keep, h->stream);
     else dc::launch_evict(h->dev, h->n, keep, h->stream);
     dc_status s = launch_error(h, "evict");

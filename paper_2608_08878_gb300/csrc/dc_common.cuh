@@ -103,6 +103,7 @@ struct Dev {
   float* part;    // [R][smax][G][4]: per-split (m, l, u2, 0)
   float* opart;   // [R][smax][G][d]
   int* holes;     // [R][stride]
+  int* nmoves;    // [R][2]: the eviction kernel's move count and hole count per row
   int smax;
   float c;        // log2(e) / sqrt(d): raw logit difference -> log2 units
 };

@@ -20,7 +20,10 @@ void launch_split_stats(const Dev& p, const Step& st, const void* q, cudaStream_
 void launch_split_v(const Dev& p, const Step& st, cudaStream_t s);
 void launch_split_out(const Dev& p, const Step& st, float* out, cudaStream_t s);
 
+// argtop_B and prune of every row (B <= 0: per-row budgets): a select kernel
+// and, when slots have to move, a move kernel (evict_kernel_count of them).
 void launch_evict(const Dev& p, int n, int B, cudaStream_t s);
+int evict_kernel_count(int n, int B);
 
 // Global token mode: pooled per-sequence features and scores after the split
 // engine's per-row pass; the sequence's selection applied to all its rows.

@@ -252,15 +252,66 @@ __device__ __forceinline__ void move_slot_1(const Dev& p, size_t src, size_t dst
 }
 
 // K/V rows a warp of the list-based compaction loads before it stores them.
-constexpr int kMoveUnroll = 6;
+constexpr int kMoveUnroll = 8;
+
+// One warp moves entries [k0, min(k0 + 32, nmv)) of a row's move lists: the
+// k-th mover (slot movers[k] >= B) fills the k-th hole (slot holes[k] < B).
+// Sources are at or above B and destinations below it, so all moves of a row
+// are independent. Lane l copies the per-token fields of move k0 + l (uniform
+// code, one slot per lane); then the warp copies the K and V rows, each lane
+// one 16-byte chunk, kMoveUnroll rows' loads in flight before their stores.
+__device__ __forceinline__ void warp_move_batch(const Dev& p, size_t base, const int* holes, const int* movers,
+                                                int k0, int nmv, int lane) {
+  const int VPR = p.d / 8;                 // 16-byte chunks per K (or V) row
+  const int rows_per = kWarp / (2 * VPR);  // slots copied per warp instruction
+  const int sub = lane / (2 * VPR), chunk = lane % (2 * VPR);
+  const int k = k0 + lane;
+  const bool live = k < nmv;
+  int src = live ? movers[k] : 0, dst = live ? holes[k] : 0;
+  if (live && !(DC_INB(p, src, p.stride, 203) && DC_INB(p, dst, p.stride, 204))) src = dst = -1;
+  if (live && src >= 0) {
+    const size_t fs = base + src, fd = base + dst;
+    const int ps_ = p.pos[fs];
+    const float vn = p.vnorm[fs];
+    const float4 sz = p.SZ[fs];
+    const float sc = p.score[fs];
+    const float ac = p.acc ? p.acc[fs] : 0.f;
+    p.pos[fd] = ps_;
+    p.vnorm[fd] = vn;
+    p.SZ[fd] = sz;
+    p.score[fd] = sc;
+    if (p.acc) p.acc[fd] = ac;
+    if (p.keep_features)
+      for (int e = 0; e < 5; ++e) p.feat[fd * 5 + e] = p.feat[fs * 5 + e];
+  }
+  const int cnt = nmv - k0 < kWarp ? nmv - k0 : kWarp;
+  const uint4* gk = reinterpret_cast<const uint4*>(chunk < VPR ? p.K : p.V);
+  uint4* gkw = reinterpret_cast<uint4*>(chunk < VPR ? p.K : p.V);
+  const int c = chunk < VPR ? chunk : chunk - VPR;
+  for (int j0 = 0; j0 < cnt; j0 += kMoveUnroll * rows_per) {
+    uint4 v[kMoveUnroll];
+    int d_[kMoveUnroll];
+#pragma unroll
+    for (int u = 0; u < kMoveUnroll; ++u) {
+      const int j = j0 + u * rows_per + sub;
+      const int sj = __shfl_sync(0xffffffffu, src, j & (kWarp - 1));
+      d_[u] = __shfl_sync(0xffffffffu, dst, j & (kWarp - 1));
+      if (j >= cnt || sj < 0) d_[u] = -1;
+      if (d_[u] >= 0) v[u] = gk[(base + sj) * VPR + c];
+    }
+#pragma unroll
+    for (int u = 0; u < kMoveUnroll; ++u)
+      if (d_[u] >= 0) gkw[(base + d_[u]) * VPR + c] = v[u];
+  }
+}
 
 // Keeps the top B of the row's n tokens (order keys keyf(i), i < n) and
 // compacts them into slots [0, B). Requires 1 <= B < n. All NT threads of the
 // team call it. Two compactions: WARP_MOVES (the eviction kernel, many moves):
-// hole and mover lists built with ballots, then each warp copies several
-// slots at a time; otherwise (the fused kernel's epilogue, where registers
-// are scarce) chunks of NT candidate slots are ranked with a team scan and
-// each mover thread copies its slot.
+// hole and mover lists built with ballots, the moves left to a kernel of their
+// own (evict_move_kernel); otherwise (the fused kernel's epilogue, where
+// registers are scarce) chunks of NT candidate slots are ranked with a team
+// scan and each mover thread copies its slot.
 template <int NT, bool WARP_MOVES, class KeyF, class Sync>
 __device__ void team_select_compact_k(const Dev& p, int r, int n, int B, KeyF key, int tid,
                                       const SelectScratch& s, Sync sync) {
@@ -349,12 +400,13 @@ __device__ void team_select_compact_k(const Dev& p, int r, int n, int B, KeyF ke
     sync();
   } else {
     // Hole and mover lists in ascending slot order: holes (evicted slots below
-    // B) in holes[0, nh), movers (survivors at or above B) in holes[B, B + nm)
-    // (the row's scratch has n >= B + nm entries). Each warp takes a contiguous
+    // B) in holes[0, nh), movers (survivors at or above B) in holes[nh, nh + nm)
+    // (the row's scratch has n >= nh + nm entries). Each warp takes a contiguous
     // run of 32-slot groups: it counts its flags with ballots, the warps' counts
-    // are prefix-summed once, and a second walk writes the indices.
+    // are prefix-summed once, and a second walk writes the indices. The moves
+    // themselves are evict_move_kernel's (warp_move_batch), with the counts
+    // left in p.nmoves.
     int* holes = p.holes + base;
-    int* movers = holes + B;
     constexpr int NW = NT / kWarp;
     const int lane = tid % kWarp, wid = tid / kWarp;
     const int ng = (n + kWarp - 1) / kWarp;
@@ -379,6 +431,7 @@ __device__ void team_select_compact_k(const Dev& p, int r, int n, int B, KeyF ke
       nh += vh;
       nm += vm;
     }
+    int* movers = holes + nh;
     const unsigned lt = (1u << lane) - 1u;
     for (int gi = g0; gi < g1; ++gi) {
       const int i = gi * kWarp + lane;
@@ -386,60 +439,15 @@ __device__ void team_select_compact_k(const Dev& p, int r, int n, int B, KeyF ke
       const bool fh = i < B && !kp, fm = i >= B && kp;
       const unsigned bh = __ballot_sync(0xffffffffu, fh), bm = __ballot_sync(0xffffffffu, fm);
       if (fh && DC_INB(p, hb + __popc(bh & lt), B, 201)) holes[hb + __popc(bh & lt)] = i;
-      if (fm && DC_INB(p, B + mb + __popc(bm & lt), p.stride, 202)) movers[mb + __popc(bm & lt)] = i;
+      if (fm && DC_INB(p, nh + mb + __popc(bm & lt), p.stride, 202)) movers[mb + __popc(bm & lt)] = i;
       hb += __popc(bh);
       mb += __popc(bm);
     }
     if (tid == 0 && nm != nh) atomicOr(p.status, kStatusBadShape);
     sync();
-    // The k-th mover fills the k-th hole. Sources are >= B and destinations < B,
-    // so the moves are independent. A warp takes 32 moves at a time: lane l
-    // copies the per-token fields of move l (uniform code, one slot per lane),
-    // then the warp copies the K and V rows, each lane one 16-byte chunk, eight
-    // rows' loads in flight before their stores.
-    const int nmv = nm < nh ? nm : nh;
-    const int VPR = p.d / 8;              // 16-byte chunks per K (or V) row
-    const int rows_per = kWarp / (2 * VPR);  // slots copied per warp instruction
-    const int sub = lane / (2 * VPR), chunk = lane % (2 * VPR);
-    for (int k0 = wid * kWarp; k0 < nmv; k0 += NW * kWarp) {
-      const int k = k0 + lane;
-      const bool live = k < nmv;
-      int src = live ? movers[k] : 0, dst = live ? holes[k] : 0;
-      if (live && !(DC_INB(p, src, p.stride, 203) && DC_INB(p, dst, p.stride, 204))) src = dst = -1;
-      if (live && src >= 0) {
-        const size_t fs = base + src, fd = base + dst;
-        const int ps_ = p.pos[fs];
-        const float vn = p.vnorm[fs];
-        const float4 sz = p.SZ[fs];
-        const float sc = p.score[fs];
-        const float ac = p.acc ? p.acc[fs] : 0.f;
-        p.pos[fd] = ps_;
-        p.vnorm[fd] = vn;
-        p.SZ[fd] = sz;
-        p.score[fd] = sc;
-        if (p.acc) p.acc[fd] = ac;
-        if (p.keep_features)
-          for (int e = 0; e < 5; ++e) p.feat[fd * 5 + e] = p.feat[fs * 5 + e];
-      }
-      const int cnt = nmv - k0 < kWarp ? nmv - k0 : kWarp;
-      const uint4* gk = reinterpret_cast<const uint4*>(chunk < VPR ? p.K : p.V);
-      uint4* gkw = reinterpret_cast<uint4*>(chunk < VPR ? p.K : p.V);
-      const int c = chunk < VPR ? chunk : chunk - VPR;
-      for (int j0 = 0; j0 < cnt; j0 += kMoveUnroll * rows_per) {
-        uint4 v[kMoveUnroll];
-        int d_[kMoveUnroll];
-#pragma unroll
-        for (int u = 0; u < kMoveUnroll; ++u) {
-          const int j = j0 + u * rows_per + sub;
-          const int sj = __shfl_sync(0xffffffffu, src, j & (kWarp - 1));
-          d_[u] = __shfl_sync(0xffffffffu, dst, j & (kWarp - 1));
-          if (j >= cnt || sj < 0) d_[u] = -1;
-          if (d_[u] >= 0) v[u] = gk[(base + sj) * VPR + c];
-        }
-#pragma unroll
-        for (int u = 0; u < kMoveUnroll; ++u)
-          if (d_[u] >= 0) gkw[(base + d_[u]) * VPR + c] = v[u];
-      }
+    if (tid == 0) {
+      p.nmoves[2 * (size_t)r] = nm < nh ? nm : nh;
+      p.nmoves[2 * (size_t)r + 1] = nh;
     }
     sync();
   }
