@@ -133,6 +133,13 @@ __device__ __forceinline__ float ex2(float x) {
   return y;
 }
 
+// Hardware base-2 logarithm (lg2.approx, relative error ~2^-22).
+__device__ __forceinline__ float lg2_approx(float x) {
+  float y;
+  asm("lg2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+
 // Attention weight a = 2^((s - m) c) / l = 2^((s - m) c + nl), nl = -log2(l),
 // of a token with raw logit s under a query whose max raw logit is m. Written
 // with explicitly rounded operations so that the value is bit-identical

@@ -922,8 +922,11 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
       for (int h = 0; h < G; ++h) {
         M[h] = Mm[h];
-        NL[h] = -log2f(Ll[h]);
-        Hh[h] = logf(Ll[h]) - 0.69314718055994531f * (Uu[h] / Ll[h]);
+        // H = ln l - ln 2 u / l = ln 2 (log2 l - u / l), with the hardware
+        // log2 and divide (l >= 1: the row's largest logit contributes 2^0)
+        const float lg = lg2_approx(Ll[h]);
+        NL[h] = -lg;
+        Hh[h] = 0.69314718055994531f * (lg - __fdividef(Uu[h], Ll[h]));
         if (tid == h) L0 = Ll[h];
       }
       // G = 8: the V pass reads the row's final statistics from shared memory
