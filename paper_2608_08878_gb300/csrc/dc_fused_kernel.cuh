@@ -1226,10 +1226,25 @@ __global__ void __launch_bounds__(kThreads, 1)
           const int op = __shfl_xor_sync(0xffffffffu, bp, off);
           if (lower(bk, bs, bp, ok, os, op)) { bk = ok; bs = os; bp = op; }
         }
-        sync();
+        if (half >= 0) sync();
         const int tw = tid / kWarp;  // warp within the team
         if (lane == 0) { scr.best[tw] = bk; scr.best_slot[tw] = bs; scr.hist[tw] = bp; }
         sync();
+        if (half < 0) {
+          // whole rows and row pairs: the warp that holds slot B reduces the
+          // team's candidates itself (in warp order, as one thread would) and
+          // fills the evicted slot; no further barrier (the candidates' next
+          // writers are behind the next item's barriers)
+          if (tid < kWarp) {
+            uint32_t fk = (uint32_t)scr.best[0];
+            int fe = scr.best_slot[0], fpos = scr.hist[0];
+            for (int w = 1; w < kTeam / kWarp; ++w)
+              if (lower(fk, fe, fpos, (uint32_t)scr.best[w], scr.best_slot[w], scr.hist[w])) {
+                fk = (uint32_t)scr.best[w]; fe = scr.best_slot[w]; fpos = scr.hist[w];
+              }
+            if (fe >= 0 && fe < Bsel && slot_ok(fe, 117)) slot_store(p, rbase + fe, tid, mv);
+          }
+        } else {
         if (tid == 0) {
           uint32_t fk = (uint32_t)scr.best[0];
           int fe = scr.best_slot[0], fpos = scr.hist[0];
@@ -1258,6 +1273,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int e = scr.sh[0];
         if (mover && e >= 0 && e < Bsel && tid < kWarp && slot_ok(e, 117)) slot_store(p, rbase + e, tid, mv);
         sync();
+        }
       } else if (fs.do_evict && Bsel < n) {
         // several evictions (whole rows only): radix select over the scores
         sync();
