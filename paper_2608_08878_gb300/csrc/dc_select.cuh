@@ -305,11 +305,68 @@ __device__ __forceinline__ void warp_move_batch(const Dev& p, size_t base, const
   }
 }
 
+// Hole and mover lists of a row in ascending slot order, for keep(i) = "slot
+// i survives": holes (evicted slots below B) in p.holes[row][0, nh), movers
+// (survivors at or above B) in p.holes[row][nh, nh + nm) (the row's scratch
+// has n >= nh + nm entries), the counts in p.nmoves[row]. Each warp takes a
+// contiguous run of 32-slot groups: it counts its flags with ballots, the
+// warps' counts are prefix-summed once, and a second walk writes the indices.
+// The moves themselves are evict_move_kernel's (warp_move_batch).
+template <int NT, class Keep, class Sync>
+__device__ void team_move_lists(const Dev& p, int r, int n, int B, Keep keep, int tid, const SelectScratch& s,
+                                Sync sync) {
+  const size_t base = (size_t)r * p.stride;
+  int* holes = p.holes + base;
+  constexpr int NW = NT / kWarp;
+  const int lane = tid % kWarp, wid = tid / kWarp;
+  const int ng = (n + kWarp - 1) / kWarp;
+  const int g0 = (int)((long long)ng * wid / NW), g1 = (int)((long long)ng * (wid + 1) / NW);
+  int ch = 0, cm = 0;
+  for (int gi = g0; gi < g1; ++gi) {
+    const int i = gi * kWarp + lane;
+    const bool kp = i < n && keep(i);
+    ch += __popc(__ballot_sync(0xffffffffu, i < B && !kp));
+    cm += __popc(__ballot_sync(0xffffffffu, i >= B && kp));
+  }
+  if (lane == 0) s.best[wid] = ((unsigned long long)(unsigned)cm << 32) | (unsigned)ch;
+  sync();
+  int hb = 0, mb = 0, nh = 0, nm = 0;
+  for (int w = 0; w < NW; ++w) {
+    const unsigned long long v = s.best[w];
+    const int vh = (int)(unsigned)(v & 0xFFFFFFFFull), vm = (int)(unsigned)(v >> 32);
+    if (w < wid) {
+      hb += vh;
+      mb += vm;
+    }
+    nh += vh;
+    nm += vm;
+  }
+  int* movers = holes + nh;
+  const unsigned lt = (1u << lane) - 1u;
+  for (int gi = g0; gi < g1; ++gi) {
+    const int i = gi * kWarp + lane;
+    const bool kp = i < n && keep(i);
+    const bool fh = i < B && !kp, fm = i >= B && kp;
+    const unsigned bh = __ballot_sync(0xffffffffu, fh), bm = __ballot_sync(0xffffffffu, fm);
+    if (fh && DC_INB(p, hb + __popc(bh & lt), B, 201)) holes[hb + __popc(bh & lt)] = i;
+    if (fm && DC_INB(p, nh + mb + __popc(bm & lt), p.stride, 202)) movers[mb + __popc(bm & lt)] = i;
+    hb += __popc(bh);
+    mb += __popc(bm);
+  }
+  if (tid == 0 && nm != nh) atomicOr(p.status, kStatusBadShape);
+  sync();
+  if (tid == 0) {
+    p.nmoves[2 * (size_t)r] = nm < nh ? nm : nh;
+    p.nmoves[2 * (size_t)r + 1] = nh;
+  }
+  sync();
+}
+
 // Keeps the top B of the row's n tokens (order keys keyf(i), i < n) and
 // compacts them into slots [0, B). Requires 1 <= B < n. All NT threads of the
 // team call it. Two compactions: WARP_MOVES (the eviction kernel, many moves):
-// hole and mover lists built with ballots, the moves left to a kernel of their
-// own (evict_move_kernel); otherwise (the fused kernel's epilogue, where
+// team_move_lists, the moves left to a kernel of their own
+// (evict_move_kernel); otherwise (the fused kernel's epilogue, where
 // registers are scarce) chunks of NT candidate slots are ranked with a team
 // scan and each mover thread copies its slot.
 template <int NT, bool WARP_MOVES, class KeyF, class Sync>
@@ -399,57 +456,7 @@ __device__ void team_select_compact_k(const Dev& p, int r, int n, int B, KeyF ke
     if (tid == 0 && nm != nh) atomicOr(p.status, kStatusBadShape);
     sync();
   } else {
-    // Hole and mover lists in ascending slot order: holes (evicted slots below
-    // B) in holes[0, nh), movers (survivors at or above B) in holes[nh, nh + nm)
-    // (the row's scratch has n >= nh + nm entries). Each warp takes a contiguous
-    // run of 32-slot groups: it counts its flags with ballots, the warps' counts
-    // are prefix-summed once, and a second walk writes the indices. The moves
-    // themselves are evict_move_kernel's (warp_move_batch), with the counts
-    // left in p.nmoves.
-    int* holes = p.holes + base;
-    constexpr int NW = NT / kWarp;
-    const int lane = tid % kWarp, wid = tid / kWarp;
-    const int ng = (n + kWarp - 1) / kWarp;
-    const int g0 = (int)((long long)ng * wid / NW), g1 = (int)((long long)ng * (wid + 1) / NW);
-    int ch = 0, cm = 0;
-    for (int gi = g0; gi < g1; ++gi) {
-      const int i = gi * kWarp + lane;
-      const bool kp = i < n && keep(i);
-      ch += __popc(__ballot_sync(0xffffffffu, i < B && !kp));
-      cm += __popc(__ballot_sync(0xffffffffu, i >= B && kp));
-    }
-    if (lane == 0) s.best[wid] = ((unsigned long long)(unsigned)cm << 32) | (unsigned)ch;
-    sync();
-    int hb = 0, mb = 0, nh = 0, nm = 0;
-    for (int w = 0; w < NW; ++w) {
-      const unsigned long long v = s.best[w];
-      const int vh = (int)(unsigned)(v & 0xFFFFFFFFull), vm = (int)(unsigned)(v >> 32);
-      if (w < wid) {
-        hb += vh;
-        mb += vm;
-      }
-      nh += vh;
-      nm += vm;
-    }
-    int* movers = holes + nh;
-    const unsigned lt = (1u << lane) - 1u;
-    for (int gi = g0; gi < g1; ++gi) {
-      const int i = gi * kWarp + lane;
-      const bool kp = i < n && keep(i);
-      const bool fh = i < B && !kp, fm = i >= B && kp;
-      const unsigned bh = __ballot_sync(0xffffffffu, fh), bm = __ballot_sync(0xffffffffu, fm);
-      if (fh && DC_INB(p, hb + __popc(bh & lt), B, 201)) holes[hb + __popc(bh & lt)] = i;
-      if (fm && DC_INB(p, nh + mb + __popc(bm & lt), p.stride, 202)) movers[mb + __popc(bm & lt)] = i;
-      hb += __popc(bh);
-      mb += __popc(bm);
-    }
-    if (tid == 0 && nm != nh) atomicOr(p.status, kStatusBadShape);
-    sync();
-    if (tid == 0) {
-      p.nmoves[2 * (size_t)r] = nm < nh ? nm : nh;
-      p.nmoves[2 * (size_t)r + 1] = nh;
-    }
-    sync();
+    team_move_lists<NT>(p, r, n, B, keep, tid, s, sync);
   }
 }
 

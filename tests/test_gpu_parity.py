@@ -275,6 +275,23 @@ def test_heuristic_scorers(engine, scorer):
             assert torch.equal(a.cache.buffer(which)[:, :n], b.cache.buffer(which)[:, :n]), (s, which)
 
 
+@pytest.mark.parametrize("n_sinks", [10000, 5000, 512])
+def test_many_evictions_with_tied_scores(n_sinks):
+    """The eviction kernel's select on a 12001-token row with budget 1024,
+    StreamingLLM scores (the first n_sinks positions tie at the top, the rest
+    are distinct): 10000 tied keys (more than the select lists in shared
+    memory, so it takes its radix passes over the whole row), 5000 tied keys
+    (listed, the cut among them by position), and 512 (the threshold among the
+    distinct scores, survivors moved into the holes). Against the oracle fed
+    the GPU's scores, then two steps with one eviction each."""
+    wl = synth.MISTRAL_1L.with_(prompt_len=12000, budget=1024, steps=3)
+    ls = LockStep(wl, [0, 5], engine=2, scorer=2, n_sinks=n_sinks)
+    ls.load_prompt()
+    for _ in range(wl.steps):
+        ls.step()
+    assert ls.cache.length()[0] == 1024
+
+
 @pytest.mark.parametrize("engine", ENGINES)
 @pytest.mark.parametrize("basis", [0, 1])
 def test_dynamic_budget(engine, basis):
