@@ -127,6 +127,32 @@ struct Step {
   int chunk;      // tokens per split
 };
 
+// Programmatic dependent launch (a grid launched with the programmatic
+// stream serialization attribute may start while the grid before it in the
+// stream still runs): grid_dep_wait returns once the grids this one depends
+// on have completed and their writes are visible (at once when there are
+// none); grid_dep_launch lets the grid after this one start launching.
+__device__ __forceinline__ void grid_dep_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void grid_dep_launch() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
+
+// Launches f with programmatic stream serialization: the grid may start while
+// the grid before it in the stream runs, and waits for it in grid_dep_wait.
+template <class... KArgs, class... Args>
+inline cudaError_t launch_pdl(void (*f)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t s,
+                              Args&&... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute la[1];
+  la[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  la[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = la;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, f, static_cast<Args&&>(args)...);
+}
+
 __device__ __forceinline__ float ex2(float x) {
   float y;
   asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));

@@ -369,6 +369,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   constexpr bool kWqSmem = G == 8;
   static_assert(!GRAPH || (!FULL && !HEUR && !GLOB && !PERROW), "device-counted steps: the plain step");
   if constexpr (GRAPH) {
+    grid_dep_wait();  // the counter is the previous launch's
     // this launch's step: the base arguments advanced by the steps taken (in
     // the steady state a step appends one token, so positions, window slots
     // and the launch epoch all advance by one per step)
@@ -435,8 +436,6 @@ __global__ void __launch_bounds__(kThreads, 1)
     mbar_init(&bar[B_DRAIN2], 1);
     *abort = 0;
     for (int e = 0; e < kItemRing; ++e) items[4 * kItemRing + e] = 0;
-    // the next launch's queue counter (this launch uses the other one)
-    if (blockIdx.x == 0) fs.work[(fs.epoch + 1u) & 1u] = 0u;
     fence_mbar_init();
   }
   // zero the stages and their per-token areas (a row's ragged last tile loads
@@ -463,6 +462,12 @@ __global__ void __launch_bounds__(kThreads, 1)
     prefetch_tmap(&tmK16);
     prefetch_tmap(&tmV16);
   }
+  // everything above touches only shared memory, TMEM and read-only inputs:
+  // with a programmatic launch it overlaps the kernel before (the append);
+  // the cache and the queue counters are read and written after this wait
+  grid_dep_wait();
+  // the next launch's queue counter (this launch uses the other one)
+  if (blockIdx.x == 0 && threadIdx.x == 0) fs.work[(fs.epoch + 1u) & 1u] = 0u;
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
@@ -1313,6 +1318,9 @@ static cudaError_t launch_t(const FusedMaps& maps, const Dev& p, const Step& st,
     if (e != cudaSuccess) return e;
     attr = true;
   }
+  if (fs.half_rows == 0 && !GRAPH)
+    return launch_pdl(fused_kernel<D, G, LONG, FULL, HEUR, GLOB, PERROW, PAIR, GRAPH>, dim3(grid), dim3(kThreads),
+                      kSmemBytes, s, maps.k, maps.v, maps.k16, maps.v16, p, st, fs, fp);
   if (fs.half_rows == 0) {
     fused_kernel<D, G, LONG, FULL, HEUR, GLOB, PERROW, PAIR, GRAPH>
         <<<grid, kThreads, kSmemBytes, s>>>(maps.k, maps.v, maps.k16, maps.v16, p, st, fs, fp);

@@ -23,6 +23,11 @@ constexpr int kTile = 128;  // tokens per tile = threads per CTA
 __global__ void __launch_bounds__(256) append_kernel(Dev p, const uint4* __restrict__ k,
                                                      const uint4* __restrict__ v, long long pairs, int T,
                                                      int n0, int seen0) {
+  // launched after the kernels that wrote k and v, or after the previous
+  // step's kernels, which still read the slots written here
+  grid_dep_wait();
+  // the fused step kernel after this one may start its set-up meanwhile
+  grid_dep_launch();
   const int vpr = p.d / 8;
   const long long e = ((long long)blockIdx.x * blockDim.x + threadIdx.x) / vpr;
   const int c = threadIdx.x % vpr;
@@ -410,7 +415,7 @@ void launch_append(const Dev& p, const void* k, const void* v, int T, int n0, in
   if (pairs == 0) return;
   const long long per_block = 256 / (p.d / 8);
   const unsigned blocks = (unsigned)((pairs + per_block - 1) / per_block);
-  append_kernel<<<blocks, 256, 0, s>>>(p, (const uint4*)k, (const uint4*)v, pairs, T, n0, seen0);
+  launch_pdl(append_kernel, dim3(blocks), dim3(256), 0, s, p, (const uint4*)k, (const uint4*)v, pairs, T, n0, seen0);
 }
 
 #define DC_DISPATCH(EXPR)                                                   \
