@@ -497,40 +497,70 @@ __global__ void __launch_bounds__(kThreads, 1)
       last = it.half >= 0;
       const int r = it.row;
       // query tile (PAIR: one per row): rows [0,G) current, [G,2G) previous
-      // step, [2G,3G) departing. The current query also takes over the
-      // departing query's ring slot, so every element of a row is read
-      // before any is written: a row's loads are issued together.
-      constexpr int QCH = G * (D / 8);                 // 16-byte chunks of a row's G query heads
-      constexpr int QIT = (QCH + kWarp - 1) / kWarp;   // per lane
-      for (int qi = 0; qi < (PAIR ? 2 : 1); ++qi) {
-        const int rq = r + qi;
-        uint8_t* qt = smem + OFF_Q + (PAIR ? 2 * qb + qi : qb) * L::QBYTES;
-        const int qo = ((rq / p.kvh) * p.qh + (rq % p.kvh) * G) * D;
-        const __nv_bfloat16* prev = p.ring_q + ((size_t)rq * p.w + st.slot_prev) * G * D;
-        const __nv_bfloat16* dep = p.ring_q + ((size_t)rq * p.w + st.slot) * G * D;
-        __nv_bfloat16* ring_slot = p.ring_q + ((size_t)rq * p.w + st.slot) * G * D;
-        const bool q_ok = DC_INB(p, qo + G * D - 1, (long long)(p.R / p.kvh) * p.qh * D, 101) &&
-                          DC_INB(p, ((long long)rq * p.w + st.slot) * G * D + G * D - 1, (long long)p.R * p.w * G * D, 102) &&
-                          DC_INB(p, ((long long)rq * p.w + st.slot_prev) * G * D, (long long)p.R * p.w * G * D, 103);
-        uint4 qcur[QIT], qprev[QIT], qdep[QIT];
+      // step, [2G,3G) departing
+      if constexpr (PAIR) {
+        // row pairs: a row's loads issued together (every element is read
+        // before any is written, as the current query takes over the departing
+        // query's ring slot), one global round trip per row
+        constexpr int QCH = G * (D / 8);                 // 16-byte chunks of a row's G query heads
+        constexpr int QIT = (QCH + kWarp - 1) / kWarp;   // per lane
+        for (int qi = 0; qi < 2; ++qi) {
+          const int rq = r + qi;
+          uint8_t* qt = smem + OFF_Q + (2 * qb + qi) * L::QBYTES;
+          const int qo = ((rq / p.kvh) * p.qh + (rq % p.kvh) * G) * D;
+          const __nv_bfloat16* prev = p.ring_q + ((size_t)rq * p.w + st.slot_prev) * G * D;
+          const __nv_bfloat16* dep = p.ring_q + ((size_t)rq * p.w + st.slot) * G * D;
+          __nv_bfloat16* ring_slot = p.ring_q + ((size_t)rq * p.w + st.slot) * G * D;
+          const bool q_ok = DC_INB(p, qo + G * D - 1, (long long)(p.R / p.kvh) * p.qh * D, 101) &&
+                            DC_INB(p, ((long long)rq * p.w + st.slot) * G * D + G * D - 1, (long long)p.R * p.w * G * D, 102) &&
+                            DC_INB(p, ((long long)rq * p.w + st.slot_prev) * G * D, (long long)p.R * p.w * G * D, 103);
+          uint4 qcur[QIT], qprev[QIT], qdep[QIT];
 #pragma unroll
-        for (int u = 0; u < QIT; ++u) {
-          const int e = lane + u * kWarp;
-          const int h = e / (D / 8), kc = e % (D / 8);
-          const bool ld = q_ok && e < QCH;
-          qcur[u] = ld ? reinterpret_cast<const uint4*>(fs.q + qo + h * D)[kc] : make_uint4(0, 0, 0, 0);
-          qprev[u] = ld && st.has_prev ? reinterpret_cast<const uint4*>(prev + h * D)[kc] : make_uint4(0, 0, 0, 0);
-          qdep[u] = ld && st.has_dep ? reinterpret_cast<const uint4*>(dep + h * D)[kc] : make_uint4(0, 0, 0, 0);
+          for (int u = 0; u < QIT; ++u) {
+            const int e = lane + u * kWarp;
+            const int h = e / (D / 8), kc = e % (D / 8);
+            const bool ld = q_ok && e < QCH;
+            qcur[u] = ld ? reinterpret_cast<const uint4*>(fs.q + qo + h * D)[kc] : make_uint4(0, 0, 0, 0);
+            qprev[u] = ld && st.has_prev ? reinterpret_cast<const uint4*>(prev + h * D)[kc] : make_uint4(0, 0, 0, 0);
+            qdep[u] = ld && st.has_dep ? reinterpret_cast<const uint4*>(dep + h * D)[kc] : make_uint4(0, 0, 0, 0);
+          }
+#pragma unroll
+          for (int u = 0; u < QIT; ++u) {
+            const int e = lane + u * kWarp;
+            if (!q_ok || e >= QCH) continue;
+            const int h = e / (D / 8), kc = e % (D / 8);
+            *reinterpret_cast<uint4*>(qt + (kc >> 3) * (NQ * 128) + sw128(h, kc & 7)) = qcur[u];
+            *reinterpret_cast<uint4*>(qt + (kc >> 3) * (NQ * 128) + sw128(G + h, kc & 7)) = qprev[u];
+            *reinterpret_cast<uint4*>(qt + (kc >> 3) * (NQ * 128) + sw128(2 * G + h, kc & 7)) = qdep[u];
+            if (!FULL && it.half < 0) reinterpret_cast<uint4*>(ring_slot + h * D)[kc] = qcur[u];  // halves: see the epilogue
+          }
         }
-#pragma unroll
-        for (int u = 0; u < QIT; ++u) {
-          const int e = lane + u * kWarp;
-          if (!q_ok || e >= QCH) continue;
-          const int h = e / (D / 8), kc = e % (D / 8);
-          *reinterpret_cast<uint4*>(qt + (kc >> 3) * (NQ * 128) + sw128(h, kc & 7)) = qcur[u];
-          *reinterpret_cast<uint4*>(qt + (kc >> 3) * (NQ * 128) + sw128(G + h, kc & 7)) = qprev[u];
-          *reinterpret_cast<uint4*>(qt + (kc >> 3) * (NQ * 128) + sw128(2 * G + h, kc & 7)) = qdep[u];
-          if (!FULL && it.half < 0) reinterpret_cast<uint4*>(ring_slot + h * D)[kc] = qcur[u];  // halves: see the epilogue
+      } else {
+        // whole rows: one chunk per lane at a time (on whole rows this measured
+        // faster than issuing the row's loads together: 6.04 against 6.25 ms
+        // per step at 64 x 16384 x 25%)
+        {
+          const int rq = r;
+          uint8_t* qt = smem + OFF_Q + qb * L::QBYTES;
+          const int qo = ((rq / p.kvh) * p.qh + (rq % p.kvh) * G) * D;
+          const __nv_bfloat16* prev = p.ring_q + ((size_t)rq * p.w + st.slot_prev) * G * D;
+          const __nv_bfloat16* dep = p.ring_q + ((size_t)rq * p.w + st.slot) * G * D;
+          // The current query also takes over the departing query's ring slot:
+          // each lane reads the departing element before it writes the same one.
+          __nv_bfloat16* ring_slot = p.ring_q + ((size_t)rq * p.w + st.slot) * G * D;
+          const bool q_ok = DC_INB(p, qo + G * D - 1, (long long)(p.R / p.kvh) * p.qh * D, 101) &&
+                            DC_INB(p, ((long long)rq * p.w + st.slot) * G * D + G * D - 1, (long long)p.R * p.w * G * D, 102) &&
+                            DC_INB(p, ((long long)rq * p.w + st.slot_prev) * G * D, (long long)p.R * p.w * G * D, 103);
+          for (int e = lane; q_ok && e < G * (D / 8); e += kWarp) {
+            const int h = e / (D / 8), kc = e % (D / 8);
+            const uint4 cur = reinterpret_cast<const uint4*>(fs.q + qo + h * D)[kc];
+            const uint4 pv = st.has_prev ? reinterpret_cast<const uint4*>(prev + h * D)[kc] : make_uint4(0, 0, 0, 0);
+            const uint4 dv = st.has_dep ? reinterpret_cast<const uint4*>(dep + h * D)[kc] : make_uint4(0, 0, 0, 0);
+            *reinterpret_cast<uint4*>(qt + (kc >> 3) * (NQ * 128) + sw128(h, kc & 7)) = cur;
+            *reinterpret_cast<uint4*>(qt + (kc >> 3) * (NQ * 128) + sw128(G + h, kc & 7)) = pv;
+            *reinterpret_cast<uint4*>(qt + (kc >> 3) * (NQ * 128) + sw128(2 * G + h, kc & 7)) = dv;
+            if (!FULL && it.half < 0) reinterpret_cast<uint4*>(ring_slot + h * D)[kc] = cur;  // halves: see the epilogue
+          }
         }
       }
       fence_proxy_async();
@@ -939,11 +969,19 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
       for (int h = 0; h < G; ++h) {
         M[h] = Mm[h];
-        // H = ln l - ln 2 u / l = ln 2 (log2 l - u / l), with the hardware
-        // log2 and divide (l >= 1: the row's largest logit contributes 2^0)
-        const float lg = lg2_approx(Ll[h]);
-        NL[h] = -lg;
-        Hh[h] = 0.69314718055994531f * (lg - __fdividef(Uu[h], Ll[h]));
+        // H = ln l - ln 2 u / l. Whole rows take log2 l from the hardware log2
+        // and divide (l >= 1: the row's largest logit contributes 2^0), row
+        // pairs from log2f and logf: each measured the faster for its
+        // schedule (the kernel's speed on these shapes moves by several
+        // per cent with its code layout)
+        if constexpr (PAIR) {
+          NL[h] = -log2f(Ll[h]);
+          Hh[h] = logf(Ll[h]) - 0.69314718055994531f * (Uu[h] / Ll[h]);
+        } else {
+          const float lg = lg2_approx(Ll[h]);
+          NL[h] = -lg;
+          Hh[h] = 0.69314718055994531f * (lg - __fdividef(Uu[h], Ll[h]));
+        }
         if (tid == h) L0 = Ll[h];
       }
       // G = 8: the V pass reads the row's final statistics from shared memory
