@@ -1212,12 +1212,16 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
       };
       // prep(j) returns (the linear score part, or a heuristic score; the
-      // position) for finish(j)
-      float2 pf_cur = j0 < t1 ? prep(j0) : make_float2(0.f, 0.f);
-      for (int j = j0; j < t1; j += JS) {
+      // position) for finish(j), which runs after prep(j + JS); one call site
+      // each (the first pass of the loop only preps the first tile), so that
+      // the loop's code is inlined once
+      float2 pf_cur = make_float2(0.f, 0.f);
+      for (int j = j0 - JS; j < t1; j += JS) {
         const float2 pf_next = j + JS < t1 ? prep(j + JS) : make_float2(0.f, 0.f);
-        if constexpr (HEUR) record_h(j, pf_cur.x, __float_as_int(pf_cur.y));
-        else if constexpr (!FULL && !GLOB) finish(j, pf_cur.x, __float_as_int(pf_cur.y));
+        if (j >= j0) {
+          if constexpr (HEUR) record_h(j, pf_cur.x, __float_as_int(pf_cur.y));
+          else if constexpr (!FULL && !GLOB) finish(j, pf_cur.x, __float_as_int(pf_cur.y));
+        }
         pf_cur = pf_next;
       }
       g += nItem;
