@@ -69,3 +69,29 @@ def test_algorithmic_bytes_are_the_documented_per_unit_figures():
     assert bench.step_bytes(wl, 8193) == 2048 * (8193 * 548 + 532 + 2 * 532)
     assert round(bench.step_bytes(wl, 8193) / 1e9, 3) == 9.198
     assert bench.step_bytes(wl, 8193, moved_per_row=0) == 2048 * (8193 * 548 + 532)
+
+
+def test_reference_arm_line_on_rank_zero(monkeypatch):
+    """The reference arm's line (the fp64 oracle on the host's cores, a bounded
+    sample extrapolated to whole steps): the GPU arm's metric, unit, direction
+    and config dict; the sample described in cpu_baseline; an e2e entry with
+    no host-device copies."""
+    import json
+    import types
+    import bench
+    monkeypatch.delenv("RANK", raising=False)
+    monkeypatch.delenv("WORLD_SIZE", raising=False)
+    args = types.SimpleNamespace(steps=2, warmup=3, cpu_seconds=0.3, global_tokens=False, hybrid=False, scorer=0,
+                                 budget_ratio=0.0)
+    line = bench.run_reference(args)
+    json.dumps(line)
+    assert line["impl"] == "reference"
+    assert (line["metric"], line["unit"], line["higher_is_better"]) == (bench.METRIC, bench.UNIT, True)
+    assert line["config"] == bench.bench_config(bench.workload(), args, 1)
+    assert line["n_gpus"] == 1 and (line["steps"], line["warmup"]) == (2, 3)
+    cb = line["cpu_baseline"]
+    assert cb["kind"] == "oracle" and cb["cores"] >= 1 and cb["host_cores"] >= cb["cores"] and cb["sample"]
+    assert cb["value"] == line["value"] > 0 and cb["row_steps_run"] >= 1
+    assert line["extrapolated"] is True and line["ms_per_step"] == pytest.approx(1e3 / line["value"])
+    assert line["e2e"] == {"value": line["value"], "unit": bench.UNIT, "h2d_bytes_per_step": 0,
+                           "d2h_bytes_per_step": 0}
